@@ -1,0 +1,121 @@
+/*
+ * Reference (oracle) implementation of one Gated VLA-Cache step.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This library is the slow, plain CPU statement
+ * of what the method computes; only the tests, the package's smoke check
+ * and the benchmark's CPU-baseline leg may load it.  It shares no code,
+ * header or table with the CUDA library.
+ *
+ * What it follows:
+ *   - Sec. III-A: image cut into (H/p)(W/p) patches, projected to token
+ *     embeddings, concatenated with the language tokens.
+ *   - Sec. III-B Stage 1: cosine similarity between corresponding patches
+ *     of I_t and I_{t-1}; similarity above tau marks a patch static.
+ *   - Sec. III-B Stage 3: a per-layer proportion of the static patches is
+ *     reused (here a caller-given per-mille schedule).
+ *   - Sec. IV-A Eq. (1): mean top-1/top-2 probability margin over the D
+ *     action tokens.
+ *   - Algorithm 1: gate on m_{t-1} < theta_m -> invalidate and run a full
+ *     pass; otherwise reuse the cache and recompute only the rest; then
+ *     decode the action tokens.
+ *
+ * Every dot product and reduction accumulates in fp64.  Stored values are
+ * rounded at fixed points: the residual stream to fp32; GEMM inputs (norm
+ * outputs, attention output, SwiGLU product), Q and the cached K/V to bf16
+ * (bf16 workloads) or fp32 (fp32 workloads).
+ */
+#ifndef ORC_H
+#define ORC_H
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct orc_dims {
+  int32_t n_layers, hidden, n_heads, head_dim, ffn, vocab, n_bins;
+  int32_t img_h, img_w, patch, n_views;
+  int32_t n_text;       /* prompt length including BOS */
+  int32_t proprio_dim;  /* 0 = no proprio token */
+  int32_t n_action;     /* action tokens (autoregressive) or block positions (parallel) */
+  int32_t parallel;     /* 0 = autoregressive decode, 1 = parallel action block */
+  int32_t bf16;         /* 1 = weights are bf16 bit patterns and storage rounds to bf16 */
+  double rope_theta, rms_eps;
+} orc_dims;
+
+/* Host pointers.  Element type: uint16 bf16 bit patterns if dims.bf16, else float.
+ * Matrices are row-major [out][in]; per-layer entries are arrays of n_layers pointers. */
+typedef struct orc_weights {
+  const void* tok_emb;     /* [vocab][hidden] */
+  const void* patch_w;     /* [hidden][patch*patch*3], column (y*patch + x)*3 + c */
+  const void* proprio_w;   /* [hidden][proprio_dim] or NULL */
+  const void* action_emb;  /* [n_action][hidden] (parallel) or NULL */
+  const void* const* attn_norm;
+  const void* const* wq;
+  const void* const* wk;
+  const void* const* wv;
+  const void* const* wo;
+  const void* const* ffn_norm;
+  const void* const* w_gate;
+  const void* const* w_up;
+  const void* const* w_down;
+  const void* final_norm;
+  const void* lm_head;     /* [vocab][hidden]; rows vocab-n_bins .. vocab-1 are read */
+} orc_weights;
+
+typedef struct orc_opts {
+  int32_t margin_kind;          /* 0 = probability p1 - p2 (Eq. 1), 1 = logit gap l1 - l2 */
+  int32_t reduction;            /* 0 = mean over the action tokens (Eq. 1), 1 = minimum */
+  const int8_t* gate_override;  /* [B]: -1 gate, 0 force cached, 1 force full; NULL = gate */
+  const int32_t* forced_ids;    /* [B][n_action] bins fed back in decode; NULL = argmax */
+} orc_opts;
+
+typedef struct orc_out {
+  int32_t* action_ids;  /* [B][n_action] argmax bin (0 .. n_bins-1) */
+  double* margins;      /* [B][n_action] p1 - p2 */
+  double* logit_gap;    /* [B][n_action] l1 - l2 */
+  double* logits;       /* [B][n_action][n_bins] or NULL */
+  uint8_t* recomputed;  /* [B] 1 = the full branch ran */
+  uint8_t* gate_auto;   /* [B] what the gate alone decided */
+  double* step_margin;  /* [B] m_t (reduced per-token signal) */
+  uint8_t* static_mask; /* [B][n_visual] or NULL */
+  int32_t* idx;         /* [B][S] recompute order or NULL */
+  int32_t* M;           /* [B][n_layers] rows recomputed per layer or NULL */
+} orc_out;
+
+typedef struct orc_ctx orc_ctx;
+typedef struct orc_cache orc_cache;
+
+enum { ORC_OK = 0, ORC_ERR_ARG = -1, ORC_ERR_OOM = -3 };
+
+int orc_create(const orc_dims* d, const orc_weights* w, orc_ctx** out);
+void orc_destroy(orc_ctx* c);
+int orc_cache_new(const orc_ctx* c, int batch, orc_cache** out);
+void orc_cache_free(orc_cache* k);
+int orc_reset(orc_cache* k, int seq);  /* seq = -1: every sequence */
+int orc_step(orc_ctx* c, orc_cache* k, const uint8_t* frames, const int32_t* prompt_ids,
+             const float* proprio, uint32_t tau_num, uint32_t tau_den, double tau_margin,
+             const uint16_t* reuse_permille, const orc_opts* opts, orc_out* out);
+/* Copies one layer of sequence `seq`'s cache: kind 0 = K, 1 = V ([cache_len][hidden]),
+ * 2 = H (layer inputs, [S][hidden]).  Values as stored (float). */
+int orc_cache_read(const orc_cache* k, int seq, int kind, int layer, float* dst);
+int orc_cache_state(const orc_cache* k, int seq, double* m_prev, int* valid);
+
+/* Pieces exposed for pin tests. */
+void orc_patch_stats(const orc_dims* d, const uint8_t* frame, const uint8_t* prev, int v,
+                     int64_t* dot, int64_t* na, int64_t* nb);
+int orc_is_static(int64_t dot, int64_t na, int64_t nb, uint32_t num, uint32_t den);
+int orc_more_similar(int64_t d_i, int64_t na_i, int64_t nb_i, int i,
+                     int64_t d_j, int64_t na_j, int64_t nb_j, int j);
+int orc_select(const orc_dims* d, const uint8_t* frame, const uint8_t* prev, int have_prev,
+               uint32_t num, uint32_t den, const uint16_t* permille, int full,
+               uint8_t* mask, int32_t* idx, int32_t* M);
+void orc_margin(const double* logits, int n, int32_t* argmax, double* pmargin, double* lgap);
+double orc_round_bf16(double v);
+void orc_rope_table(const orc_dims* d, int n_pos, float* cos_t, float* sin_t);
+
+#ifdef __cplusplus
+}
+#endif
+#endif
