@@ -1,0 +1,175 @@
+/*
+ * vlac — one Gated VLA-Cache step on a single GB300 (sm_103a).
+ *
+ * The step is Algorithm 1 of the paper: a logit-margin gate on the previous
+ * step's Eq. (1) margin either invalidates the cache and runs the full
+ * forward pass, or detects static patches (Sec. III-B, Stage 1), applies the
+ * per-layer reuse proportion (Stage 3) and recomputes only the remaining
+ * tokens; then the D action tokens are decoded and their margins reduced.
+ *
+ * Conventions for every call:
+ *   - Return value: VLAC_OK (0) or a negative VLAC_ERR_* code.  No call
+ *     aborts or exits the process.  vlac_strerror() names a code.
+ *   - "device" pointers are CUDA device memory of the context's device;
+ *     "host" pointers are ordinary host memory read during the call.
+ *   - Work is enqueued asynchronously on `stream` (a cudaStream_t, NULL =
+ *     the legacy default stream); outputs are valid once the stream has
+ *     reached the end of the call's work.
+ *   - Errors detected on the device (bad token ids, a bounded wait that gave
+ *     up) are latched in a per-context error word; the next call on the
+ *     context returns them, and vlac_sync_error() waits for the device and
+ *     returns them.
+ */
+#ifndef VLAC_H
+#define VLAC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define VLAC_OK 0
+#define VLAC_ERR_INVALID_ARG (-1)  /* a pointer, size or value is out of its documented range */
+#define VLAC_ERR_CUDA (-2)         /* a CUDA runtime call or kernel launch failed */
+#define VLAC_ERR_OOM (-3)          /* device or host allocation failed */
+#define VLAC_ERR_TIMEOUT (-4)      /* a bounded device-side wait gave up */
+#define VLAC_ERR_DEVICE_CHECK (-5) /* a device-side bounds check rejected an input value */
+#define VLAC_ERR_STATE (-6)        /* cache and context (or batch) do not match */
+#define VLAC_ERR_UNSUPPORTED (-7)  /* valid dims this build does not implement */
+
+#define VLAC_F32 0  /* fp32 weights and activations */
+#define VLAC_BF16 1 /* bf16 weights and GEMM inputs, fp32 residual stream and accumulation */
+
+#define VLAC_MARGIN_PROB 0  /* gate signal p1 - p2 of the softmax over the action bins (Eq. 1) */
+#define VLAC_MARGIN_LOGIT 1 /* gate signal l1 - l2, the top-2 logit gap */
+#define VLAC_REDUCE_DEFAULT (-1) /* mean for autoregressive decode (Eq. 1), min for a parallel block */
+#define VLAC_REDUCE_MEAN 0
+#define VLAC_REDUCE_MIN 1
+
+/* Backbone and input geometry (Sec. III-A).  Token layout of a sequence:
+ * position 0 = BOS (prompt id 0), 1..n_visual = patches (view-major, row-major),
+ * then one proprio token if proprio_dim > 0, then prompt ids 1..n_text-1, then,
+ * if parallel, n_action action positions computed in the same pass. */
+typedef struct vlac_dims {
+  int32_t n_layers, hidden, n_heads, head_dim, ffn, vocab, n_bins;
+  int32_t img_h, img_w, patch, n_views;
+  int32_t n_text;      /* prompt length including BOS (>= 2 when parallel == 0) */
+  int32_t proprio_dim; /* 0 = no proprio token */
+  int32_t n_action;    /* D action tokens (autoregressive) or block positions (parallel) */
+  int32_t parallel;    /* 0 = autoregressive decode of D tokens, 1 = one parallel block */
+  int32_t dtype;       /* VLAC_F32 or VLAC_BF16 */
+  float rope_theta, rms_eps;
+  int32_t max_batch;   /* largest batch a cache of this context may hold */
+} vlac_dims;
+
+/* Weights: device pointers of element type dims.dtype, row-major [out][in].
+ * Per-layer members are HOST arrays of n_layers device pointers.  All are read
+ * during vlac_create (copied / repacked), so the caller may free them after. */
+typedef struct vlac_weights {
+  const void* tok_emb;    /* [vocab][hidden] */
+  const void* patch_w;    /* [hidden][patch*patch*3], column index (y*patch + x)*3 + c */
+  const void* proprio_w;  /* [hidden][proprio_dim], or NULL when proprio_dim == 0 */
+  const void* action_emb; /* [n_action][hidden] when parallel, else NULL */
+  const void* const* attn_norm; /* [hidden] RMSNorm gains */
+  const void* const* wq;        /* [hidden][hidden] */
+  const void* const* wk;
+  const void* const* wv;
+  const void* const* wo;
+  const void* const* ffn_norm;
+  const void* const* w_gate;    /* [ffn][hidden] */
+  const void* const* w_up;      /* [ffn][hidden] */
+  const void* const* w_down;    /* [hidden][ffn] */
+  const void* final_norm;       /* [hidden] */
+  const void* lm_head;          /* [vocab][hidden]; only rows vocab-n_bins .. vocab-1 are read */
+} vlac_weights;
+
+/* Stage-1 threshold as an exact fraction: a patch is static iff cos > num/den. */
+typedef struct vlac_rational {
+  uint32_t num, den; /* den > 0 */
+} vlac_rational;
+
+typedef struct vlac_step_opts {
+  int32_t margin_kind;         /* VLAC_MARGIN_PROB (default) or VLAC_MARGIN_LOGIT */
+  int32_t reduction;           /* VLAC_REDUCE_* */
+  const int8_t* gate_override; /* device [B]: -1 gate decides, 0 force the cached branch,
+                                  1 force the full branch; NULL = gate decides.  An empty
+                                  cache always runs the full branch. */
+  const int32_t* forced_ids;   /* device [B][n_action]: bins fed back during autoregressive
+                                  decode instead of the argmax (lock-step replay); NULL = argmax */
+} vlac_step_opts;
+
+/* Device output buffers of one step (B = the cache's batch, D = n_action,
+ * S = positions of the prefix pass, Nv = visual tokens, L = n_layers). */
+typedef struct vlac_step_out {
+  int32_t* action_ids;  /* [B][D] argmax bin, 0 .. n_bins-1 (token id vocab-n_bins+bin) */
+  float* margins;       /* [B][D] p1 - p2 of each action token (Eq. 1 summand) */
+  float* logit_gap;     /* [B][D] l1 - l2 */
+  uint8_t* recomputed;  /* [B] 1 = the full branch ran this step */
+  float* step_margin;   /* [B] m_t: the reduced signal that gates the next step */
+  uint8_t* gate_auto;   /* optional [B]: what the gate alone decided */
+  float* logits;        /* optional [B][D][n_bins] action-bin logits (fp32) */
+  uint8_t* static_mask; /* optional [B][Nv] Stage-1 result (0 without a previous frame) */
+  int32_t* idx;         /* optional [B][S] recompute order: rows of layer l are idx[0..M[l]) */
+  int32_t* M;           /* optional [B][L] rows recomputed at each layer */
+} vlac_step_out;
+
+typedef struct vlac_ctx vlac_ctx;
+typedef struct vlac_cache vlac_cache;
+
+/* Validates dims, copies and repacks the weights into device memory owned by
+ * the context, builds RoPE tables and TMA descriptors, and allocates the
+ * step workspace for dims.max_batch sequences.  *out is set on success. */
+int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ctx** out);
+int vlac_destroy(vlac_ctx* ctx);
+
+/* Bytes of device memory a cache for `batch` (1 .. max_batch) sequences needs:
+ * per sequence the K/V of every layer and position, the fp32 input of every
+ * layer for the prefix positions (tokens that rejoin at a deeper layer start
+ * from it), the previous frame, m_{t-1} and a valid flag. */
+int vlac_cache_bytes(const vlac_ctx* ctx, int batch, size_t* bytes);
+/* Formats caller-owned device memory (>= vlac_cache_bytes, 256-byte aligned)
+ * as an empty cache; the memory must outlive the cache handle.  Synchronous. */
+int vlac_cache_init(vlac_ctx* ctx, void* dev_mem, size_t bytes, int batch, vlac_cache** out);
+int vlac_cache_destroy(vlac_cache* cache);
+
+/* One step of Algorithm 1 for every sequence of the cache.
+ *   frames:          device [B][n_views][img_h][img_w][3] uint8 (HWC)
+ *   prompt_ids:      device [B][n_text] int32 token ids (BOS first)
+ *   proprio:         device [B][proprio_dim] fp32, NULL when proprio_dim == 0
+ *   tau_sim:         Stage-1 threshold (static iff cos > num/den)
+ *   tau_margin:      the gate fires iff m_{t-1} < tau_margin (strict)
+ *   reuse_permille:  host [n_layers]: k_l = floor(permille[l] * |static| / 1000)
+ *                    static patches (the most similar) are reused at layer l; each <= 1000
+ *   opts:            NULL = defaults
+ *   out:             device output buffers (required members non-NULL)
+ * Returns VLAC_ERR_STATE if the cache belongs to another context. */
+int vlac_step(vlac_ctx* ctx, vlac_cache* cache, const uint8_t* frames, const int32_t* prompt_ids,
+              const float* proprio, vlac_rational tau_sim, float tau_margin,
+              const uint16_t* reuse_permille, const vlac_step_opts* opts, const vlac_step_out* out,
+              void* stream);
+
+/* Invalidates sequence `seq` (-1 = all): its next step runs the full pass as if
+ * no cache existed (Algorithm 1, cache invalidation). */
+int vlac_reset(vlac_cache* cache, int seq, void* stream);
+
+/* Waits for the context's device work and returns (and clears) the latched
+ * device error word. */
+int vlac_sync_error(vlac_ctx* ctx);
+
+/* Kernels this context has launched so far (every launch of the library's own kernels). */
+uint64_t vlac_launch_count(const vlac_ctx* ctx);
+
+/* Self-test of the bounded device wait: one kernel waits on an mbarrier that
+ * nothing completes, for at most `spin_limit` polls, then records
+ * VLAC_ERR_TIMEOUT in the error word and returns.  Synchronous; returns the
+ * recorded status (VLAC_ERR_TIMEOUT when the wait gave up). */
+int vlac_selftest_wait(vlac_ctx* ctx, uint32_t spin_limit);
+
+const char* vlac_strerror(int code);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* VLAC_H */

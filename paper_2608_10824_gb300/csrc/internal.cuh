@@ -1,0 +1,143 @@
+// Internal declarations shared by the CUDA translation units of libvlac.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/vlac.h"
+
+namespace vlac {
+
+typedef __nv_bfloat16 bf16;
+
+constexpr int kMaxLayers = 256;
+
+// Per-step scalars, written to device memory before the step's kernels run.
+struct StepParams {
+  uint32_t tau_num, tau_den;
+  float tau_margin;
+  int32_t margin_kind;
+  int32_t reduction;  // resolved: 0 mean, 1 min
+  int32_t has_override;
+  int32_t has_forced;
+  int32_t pad;
+  uint16_t permille[kMaxLayers];
+};
+
+// A set of rows processed by one layer: per sequence b, rows i < count_b with
+// count_b = off[b+1] - off[b]; the compacted row index is off[b] + i, the
+// token position is idx[b * idx_stride + i], and the fp32 residual row lives at
+// X + (b * idx_stride + i) * hidden.
+struct Rows {
+  const int* off;
+  const int* idx;
+  int idx_stride;
+  float* X;
+};
+
+// ---- scalar helpers --------------------------------------------------------
+template <typename T> __device__ __forceinline__ float to_f(T v);
+template <> __device__ __forceinline__ float to_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ float to_f<bf16>(bf16 v) { return __bfloat162float(v); }
+template <typename T> __device__ __forceinline__ T from_f(float v);
+template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
+
+__device__ __forceinline__ void set_error(int* err, int code) {
+  if (err) atomicCAS(err, 0, code);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// Block-wide sum in a fixed order (warp butterflies, then warp 0 over the
+// per-warp partials).  `red` holds >= 32 floats.  All threads get the result.
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  v = warp_sum(v);
+  __syncthreads();
+  if (lane == 0) red[w] = v;
+  __syncthreads();
+  float t = (threadIdx.x < (unsigned)nw) ? red[threadIdx.x] : 0.f;
+  if (w == 0) {
+    t = warp_sum(t);
+    if (lane == 0) red[0] = t;
+  }
+  __syncthreads();
+  float r = red[0];
+  __syncthreads();
+  return r;
+}
+
+}  // namespace vlac
+
+// ---- launchers (defined in the kernel translation units) -------------------
+namespace vlac {
+
+void launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid,
+                        const StepParams* prm, int B, int n_views, int img_h, int img_w, int patch,
+                        int3* stats, uint8_t* mask, uint8_t* user_mask, cudaStream_t st);
+void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
+                   const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
+                   int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
+                   uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
+                   cudaStream_t st);
+
+template <typename T>
+void launch_im2col(Rows rows, int B, int S, const uint8_t* frames, int n_views, int img_h, int img_w,
+                   int patch, int kpad, T* col, cudaStream_t st);
+template <typename T>
+void launch_embed(Rows rows, int B, int S, int hidden, int Nv, int P, int has_proprio, int proprio_dim,
+                  int n_text, int vocab, const int32_t* prompt, const float* proprio, const T* tok_emb,
+                  const float* patch_part, const T* proprio_w, const T* action_emb, int* err,
+                  cudaStream_t st);
+template <typename T>
+void launch_layer_in(Rows rows, const int* off_prev, int B, int S, int hidden, float* H, size_t h_seq_stride,
+                     const T* gain, float eps, T* A, cudaStream_t st);
+template <typename T>
+void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, int splits,
+                         size_t split_stride, const float* rope_cos, const float* rope_sin, T* Q, T* Kc,
+                         T* Vc, size_t kv_seq_stride, int Tc, cudaStream_t st);
+template <typename T>
+void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part, int splits,
+                          size_t split_stride, const T* gain, float eps, T* A, cudaStream_t st);
+template <typename T>
+void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, int splits, size_t split_stride, T* G,
+                   cudaStream_t st);
+void launch_residual(Rows rows, int B, int S, int hidden, const float* part, int splits, size_t split_stride,
+                     cudaStream_t st);
+template <typename T>
+void launch_attention(Rows rows, int B, int S, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc,
+                      size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, T* O, cudaStream_t st);
+template <typename T>
+void launch_head(const float* X, const int* row_of_seq, size_t x_seq_stride, int rows_per_seq, int B,
+                 int hidden, int n_bins, const T* final_norm, const T* head_w, float eps, int D, int tok0,
+                 int32_t* ids, float* margins, float* gaps, float* logits, cudaStream_t st);
+template <typename T>
+void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
+                         const int32_t* ids, const int32_t* forced, const StepParams* prm, float* Xd,
+                         int* idx_dec, int* err, cudaStream_t st);
+void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps,
+                   float* m_prev, uint8_t* valid, float* user_step_margin, cudaStream_t st);
+
+// GEMMs: out[s][m][n] = sum over split s of A[m][k] * W[n][k]; rows m < *m_ptr.
+void launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
+                    int splits, float* out, int* err, uint32_t wait_limit, cudaStream_t st);
+template <typename T>
+void launch_gemm_simt(const T* A, const T* W, const int* m_ptr, int m_cap, int N, int K, float* out,
+                      cudaStream_t st);
+template <typename T>
+void launch_gemv(const T* W, int N, int K, const T* x, int nb, float* y, cudaStream_t st);
+int launch_wait_selftest(int* err, uint32_t spin_limit, cudaStream_t st);
+
+}  // namespace vlac

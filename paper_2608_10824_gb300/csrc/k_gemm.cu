@@ -1,0 +1,506 @@
+// Projections of the layer loop: out[s][m][n] = sum_k A[m][k] * W[n][k] over
+// the k range of split s.  Three kernels, one per regime:
+//   - gemm_tc:   bf16 prefix pass (M = recomputed rows, device-resident),
+//                tcgen05 MMA with fp32 accumulators in TMEM, operands staged
+//                by TMA into 128B-swizzled shared memory.  The weight tile is
+//                the 128-row MMA operand and the token rows are the N side
+//                ("swap-AB"), so one weight tile feeds every recomputed row.
+//   - gemv:      decode passes (M = batch <= 8): HBM-bound weight streaming
+//                with 16-byte non-allocating loads and fp32 FMAs.
+//   - gemm_simt: the fp32 tiny model.
+#include "internal.cuh"
+
+namespace vlac {
+
+// =============================================================================
+// tcgen05 GEMM
+// =============================================================================
+namespace tc {
+
+constexpr int kBM = 128;        // weight rows per CTA (MMA M)
+constexpr int kBK = 64;         // K elements per stage = one 128-byte swizzle row
+constexpr int kBoxRows = 32;    // token rows per TMA box of the activation operand
+constexpr int kMaxTok = 512;    // token columns per pass (TMEM has 512 fp32 columns)
+constexpr int kMaxStages = 8;
+constexpr int kWTileBytes = kBM * kBK * 2;  // 16 KB
+constexpr int kSmemBytes = 212 * 1024;      // dynamic shared memory (tiles only)
+constexpr int kThreads = 192;               // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase with `parity` to complete.  Gives up after
+// `limit` polls or when another role raised `abort`; returns false then.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t limit, volatile int* abort) {
+  for (uint32_t i = 0; i < limit; ++i) {
+    if (mbar_test(bar, parity)) return true;
+    if (*abort) return false;
+  }
+  return false;
+}
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, int x, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
+          "r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// D[tmem] (+)= A[smem] * B[smem]^T, bf16 inputs, fp32 accumulate.
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrives on `bar` once every MMA issued so far by this thread has completed.
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+}
+
+// Shared-memory matrix descriptor of a K-major operand in 128B-swizzled rows
+// (8-row groups 1024 bytes apart).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);        // start address
+  d |= (uint64_t)1 << 16;                          // leading byte offset (unused for swizzled K-major)
+  d |= (uint64_t)((1024u >> 4) & 0x3FFFu) << 32;   // stride byte offset: next 8-row group
+  d |= (uint64_t)1 << 46;                          // descriptor version
+  d |= (uint64_t)2 << 61;                          // 128-byte swizzle
+  return d;
+}
+// Instruction descriptor: bf16 x bf16 -> fp32, both operands K-major, M = 128.
+__device__ __forceinline__ uint32_t idesc_bf16(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
+                   const int* __restrict__ m_ptr, int m_cap, int N, int k_chunks, int chunks_per_split,
+                   float* __restrict__ out, size_t split_stride, int* __restrict__ err, uint32_t wait_limit) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t acc_full, acc_empty;
+  __shared__ uint32_t tmem_slot;
+  __shared__ __align__(8) uint64_t drain_bar;
+  __shared__ int abort_flag, never;
+  __shared__ int prod_cnt[kMaxStages], cons_cnt[kMaxStages];
+  __shared__ uint32_t last_par[kMaxStages];
+
+  uint8_t* tiles = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int M = min(*m_ptr, m_cap);
+  if (M <= 0) return;
+  const int n0 = blockIdx.x * kBM;
+  const int kc0 = blockIdx.y * chunks_per_split;
+  const int kc1 = min(kc0 + chunks_per_split, k_chunks);
+  const int nk = kc1 - kc0;
+  if (nk <= 0) return;
+  const int tok_layout = ((min(M, kMaxTok) + kBoxRows - 1) / kBoxRows) * kBoxRows;
+  const uint32_t stage_bytes = kWTileBytes + (uint32_t)tok_layout * 128u;
+  const int n_stages = min(kMaxStages, (int)((kSmemBytes - 1024) / stage_bytes));
+  const int n_pass = (M + kMaxTok - 1) / kMaxTok;
+  uint32_t ncols = 32;
+  while (ncols < (uint32_t)tok_layout) ncols <<= 1;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kMaxStages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+      prod_cnt[s] = 0;
+      cons_cnt[s] = 0;
+      last_par[s] = 0;
+    }
+    mbar_init(&acc_full, 1);
+    mbar_init(&acc_empty, 4);
+    mbar_init(&drain_bar, 1);
+    abort_flag = 0;
+    never = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    tmem_alloc(&tmem_slot, ncols);
+    tmem_relinquish();
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem_base = tmem_slot;
+  volatile int* abort = &abort_flag;
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int pass = 0; pass < n_pass && !*abort; ++pass) {
+        const int row0 = pass * kMaxTok;
+        const int rows = min(M - row0, kMaxTok);
+        const int nbox = (rows + kBoxRows - 1) / kBoxRows;
+        for (int kc = kc0; kc < kc1; ++kc) {
+          if (!mbar_wait(&empty_bar[stage], phase ^ 1u, wait_limit, abort)) {
+            set_error(err, VLAC_ERR_TIMEOUT);
+            *abort = 1;
+            break;
+          }
+          uint8_t* wt = tiles + (size_t)stage * stage_bytes;
+          uint8_t* at = wt + kWTileBytes;
+          mbar_expect_tx(&full_bar[stage], kWTileBytes + (uint32_t)nbox * kBoxRows * 128u);
+          tma_load_2d(wt, &tmW, kc * kBK, n0, &full_bar[stage]);
+          for (int bx = 0; bx < nbox; ++bx)
+            tma_load_2d(at + (size_t)bx * kBoxRows * 128, &tmA, kc * kBK, row0 + bx * kBoxRows, &full_bar[stage]);
+          prod_cnt[stage] += 1;
+          last_par[stage] = phase;
+          if (++stage == n_stages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int pass = 0; pass < n_pass && !*abort; ++pass) {
+        const int rows = min(M - pass * kMaxTok, kMaxTok);
+        if (pass > 0 && !mbar_wait(&acc_empty, (uint32_t)(pass - 1) & 1u, wait_limit, abort)) {
+          set_error(err, VLAC_ERR_TIMEOUT);
+          *abort = 1;
+          break;
+        }
+        fence_after();
+        for (int i = 0; i < nk; ++i) {
+          if (!mbar_wait(&full_bar[stage], phase, wait_limit, abort)) {
+            set_error(err, VLAC_ERR_TIMEOUT);
+            *abort = 1;
+            break;
+          }
+          cons_cnt[stage] += 1;
+          fence_after();
+          const uint32_t wt = smem_u32(tiles + (size_t)stage * stage_bytes);
+          const uint32_t at = wt + kWTileBytes;
+#pragma unroll
+          for (int k16 = 0; k16 < kBK / 16; ++k16) {
+            const uint64_t adesc = sw128_desc(wt + k16 * 32);
+            for (int sub = 0; sub * 256 < rows; ++sub) {
+              const int n = min(256, ((rows - sub * 256 + 15) / 16) * 16);
+              const uint64_t bdesc = sw128_desc(at + sub * 256 * 128 + k16 * 32);
+              umma_bf16(tmem_base + sub * 256, adesc, bdesc, idesc_bf16(n), (i > 0 || k16 > 0) ? 1u : 0u);
+            }
+          }
+          umma_commit(&empty_bar[stage]);
+          if (++stage == n_stages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        umma_commit(&acc_full);
+      }
+      if (*abort) {
+        // every MMA issued so far must finish before TMEM and the tiles go away
+        umma_commit(&drain_bar);
+        mbar_wait(&drain_bar, 0, wait_limit, &never);
+      }
+    }
+  } else {
+    // ---------------- epilogue: TMEM -> fp32 partials ----------------
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int n = n0 + q * 32 + lane;
+    float* dst = out + (size_t)blockIdx.y * split_stride;
+    for (int pass = 0; pass < n_pass; ++pass) {
+      const int row0 = pass * kMaxTok;
+      const int rows = min(M - row0, kMaxTok);
+      bool ok = true;
+      if (lane == 0) ok = mbar_wait(&acc_full, (uint32_t)pass & 1u, wait_limit, abort);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) {
+        if (lane == 0) {
+          set_error(err, VLAC_ERR_TIMEOUT);
+          *abort = 1;
+        }
+        break;
+      }
+      fence_after();
+      for (int c0 = 0; c0 < rows; c0 += 16) {
+        float v[16];
+        tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, v);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int m = row0 + c0 + j;
+          if (m < M) dst[(size_t)m * N + n] = v[j];
+        }
+      }
+      fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty);
+    }
+  }
+
+  __syncthreads();
+  if (threadIdx.x == 0 && abort_flag) {
+    // let every bulk copy that was issued but not consumed land before exit
+    for (int s = 0; s < n_stages; ++s)
+      if (prod_cnt[s] > cons_cnt[s]) mbar_wait(&full_bar[s], last_par[s], wait_limit, &never);
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, ncols);
+}
+
+}  // namespace tc
+
+void launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
+                    int splits, float* out, int* err, uint32_t wait_limit, cudaStream_t st) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaFuncSetAttribute(tc::gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, tc::kSmemBytes);
+    attr_set = true;
+  }
+  const int k_chunks = K / tc::kBK;
+  const int cps = (k_chunks + splits - 1) / splits;
+  dim3 grid(N / tc::kBM, splits);
+  tc::gemm_tc_kernel<<<grid, tc::kThreads, tc::kSmemBytes, st>>>(*tmA, *tmW, m_ptr, m_cap, N, k_chunks, cps, out,
+                                                                 (size_t)m_cap * N, err, wait_limit);
+}
+
+// =============================================================================
+// Decode GEMV: y[b][n] = sum_k x[b][k] * W[n][k] for nb <= 8 rows of x.
+// =============================================================================
+
+__device__ __forceinline__ uint4 ld_stream(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+template <typename T> struct Vec;
+template <> struct Vec<bf16> { static constexpr int n = 8; };
+template <> struct Vec<float> { static constexpr int n = 4; };
+
+template <typename T>
+__device__ __forceinline__ void unpack(const uint4& u, float* f) {
+  if constexpr (sizeof(T) == 2) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      f[2 * i] = __uint_as_float(w[i] << 16);
+      f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+  } else {
+    f[0] = __uint_as_float(u.x);
+    f[1] = __uint_as_float(u.y);
+    f[2] = __uint_as_float(u.z);
+    f[3] = __uint_as_float(u.w);
+  }
+}
+
+// Each warp owns ROWS consecutive weight rows; lanes stride over K in
+// 16-byte vectors, UNROLL vectors in flight per row.  Fixed reduction order.
+template <typename T, int NB, int ROWS, int UNROLL>
+__global__ void __launch_bounds__(256) gemv_kernel(const T* __restrict__ W, int N, int K, const T* __restrict__ x,
+                                                   float* __restrict__ y) {
+  constexpr int V = Vec<T>::n;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row0 = (blockIdx.x * (blockDim.x >> 5) + warp) * ROWS;
+  if (row0 >= N) return;
+  const int kv = K / V;  // vectors per row
+  float acc[ROWS][NB];
+#pragma unroll
+  for (int r = 0; r < ROWS; ++r)
+#pragma unroll
+    for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
+  const uint4* Wv = reinterpret_cast<const uint4*>(W);
+  const uint4* xv = reinterpret_cast<const uint4*>(x);
+  for (int k0 = lane; k0 < kv; k0 += 32 * UNROLL) {
+    uint4 wr[UNROLL][ROWS];
+#pragma unroll
+    for (int u = 0; u < UNROLL; ++u) {
+      const int k = k0 + u * 32;
+#pragma unroll
+      for (int r = 0; r < ROWS; ++r)
+        if (k < kv && row0 + r < N) wr[u][r] = ld_stream(Wv + (size_t)(row0 + r) * kv + k);
+        else wr[u][r] = make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < UNROLL; ++u) {
+      const int k = k0 + u * 32;
+      if (k >= kv) break;
+#pragma unroll
+      for (int b = 0; b < NB; ++b) {
+        float xf[V];
+        unpack<T>(__ldg(xv + (size_t)b * kv + k), xf);
+#pragma unroll
+        for (int r = 0; r < ROWS; ++r) {
+          float wf[V];
+          unpack<T>(wr[u][r], wf);
+#pragma unroll
+          for (int e = 0; e < V; ++e) acc[r][b] = fmaf(wf[e], xf[e], acc[r][b]);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < ROWS; ++r)
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      const float s = warp_sum(acc[r][b]);
+      if (lane == 0 && row0 + r < N) y[(size_t)b * N + row0 + r] = s;
+    }
+}
+
+template <typename T, int NB>
+static void gemv_nb(const T* W, int N, int K, const T* x, float* y, cudaStream_t st) {
+  constexpr int ROWS = NB <= 2 ? 2 : 1;
+  constexpr int UNROLL = NB <= 2 ? 4 : 2;
+  const int warps = 8;
+  const int blocks = (N + warps * ROWS - 1) / (warps * ROWS);
+  gemv_kernel<T, NB, ROWS, UNROLL><<<blocks, warps * 32, 0, st>>>(W, N, K, x, y);
+}
+
+template <typename T>
+void launch_gemv(const T* W, int N, int K, const T* x, int nb, float* y, cudaStream_t st) {
+  switch (nb) {
+    case 1: gemv_nb<T, 1>(W, N, K, x, y, st); break;
+    case 2: gemv_nb<T, 2>(W, N, K, x, y, st); break;
+    case 3: gemv_nb<T, 3>(W, N, K, x, y, st); break;
+    case 4: gemv_nb<T, 4>(W, N, K, x, y, st); break;
+    case 5: gemv_nb<T, 5>(W, N, K, x, y, st); break;
+    case 6: gemv_nb<T, 6>(W, N, K, x, y, st); break;
+    case 7: gemv_nb<T, 7>(W, N, K, x, y, st); break;
+    default: gemv_nb<T, 8>(W, N, K, x, y, st); break;
+  }
+}
+template void launch_gemv<float>(const float*, int, int, const float*, int, float*, cudaStream_t);
+template void launch_gemv<bf16>(const bf16*, int, int, const bf16*, int, float*, cudaStream_t);
+
+// =============================================================================
+// SIMT GEMM (fp32 tiny model): 64x64 output tile, 4x4 per thread.
+// =============================================================================
+template <typename T>
+__global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A, const T* __restrict__ W,
+                                                        const int* __restrict__ m_ptr, int m_cap, int N, int K,
+                                                        float* __restrict__ out) {
+  __shared__ float As[16][64 + 1];
+  __shared__ float Ws[16][64 + 1];
+  const int M = min(*m_ptr, m_cap);
+  const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
+  if (m0 >= M) return;
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  float acc[4][4] = {};
+  for (int k0 = 0; k0 < K; k0 += 16) {
+    for (int t = threadIdx.x; t < 16 * 64; t += 256) {
+      const int kk = t & 15, rr = t >> 4;
+      const int m = m0 + rr, n = n0 + rr, k = k0 + kk;
+      As[kk][rr] = (m < M && k < K) ? to_f(A[(size_t)m * K + k]) : 0.f;
+      Ws[kk][rr] = (n < N && k < K) ? to_f(W[(size_t)n * K + k]) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < 16; ++kk) {
+      float a[4], w[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        a[i] = As[kk][ty * 4 + i];
+        w[i] = Ws[kk][tx * 4 + i];
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], w[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int m = m0 + ty * 4 + i, n = n0 + tx * 4 + j;
+      if (m < M && n < N) out[(size_t)m * N + n] = acc[i][j];
+    }
+}
+
+template <typename T>
+void launch_gemm_simt(const T* A, const T* W, const int* m_ptr, int m_cap, int N, int K, float* out,
+                      cudaStream_t st) {
+  dim3 grid((N + 63) / 64, (m_cap + 63) / 64);
+  gemm_simt_kernel<T><<<grid, 256, 0, st>>>(A, W, m_ptr, m_cap, N, K, out);
+}
+template void launch_gemm_simt<float>(const float*, const float*, const int*, int, int, int, float*, cudaStream_t);
+
+// =============================================================================
+// Bounded-wait self-test: waits on an mbarrier that nothing completes.
+// =============================================================================
+__global__ void wait_selftest_kernel(int* err, uint32_t limit) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&bar, 1);
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !tc::mbar_wait(&bar, 0, limit, &abort_flag)) set_error(err, VLAC_ERR_TIMEOUT);
+}
+
+int launch_wait_selftest(int* err, uint32_t spin_limit, cudaStream_t st) {
+  wait_selftest_kernel<<<1, 32, 0, st>>>(err, spin_limit);
+  return cudaGetLastError() == cudaSuccess ? 0 : -1;
+}
+
+}  // namespace vlac

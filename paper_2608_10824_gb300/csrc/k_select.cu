@@ -1,0 +1,195 @@
+// Stage 1 (static patch detection) and the gate + Stage-3 selection.
+//
+// Sec. III-B, Stage 1: cosine similarity between corresponding patches of
+// I_t and I_{t-1}; a patch is static when the similarity is above tau.  The
+// similarity vector is the raw uint8 RGB values of the patch, and the
+// comparison against tau = num/den is decided exactly in integers.
+// Algorithm 1: m_{t-1} < theta_m (strict) invalidates the cache and runs the
+// full pass; otherwise Stage 3 reuses, at layer l, the floor(s_l * |S| / 1000)
+// most similar static patches and recomputes the rest.
+#include "internal.cuh"
+
+namespace vlac {
+
+typedef unsigned __int128 u128;
+
+// cos > num/den, exact.  Both patches all-zero: cos = 1; exactly one: cos = 0.
+__device__ __forceinline__ bool cos_above(uint32_t d, uint32_t na, uint32_t nb, uint32_t num, uint32_t den) {
+  if (den == 0) return false;
+  if (na == 0 && nb == 0) return num < den;
+  if (na == 0 || nb == 0 || d == 0) return false;
+  const u128 lhs = (u128)((uint64_t)d * d) * (u128)((uint64_t)den * den);
+  const u128 rhs = (u128)((uint64_t)num * num) * (u128)((uint64_t)na * nb);
+  return lhs > rhs;
+}
+
+// cos^2 as a fraction with a positive denominator.
+__device__ __forceinline__ void cos2_frac(int3 s, uint64_t& n2, uint64_t& d2) {
+  const uint32_t d = (uint32_t)s.x, na = (uint32_t)s.y, nb = (uint32_t)s.z;
+  if (na == 0 && nb == 0) { n2 = 1; d2 = 1; return; }
+  if (na == 0 || nb == 0) { n2 = 0; d2 = 1; return; }
+  n2 = (uint64_t)d * d;
+  d2 = (uint64_t)na * nb;
+}
+
+// Reuse order: patch u precedes patch v when its cosine is higher, ties by index.
+__device__ __forceinline__ bool more_similar(int3 su, int u, int3 sv, int v) {
+  uint64_t nu, du, nv, dv;
+  cos2_frac(su, nu, du);
+  cos2_frac(sv, nv, dv);
+  const u128 l = (u128)nu * dv, r = (u128)nv * du;
+  if (l != r) return l > r;
+  return u < v;
+}
+
+// One warp per (sequence, patch): integer dot product and squared norms.
+__global__ void patch_stats_kernel(const uint8_t* __restrict__ frames, const uint8_t* __restrict__ prev,
+                                   const uint8_t* __restrict__ valid, const StepParams* __restrict__ prm,
+                                   int n_views, int img_h, int img_w, int patch, int Nv, int3* __restrict__ stats,
+                                   uint8_t* __restrict__ mask, uint8_t* __restrict__ user_mask) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int v = blockIdx.x * (blockDim.x >> 5) + warp;
+  const int b = blockIdx.y;
+  if (v >= Nv) return;
+  const size_t fb = (size_t)n_views * img_h * img_w * 3;
+  const uint8_t* fa = frames + (size_t)b * fb;
+  const uint8_t* fp = prev + (size_t)b * fb;
+  const int gw = img_w / patch, gh = img_h / patch;
+  const int view = v / (gw * gh), r = v % (gw * gh), py = r / gw, px = r % gw;
+  const int n = patch * patch * 3, row_bytes = patch * 3;
+  uint32_t d = 0, na = 0, nb = 0;
+  for (int e = lane; e < n; e += 32) {
+    const int ry = e / row_bytes, rem = e - ry * row_bytes;
+    const size_t o = ((size_t)(view * img_h + py * patch + ry) * img_w + (size_t)px * patch) * 3 + rem;
+    const uint32_t a = fa[o], c = fp[o];
+    d += a * c;
+    na += a * a;
+    nb += c * c;
+  }
+  d = __reduce_add_sync(0xffffffffu, d);
+  na = __reduce_add_sync(0xffffffffu, na);
+  nb = __reduce_add_sync(0xffffffffu, nb);
+  if (lane == 0) {
+    const bool st = valid[b] && cos_above(d, na, nb, prm->tau_num, prm->tau_den);
+    stats[(size_t)b * Nv + v] = make_int3((int)d, (int)na, (int)nb);
+    mask[(size_t)b * Nv + v] = st;
+    if (user_mask) user_mask[(size_t)b * Nv + v] = st;
+  }
+}
+
+// One block per sequence: gate decision, reuse ranking and the ordered
+// recompute list.  idx = [non-static positions ascending] ++ [static patches,
+// least similar first], so the rows recomputed at layer l are idx[0 .. M[l]).
+__global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __restrict__ mask,
+                              const uint8_t* __restrict__ valid, const float* __restrict__ m_prev,
+                              const StepParams* __restrict__ prm, const int8_t* __restrict__ override_,
+                              int Nv, int S, int L, int P, int parallel, int n_action, uint8_t* __restrict__ full_out,
+                              int* __restrict__ idx, int* __restrict__ M, int* __restrict__ emit_slot,
+                              uint8_t* __restrict__ user_recomputed, uint8_t* __restrict__ user_gate_auto,
+                              int* __restrict__ user_idx, int* __restrict__ user_M) {
+  extern __shared__ uint8_t smem[];
+  int3* s_st = reinterpret_cast<int3*>(smem);
+  int* s_rank = reinterpret_cast<int*>(s_st + Nv);
+  uint8_t* s_stat = reinterpret_cast<uint8_t*>(s_rank + Nv);
+  __shared__ int s_full;
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+
+  if (tid == 0) {
+    const bool ok = valid[b] != 0;
+    const bool gate = !ok || m_prev[b] < prm->tau_margin;
+    bool full = gate;
+    if (prm->has_override && override_ && override_[b] >= 0) full = override_[b] != 0;
+    if (!ok) full = true;
+    s_full = full;
+    full_out[b] = full;
+    if (user_recomputed) user_recomputed[b] = full;
+    if (user_gate_auto) user_gate_auto[b] = gate;
+  }
+  for (int v = tid; v < Nv; v += blockDim.x) {
+    s_st[v] = stats[(size_t)b * Nv + v];
+    s_stat[v] = mask[(size_t)b * Nv + v];
+  }
+  __syncthreads();
+  const bool full = s_full != 0;
+  int* idx_b = idx + (size_t)b * S;
+  if (full) {
+    for (int i = tid; i < S; i += blockDim.x) idx_b[i] = i;
+    for (int l = tid; l < L; l += blockDim.x) M[(size_t)b * L + l] = S;
+    if (tid == 0) emit_slot[b] = parallel ? P : P - 1;
+  }
+  __syncthreads();
+  if (!full) {
+    // |S| and the reuse rank of every static patch (0 = most similar)
+    __shared__ int s_ns;
+    if (tid == 0) s_ns = 0;
+    __syncthreads();
+    int local = 0;
+    for (int v = tid; v < Nv; v += blockDim.x) local += s_stat[v];
+    if (local) atomicAdd(&s_ns, local);
+    for (int v = tid; v < Nv; v += blockDim.x) {
+      if (!s_stat[v]) continue;
+      int rank = 0;
+      const int3 sv = s_st[v];
+      for (int u = 0; u < Nv; ++u)
+        if (u != v && s_stat[u] && more_similar(s_st[u], u, sv, v)) ++rank;
+      s_rank[v] = rank;
+    }
+    __syncthreads();
+    const int nS = s_ns, n_always = S - nS;
+    if (warp == 0) {
+      int base = 0;
+      for (int p0 = 0; p0 < S; p0 += 32) {
+        const int p = p0 + lane;
+        const bool always = p < S && !(p >= 1 && p <= Nv && s_stat[p - 1]);
+        const unsigned bal = __ballot_sync(0xffffffffu, always);
+        if (always) idx_b[base + __popc(bal & ((1u << lane) - 1u))] = p;
+        base += __popc(bal);
+      }
+    }
+    for (int v = tid; v < Nv; v += blockDim.x)
+      if (s_stat[v]) idx_b[n_always + (nS - 1 - s_rank[v])] = 1 + v;
+    for (int l = tid; l < L; l += blockDim.x)
+      M[(size_t)b * L + l] = S - (int)(((uint32_t)prm->permille[l] * (uint32_t)nS) / 1000u);
+    if (tid == 0) emit_slot[b] = parallel ? n_always - n_action : n_always - 1;
+  }
+  __syncthreads();
+  if (user_idx)
+    for (int i = tid; i < S; i += blockDim.x) user_idx[(size_t)b * S + i] = idx_b[i];
+  if (user_M)
+    for (int l = tid; l < L; l += blockDim.x) user_M[(size_t)b * L + l] = M[(size_t)b * L + l];
+}
+
+// Row offsets of every layer: off[l][b] = sum of M[b'][l] over b' < b.
+__global__ void plan_kernel(const int* __restrict__ M, int B, int L, int* __restrict__ off) {
+  for (int l = threadIdx.x; l < L; l += blockDim.x) {
+    int acc = 0;
+    off[(size_t)l * (B + 1)] = 0;
+    for (int b = 0; b < B; ++b) {
+      acc += M[(size_t)b * L + l];
+      off[(size_t)l * (B + 1) + b + 1] = acc;
+    }
+  }
+}
+
+void launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid, const StepParams* prm,
+                        int B, int n_views, int img_h, int img_w, int patch, int3* stats, uint8_t* mask,
+                        uint8_t* user_mask, cudaStream_t st) {
+  const int Nv = n_views * (img_h / patch) * (img_w / patch);
+  dim3 grid((Nv + 7) / 8, B);
+  patch_stats_kernel<<<grid, 256, 0, st>>>(frames, prev, valid, prm, n_views, img_h, img_w, patch, Nv, stats,
+                                           mask, user_mask);
+}
+
+void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
+                   const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
+                   int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
+                   uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
+                   cudaStream_t st) {
+  const size_t smem = (size_t)Nv * (sizeof(int3) + sizeof(int) + 1) + 16;
+  select_kernel<<<B, 512, smem, st>>>(stats, mask, valid, m_prev, prm, override_, Nv, S, L, P, parallel,
+                                      n_action, full, idx, M, emit_slot, user_recomputed, user_gate_auto,
+                                      user_idx, user_M);
+  plan_kernel<<<1, 256, 0, st>>>(M, B, L, off);
+}
+
+}  // namespace vlac

@@ -1,0 +1,566 @@
+// C-ABI of libvlac: context (repacked weights, TMA descriptors, workspace),
+// caller-owned caches and the step of Algorithm 1.
+#include <algorithm>
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "internal.cuh"
+
+using namespace vlac;
+
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+constexpr uint32_t kDefaultWaitLimit = 1u << 24;
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// A bump allocator over one device allocation.
+struct Carve {
+  size_t off = 0;
+  template <typename P>
+  void take(P*& p, size_t bytes, char* base) {
+    off = align_up(off, 256);
+    p = base ? reinterpret_cast<P*>(base + off) : nullptr;
+    off += bytes;
+  }
+};
+
+}  // namespace
+
+struct vlac_ctx {
+  vlac_dims d;
+  int P, S, Tc, Nv, pdim, kpad, has_p, rows_cap;
+  bool bf16;
+  size_t esz;
+  int dev;
+  // weights
+  char* wmem = nullptr;
+  void *tok_emb, *patch_w, *proprio_w, *action_emb, *final_norm, *head_w;
+  std::vector<void*> attn_norm, ffn_norm, wqkv, wo, wgu, wd;
+  float *rope_cos, *rope_sin;
+  // TMA descriptors (bf16 only)
+  std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_d;
+  CUtensorMap tm_patch, tm_A, tm_AO, tm_G, tm_col;
+  int split_qkv = 1, split_o = 1, split_gu = 1, split_d = 1;
+  // workspace
+  char* wsmem = nullptr;
+  float *X, *Xd, *part;
+  void *A, *Q, *AO, *G, *col;
+  StepParams* prm;
+  int3* stats;
+  uint8_t *mask, *full;
+  int *idx, *M, *off, *emit_slot, *off_dec, *idx_dec, *err;
+  int* err_host = nullptr;  // pinned
+  uint64_t launches = 0;
+  uint32_t wait_limit = kDefaultWaitLimit;
+};
+
+struct vlac_cache {
+  vlac_ctx* ctx;
+  int B;
+  void *K, *V;
+  float* H;
+  uint8_t *prev, *valid;
+  float* m_prev;
+  size_t kv_seq_stride, h_seq_stride;  // elements per sequence
+};
+
+#define CK(x)                                  \
+  do {                                         \
+    if ((x) != cudaSuccess) {                  \
+      (void)cudaGetLastError();                \
+      return VLAC_ERR_CUDA;                    \
+    }                                          \
+  } while (0)
+
+// ---- dims ------------------------------------------------------------------
+
+static int check_dims(const vlac_dims* d) {
+  if (!d) return VLAC_ERR_INVALID_ARG;
+  if (d->n_layers < 1 || d->n_layers > kMaxLayers || d->n_heads < 1 || d->n_heads * d->head_dim != d->hidden ||
+      d->ffn < 1 || d->vocab < 1 || d->n_bins < 2 || d->n_bins > d->vocab || d->n_bins > 4096 || d->patch < 1 ||
+      d->img_h < d->patch || d->img_w < d->patch || d->img_h % d->patch || d->img_w % d->patch || d->n_views < 1 ||
+      d->n_text < 1 || d->n_action < 1 || d->proprio_dim < 0 || d->proprio_dim > 256 || d->max_batch < 1 ||
+      d->max_batch > 8 || (d->parallel != 0 && d->parallel != 1) || (!d->parallel && d->n_text < 2) ||
+      !(d->rms_eps >= 0.f) || !(d->rope_theta > 0.f))
+    return VLAC_ERR_INVALID_ARG;
+  if (d->dtype != VLAC_F32 && d->dtype != VLAC_BF16) return VLAC_ERR_INVALID_ARG;
+  if (d->head_dim != 64 && d->head_dim != 128) return VLAC_ERR_UNSUPPORTED;
+  const int nv = d->n_views * (d->img_h / d->patch) * (d->img_w / d->patch);
+  if (nv > 4096) return VLAC_ERR_UNSUPPORTED;
+  if (d->dtype == VLAC_BF16) {
+    if (d->hidden % 128 || d->ffn % 64) return VLAC_ERR_UNSUPPORTED;
+  } else {
+    if (d->hidden % 4 || d->ffn % 4) return VLAC_ERR_UNSUPPORTED;
+  }
+  return VLAC_OK;
+}
+
+static EncodeTiledFn get_encode() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 2D bf16 tensor [rows][cols] (cols contiguous), box = 64 columns x box_rows, 128B swizzle.
+static bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  EncodeTiledFn enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// ---- create / destroy -----------------------------------------------------------
+
+extern "C" int vlac_destroy(vlac_ctx* c) {
+  if (!c) return VLAC_ERR_INVALID_ARG;
+  if (c->wmem) cudaFree(c->wmem);
+  if (c->wsmem) cudaFree(c->wsmem);
+  if (c->err_host) cudaFreeHost(c->err_host);
+  delete c;
+  return VLAC_OK;
+}
+
+extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ctx** out) {
+  int rc = check_dims(dims);
+  if (rc) return rc;
+  if (!w || !out || !w->tok_emb || !w->patch_w || !w->attn_norm || !w->wq || !w->wk || !w->wv || !w->wo ||
+      !w->ffn_norm || !w->w_gate || !w->w_up || !w->w_down || !w->final_norm || !w->lm_head)
+    return VLAC_ERR_INVALID_ARG;
+  if (dims->proprio_dim > 0 && !w->proprio_w) return VLAC_ERR_INVALID_ARG;
+  if (dims->parallel && !w->action_emb) return VLAC_ERR_INVALID_ARG;
+  for (int l = 0; l < dims->n_layers; ++l)
+    if (!w->attn_norm[l] || !w->wq[l] || !w->wk[l] || !w->wv[l] || !w->wo[l] || !w->ffn_norm[l] || !w->w_gate[l] ||
+        !w->w_up[l] || !w->w_down[l])
+      return VLAC_ERR_INVALID_ARG;
+
+  vlac_ctx* c = new (std::nothrow) vlac_ctx();
+  if (!c) return VLAC_ERR_OOM;
+  c->d = *dims;
+  const vlac_dims& d = c->d;
+  c->bf16 = d.dtype == VLAC_BF16;
+  c->esz = c->bf16 ? 2 : 4;
+  c->Nv = d.n_views * (d.img_h / d.patch) * (d.img_w / d.patch);
+  c->has_p = d.proprio_dim > 0;
+  c->P = d.n_text + c->Nv + c->has_p;
+  c->S = c->P + (d.parallel ? d.n_action : 0);
+  c->Tc = c->S + (d.parallel ? 0 : d.n_action - 1);
+  c->pdim = d.patch * d.patch * 3;
+  c->kpad = c->bf16 ? (int)align_up(c->pdim, 64) : c->pdim;
+  c->rows_cap = d.max_batch * c->S;
+  if (cudaGetDevice(&c->dev) != cudaSuccess) {
+    delete c;
+    return VLAC_ERR_CUDA;
+  }
+  const size_t L = d.n_layers, Hd = d.hidden, F = d.ffn, E = c->esz;
+
+  // ---- weights: one allocation, fused [q|k|v] and [gate|up] projections ----
+  Carve wc;
+  auto plan_w = [&](char* base) {
+    wc = Carve();
+    wc.take(c->tok_emb, (size_t)d.vocab * Hd * E, base);
+    wc.take(c->patch_w, Hd * c->kpad * E, base);
+    wc.take(c->proprio_w, Hd * std::max(d.proprio_dim, 1) * E, base);
+    wc.take(c->action_emb, (size_t)d.n_action * Hd * E, base);
+    wc.take(c->final_norm, Hd * E, base);
+    wc.take(c->head_w, (size_t)d.n_bins * Hd * E, base);
+    c->attn_norm.resize(L); c->ffn_norm.resize(L); c->wqkv.resize(L); c->wo.resize(L); c->wgu.resize(L); c->wd.resize(L);
+    for (size_t l = 0; l < L; ++l) {
+      wc.take(c->attn_norm[l], Hd * E, base);
+      wc.take(c->wqkv[l], 3 * Hd * Hd * E, base);
+      wc.take(c->wo[l], Hd * Hd * E, base);
+      wc.take(c->ffn_norm[l], Hd * E, base);
+      wc.take(c->wgu[l], 2 * F * Hd * E, base);
+      wc.take(c->wd[l], Hd * F * E, base);
+    }
+    const size_t half = d.head_dim / 2;
+    wc.take(c->rope_cos, (size_t)c->Tc * half * 4, base);
+    wc.take(c->rope_sin, (size_t)c->Tc * half * 4, base);
+  };
+  plan_w(nullptr);
+  if (cudaMalloc(&c->wmem, wc.off) != cudaSuccess) {
+    (void)cudaGetLastError();
+    delete c;
+    return VLAC_ERR_OOM;
+  }
+  plan_w(c->wmem);
+  auto fail = [&](int code) {
+    vlac_destroy(c);
+    return code;
+  };
+  auto cp = [&](void* dst, const void* src, size_t bytes) {
+    return cudaMemcpy(dst, src, bytes, cudaMemcpyDeviceToDevice) == cudaSuccess;
+  };
+  bool ok = cp(c->tok_emb, w->tok_emb, (size_t)d.vocab * Hd * E);
+  ok = ok && cudaMemset(c->patch_w, 0, Hd * c->kpad * E) == cudaSuccess;
+  ok = ok && cudaMemcpy2D(c->patch_w, c->kpad * E, w->patch_w, c->pdim * E, c->pdim * E, Hd,
+                          cudaMemcpyDeviceToDevice) == cudaSuccess;
+  if (d.proprio_dim) ok = ok && cp(c->proprio_w, w->proprio_w, Hd * d.proprio_dim * E);
+  if (d.parallel) ok = ok && cp(c->action_emb, w->action_emb, (size_t)d.n_action * Hd * E);
+  ok = ok && cp(c->final_norm, w->final_norm, Hd * E);
+  ok = ok && cp(c->head_w, static_cast<const char*>(w->lm_head) + (size_t)(d.vocab - d.n_bins) * Hd * E,
+                (size_t)d.n_bins * Hd * E);
+  for (size_t l = 0; l < L && ok; ++l) {
+    char* qkv = static_cast<char*>(c->wqkv[l]);
+    char* gu = static_cast<char*>(c->wgu[l]);
+    ok = cp(c->attn_norm[l], w->attn_norm[l], Hd * E) && cp(qkv, w->wq[l], Hd * Hd * E) &&
+         cp(qkv + Hd * Hd * E, w->wk[l], Hd * Hd * E) && cp(qkv + 2 * Hd * Hd * E, w->wv[l], Hd * Hd * E) &&
+         cp(c->wo[l], w->wo[l], Hd * Hd * E) && cp(c->ffn_norm[l], w->ffn_norm[l], Hd * E) &&
+         cp(gu, w->w_gate[l], F * Hd * E) && cp(gu + F * Hd * E, w->w_up[l], F * Hd * E) &&
+         cp(c->wd[l], w->w_down[l], Hd * F * E);
+  }
+  if (!ok) return fail(VLAC_ERR_CUDA);
+  {  // RoPE tables: angle pos * theta^(-2i/head_dim) in fp64, stored fp32
+    const int half = d.head_dim / 2;
+    std::vector<float> cs((size_t)c->Tc * half), sn((size_t)c->Tc * half);
+    for (int p = 0; p < c->Tc; ++p)
+      for (int i = 0; i < half; ++i) {
+        const double a = (double)p * std::pow((double)d.rope_theta, -2.0 * i / d.head_dim);
+        cs[(size_t)p * half + i] = (float)std::cos(a);
+        sn[(size_t)p * half + i] = (float)std::sin(a);
+      }
+    if (cudaMemcpy(c->rope_cos, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(c->rope_sin, sn.data(), sn.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(VLAC_ERR_CUDA);
+  }
+
+  // ---- workspace ----
+  if (c->bf16) {
+    c->split_o = 4;
+    c->split_d = 4;
+  }
+  const size_t rc_ = c->rows_cap, Bm = d.max_batch;
+  const size_t part_n = std::max({3 * Hd, 2 * F, (size_t)c->split_o * Hd, (size_t)c->split_d * Hd});
+  Carve sc;
+  auto plan_s = [&](char* base) {
+    sc = Carve();
+    sc.take(c->X, rc_ * Hd * 4, base);
+    sc.take(c->Xd, Bm * Hd * 4, base);
+    sc.take(c->part, rc_ * part_n * 4, base);
+    sc.take(c->A, rc_ * Hd * E, base);
+    sc.take(c->Q, rc_ * Hd * E, base);
+    sc.take(c->AO, rc_ * Hd * E, base);
+    sc.take(c->G, rc_ * F * E, base);
+    sc.take(c->col, rc_ * c->kpad * E, base);
+    sc.take(c->prm, sizeof(StepParams), base);
+    sc.take(c->stats, Bm * c->Nv * sizeof(int3), base);
+    sc.take(c->mask, Bm * c->Nv, base);
+    sc.take(c->full, Bm, base);
+    sc.take(c->idx, Bm * c->S * 4, base);
+    sc.take(c->M, Bm * L * 4, base);
+    sc.take(c->off, L * (Bm + 1) * 4, base);
+    sc.take(c->emit_slot, Bm * 4, base);
+    sc.take(c->off_dec, (Bm + 1) * 4, base);
+    sc.take(c->idx_dec, Bm * 4, base);
+    sc.take(c->err, 4, base);
+  };
+  plan_s(nullptr);
+  if (cudaMalloc(&c->wsmem, sc.off) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return fail(VLAC_ERR_OOM);
+  }
+  plan_s(c->wsmem);
+  if (cudaMemset(c->wsmem, 0, sc.off) != cudaSuccess) return fail(VLAC_ERR_CUDA);
+  {
+    std::vector<int> od(Bm + 1);
+    for (size_t b = 0; b <= Bm; ++b) od[b] = (int)b;
+    if (cudaMemcpy(c->off_dec, od.data(), od.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(VLAC_ERR_CUDA);
+  }
+  if (cudaMallocHost(&c->err_host, sizeof(int)) != cudaSuccess) {
+    (void)cudaGetLastError();
+    c->err_host = nullptr;
+    return fail(VLAC_ERR_OOM);
+  }
+  *c->err_host = 0;
+
+  // ---- TMA descriptors ----
+  if (c->bf16) {
+    c->tm_qkv.resize(L); c->tm_o.resize(L); c->tm_gu.resize(L); c->tm_d.resize(L);
+    bool mok = make_map(&c->tm_patch, c->patch_w, Hd, c->kpad, 128) && make_map(&c->tm_A, c->A, rc_, Hd, 32) &&
+               make_map(&c->tm_AO, c->AO, rc_, Hd, 32) && make_map(&c->tm_G, c->G, rc_, F, 32) &&
+               make_map(&c->tm_col, c->col, rc_, c->kpad, 32);
+    for (size_t l = 0; l < L && mok; ++l)
+      mok = make_map(&c->tm_qkv[l], c->wqkv[l], 3 * Hd, Hd, 128) && make_map(&c->tm_o[l], c->wo[l], Hd, Hd, 128) &&
+            make_map(&c->tm_gu[l], c->wgu[l], 2 * F, Hd, 128) && make_map(&c->tm_d[l], c->wd[l], Hd, F, 128);
+    if (!mok) return fail(VLAC_ERR_CUDA);
+  }
+  if (cudaDeviceSynchronize() != cudaSuccess) return fail(VLAC_ERR_CUDA);
+  *out = c;
+  return VLAC_OK;
+}
+
+// ---- caches -----------------------------------------------------------------------
+
+static size_t cache_layout(const vlac_ctx* c, int B, char* base, vlac_cache* k) {
+  const vlac_dims& d = c->d;
+  Carve cv;
+  void* K;
+  void* V;
+  float* H;
+  uint8_t *prev, *valid;
+  float* m_prev;
+  const size_t kv = (size_t)d.n_layers * d.n_heads * c->Tc * d.head_dim;
+  const size_t hs = (size_t)d.n_layers * c->S * d.hidden;
+  cv.take(K, B * kv * c->esz, base);
+  cv.take(V, B * kv * c->esz, base);
+  cv.take(H, B * hs * 4, base);
+  cv.take(prev, (size_t)B * d.n_views * d.img_h * d.img_w * 3, base);
+  cv.take(m_prev, (size_t)B * 4, base);
+  cv.take(valid, (size_t)B, base);
+  if (k) {
+    k->K = K; k->V = V; k->H = H; k->prev = prev; k->m_prev = m_prev; k->valid = valid;
+    k->kv_seq_stride = kv;
+    k->h_seq_stride = hs;
+  }
+  return align_up(cv.off, 256);
+}
+
+extern "C" int vlac_cache_bytes(const vlac_ctx* c, int batch, size_t* bytes) {
+  if (!c || !bytes || batch < 1 || batch > c->d.max_batch) return VLAC_ERR_INVALID_ARG;
+  *bytes = cache_layout(c, batch, nullptr, nullptr);
+  return VLAC_OK;
+}
+
+extern "C" int vlac_cache_init(vlac_ctx* c, void* mem, size_t bytes, int batch, vlac_cache** out) {
+  if (!c || !mem || !out || batch < 1 || batch > c->d.max_batch) return VLAC_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(mem) % 256) return VLAC_ERR_INVALID_ARG;
+  const size_t need = cache_layout(c, batch, nullptr, nullptr);
+  if (bytes < need) return VLAC_ERR_INVALID_ARG;
+  vlac_cache* k = new (std::nothrow) vlac_cache();
+  if (!k) return VLAC_ERR_OOM;
+  k->ctx = c;
+  k->B = batch;
+  cache_layout(c, batch, static_cast<char*>(mem), k);
+  if (cudaMemset(mem, 0, need) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
+    (void)cudaGetLastError();
+    delete k;
+    return VLAC_ERR_CUDA;
+  }
+  *out = k;
+  return VLAC_OK;
+}
+
+extern "C" int vlac_cache_destroy(vlac_cache* k) {
+  if (!k) return VLAC_ERR_INVALID_ARG;
+  delete k;
+  return VLAC_OK;
+}
+
+extern "C" int vlac_reset(vlac_cache* k, int seq, void* stream) {
+  if (!k || seq < -1 || seq >= k->B) return VLAC_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (seq < 0) CK(cudaMemsetAsync(k->valid, 0, (size_t)k->B, st));
+  else CK(cudaMemsetAsync(k->valid + seq, 0, 1, st));
+  return VLAC_OK;
+}
+
+// ---- the step ------------------------------------------------------------------
+
+namespace {
+
+template <typename T>
+void gemm(vlac_ctx* c, const CUtensorMap* tmA, const CUtensorMap* tmW, const T* A, const void* W, const int* m_ptr,
+          int N, int K, int splits, cudaStream_t st) {
+  if constexpr (sizeof(T) == 2) {
+    launch_gemm_tc(tmA, tmW, m_ptr, c->rows_cap, N, K, splits, c->part, c->err, c->wait_limit, st);
+  } else {
+    launch_gemm_simt<T>(A, static_cast<const T*>(W), m_ptr, c->rows_cap, N, K, c->part, st);
+  }
+  c->launches += 1;
+}
+
+template <typename T>
+int step_impl(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, const int32_t* prompt, const float* proprio,
+              const vlac_step_opts* opts, const vlac_step_out* out, cudaStream_t st) {
+  const vlac_dims& d = c->d;
+  const int B = k->B, S = c->S, L = d.n_layers, Hd = d.hidden, F = d.ffn, D = d.n_action, nb = d.n_bins;
+  const int nh = d.n_heads, hd = d.head_dim;
+  const float eps = d.rms_eps;
+  T* A = static_cast<T*>(c->A);
+  T* Q = static_cast<T*>(c->Q);
+  T* AO = static_cast<T*>(c->AO);
+  T* G = static_cast<T*>(c->G);
+  T* col = static_cast<T*>(c->col);
+  T* Kc = static_cast<T*>(k->K);
+  T* Vc = static_cast<T*>(k->V);
+  const size_t kv_layer = (size_t)nh * c->Tc * hd;
+  const int8_t* ovr = opts ? opts->gate_override : nullptr;
+  const int32_t* forced = opts ? opts->forced_ids : nullptr;
+  auto W = [](void* p) { return static_cast<const T*>(p); };
+
+  // Stage 1 and the gate + Stage-3 plan
+  launch_patch_stats(frames, k->prev, k->valid, c->prm, B, d.n_views, d.img_h, d.img_w, d.patch, c->stats, c->mask,
+                     out->static_mask, st);
+  launch_select(c->stats, c->mask, k->valid, k->m_prev, c->prm, ovr, B, c->Nv, S, L, c->P, d.parallel, D, c->full,
+                c->idx, c->M, c->off, c->emit_slot, out->recomputed, out->gate_auto, out->idx, out->M, st);
+  c->launches += 3;
+
+  // layer-0 inputs of the recomputed rows
+  Rows r0{c->off, c->idx, S, c->X};
+  const int* m0 = c->off + B;
+  launch_im2col<T>(r0, B, S, frames, d.n_views, d.img_h, d.img_w, d.patch, c->kpad, col, st);
+  gemm<T>(c, &c->tm_col, &c->tm_patch, col, c->patch_w, m0, Hd, c->kpad, 1, st);
+  launch_embed<T>(r0, B, S, Hd, c->Nv, c->P, c->has_p, d.proprio_dim, d.n_text, d.vocab, prompt, proprio,
+                  W(c->tok_emb), c->part, W(c->proprio_w), W(c->action_emb), c->err, st);
+  c->launches += 2;
+
+  const size_t rs = (size_t)c->rows_cap;
+  for (int l = 0; l < L; ++l) {
+    Rows rl{c->off + (size_t)l * (B + 1), c->idx, S, c->X};
+    const int* ml = rl.off + B;
+    const int* off_prev = l == 0 ? rl.off : c->off + (size_t)(l - 1) * (B + 1);
+    launch_layer_in<T>(rl, off_prev, B, S, Hd, l == 0 ? nullptr : k->H + (size_t)l * S * Hd, k->h_seq_stride,
+                       W(c->attn_norm[l]), eps, A, st);
+    gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_qkv[l] : nullptr, A, c->wqkv[l], ml, 3 * Hd, Hd, c->split_qkv, st);
+    launch_qkv_epilogue<T>(rl, B, S, nh, hd, c->part, c->split_qkv, rs * 3 * Hd, c->rope_cos, c->rope_sin, Q,
+                           Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, st);
+    launch_attention<T>(rl, B, S, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, c->P,
+                        d.parallel, D, AO, st);
+    gemm<T>(c, &c->tm_AO, c->bf16 ? &c->tm_o[l] : nullptr, AO, c->wo[l], ml, Hd, Hd, c->split_o, st);
+    launch_residual_norm<T>(rl, B, S, Hd, c->part, c->split_o, rs * Hd, W(c->ffn_norm[l]), eps, A, st);
+    gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_gu[l] : nullptr, A, c->wgu[l], ml, 2 * F, Hd, c->split_gu, st);
+    launch_swiglu<T>(rl, B, S, F, c->part, c->split_gu, rs * 2 * F, G, st);
+    gemm<T>(c, &c->tm_G, c->bf16 ? &c->tm_d[l] : nullptr, G, c->wd[l], ml, Hd, F, c->split_d, st);
+    launch_residual(rl, B, S, Hd, c->part, c->split_d, rs * Hd, st);
+    c->launches += 6;
+  }
+  // action head on the prefix pass: the last text row, or the parallel action block
+  launch_head<T>(c->X, c->emit_slot, (size_t)S * Hd, d.parallel ? D : 1, B, Hd, nb, W(c->final_norm), W(c->head_w),
+                 eps, D, 0, out->action_ids, out->margins, out->logit_gap, out->logits, st);
+  c->launches += 1;
+
+  if (!d.parallel) {
+    Rows rd{c->off_dec, c->idx_dec, 1, c->Xd};
+    for (int a = 1; a < D; ++a) {
+      launch_decode_embed<T>(B, a, D, c->P, Hd, d.vocab, nb, W(c->tok_emb), out->action_ids, forced, c->prm, c->Xd,
+                             c->idx_dec, c->err, st);
+      c->launches += 1;
+      for (int l = 0; l < L; ++l) {
+        launch_layer_in<T>(rd, rd.off, B, 1, Hd, nullptr, 0, W(c->attn_norm[l]), eps, A, st);
+        launch_gemv<T>(W(c->wqkv[l]), 3 * Hd, Hd, A, B, c->part, st);
+        launch_qkv_epilogue<T>(rd, B, 1, nh, hd, c->part, 1, 0, c->rope_cos, c->rope_sin, Q, Kc + l * kv_layer,
+                               Vc + l * kv_layer, k->kv_seq_stride, c->Tc, st);
+        launch_attention<T>(rd, B, 1, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc,
+                            c->P, 0, D, AO, st);
+        launch_gemv<T>(W(c->wo[l]), Hd, Hd, AO, B, c->part, st);
+        launch_residual_norm<T>(rd, B, 1, Hd, c->part, 1, 0, W(c->ffn_norm[l]), eps, A, st);
+        launch_gemv<T>(W(c->wgu[l]), 2 * F, Hd, A, B, c->part, st);
+        launch_swiglu<T>(rd, B, 1, F, c->part, 1, 0, G, st);
+        launch_gemv<T>(W(c->wd[l]), Hd, F, G, B, c->part, st);
+        launch_residual(rd, B, 1, Hd, c->part, 1, 0, st);
+        c->launches += 10;
+      }
+      launch_head<T>(c->Xd, nullptr, Hd, 1, B, Hd, nb, W(c->final_norm), W(c->head_w), eps, D, a, out->action_ids,
+                     out->margins, out->logit_gap, out->logits, st);
+      c->launches += 1;
+    }
+  }
+  launch_finish(B, D, c->prm, out->margins, out->logit_gap, k->m_prev, k->valid, out->step_margin, st);
+  c->launches += 1;
+  const size_t fb = (size_t)d.n_views * d.img_h * d.img_w * 3;
+  CK(cudaMemcpyAsync(k->prev, frames, (size_t)B * fb, cudaMemcpyDeviceToDevice, st));
+  CK(cudaMemcpyAsync(c->err_host, c->err, sizeof(int), cudaMemcpyDeviceToHost, st));
+  CK(cudaGetLastError());
+  return VLAC_OK;
+}
+
+}  // namespace
+
+extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, const int32_t* prompt_ids,
+                         const float* proprio, vlac_rational tau_sim, float tau_margin,
+                         const uint16_t* reuse_permille, const vlac_step_opts* opts, const vlac_step_out* out,
+                         void* stream) {
+  if (!c || !k || !frames || !prompt_ids || !reuse_permille || !out || !out->action_ids || !out->margins ||
+      !out->logit_gap || !out->recomputed || !out->step_margin || tau_sim.den == 0)
+    return VLAC_ERR_INVALID_ARG;
+  if (k->ctx != c) return VLAC_ERR_STATE;
+  if (c->d.proprio_dim > 0 && !proprio) return VLAC_ERR_INVALID_ARG;
+  if (tau_margin != tau_margin) return VLAC_ERR_INVALID_ARG;
+  StepParams p;
+  std::memset(&p, 0, sizeof(p));
+  for (int l = 0; l < c->d.n_layers; ++l) {
+    if (reuse_permille[l] > 1000) return VLAC_ERR_INVALID_ARG;
+    p.permille[l] = reuse_permille[l];
+  }
+  int mk = opts ? opts->margin_kind : VLAC_MARGIN_PROB;
+  int red = opts ? opts->reduction : VLAC_REDUCE_DEFAULT;
+  if (mk != VLAC_MARGIN_PROB && mk != VLAC_MARGIN_LOGIT) return VLAC_ERR_INVALID_ARG;
+  if (red == VLAC_REDUCE_DEFAULT) red = c->d.parallel ? VLAC_REDUCE_MIN : VLAC_REDUCE_MEAN;
+  if (red != VLAC_REDUCE_MEAN && red != VLAC_REDUCE_MIN) return VLAC_ERR_INVALID_ARG;
+  p.tau_num = tau_sim.num;
+  p.tau_den = tau_sim.den;
+  p.tau_margin = tau_margin;
+  p.margin_kind = mk;
+  p.reduction = red;
+  p.has_override = (opts && opts->gate_override) ? 1 : 0;
+  p.has_forced = (opts && opts->forced_ids) ? 1 : 0;
+  // an error latched by an earlier step on this context is reported first
+  if (*c->err_host) {
+    const int e = *c->err_host;
+    *c->err_host = 0;
+    cudaMemsetAsync(c->err, 0, sizeof(int), static_cast<cudaStream_t>(stream));
+    return e;
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  CK(cudaMemcpyAsync(c->prm, &p, sizeof(p), cudaMemcpyHostToDevice, st));
+  return c->bf16 ? step_impl<bf16>(c, k, frames, prompt_ids, proprio, opts, out, st)
+                 : step_impl<float>(c, k, frames, prompt_ids, proprio, opts, out, st);
+}
+
+extern "C" int vlac_sync_error(vlac_ctx* c) {
+  if (!c) return VLAC_ERR_INVALID_ARG;
+  CK(cudaDeviceSynchronize());
+  int e = 0;
+  CK(cudaMemcpy(&e, c->err, sizeof(int), cudaMemcpyDeviceToHost));
+  CK(cudaMemset(c->err, 0, sizeof(int)));
+  *c->err_host = 0;
+  return e;
+}
+
+extern "C" uint64_t vlac_launch_count(const vlac_ctx* c) { return c ? c->launches : 0; }
+
+extern "C" int vlac_selftest_wait(vlac_ctx* c, uint32_t spin_limit) {
+  if (!c) return VLAC_ERR_INVALID_ARG;
+  CK(cudaDeviceSynchronize());
+  CK(cudaMemset(c->err, 0, sizeof(int)));
+  if (launch_wait_selftest(c->err, spin_limit, 0)) return VLAC_ERR_CUDA;
+  c->launches += 1;
+  CK(cudaDeviceSynchronize());
+  int e = 0;
+  CK(cudaMemcpy(&e, c->err, sizeof(int), cudaMemcpyDeviceToHost));
+  CK(cudaMemset(c->err, 0, sizeof(int)));
+  return e;
+}
+
+extern "C" const char* vlac_strerror(int code) {
+  switch (code) {
+    case VLAC_OK: return "ok";
+    case VLAC_ERR_INVALID_ARG: return "invalid argument";
+    case VLAC_ERR_CUDA: return "CUDA runtime error";
+    case VLAC_ERR_OOM: return "out of memory";
+    case VLAC_ERR_TIMEOUT: return "a bounded device wait gave up";
+    case VLAC_ERR_DEVICE_CHECK: return "a device-side bounds check rejected an input";
+    case VLAC_ERR_STATE: return "cache does not belong to this context";
+    case VLAC_ERR_UNSUPPORTED: return "dims not supported by this build";
+    default: return "unknown error";
+  }
+}

@@ -1,0 +1,241 @@
+"""ctypes binding of libvlac (include/vlac.h).
+
+Argument marshalling only: every step of the method runs in the library's
+CUDA kernels.  PyTorch supplies device memory and streams.  Importing this
+module does not load the library; the first call does, and raises
+``RuntimeError`` if ``libvlac.so`` is missing or fails to load.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import threading
+from typing import Dict, Optional, Sequence
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libvlac.so")
+_lock = threading.Lock()
+_lib = None
+
+VLAC_OK = 0
+ERRORS = {-1: "VLAC_ERR_INVALID_ARG", -2: "VLAC_ERR_CUDA", -3: "VLAC_ERR_OOM", -4: "VLAC_ERR_TIMEOUT",
+          -5: "VLAC_ERR_DEVICE_CHECK", -6: "VLAC_ERR_STATE", -7: "VLAC_ERR_UNSUPPORTED"}
+F32, BF16 = 0, 1
+MARGIN_PROB, MARGIN_LOGIT = 0, 1
+REDUCE_DEFAULT, REDUCE_MEAN, REDUCE_MIN = -1, 0, 1
+
+
+class VlacError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {ERRORS.get(code, code)} ({code})")
+
+
+class Dims(C.Structure):
+    _fields_ = [(n, C.c_int32) for n in (
+        "n_layers", "hidden", "n_heads", "head_dim", "ffn", "vocab", "n_bins", "img_h", "img_w", "patch",
+        "n_views", "n_text", "proprio_dim", "n_action", "parallel", "dtype")] + [
+        ("rope_theta", C.c_float), ("rms_eps", C.c_float), ("max_batch", C.c_int32)]
+
+
+_PP = C.POINTER(C.c_void_p)
+
+
+class Weights(C.Structure):
+    _fields_ = [("tok_emb", C.c_void_p), ("patch_w", C.c_void_p), ("proprio_w", C.c_void_p),
+                ("action_emb", C.c_void_p)] + [(n, _PP) for n in (
+                    "attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate", "w_up", "w_down")] + [
+                ("final_norm", C.c_void_p), ("lm_head", C.c_void_p)]
+
+
+class Rational(C.Structure):
+    _fields_ = [("num", C.c_uint32), ("den", C.c_uint32)]
+
+
+class StepOpts(C.Structure):
+    _fields_ = [("margin_kind", C.c_int32), ("reduction", C.c_int32), ("gate_override", C.c_void_p),
+                ("forced_ids", C.c_void_p)]
+
+
+class StepOut(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in (
+        "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
+        "static_mask", "idx", "M")]
+
+
+EXPORTS = ["vlac_create", "vlac_destroy", "vlac_cache_bytes", "vlac_cache_init", "vlac_cache_destroy",
+           "vlac_step", "vlac_reset", "vlac_sync_error", "vlac_launch_count", "vlac_selftest_wait",
+           "vlac_strerror"]
+
+
+def lib():
+    """Loads libvlac.so (once) and declares its signatures."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(f"libvlac.so is not built ({LIB_PATH}); run paper_2608_10824_gb300.build()")
+            L = C.CDLL(LIB_PATH)
+            vp, i32 = C.c_void_p, C.c_int
+            L.vlac_create.argtypes = [C.POINTER(Dims), C.POINTER(Weights), C.POINTER(vp)]
+            L.vlac_destroy.argtypes = [vp]
+            L.vlac_cache_bytes.argtypes = [vp, i32, C.POINTER(C.c_size_t)]
+            L.vlac_cache_init.argtypes = [vp, vp, C.c_size_t, i32, C.POINTER(vp)]
+            L.vlac_cache_destroy.argtypes = [vp]
+            L.vlac_step.argtypes = [vp, vp, vp, vp, vp, Rational, C.c_float, vp, C.POINTER(StepOpts),
+                                    C.POINTER(StepOut), vp]
+            L.vlac_reset.argtypes = [vp, i32, vp]
+            L.vlac_sync_error.argtypes = [vp]
+            L.vlac_launch_count.argtypes = [vp]
+            L.vlac_launch_count.restype = C.c_uint64
+            L.vlac_selftest_wait.argtypes = [vp, C.c_uint32]
+            L.vlac_strerror.argtypes = [i32]
+            L.vlac_strerror.restype = C.c_char_p
+            for name in EXPORTS:
+                if name not in ("vlac_launch_count", "vlac_strerror"):
+                    getattr(L, name).restype = C.c_int
+            _lib = L
+    return _lib
+
+
+def _check(rc: int, where: str):
+    if rc != VLAC_OK:
+        raise VlacError(rc, where)
+
+
+def c_dims(d, max_batch: Optional[int] = None) -> Dims:
+    return Dims(d.n_layers, d.hidden, d.n_heads, d.head_dim, d.ffn, d.vocab, d.n_bins, d.img_h, d.img_w,
+                d.patch, d.n_views, d.n_text, d.proprio_dim, d.n_action, d.parallel,
+                BF16 if d.dtype == "bf16" else F32, float(d.rope_theta), float(d.rms_eps),
+                int(max_batch if max_batch is not None else d.max_batch))
+
+
+def _ptr(t) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _stream_ptr(stream) -> Optional[int]:
+    import torch
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+class Context:
+    """A model on the current CUDA device: repacked weights and workspace."""
+
+    def __init__(self, d, weights: Dict, max_batch: Optional[int] = None):
+        self.d = d
+        self.max_batch = int(max_batch if max_batch is not None else d.max_batch)
+        keep = []
+
+        def arr(name):
+            a = (C.c_void_p * d.n_layers)(*[lay[name].data_ptr() for lay in weights["layers"]])
+            keep.append(a)
+            return C.cast(a, _PP)
+
+        w = Weights(_ptr(weights["tok_emb"]), _ptr(weights["patch_w"]), _ptr(weights.get("proprio_w")),
+                    _ptr(weights.get("action_emb")), arr("attn_norm"), arr("wq"), arr("wk"), arr("wv"),
+                    arr("wo"), arr("ffn_norm"), arr("w_gate"), arr("w_up"), arr("w_down"),
+                    _ptr(weights["final_norm"]), _ptr(weights["lm_head"]))
+        self._dims = c_dims(d, self.max_batch)
+        h = C.c_void_p()
+        _check(lib().vlac_create(C.byref(self._dims), C.byref(w), C.byref(h)), "vlac_create")
+        self._h = h
+
+    def close(self):
+        h = getattr(self, "_h", None)
+        if h is not None and h.value:
+            lib().vlac_destroy(h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def cache_bytes(self, batch: int) -> int:
+        n = C.c_size_t()
+        _check(lib().vlac_cache_bytes(self._h, batch, C.byref(n)), "vlac_cache_bytes")
+        return n.value
+
+    def new_cache(self, batch: int = 1) -> "Cache":
+        return Cache(self, batch)
+
+    def alloc_outputs(self, batch: int, want: Sequence[str] = ()) -> Dict:
+        import torch
+        d, dev = self.d, torch.device("cuda")
+        D = d.n_action
+        out = {
+            "action_ids": torch.zeros((batch, D), dtype=torch.int32, device=dev),
+            "margins": torch.zeros((batch, D), dtype=torch.float32, device=dev),
+            "logit_gap": torch.zeros((batch, D), dtype=torch.float32, device=dev),
+            "recomputed": torch.zeros((batch,), dtype=torch.uint8, device=dev),
+            "step_margin": torch.zeros((batch,), dtype=torch.float32, device=dev),
+        }
+        shapes = {"gate_auto": ((batch,), torch.uint8), "logits": ((batch, D, d.n_bins), torch.float32),
+                  "static_mask": ((batch, d.n_visual), torch.uint8), "idx": ((batch, d.pass_len), torch.int32),
+                  "M": ((batch, d.n_layers), torch.int32)}
+        for k in want:
+            shp, dt = shapes[k]
+            out[k] = torch.zeros(shp, dtype=dt, device=dev)
+        return out
+
+    def step(self, cache: "Cache", frames, prompt, proprio=None, tau_sim=(996, 1000), tau_margin: float = 0.0,
+             permille=None, margin_kind: int = MARGIN_PROB, reduction: int = REDUCE_DEFAULT, gate_override=None,
+             forced_ids=None, out: Optional[Dict] = None, want: Sequence[str] = (), stream=None) -> Dict:
+        """One step for every sequence of `cache`; inputs are CUDA tensors.
+        Returns the dict of device output tensors (allocated unless given)."""
+        d = self.d
+        if permille is None:
+            permille = np.full(d.n_layers, 1000, dtype=np.uint16)
+        permille = np.ascontiguousarray(permille, dtype=np.uint16)
+        if out is None:
+            out = self.alloc_outputs(cache.batch, want)
+        so = StepOut(*[_ptr(out.get(k)) for k in (
+            "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
+            "static_mask", "idx", "M")])
+        opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids))
+        rc = lib().vlac_step(self._h, cache._h, frames.data_ptr(), prompt.data_ptr(), _ptr(proprio),
+                             Rational(int(tau_sim[0]), int(tau_sim[1])), float(tau_margin),
+                             permille.ctypes.data, C.byref(opts), C.byref(so), _stream_ptr(stream))
+        _check(rc, "vlac_step")
+        return out
+
+    def reset(self, cache: "Cache", seq: int = -1, stream=None):
+        _check(lib().vlac_reset(cache._h, seq, _stream_ptr(stream)), "vlac_reset")
+
+    def sync_error(self) -> int:
+        return lib().vlac_sync_error(self._h)
+
+    def launch_count(self) -> int:
+        return int(lib().vlac_launch_count(self._h))
+
+    def selftest_wait(self, spin_limit: int) -> int:
+        return lib().vlac_selftest_wait(self._h, spin_limit)
+
+
+class Cache:
+    """Device memory (a torch uint8 tensor) formatted by the library as a cache."""
+
+    def __init__(self, ctx: Context, batch: int):
+        import torch
+        self.ctx, self.batch = ctx, batch
+        nbytes = ctx.cache_bytes(batch)
+        self.mem = torch.empty(nbytes + 256, dtype=torch.uint8, device="cuda")
+        base = self.mem.data_ptr()
+        off = (-base) % 256
+        h = C.c_void_p()
+        _check(lib().vlac_cache_init(ctx._h, base + off, nbytes, batch, C.byref(h)), "vlac_cache_init")
+        self._h = h
+
+    def __del__(self):
+        h = getattr(self, "_h", None)
+        if h is not None and h.value:
+            try:
+                lib().vlac_cache_destroy(h)
+            except Exception:
+                pass
+            self._h = None

@@ -1,0 +1,110 @@
+"""Shared pieces of the GPU parity tests: small workloads the oracle finishes
+in seconds, and a lock-step driver that runs the oracle and the CUDA library
+on the same seeded inputs and compares every step."""
+from __future__ import annotations
+
+import numpy as np
+
+import synth
+
+# Tolerances.  Logits: the stated bar for bf16 weights is abs 2e-2; the fp32
+# model is held to 1e-3.  Action ids may differ only where the oracle's
+# probability margin p1 - p2 is below 1e-3.  Flags may differ only where the
+# oracle's m_{t-1} is within 1e-4 of theta_m (the step is then re-synced by
+# forcing the oracle's branch).
+LOGIT_TOL = {"bf16": 2e-2, "f32": 1e-3}
+ID_EXEMPT_MARGIN = 1e-3
+FLAG_TIE = 1e-4
+
+SMALL = {
+    # bf16 path (tcgen05 GEMMs), head_dim 128, autoregressive decode
+    "small": synth.Dims(n_layers=2, hidden=256, n_heads=2, head_dim=128, ffn=768, vocab=1024, n_bins=256,
+                        img_h=112, img_w=112, patch=14, n_views=1, n_text=8, proprio_dim=0, n_action=7,
+                        parallel=0, dtype="bf16"),
+    # bf16, two 224x224 views + proprio + 56-position parallel block: 596 rows (> 512, two GEMM passes)
+    "small_oft": synth.Dims(n_layers=2, hidden=256, n_heads=4, head_dim=64, ffn=512, vocab=512, n_bins=256,
+                            img_h=224, img_w=224, patch=14, n_views=2, n_text=27, proprio_dim=8, n_action=56,
+                            parallel=1, dtype="bf16"),
+    # bf16, batch of three sequences with ragged recompute sets
+    "small_batch": synth.Dims(n_layers=2, hidden=256, n_heads=2, head_dim=128, ffn=768, vocab=1024, n_bins=256,
+                              img_h=112, img_w=112, patch=14, n_views=1, n_text=8, proprio_dim=0, n_action=7,
+                              parallel=0, dtype="bf16", max_batch=3),
+    # fp32 tiny model (SIMT path)
+    "tiny": synth.dims_for("tiny"),
+}
+
+
+def episode(d, n_frames: int, seed: int, batch: int = 1, kind=None):
+    frames = synth.make_episode(d, n_frames, seed=seed, batch=batch, kind=kind)
+    prompt = synth.make_prompt(d, seed=seed, batch=batch)
+    prop = synth.make_proprio(d, n_frames, seed=seed, batch=batch)
+    return frames, prompt, prop
+
+
+class Lockstep:
+    """Runs the oracle and the library side by side, one step at a time."""
+
+    def __init__(self, d, w_cpu, w_gpu=None, batch: int = 1):
+        import torch
+
+        import oracle
+        from paper_2608_10824_gb300 import Context
+        self.d, self.B = d, batch
+        if w_gpu is None:
+            w_gpu = synth.weights_to(w_cpu, "cuda")
+        self.orc = oracle.Oracle(d, w_cpu)
+        self.oc = self.orc.new_cache(batch)
+        self.ctx = Context(d, w_gpu, max_batch=batch)
+        self.gc = self.ctx.new_cache(batch)
+        self.torch = torch
+        self.prev_m = None
+        self.log = []
+
+    def step(self, frames, prompt, proprio, tau_sim, tau_m, permille, margin_kind=0, force_branch=None):
+        torch = self.torch
+        d, B = self.d, self.B
+        o = self.orc.step(self.oc, frames, prompt, proprio, tau_sim=tau_sim, tau_margin=tau_m,
+                          permille=permille, margin_kind=margin_kind,
+                          gate_override=None if force_branch is None else np.full(B, force_branch, np.int8))
+        # branch: free-running, except where the oracle's m_{t-1} sits in the tie zone
+        ovr = np.full(B, -1, np.int8) if force_branch is None else np.full(B, force_branch, np.int8)
+        if self.prev_m is not None and force_branch is None:
+            tie = np.abs(self.prev_m - tau_m) < FLAG_TIE
+            ovr[tie] = o["recomputed"][tie]
+        g = self.ctx.step(
+            self.gc, torch.from_numpy(np.ascontiguousarray(frames)).cuda(),
+            torch.from_numpy(np.ascontiguousarray(prompt)).cuda(),
+            None if proprio is None else torch.from_numpy(np.ascontiguousarray(proprio, np.float32)).cuda(),
+            tau_sim=tau_sim, tau_margin=tau_m, permille=permille, margin_kind=margin_kind,
+            gate_override=torch.from_numpy(ovr).cuda(),
+            forced_ids=torch.from_numpy(o["action_ids"].astype(np.int32)).cuda(),
+            want=("gate_auto", "logits", "static_mask", "idx", "M"))
+        torch.cuda.synchronize()
+        g = {k: v.cpu().numpy() for k, v in g.items()}
+        err = self.ctx.sync_error()
+        assert err == 0, f"device error {err}"
+        rep = compare(d, o, g, self.prev_m, tau_m)
+        self.prev_m = o["step_margin"].copy()
+        self.log.append(rep)
+        return o, g, rep
+
+
+def compare(d, o, g, prev_m, tau_m):
+    """Checks one step; returns a small report of the numeric gaps."""
+    B = o["action_ids"].shape[0]
+    for k in ("static_mask", "idx", "M", "recomputed"):
+        np.testing.assert_array_equal(g[k], o[k], err_msg=k)
+    for b in range(B):
+        tie = prev_m is not None and abs(prev_m[b] - tau_m) < FLAG_TIE
+        if not tie:
+            assert g["gate_auto"][b] == o["gate_auto"][b], f"gate_auto[{b}]"
+    tol = LOGIT_TOL[d.dtype]
+    diff = np.abs(g["logits"].astype(np.float64) - o["logits"])
+    assert diff.max() <= tol, f"logits differ by {diff.max():.3e} > {tol}"
+    mism = g["action_ids"] != o["action_ids"]
+    exempt = o["margins"] < ID_EXEMPT_MARGIN
+    bad = mism & ~exempt
+    assert not bad.any(), f"action ids differ outside the exemption: {np.argwhere(bad)}"
+    np.testing.assert_allclose(g["margins"], o["margins"], atol=max(tol * 0.05, 1e-6), rtol=0.05)
+    return {"max_logit_diff": float(diff.max()), "id_mismatch": int(mism.sum()),
+            "id_exempt": int(exempt.sum()), "recomputed": o["recomputed"].tolist()}

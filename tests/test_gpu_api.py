@@ -1,0 +1,76 @@
+"""Error behaviour of the C-ABI on a GPU: documented status codes for bad
+arguments and bounded device waits (a wait that nothing completes gives up,
+records VLAC_ERR_TIMEOUT and leaves the context usable)."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from tests.gpu_common import SMALL, episode
+
+pytestmark = pytest.mark.gpu
+
+
+def _ctx(name="small"):
+    from paper_2608_10824_gb300 import Context
+    d = SMALL[name]
+    return d, Context(d, synth.weights_to(synth.make_weights(d, seed=1), "cuda"), max_batch=2)
+
+
+def test_bounded_wait_gives_up_and_context_stays_usable(cuda_device):
+    from paper_2608_10824_gb300.vlac import ERRORS
+    d, ctx = _ctx()
+    rc = ctx.selftest_wait(1000)
+    assert ERRORS[rc] == "VLAC_ERR_TIMEOUT"
+    frames, prompt, _ = episode(d, 1, seed=2)
+    c = ctx.new_cache(1)
+    out = ctx.step(c, torch.from_numpy(frames[0]).cuda(), torch.from_numpy(prompt).cuda())
+    torch.cuda.synchronize()
+    assert ctx.sync_error() == 0
+    assert out["recomputed"].item() == 1
+
+
+def test_invalid_arguments(cuda_device):
+    from paper_2608_10824_gb300 import VlacError
+    d, ctx = _ctx()
+    frames, prompt, _ = episode(d, 1, seed=2)
+    f, p = torch.from_numpy(frames[0]).cuda(), torch.from_numpy(prompt).cuda()
+    c = ctx.new_cache(1)
+    with pytest.raises(VlacError) as e:
+        ctx.step(c, f, p, permille=np.full(d.n_layers, 1001, np.uint16))
+    assert e.value.code == -1
+    with pytest.raises(VlacError) as e:
+        ctx.step(c, f, p, tau_sim=(1, 0))
+    assert e.value.code == -1
+    with pytest.raises(VlacError) as e:
+        ctx.new_cache(3)  # above max_batch
+    assert e.value.code == -1
+    with pytest.raises(VlacError) as e:
+        ctx.reset(c, 1)  # out-of-range sequence
+    assert e.value.code == -1
+    # a cache of another context is a state error
+    d2, ctx2 = _ctx()
+    with pytest.raises(VlacError) as e:
+        ctx2.step(c, f, p)
+    assert e.value.code == -6
+
+
+def test_bad_prompt_id_is_a_device_check(cuda_device):
+    d, ctx = _ctx()
+    frames, prompt, _ = episode(d, 1, seed=2)
+    bad = prompt.copy()
+    bad[0, 3] = d.vocab + 5
+    c = ctx.new_cache(1)
+    ctx.step(c, torch.from_numpy(frames[0]).cuda(), torch.from_numpy(bad).cuda())
+    torch.cuda.synchronize()
+    assert ctx.sync_error() == -5
+    assert ctx.sync_error() == 0  # cleared once reported
+
+
+def test_unsupported_dims():
+    from paper_2608_10824_gb300 import VlacError
+    from paper_2608_10824_gb300.vlac import Context
+    d = SMALL["small"].replace(head_dim=96, n_heads=2, hidden=192)
+    with pytest.raises(VlacError) as e:
+        Context(d, synth.weights_to(synth.make_weights(d, seed=1), "cuda"))
+    assert e.value.code in (-7, -1)
