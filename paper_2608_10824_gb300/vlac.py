@@ -224,9 +224,10 @@ class Cache:
         import torch
         self.ctx, self.batch = ctx, batch
         nbytes = ctx.cache_bytes(batch)
-        self.mem = torch.empty(nbytes + 256, dtype=torch.uint8, device="cuda")
-        base = self.mem.data_ptr()
+        self._buf = torch.zeros(nbytes + 256, dtype=torch.uint8, device="cuda")
+        base = self._buf.data_ptr()
         off = (-base) % 256
+        self.mem = self._buf[off:off + nbytes]  # the formatted cache region
         h = C.c_void_p()
         _check(lib().vlac_cache_init(ctx._h, base + off, nbytes, batch, C.byref(h)), "vlac_cache_init")
         self._h = h
