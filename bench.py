@@ -1,0 +1,381 @@
+#!/usr/bin/env python
+"""Throughput of the gated cached VLA step at the OpenVLA-7B shape.
+
+One step = Algorithm 1 for one frame: gate, Stage-1 patch similarity,
+Stage-3 selection, the partial (or full) 32-layer prefix pass, 6 decode
+passes and the Eq. (1) margin.  Workload: a seeded 50-frame synthetic scene
+episode (224x224 frames, 256 patches, 27 text tokens, 7 action tokens),
+tau_sim = 0.996, reuse 0.9 -> 0.5 over the layers, tau_margin = 0.05;
+random-init bf16 weights.  Episodes restart (cache reset) every 50 steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  With N > 1 (torchrun), every rank runs an
+independent replica on its own GPU with its own episode; there is no
+collective on the data path.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "cached VLA steps/sec at OpenVLA-7B shape (1 GB300) and % of step roofline"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+EPISODE = 50
+TAU_SIM = (996, 1000)
+CPU_LAYERS = 2  # the CPU oracle sample runs this many of the 32 layers
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return {k: float(j[k]) for k in FALLBACK_PEAKS}, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ---------------------------------------------------------------------------
+# Algorithmic work of one step (2 FLOPs per multiply-add)
+# ---------------------------------------------------------------------------
+
+def step_work(d, M_seq, idx_seq, recomputed: bool):
+    """FLOPs and bytes one sequence's step must move, from its per-layer row
+    counts M[l] and recompute order idx (what the method computes)."""
+    Hd, F, L, nb = d.hidden, d.ffn, d.n_layers, d.n_bins
+    P, D = d.prefix_len, d.n_action
+    per_row = 2 * (4 * Hd * Hd + 3 * F * Hd)            # QKV + O + gate/up + down
+    w_bytes = L * (4 * Hd * Hd + 3 * F * Hd) * 2        # bf16 weights of one pass
+    head_bytes = nb * Hd * 2
+    flops = 0.0
+    byts = 0.0
+    passes = []
+    # prefix pass
+    fp = 0.0
+    bp = w_bytes + head_bytes
+    for l in range(L):
+        rows = idx_seq[:M_seq[l]]
+        fp += M_seq[l] * per_row + 4 * Hd * float(np.sum(rows + 1))   # QK^T and PV over j <= pos
+        bp += 2 * d.pass_len * Hd * 2                                   # read K and V of the layer
+        bp += M_seq[l] * 2 * Hd * 2                                     # write fresh K/V
+        if l > 0:
+            bp += max(M_seq[l - 1], M_seq[l]) * Hd * 4                  # record / reload layer inputs
+    n_vis0 = int(np.sum((idx_seq[:M_seq[0]] >= 1) & (idx_seq[:M_seq[0]] <= d.n_visual)))
+    fp += 2 * n_vis0 * d.patch_dim * Hd + 2 * nb * Hd
+    bp += Hd * d.patch_dim * 2 + 2 * d.n_views * d.img_h * d.img_w * 3
+    passes.append((fp, bp))
+    # autoregressive decode passes
+    if not d.parallel:
+        for a in range(1, D):
+            pos = P + a - 1
+            fd = L * (per_row + 4 * Hd * (pos + 1)) + 2 * nb * Hd
+            bd = w_bytes + head_bytes + L * (2 * (pos + 1) * Hd * 2 + 2 * Hd * 2) + Hd * 2
+            passes.append((fd, bd))
+    for f_, b_ in passes:
+        flops += f_
+        byts += b_
+    return flops, byts, passes
+
+
+# ---------------------------------------------------------------------------
+# Clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class Clocks:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, dev_index: int):
+        self.p = None
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                                       "-lms", "200", "-i", str(dev_index)], stdout=subprocess.PIPE,
+                                      stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.p.terminate()
+        try:
+            out, _ = self.p.communicate(timeout=5)
+        except Exception:
+            self.p.kill()
+            out = ""
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() in ("active", "0x1", "1"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle sample (the cpu_baseline leg and the reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_sample(d, frames, prompt, pm, tau_m, n_steps, seed, budget_s=None):
+    """Times the CPU oracle on the first CPU_LAYERS layers of each step of the
+    same episode and scales the step time by n_layers / CPU_LAYERS."""
+    import torch
+
+    import oracle
+    ds = d.replace(n_layers=CPU_LAYERS)
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    w = synth.make_weights(ds, seed=seed, device=dev, lm_head_rows=d.n_bins)
+    w = synth.weights_to(w, "cpu")
+    orc = oracle.Oracle(ds, w)
+    cache = orc.new_cache(1)
+    times = []
+    t_begin = time.perf_counter()
+    for t in range(n_steps):
+        if t % EPISODE == 0:
+            cache.reset()
+        t0 = time.perf_counter()
+        orc.step(cache, frames[t % EPISODE], prompt, tau_sim=TAU_SIM, tau_margin=tau_m, permille=pm[:CPU_LAYERS],
+                 want_logits=False)
+        times.append((time.perf_counter() - t0) * d.n_layers / CPU_LAYERS)
+        if budget_s is not None and time.perf_counter() - t_begin > budget_s:
+            break
+    return times
+
+
+def cores_used():
+    n = os.environ.get("OMP_NUM_THREADS")
+    return int(n) if n else (os.cpu_count() or 1)
+
+
+def run_reference(args, d, frames, prompt, pm, rank):
+    if rank != 0:
+        return
+    times = oracle_sample(d, frames, prompt, pm, args.tau_margin, args.warmup + args.steps, seed=args.seed)
+    timed = times[args.warmup:]
+    total = sum(timed)
+    v = len(timed) / total
+    sample = (f"each step: the CPU oracle (fp64, plain C + OpenMP) runs the first {CPU_LAYERS} of "
+              f"{d.n_layers} layers of the step (prefix pass and every decode pass), time scaled by "
+              f"{d.n_layers}/{CPU_LAYERS}")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": v, "unit": "steps/s", "n_gpus": args.gpus,
+        "steps": len(timed), "warmup": args.warmup, "ms_per_step": 1e3 * total / len(timed),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": config_block(d, args),
+        "cpu_baseline": {"value": v, "unit": "steps/s", "cores": cores_used(), "kind": "oracle", "sample": sample},
+        "e2e": {"value": v, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def config_block(d, args):
+    return {"workload": f"{args.config}: OpenVLA-7B-shaped Llama-2 backbone (32 layers, hidden 4096, "
+                        f"32x128 heads, SwiGLU 11008, vocab 32000, 256 action bins), 224x224 frame -> "
+                        f"256 patches, 27 text tokens, 7 autoregressive action tokens, 50-frame scene episode",
+            "global_batch": 1 * args.gpus, "seq_len": d.pass_len, "parallelism": f"replicas x{args.gpus}",
+            "tau_sim": f"{TAU_SIM[0]}/{TAU_SIM[1]}", "tau_margin": args.tau_margin,
+            "reuse_permille": "linear 900 -> 500", "l2": "inputs larger than L2 (13 GB of weights per pass)"}
+
+
+# ---------------------------------------------------------------------------
+# Our arm
+# ---------------------------------------------------------------------------
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default="openvla7b")
+    ap.add_argument("--tau-margin", type=float, default=0.05)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--cpu-budget", type=float, default=25.0, help="seconds of oracle work for cpu_baseline")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    d = synth.dims_for(args.config)
+    seed = args.seed + rank
+    frames = synth.make_episode(d, EPISODE, seed=seed, kind="scene")
+    prompt = synth.make_prompt(d, seed=seed)
+    pm = synth.linear_schedule(d.n_layers)
+
+    if args.impl == "reference":
+        run_reference(args, d, frames, prompt, pm, rank)
+        return
+
+    import torch
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    from paper_2608_10824_gb300 import Context
+
+    dev = torch.device("cuda", local)
+    w = synth.make_weights(d, seed=args.seed, device=dev)
+    ctx = Context(d, w, max_batch=1)
+    del w
+    torch.cuda.empty_cache()
+    cache = ctx.new_cache(1)
+    fr_dev = torch.from_numpy(frames).to(dev)          # [T][1][1][H][W][3]
+    pr_dev = torch.from_numpy(prompt).to(dev)
+    K, W = args.steps, args.warmup
+    outs = ctx.alloc_outputs(1, want=("M", "idx", "gate_auto"))
+    hist = {k: torch.zeros((K,) + tuple(v.shape), dtype=v.dtype, device=dev) for k, v in outs.items()}
+
+    def one_step(t, out):
+        if t % EPISODE == 0:
+            ctx.reset(cache)
+        ctx.step(cache, fr_dev[t % EPISODE], pr_dev, tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm,
+                 out=out)
+
+    def barrier():
+        torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+            torch.cuda.synchronize()
+
+    for t in range(W):
+        one_step(t, outs)
+    barrier()
+    assert ctx.sync_error() == 0
+    # ---- timed region: device-resident inputs ----
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk = Clocks(local)
+    time.sleep(0.3)
+    n0 = ctx.launch_count()
+    e0.record(stream)
+    for k in range(K):
+        one_step(W + k, {n: hist[n][k] for n in hist})
+    e1.record(stream)
+    barrier()
+    clocks = clk.stop()
+    launches = ctx.launch_count() - n0
+    ms = e0.elapsed_time(e1)
+    if dist is not None:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    assert ctx.sync_error() == 0
+    value = world * K / (ms / 1e3)
+
+    # ---- algorithmic work of the timed steps ----
+    Ms = hist["M"].cpu().numpy()[:, 0]
+    idxs = hist["idx"].cpu().numpy()[:, 0]
+    rec = hist["recomputed"].cpu().numpy()[:, 0]
+    pk, src = peaks()
+    F_tot = B_tot = 0.0
+    t_roof_step = t_roof_pass = 0.0
+    for k in range(K):
+        f_, b_, passes = step_work(d, Ms[k], idxs[k], bool(rec[k]))
+        F_tot += f_
+        B_tot += b_
+        t_roof_step += max(f_ / (pk["bf16_tflops"] * 1e12), b_ / (pk["hbm_gbs"] * 1e9))
+        t_roof_pass += sum(max(fp / (pk["bf16_tflops"] * 1e12), bp / (pk["hbm_gbs"] * 1e9)) for fp, bp in passes)
+    t_meas = ms / 1e3 / K
+
+    # ---- roofline of the dominant kernel (decode GEMV), second pass with per-launch events ----
+    ctx.prof_enable(True)
+    for k in range(K):
+        one_step(W + K + k, outs)
+    barrier()
+    ctx.prof_enable(False)
+    g_ms, g_n, g_bytes = ctx.prof_read(0)
+    p_ms, p_n, p_bytes = ctx.prof_read(1)
+    gemv_gbs = g_bytes / (g_ms / 1e3) / 1e9 if g_ms > 0 else None
+    gemm_gbs = p_bytes / (p_ms / 1e3) / 1e9 if p_ms > 0 else None
+
+    # ---- end to end through the public API with host buffers ----
+    fr_host = torch.from_numpy(frames).pin_memory()
+    pr_host = torch.from_numpy(prompt).pin_memory()
+    f_buf = torch.empty_like(fr_dev[0])
+    p_buf = torch.empty_like(pr_dev)
+    res_host = {n: torch.empty(outs[n].shape, dtype=outs[n].dtype).pin_memory()
+                for n in ("action_ids", "margins", "recomputed", "step_margin")}
+    h2d = f_buf.numel() * f_buf.element_size() + p_buf.numel() * p_buf.element_size()
+    d2h = sum(v.numel() * v.element_size() for v in res_host.values())
+    barrier()
+    t0 = time.perf_counter()
+    for k in range(K):
+        t = W + 2 * K + k
+        f_buf.copy_(fr_host[t % EPISODE], non_blocking=True)
+        p_buf.copy_(pr_host, non_blocking=True)
+        if t % EPISODE == 0:
+            ctx.reset(cache)
+        ctx.step(cache, f_buf, p_buf, tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm, out=outs)
+        for n, hbuf in res_host.items():
+            hbuf.copy_(outs[n], non_blocking=True)
+        torch.cuda.current_stream().synchronize()  # the action is needed before the next frame
+    e2e_s = time.perf_counter() - t0
+    if dist is not None:
+        t_ = torch.tensor([e2e_s], device=dev)
+        dist.all_reduce(t_, op=dist.ReduceOp.MAX)
+        e2e_s = float(t_.item())
+    e2e = world * K / e2e_s
+
+    # ---- CPU oracle baseline (rank 0, N = 1 only) ----
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        times = oracle_sample(d, frames, prompt, pm, args.tau_margin, 10 ** 6, seed=args.seed,
+                              budget_s=args.cpu_budget)
+        cpu = {"value": len(times) / sum(times), "unit": "steps/s", "cores": cores_used(), "kind": "oracle",
+               "sample": f"{len(times)} steps of the same episode; the oracle runs the first {CPU_LAYERS} of "
+                         f"{d.n_layers} layers of each step, time scaled by {d.n_layers}/{CPU_LAYERS}"}
+
+    if rank != 0:
+        return
+    line = {
+        "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": K, "warmup": W,
+        "ms_per_step": ms / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic (seeded scene frames, random-init N(0,0.02) bf16 weights)",
+        "config": config_block(d, args),
+        "step_roofline": {"frac": t_roof_step / K / t_meas, "frac_per_pass": t_roof_pass / K / t_meas,
+                          "t_roof_ms": 1e3 * t_roof_step / K, "t_meas_ms": 1e3 * t_meas,
+                          "alg_tflop_per_step": F_tot / K / 1e12, "alg_gb_per_step": B_tot / K / 1e9,
+                          "peaks": src, "fire_rate": float(rec.mean())},
+        "roofline": {"bound": "hbm", "achieved": gemv_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                     "frac": (gemv_gbs / pk["hbm_gbs"]) if gemv_gbs else None, "traffic": None,
+                     "kernel": "gemv_kernel (decode weight streaming)", "launches": g_n,
+                     "avg_launch_us": 1e3 * g_ms / max(g_n, 1), "peak_source": f"{src} hbm_gbs"},
+        "prefix_gemm": {"weight_gbs": gemm_gbs, "launches": p_n, "avg_launch_us": 1e3 * p_ms / max(p_n, 1)},
+        "clocks": clocks,
+        "e2e": {"value": e2e, "unit": "steps/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "note": "frame + prompt H2D from pinned memory, action ids/margins/flag D2H, synchronised "
+                        "every step (closed loop)"},
+        "gpu_launches": int(launches),
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -167,6 +167,18 @@ uint64_t vlac_launch_count(const vlac_ctx* ctx);
  * recorded status (VLAC_ERR_TIMEOUT when the wait gave up). */
 int vlac_selftest_wait(vlac_ctx* ctx, uint32_t spin_limit);
 
+/* Per-launch timing of the weight-streaming kernels, for roofline reports.
+ * While enabled, each launch of the kernel kinds below is bracketed by CUDA
+ * events recorded on the launching stream.  vlac_prof_read waits for those
+ * events, returns the summed device time, the number of launches and their
+ * algorithmic bytes, and forgets them.  kind 0 = decode GEMV (bytes: weights
+ * + inputs + outputs); kind 1 = prefix GEMM (bytes: weights only, the row
+ * count being device-resident). */
+#define VLAC_PROF_DECODE_GEMV 0
+#define VLAC_PROF_PREFIX_GEMM 1
+int vlac_prof_enable(vlac_ctx* ctx, int on);
+int vlac_prof_read(vlac_ctx* ctx, int kind, double* total_ms, uint64_t* launches, double* bytes);
+
 const char* vlac_strerror(int code);
 
 #ifdef __cplusplus

@@ -60,6 +60,15 @@ struct vlac_ctx {
   int* err_host = nullptr;  // pinned
   uint64_t launches = 0;
   uint32_t wait_limit = kDefaultWaitLimit;
+  // optional per-launch timing
+  struct ProfRec {
+    int kind;
+    double bytes;
+    cudaEvent_t a, b;
+  };
+  bool prof_on = false;
+  std::vector<ProfRec> prof;
+  std::vector<cudaEvent_t> ev_pool;
 };
 
 struct vlac_cache {
@@ -132,6 +141,11 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t c
 
 extern "C" int vlac_destroy(vlac_ctx* c) {
   if (!c) return VLAC_ERR_INVALID_ARG;
+  for (auto& r : c->prof) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  for (auto e : c->ev_pool) cudaEventDestroy(e);
   if (c->wmem) cudaFree(c->wmem);
   if (c->wsmem) cudaFree(c->wsmem);
   if (c->err_host) cudaFreeHost(c->err_host);
@@ -377,9 +391,49 @@ extern "C" int vlac_reset(vlac_cache* k, int seq, void* stream) {
 
 namespace {
 
+cudaEvent_t prof_event(vlac_ctx* c) {
+  if (!c->ev_pool.empty()) {
+    cudaEvent_t e = c->ev_pool.back();
+    c->ev_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Records events around one launch of a profiled kernel kind.
+struct ProfScope {
+  vlac_ctx* c;
+  cudaStream_t st;
+  vlac_ctx::ProfRec rec;
+  ProfScope(vlac_ctx* c_, int kind, double bytes, cudaStream_t s) : c(c_), st(s) {
+    if (!c->prof_on) return;
+    rec.kind = kind;
+    rec.bytes = bytes;
+    rec.a = prof_event(c);
+    rec.b = prof_event(c);
+    cudaEventRecord(rec.a, st);
+  }
+  ~ProfScope() {
+    if (!c->prof_on) return;
+    cudaEventRecord(rec.b, st);
+    c->prof.push_back(rec);
+  }
+};
+
+template <typename T>
+void gemv(vlac_ctx* c, const void* W, int N, int K, const T* x, int nb, cudaStream_t st) {
+  ProfScope ps(c, VLAC_PROF_DECODE_GEMV, (double)N * K * sizeof(T) + (double)nb * K * sizeof(T) + (double)nb * N * 4,
+               st);
+  launch_gemv<T>(static_cast<const T*>(W), N, K, x, nb, c->part, st);
+  c->launches += 1;
+}
+
 template <typename T>
 void gemm(vlac_ctx* c, const CUtensorMap* tmA, const CUtensorMap* tmW, const T* A, const void* W, const int* m_ptr,
           int N, int K, int splits, cudaStream_t st) {
+  ProfScope ps(c, VLAC_PROF_PREFIX_GEMM, (double)N * K * sizeof(T), st);
   if constexpr (sizeof(T) == 2) {
     launch_gemm_tc(tmA, tmW, m_ptr, c->rows_cap, N, K, splits, c->part, c->err, c->wait_limit, st);
   } else {
@@ -456,18 +510,18 @@ int step_impl(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, const int32_t* 
       c->launches += 1;
       for (int l = 0; l < L; ++l) {
         launch_layer_in<T>(rd, rd.off, B, 1, Hd, nullptr, 0, W(c->attn_norm[l]), eps, A, st);
-        launch_gemv<T>(W(c->wqkv[l]), 3 * Hd, Hd, A, B, c->part, st);
+        gemv<T>(c, c->wqkv[l], 3 * Hd, Hd, A, B, st);
         launch_qkv_epilogue<T>(rd, B, 1, nh, hd, c->part, 1, 0, c->rope_cos, c->rope_sin, Q, Kc + l * kv_layer,
                                Vc + l * kv_layer, k->kv_seq_stride, c->Tc, st);
         launch_attention<T>(rd, B, 1, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc,
                             c->P, 0, D, AO, st);
-        launch_gemv<T>(W(c->wo[l]), Hd, Hd, AO, B, c->part, st);
+        gemv<T>(c, c->wo[l], Hd, Hd, AO, B, st);
         launch_residual_norm<T>(rd, B, 1, Hd, c->part, 1, 0, W(c->ffn_norm[l]), eps, A, st);
-        launch_gemv<T>(W(c->wgu[l]), 2 * F, Hd, A, B, c->part, st);
+        gemv<T>(c, c->wgu[l], 2 * F, Hd, A, B, st);
         launch_swiglu<T>(rd, B, 1, F, c->part, 1, 0, G, st);
-        launch_gemv<T>(W(c->wd[l]), Hd, F, G, B, c->part, st);
+        gemv<T>(c, c->wd[l], Hd, F, G, B, st);
         launch_residual(rd, B, 1, Hd, c->part, 1, 0, st);
-        c->launches += 10;
+        c->launches += 6;
       }
       launch_head<T>(c->Xd, nullptr, Hd, 1, B, Hd, nb, W(c->final_norm), W(c->head_w), eps, D, a, out->action_ids,
                      out->margins, out->logit_gap, out->logits, st);
@@ -549,6 +603,40 @@ extern "C" int vlac_selftest_wait(vlac_ctx* c, uint32_t spin_limit) {
   CK(cudaMemcpy(&e, c->err, sizeof(int), cudaMemcpyDeviceToHost));
   CK(cudaMemset(c->err, 0, sizeof(int)));
   return e;
+}
+
+extern "C" int vlac_prof_enable(vlac_ctx* c, int on) {
+  if (!c) return VLAC_ERR_INVALID_ARG;
+  c->prof_on = on != 0;
+  return VLAC_OK;
+}
+
+extern "C" int vlac_prof_read(vlac_ctx* c, int kind, double* total_ms, uint64_t* launches, double* bytes) {
+  if (!c || !total_ms || !launches || !bytes) return VLAC_ERR_INVALID_ARG;
+  double ms = 0, by = 0;
+  uint64_t n = 0;
+  std::vector<vlac_ctx::ProfRec> keep;
+  for (auto& r : c->prof) {
+    if (r.kind != kind) {
+      keep.push_back(r);
+      continue;
+    }
+    float t = 0.f;
+    if (cudaEventSynchronize(r.b) != cudaSuccess || cudaEventElapsedTime(&t, r.a, r.b) != cudaSuccess) {
+      (void)cudaGetLastError();
+      return VLAC_ERR_CUDA;
+    }
+    ms += t;
+    by += r.bytes;
+    ++n;
+    c->ev_pool.push_back(r.a);
+    c->ev_pool.push_back(r.b);
+  }
+  c->prof.swap(keep);
+  *total_ms = ms;
+  *launches = n;
+  *bytes = by;
+  return VLAC_OK;
 }
 
 extern "C" const char* vlac_strerror(int code) {

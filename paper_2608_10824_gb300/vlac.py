@@ -67,7 +67,7 @@ class StepOut(C.Structure):
 
 EXPORTS = ["vlac_create", "vlac_destroy", "vlac_cache_bytes", "vlac_cache_init", "vlac_cache_destroy",
            "vlac_step", "vlac_reset", "vlac_sync_error", "vlac_launch_count", "vlac_selftest_wait",
-           "vlac_strerror"]
+           "vlac_prof_enable", "vlac_prof_read", "vlac_strerror"]
 
 
 def lib():
@@ -91,6 +91,9 @@ def lib():
             L.vlac_launch_count.argtypes = [vp]
             L.vlac_launch_count.restype = C.c_uint64
             L.vlac_selftest_wait.argtypes = [vp, C.c_uint32]
+            L.vlac_prof_enable.argtypes = [vp, i32]
+            L.vlac_prof_read.argtypes = [vp, i32, C.POINTER(C.c_double), C.POINTER(C.c_uint64),
+                                         C.POINTER(C.c_double)]
             L.vlac_strerror.argtypes = [i32]
             L.vlac_strerror.restype = C.c_char_p
             for name in EXPORTS:
@@ -212,6 +215,15 @@ class Context:
 
     def launch_count(self) -> int:
         return int(lib().vlac_launch_count(self._h))
+
+    def prof_enable(self, on: bool = True):
+        _check(lib().vlac_prof_enable(self._h, int(on)), "vlac_prof_enable")
+
+    def prof_read(self, kind: int):
+        """(total device ms, launches, algorithmic bytes) of the timed launches of `kind`."""
+        ms, n, by = C.c_double(), C.c_uint64(), C.c_double()
+        _check(lib().vlac_prof_read(self._h, kind, C.byref(ms), C.byref(n), C.byref(by)), "vlac_prof_read")
+        return ms.value, n.value, by.value
 
     def selftest_wait(self, spin_limit: int) -> int:
         return lib().vlac_selftest_wait(self._h, spin_limit)
