@@ -56,6 +56,8 @@ def step_work(d, M_seq, idx_seq, recomputed: bool):
     counts M[l] and recompute order idx (what the method computes)."""
     Hd, F, L, nb = d.hidden, d.ffn, d.n_layers, d.n_bins
     P, D = d.prefix_len, d.n_action
+    M_seq = [int(m) for m in M_seq]
+    idx_seq = np.asarray(idx_seq, dtype=np.int64)
     per_row = 2 * (4 * Hd * Hd + 3 * F * Hd)            # QKV + O + gate/up + down
     w_bytes = L * (4 * Hd * Hd + 3 * F * Hd) * 2        # bf16 weights of one pass
     head_bytes = nb * Hd * 2
@@ -64,7 +66,7 @@ def step_work(d, M_seq, idx_seq, recomputed: bool):
     passes = []
     # prefix pass
     fp = 0.0
-    bp = w_bytes + head_bytes
+    bp = float(w_bytes + head_bytes)
     for l in range(L):
         rows = idx_seq[:M_seq[l]]
         fp += M_seq[l] * per_row + 4 * Hd * float(np.sum(rows + 1))   # QK^T and PV over j <= pos
