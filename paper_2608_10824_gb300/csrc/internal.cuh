@@ -37,6 +37,31 @@ struct Rows {
   float* X;
 };
 
+// Arguments of the fused decode GEMV (one new row per sequence).  Output row
+// pairs: QKV -> (i, i + head_dim/2) of one head of q, k or v; SwiGLU ->
+// (gate j, up j); residual -> (2p, 2p + 1).
+enum { kEpiQkvRope = 0, kEpiResid = 1, kEpiSwiglu = 2 };
+struct DGemv {
+  const void* W;  // [rows][K] weights (T)
+  int n_pairs;
+  int K;
+  const float* X;     // RMSNorm prologue: fp32 residual rows [nb][K]
+  const void* gain;   // RMSNorm gains (T)
+  float eps;
+  const void* xin;    // plain input rows [nb][K] (T) when there is no prologue
+  float* Xres;        // residual epilogue: Xres[b][n] += y
+  int n_out;          // row stride of Xres
+  void* Q;            // QKV epilogue
+  void* Kc;
+  void* Vc;
+  size_t kv_seq_stride;
+  int Tc, pos, n_heads, head_dim;
+  const float* rope_cos;
+  const float* rope_sin;
+  void* G;            // SwiGLU epilogue: G[b][j]
+  int ffn;
+};
+
 // ---- scalar helpers --------------------------------------------------------
 template <typename T> __device__ __forceinline__ float to_f(T v);
 template <> __device__ __forceinline__ float to_f<float>(float v) { return v; }
@@ -139,5 +164,14 @@ void launch_gemm_simt(const T* A, const T* W, const int* m_ptr, int m_cap, int N
 template <typename T>
 void launch_gemv(const T* W, int N, int K, const T* x, int nb, float* y, cudaStream_t st);
 int launch_wait_selftest(int* err, uint32_t spin_limit, cudaStream_t st);
+template <typename T>
+void launch_dgemv(const DGemv& a, int epi, int nb, cudaStream_t st);
+template <typename T>
+void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride,
+                          int Tc, int pos, float* part, T* O, cudaStream_t st);
+template <typename T>
+void launch_head2(const float* X, const int* row_of_seq, size_t x_seq_stride, int rows_per_seq, int B, int hidden,
+                  int n_bins, const T* final_norm, const T* head_w, float eps, float* logits_ws, int D, int tok0,
+                  int32_t* ids, float* margins, float* gaps, float* logits, cudaStream_t st);
 
 }  // namespace vlac

@@ -57,6 +57,7 @@ struct vlac_ctx {
   int3* stats;
   uint8_t *mask, *full;
   int *idx, *M, *off, *emit_slot, *off_dec, *idx_dec, *err;
+  float *logits_ws, *attn_part;
   int* err_host = nullptr;  // pinned
   uint64_t launches = 0;
   uint32_t wait_limit = kDefaultWaitLimit;
@@ -98,6 +99,7 @@ static int check_dims(const vlac_dims* d) {
       d->img_h < d->patch || d->img_w < d->patch || d->img_h % d->patch || d->img_w % d->patch || d->n_views < 1 ||
       d->n_text < 1 || d->n_action < 1 || d->proprio_dim < 0 || d->proprio_dim > 256 || d->max_batch < 1 ||
       d->max_batch > 8 || (d->parallel != 0 && d->parallel != 1) || (!d->parallel && d->n_text < 2) ||
+      d->n_bins % 16 ||
       !(d->rms_eps >= 0.f) || !(d->rope_theta > 0.f))
     return VLAC_ERR_INVALID_ARG;
   if (d->dtype != VLAC_F32 && d->dtype != VLAC_BF16) return VLAC_ERR_INVALID_ARG;
@@ -285,6 +287,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->off_dec, (Bm + 1) * 4, base);
     sc.take(c->idx_dec, Bm * 4, base);
     sc.take(c->err, 4, base);
+    sc.take(c->logits_ws, Bm * (d.parallel ? d.n_action : 1) * d.n_bins * 4, base);
+    sc.take(c->attn_part, Bm * d.n_heads * ((c->Tc + 31) / 32) * (d.head_dim + 2) * 4, base);
   };
   plan_s(nullptr);
   if (cudaMalloc(&c->wsmem, sc.off) != cudaSuccess) {
@@ -423,10 +427,11 @@ struct ProfScope {
 };
 
 template <typename T>
-void gemv(vlac_ctx* c, const void* W, int N, int K, const T* x, int nb, cudaStream_t st) {
-  ProfScope ps(c, VLAC_PROF_DECODE_GEMV, (double)N * K * sizeof(T) + (double)nb * K * sizeof(T) + (double)nb * N * 4,
+void dgemv(vlac_ctx* c, const DGemv& a, int epi, int nb, cudaStream_t st) {
+  ProfScope ps(c, VLAC_PROF_DECODE_GEMV,
+               (double)2 * a.n_pairs * a.K * sizeof(T) + (double)nb * a.K * sizeof(T) + (double)nb * 2 * a.n_pairs * 4,
                st);
-  launch_gemv<T>(static_cast<const T*>(W), N, K, x, nb, c->part, st);
+  launch_dgemv<T>(a, epi, nb, st);
   c->launches += 1;
 }
 
@@ -498,34 +503,74 @@ int step_impl(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, const int32_t* 
     c->launches += 6;
   }
   // action head on the prefix pass: the last text row, or the parallel action block
-  launch_head<T>(c->X, c->emit_slot, (size_t)S * Hd, d.parallel ? D : 1, B, Hd, nb, W(c->final_norm), W(c->head_w),
-                 eps, D, 0, out->action_ids, out->margins, out->logit_gap, out->logits, st);
-  c->launches += 1;
+  launch_head2<T>(c->X, c->emit_slot, (size_t)S * Hd, d.parallel ? D : 1, B, Hd, nb, W(c->final_norm),
+                  W(c->head_w), eps, c->logits_ws, D, 0, out->action_ids, out->margins, out->logit_gap, out->logits,
+                  st);
+  c->launches += 2;
 
   if (!d.parallel) {
-    Rows rd{c->off_dec, c->idx_dec, 1, c->Xd};
+    // autoregressive decode: one row per sequence, fused GEMVs
     for (int a = 1; a < D; ++a) {
+      const int pos = c->P + a - 1;
       launch_decode_embed<T>(B, a, D, c->P, Hd, d.vocab, nb, W(c->tok_emb), out->action_ids, forced, c->prm, c->Xd,
                              c->idx_dec, c->err, st);
       c->launches += 1;
       for (int l = 0; l < L; ++l) {
-        launch_layer_in<T>(rd, rd.off, B, 1, Hd, nullptr, 0, W(c->attn_norm[l]), eps, A, st);
-        gemv<T>(c, c->wqkv[l], 3 * Hd, Hd, A, B, st);
-        launch_qkv_epilogue<T>(rd, B, 1, nh, hd, c->part, 1, 0, c->rope_cos, c->rope_sin, Q, Kc + l * kv_layer,
-                               Vc + l * kv_layer, k->kv_seq_stride, c->Tc, st);
-        launch_attention<T>(rd, B, 1, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc,
-                            c->P, 0, D, AO, st);
-        gemv<T>(c, c->wo[l], Hd, Hd, AO, B, st);
-        launch_residual_norm<T>(rd, B, 1, Hd, c->part, 1, 0, W(c->ffn_norm[l]), eps, A, st);
-        gemv<T>(c, c->wgu[l], 2 * F, Hd, A, B, st);
-        launch_swiglu<T>(rd, B, 1, F, c->part, 1, 0, G, st);
-        gemv<T>(c, c->wd[l], Hd, F, G, B, st);
-        launch_residual(rd, B, 1, Hd, c->part, 1, 0, st);
-        c->launches += 6;
+        DGemv g{};
+        g.eps = eps;
+        g.n_heads = nh;
+        g.head_dim = hd;
+        // q, k, v with the attention RMSNorm prologue, RoPE and the K/V scatter
+        g.W = c->wqkv[l];
+        g.n_pairs = 3 * Hd / 2;
+        g.K = Hd;
+        g.X = c->Xd;
+        g.gain = c->attn_norm[l];
+        g.Q = Q;
+        g.Kc = Kc + l * kv_layer;
+        g.Vc = Vc + l * kv_layer;
+        g.kv_seq_stride = k->kv_seq_stride;
+        g.Tc = c->Tc;
+        g.pos = pos;
+        g.rope_cos = c->rope_cos;
+        g.rope_sin = c->rope_sin;
+        dgemv<T>(c, g, kEpiQkvRope, B, st);
+        launch_dec_attention<T>(B, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, pos,
+                                c->attn_part, AO, st);
+        c->launches += 2;
+        // o-projection + residual
+        DGemv o{};
+        o.W = c->wo[l];
+        o.n_pairs = Hd / 2;
+        o.K = Hd;
+        o.xin = AO;
+        o.Xres = c->Xd;
+        o.n_out = Hd;
+        dgemv<T>(c, o, kEpiResid, B, st);
+        // gate/up with the MLP RMSNorm prologue and SwiGLU
+        DGemv u{};
+        u.W = c->wgu[l];
+        u.n_pairs = F;
+        u.K = Hd;
+        u.X = c->Xd;
+        u.gain = c->ffn_norm[l];
+        u.eps = eps;
+        u.G = G;
+        u.ffn = F;
+        dgemv<T>(c, u, kEpiSwiglu, B, st);
+        // down-projection + residual
+        DGemv dn{};
+        dn.W = c->wd[l];
+        dn.n_pairs = Hd / 2;
+        dn.K = F;
+        dn.xin = G;
+        dn.Xres = c->Xd;
+        dn.n_out = Hd;
+        dgemv<T>(c, dn, kEpiResid, B, st);
       }
-      launch_head<T>(c->Xd, nullptr, Hd, 1, B, Hd, nb, W(c->final_norm), W(c->head_w), eps, D, a, out->action_ids,
-                     out->margins, out->logit_gap, out->logits, st);
-      c->launches += 1;
+      launch_head2<T>(c->Xd, nullptr, Hd, 1, B, Hd, nb, W(c->final_norm), W(c->head_w), eps, c->logits_ws, D, a,
+                      out->action_ids, out->margins, out->logit_gap, out->logits, st);
+      c->launches += 2;
     }
   }
   launch_finish(B, D, c->prm, out->margins, out->logit_gap, k->m_prev, k->valid, out->step_margin, st);
