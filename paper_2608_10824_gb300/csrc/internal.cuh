@@ -70,6 +70,18 @@ template <typename T> __device__ __forceinline__ T from_f(float v);
 template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
 template <> __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
 
+// Programmatic dependent launch.  Every kernel of the step calls pdl_wait()
+// before it touches data written by an earlier kernel of the stream (a no-op
+// when the launch did not allow early start), and pdl_trigger() once its
+// dependents may be scheduled.  Work that reads only constant data (weight
+// prefetches) may run before pdl_wait().
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+// Starts pulling [p, p + bytes) into L2 (bytes: multiple of 16, p 16-byte aligned).
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
 __device__ __forceinline__ void set_error(int* err, int code) {
   if (err) atomicCAS(err, 0, code);
 }
@@ -102,6 +114,24 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   float r = red[0];
   __syncthreads();
   return r;
+}
+
+// Launch with optional programmatic stream serialization (the kernel may
+// start while its predecessor drains; it must call pdl_wait()).
+extern bool g_pdl;
+template <typename... KArgs, typename... Args>
+inline void launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = g_pdl ? 1 : 0;
+  cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
 }  // namespace vlac
@@ -145,15 +175,27 @@ template <typename T>
 void launch_attention(Rows rows, int B, int S, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc,
                       size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, T* O, cudaStream_t st);
 template <typename T>
-void launch_head(const float* X, const int* row_of_seq, size_t x_seq_stride, int rows_per_seq, int B,
-                 int hidden, int n_bins, const T* final_norm, const T* head_w, float eps, int D, int tok0,
-                 int32_t* ids, float* margins, float* gaps, float* logits, cudaStream_t st);
-template <typename T>
 void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
                          const int32_t* ids, const int32_t* forced, const StepParams* prm, float* Xd,
                          int* idx_dec, int* err, cudaStream_t st);
 void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps,
                    float* m_prev, uint8_t* valid, float* user_step_margin, cudaStream_t st);
+
+// Copies of the caller's per-step inputs into the context's staging buffers
+// (and the step scalars into device memory), and of the step's outputs back
+// to the caller's buffers.  A NULL source (or destination) is skipped.
+struct CopySpan {
+  const void* src;
+  void* dst;
+  size_t bytes;
+};
+constexpr int kMaxSpans = 12;
+struct CopyList {
+  CopySpan span[kMaxSpans];
+  int n;
+};
+void launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st);
+void launch_copies(const CopyList& list, cudaStream_t st);
 
 // GEMMs: out[s][m][n] = sum over split s of A[m][k] * W[n][k]; rows m < *m_ptr.
 void launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
@@ -161,8 +203,6 @@ void launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmW, const int* m
 template <typename T>
 void launch_gemm_simt(const T* A, const T* W, const int* m_ptr, int m_cap, int N, int K, float* out,
                       cudaStream_t st);
-template <typename T>
-void launch_gemv(const T* W, int N, int K, const T* x, int nb, float* y, cudaStream_t st);
 int launch_wait_selftest(int* err, uint32_t spin_limit, cudaStream_t st);
 template <typename T>
 void launch_dgemv(const DGemv& a, int epi, int nb, cudaStream_t st);

@@ -17,6 +17,8 @@ __global__ void __launch_bounds__(256) attn_kernel(Rows rows, int n_heads, const
                                                    const T* __restrict__ Kc, const T* __restrict__ Vc,
                                                    size_t kv_seq_stride, int Tc, int P, int parallel, int n_action,
                                                    float scale, T* __restrict__ O) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int QT = 16, KT = 32, NC = HD / 32;
   __shared__ float Kt[HD][KT + 1];  // padded: conflict-free transposed stores
   __shared__ float Vs[KT][HD];
@@ -120,11 +122,11 @@ void launch_attention(Rows rows, int B, int S, int n_heads, int head_dim, const 
   dim3 grid((S + 15) / 16, n_heads, B);
   const float scale = 1.0f / sqrtf((float)head_dim);
   if (head_dim == 128)
-    attn_kernel<T, 128><<<grid, 256, 0, st>>>(rows, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, P, parallel, n_action,
-                                              scale, O);
+    launch_k(attn_kernel<T, 128>, grid, dim3(256), 0, st, rows, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, P, parallel,
+             n_action, scale, O);
   else
-    attn_kernel<T, 64><<<grid, 256, 0, st>>>(rows, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, P, parallel, n_action,
-                                             scale, O);
+    launch_k(attn_kernel<T, 64>, grid, dim3(256), 0, st, rows, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, P, parallel,
+             n_action, scale, O);
 }
 
 template void launch_attention<float>(Rows, int, int, int, int, const float*, const float*, const float*, size_t,

@@ -95,11 +95,9 @@ __global__ void __launch_bounds__(256) dgemv_kernel(DGemv a) {
   extern __shared__ __align__(16) uint8_t dsm[];
   T* xs = reinterpret_cast<T*>(dsm);
   const int K = a.K;
-  if constexpr (NORM) norm_rows_to_smem<T, NB>(a.X, static_cast<const T*>(a.gain), K, a.eps, xs);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int p = blockIdx.x * (blockDim.x >> 5) + warp;
-  if (p >= a.n_pairs) return;
-  int r1, r2;
+  int r1 = 0, r2 = 0;
   int sec = 0, h = 0, e = 0;
   const int hd = a.head_dim, half = hd >> 1;
   if constexpr (EPI == kEpiQkvRope) {
@@ -117,6 +115,16 @@ __global__ void __launch_bounds__(256) dgemv_kernel(DGemv a) {
     r1 = 2 * p;
     r2 = 2 * p + 1;
   }
+  // the weight rows do not depend on earlier kernels: start pulling them into
+  // L2 while the previous kernel of the stream drains
+  if (p < a.n_pairs && lane == 0) {
+    prefetch_l2(static_cast<const T*>(a.W) + (size_t)r1 * K, (uint32_t)(K * sizeof(T)));
+    prefetch_l2(static_cast<const T*>(a.W) + (size_t)r2 * K, (uint32_t)(K * sizeof(T)));
+  }
+  pdl_wait();
+  pdl_trigger();
+  if constexpr (NORM) norm_rows_to_smem<T, NB>(a.X, static_cast<const T*>(a.gain), K, a.eps, xs);
+  if (p >= a.n_pairs) return;
   const T* W = static_cast<const T*>(a.W);
   const int kv = K / V;
   const uint4* w1 = reinterpret_cast<const uint4*>(W + (size_t)r1 * K);
@@ -205,9 +213,12 @@ static void dgemv_nb(const DGemv& a, cudaStream_t st) {
   const int blocks = (a.n_pairs + warps - 1) / warps;
   const size_t smem = NORM ? (size_t)NB * a.K * sizeof(T) : 0;
   constexpr int U = NB <= 2 ? 4 : 2;
-  if (smem > 48 * 1024) cudaFuncSetAttribute(dgemv_kernel<T, NB, EPI, NORM, U>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  dgemv_kernel<T, NB, EPI, NORM, U><<<blocks, warps * 32, smem, st>>>(a);
+  static size_t smem_set = 48 * 1024;  // raised once per instantiation, before any graph capture of it
+  if (smem > smem_set) {
+    cudaFuncSetAttribute(dgemv_kernel<T, NB, EPI, NORM, U>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    smem_set = smem;
+  }
+  launch_k(dgemv_kernel<T, NB, EPI, NORM, U>, dim3(blocks), dim3(warps * 32), smem, st, a);
 }
 
 template <typename T, int EPI, bool NORM>
@@ -244,6 +255,8 @@ __global__ void __launch_bounds__(32) dec_attn_partial_kernel(const T* __restric
                                                               const T* __restrict__ Vc, size_t kv_seq_stride, int Tc,
                                                               int pos, int n_heads, float scale,
                                                               float* __restrict__ part, int nchunk) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int EPL = HD / 32;
   const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z, lane = threadIdx.x;
   const int hidden = n_heads * HD;
@@ -287,6 +300,8 @@ __global__ void __launch_bounds__(32) dec_attn_partial_kernel(const T* __restric
 template <typename T, int HD>
 __global__ void __launch_bounds__(HD) dec_attn_combine_kernel(const float* __restrict__ part, int nchunk,
                                                               int n_heads, T* __restrict__ O) {
+  pdl_wait();
+  pdl_trigger();
   const int h = blockIdx.x, b = blockIdx.y, e = threadIdx.x;
   const float* base = part + ((size_t)b * n_heads + h) * nchunk * (HD + 2);
   float M = -INFINITY;
@@ -307,13 +322,13 @@ void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T*
   const int nchunk = (pos + 1 + 31) / 32;
   const float scale = 1.0f / sqrtf((float)head_dim);
   if (head_dim == 128) {
-    dec_attn_partial_kernel<T, 128><<<dim3(nchunk, n_heads, B), 32, 0, st>>>(Q, Kc, Vc, kv_seq_stride, Tc, pos,
-                                                                             n_heads, scale, part, nchunk);
-    dec_attn_combine_kernel<T, 128><<<dim3(n_heads, B), 128, 0, st>>>(part, nchunk, n_heads, O);
+    launch_k(dec_attn_partial_kernel<T, 128>, dim3(nchunk, n_heads, B), dim3(32), 0, st, Q, Kc, Vc, kv_seq_stride,
+             Tc, pos, n_heads, scale, part, nchunk);
+    launch_k(dec_attn_combine_kernel<T, 128>, dim3(n_heads, B), dim3(128), 0, st, part, nchunk, n_heads, O);
   } else {
-    dec_attn_partial_kernel<T, 64><<<dim3(nchunk, n_heads, B), 32, 0, st>>>(Q, Kc, Vc, kv_seq_stride, Tc, pos,
-                                                                            n_heads, scale, part, nchunk);
-    dec_attn_combine_kernel<T, 64><<<dim3(n_heads, B), 64, 0, st>>>(part, nchunk, n_heads, O);
+    launch_k(dec_attn_partial_kernel<T, 64>, dim3(nchunk, n_heads, B), dim3(32), 0, st, Q, Kc, Vc, kv_seq_stride,
+             Tc, pos, n_heads, scale, part, nchunk);
+    launch_k(dec_attn_combine_kernel<T, 64>, dim3(n_heads, B), dim3(64), 0, st, part, nchunk, n_heads, O);
   }
 }
 template void launch_dec_attention<float>(int, int, int, const float*, const float*, const float*, size_t, int, int,
@@ -332,6 +347,8 @@ __global__ void __launch_bounds__(256) head_logits_kernel(const float* __restric
                                                           const T* __restrict__ final_norm,
                                                           const T* __restrict__ head_w, float eps,
                                                           float* __restrict__ logits_ws) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ __align__(16) uint8_t dsm[];
   T* xs = reinterpret_cast<T*>(dsm);
   const int j = blockIdx.y, b = blockIdx.z;
@@ -370,6 +387,8 @@ __global__ void __launch_bounds__(256) head_logits_kernel(const float* __restric
 __global__ void __launch_bounds__(32) head_margin_kernel(const float* __restrict__ logits_ws, int n_bins, int D, int tok0,
                                                          int32_t* __restrict__ ids, float* __restrict__ margins,
                                                          float* __restrict__ gaps, float* __restrict__ logits) {
+  pdl_wait();
+  pdl_trigger();
   const int j = blockIdx.x, b = blockIdx.y, lane = threadIdx.x;
   const float* lg = logits_ws + ((size_t)b * gridDim.x + j) * n_bins;
   float bv = -INFINITY;
@@ -411,10 +430,10 @@ void launch_head2(const float* X, const int* row_of_seq, size_t x_seq_stride, in
                   int n_bins, const T* final_norm, const T* head_w, float eps, float* logits_ws, int D, int tok0,
                   int32_t* ids, float* margins, float* gaps, float* logits, cudaStream_t st) {
   const size_t smem = (size_t)hidden * sizeof(T);
-  head_logits_kernel<T><<<dim3(n_bins / 16, rows_per_seq, B), 256, smem, st>>>(X, row_of_seq, x_seq_stride, hidden,
-                                                                              n_bins, final_norm, head_w, eps,
-                                                                              logits_ws);
-  head_margin_kernel<<<dim3(rows_per_seq, B), 32, 0, st>>>(logits_ws, n_bins, D, tok0, ids, margins, gaps, logits);
+  launch_k(head_logits_kernel<T>, dim3(n_bins / 16, rows_per_seq, B), dim3(256), smem, st, X, row_of_seq,
+           x_seq_stride, hidden, n_bins, final_norm, head_w, eps, logits_ws);
+  launch_k(head_margin_kernel, dim3(rows_per_seq, B), dim3(32), 0, st, logits_ws, n_bins, D, tok0, ids, margins, gaps,
+           logits);
 }
 template void launch_head2<float>(const float*, const int*, size_t, int, int, int, int, const float*, const float*,
                                   float, float*, int, int, int32_t*, float*, float*, float*, cudaStream_t);

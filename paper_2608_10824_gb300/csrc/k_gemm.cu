@@ -25,6 +25,7 @@ constexpr int kMaxStages = 8;
 constexpr int kWTileBytes = kBM * kBK * 2;  // 16 KB
 constexpr int kSmemBytes = 212 * 1024;      // dynamic shared memory (tiles only)
 constexpr int kThreads = 192;               // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
+constexpr int kPrefetchChunks = 16;         // weight K-chunks pulled into L2 before the dependency wait
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -139,6 +140,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   uint8_t* tiles = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    // the weight tiles do not depend on earlier kernels: start pulling the
+    // first ones into L2 while the previous kernel drains
+    const int k0 = blockIdx.y * chunks_per_split;
+    const int k1 = min(min(k0 + chunks_per_split, k_chunks), k0 + kPrefetchChunks);
+    for (int kc = k0; kc < k1; ++kc)
+      asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                       reinterpret_cast<uint64_t>(&tmW)),
+                   "r"(kc * kBK), "r"((int)blockIdx.x * kBM)
+                   : "memory");
+  }
+  pdl_wait();
+  pdl_trigger();
   const int M = min(*m_ptr, m_cap);
   if (M <= 0) return;
   const int n0 = blockIdx.x * kBM;
@@ -313,121 +327,9 @@ void launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmW, const int* m
   const int k_chunks = K / tc::kBK;
   const int cps = (k_chunks + splits - 1) / splits;
   dim3 grid(N / tc::kBM, splits);
-  tc::gemm_tc_kernel<<<grid, tc::kThreads, tc::kSmemBytes, st>>>(*tmA, *tmW, m_ptr, m_cap, N, k_chunks, cps, out,
-                                                                 (size_t)m_cap * N, err, wait_limit);
+  launch_k(tc::gemm_tc_kernel, grid, dim3(tc::kThreads), tc::kSmemBytes, st, *tmA, *tmW, m_ptr, m_cap, N, k_chunks,
+           cps, out, (size_t)m_cap * N, err, wait_limit);
 }
-
-// =============================================================================
-// Decode GEMV: y[b][n] = sum_k x[b][k] * W[n][k] for nb <= 8 rows of x.
-// =============================================================================
-
-__device__ __forceinline__ uint4 ld_stream(const void* p) {
-  uint4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "l"(p));
-  return v;
-}
-
-template <typename T> struct Vec;
-template <> struct Vec<bf16> { static constexpr int n = 8; };
-template <> struct Vec<float> { static constexpr int n = 4; };
-
-template <typename T>
-__device__ __forceinline__ void unpack(const uint4& u, float* f) {
-  if constexpr (sizeof(T) == 2) {
-    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      f[2 * i] = __uint_as_float(w[i] << 16);
-      f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
-    }
-  } else {
-    f[0] = __uint_as_float(u.x);
-    f[1] = __uint_as_float(u.y);
-    f[2] = __uint_as_float(u.z);
-    f[3] = __uint_as_float(u.w);
-  }
-}
-
-// Each warp owns ROWS consecutive weight rows; lanes stride over K in
-// 16-byte vectors, UNROLL vectors in flight per row.  Fixed reduction order.
-template <typename T, int NB, int ROWS, int UNROLL>
-__global__ void __launch_bounds__(256) gemv_kernel(const T* __restrict__ W, int N, int K, const T* __restrict__ x,
-                                                   float* __restrict__ y) {
-  constexpr int V = Vec<T>::n;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int row0 = (blockIdx.x * (blockDim.x >> 5) + warp) * ROWS;
-  if (row0 >= N) return;
-  const int kv = K / V;  // vectors per row
-  float acc[ROWS][NB];
-#pragma unroll
-  for (int r = 0; r < ROWS; ++r)
-#pragma unroll
-    for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
-  const uint4* Wv = reinterpret_cast<const uint4*>(W);
-  const uint4* xv = reinterpret_cast<const uint4*>(x);
-  for (int k0 = lane; k0 < kv; k0 += 32 * UNROLL) {
-    uint4 wr[UNROLL][ROWS];
-#pragma unroll
-    for (int u = 0; u < UNROLL; ++u) {
-      const int k = k0 + u * 32;
-#pragma unroll
-      for (int r = 0; r < ROWS; ++r)
-        if (k < kv && row0 + r < N) wr[u][r] = ld_stream(Wv + (size_t)(row0 + r) * kv + k);
-        else wr[u][r] = make_uint4(0, 0, 0, 0);
-    }
-#pragma unroll
-    for (int u = 0; u < UNROLL; ++u) {
-      const int k = k0 + u * 32;
-      if (k >= kv) break;
-#pragma unroll
-      for (int b = 0; b < NB; ++b) {
-        float xf[V];
-        unpack<T>(__ldg(xv + (size_t)b * kv + k), xf);
-#pragma unroll
-        for (int r = 0; r < ROWS; ++r) {
-          float wf[V];
-          unpack<T>(wr[u][r], wf);
-#pragma unroll
-          for (int e = 0; e < V; ++e) acc[r][b] = fmaf(wf[e], xf[e], acc[r][b]);
-        }
-      }
-    }
-  }
-#pragma unroll
-  for (int r = 0; r < ROWS; ++r)
-#pragma unroll
-    for (int b = 0; b < NB; ++b) {
-      const float s = warp_sum(acc[r][b]);
-      if (lane == 0 && row0 + r < N) y[(size_t)b * N + row0 + r] = s;
-    }
-}
-
-template <typename T, int NB>
-static void gemv_nb(const T* W, int N, int K, const T* x, float* y, cudaStream_t st) {
-  constexpr int ROWS = NB <= 2 ? 2 : 1;
-  constexpr int UNROLL = NB <= 2 ? 4 : 2;
-  const int warps = 8;
-  const int blocks = (N + warps * ROWS - 1) / (warps * ROWS);
-  gemv_kernel<T, NB, ROWS, UNROLL><<<blocks, warps * 32, 0, st>>>(W, N, K, x, y);
-}
-
-template <typename T>
-void launch_gemv(const T* W, int N, int K, const T* x, int nb, float* y, cudaStream_t st) {
-  switch (nb) {
-    case 1: gemv_nb<T, 1>(W, N, K, x, y, st); break;
-    case 2: gemv_nb<T, 2>(W, N, K, x, y, st); break;
-    case 3: gemv_nb<T, 3>(W, N, K, x, y, st); break;
-    case 4: gemv_nb<T, 4>(W, N, K, x, y, st); break;
-    case 5: gemv_nb<T, 5>(W, N, K, x, y, st); break;
-    case 6: gemv_nb<T, 6>(W, N, K, x, y, st); break;
-    case 7: gemv_nb<T, 7>(W, N, K, x, y, st); break;
-    default: gemv_nb<T, 8>(W, N, K, x, y, st); break;
-  }
-}
-template void launch_gemv<float>(const float*, int, int, const float*, int, float*, cudaStream_t);
-template void launch_gemv<bf16>(const bf16*, int, int, const bf16*, int, float*, cudaStream_t);
 
 // =============================================================================
 // SIMT GEMM (fp32 tiny model): 64x64 output tile, 4x4 per thread.
@@ -436,6 +338,8 @@ template <typename T>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A, const T* __restrict__ W,
                                                         const int* __restrict__ m_ptr, int m_cap, int N, int K,
                                                         float* __restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float As[16][64 + 1];
   __shared__ float Ws[16][64 + 1];
   const int M = min(*m_ptr, m_cap);
@@ -479,7 +383,7 @@ template <typename T>
 void launch_gemm_simt(const T* A, const T* W, const int* m_ptr, int m_cap, int N, int K, float* out,
                       cudaStream_t st) {
   dim3 grid((N + 63) / 64, (m_cap + 63) / 64);
-  gemm_simt_kernel<T><<<grid, 256, 0, st>>>(A, W, m_ptr, m_cap, N, K, out);
+  launch_k(gemm_simt_kernel<T>, grid, dim3(256), 0, st, A, W, m_ptr, m_cap, N, K, out);
 }
 template void launch_gemm_simt<float>(const float*, const float*, const int*, int, int, int, float*, cudaStream_t);
 

@@ -15,6 +15,8 @@ namespace vlac {
 template <typename T>
 __global__ void im2col_kernel(Rows rows, const uint8_t* __restrict__ frames, int n_views, int img_h, int img_w,
                               int patch, int kpad, T* __restrict__ col) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.y, i = blockIdx.x;
   const int cnt = rows.off[b + 1] - rows.off[b];
   if (i >= cnt) return;
@@ -47,6 +49,8 @@ __global__ void embed_kernel(Rows rows, int hidden, int Nv, int P, int has_propr
                              int vocab, const int32_t* __restrict__ prompt, const float* __restrict__ proprio,
                              const T* __restrict__ tok_emb, const float* __restrict__ patch_part,
                              const T* __restrict__ proprio_w, const T* __restrict__ action_emb, int* err) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.y, i = blockIdx.x;
   const int cnt = rows.off[b + 1] - rows.off[b];
   if (i >= cnt) return;
@@ -98,6 +102,8 @@ __device__ __forceinline__ void rmsnorm_row(const float* __restrict__ x, const T
 template <typename T>
 __global__ void layer_in_kernel(Rows rows, const int* __restrict__ off_prev, int hidden, float* __restrict__ H,
                                 size_t h_seq_stride, const T* __restrict__ gain, float eps, T* __restrict__ A) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float red[32];
   const int b = blockIdx.y, i = blockIdx.x;
   const int cnt = rows.off[b + 1] - rows.off[b];
@@ -132,6 +138,8 @@ __global__ void qkv_epilogue_kernel(Rows rows, int n_heads, int head_dim, const 
                                     int splits, size_t split_stride, const float* __restrict__ rope_cos,
                                     const float* __restrict__ rope_sin, T* __restrict__ Q, T* __restrict__ Kc,
                                     T* __restrict__ Vc, size_t kv_seq_stride, int Tc) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.y, i = blockIdx.x;
   const int cnt = rows.off[b + 1] - rows.off[b];
   if (i >= cnt) return;
@@ -164,6 +172,8 @@ __global__ void qkv_epilogue_kernel(Rows rows, int n_heads, int head_dim, const 
 template <typename T>
 __global__ void residual_norm_kernel(Rows rows, int hidden, const float* __restrict__ part, int splits,
                                      size_t split_stride, const T* __restrict__ gain, float eps, T* __restrict__ A) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float red[32];
   const int b = blockIdx.y, i = blockIdx.x;
   const int cnt = rows.off[b + 1] - rows.off[b];
@@ -180,6 +190,8 @@ __global__ void residual_norm_kernel(Rows rows, int hidden, const float* __restr
 template <typename T>
 __global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part, int splits, size_t split_stride,
                               T* __restrict__ G) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.y, i = blockIdx.x;
   const int cnt = rows.off[b + 1] - rows.off[b];
   if (i >= cnt) return;
@@ -195,6 +207,8 @@ __global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part
 // x += down-projection (summed over splits).
 __global__ void residual_kernel(Rows rows, int hidden, const float* __restrict__ part, int splits,
                                 size_t split_stride) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.y, i = blockIdx.x;
   const int cnt = rows.off[b + 1] - rows.off[b];
   if (i >= cnt) return;
@@ -204,70 +218,6 @@ __global__ void residual_kernel(Rows rows, int hidden, const float* __restrict__
   for (int k = threadIdx.x; k < hidden; k += blockDim.x) x[k] = x[k] + sum_splits(pr, splits, split_stride, k);
 }
 
-// ---- action head: final norm, action-bin logits, Eq. (1) margin ------------
-
-// One block (256 threads) per action row.  Rows of sequence b are
-// X + b * x_seq_stride + (row_of_seq[b] + j) * hidden for j < rows_per_seq and
-// write action token tok0 + j.
-template <typename T>
-__global__ void __launch_bounds__(256) head_kernel(const float* __restrict__ X, const int* __restrict__ row_of_seq,
-                                                   size_t x_seq_stride, int hidden, int n_bins,
-                                                   const T* __restrict__ final_norm, const T* __restrict__ head_w,
-                                                   float eps, int D, int tok0, int32_t* __restrict__ ids,
-                                                   float* __restrict__ margins, float* __restrict__ gaps,
-                                                   float* __restrict__ logits) {
-  extern __shared__ float sm[];
-  float* h = sm;               // [hidden]
-  float* lg = sm + hidden;     // [n_bins]
-  __shared__ float red[32];
-  const int j = blockIdx.x, b = blockIdx.y;
-  const int row = row_of_seq ? row_of_seq[b] + j : j;
-  const float* x = X + (size_t)b * x_seq_stride + (size_t)row * hidden;
-  float ss = 0.f;
-  for (int k = threadIdx.x; k < hidden; k += blockDim.x) ss = fmaf(x[k], x[k], ss);
-  ss = block_sum(ss, red);
-  const float rr = 1.0f / sqrtf(ss / (float)hidden + eps);
-  for (int k = threadIdx.x; k < hidden; k += blockDim.x)
-    h[k] = to_f(from_f<T>((x[k] * rr) * to_f(final_norm[k])));
-  __syncthreads();
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  for (int c = warp; c < n_bins; c += nw) {
-    const T* w = head_w + (size_t)c * hidden;
-    float acc = 0.f;
-    for (int k = lane; k < hidden; k += 32) acc = fmaf(h[k], to_f(w[k]), acc);
-    acc = warp_sum(acc);
-    if (lane == 0) lg[c] = acc;
-  }
-  __syncthreads();
-  if (warp == 0) {
-    // argmax (lowest bin on ties), second-largest logit, sum of exp(l - l1)
-    float bv = -INFINITY;
-    int bi = 0x7fffffff;
-    for (int c = lane; c < n_bins; c += 32)
-      if (lg[c] > bv) { bv = lg[c]; bi = c; }
-    for (int o = 16; o > 0; o >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-      if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
-    }
-    float v2 = -INFINITY, z = 0.f;
-    for (int c = lane; c < n_bins; c += 32) {
-      if (c != bi) v2 = fmaxf(v2, lg[c]);
-      z += expf(lg[c] - bv);
-    }
-    v2 = warp_max(v2);
-    z = warp_sum(z);
-    if (lane == 0) {
-      const int t = tok0 + j;
-      ids[(size_t)b * D + t] = bi;
-      margins[(size_t)b * D + t] = -expm1f(v2 - bv) / z;
-      gaps[(size_t)b * D + t] = bv - v2;
-    }
-    if (logits)
-      for (int c = lane; c < n_bins; c += 32) logits[((size_t)b * D + tok0 + j) * n_bins + c] = lg[c];
-  }
-}
-
 // Autoregressive decode input: the bin fed back (argmax, or the forced replay
 // bin) selects token vocab - n_bins + bin at position P + d - 1.
 template <typename T>
@@ -275,6 +225,8 @@ __global__ void decode_embed_kernel(int d, int D, int P, int hidden, int vocab, 
                                     const T* __restrict__ tok_emb, const int32_t* __restrict__ ids,
                                     const int32_t* __restrict__ forced, const StepParams* __restrict__ prm,
                                     float* __restrict__ Xd, int* __restrict__ idx_dec, int* err) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.x;
   int bin = (prm->has_forced && forced) ? forced[(size_t)b * D + d - 1] : ids[(size_t)b * D + d - 1];
   if (bin < 0 || bin >= n_bins) {
@@ -291,6 +243,8 @@ __global__ void decode_embed_kernel(int d, int D, int P, int hidden, int vocab, 
 __global__ void finish_kernel(int B, int D, const StepParams* __restrict__ prm, const float* __restrict__ margins,
                               const float* __restrict__ gaps, float* __restrict__ m_prev, uint8_t* __restrict__ valid,
                               float* __restrict__ user_step_margin) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   const float* sig = (prm->margin_kind == VLAC_MARGIN_LOGIT ? gaps : margins) + (size_t)b * D;
@@ -308,64 +262,90 @@ __global__ void finish_kernel(int B, int D, const StepParams* __restrict__ prm, 
   user_step_margin[b] = m;
 }
 
+// ---- per-step staging -------------------------------------------------------------
+
+// Block-strided byte copies of every span (16-byte vectors when both ends are
+// aligned); block 0 also writes the step scalars.
+__global__ void copy_spans_kernel(CopyList list, StepParams p, StepParams* prm) {
+  pdl_wait();
+  pdl_trigger();
+  if (prm && blockIdx.x == 0 && threadIdx.x == 0) *prm = p;
+  for (int s = 0; s < list.n; ++s) {
+    const CopySpan c = list.span[s];
+    const uint8_t* src = static_cast<const uint8_t*>(c.src);
+    uint8_t* dst = static_cast<uint8_t*>(c.dst);
+    const size_t tid = (size_t)blockIdx.x * blockDim.x + threadIdx.x, nth = (size_t)gridDim.x * blockDim.x;
+    if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0) {
+      const size_t nv = c.bytes / 16;
+      for (size_t i = tid; i < nv; i += nth)
+        reinterpret_cast<uint4*>(dst)[i] = reinterpret_cast<const uint4*>(src)[i];
+      for (size_t i = nv * 16 + tid; i < c.bytes; i += nth) dst[i] = src[i];
+    } else {
+      for (size_t i = tid; i < c.bytes; i += nth) dst[i] = src[i];
+    }
+  }
+}
+
+void launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st) {
+  launch_k(copy_spans_kernel, dim3(64), dim3(256), 0, st, list, p, prm);
+}
+void launch_copies(const CopyList& list, cudaStream_t st) {
+  StepParams none{};
+  launch_k(copy_spans_kernel, dim3(8), dim3(256), 0, st, list, none, (StepParams*)nullptr);
+}
+
 // ---- launchers -----------------------------------------------------------------
 
 template <typename T>
 void launch_im2col(Rows rows, int B, int S, const uint8_t* frames, int n_views, int img_h, int img_w, int patch,
                    int kpad, T* col, cudaStream_t st) {
-  im2col_kernel<T><<<dim3(S, B), 128, 0, st>>>(rows, frames, n_views, img_h, img_w, patch, kpad, col);
+  launch_k(im2col_kernel<T>, dim3(S, B), dim3(128), 0, st, rows, frames, n_views, img_h, img_w, patch, kpad, col);
 }
 template <typename T>
 void launch_embed(Rows rows, int B, int S, int hidden, int Nv, int P, int has_proprio, int proprio_dim, int n_text,
                   int vocab, const int32_t* prompt, const float* proprio, const T* tok_emb, const float* patch_part,
                   const T* proprio_w, const T* action_emb, int* err, cudaStream_t st) {
-  embed_kernel<T><<<dim3(S, B), 256, 0, st>>>(rows, hidden, Nv, P, has_proprio, proprio_dim, n_text, vocab, prompt,
-                                              proprio, tok_emb, patch_part, proprio_w, action_emb, err);
+  launch_k(embed_kernel<T>, dim3(S, B), dim3(256), 0, st, rows, hidden, Nv, P, has_proprio, proprio_dim, n_text,
+           vocab, prompt, proprio, tok_emb, patch_part, proprio_w, action_emb, err);
 }
 template <typename T>
 void launch_layer_in(Rows rows, const int* off_prev, int B, int S, int hidden, float* H, size_t h_seq_stride,
                      const T* gain, float eps, T* A, cudaStream_t st) {
-  layer_in_kernel<T><<<dim3(S, B), 256, 0, st>>>(rows, off_prev, hidden, H, h_seq_stride, gain, eps, A);
+  launch_k(layer_in_kernel<T>, dim3(S, B), dim3(256), 0, st, rows, off_prev, hidden, H, h_seq_stride, gain, eps, A);
 }
 template <typename T>
 void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, int splits,
                          size_t split_stride, const float* rope_cos, const float* rope_sin, T* Q, T* Kc, T* Vc,
                          size_t kv_seq_stride, int Tc, cudaStream_t st) {
-  qkv_epilogue_kernel<T><<<dim3(S, B), 256, 0, st>>>(rows, n_heads, head_dim, part, splits, split_stride, rope_cos,
-                                                     rope_sin, Q, Kc, Vc, kv_seq_stride, Tc);
+  launch_k(qkv_epilogue_kernel<T>, dim3(S, B), dim3(256), 0, st, rows, n_heads, head_dim, part, splits, split_stride,
+           rope_cos, rope_sin, Q, Kc, Vc, kv_seq_stride, Tc);
 }
 template <typename T>
 void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part, int splits, size_t split_stride,
                           const T* gain, float eps, T* A, cudaStream_t st) {
-  residual_norm_kernel<T><<<dim3(S, B), 256, 0, st>>>(rows, hidden, part, splits, split_stride, gain, eps, A);
+  launch_k(residual_norm_kernel<T>, dim3(S, B), dim3(256), 0, st, rows, hidden, part, splits, split_stride, gain, eps,
+           A);
 }
 template <typename T>
 void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, int splits, size_t split_stride, T* G,
                    cudaStream_t st) {
-  swiglu_kernel<T><<<dim3(S, B), 256, 0, st>>>(rows, ffn, part, splits, split_stride, G);
+  launch_k(swiglu_kernel<T>, dim3(S, B), dim3(256), 0, st, rows, ffn, part, splits, split_stride, G);
 }
 void launch_residual(Rows rows, int B, int S, int hidden, const float* part, int splits, size_t split_stride,
                      cudaStream_t st) {
-  residual_kernel<<<dim3(S, B), 256, 0, st>>>(rows, hidden, part, splits, split_stride);
-}
-template <typename T>
-void launch_head(const float* X, const int* row_of_seq, size_t x_seq_stride, int rows_per_seq, int B, int hidden,
-                 int n_bins, const T* final_norm, const T* head_w, float eps, int D, int tok0, int32_t* ids,
-                 float* margins, float* gaps, float* logits, cudaStream_t st) {
-  const size_t smem = sizeof(float) * (size_t)(hidden + n_bins);
-  head_kernel<T><<<dim3(rows_per_seq, B), 256, smem, st>>>(X, row_of_seq, x_seq_stride, hidden, n_bins, final_norm,
-                                                          head_w, eps, D, tok0, ids, margins, gaps, logits);
+  launch_k(residual_kernel, dim3(S, B), dim3(256), 0, st, rows, hidden, part, splits, split_stride);
 }
 template <typename T>
 void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
                          const int32_t* ids, const int32_t* forced, const StepParams* prm, float* Xd, int* idx_dec,
                          int* err, cudaStream_t st) {
-  decode_embed_kernel<T><<<B, 256, 0, st>>>(d, D, P, hidden, vocab, n_bins, tok_emb, ids, forced, prm, Xd, idx_dec,
-                                            err);
+  launch_k(decode_embed_kernel<T>, dim3(B), dim3(256), 0, st, d, D, P, hidden, vocab, n_bins, tok_emb, ids, forced,
+           prm, Xd, idx_dec, err);
 }
 void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps, float* m_prev,
                    uint8_t* valid, float* user_step_margin, cudaStream_t st) {
-  finish_kernel<<<(B + 63) / 64, 64, 0, st>>>(B, D, prm, margins, gaps, m_prev, valid, user_step_margin);
+  launch_k(finish_kernel, dim3((B + 63) / 64), dim3(64), 0, st, B, D, prm, margins, gaps, m_prev, valid,
+           user_step_margin);
 }
 
 #define VLAC_INST(T)                                                                                              \
@@ -379,8 +359,6 @@ void launch_finish(int B, int D, const StepParams* prm, const float* margins, co
   template void launch_residual_norm<T>(Rows, int, int, int, const float*, int, size_t, const T*, float, T*,      \
                                         cudaStream_t);                                                            \
   template void launch_swiglu<T>(Rows, int, int, int, const float*, int, size_t, T*, cudaStream_t);               \
-  template void launch_head<T>(const float*, const int*, size_t, int, int, int, int, const T*, const T*, float,   \
-                               int, int, int32_t*, float*, float*, float*, cudaStream_t);                         \
   template void launch_decode_embed<T>(int, int, int, int, int, int, int, const T*, const int32_t*,               \
                                        const int32_t*, const StepParams*, float*, int*, int*, cudaStream_t);
 VLAC_INST(float)

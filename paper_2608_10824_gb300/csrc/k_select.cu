@@ -47,6 +47,8 @@ __global__ void patch_stats_kernel(const uint8_t* __restrict__ frames, const uin
                                    const uint8_t* __restrict__ valid, const StepParams* __restrict__ prm,
                                    int n_views, int img_h, int img_w, int patch, int Nv, int3* __restrict__ stats,
                                    uint8_t* __restrict__ mask, uint8_t* __restrict__ user_mask) {
+  pdl_wait();
+  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int v = blockIdx.x * (blockDim.x >> 5) + warp;
   const int b = blockIdx.y;
@@ -87,6 +89,8 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
                               int* __restrict__ idx, int* __restrict__ M, int* __restrict__ emit_slot,
                               uint8_t* __restrict__ user_recomputed, uint8_t* __restrict__ user_gate_auto,
                               int* __restrict__ user_idx, int* __restrict__ user_M) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ uint8_t smem[];
   int3* s_st = reinterpret_cast<int3*>(smem);
   int* s_rank = reinterpret_cast<int*>(s_st + Nv);
@@ -161,6 +165,8 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
 
 // Row offsets of every layer: off[l][b] = sum of M[b'][l] over b' < b.
 __global__ void plan_kernel(const int* __restrict__ M, int B, int L, int* __restrict__ off) {
+  pdl_wait();
+  pdl_trigger();
   for (int l = threadIdx.x; l < L; l += blockDim.x) {
     int acc = 0;
     off[(size_t)l * (B + 1)] = 0;
@@ -176,8 +182,8 @@ void launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_
                         uint8_t* user_mask, cudaStream_t st) {
   const int Nv = n_views * (img_h / patch) * (img_w / patch);
   dim3 grid((Nv + 7) / 8, B);
-  patch_stats_kernel<<<grid, 256, 0, st>>>(frames, prev, valid, prm, n_views, img_h, img_w, patch, Nv, stats,
-                                           mask, user_mask);
+  launch_k(patch_stats_kernel, grid, dim3(256), 0, st, frames, prev, valid, prm, n_views, img_h, img_w, patch, Nv,
+           stats, mask, user_mask);
 }
 
 void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
@@ -186,10 +192,9 @@ void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid,
                    uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
                    cudaStream_t st) {
   const size_t smem = (size_t)Nv * (sizeof(int3) + sizeof(int) + 1) + 16;
-  select_kernel<<<B, 512, smem, st>>>(stats, mask, valid, m_prev, prm, override_, Nv, S, L, P, parallel,
-                                      n_action, full, idx, M, emit_slot, user_recomputed, user_gate_auto,
-                                      user_idx, user_M);
-  plan_kernel<<<1, 256, 0, st>>>(M, B, L, off);
+  launch_k(select_kernel, dim3(B), dim3(512), smem, st, stats, mask, valid, m_prev, prm, override_, Nv, S, L, P,
+           parallel, n_action, full, idx, M, emit_slot, user_recomputed, user_gate_auto, user_idx, user_M);
+  launch_k(plan_kernel, dim3(1), dim3(256), 0, st, M, B, L, off);
 }
 
 }  // namespace vlac

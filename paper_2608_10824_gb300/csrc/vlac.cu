@@ -11,6 +11,10 @@
 
 using namespace vlac;
 
+namespace vlac {
+bool g_pdl = true;
+}
+
 namespace {
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -58,6 +62,18 @@ struct vlac_ctx {
   uint8_t *mask, *full;
   int *idx, *M, *off, *emit_slot, *off_dec, *idx_dec, *err;
   float *logits_ws, *attn_part;
+  // staged per-step inputs and outputs (fixed addresses, so a step can be a graph)
+  uint8_t* in_frames;
+  int32_t* in_prompt;
+  float* in_proprio;
+  int8_t* in_override;
+  int32_t* in_forced;
+  int32_t* o_ids;
+  float *o_margins, *o_gaps, *o_step_margin, *o_logits;
+  uint8_t *o_recomputed, *o_gate_auto, *o_mask;
+  int32_t *o_idx, *o_M;
+  cudaStream_t cap_stream = nullptr;
+  bool use_graph = true;
   int* err_host = nullptr;  // pinned
   uint64_t launches = 0;
   uint32_t wait_limit = kDefaultWaitLimit;
@@ -75,6 +91,10 @@ struct vlac_ctx {
 struct vlac_cache {
   vlac_ctx* ctx;
   int B;
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t gexec = nullptr;
+  int eager_steps = 0;
+  uint64_t graph_launches = 0;
   void *K, *V;
   float* H;
   uint8_t *prev, *valid;
@@ -148,6 +168,7 @@ extern "C" int vlac_destroy(vlac_ctx* c) {
     cudaEventDestroy(r.b);
   }
   for (auto e : c->ev_pool) cudaEventDestroy(e);
+  if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
   if (c->wmem) cudaFree(c->wmem);
   if (c->wsmem) cudaFree(c->wsmem);
   if (c->err_host) cudaFreeHost(c->err_host);
@@ -170,6 +191,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
 
   vlac_ctx* c = new (std::nothrow) vlac_ctx();
   if (!c) return VLAC_ERR_OOM;
+  if (const char* e = std::getenv("VLAC_PDL")) g_pdl = std::atoi(e) != 0;
+  if (const char* e = std::getenv("VLAC_GRAPH")) c->use_graph = std::atoi(e) != 0;
   c->d = *dims;
   const vlac_dims& d = c->d;
   c->bf16 = d.dtype == VLAC_BF16;
@@ -289,6 +312,22 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->err, 4, base);
     sc.take(c->logits_ws, Bm * (d.parallel ? d.n_action : 1) * d.n_bins * 4, base);
     sc.take(c->attn_part, Bm * d.n_heads * ((c->Tc + 31) / 32) * (d.head_dim + 2) * 4, base);
+    const size_t fbytes = (size_t)d.n_views * d.img_h * d.img_w * 3;
+    sc.take(c->in_frames, Bm * fbytes, base);
+    sc.take(c->in_prompt, Bm * d.n_text * 4, base);
+    sc.take(c->in_proprio, Bm * std::max(d.proprio_dim, 1) * 4, base);
+    sc.take(c->in_override, Bm, base);
+    sc.take(c->in_forced, Bm * d.n_action * 4, base);
+    sc.take(c->o_ids, Bm * d.n_action * 4, base);
+    sc.take(c->o_margins, Bm * d.n_action * 4, base);
+    sc.take(c->o_gaps, Bm * d.n_action * 4, base);
+    sc.take(c->o_step_margin, Bm * 4, base);
+    sc.take(c->o_logits, Bm * d.n_action * d.n_bins * 4, base);
+    sc.take(c->o_recomputed, Bm, base);
+    sc.take(c->o_gate_auto, Bm, base);
+    sc.take(c->o_mask, Bm * c->Nv, base);
+    sc.take(c->o_idx, Bm * c->S * 4, base);
+    sc.take(c->o_M, Bm * L * 4, base);
   };
   plan_s(nullptr);
   if (cudaMalloc(&c->wsmem, sc.off) != cudaSuccess) {
@@ -309,6 +348,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     return fail(VLAC_ERR_OOM);
   }
   *c->err_host = 0;
+  if (cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess) return fail(VLAC_ERR_CUDA);
 
   // ---- TMA descriptors ----
   if (c->bf16) {
@@ -379,6 +419,8 @@ extern "C" int vlac_cache_init(vlac_ctx* c, void* mem, size_t bytes, int batch, 
 
 extern "C" int vlac_cache_destroy(vlac_cache* k) {
   if (!k) return VLAC_ERR_INVALID_ARG;
+  if (k->gexec) cudaGraphExecDestroy(k->gexec);
+  if (k->graph) cudaGraphDestroy(k->graph);
   delete k;
   return VLAC_OK;
 }
@@ -447,9 +489,16 @@ void gemm(vlac_ctx* c, const CUtensorMap* tmA, const CUtensorMap* tmW, const T* 
   c->launches += 1;
 }
 
+// The step body: reads only the staged inputs and writes only the context's
+// output buffers, so its launches can be captured once and replayed.
 template <typename T>
-int step_impl(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, const int32_t* prompt, const float* proprio,
-              const vlac_step_opts* opts, const vlac_step_out* out, cudaStream_t st) {
+int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
+  vlac_step_out outv{c->o_ids, c->o_margins, c->o_gaps, c->o_recomputed, c->o_step_margin, c->o_gate_auto,
+                     c->o_logits, c->o_mask, c->o_idx, c->o_M};
+  const vlac_step_out* out = &outv;
+  const uint8_t* frames = c->in_frames;
+  const int32_t* prompt = c->in_prompt;
+  const float* proprio = c->in_proprio;
   const vlac_dims& d = c->d;
   const int B = k->B, S = c->S, L = d.n_layers, Hd = d.hidden, F = d.ffn, D = d.n_action, nb = d.n_bins;
   const int nh = d.n_heads, hd = d.head_dim;
@@ -462,8 +511,8 @@ int step_impl(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, const int32_t* 
   T* Kc = static_cast<T*>(k->K);
   T* Vc = static_cast<T*>(k->V);
   const size_t kv_layer = (size_t)nh * c->Tc * hd;
-  const int8_t* ovr = opts ? opts->gate_override : nullptr;
-  const int32_t* forced = opts ? opts->forced_ids : nullptr;
+  const int8_t* ovr = c->in_override;
+  const int32_t* forced = c->in_forced;
   auto W = [](void* p) { return static_cast<const T*>(p); };
 
   // Stage 1 and the gate + Stage-3 plan
@@ -582,6 +631,41 @@ int step_impl(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, const int32_t* 
   return VLAC_OK;
 }
 
+int run_body(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
+  return c->bf16 ? step_impl<bf16>(c, k, st) : step_impl<float>(c, k, st);
+}
+
+// First step of a cache runs eagerly (lazy per-kernel set-up happens there);
+// the second captures the body into a graph, which every later step replays.
+int run_step(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
+  if (!c->use_graph || c->prof_on) return run_body(c, k, st);
+  if (!k->gexec) {
+    if (k->eager_steps++ == 0) return run_body(c, k, st);
+    const uint64_t n0 = c->launches;
+    CK(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal));
+    const int rc = run_body(c, k, c->cap_stream);
+    cudaGraph_t g = nullptr;
+    const cudaError_t e = cudaStreamEndCapture(c->cap_stream, &g);
+    if (rc != VLAC_OK || e != cudaSuccess) {
+      if (g) cudaGraphDestroy(g);
+      (void)cudaGetLastError();
+      return rc != VLAC_OK ? rc : VLAC_ERR_CUDA;
+    }
+    if (cudaGraphInstantiate(&k->gexec, g, 0) != cudaSuccess) {
+      cudaGraphDestroy(g);
+      k->gexec = nullptr;
+      (void)cudaGetLastError();
+      return VLAC_ERR_CUDA;
+    }
+    k->graph = g;
+    k->graph_launches = c->launches - n0;
+    c->launches = n0;
+  }
+  CK(cudaGraphLaunch(k->gexec, st));
+  c->launches += k->graph_launches;
+  return VLAC_OK;
+}
+
 }  // namespace
 
 extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, const int32_t* prompt_ids,
@@ -620,9 +704,37 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
     return e;
   }
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  CK(cudaMemcpyAsync(c->prm, &p, sizeof(p), cudaMemcpyHostToDevice, st));
-  return c->bf16 ? step_impl<bf16>(c, k, frames, prompt_ids, proprio, opts, out, st)
-                 : step_impl<float>(c, k, frames, prompt_ids, proprio, opts, out, st);
+  const vlac_dims& d = c->d;
+  const int B = k->B, D = d.n_action;
+  const size_t fb = (size_t)d.n_views * d.img_h * d.img_w * 3;
+  CopyList in{};
+  auto add = [](CopyList& l, const void* src, void* dst, size_t bytes) {
+    if (src && dst && bytes) l.span[l.n++] = CopySpan{src, dst, bytes};
+  };
+  add(in, frames, c->in_frames, (size_t)B * fb);
+  add(in, prompt_ids, c->in_prompt, (size_t)B * d.n_text * 4);
+  if (d.proprio_dim) add(in, proprio, c->in_proprio, (size_t)B * d.proprio_dim * 4);
+  if (p.has_override) add(in, opts->gate_override, c->in_override, (size_t)B);
+  if (p.has_forced) add(in, opts->forced_ids, c->in_forced, (size_t)B * D * 4);
+  launch_stage(p, c->prm, in, st);
+  c->launches += 1;
+  int rc = run_step(c, k, st);
+  if (rc) return rc;
+  CopyList o{};
+  add(o, c->o_ids, out->action_ids, (size_t)B * D * 4);
+  add(o, c->o_margins, out->margins, (size_t)B * D * 4);
+  add(o, c->o_gaps, out->logit_gap, (size_t)B * D * 4);
+  add(o, c->o_recomputed, out->recomputed, (size_t)B);
+  add(o, c->o_step_margin, out->step_margin, (size_t)B * 4);
+  add(o, c->o_gate_auto, out->gate_auto, (size_t)B);
+  add(o, c->o_logits, out->logits, (size_t)B * D * d.n_bins * 4);
+  add(o, c->o_mask, out->static_mask, (size_t)B * c->Nv);
+  add(o, c->o_idx, out->idx, (size_t)B * c->S * 4);
+  add(o, c->o_M, out->M, (size_t)B * d.n_layers * 4);
+  launch_copies(o, st);
+  c->launches += 1;
+  CK(cudaGetLastError());
+  return VLAC_OK;
 }
 
 extern "C" int vlac_sync_error(vlac_ctx* c) {
