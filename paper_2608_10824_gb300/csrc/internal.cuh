@@ -60,7 +60,11 @@ struct DGemv {
   const float* rope_sin;
   void* G;            // SwiGLU epilogue: G[b][j]
   int ffn;
+  const float* ssq_in;  // normalising GEMV: per-producer-CTA sums of squares [nb][n_ssq]
+  int n_ssq;
+  float* ssq_out;       // residual GEMV: this launch's per-CTA sums of squares [nb][grid]
 };
+constexpr int kDecodeRowsPerCta = 4;  // residual rows per decode-GEMV CTA (2 row pairs)
 
 // ---- scalar helpers --------------------------------------------------------
 template <typename T> __device__ __forceinline__ float to_f(T v);
@@ -177,7 +181,7 @@ void launch_attention(Rows rows, int B, int S, int n_heads, int head_dim, const 
 template <typename T>
 void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
                          const int32_t* ids, const int32_t* forced, const StepParams* prm, float* Xd,
-                         int* idx_dec, int* err, cudaStream_t st);
+                         int* idx_dec, float* ssq_out, int* err, cudaStream_t st);
 void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps,
                    float* m_prev, uint8_t* valid, float* user_step_margin, cudaStream_t st);
 

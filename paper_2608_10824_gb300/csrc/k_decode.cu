@@ -88,137 +88,185 @@ __device__ __forceinline__ void norm_rows_to_smem(const float* __restrict__ X, c
 }  // namespace
 
 // ---- fused decode GEMV ----------------------------------------------------------
+//
+// A CTA owns RP row pairs (2*RP weight rows) over the full K; its 8 warps split
+// K into 8 contiguous segments and the per-warp partial dot products are
+// summed in warp order.  Small CTAs keep the last wave short.
+//
+// RMSNorm without a second pass: every residual-writing GEMV (and the decode
+// embedding) stores, per CTA and sequence, the sum of squares of the residual
+// elements it produced; a normalising GEMV sums those partials in index order
+// to get the row's mean square, then normalises its own K segment on the fly
+// (x * r * g rounded to T, as the GEMM input).
 
-template <typename T, int NB, int EPI, bool NORM, int UNROLL>
-__global__ void __launch_bounds__(256) dgemv_kernel(DGemv a) {
+constexpr int kDW = 8;  // warps per decode-GEMV CTA
+
+template <typename T, int NB, int EPI, bool NORM, int RP, int UNROLL>
+__global__ void __launch_bounds__(kDW * 32) dgemv_kernel(DGemv a) {
   constexpr int V = Vec<T>::n;
-  extern __shared__ __align__(16) uint8_t dsm[];
-  T* xs = reinterpret_cast<T*>(dsm);
+  constexpr int NR = 2 * RP;
+  __shared__ float red[kDW][NR][NB];
+  __shared__ float rr[NB];
+  __shared__ float xnew[NR][NB];
   const int K = a.K;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int p = blockIdx.x * (blockDim.x >> 5) + warp;
-  int r1 = 0, r2 = 0;
-  int sec = 0, h = 0, e = 0;
   const int hd = a.head_dim, half = hd >> 1;
-  if constexpr (EPI == kEpiQkvRope) {
-    const int hidden = a.n_heads * hd;
-    sec = p / (hidden / 2);
-    const int within = p - sec * (hidden / 2);
-    h = within / half;
-    e = within - h * half;
-    r1 = sec * hidden + h * hd + e;
-    r2 = r1 + half;
-  } else if constexpr (EPI == kEpiSwiglu) {
-    r1 = p;
-    r2 = a.ffn + p;
-  } else {
-    r1 = 2 * p;
-    r2 = 2 * p + 1;
+  // weight rows of this CTA: pair q -> rows (row[2q], row[2q+1])
+  int row[NR];
+#pragma unroll
+  for (int q = 0; q < RP; ++q) {
+    const int p = blockIdx.x * RP + q;
+    if constexpr (EPI == kEpiQkvRope) {
+      const int hidden = a.n_heads * hd;
+      const int sec = p / (hidden / 2), within = p - sec * (hidden / 2);
+      const int h = within / half, e = within - h * half;
+      row[2 * q] = sec * hidden + h * hd + e;
+      row[2 * q + 1] = row[2 * q] + half;
+    } else if constexpr (EPI == kEpiSwiglu) {
+      row[2 * q] = p;
+      row[2 * q + 1] = a.ffn + p;
+    } else {
+      row[2 * q] = 2 * p;
+      row[2 * q + 1] = 2 * p + 1;
+    }
   }
-  // the weight rows do not depend on earlier kernels: start pulling them into
-  // L2 while the previous kernel of the stream drains
-  if (p < a.n_pairs && lane == 0) {
-    prefetch_l2(static_cast<const T*>(a.W) + (size_t)r1 * K, (uint32_t)(K * sizeof(T)));
-    prefetch_l2(static_cast<const T*>(a.W) + (size_t)r2 * K, (uint32_t)(K * sizeof(T)));
-  }
+  const T* W = static_cast<const T*>(a.W);
+  // weights are constant: pull this CTA's rows into L2 before the dependency wait
+  if (warp < NR && lane == 0) prefetch_l2(W + (size_t)row[warp] * K, (uint32_t)(K * sizeof(T)));
   pdl_wait();
   pdl_trigger();
-  if constexpr (NORM) norm_rows_to_smem<T, NB>(a.X, static_cast<const T*>(a.gain), K, a.eps, xs);
-  if (p >= a.n_pairs) return;
-  const T* W = static_cast<const T*>(a.W);
   const int kv = K / V;
-  const uint4* w1 = reinterpret_cast<const uint4*>(W + (size_t)r1 * K);
-  const uint4* w2 = reinterpret_cast<const uint4*>(W + (size_t)r2 * K);
-  const uint4* xv = reinterpret_cast<const uint4*>(NORM ? (const T*)xs : static_cast<const T*>(a.xin));
-  float acc1[NB], acc2[NB];
+  const int seg = (kv + kDW - 1) / kDW;
+  const int k_beg = warp * seg, k_end = min(kv, k_beg + seg);
+  float acc[NR][NB];
 #pragma unroll
-  for (int b = 0; b < NB; ++b) acc1[b] = acc2[b] = 0.f;
-  for (int k0 = lane; k0 < kv; k0 += 32 * UNROLL) {
-    uint4 q1[UNROLL], q2[UNROLL];
+  for (int r = 0; r < NR; ++r)
+#pragma unroll
+    for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
+  if constexpr (NORM) {
+    // mean square of each residual row from the producers' partials (index order)
+    float s[NB];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) s[b] = 0.f;
+    for (int c = threadIdx.x; c < a.n_ssq; c += blockDim.x)
+#pragma unroll
+      for (int b = 0; b < NB; ++b) s[b] += a.ssq_in[(size_t)b * a.n_ssq + c];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      const float t = warp_allsum(s[b]);
+      if (lane == 0) red[warp][0][b] = t;
+    }
+    __syncthreads();
+    if (threadIdx.x < NB) {
+      float t = 0.f;
+      for (int w = 0; w < kDW; ++w) t += red[w][0][threadIdx.x];
+      rr[threadIdx.x] = 1.0f / sqrtf(t / (float)K + a.eps);
+    }
+    __syncthreads();
+  }
+  const uint4* xv = reinterpret_cast<const uint4*>(static_cast<const T*>(a.xin));
+  const T* gain = static_cast<const T*>(a.gain);
+  for (int k0 = k_beg + lane; k0 < k_end; k0 += 32 * UNROLL) {
+    uint4 wq[UNROLL][NR];
 #pragma unroll
     for (int u = 0; u < UNROLL; ++u) {
       const int k = k0 + u * 32;
-      if (k < kv) {
-        q1[u] = ld_stream(w1 + k);
-        q2[u] = ld_stream(w2 + k);
-      }
+#pragma unroll
+      for (int r = 0; r < NR; ++r)
+        if (k < k_end) wq[u][r] = ld_stream(reinterpret_cast<const uint4*>(W + (size_t)row[r] * K) + k);
     }
 #pragma unroll
     for (int u = 0; u < UNROLL; ++u) {
       const int k = k0 + u * 32;
-      if (k >= kv) break;
-      float f1[V], f2[V];
-      unpack<T>(q1[u], f1);
-      unpack<T>(q2[u], f2);
+      if (k >= k_end) break;
+      float xf[NB][V];
+      if constexpr (NORM) {
+        float g[V];
+        unpack<T>(__ldg(reinterpret_cast<const uint4*>(gain) + k), g);
 #pragma unroll
-      for (int b = 0; b < NB; ++b) {
-        float xf[V];
-        uint4 xu;
-        if constexpr (NORM) xu = xv[(size_t)b * kv + k];
-        else xu = __ldg(xv + (size_t)b * kv + k);
-        unpack<T>(xu, xf);
+        for (int b = 0; b < NB; ++b) {
+          const float4* x4 = reinterpret_cast<const float4*>(a.X + (size_t)b * K + (size_t)k * V);
 #pragma unroll
-        for (int i = 0; i < V; ++i) {
-          acc1[b] = fmaf(f1[i], xf[i], acc1[b]);
-          acc2[b] = fmaf(f2[i], xf[i], acc2[b]);
+          for (int i = 0; i < V / 4; ++i) {
+            const float4 v4 = x4[i];
+            xf[b][4 * i + 0] = to_f(from_f<T>((v4.x * rr[b]) * g[4 * i + 0]));
+            xf[b][4 * i + 1] = to_f(from_f<T>((v4.y * rr[b]) * g[4 * i + 1]));
+            xf[b][4 * i + 2] = to_f(from_f<T>((v4.z * rr[b]) * g[4 * i + 2]));
+            xf[b][4 * i + 3] = to_f(from_f<T>((v4.w * rr[b]) * g[4 * i + 3]));
+          }
         }
+      } else {
+#pragma unroll
+        for (int b = 0; b < NB; ++b) unpack<T>(__ldg(xv + (size_t)b * kv + k), xf[b]);
+      }
+#pragma unroll
+      for (int r = 0; r < NR; ++r) {
+        float wf[V];
+        unpack<T>(wq[u][r], wf);
+#pragma unroll
+        for (int b = 0; b < NB; ++b)
+#pragma unroll
+          for (int i = 0; i < V; ++i) acc[r][b] = fmaf(wf[i], xf[b][i], acc[r][b]);
       }
     }
   }
 #pragma unroll
-  for (int b = 0; b < NB; ++b) {
-    acc1[b] = warp_allsum(acc1[b]);
-    acc2[b] = warp_allsum(acc2[b]);
-  }
-  if (lane >= NB) return;
-  // lane b writes sequence b
-  float y1 = acc1[0], y2 = acc2[0];
+  for (int r = 0; r < NR; ++r)
 #pragma unroll
-  for (int b = 1; b < NB; ++b)
-    if (lane == b) {
-      y1 = acc1[b];
-      y2 = acc2[b];
+    for (int b = 0; b < NB; ++b) {
+      const float t = warp_allsum(acc[r][b]);
+      if (lane == 0) red[warp][r][b] = t;
     }
-  const int b = lane;
-  if constexpr (EPI == kEpiQkvRope) {
-    const int hidden = a.n_heads * hd;
-    float o1 = y1, o2 = y2;
-    if (sec < 2) {
-      const float c = a.rope_cos[(size_t)a.pos * half + e], s = a.rope_sin[(size_t)a.pos * half + e];
-      o1 = y1 * c - y2 * s;
-      o2 = y2 * c + y1 * s;
+  __syncthreads();
+  if (threadIdx.x < RP * NB) {
+    const int q = threadIdx.x / NB, b = threadIdx.x - q * NB;
+    float y1 = 0.f, y2 = 0.f;
+    for (int w = 0; w < kDW; ++w) {
+      y1 += red[w][2 * q][b];
+      y2 += red[w][2 * q + 1][b];
     }
-    if (sec == 0) {
-      T* q = static_cast<T*>(a.Q) + (size_t)b * hidden + (size_t)h * hd;
-      q[e] = from_f<T>(o1);
-      q[e + half] = from_f<T>(o2);
+    const int p = blockIdx.x * RP + q;
+    if constexpr (EPI == kEpiQkvRope) {
+      const int hidden = a.n_heads * hd;
+      const int sec = p / (hidden / 2), within = p - sec * (hidden / 2);
+      const int h = within / half, e = within - h * half;
+      float o1 = y1, o2 = y2;
+      if (sec < 2) {
+        const float c = a.rope_cos[(size_t)a.pos * half + e], sn = a.rope_sin[(size_t)a.pos * half + e];
+        o1 = y1 * c - y2 * sn;
+        o2 = y2 * c + y1 * sn;
+      }
+      T* dst = sec == 0 ? static_cast<T*>(a.Q) + (size_t)b * hidden + (size_t)h * hd
+                        : static_cast<T*>(sec == 1 ? a.Kc : a.Vc) + (size_t)b * a.kv_seq_stride +
+                              ((size_t)h * a.Tc + a.pos) * hd;
+      dst[e] = from_f<T>(o1);
+      dst[e + half] = from_f<T>(o2);
+    } else if constexpr (EPI == kEpiSwiglu) {
+      static_cast<T*>(a.G)[(size_t)b * a.ffn + p] = from_f<T>((y1 / (1.0f + expf(-y1))) * y2);
     } else {
-      T* c = static_cast<T*>(sec == 1 ? a.Kc : a.Vc) + (size_t)b * a.kv_seq_stride +
-             ((size_t)h * a.Tc + a.pos) * hd;
-      c[e] = from_f<T>(o1);
-      c[e + half] = from_f<T>(o2);
+      float* x = a.Xres + (size_t)b * a.n_out;
+      const float n1 = x[row[2 * q]] + y1, n2 = x[row[2 * q + 1]] + y2;
+      x[row[2 * q]] = n1;
+      x[row[2 * q + 1]] = n2;
+      xnew[2 * q][b] = n1;
+      xnew[2 * q + 1][b] = n2;
     }
-  } else if constexpr (EPI == kEpiSwiglu) {
-    static_cast<T*>(a.G)[(size_t)b * a.ffn + p] = from_f<T>((y1 / (1.0f + expf(-y1))) * y2);
-  } else {
-    float* x = a.Xres + (size_t)b * a.n_out;
-    x[r1] += y1;
-    x[r2] += y2;
+  }
+  if constexpr (EPI == kEpiResid) {
+    __syncthreads();
+    if (threadIdx.x < NB) {
+      float t = 0.f;
+      for (int r = 0; r < NR; ++r) t = fmaf(xnew[r][threadIdx.x], xnew[r][threadIdx.x], t);
+      a.ssq_out[(size_t)threadIdx.x * gridDim.x + blockIdx.x] = t;
+    }
   }
 }
 
 template <typename T, int NB, int EPI, bool NORM>
 static void dgemv_nb(const DGemv& a, cudaStream_t st) {
-  const int warps = 8;
-  const int blocks = (a.n_pairs + warps - 1) / warps;
-  const size_t smem = NORM ? (size_t)NB * a.K * sizeof(T) : 0;
-  constexpr int U = NB <= 2 ? 4 : 2;
-  static size_t smem_set = 48 * 1024;  // raised once per instantiation, before any graph capture of it
-  if (smem > smem_set) {
-    cudaFuncSetAttribute(dgemv_kernel<T, NB, EPI, NORM, U>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    smem_set = smem;
-  }
-  launch_k(dgemv_kernel<T, NB, EPI, NORM, U>, dim3(blocks), dim3(warps * 32), smem, st, a);
+  constexpr int RP = 2;
+  constexpr int U = NB <= 2 ? 2 : 1;
+  launch_k(dgemv_kernel<T, NB, EPI, NORM, RP, U>, dim3(a.n_pairs / RP), dim3(kDW * 32), 0, st, a);
 }
 
 template <typename T, int EPI, bool NORM>
@@ -247,89 +295,95 @@ template void launch_dgemv<float>(const DGemv&, int, int, cudaStream_t);
 template void launch_dgemv<bf16>(const DGemv&, int, int, cudaStream_t);
 
 // ---- decode attention: one query per (sequence, head) ----------------------------
-
-// Partial softmax of one 32-key chunk: m = max score, l = sum exp(s - m),
-// acc = sum exp(s - m) * v.  Lane holds elements [lane*EPL, lane*EPL + EPL).
+//
+// One CTA per (head, sequence).  Each warp takes 32-key tiles (lane = key for
+// the scores, lane = output elements for P.V) with a running softmax; the
+// warps' partial results are combined in warp order.
 template <typename T, int HD>
-__global__ void __launch_bounds__(32) dec_attn_partial_kernel(const T* __restrict__ Q, const T* __restrict__ Kc,
-                                                              const T* __restrict__ Vc, size_t kv_seq_stride, int Tc,
-                                                              int pos, int n_heads, float scale,
-                                                              float* __restrict__ part, int nchunk) {
+__global__ void __launch_bounds__(256) dec_attn_kernel(const T* __restrict__ Q, const T* __restrict__ Kc,
+                                                       const T* __restrict__ Vc, size_t kv_seq_stride, int Tc, int pos,
+                                                       int n_heads, float scale, T* __restrict__ O) {
+  constexpr int EPL = HD / 32, NW = 8, V = Vec<T>::n;
+  __shared__ float qs[HD];
+  __shared__ float wm[NW], wl[NW];
+  __shared__ float wacc[NW][HD];
   pdl_wait();
   pdl_trigger();
-  constexpr int EPL = HD / 32;
-  const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z, lane = threadIdx.x;
+  const int h = blockIdx.x, b = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int hidden = n_heads * HD;
-  float q[EPL];
-#pragma unroll
-  for (int i = 0; i < EPL; ++i) q[i] = to_f(Q[(size_t)b * hidden + (size_t)h * HD + lane * EPL + i]);
+  for (int e = threadIdx.x; e < HD; e += blockDim.x) qs[e] = to_f(Q[(size_t)b * hidden + (size_t)h * HD + e]);
+  __syncthreads();
   const T* Kh = Kc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
   const T* Vh = Vc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
-  const int j0 = c * 32, j1 = min(j0 + 32, pos + 1);
-  float s_mine = -INFINITY;  // lane j keeps the score of key j0 + j
-  for (int j = j0; j < j1; ++j) {
-    float d = 0.f;
+  const int nkeys = min(pos + 1, Tc);
+  float m = -INFINITY, l = 0.f, acc[EPL];
 #pragma unroll
-    for (int i = 0; i < EPL; ++i) d = fmaf(q[i], to_f(Kh[(size_t)j * HD + lane * EPL + i]), d);
-    d = warp_allsum(d) * scale;
-    if (lane == j - j0) s_mine = d;
+  for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
+  for (int j0 = warp * 32; j0 < nkeys; j0 += NW * 32) {
+    const int j = j0 + lane;
+    float sc = -INFINITY;
+    if (j < nkeys) {
+      const uint4* kr = reinterpret_cast<const uint4*>(Kh + (size_t)j * HD);
+      float d = 0.f;
+#pragma unroll
+      for (int v = 0; v < HD / V; ++v) {
+        float f[V];
+        unpack<T>(kr[v], f);
+#pragma unroll
+        for (int i = 0; i < V; ++i) d = fmaf(f[i], qs[v * V + i], d);
+      }
+      sc = d * scale;
+    }
+    float mt = sc;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
+    const float mn = fmaxf(m, mt);
+    const float p = (sc == -INFINITY) ? 0.f : expf(sc - mn);
+    const float corr = (m == -INFINITY) ? 0.f : expf(m - mn);
+    l = l * corr + warp_allsum(p);
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) acc[e] *= corr;
+    const int jn = min(32, nkeys - j0);
+#pragma unroll 4
+    for (int jj = 0; jj < jn; ++jj) {
+      const float pj = __shfl_sync(0xffffffffu, p, jj);
+      const T* vr = Vh + (size_t)(j0 + jj) * HD + lane * EPL;
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) acc[e] = fmaf(pj, to_f(vr[e]), acc[e]);
+    }
+    m = mn;
   }
-  float m = s_mine;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-  const float pj = (s_mine == -INFINITY) ? 0.f : expf(s_mine - m);
-  const float l = warp_allsum(pj);
-  float acc[EPL];
-#pragma unroll
-  for (int i = 0; i < EPL; ++i) acc[i] = 0.f;
-  for (int j = j0; j < j1; ++j) {
-    const float p = __shfl_sync(0xffffffffu, pj, j - j0);
-#pragma unroll
-    for (int i = 0; i < EPL; ++i) acc[i] = fmaf(p, to_f(Vh[(size_t)j * HD + lane * EPL + i]), acc[i]);
-  }
-  float* o = part + (((size_t)b * n_heads + h) * nchunk + c) * (HD + 2);
-#pragma unroll
-  for (int i = 0; i < EPL; ++i) o[lane * EPL + i] = acc[i];
   if (lane == 0) {
-    o[HD] = m;
-    o[HD + 1] = l;
+    wm[warp] = m;
+    wl[warp] = l;
   }
-}
-
-// Combines the chunks of one (sequence, head) in chunk order.
-template <typename T, int HD>
-__global__ void __launch_bounds__(HD) dec_attn_combine_kernel(const float* __restrict__ part, int nchunk,
-                                                              int n_heads, T* __restrict__ O) {
-  pdl_wait();
-  pdl_trigger();
-  const int h = blockIdx.x, b = blockIdx.y, e = threadIdx.x;
-  const float* base = part + ((size_t)b * n_heads + h) * nchunk * (HD + 2);
-  float M = -INFINITY;
-  for (int c = 0; c < nchunk; ++c) M = fmaxf(M, base[(size_t)c * (HD + 2) + HD]);
-  float L = 0.f, acc = 0.f;
-  for (int c = 0; c < nchunk; ++c) {
-    const float* pc = base + (size_t)c * (HD + 2);
-    const float f = expf(pc[HD] - M);
-    L = fmaf(pc[HD + 1], f, L);
-    acc = fmaf(pc[e], f, acc);
+#pragma unroll
+  for (int e = 0; e < EPL; ++e) wacc[warp][lane * EPL + e] = acc[e];
+  __syncthreads();
+  for (int e = threadIdx.x; e < HD; e += blockDim.x) {
+    float M = -INFINITY;
+    for (int w = 0; w < NW; ++w) M = fmaxf(M, wm[w]);
+    float L = 0.f, o = 0.f;
+    for (int w = 0; w < NW; ++w) {
+      const float f = expf(wm[w] - M);
+      L = fmaf(wl[w], f, L);
+      o = fmaf(wacc[w][e], f, o);
+    }
+    O[(size_t)b * hidden + (size_t)h * HD + e] = from_f<T>(o / L);
   }
-  O[(size_t)b * n_heads * HD + (size_t)h * HD + e] = from_f<T>(acc / L);
 }
 
 template <typename T>
 void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride,
                           int Tc, int pos, float* part, T* O, cudaStream_t st) {
-  const int nchunk = (pos + 1 + 31) / 32;
+  (void)part;
   const float scale = 1.0f / sqrtf((float)head_dim);
-  if (head_dim == 128) {
-    launch_k(dec_attn_partial_kernel<T, 128>, dim3(nchunk, n_heads, B), dim3(32), 0, st, Q, Kc, Vc, kv_seq_stride,
-             Tc, pos, n_heads, scale, part, nchunk);
-    launch_k(dec_attn_combine_kernel<T, 128>, dim3(n_heads, B), dim3(128), 0, st, part, nchunk, n_heads, O);
-  } else {
-    launch_k(dec_attn_partial_kernel<T, 64>, dim3(nchunk, n_heads, B), dim3(32), 0, st, Q, Kc, Vc, kv_seq_stride,
-             Tc, pos, n_heads, scale, part, nchunk);
-    launch_k(dec_attn_combine_kernel<T, 64>, dim3(n_heads, B), dim3(64), 0, st, part, nchunk, n_heads, O);
-  }
+  if (head_dim == 128)
+    launch_k(dec_attn_kernel<T, 128>, dim3(n_heads, B), dim3(256), 0, st, Q, Kc, Vc, kv_seq_stride, Tc, pos, n_heads,
+             scale, O);
+  else
+    launch_k(dec_attn_kernel<T, 64>, dim3(n_heads, B), dim3(256), 0, st, Q, Kc, Vc, kv_seq_stride, Tc, pos, n_heads,
+             scale, O);
 }
 template void launch_dec_attention<float>(int, int, int, const float*, const float*, const float*, size_t, int, int,
                                           float*, float*, cudaStream_t);

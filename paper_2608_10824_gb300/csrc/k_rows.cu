@@ -224,7 +224,8 @@ template <typename T>
 __global__ void decode_embed_kernel(int d, int D, int P, int hidden, int vocab, int n_bins,
                                     const T* __restrict__ tok_emb, const int32_t* __restrict__ ids,
                                     const int32_t* __restrict__ forced, const StepParams* __restrict__ prm,
-                                    float* __restrict__ Xd, int* __restrict__ idx_dec, int* err) {
+                                    float* __restrict__ Xd, int* __restrict__ idx_dec, float* __restrict__ ssq_out,
+                                    int* err) {
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.x;
@@ -235,6 +236,16 @@ __global__ void decode_embed_kernel(int d, int D, int P, int hidden, int vocab, 
   }
   const T* e = tok_emb + (size_t)(vocab - n_bins + bin) * hidden;
   for (int k = threadIdx.x; k < hidden; k += blockDim.x) Xd[(size_t)b * hidden + k] = to_f(e[k]);
+  // sums of squares of the new residual row, in the decode GEMVs' groups of rows
+  const int ng = hidden / kDecodeRowsPerCta;
+  for (int g = threadIdx.x; g < ng; g += blockDim.x) {
+    float t = 0.f;
+    for (int r = 0; r < kDecodeRowsPerCta; ++r) {
+      const float v = to_f(e[g * kDecodeRowsPerCta + r]);
+      t = fmaf(v, v, t);
+    }
+    ssq_out[(size_t)b * ng + g] = t;
+  }
   if (threadIdx.x == 0) idx_dec[b] = P + d - 1;
 }
 
@@ -338,9 +349,9 @@ void launch_residual(Rows rows, int B, int S, int hidden, const float* part, int
 template <typename T>
 void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
                          const int32_t* ids, const int32_t* forced, const StepParams* prm, float* Xd, int* idx_dec,
-                         int* err, cudaStream_t st) {
+                         float* ssq_out, int* err, cudaStream_t st) {
   launch_k(decode_embed_kernel<T>, dim3(B), dim3(256), 0, st, d, D, P, hidden, vocab, n_bins, tok_emb, ids, forced,
-           prm, Xd, idx_dec, err);
+           prm, Xd, idx_dec, ssq_out, err);
 }
 void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps, float* m_prev,
                    uint8_t* valid, float* user_step_margin, cudaStream_t st) {
@@ -360,7 +371,7 @@ void launch_finish(int B, int D, const StepParams* prm, const float* margins, co
                                         cudaStream_t);                                                            \
   template void launch_swiglu<T>(Rows, int, int, int, const float*, int, size_t, T*, cudaStream_t);               \
   template void launch_decode_embed<T>(int, int, int, int, int, int, int, const T*, const int32_t*,               \
-                                       const int32_t*, const StepParams*, float*, int*, int*, cudaStream_t);
+                                       const int32_t*, const StepParams*, float*, int*, float*, int*, cudaStream_t);
 VLAC_INST(float)
 VLAC_INST(bf16)
 

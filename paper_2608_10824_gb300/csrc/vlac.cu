@@ -61,7 +61,7 @@ struct vlac_ctx {
   int3* stats;
   uint8_t *mask, *full;
   int *idx, *M, *off, *emit_slot, *off_dec, *idx_dec, *err;
-  float *logits_ws, *attn_part;
+  float *logits_ws, *attn_part, *ssq_a, *ssq_b;
   // staged per-step inputs and outputs (fixed addresses, so a step can be a graph)
   uint8_t* in_frames;
   int32_t* in_prompt;
@@ -312,6 +312,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->err, 4, base);
     sc.take(c->logits_ws, Bm * (d.parallel ? d.n_action : 1) * d.n_bins * 4, base);
     sc.take(c->attn_part, Bm * d.n_heads * ((c->Tc + 31) / 32) * (d.head_dim + 2) * 4, base);
+    sc.take(c->ssq_a, Bm * (Hd / kDecodeRowsPerCta) * 4, base);
+    sc.take(c->ssq_b, Bm * (Hd / kDecodeRowsPerCta) * 4, base);
     const size_t fbytes = (size_t)d.n_views * d.img_h * d.img_w * 3;
     sc.take(c->in_frames, Bm * fbytes, base);
     sc.take(c->in_prompt, Bm * d.n_text * 4, base);
@@ -562,7 +564,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
     for (int a = 1; a < D; ++a) {
       const int pos = c->P + a - 1;
       launch_decode_embed<T>(B, a, D, c->P, Hd, d.vocab, nb, W(c->tok_emb), out->action_ids, forced, c->prm, c->Xd,
-                             c->idx_dec, c->err, st);
+                             c->idx_dec, c->ssq_b, c->err, st);
       c->launches += 1;
       for (int l = 0; l < L; ++l) {
         DGemv g{};
@@ -583,10 +585,12 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         g.pos = pos;
         g.rope_cos = c->rope_cos;
         g.rope_sin = c->rope_sin;
+        g.ssq_in = c->ssq_b;
+        g.n_ssq = Hd / kDecodeRowsPerCta;
         dgemv<T>(c, g, kEpiQkvRope, B, st);
         launch_dec_attention<T>(B, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, pos,
                                 c->attn_part, AO, st);
-        c->launches += 2;
+        c->launches += 1;
         // o-projection + residual
         DGemv o{};
         o.W = c->wo[l];
@@ -595,6 +599,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         o.xin = AO;
         o.Xres = c->Xd;
         o.n_out = Hd;
+        o.ssq_out = c->ssq_a;
         dgemv<T>(c, o, kEpiResid, B, st);
         // gate/up with the MLP RMSNorm prologue and SwiGLU
         DGemv u{};
@@ -606,6 +611,8 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         u.eps = eps;
         u.G = G;
         u.ffn = F;
+        u.ssq_in = c->ssq_a;
+        u.n_ssq = Hd / kDecodeRowsPerCta;
         dgemv<T>(c, u, kEpiSwiglu, B, st);
         // down-projection + residual
         DGemv dn{};
@@ -615,6 +622,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         dn.xin = G;
         dn.Xres = c->Xd;
         dn.n_out = Hd;
+        dn.ssq_out = c->ssq_b;
         dgemv<T>(c, dn, kEpiResid, B, st);
       }
       launch_head2<T>(c->Xd, nullptr, Hd, 1, B, Hd, nb, W(c->final_norm), W(c->head_w), eps, c->logits_ws, D, a,
