@@ -311,6 +311,10 @@ def main():
     ctx.prof_enable(False)
     g_ms, g_n, g_bytes = ctx.prof_read(0)
     p_ms, p_n, p_bytes = ctx.prof_read(1)
+    kinds = ["decode_gemv", "prefix_gemm", "prefix_attn", "decode_attn", "prefix_rows", "head", "other"]
+    breakdown = {"decode_gemv": g_ms / K, "prefix_gemm": p_ms / K}
+    for i in range(2, len(kinds)):
+        breakdown[kinds[i]] = ctx.prof_read(i)[0] / K
     gemv_gbs = g_bytes / (g_ms / 1e3) / 1e9 if g_ms > 0 else None
     gemm_gbs = p_bytes / (p_ms / 1e3) / 1e9 if p_ms > 0 else None
 
@@ -367,6 +371,7 @@ def main():
                      "kernel": "gemv_kernel (decode weight streaming)", "launches": g_n,
                      "avg_launch_us": 1e3 * g_ms / max(g_n, 1), "peak_source": f"{src} hbm_gbs"},
         "prefix_gemm": {"weight_gbs": gemm_gbs, "launches": p_n, "avg_launch_us": 1e3 * p_ms / max(p_n, 1)},
+        "device_ms_per_step_by_kind": {k: round(v, 4) for k, v in breakdown.items()},
         "clocks": clocks,
         "e2e": {"value": e2e, "unit": "steps/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "note": "frame + prompt H2D from pinned memory, action ids/margins/flag D2H, synchronised "

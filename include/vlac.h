@@ -167,15 +167,22 @@ uint64_t vlac_launch_count(const vlac_ctx* ctx);
  * recorded status (VLAC_ERR_TIMEOUT when the wait gave up). */
 int vlac_selftest_wait(vlac_ctx* ctx, uint32_t spin_limit);
 
-/* Per-launch timing of the weight-streaming kernels, for roofline reports.
- * While enabled, each launch of the kernel kinds below is bracketed by CUDA
- * events recorded on the launching stream.  vlac_prof_read waits for those
- * events, returns the summed device time, the number of launches and their
- * algorithmic bytes, and forgets them.  kind 0 = decode GEMV (bytes: weights
- * + inputs + outputs); kind 1 = prefix GEMM (bytes: weights only, the row
- * count being device-resident). */
+/* Per-launch timing, for roofline reports and time breakdowns.  While
+ * enabled (steps then run without graph replay), each kernel launch of the
+ * step is bracketed by CUDA events recorded on the launching stream and
+ * filed under one of the kinds below.  vlac_prof_read waits for the events of
+ * one kind, returns their summed device time, the number of launches and
+ * their algorithmic bytes, and forgets them.  Bytes are counted for kind 0
+ * (decode GEMV: weights + inputs + outputs) and kind 1 (prefix GEMM: weights
+ * only, the row count being device-resident); other kinds report 0 bytes. */
 #define VLAC_PROF_DECODE_GEMV 0
 #define VLAC_PROF_PREFIX_GEMM 1
+#define VLAC_PROF_PREFIX_ATTN 2 /* attention of the prefix pass */
+#define VLAC_PROF_DECODE_ATTN 3 /* attention of the decode passes */
+#define VLAC_PROF_ROWS 4        /* prefix row kernels: embedding, norms, epilogues */
+#define VLAC_PROF_HEAD 5        /* action head: logits and margins */
+#define VLAC_PROF_OTHER 6       /* selection, decode inputs, state update, staging */
+#define VLAC_PROF_KINDS 7
 int vlac_prof_enable(vlac_ctx* ctx, int on);
 int vlac_prof_read(vlac_ctx* ctx, int kind, double* total_ms, uint64_t* launches, double* bytes);
 

@@ -518,19 +518,31 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   auto W = [](void* p) { return static_cast<const T*>(p); };
 
   // Stage 1 and the gate + Stage-3 plan
-  launch_patch_stats(frames, k->prev, k->valid, c->prm, B, d.n_views, d.img_h, d.img_w, d.patch, c->stats, c->mask,
-                     out->static_mask, st);
-  launch_select(c->stats, c->mask, k->valid, k->m_prev, c->prm, ovr, B, c->Nv, S, L, c->P, d.parallel, D, c->full,
-                c->idx, c->M, c->off, c->emit_slot, out->recomputed, out->gate_auto, out->idx, out->M, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
+    launch_patch_stats(frames, k->prev, k->valid, c->prm, B, d.n_views, d.img_h, d.img_w, d.patch, c->stats, c->mask,
+                       out->static_mask, st);
+  }
+  {
+    ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
+    launch_select(c->stats, c->mask, k->valid, k->m_prev, c->prm, ovr, B, c->Nv, S, L, c->P, d.parallel, D, c->full,
+                  c->idx, c->M, c->off, c->emit_slot, out->recomputed, out->gate_auto, out->idx, out->M, st);
+  }
   c->launches += 3;
 
   // layer-0 inputs of the recomputed rows
   Rows r0{c->off, c->idx, S, c->X};
   const int* m0 = c->off + B;
-  launch_im2col<T>(r0, B, S, frames, d.n_views, d.img_h, d.img_w, d.patch, c->kpad, col, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_im2col<T>(r0, B, S, frames, d.n_views, d.img_h, d.img_w, d.patch, c->kpad, col, st);
+  }
   gemm<T>(c, &c->tm_col, &c->tm_patch, col, c->patch_w, m0, Hd, c->kpad, 1, st);
-  launch_embed<T>(r0, B, S, Hd, c->Nv, c->P, c->has_p, d.proprio_dim, d.n_text, d.vocab, prompt, proprio,
-                  W(c->tok_emb), c->part, W(c->proprio_w), W(c->action_emb), c->err, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_embed<T>(r0, B, S, Hd, c->Nv, c->P, c->has_p, d.proprio_dim, d.n_text, d.vocab, prompt, proprio,
+                    W(c->tok_emb), c->part, W(c->proprio_w), W(c->action_emb), c->err, st);
+  }
   c->launches += 2;
 
   const size_t rs = (size_t)c->rows_cap;
@@ -538,33 +550,57 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
     Rows rl{c->off + (size_t)l * (B + 1), c->idx, S, c->X};
     const int* ml = rl.off + B;
     const int* off_prev = l == 0 ? rl.off : c->off + (size_t)(l - 1) * (B + 1);
-    launch_layer_in<T>(rl, off_prev, B, S, Hd, l == 0 ? nullptr : k->H + (size_t)l * S * Hd, k->h_seq_stride,
-                       W(c->attn_norm[l]), eps, A, st);
+    {
+      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+      launch_layer_in<T>(rl, off_prev, B, S, Hd, l == 0 ? nullptr : k->H + (size_t)l * S * Hd, k->h_seq_stride,
+                         W(c->attn_norm[l]), eps, A, st);
+    }
     gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_qkv[l] : nullptr, A, c->wqkv[l], ml, 3 * Hd, Hd, c->split_qkv, st);
-    launch_qkv_epilogue<T>(rl, B, S, nh, hd, c->part, c->split_qkv, rs * 3 * Hd, c->rope_cos, c->rope_sin, Q,
-                           Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, st);
-    launch_attention<T>(rl, B, S, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, c->P,
-                        d.parallel, D, AO, st);
+    {
+      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+      launch_qkv_epilogue<T>(rl, B, S, nh, hd, c->part, c->split_qkv, rs * 3 * Hd, c->rope_cos, c->rope_sin, Q,
+                             Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, st);
+    }
+    {
+      ProfScope ps_(c, VLAC_PROF_PREFIX_ATTN, 0, st);
+      launch_attention<T>(rl, B, S, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, c->P,
+                          d.parallel, D, AO, st);
+    }
     gemm<T>(c, &c->tm_AO, c->bf16 ? &c->tm_o[l] : nullptr, AO, c->wo[l], ml, Hd, Hd, c->split_o, st);
-    launch_residual_norm<T>(rl, B, S, Hd, c->part, c->split_o, rs * Hd, W(c->ffn_norm[l]), eps, A, st);
+    {
+      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+      launch_residual_norm<T>(rl, B, S, Hd, c->part, c->split_o, rs * Hd, W(c->ffn_norm[l]), eps, A, st);
+    }
     gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_gu[l] : nullptr, A, c->wgu[l], ml, 2 * F, Hd, c->split_gu, st);
-    launch_swiglu<T>(rl, B, S, F, c->part, c->split_gu, rs * 2 * F, G, st);
+    {
+      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+      launch_swiglu<T>(rl, B, S, F, c->part, c->split_gu, rs * 2 * F, G, st);
+    }
     gemm<T>(c, &c->tm_G, c->bf16 ? &c->tm_d[l] : nullptr, G, c->wd[l], ml, Hd, F, c->split_d, st);
-    launch_residual(rl, B, S, Hd, c->part, c->split_d, rs * Hd, st);
+    {
+      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+      launch_residual(rl, B, S, Hd, c->part, c->split_d, rs * Hd, st);
+    }
     c->launches += 6;
   }
   // action head on the prefix pass: the last text row, or the parallel action block
-  launch_head2<T>(c->X, c->emit_slot, (size_t)S * Hd, d.parallel ? D : 1, B, Hd, nb, W(c->final_norm),
-                  W(c->head_w), eps, c->logits_ws, D, 0, out->action_ids, out->margins, out->logit_gap, out->logits,
-                  st);
+  {
+    ProfScope ps_(c, VLAC_PROF_HEAD, 0, st);
+    launch_head2<T>(c->X, c->emit_slot, (size_t)S * Hd, d.parallel ? D : 1, B, Hd, nb, W(c->final_norm),
+                    W(c->head_w), eps, c->logits_ws, D, 0, out->action_ids, out->margins, out->logit_gap, out->logits,
+                    st);
+  }
   c->launches += 2;
 
   if (!d.parallel) {
     // autoregressive decode: one row per sequence, fused GEMVs
     for (int a = 1; a < D; ++a) {
       const int pos = c->P + a - 1;
-      launch_decode_embed<T>(B, a, D, c->P, Hd, d.vocab, nb, W(c->tok_emb), out->action_ids, forced, c->prm, c->Xd,
-                             c->idx_dec, c->ssq_b, c->err, st);
+      {
+        ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
+        launch_decode_embed<T>(B, a, D, c->P, Hd, d.vocab, nb, W(c->tok_emb), out->action_ids, forced, c->prm, c->Xd,
+                               c->idx_dec, c->ssq_b, c->err, st);
+      }
       c->launches += 1;
       for (int l = 0; l < L; ++l) {
         DGemv g{};
@@ -588,8 +624,11 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         g.ssq_in = c->ssq_b;
         g.n_ssq = Hd / kDecodeRowsPerCta;
         dgemv<T>(c, g, kEpiQkvRope, B, st);
-        launch_dec_attention<T>(B, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, pos,
-                                c->attn_part, AO, st);
+        {
+          ProfScope ps_(c, VLAC_PROF_DECODE_ATTN, 0, st);
+          launch_dec_attention<T>(B, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, pos,
+                                  c->attn_part, AO, st);
+        }
         c->launches += 1;
         // o-projection + residual
         DGemv o{};
@@ -625,12 +664,18 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         dn.ssq_out = c->ssq_b;
         dgemv<T>(c, dn, kEpiResid, B, st);
       }
-      launch_head2<T>(c->Xd, nullptr, Hd, 1, B, Hd, nb, W(c->final_norm), W(c->head_w), eps, c->logits_ws, D, a,
-                      out->action_ids, out->margins, out->logit_gap, out->logits, st);
+      {
+        ProfScope ps_(c, VLAC_PROF_HEAD, 0, st);
+        launch_head2<T>(c->Xd, nullptr, Hd, 1, B, Hd, nb, W(c->final_norm), W(c->head_w), eps, c->logits_ws, D, a,
+                        out->action_ids, out->margins, out->logit_gap, out->logits, st);
+      }
       c->launches += 2;
     }
   }
-  launch_finish(B, D, c->prm, out->margins, out->logit_gap, k->m_prev, k->valid, out->step_margin, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
+    launch_finish(B, D, c->prm, out->margins, out->logit_gap, k->m_prev, k->valid, out->step_margin, st);
+  }
   c->launches += 1;
   const size_t fb = (size_t)d.n_views * d.img_h * d.img_w * 3;
   CK(cudaMemcpyAsync(k->prev, frames, (size_t)B * fb, cudaMemcpyDeviceToDevice, st));
@@ -724,7 +769,10 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   if (d.proprio_dim) add(in, proprio, c->in_proprio, (size_t)B * d.proprio_dim * 4);
   if (p.has_override) add(in, opts->gate_override, c->in_override, (size_t)B);
   if (p.has_forced) add(in, opts->forced_ids, c->in_forced, (size_t)B * D * 4);
-  launch_stage(p, c->prm, in, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
+    launch_stage(p, c->prm, in, st);
+  }
   c->launches += 1;
   int rc = run_step(c, k, st);
   if (rc) return rc;
@@ -739,7 +787,10 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   add(o, c->o_mask, out->static_mask, (size_t)B * c->Nv);
   add(o, c->o_idx, out->idx, (size_t)B * c->S * 4);
   add(o, c->o_M, out->M, (size_t)B * d.n_layers * 4);
-  launch_copies(o, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
+    launch_copies(o, st);
+  }
   c->launches += 1;
   CK(cudaGetLastError());
   return VLAC_OK;
@@ -780,6 +831,7 @@ extern "C" int vlac_prof_read(vlac_ctx* c, int kind, double* total_ms, uint64_t*
   if (!c || !total_ms || !launches || !bytes) return VLAC_ERR_INVALID_ARG;
   double ms = 0, by = 0;
   uint64_t n = 0;
+  if (kind < 0 || kind >= VLAC_PROF_KINDS) return VLAC_ERR_INVALID_ARG;
   std::vector<vlac_ctx::ProfRec> keep;
   for (auto& r : c->prof) {
     if (r.kind != kind) {
