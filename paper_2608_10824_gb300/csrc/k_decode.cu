@@ -7,6 +7,9 @@
 // Attention of the single query per head is split over key chunks and
 // combined in a fixed order.  The action head (final norm, bin logits) is a
 // multi-CTA GEMV followed by a one-warp top-2 / margin reduction per row.
+#include <algorithm>
+#include <type_traits>
+
 #include "internal.cuh"
 
 namespace vlac {
@@ -296,34 +299,55 @@ template void launch_dgemv<bf16>(const DGemv&, int, int, cudaStream_t);
 
 // ---- decode attention: one query per (sequence, head) ----------------------------
 //
-// One CTA per (head, sequence).  Each warp takes 32-key tiles (lane = key for
-// the scores, lane = output elements for P.V) with a running softmax; the
-// warps' partial results are combined in warp order.
+// One CTA per (head, sequence) with one warp per 32-key tile (up to 32 tiles).
+// A warp issues all loads of its tile at once -- lane j reads key j's K row,
+// and the V elements [lane*EPL, lane*EPL + EPL) of all 32 keys -- so the tile
+// costs one memory round trip.  Tiles are combined in tile order.
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
+               "l"(gmem)
+               : "memory");
+}
+
 template <typename T, int HD>
-__global__ void __launch_bounds__(256) dec_attn_kernel(const T* __restrict__ Q, const T* __restrict__ Kc,
+__global__ void __launch_bounds__(512) dec_attn_kernel(const T* __restrict__ Q, const T* __restrict__ Kc,
                                                        const T* __restrict__ Vc, size_t kv_seq_stride, int Tc, int pos,
                                                        int n_heads, float scale, T* __restrict__ O) {
-  constexpr int EPL = HD / 32, NW = 8, V = Vec<T>::n;
+  constexpr int EPL = HD / 32, V = Vec<T>::n, CPR = HD * (int)sizeof(T) / 16;  // 16-byte chunks per row
+  extern __shared__ __align__(16) uint8_t dsm[];
   __shared__ float qs[HD];
-  __shared__ float wm[NW], wl[NW];
-  __shared__ float wacc[NW][HD];
+  __shared__ float wm[16], wl[16];
+  __shared__ float wacc[16][HD];
   pdl_wait();
   pdl_trigger();
   const int h = blockIdx.x, b = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nw = blockDim.x >> 5;
   const int hidden = n_heads * HD;
-  for (int e = threadIdx.x; e < HD; e += blockDim.x) qs[e] = to_f(Q[(size_t)b * hidden + (size_t)h * HD + e]);
-  __syncthreads();
+  T* vbuf = reinterpret_cast<T*>(dsm) + (size_t)warp * 32 * HD;
   const T* Kh = Kc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
   const T* Vh = Vc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
   const int nkeys = min(pos + 1, Tc);
-  float m = -INFINITY, l = 0.f, acc[EPL];
+  for (int e = threadIdx.x; e < HD; e += blockDim.x) qs[e] = to_f(Q[(size_t)b * hidden + (size_t)h * HD + e]);
+  __syncthreads();
+  float m_run = -INFINITY, l_run = 0.f, acc[EPL];
 #pragma unroll
   for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
-  for (int j0 = warp * 32; j0 < nkeys; j0 += NW * 32) {
-    const int j = j0 + lane;
+  for (int j0 = warp * 32; j0 < nkeys; j0 += nw * 32) {
+    const int j = j0 + lane, jn = min(32, nkeys - j0);
+    // the tile's V rows go to shared memory asynchronously, its K rows to registers
+    for (int c = lane; c < jn * CPR; c += 32) {
+      const int jj = c / CPR, q = c - jj * CPR;
+      cp_async16(vbuf + (size_t)jj * HD + q * (16 / sizeof(T)), Vh + (size_t)(j0 + jj) * HD + q * (16 / sizeof(T)));
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    uint4 kr[HD / V];
+    if (j < nkeys) {
+      const uint4* src = reinterpret_cast<const uint4*>(Kh + (size_t)j * HD);
+#pragma unroll
+      for (int v = 0; v < HD / V; ++v) kr[v] = src[v];
+    }
     float sc = -INFINITY;
     if (j < nkeys) {
-      const uint4* kr = reinterpret_cast<const uint4*>(Kh + (size_t)j * HD);
       float d = 0.f;
 #pragma unroll
       for (int v = 0; v < HD / V; ++v) {
@@ -337,34 +361,36 @@ __global__ void __launch_bounds__(256) dec_attn_kernel(const T* __restrict__ Q, 
     float mt = sc;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
-    const float mn = fmaxf(m, mt);
+    const float mn = fmaxf(m_run, mt);
     const float p = (sc == -INFINITY) ? 0.f : expf(sc - mn);
-    const float corr = (m == -INFINITY) ? 0.f : expf(m - mn);
-    l = l * corr + warp_allsum(p);
+    const float corr = (m_run == -INFINITY) ? 0.f : expf(m_run - mn);
+    l_run = l_run * corr + warp_allsum(p);
 #pragma unroll
     for (int e = 0; e < EPL; ++e) acc[e] *= corr;
-    const int jn = min(32, nkeys - j0);
-#pragma unroll 4
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncwarp();
+#pragma unroll 8
     for (int jj = 0; jj < jn; ++jj) {
       const float pj = __shfl_sync(0xffffffffu, p, jj);
-      const T* vr = Vh + (size_t)(j0 + jj) * HD + lane * EPL;
+      const T* vr = vbuf + (size_t)jj * HD + lane * EPL;
 #pragma unroll
       for (int e = 0; e < EPL; ++e) acc[e] = fmaf(pj, to_f(vr[e]), acc[e]);
     }
-    m = mn;
+    __syncwarp();
+    m_run = mn;
   }
   if (lane == 0) {
-    wm[warp] = m;
-    wl[warp] = l;
+    wm[warp] = m_run;
+    wl[warp] = l_run;
   }
 #pragma unroll
   for (int e = 0; e < EPL; ++e) wacc[warp][lane * EPL + e] = acc[e];
   __syncthreads();
   for (int e = threadIdx.x; e < HD; e += blockDim.x) {
     float M = -INFINITY;
-    for (int w = 0; w < NW; ++w) M = fmaxf(M, wm[w]);
+    for (int w = 0; w < nw; ++w) M = fmaxf(M, wm[w]);
     float L = 0.f, o = 0.f;
-    for (int w = 0; w < NW; ++w) {
+    for (int w = 0; w < nw; ++w) {
       const float f = expf(wm[w] - M);
       L = fmaf(wl[w], f, L);
       o = fmaf(wacc[w][e], f, o);
@@ -373,17 +399,29 @@ __global__ void __launch_bounds__(256) dec_attn_kernel(const T* __restrict__ Q, 
   }
 }
 
+template <typename T, int HD>
+static void dec_attn_launch(int B, int n_heads, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride, int Tc,
+                            int pos, float scale, T* O, cudaStream_t st) {
+  const size_t per_warp = (size_t)32 * HD * sizeof(T);
+  const int tiles = (std::min(pos + 1, Tc) + 31) / 32;
+  const int warps = std::max(1, std::min({16, tiles, (int)((200 * 1024) / per_warp)}));
+  const size_t smem = per_warp * warps;
+  static size_t smem_set = 48 * 1024;  // raised once, before any graph capture of the kernel
+  if (smem > smem_set) {
+    cudaFuncSetAttribute(dec_attn_kernel<T, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(200 * 1024));
+    smem_set = 200 * 1024;
+  }
+  launch_k(dec_attn_kernel<T, HD>, dim3(n_heads, B), dim3(warps * 32), smem, st, Q, Kc, Vc, kv_seq_stride, Tc, pos,
+           n_heads, scale, O);
+}
+
 template <typename T>
 void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride,
                           int Tc, int pos, float* part, T* O, cudaStream_t st) {
   (void)part;
   const float scale = 1.0f / sqrtf((float)head_dim);
-  if (head_dim == 128)
-    launch_k(dec_attn_kernel<T, 128>, dim3(n_heads, B), dim3(256), 0, st, Q, Kc, Vc, kv_seq_stride, Tc, pos, n_heads,
-             scale, O);
-  else
-    launch_k(dec_attn_kernel<T, 64>, dim3(n_heads, B), dim3(256), 0, st, Q, Kc, Vc, kv_seq_stride, Tc, pos, n_heads,
-             scale, O);
+  if (head_dim == 128) dec_attn_launch<T, 128>(B, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, pos, scale, O, st);
+  else dec_attn_launch<T, 64>(B, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, pos, scale, O, st);
 }
 template void launch_dec_attention<float>(int, int, int, const float*, const float*, const float*, size_t, int, int,
                                           float*, float*, cudaStream_t);
