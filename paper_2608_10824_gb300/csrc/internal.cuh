@@ -63,6 +63,7 @@ struct DGemv {
   const float* ssq_in;  // normalising GEMV: per-producer-CTA sums of squares [nb][n_ssq]
   int n_ssq;
   float* ssq_out;       // residual GEMV: this launch's per-CTA sums of squares [nb][grid]
+  int* err;             // device error word (bounded waits)
 };
 constexpr int kDecodeRowsPerCta = 4;  // residual rows per decode-GEMV CTA (2 row pairs)
 
@@ -85,6 +86,53 @@ __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.lau
 __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
+
+// ---- mbarrier and bulk-copy helpers ------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase with `parity`; false after `limit` polls or once
+// another role raised *abort.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t limit, volatile int* abort) {
+  for (uint32_t i = 0; i < limit; ++i) {
+    if (mbar_test(bar, parity)) return true;
+    if (*abort) return false;
+  }
+  return false;
+}
+// 1-D bulk copy global -> shared completing on `bar` (16-byte aligned, bytes % 16 == 0).
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+constexpr uint32_t kWaitLimit = 1u << 24;
 
 __device__ __forceinline__ void set_error(int* err, int code) {
   if (err) atomicCAS(err, 0, code);
@@ -209,7 +257,8 @@ void launch_gemm_simt(const T* A, const T* W, const int* m_ptr, int m_cap, int N
                       cudaStream_t st);
 int launch_wait_selftest(int* err, uint32_t spin_limit, cudaStream_t st);
 template <typename T>
-void launch_dgemv(const DGemv& a, int epi, int nb, cudaStream_t st);
+void launch_dgemv(const DGemv& a, int epi, int nb, int n_sm, cudaStream_t st);
+int dgemv_grid(int n_pairs, int n_sm);  // CTAs (and sum-of-squares partials) of one decode GEMV
 template <typename T>
 void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride,
                           int Tc, int pos, float* part, T* O, cudaStream_t st);

@@ -92,210 +92,297 @@ __device__ __forceinline__ void norm_rows_to_smem(const float* __restrict__ X, c
 
 // ---- fused decode GEMV ----------------------------------------------------------
 //
-// A CTA owns RP row pairs (2*RP weight rows) over the full K; its 8 warps split
-// K into 8 contiguous segments and the per-warp partial dot products are
-// summed in warp order.  Small CTAs keep the last wave short.
+// Persistent weight-streaming GEMV: one CTA per SM owns a contiguous, byte-
+// balanced range of output row pairs.  A producer warp streams the pairs'
+// weight rows in chunks of kKC elements into a ring of kNS shared-memory
+// stages with 1-D bulk copies; 8 consumer warps (one row pair each per group
+// of 8 pairs) read the stages and the input vector from shared memory.  The
+// producer starts before the dependency wait (weights are constant), so a
+// kernel's first stages stream in while its predecessor drains.
 //
-// RMSNorm without a second pass: every residual-writing GEMV (and the decode
-// embedding) stores, per CTA and sequence, the sum of squares of the residual
-// elements it produced; a normalising GEMV sums those partials in index order
-// to get the row's mean square, then normalises its own K segment on the fly
-// (x * r * g rounded to T, as the GEMM input).
+// RMSNorm without a second pass over the row: every residual-writing GEMV
+// (and the decode embedding) stores per CTA and sequence the sum of squares
+// of the residual elements it produced; a normalising GEMV sums those
+// partials in index order for the mean square and normalises the input
+// vector once into shared memory (x * r * g rounded to T).
 
-constexpr int kDW = 8;  // warps per decode-GEMV CTA
+constexpr int kNC = 8;          // consumer warps
+constexpr int kNS = 5;          // stages
+constexpr int kRowChunkB = 1024;  // bytes of one row chunk in a stage
 
-template <typename T, int NB, int EPI, bool NORM, int RP, int UNROLL>
-__global__ void __launch_bounds__(kDW * 32) dgemv_kernel(DGemv a) {
+template <typename T>
+__host__ __device__ constexpr int row_chunk_elems() { return kRowChunkB / (int)sizeof(T); }
+
+__host__ __device__ inline size_t sgemv_xs_bytes(int nb, int K, int esz) {
+  return ((size_t)nb * K * esz + 1023) / 1024 * 1024;
+}
+constexpr size_t kStageB = (size_t)2 * kNC * kRowChunkB;
+
+template <typename T, int NB, int EPI, bool NORM, bool XG>
+__global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
   constexpr int V = Vec<T>::n;
-  constexpr int NR = 2 * RP;
-  __shared__ float red[kDW][NR][NB];
+  constexpr int KC = row_chunk_elems<T>();
+  extern __shared__ __align__(1024) uint8_t dsm[];
+  __shared__ __align__(8) uint64_t full_bar[kNS];
+  __shared__ __align__(8) uint64_t empty_bar[kNS];
+  __shared__ float red[kNC][NB];
   __shared__ float rr[NB];
-  __shared__ float xnew[NR][NB];
-  const int K = a.K;
+  __shared__ int abort_flag;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int K = a.K, nchunk = (K + KC - 1) / KC;
+  const int P = a.n_pairs;
+  const int p0 = (int)(((long long)P * blockIdx.x) / gridDim.x);
+  const int p1 = (int)(((long long)P * (blockIdx.x + 1)) / gridDim.x);
+  const int ngroups = (p1 - p0 + kNC - 1) / kNC;
   const int hd = a.head_dim, half = hd >> 1;
-  // weight rows of this CTA: pair q -> rows (row[2q], row[2q+1])
-  int row[NR];
-#pragma unroll
-  for (int q = 0; q < RP; ++q) {
-    const int p = blockIdx.x * RP + q;
+  T* xs = reinterpret_cast<T*>(dsm);
+  uint8_t* stages = dsm + (XG ? 0 : sgemv_xs_bytes(NB, K, (int)sizeof(T)));
+  const T* W = static_cast<const T*>(a.W);
+  auto pair_rows = [&](int p, int& r1, int& r2) {
     if constexpr (EPI == kEpiQkvRope) {
       const int hidden = a.n_heads * hd;
       const int sec = p / (hidden / 2), within = p - sec * (hidden / 2);
       const int h = within / half, e = within - h * half;
-      row[2 * q] = sec * hidden + h * hd + e;
-      row[2 * q + 1] = row[2 * q] + half;
+      r1 = sec * hidden + h * hd + e;
+      r2 = r1 + half;
     } else if constexpr (EPI == kEpiSwiglu) {
-      row[2 * q] = p;
-      row[2 * q + 1] = a.ffn + p;
+      r1 = p;
+      r2 = a.ffn + p;
     } else {
-      row[2 * q] = 2 * p;
-      row[2 * q + 1] = 2 * p + 1;
+      r1 = 2 * p;
+      r2 = 2 * p + 1;
     }
+  };
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kNS; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], kNC);
+    }
+    abort_flag = 0;
+    mbar_fence_init();
   }
-  const T* W = static_cast<const T*>(a.W);
-  // weights are constant: pull this CTA's rows into L2 before the dependency wait
-  if (warp < NR && lane == 0) prefetch_l2(W + (size_t)row[warp] * K, (uint32_t)(K * sizeof(T)));
-  pdl_wait();
-  pdl_trigger();
-  const int kv = K / V;
-  const int seg = (kv + kDW - 1) / kDW;
-  const int k_beg = warp * seg, k_end = min(kv, k_beg + seg);
-  float acc[NR][NB];
-#pragma unroll
-  for (int r = 0; r < NR; ++r)
-#pragma unroll
-    for (int b = 0; b < NB; ++b) acc[r][b] = 0.f;
-  if constexpr (NORM) {
-    // mean square of each residual row from the producers' partials (index order)
-    float s[NB];
-#pragma unroll
-    for (int b = 0; b < NB; ++b) s[b] = 0.f;
-    for (int c = threadIdx.x; c < a.n_ssq; c += blockDim.x)
-#pragma unroll
-      for (int b = 0; b < NB; ++b) s[b] += a.ssq_in[(size_t)b * a.n_ssq + c];
-#pragma unroll
-    for (int b = 0; b < NB; ++b) {
-      const float t = warp_allsum(s[b]);
-      if (lane == 0) red[warp][0][b] = t;
-    }
-    __syncthreads();
-    if (threadIdx.x < NB) {
-      float t = 0.f;
-      for (int w = 0; w < kDW; ++w) t += red[w][0][threadIdx.x];
-      rr[threadIdx.x] = 1.0f / sqrtf(t / (float)K + a.eps);
-    }
-    __syncthreads();
-  }
-  const uint4* xv = reinterpret_cast<const uint4*>(static_cast<const T*>(a.xin));
-  const T* gain = static_cast<const T*>(a.gain);
-  for (int k0 = k_beg + lane; k0 < k_end; k0 += 32 * UNROLL) {
-    uint4 wq[UNROLL][NR];
-#pragma unroll
-    for (int u = 0; u < UNROLL; ++u) {
-      const int k = k0 + u * 32;
-#pragma unroll
-      for (int r = 0; r < NR; ++r)
-        if (k < k_end) wq[u][r] = ld_stream(reinterpret_cast<const uint4*>(W + (size_t)row[r] * K) + k);
-    }
-#pragma unroll
-    for (int u = 0; u < UNROLL; ++u) {
-      const int k = k0 + u * 32;
-      if (k >= k_end) break;
-      float xf[NB][V];
-      if constexpr (NORM) {
-        float g[V];
-        unpack<T>(__ldg(reinterpret_cast<const uint4*>(gain) + k), g);
-#pragma unroll
-        for (int b = 0; b < NB; ++b) {
-          const float4* x4 = reinterpret_cast<const float4*>(a.X + (size_t)b * K + (size_t)k * V);
-#pragma unroll
-          for (int i = 0; i < V / 4; ++i) {
-            const float4 v4 = x4[i];
-            xf[b][4 * i + 0] = to_f(from_f<T>((v4.x * rr[b]) * g[4 * i + 0]));
-            xf[b][4 * i + 1] = to_f(from_f<T>((v4.y * rr[b]) * g[4 * i + 1]));
-            xf[b][4 * i + 2] = to_f(from_f<T>((v4.z * rr[b]) * g[4 * i + 2]));
-            xf[b][4 * i + 3] = to_f(from_f<T>((v4.w * rr[b]) * g[4 * i + 3]));
+  __syncthreads();
+  volatile int* abort = &abort_flag;
+
+  if (warp == kNC) {
+    // ---- producer: weights only, so it runs ahead of the dependency wait ----
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int g = 0; g < ngroups && !*abort; ++g) {
+        const int q0 = p0 + g * kNC, nq = min(kNC, p1 - q0);
+        for (int c = 0; c < nchunk; ++c) {
+          const int k0 = c * KC, kn = min(KC, K - k0);
+          if (!mbar_wait(&empty_bar[stage], phase ^ 1u, kWaitLimit, abort)) {
+            set_error(a.err, VLAC_ERR_TIMEOUT);
+            *abort = 1;
+            break;
+          }
+          uint8_t* st = stages + (size_t)stage * kStageB;
+          mbar_expect_tx(&full_bar[stage], (uint32_t)(nq * 2 * kn * sizeof(T)));
+          for (int q = 0; q < nq; ++q) {
+            int r1, r2;
+            pair_rows(q0 + q, r1, r2);
+            bulk_g2s(st + (size_t)(2 * q) * kRowChunkB, W + (size_t)r1 * K + k0, (uint32_t)(kn * sizeof(T)),
+                     &full_bar[stage]);
+            bulk_g2s(st + (size_t)(2 * q + 1) * kRowChunkB, W + (size_t)r2 * K + k0, (uint32_t)(kn * sizeof(T)),
+                     &full_bar[stage]);
+          }
+          if (++stage == kNS) {
+            stage = 0;
+            phase ^= 1u;
           }
         }
-      } else {
-#pragma unroll
-        for (int b = 0; b < NB; ++b) unpack<T>(__ldg(xv + (size_t)b * kv + k), xf[b]);
-      }
-#pragma unroll
-      for (int r = 0; r < NR; ++r) {
-        float wf[V];
-        unpack<T>(wq[u][r], wf);
-#pragma unroll
-        for (int b = 0; b < NB; ++b)
-#pragma unroll
-          for (int i = 0; i < V; ++i) acc[r][b] = fmaf(wf[i], xf[b][i], acc[r][b]);
       }
     }
+    pdl_wait();
+    pdl_trigger();
+    return;
   }
+
+  // ---- consumers ----
+  pdl_wait();
+  pdl_trigger();
+  const int tid = threadIdx.x;  // 0 .. kNC*32-1
+  if constexpr (NORM) {
+    float sacc[NB];
 #pragma unroll
-  for (int r = 0; r < NR; ++r)
+    for (int b = 0; b < NB; ++b) sacc[b] = 0.f;
+    for (int c = tid; c < a.n_ssq; c += kNC * 32)
+#pragma unroll
+      for (int b = 0; b < NB; ++b) sacc[b] += a.ssq_in[(size_t)b * a.n_ssq + c];
 #pragma unroll
     for (int b = 0; b < NB; ++b) {
-      const float t = warp_allsum(acc[r][b]);
-      if (lane == 0) red[warp][r][b] = t;
+      const float t = warp_allsum(sacc[b]);
+      if (lane == 0) red[warp][b] = t;
     }
-  __syncthreads();
-  if (threadIdx.x < RP * NB) {
-    const int q = threadIdx.x / NB, b = threadIdx.x - q * NB;
-    float y1 = 0.f, y2 = 0.f;
-    for (int w = 0; w < kDW; ++w) {
-      y1 += red[w][2 * q][b];
-      y2 += red[w][2 * q + 1][b];
+    asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
+    if (tid < NB) {
+      float t = 0.f;
+      for (int w = 0; w < kNC; ++w) t += red[w][tid];
+      rr[tid] = 1.0f / sqrtf(t / (float)K + a.eps);
     }
-    const int p = blockIdx.x * RP + q;
-    if constexpr (EPI == kEpiQkvRope) {
-      const int hidden = a.n_heads * hd;
-      const int sec = p / (hidden / 2), within = p - sec * (hidden / 2);
-      const int h = within / half, e = within - h * half;
-      float o1 = y1, o2 = y2;
-      if (sec < 2) {
-        const float c = a.rope_cos[(size_t)a.pos * half + e], sn = a.rope_sin[(size_t)a.pos * half + e];
-        o1 = y1 * c - y2 * sn;
-        o2 = y2 * c + y1 * sn;
+    asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
+    const T* g = static_cast<const T*>(a.gain);
+    for (int k = tid; k < K; k += kNC * 32) {
+      const float gk = to_f(g[k]);
+#pragma unroll
+      for (int b = 0; b < NB; ++b) xs[(size_t)b * K + k] = from_f<T>((a.X[(size_t)b * K + k] * rr[b]) * gk);
+    }
+  } else if constexpr (!XG) {
+    const uint4* src = reinterpret_cast<const uint4*>(static_cast<const T*>(a.xin));
+    uint4* dst = reinterpret_cast<uint4*>(xs);
+    for (int i = tid; i < NB * K / V; i += kNC * 32) dst[i] = src[i];
+  }
+  asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
+  const T* xsrc = XG ? static_cast<const T*>(a.xin) : xs;
+  bool aborted = false;
+
+  float ssq[NB];
+#pragma unroll
+  for (int b = 0; b < NB; ++b) ssq[b] = 0.f;
+  int stage = 0;
+  uint32_t phase = 0;
+  for (int g = 0; g < ngroups; ++g) {
+    const int q0 = p0 + g * kNC, nq = min(kNC, p1 - q0);
+    const bool mine = warp < nq;
+    float acc1[NB], acc2[NB];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) acc1[b] = acc2[b] = 0.f;
+    for (int c = 0; c < nchunk; ++c) {
+      const int k0 = c * KC, kn = min(KC, K - k0);
+      bool ok = true;
+      if (lane == 0) ok = mbar_wait(&full_bar[stage], phase, kWaitLimit, abort);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) {
+        if (lane == 0) {
+          set_error(a.err, VLAC_ERR_TIMEOUT);
+          *abort = 1;
+        }
+        aborted = true;
+        break;
       }
-      T* dst = sec == 0 ? static_cast<T*>(a.Q) + (size_t)b * hidden + (size_t)h * hd
-                        : static_cast<T*>(sec == 1 ? a.Kc : a.Vc) + (size_t)b * a.kv_seq_stride +
-                              ((size_t)h * a.Tc + a.pos) * hd;
-      dst[e] = from_f<T>(o1);
-      dst[e + half] = from_f<T>(o2);
-    } else if constexpr (EPI == kEpiSwiglu) {
-      static_cast<T*>(a.G)[(size_t)b * a.ffn + p] = from_f<T>((y1 / (1.0f + expf(-y1))) * y2);
-    } else {
-      float* x = a.Xres + (size_t)b * a.n_out;
-      const float n1 = x[row[2 * q]] + y1, n2 = x[row[2 * q + 1]] + y2;
-      x[row[2 * q]] = n1;
-      x[row[2 * q + 1]] = n2;
-      xnew[2 * q][b] = n1;
-      xnew[2 * q + 1][b] = n2;
+      if (mine) {
+        const uint8_t* st = stages + (size_t)stage * kStageB;
+        const uint4* w1 = reinterpret_cast<const uint4*>(st + (size_t)(2 * warp) * kRowChunkB);
+        const uint4* w2 = reinterpret_cast<const uint4*>(st + (size_t)(2 * warp + 1) * kRowChunkB);
+        for (int v = lane; v < kn / V; v += 32) {
+          float f1[V], f2[V];
+          unpack<T>(w1[v], f1);
+          unpack<T>(w2[v], f2);
+#pragma unroll
+          for (int b = 0; b < NB; ++b) {
+            float xf[V];
+            uint4 xu;
+            if constexpr (XG) xu = __ldg(reinterpret_cast<const uint4*>(xsrc + (size_t)b * K + k0) + v);
+            else xu = reinterpret_cast<const uint4*>(xsrc + (size_t)b * K + k0)[v];
+            unpack<T>(xu, xf);
+#pragma unroll
+            for (int i = 0; i < V; ++i) {
+              acc1[b] = fmaf(f1[i], xf[i], acc1[b]);
+              acc2[b] = fmaf(f2[i], xf[i], acc2[b]);
+            }
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_bar[stage]);
+      if (++stage == kNS) {
+        stage = 0;
+        phase ^= 1u;
+      }
+    }
+    if (aborted) break;
+    if (!mine) continue;
+    float y1 = 0.f, y2 = 0.f;
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      const float t1 = warp_allsum(acc1[b]), t2 = warp_allsum(acc2[b]);
+      if (lane == b) {
+        y1 = t1;
+        y2 = t2;
+      }
+    }
+    if (lane < NB) {
+      const int b = lane, p = q0 + warp;
+      if constexpr (EPI == kEpiQkvRope) {
+        const int hidden = a.n_heads * hd;
+        const int sec = p / (hidden / 2), within = p - sec * (hidden / 2);
+        const int h = within / half, e = within - h * half;
+        float o1 = y1, o2 = y2;
+        if (sec < 2) {
+          const float cs = a.rope_cos[(size_t)a.pos * half + e], sn = a.rope_sin[(size_t)a.pos * half + e];
+          o1 = y1 * cs - y2 * sn;
+          o2 = y2 * cs + y1 * sn;
+        }
+        T* dst = sec == 0 ? static_cast<T*>(a.Q) + (size_t)b * hidden + (size_t)h * hd
+                          : static_cast<T*>(sec == 1 ? a.Kc : a.Vc) + (size_t)b * a.kv_seq_stride +
+                                ((size_t)h * a.Tc + a.pos) * hd;
+        dst[e] = from_f<T>(o1);
+        dst[e + half] = from_f<T>(o2);
+      } else if constexpr (EPI == kEpiSwiglu) {
+        static_cast<T*>(a.G)[(size_t)b * a.ffn + p] = from_f<T>((y1 / (1.0f + expf(-y1))) * y2);
+      } else {
+        float* x = a.Xres + (size_t)b * a.n_out;
+        const float n1 = x[2 * p] + y1, n2 = x[2 * p + 1] + y2;
+        x[2 * p] = n1;
+        x[2 * p + 1] = n2;
+        ssq[0] = fmaf(n1, n1, fmaf(n2, n2, ssq[0]));  // lane b keeps sequence b's sum in ssq[0]
+      }
     }
   }
   if constexpr (EPI == kEpiResid) {
-    __syncthreads();
-    if (threadIdx.x < NB) {
+    if (lane < NB) red[warp][lane] = ssq[0];
+    asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
+    if (tid < NB) {
       float t = 0.f;
-      for (int r = 0; r < NR; ++r) t = fmaf(xnew[r][threadIdx.x], xnew[r][threadIdx.x], t);
-      a.ssq_out[(size_t)threadIdx.x * gridDim.x + blockIdx.x] = t;
+      for (int w = 0; w < kNC; ++w) t += red[w][tid];
+      a.ssq_out[(size_t)tid * gridDim.x + blockIdx.x] = t;
     }
   }
 }
 
 template <typename T, int NB, int EPI, bool NORM>
-static void dgemv_nb(const DGemv& a, cudaStream_t st) {
-  constexpr int RP = 2;
-  constexpr int U = NB <= 2 ? 2 : 1;
-  launch_k(dgemv_kernel<T, NB, EPI, NORM, RP, U>, dim3(a.n_pairs / RP), dim3(kDW * 32), 0, st, a);
+static void dgemv_nb(const DGemv& a, int grid, cudaStream_t st) {
+  // the input vector lives in shared memory unless it is large (then it is read through L1)
+  const bool xg = !NORM && (size_t)NB * a.K * sizeof(T) > 64 * 1024;
+  const size_t smem = (xg ? 0 : sgemv_xs_bytes(NB, a.K, (int)sizeof(T))) + (size_t)kNS * kStageB;
+  auto kern = xg ? dgemv_kernel<T, NB, EPI, NORM, true> : dgemv_kernel<T, NB, EPI, NORM, false>;
+  static size_t smem_set[2] = {48 * 1024, 48 * 1024};  // raised once per kernel, before any graph capture of it
+  if (smem > smem_set[xg]) {
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    smem_set[xg] = smem;
+  }
+  launch_k(kern, dim3(grid), dim3((kNC + 1) * 32), smem, st, a);
 }
 
 template <typename T, int EPI, bool NORM>
-static void dgemv_dispatch(const DGemv& a, int nb, cudaStream_t st) {
+static void dgemv_dispatch(const DGemv& a, int nb, int grid, cudaStream_t st) {
   switch (nb) {
-    case 1: dgemv_nb<T, 1, EPI, NORM>(a, st); break;
-    case 2: dgemv_nb<T, 2, EPI, NORM>(a, st); break;
-    case 3: dgemv_nb<T, 3, EPI, NORM>(a, st); break;
-    case 4: dgemv_nb<T, 4, EPI, NORM>(a, st); break;
-    case 5: dgemv_nb<T, 5, EPI, NORM>(a, st); break;
-    case 6: dgemv_nb<T, 6, EPI, NORM>(a, st); break;
-    case 7: dgemv_nb<T, 7, EPI, NORM>(a, st); break;
-    default: dgemv_nb<T, 8, EPI, NORM>(a, st); break;
+    case 1: dgemv_nb<T, 1, EPI, NORM>(a, grid, st); break;
+    case 2: dgemv_nb<T, 2, EPI, NORM>(a, grid, st); break;
+    case 3: dgemv_nb<T, 3, EPI, NORM>(a, grid, st); break;
+    case 4: dgemv_nb<T, 4, EPI, NORM>(a, grid, st); break;
+    case 5: dgemv_nb<T, 5, EPI, NORM>(a, grid, st); break;
+    case 6: dgemv_nb<T, 6, EPI, NORM>(a, grid, st); break;
+    case 7: dgemv_nb<T, 7, EPI, NORM>(a, grid, st); break;
+    default: dgemv_nb<T, 8, EPI, NORM>(a, grid, st); break;
   }
 }
 
+// Grid: one CTA per SM (at most one pair per CTA).
 template <typename T>
-void launch_dgemv(const DGemv& a, int epi, int nb, cudaStream_t st) {
+void launch_dgemv(const DGemv& a, int epi, int nb, int n_sm, cudaStream_t st) {
+  const int grid = std::min(a.n_pairs, n_sm);
   switch (epi) {
-    case kEpiQkvRope: dgemv_dispatch<T, kEpiQkvRope, true>(a, nb, st); break;
-    case kEpiSwiglu: dgemv_dispatch<T, kEpiSwiglu, true>(a, nb, st); break;
-    default: dgemv_dispatch<T, kEpiResid, false>(a, nb, st); break;
+    case kEpiQkvRope: dgemv_dispatch<T, kEpiQkvRope, true>(a, nb, grid, st); break;
+    case kEpiSwiglu: dgemv_dispatch<T, kEpiSwiglu, true>(a, nb, grid, st); break;
+    default: dgemv_dispatch<T, kEpiResid, false>(a, nb, grid, st); break;
   }
 }
-template void launch_dgemv<float>(const DGemv&, int, int, cudaStream_t);
-template void launch_dgemv<bf16>(const DGemv&, int, int, cudaStream_t);
+template void launch_dgemv<float>(const DGemv&, int, int, int, cudaStream_t);
+template void launch_dgemv<bf16>(const DGemv&, int, int, int, cudaStream_t);
+int dgemv_grid(int n_pairs, int n_sm) { return std::min(n_pairs, n_sm); }
 
 // ---- decode attention: one query per (sequence, head) ----------------------------
 //

@@ -44,6 +44,7 @@ struct vlac_ctx {
   bool bf16;
   size_t esz;
   int dev;
+  int n_sm = 1;
   // weights
   char* wmem = nullptr;
   void *tok_emb, *patch_w, *proprio_w, *action_emb, *final_norm, *head_w;
@@ -205,7 +206,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   c->pdim = d.patch * d.patch * 3;
   c->kpad = c->bf16 ? (int)align_up(c->pdim, 64) : c->pdim;
   c->rows_cap = d.max_batch * c->S;
-  if (cudaGetDevice(&c->dev) != cudaSuccess) {
+  if (cudaGetDevice(&c->dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&c->n_sm, cudaDevAttrMultiProcessorCount, c->dev) != cudaSuccess) {
     delete c;
     return VLAC_ERR_CUDA;
   }
@@ -312,8 +314,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->err, 4, base);
     sc.take(c->logits_ws, Bm * (d.parallel ? d.n_action : 1) * d.n_bins * 4, base);
     sc.take(c->attn_part, Bm * d.n_heads * ((c->Tc + 31) / 32) * (d.head_dim + 2) * 4, base);
-    sc.take(c->ssq_a, Bm * (Hd / kDecodeRowsPerCta) * 4, base);
-    sc.take(c->ssq_b, Bm * (Hd / kDecodeRowsPerCta) * 4, base);
+    sc.take(c->ssq_a, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
+    sc.take(c->ssq_b, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
     const size_t fbytes = (size_t)d.n_views * d.img_h * d.img_w * 3;
     sc.take(c->in_frames, Bm * fbytes, base);
     sc.take(c->in_prompt, Bm * d.n_text * 4, base);
@@ -475,7 +477,7 @@ void dgemv(vlac_ctx* c, const DGemv& a, int epi, int nb, cudaStream_t st) {
   ProfScope ps(c, VLAC_PROF_DECODE_GEMV,
                (double)2 * a.n_pairs * a.K * sizeof(T) + (double)nb * a.K * sizeof(T) + (double)nb * 2 * a.n_pairs * 4,
                st);
-  launch_dgemv<T>(a, epi, nb, st);
+  launch_dgemv<T>(a, epi, nb, c->n_sm, st);
   c->launches += 1;
 }
 
@@ -622,7 +624,8 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         g.rope_cos = c->rope_cos;
         g.rope_sin = c->rope_sin;
         g.ssq_in = c->ssq_b;
-        g.n_ssq = Hd / kDecodeRowsPerCta;
+        g.n_ssq = l == 0 ? Hd / kDecodeRowsPerCta : dgemv_grid(Hd / 2, c->n_sm);  // embedding or down-projection
+        g.err = c->err;
         dgemv<T>(c, g, kEpiQkvRope, B, st);
         {
           ProfScope ps_(c, VLAC_PROF_DECODE_ATTN, 0, st);
@@ -639,6 +642,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         o.Xres = c->Xd;
         o.n_out = Hd;
         o.ssq_out = c->ssq_a;
+        o.err = c->err;
         dgemv<T>(c, o, kEpiResid, B, st);
         // gate/up with the MLP RMSNorm prologue and SwiGLU
         DGemv u{};
@@ -651,7 +655,8 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         u.G = G;
         u.ffn = F;
         u.ssq_in = c->ssq_a;
-        u.n_ssq = Hd / kDecodeRowsPerCta;
+        u.n_ssq = dgemv_grid(Hd / 2, c->n_sm);  // o-projection
+        u.err = c->err;
         dgemv<T>(c, u, kEpiSwiglu, B, st);
         // down-projection + residual
         DGemv dn{};
@@ -662,6 +667,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         dn.Xres = c->Xd;
         dn.n_out = Hd;
         dn.ssq_out = c->ssq_b;
+        dn.err = c->err;
         dgemv<T>(c, dn, kEpiResid, B, st);
       }
       {
