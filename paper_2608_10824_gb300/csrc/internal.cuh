@@ -64,6 +64,8 @@ struct DGemv {
   int n_ssq;
   float* ssq_out;       // residual GEMV: this launch's per-CTA sums of squares [nb][grid]
   int* err;             // device error word (bounded waits)
+  int ns;               // stages of the weight ring
+  int chunk_b;          // bytes of one weight row chunk (multiple of 16)
 };
 constexpr int kDecodeRowsPerCta = 4;  // residual rows per decode-GEMV CTA (2 row pairs)
 

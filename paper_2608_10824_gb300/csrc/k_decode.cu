@@ -107,24 +107,22 @@ __device__ __forceinline__ void norm_rows_to_smem(const float* __restrict__ X, c
 // vector once into shared memory (x * r * g rounded to T).
 
 constexpr int kNC = 8;          // consumer warps
-constexpr int kNS = 5;          // stages
-constexpr int kRowChunkB = 1024;  // bytes of one row chunk in a stage
-
-template <typename T>
-__host__ __device__ constexpr int row_chunk_elems() { return kRowChunkB / (int)sizeof(T); }
+constexpr int kMaxNS = 24;      // stage ring capacity
 
 __host__ __device__ inline size_t sgemv_xs_bytes(int nb, int K, int esz) {
   return ((size_t)nb * K * esz + 1023) / 1024 * 1024;
 }
-constexpr size_t kStageB = (size_t)2 * kNC * kRowChunkB;
 
 template <typename T, int NB, int EPI, bool NORM, bool XG>
 __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
   constexpr int V = Vec<T>::n;
-  constexpr int KC = row_chunk_elems<T>();
+  const int kNS = a.ns;                       // stages
+  const int kRowChunkB = a.chunk_b;           // bytes of one row chunk in a stage
+  const size_t kStageB = (size_t)2 * kNC * kRowChunkB;
+  const int KC = kRowChunkB / (int)sizeof(T);
   extern __shared__ __align__(1024) uint8_t dsm[];
-  __shared__ __align__(8) uint64_t full_bar[kNS];
-  __shared__ __align__(8) uint64_t empty_bar[kNS];
+  __shared__ __align__(8) uint64_t full_bar[kMaxNS];
+  __shared__ __align__(8) uint64_t empty_bar[kMaxNS];
   __shared__ float red[kNC][NB];
   __shared__ float rr[NB];
   __shared__ int abort_flag;
@@ -346,7 +344,7 @@ template <typename T, int NB, int EPI, bool NORM>
 static void dgemv_nb(const DGemv& a, int grid, cudaStream_t st) {
   // the input vector lives in shared memory unless it is large (then it is read through L1)
   const bool xg = !NORM && (size_t)NB * a.K * sizeof(T) > 64 * 1024;
-  const size_t smem = (xg ? 0 : sgemv_xs_bytes(NB, a.K, (int)sizeof(T))) + (size_t)kNS * kStageB;
+  const size_t smem = (xg ? 0 : sgemv_xs_bytes(NB, a.K, (int)sizeof(T))) + (size_t)a.ns * 2 * kNC * a.chunk_b;
   auto kern = xg ? dgemv_kernel<T, NB, EPI, NORM, true> : dgemv_kernel<T, NB, EPI, NORM, false>;
   static size_t smem_set[2] = {48 * 1024, 48 * 1024};  // raised once per kernel, before any graph capture of it
   if (smem > smem_set[xg]) {

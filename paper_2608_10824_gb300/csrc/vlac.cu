@@ -45,6 +45,7 @@ struct vlac_ctx {
   size_t esz;
   int dev;
   int n_sm = 1;
+  int gemv_ns = 10, gemv_chunk_b = 1024;  // decode-GEMV weight ring
   // weights
   char* wmem = nullptr;
   void *tok_emb, *patch_w, *proprio_w, *action_emb, *final_norm, *head_w;
@@ -194,6 +195,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (!c) return VLAC_ERR_OOM;
   if (const char* e = std::getenv("VLAC_PDL")) g_pdl = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_GRAPH")) c->use_graph = std::atoi(e) != 0;
+  if (const char* e = std::getenv("VLAC_GEMV_NS")) c->gemv_ns = std::max(2, std::min(24, std::atoi(e)));
+  if (const char* e = std::getenv("VLAC_GEMV_CHUNK")) c->gemv_chunk_b = std::max(256, std::atoi(e)) / 256 * 256;
   c->d = *dims;
   const vlac_dims& d = c->d;
   c->bf16 = d.dtype == VLAC_BF16;
@@ -473,7 +476,13 @@ struct ProfScope {
 };
 
 template <typename T>
-void dgemv(vlac_ctx* c, const DGemv& a, int epi, int nb, cudaStream_t st) {
+void dgemv(vlac_ctx* c, const DGemv& a_in, int epi, int nb, cudaStream_t st) {
+  DGemv a = a_in;
+  a.ns = c->gemv_ns;
+  a.chunk_b = c->gemv_chunk_b;
+  // the stage ring must fit next to the input vector in shared memory
+  const size_t xs = ((size_t)nb * a.K * sizeof(T) + 1023) / 1024 * 1024;
+  while (a.ns > 2 && (size_t)a.ns * 16 * a.chunk_b + (xs > 64 * 1024 ? 0 : xs) > 200 * 1024) --a.ns;
   ProfScope ps(c, VLAC_PROF_DECODE_GEMV,
                (double)2 * a.n_pairs * a.K * sizeof(T) + (double)nb * a.K * sizeof(T) + (double)nb * 2 * a.n_pairs * 4,
                st);
