@@ -65,7 +65,6 @@ struct DGemv {
   float* ssq_out;       // residual GEMV: this launch's per-CTA sums of squares [nb][grid]
   int* err;             // device error word (bounded waits)
   int ns;               // stages of the weight ring
-  int chunk_b;          // bytes of one weight row chunk (multiple of 16)
 };
 constexpr int kDecodeRowsPerCta = 4;  // residual rows per decode-GEMV CTA (2 row pairs)
 
@@ -261,6 +260,11 @@ int launch_wait_selftest(int* err, uint32_t spin_limit, cudaStream_t st);
 template <typename T>
 void launch_dgemv(const DGemv& a, int epi, int nb, int n_sm, cudaStream_t st);
 int dgemv_grid(int n_pairs, int n_sm);  // CTAs (and sum-of-squares partials) of one decode GEMV
+// Decode-streaming copy of a projection (W: [rows][K]); see k_decode.cu for the layout.
+template <typename T>
+void launch_tile_decode_weights(const T* W, int K, int n_pairs, int epi, int n_heads, int head_dim, int ffn, T* out,
+                                cudaStream_t st);
+size_t tiled_decode_elems(int K, int n_pairs);
 template <typename T>
 void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride,
                           int Tc, int pos, float* part, T* O, cudaStream_t st);

@@ -92,13 +92,21 @@ __device__ __forceinline__ void norm_rows_to_smem(const float* __restrict__ X, c
 
 // ---- fused decode GEMV ----------------------------------------------------------
 //
-// Persistent weight-streaming GEMV: one CTA per SM owns a contiguous, byte-
-// balanced range of output row pairs.  A producer warp streams the pairs'
-// weight rows in chunks of kKC elements into a ring of kNS shared-memory
-// stages with 1-D bulk copies; 8 consumer warps (one row pair each per group
-// of 8 pairs) read the stages and the input vector from shared memory.  The
-// producer starts before the dependency wait (weights are constant), so a
-// kernel's first stages stream in while its predecessor drains.
+// Weight layout for decode streaming (built once at create time): output row
+// pairs are grouped 4 at a time (8 weight rows); a group's K range is cut into
+// chunks of kDecKC elements; the tile [8 rows][chunk] is contiguous, and the
+// tiles of a group follow each other, then the next group.  Pair p's rows:
+//   QKV:     (i, i + head_dim/2) of one head of q, k or v;
+//   SwiGLU:  (gate j, up j);
+//   other:   (2p, 2p + 1).
+//
+// Persistent GEMV: one CTA per SM owns a contiguous, balanced range of groups
+// and so one contiguous region of the tiled weights.  A producer warp streams
+// it tile by tile into a ring of shared-memory stages with 1-D bulk copies;
+// the producer starts before the dependency wait (weights are constant), so a
+// kernel's first stages stream in while its predecessor drains.  8 consumer
+// warps: warp w handles pair w/2 over half of each tile's K range; the halves
+// are added in order at the end of the group.
 //
 // RMSNorm without a second pass over the row: every residual-writing GEMV
 // (and the decode embedding) stores per CTA and sequence the sum of squares
@@ -107,52 +115,89 @@ __device__ __forceinline__ void norm_rows_to_smem(const float* __restrict__ X, c
 // vector once into shared memory (x * r * g rounded to T).
 
 constexpr int kNC = 8;          // consumer warps
+constexpr int kGP = 4;          // row pairs per group
 constexpr int kMaxNS = 24;      // stage ring capacity
+constexpr int kDecTileB = 4096; // bytes of one tile row (K chunk)
 
 __host__ __device__ inline size_t sgemv_xs_bytes(int nb, int K, int esz) {
   return ((size_t)nb * K * esz + 1023) / 1024 * 1024;
 }
 
+template <int EPI>
+__host__ __device__ __forceinline__ void dec_pair_rows(int p, int n_heads, int head_dim, int ffn, int& r1, int& r2) {
+  if (EPI == kEpiQkvRope) {
+    const int half = head_dim >> 1, hidden = n_heads * head_dim;
+    const int sec = p / (hidden / 2), within = p - sec * (hidden / 2);
+    const int h = within / half, e = within - h * half;
+    r1 = sec * hidden + h * head_dim + e;
+    r2 = r1 + half;
+  } else if (EPI == kEpiSwiglu) {
+    r1 = p;
+    r2 = ffn + p;
+  } else {
+    r1 = 2 * p;
+    r2 = 2 * p + 1;
+  }
+}
+
+// Builds the tiled copy: one block per (group, tile row).
+template <typename T, int EPI>
+__global__ void tile_decode_weights_kernel(const T* __restrict__ W, int K, int n_pairs, int n_heads, int head_dim,
+                                           int ffn, T* __restrict__ out) {
+  const int KC = kDecTileB / (int)sizeof(T);
+  const int g = blockIdx.x, r = blockIdx.y;  // r: 0..7
+  const int p = g * kGP + r / 2;
+  int r1 = 0, r2 = 0;
+  if (p < n_pairs) dec_pair_rows<EPI>(p, n_heads, head_dim, ffn, r1, r2);
+  const T* src = W + (size_t)((r & 1) ? r2 : r1) * K;
+  T* base = out + (size_t)g * 2 * kGP * K;
+  for (int k = threadIdx.x; k < K; k += blockDim.x) {
+    const int c = k / KC, kk = k - c * KC, kn = min(KC, K - c * KC);
+    base[(size_t)2 * kGP * c * KC + (size_t)r * kn + kk] = p < n_pairs ? src[k] : from_f<T>(0.f);
+  }
+}
+
+template <typename T>
+void launch_tile_decode_weights(const T* W, int K, int n_pairs, int epi, int n_heads, int head_dim, int ffn, T* out,
+                                cudaStream_t st) {
+  const int n_groups = (n_pairs + kGP - 1) / kGP;
+  dim3 grid(n_groups, 2 * kGP);
+  if (epi == kEpiQkvRope)
+    tile_decode_weights_kernel<T, kEpiQkvRope><<<grid, 256, 0, st>>>(W, K, n_pairs, n_heads, head_dim, ffn, out);
+  else if (epi == kEpiSwiglu)
+    tile_decode_weights_kernel<T, kEpiSwiglu><<<grid, 256, 0, st>>>(W, K, n_pairs, n_heads, head_dim, ffn, out);
+  else
+    tile_decode_weights_kernel<T, kEpiResid><<<grid, 256, 0, st>>>(W, K, n_pairs, n_heads, head_dim, ffn, out);
+}
+template void launch_tile_decode_weights<float>(const float*, int, int, int, int, int, int, float*, cudaStream_t);
+template void launch_tile_decode_weights<bf16>(const bf16*, int, int, int, int, int, int, bf16*, cudaStream_t);
+size_t tiled_decode_elems(int K, int n_pairs) { return (size_t)((n_pairs + kGP - 1) / kGP) * 2 * kGP * K; }
+
 template <typename T, int NB, int EPI, bool NORM, bool XG>
 __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
   constexpr int V = Vec<T>::n;
-  const int kNS = a.ns;                       // stages
-  const int kRowChunkB = a.chunk_b;           // bytes of one row chunk in a stage
-  const size_t kStageB = (size_t)2 * kNC * kRowChunkB;
-  const int KC = kRowChunkB / (int)sizeof(T);
+  constexpr int KC = kDecTileB / (int)sizeof(T);
+  constexpr int TR = 2 * kGP;  // tile rows
+  const int NS = a.ns;
+  const size_t stage_b = (size_t)TR * kDecTileB;
   extern __shared__ __align__(1024) uint8_t dsm[];
   __shared__ __align__(8) uint64_t full_bar[kMaxNS];
   __shared__ __align__(8) uint64_t empty_bar[kMaxNS];
   __shared__ float red[kNC][NB];
+  __shared__ float half_acc[kGP][2][NB];
   __shared__ float rr[NB];
   __shared__ int abort_flag;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int K = a.K, nchunk = (K + KC - 1) / KC;
-  const int P = a.n_pairs;
-  const int p0 = (int)(((long long)P * blockIdx.x) / gridDim.x);
-  const int p1 = (int)(((long long)P * (blockIdx.x + 1)) / gridDim.x);
-  const int ngroups = (p1 - p0 + kNC - 1) / kNC;
+  const int G = (a.n_pairs + kGP - 1) / kGP;
+  const int g0 = (int)(((long long)G * blockIdx.x) / gridDim.x);
+  const int g1 = (int)(((long long)G * (blockIdx.x + 1)) / gridDim.x);
   const int hd = a.head_dim, half = hd >> 1;
   T* xs = reinterpret_cast<T*>(dsm);
   uint8_t* stages = dsm + (XG ? 0 : sgemv_xs_bytes(NB, K, (int)sizeof(T)));
-  const T* W = static_cast<const T*>(a.W);
-  auto pair_rows = [&](int p, int& r1, int& r2) {
-    if constexpr (EPI == kEpiQkvRope) {
-      const int hidden = a.n_heads * hd;
-      const int sec = p / (hidden / 2), within = p - sec * (hidden / 2);
-      const int h = within / half, e = within - h * half;
-      r1 = sec * hidden + h * hd + e;
-      r2 = r1 + half;
-    } else if constexpr (EPI == kEpiSwiglu) {
-      r1 = p;
-      r2 = a.ffn + p;
-    } else {
-      r1 = 2 * p;
-      r2 = 2 * p + 1;
-    }
-  };
+  const T* Wt = static_cast<const T*>(a.W);
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kNS; ++s) {
+    for (int s = 0; s < NS; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], kNC);
     }
@@ -167,26 +212,19 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      for (int g = 0; g < ngroups && !*abort; ++g) {
-        const int q0 = p0 + g * kNC, nq = min(kNC, p1 - q0);
+      for (int g = g0; g < g1 && !*abort; ++g) {
+        const T* gbase = Wt + (size_t)g * TR * K;
         for (int c = 0; c < nchunk; ++c) {
-          const int k0 = c * KC, kn = min(KC, K - k0);
+          const int kn = min(KC, K - c * KC);
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, kWaitLimit, abort)) {
             set_error(a.err, VLAC_ERR_TIMEOUT);
             *abort = 1;
             break;
           }
-          uint8_t* st = stages + (size_t)stage * kStageB;
-          mbar_expect_tx(&full_bar[stage], (uint32_t)(nq * 2 * kn * sizeof(T)));
-          for (int q = 0; q < nq; ++q) {
-            int r1, r2;
-            pair_rows(q0 + q, r1, r2);
-            bulk_g2s(st + (size_t)(2 * q) * kRowChunkB, W + (size_t)r1 * K + k0, (uint32_t)(kn * sizeof(T)),
-                     &full_bar[stage]);
-            bulk_g2s(st + (size_t)(2 * q + 1) * kRowChunkB, W + (size_t)r2 * K + k0, (uint32_t)(kn * sizeof(T)),
-                     &full_bar[stage]);
-          }
-          if (++stage == kNS) {
+          const uint32_t bytes = (uint32_t)(TR * kn * sizeof(T));
+          mbar_expect_tx(&full_bar[stage], bytes);
+          bulk_g2s(stages + (size_t)stage * stage_b, gbase + (size_t)TR * c * KC, bytes, &full_bar[stage]);
+          if (++stage == NS) {
             stage = 0;
             phase ^= 1u;
           }
@@ -234,21 +272,20 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
   }
   asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
   const T* xsrc = XG ? static_cast<const T*>(a.xin) : xs;
-  bool aborted = false;
 
+  const int q = warp >> 1, hk = warp & 1;  // pair within the group, K half
   float ssq[NB];
 #pragma unroll
   for (int b = 0; b < NB; ++b) ssq[b] = 0.f;
+  bool aborted = false;
   int stage = 0;
   uint32_t phase = 0;
-  for (int g = 0; g < ngroups; ++g) {
-    const int q0 = p0 + g * kNC, nq = min(kNC, p1 - q0);
-    const bool mine = warp < nq;
+  for (int g = g0; g < g1; ++g) {
     float acc1[NB], acc2[NB];
 #pragma unroll
     for (int b = 0; b < NB; ++b) acc1[b] = acc2[b] = 0.f;
     for (int c = 0; c < nchunk; ++c) {
-      const int k0 = c * KC, kn = min(KC, K - k0);
+      const int k0 = c * KC, kn = min(KC, K - k0), kh = kn >> 1;
       bool ok = true;
       if (lane == 0) ok = mbar_wait(&full_bar[stage], phase, kWaitLimit, abort);
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -260,49 +297,58 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
         aborted = true;
         break;
       }
-      if (mine) {
-        const uint8_t* st = stages + (size_t)stage * kStageB;
-        const uint4* w1 = reinterpret_cast<const uint4*>(st + (size_t)(2 * warp) * kRowChunkB);
-        const uint4* w2 = reinterpret_cast<const uint4*>(st + (size_t)(2 * warp + 1) * kRowChunkB);
-        for (int v = lane; v < kn / V; v += 32) {
-          float f1[V], f2[V];
-          unpack<T>(w1[v], f1);
-          unpack<T>(w2[v], f2);
+      const T* st = reinterpret_cast<const T*>(stages + (size_t)stage * stage_b);
+      const uint4* w1 = reinterpret_cast<const uint4*>(st + (size_t)(2 * q) * kn + hk * kh);
+      const uint4* w2 = reinterpret_cast<const uint4*>(st + (size_t)(2 * q + 1) * kn + hk * kh);
+      for (int v = lane; v < kh / V; v += 32) {
+        float f1[V], f2[V];
+        unpack<T>(w1[v], f1);
+        unpack<T>(w2[v], f2);
 #pragma unroll
-          for (int b = 0; b < NB; ++b) {
-            float xf[V];
-            uint4 xu;
-            if constexpr (XG) xu = __ldg(reinterpret_cast<const uint4*>(xsrc + (size_t)b * K + k0) + v);
-            else xu = reinterpret_cast<const uint4*>(xsrc + (size_t)b * K + k0)[v];
-            unpack<T>(xu, xf);
+        for (int b = 0; b < NB; ++b) {
+          float xf[V];
+          const uint4* xp = reinterpret_cast<const uint4*>(xsrc + (size_t)b * K + k0 + hk * kh);
+          uint4 xu;
+          if constexpr (XG) xu = __ldg(xp + v);
+          else xu = xp[v];
+          unpack<T>(xu, xf);
 #pragma unroll
-            for (int i = 0; i < V; ++i) {
-              acc1[b] = fmaf(f1[i], xf[i], acc1[b]);
-              acc2[b] = fmaf(f2[i], xf[i], acc2[b]);
-            }
+          for (int i = 0; i < V; ++i) {
+            acc1[b] = fmaf(f1[i], xf[i], acc1[b]);
+            acc2[b] = fmaf(f2[i], xf[i], acc2[b]);
           }
         }
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty_bar[stage]);
-      if (++stage == kNS) {
+      if (++stage == NS) {
         stage = 0;
         phase ^= 1u;
       }
     }
     if (aborted) break;
-    if (!mine) continue;
-    float y1 = 0.f, y2 = 0.f;
+    // add the two K halves of every pair in order, then the epilogue
 #pragma unroll
     for (int b = 0; b < NB; ++b) {
       const float t1 = warp_allsum(acc1[b]), t2 = warp_allsum(acc2[b]);
-      if (lane == b) {
-        y1 = t1;
-        y2 = t2;
+      if (hk == 1 && lane == 0) {
+        half_acc[q][0][b] = t1;
+        half_acc[q][1][b] = t2;
       }
+      acc1[b] = t1;
+      acc2[b] = t2;
     }
-    if (lane < NB) {
-      const int b = lane, p = q0 + warp;
+    asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
+    const int p = g * kGP + q;
+    if (hk == 0 && lane < NB && p < a.n_pairs) {
+      const int b = lane;
+      float y1 = 0.f, y2 = 0.f;
+#pragma unroll
+      for (int bb = 0; bb < NB; ++bb)
+        if (bb == b) {
+          y1 = acc1[bb] + half_acc[q][0][bb];
+          y2 = acc2[bb] + half_acc[q][1][bb];
+        }
       if constexpr (EPI == kEpiQkvRope) {
         const int hidden = a.n_heads * hd;
         const int sec = p / (hidden / 2), within = p - sec * (hidden / 2);
@@ -328,9 +374,10 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
         ssq[0] = fmaf(n1, n1, fmaf(n2, n2, ssq[0]));  // lane b keeps sequence b's sum in ssq[0]
       }
     }
+    asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));  // half_acc is reused by the next group
   }
   if constexpr (EPI == kEpiResid) {
-    if (lane < NB) red[warp][lane] = ssq[0];
+    if (lane < NB) red[warp][lane] = (hk == 0) ? ssq[0] : 0.f;
     asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
     if (tid < NB) {
       float t = 0.f;
@@ -344,7 +391,7 @@ template <typename T, int NB, int EPI, bool NORM>
 static void dgemv_nb(const DGemv& a, int grid, cudaStream_t st) {
   // the input vector lives in shared memory unless it is large (then it is read through L1)
   const bool xg = !NORM && (size_t)NB * a.K * sizeof(T) > 64 * 1024;
-  const size_t smem = (xg ? 0 : sgemv_xs_bytes(NB, a.K, (int)sizeof(T))) + (size_t)a.ns * 2 * kNC * a.chunk_b;
+  const size_t smem = (xg ? 0 : sgemv_xs_bytes(NB, a.K, (int)sizeof(T))) + (size_t)a.ns * 2 * kGP * kDecTileB;
   auto kern = xg ? dgemv_kernel<T, NB, EPI, NORM, true> : dgemv_kernel<T, NB, EPI, NORM, false>;
   static size_t smem_set[2] = {48 * 1024, 48 * 1024};  // raised once per kernel, before any graph capture of it
   if (smem > smem_set[xg]) {
@@ -368,10 +415,11 @@ static void dgemv_dispatch(const DGemv& a, int nb, int grid, cudaStream_t st) {
   }
 }
 
-// Grid: one CTA per SM (at most one pair per CTA).
+int dgemv_grid(int n_pairs, int n_sm) { return std::min((n_pairs + kGP - 1) / kGP, n_sm); }
+
 template <typename T>
 void launch_dgemv(const DGemv& a, int epi, int nb, int n_sm, cudaStream_t st) {
-  const int grid = std::min(a.n_pairs, n_sm);
+  const int grid = dgemv_grid(a.n_pairs, n_sm);
   switch (epi) {
     case kEpiQkvRope: dgemv_dispatch<T, kEpiQkvRope, true>(a, nb, grid, st); break;
     case kEpiSwiglu: dgemv_dispatch<T, kEpiSwiglu, true>(a, nb, grid, st); break;
@@ -380,7 +428,6 @@ void launch_dgemv(const DGemv& a, int epi, int nb, int n_sm, cudaStream_t st) {
 }
 template void launch_dgemv<float>(const DGemv&, int, int, int, cudaStream_t);
 template void launch_dgemv<bf16>(const DGemv&, int, int, int, cudaStream_t);
-int dgemv_grid(int n_pairs, int n_sm) { return std::min(n_pairs, n_sm); }
 
 // ---- decode attention: one query per (sequence, head) ----------------------------
 //

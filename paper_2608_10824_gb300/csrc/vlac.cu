@@ -45,7 +45,9 @@ struct vlac_ctx {
   size_t esz;
   int dev;
   int n_sm = 1;
-  int gemv_ns = 10, gemv_chunk_b = 1024;  // decode-GEMV weight ring
+  int gemv_ns = 6;  // decode-GEMV weight ring stages (32 KB each)
+  char* dmem = nullptr;  // decode-streaming copies of the projections
+  std::vector<void*> dqkv, dwo, dgu, dwd;
   // weights
   char* wmem = nullptr;
   void *tok_emb, *patch_w, *proprio_w, *action_emb, *final_norm, *head_w;
@@ -172,6 +174,7 @@ extern "C" int vlac_destroy(vlac_ctx* c) {
   for (auto e : c->ev_pool) cudaEventDestroy(e);
   if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
   if (c->wmem) cudaFree(c->wmem);
+  if (c->dmem) cudaFree(c->dmem);
   if (c->wsmem) cudaFree(c->wsmem);
   if (c->err_host) cudaFreeHost(c->err_host);
   delete c;
@@ -196,7 +199,6 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (const char* e = std::getenv("VLAC_PDL")) g_pdl = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_GRAPH")) c->use_graph = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_GEMV_NS")) c->gemv_ns = std::max(2, std::min(24, std::atoi(e)));
-  if (const char* e = std::getenv("VLAC_GEMV_CHUNK")) c->gemv_chunk_b = std::max(256, std::atoi(e)) / 256 * 256;
   c->d = *dims;
   const vlac_dims& d = c->d;
   c->bf16 = d.dtype == VLAC_BF16;
@@ -272,6 +274,49 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
          cp(c->wd[l], w->w_down[l], Hd * F * E);
   }
   if (!ok) return fail(VLAC_ERR_CUDA);
+  {  // decode-streaming copies: pair-grouped, K-chunked tiles (one bulk copy per pipeline stage)
+    const size_t e_qkv = tiled_decode_elems(Hd, 3 * Hd / 2), e_o = tiled_decode_elems(Hd, Hd / 2);
+    const size_t e_gu = tiled_decode_elems(Hd, F), e_d = tiled_decode_elems(F, Hd / 2);
+    Carve dc;
+    auto plan_d = [&](char* base) {
+      dc = Carve();
+      c->dqkv.resize(L); c->dwo.resize(L); c->dgu.resize(L); c->dwd.resize(L);
+      for (size_t l = 0; l < L; ++l) {
+        dc.take(c->dqkv[l], e_qkv * E, base);
+        dc.take(c->dwo[l], e_o * E, base);
+        dc.take(c->dgu[l], e_gu * E, base);
+        dc.take(c->dwd[l], e_d * E, base);
+      }
+    };
+    plan_d(nullptr);
+    if (cudaMalloc(&c->dmem, dc.off) != cudaSuccess) {
+      (void)cudaGetLastError();
+      return fail(VLAC_ERR_OOM);
+    }
+    plan_d(c->dmem);
+    for (size_t l = 0; l < L; ++l) {
+      if (c->bf16) {
+        launch_tile_decode_weights<bf16>((const bf16*)c->wqkv[l], Hd, 3 * Hd / 2, kEpiQkvRope, d.n_heads, d.head_dim, F,
+                                         (bf16*)c->dqkv[l], 0);
+        launch_tile_decode_weights<bf16>((const bf16*)c->wo[l], Hd, Hd / 2, kEpiResid, d.n_heads, d.head_dim, F,
+                                         (bf16*)c->dwo[l], 0);
+        launch_tile_decode_weights<bf16>((const bf16*)c->wgu[l], Hd, F, kEpiSwiglu, d.n_heads, d.head_dim, F,
+                                         (bf16*)c->dgu[l], 0);
+        launch_tile_decode_weights<bf16>((const bf16*)c->wd[l], F, Hd / 2, kEpiResid, d.n_heads, d.head_dim, F,
+                                         (bf16*)c->dwd[l], 0);
+      } else {
+        launch_tile_decode_weights<float>((const float*)c->wqkv[l], Hd, 3 * Hd / 2, kEpiQkvRope, d.n_heads,
+                                          d.head_dim, F, (float*)c->dqkv[l], 0);
+        launch_tile_decode_weights<float>((const float*)c->wo[l], Hd, Hd / 2, kEpiResid, d.n_heads, d.head_dim, F,
+                                          (float*)c->dwo[l], 0);
+        launch_tile_decode_weights<float>((const float*)c->wgu[l], Hd, F, kEpiSwiglu, d.n_heads, d.head_dim, F,
+                                          (float*)c->dgu[l], 0);
+        launch_tile_decode_weights<float>((const float*)c->wd[l], F, Hd / 2, kEpiResid, d.n_heads, d.head_dim, F,
+                                          (float*)c->dwd[l], 0);
+      }
+    }
+    if (cudaGetLastError() != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) return fail(VLAC_ERR_CUDA);
+  }
   {  // RoPE tables: angle pos * theta^(-2i/head_dim) in fp64, stored fp32
     const int half = d.head_dim / 2;
     std::vector<float> cs((size_t)c->Tc * half), sn((size_t)c->Tc * half);
@@ -479,10 +524,9 @@ template <typename T>
 void dgemv(vlac_ctx* c, const DGemv& a_in, int epi, int nb, cudaStream_t st) {
   DGemv a = a_in;
   a.ns = c->gemv_ns;
-  a.chunk_b = c->gemv_chunk_b;
-  // the stage ring must fit next to the input vector in shared memory
+  // the stage ring (32 KB stages) must fit next to the input vector in shared memory
   const size_t xs = ((size_t)nb * a.K * sizeof(T) + 1023) / 1024 * 1024;
-  while (a.ns > 2 && (size_t)a.ns * 16 * a.chunk_b + (xs > 64 * 1024 ? 0 : xs) > 200 * 1024) --a.ns;
+  while (a.ns > 2 && (size_t)a.ns * 32 * 1024 + (xs > 64 * 1024 ? 0 : xs) > 200 * 1024) --a.ns;
   ProfScope ps(c, VLAC_PROF_DECODE_GEMV,
                (double)2 * a.n_pairs * a.K * sizeof(T) + (double)nb * a.K * sizeof(T) + (double)nb * 2 * a.n_pairs * 4,
                st);
@@ -619,7 +663,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         g.n_heads = nh;
         g.head_dim = hd;
         // q, k, v with the attention RMSNorm prologue, RoPE and the K/V scatter
-        g.W = c->wqkv[l];
+        g.W = c->dqkv[l];
         g.n_pairs = 3 * Hd / 2;
         g.K = Hd;
         g.X = c->Xd;
@@ -644,7 +688,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         c->launches += 1;
         // o-projection + residual
         DGemv o{};
-        o.W = c->wo[l];
+        o.W = c->dwo[l];
         o.n_pairs = Hd / 2;
         o.K = Hd;
         o.xin = AO;
@@ -655,7 +699,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         dgemv<T>(c, o, kEpiResid, B, st);
         // gate/up with the MLP RMSNorm prologue and SwiGLU
         DGemv u{};
-        u.W = c->wgu[l];
+        u.W = c->dgu[l];
         u.n_pairs = F;
         u.K = Hd;
         u.X = c->Xd;
@@ -669,7 +713,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         dgemv<T>(c, u, kEpiSwiglu, B, st);
         // down-projection + residual
         DGemv dn{};
-        dn.W = c->wd[l];
+        dn.W = c->dwd[l];
         dn.n_pairs = Hd / 2;
         dn.K = F;
         dn.xin = G;
