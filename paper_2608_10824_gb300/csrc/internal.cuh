@@ -250,8 +250,12 @@ struct CopyList {
 void launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st);
 void launch_copies(const CopyList& list, cudaStream_t st);
 
+// Tensor maps of one activation buffer with boxes of 32, 64, 128 and 256 rows.
+struct ActMaps {
+  CUtensorMap m[4];
+};
 // GEMMs: out[s][m][n] = sum over split s of A[m][k] * W[n][k]; rows m < *m_ptr.
-void launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
+void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
                     int splits, float* out, int* err, uint32_t wait_limit, cudaStream_t st);
 template <typename T>
 void launch_gemm_simt(const T* A, const T* W, const int* m_ptr, int m_cap, int N, int K, float* out,

@@ -19,7 +19,7 @@ namespace tc {
 
 constexpr int kBM = 128;        // weight rows per CTA (MMA M)
 constexpr int kBK = 64;         // K elements per stage = one 128-byte swizzle row
-constexpr int kBoxRows = 32;    // token rows per TMA box of the activation operand
+constexpr int kBoxRows = 32;    // granularity of the activation operand's token rows (boxes of 32..256 rows)
 constexpr int kMaxTok = 512;    // token columns per pass (TMEM has 512 fp32 columns)
 constexpr int kMaxStages = 8;
 constexpr int kWTileBytes = kBM * kBK * 2;  // 16 KB
@@ -92,7 +92,7 @@ __device__ __forceinline__ uint32_t idesc_bf16(int n) {
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
+    gemm_tc_kernel(const __grid_constant__ ActMaps tmA, const __grid_constant__ CUtensorMap tmW,
                    const int* __restrict__ m_ptr, int m_cap, int N, int k_chunks, int chunks_per_split,
                    float* __restrict__ out, size_t split_stride, int* __restrict__ err, uint32_t wait_limit) {
   extern __shared__ uint8_t smem_raw[];
@@ -179,8 +179,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint8_t* at = wt + kWTileBytes;
           mbar_expect_tx(&full_bar[stage], kWTileBytes + (uint32_t)nbox * kBoxRows * 128u);
           tma_load_2d(wt, &tmW, kc * kBK, n0, &full_bar[stage]);
-          for (int bx = 0; bx < nbox; ++bx)
-            tma_load_2d(at + (size_t)bx * kBoxRows * 128, &tmA, kc * kBK, row0 + bx * kBoxRows, &full_bar[stage]);
+          // the token rows in as few boxes as possible: 256, 128, 64 and 32 rows
+          for (int done = 0, left = nbox; left > 0;) {
+            const int lg = left >= 8 ? 3 : left >= 4 ? 2 : left >= 2 ? 1 : 0;
+            tma_load_2d(at + (size_t)done * kBoxRows * 128, &tmA.m[lg], kc * kBK, row0 + done * kBoxRows,
+                        &full_bar[stage]);
+            done += 1 << lg;
+            left -= 1 << lg;
+          }
           prod_cnt[stage] += 1;
           last_par[stage] = phase;
           if (++stage == n_stages) {
@@ -284,7 +290,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace tc
 
-void launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
+void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
                     int splits, float* out, int* err, uint32_t wait_limit, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {

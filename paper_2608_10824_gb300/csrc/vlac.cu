@@ -55,7 +55,8 @@ struct vlac_ctx {
   float *rope_cos, *rope_sin;
   // TMA descriptors (bf16 only)
   std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_d;
-  CUtensorMap tm_patch, tm_A, tm_AO, tm_G, tm_col;
+  CUtensorMap tm_patch;
+  ActMaps tm_A, tm_AO, tm_G, tm_col;
   int split_qkv = 1, split_o = 1, split_gu = 1, split_d = 1;
   // workspace
   char* wsmem = nullptr;
@@ -405,9 +406,13 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   // ---- TMA descriptors ----
   if (c->bf16) {
     c->tm_qkv.resize(L); c->tm_o.resize(L); c->tm_gu.resize(L); c->tm_d.resize(L);
-    bool mok = make_map(&c->tm_patch, c->patch_w, Hd, c->kpad, 128) && make_map(&c->tm_A, c->A, rc_, Hd, 32) &&
-               make_map(&c->tm_AO, c->AO, rc_, Hd, 32) && make_map(&c->tm_G, c->G, rc_, F, 32) &&
-               make_map(&c->tm_col, c->col, rc_, c->kpad, 32);
+    auto act = [&](ActMaps* am, const void* base, size_t cols) {
+      bool r = true;
+      for (int i = 0; i < 4; ++i) r = r && make_map(&am->m[i], base, rc_, cols, 32u << i);
+      return r;
+    };
+    bool mok = make_map(&c->tm_patch, c->patch_w, Hd, c->kpad, 128) && act(&c->tm_A, c->A, Hd) &&
+               act(&c->tm_AO, c->AO, Hd) && act(&c->tm_G, c->G, F) && act(&c->tm_col, c->col, c->kpad);
     for (size_t l = 0; l < L && mok; ++l)
       mok = make_map(&c->tm_qkv[l], c->wqkv[l], 3 * Hd, Hd, 128) && make_map(&c->tm_o[l], c->wo[l], Hd, Hd, 128) &&
             make_map(&c->tm_gu[l], c->wgu[l], 2 * F, Hd, 128) && make_map(&c->tm_d[l], c->wd[l], Hd, F, 128);
@@ -535,7 +540,7 @@ void dgemv(vlac_ctx* c, const DGemv& a_in, int epi, int nb, cudaStream_t st) {
 }
 
 template <typename T>
-void gemm(vlac_ctx* c, const CUtensorMap* tmA, const CUtensorMap* tmW, const T* A, const void* W, const int* m_ptr,
+void gemm(vlac_ctx* c, const ActMaps* tmA, const CUtensorMap* tmW, const T* A, const void* W, const int* m_ptr,
           int N, int K, int splits, cudaStream_t st) {
   ProfScope ps(c, VLAC_PROF_PREFIX_GEMM, (double)N * K * sizeof(T), st);
   if constexpr (sizeof(T) == 2) {
