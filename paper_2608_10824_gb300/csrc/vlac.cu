@@ -67,6 +67,8 @@ struct vlac_ctx {
   uint8_t *mask, *full;
   int *idx, *M, *off, *emit_slot, *off_dec, *idx_dec, *err;
   float *logits_ws, *attn_part, *ssq_a, *ssq_b;
+  float* sk_ws;    // stream-K partial tiles, one per CTA
+  int* sk_flags;   // stream-K partial-ready flags, one per CTA
   // staged per-step inputs and outputs (fixed addresses, so a step can be a graph)
   uint8_t* in_frames;
   int32_t* in_prompt;
@@ -333,10 +335,6 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   }
 
   // ---- workspace ----
-  if (c->bf16) {
-    c->split_o = 4;
-    c->split_d = 4;
-  }
   const size_t rc_ = c->rows_cap, Bm = d.max_batch;
   const size_t part_n = std::max({3 * Hd, 2 * F, (size_t)c->split_o * Hd, (size_t)c->split_d * Hd});
   Carve sc;
@@ -363,6 +361,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->err, 4, base);
     sc.take(c->logits_ws, Bm * (d.parallel ? d.n_action : 1) * d.n_bins * 4, base);
     sc.take(c->attn_part, Bm * d.n_heads * ((c->Tc + 31) / 32) * (d.head_dim + 2) * 4, base);
+    sc.take(c->sk_ws, c->bf16 ? (size_t)c->n_sm * 128 * 512 * 4 : 16, base);
+    sc.take(c->sk_flags, (size_t)c->n_sm * 4, base);
     sc.take(c->ssq_a, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
     sc.take(c->ssq_b, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
     const size_t fbytes = (size_t)d.n_views * d.img_h * d.img_w * 3;
@@ -544,7 +544,9 @@ void gemm(vlac_ctx* c, const ActMaps* tmA, const CUtensorMap* tmW, const T* A, c
           int N, int K, int splits, cudaStream_t st) {
   ProfScope ps(c, VLAC_PROF_PREFIX_GEMM, (double)N * K * sizeof(T), st);
   if constexpr (sizeof(T) == 2) {
-    launch_gemm_tc(tmA, tmW, m_ptr, c->rows_cap, N, K, splits, c->part, c->err, c->wait_limit, st);
+    (void)splits;
+    launch_gemm_tc(tmA, tmW, m_ptr, c->rows_cap, N, K, gemm_tc_grid(N, K, c->rows_cap, c->n_sm), c->part, c->sk_ws,
+                   c->sk_flags, c->err, c->wait_limit, st);
   } else {
     launch_gemm_simt<T>(A, static_cast<const T*>(W), m_ptr, c->rows_cap, N, K, c->part, st);
   }
