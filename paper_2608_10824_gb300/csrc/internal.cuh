@@ -254,13 +254,9 @@ void launch_copies(const CopyList& list, cudaStream_t st);
 struct ActMaps {
   CUtensorMap m[4];
 };
-// GEMMs: out[m][n] = sum_k A[m][k] * W[n][k] for rows m < *m_ptr.
-// tcgen05 stream-K GEMM: `grid` CTAs from gemm_tc_grid(); ws holds one
-// partial tile (128 x 512 fp32) per CTA and flags one int per CTA (zero
-// between launches).
-int gemm_tc_grid(int N, int K, int max_rows, int n_sm);
-void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K, int grid,
-                    float* out, float* ws, int* flags, int* err, uint32_t wait_limit, cudaStream_t st);
+// GEMMs: out[s][m][n] = sum over split s of A[m][k] * W[n][k]; rows m < *m_ptr.
+void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
+                    int splits, float* out, int* err, uint32_t wait_limit, cudaStream_t st);
 template <typename T>
 void launch_gemm_simt(const T* A, const T* W, const int* m_ptr, int m_cap, int N, int K, float* out,
                       cudaStream_t st);

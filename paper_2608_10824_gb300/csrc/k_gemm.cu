@@ -8,8 +8,6 @@
 //   - gemv:      decode passes (M = batch <= 8): HBM-bound weight streaming
 //                with 16-byte non-allocating loads and fp32 FMAs.
 //   - gemm_simt: the fp32 tiny model.
-#include <algorithm>
-
 #include "internal.cuh"
 
 namespace vlac {
@@ -93,21 +91,10 @@ __device__ __forceinline__ uint32_t idesc_bf16(int n) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
 }
 
-// Segments of a stream-K schedule: the (pass, weight tile, K chunk) units of
-// the GEMM are numbered tile-major and CTA c owns units [c*U/G, (c+1)*U/G).
-// A CTA's range is a run of segments, each a K-chunk range of one tile; only
-// its first segment can start inside a tile.  The CTA holding a tile's first
-// K chunk adds the other segments' partial sums in K order (deterministic).
-struct SkPlan {
-  int tiles, k_chunks, G;
-  long long U;
-  __device__ long long start(int c) const { return (U * c) / G; }
-};
-
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ ActMaps tmA, const __grid_constant__ CUtensorMap tmW,
-                   const int* __restrict__ m_ptr, int m_cap, int N, int k_chunks, float* __restrict__ out,
-                   float* __restrict__ ws, int* __restrict__ flags, int* __restrict__ err, uint32_t wait_limit) {
+                   const int* __restrict__ m_ptr, int m_cap, int N, int k_chunks, int chunks_per_split,
+                   float* __restrict__ out, size_t split_stride, int* __restrict__ err, uint32_t wait_limit) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kMaxStages];
   __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
@@ -120,35 +107,33 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   uint8_t* tiles = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int G = gridDim.x, c = blockIdx.x;
-  const int n_tiles = N / kBM;
   if (threadIdx.x == 0) {
-    // weights do not depend on earlier kernels: pull this CTA's first tiles into
-    // L2 while the previous kernel drains (assuming a single token pass)
-    SkPlan pl{n_tiles, k_chunks, G, (long long)n_tiles * k_chunks};
-    const long long u0 = pl.start(c), u1 = pl.start(c + 1);
-    for (long long u = u0; u < u1 && u < u0 + kPrefetchChunks; ++u) {
-      const int t = (int)(u / k_chunks), kc = (int)(u % k_chunks);
+    // the weight tiles do not depend on earlier kernels: start pulling the
+    // first ones into L2 while the previous kernel drains
+    const int k0 = blockIdx.y * chunks_per_split;
+    const int k1 = min(min(k0 + chunks_per_split, k_chunks), k0 + kPrefetchChunks);
+    for (int kc = k0; kc < k1; ++kc)
       asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
                        reinterpret_cast<uint64_t>(&tmW)),
-                   "r"(kc * kBK), "r"(t * kBM)
+                   "r"(kc * kBK), "r"((int)blockIdx.x * kBM)
                    : "memory");
-    }
   }
   pdl_wait();
   pdl_trigger();
   const int M = min(*m_ptr, m_cap);
   if (M <= 0) return;
-  const int n_pass = (M + kMaxTok - 1) / kMaxTok;
-  SkPlan pl{n_tiles, k_chunks, G, (long long)n_pass * n_tiles * k_chunks};
-  const long long u_beg = pl.start(c), u_end = pl.start(c + 1);
-  if (u_beg >= u_end) return;
+  const int n0 = blockIdx.x * kBM;
+  const int kc0 = blockIdx.y * chunks_per_split;
+  const int kc1 = min(kc0 + chunks_per_split, k_chunks);
+  const int nk = kc1 - kc0;
+  if (nk <= 0) return;
   const int tok_layout = ((min(M, kMaxTok) + kBoxRows - 1) / kBoxRows) * kBoxRows;
-  // independent accumulator chains (MMAs into one accumulator serialise)
-  const int C = tok_layout <= 128 ? 4 : tok_layout <= 256 ? 2 : 1;
-  const int chain_cols = C == 1 ? 256 : tok_layout;  // column stride between chains (C > 1)
   const uint32_t stage_bytes = kWTileBytes + (uint32_t)tok_layout * 128u;
   const int n_stages = min(kMaxStages, (int)((kSmemBytes - 1024) / stage_bytes));
+  const int n_pass = (M + kMaxTok - 1) / kMaxTok;
+  // independent accumulator chains: MMAs into one accumulator serialise, so
+  // short token sets spread the K steps over 2 or 4 accumulators
+  const int C = tok_layout <= 128 ? 4 : tok_layout <= 256 ? 2 : 1;
   const uint32_t ncols = 512;
 
   if (threadIdx.x == 0) {
@@ -164,7 +149,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&drain_bar, 1);
     abort_flag = 0;
     never = 0;
-    mbar_fence_init();
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   if (warp == 1) {
     tmem_alloc(&tmem_slot, ncols);
@@ -181,13 +167,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      for (long long u = u_beg; u < u_end && !*abort;) {
-        const int t = (int)(u / k_chunks), kb = (int)(u % k_chunks);
-        const int ke = (int)min((long long)k_chunks, kb + (u_end - u));
-        const int pass = t / n_tiles, tile = t - pass * n_tiles;
-        const int row0 = pass * kMaxTok, rows = min(M - row0, kMaxTok);
+      for (int pass = 0; pass < n_pass && !*abort; ++pass) {
+        const int row0 = pass * kMaxTok;
+        const int rows = min(M - row0, kMaxTok);
         const int nbox = (rows + kBoxRows - 1) / kBoxRows;
-        for (int kc = kb; kc < ke; ++kc) {
+        for (int kc = kc0; kc < kc1; ++kc) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, wait_limit, abort)) {
             set_error(err, VLAC_ERR_TIMEOUT);
             *abort = 1;
@@ -196,7 +180,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint8_t* wt = tiles + (size_t)stage * stage_bytes;
           uint8_t* at = wt + kWTileBytes;
           mbar_expect_tx(&full_bar[stage], kWTileBytes + (uint32_t)nbox * kBoxRows * 128u);
-          tma_load_2d(wt, &tmW, kc * kBK, tile * kBM, &full_bar[stage]);
+          tma_load_2d(wt, &tmW, kc * kBK, n0, &full_bar[stage]);
+          // the token rows in as few boxes as possible: 256, 128, 64 and 32 rows
           for (int done = 0, left = nbox; left > 0;) {
             const int lg = left >= 8 ? 3 : left >= 4 ? 2 : left >= 2 ? 1 : 0;
             tma_load_2d(at + (size_t)done * kBoxRows * 128, &tmA.m[lg], kc * kBK, row0 + done * kBoxRows,
@@ -211,7 +196,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             phase ^= 1u;
           }
         }
-        u += ke - kb;
       }
     }
   } else if (warp == 1) {
@@ -219,19 +203,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      int seg = 0;
-      for (long long u = u_beg; u < u_end && !*abort; ++seg) {
-        const int t = (int)(u / k_chunks), kb = (int)(u % k_chunks);
-        const int ke = (int)min((long long)k_chunks, kb + (u_end - u));
-        const int pass = t / n_tiles;
+      for (int pass = 0; pass < n_pass && !*abort; ++pass) {
         const int rows = min(M - pass * kMaxTok, kMaxTok);
-        if (seg > 0 && !mbar_wait(&acc_empty, (uint32_t)(seg - 1) & 1u, wait_limit, abort)) {
+        if (pass > 0 && !mbar_wait(&acc_empty, (uint32_t)(pass - 1) & 1u, wait_limit, abort)) {
           set_error(err, VLAC_ERR_TIMEOUT);
           *abort = 1;
           break;
         }
         fence_after();
-        for (int kc = kb; kc < ke; ++kc) {
+        for (int i = 0; i < nk; ++i) {
           if (!mbar_wait(&full_bar[stage], phase, wait_limit, abort)) {
             set_error(err, VLAC_ERR_TIMEOUT);
             *abort = 1;
@@ -241,22 +221,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           fence_after();
           const uint32_t wt = smem_u32(tiles + (size_t)stage * stage_bytes);
           const uint32_t at = wt + kWTileBytes;
-          const bool first = kc == kb;
 #pragma unroll
           for (int k16 = 0; k16 < kBK / 16; ++k16) {
             const uint64_t adesc = sw128_desc(wt + k16 * 32);
             if (C > 1) {
-              // chain k16 % C accumulates every C-th K step of the segment
-              const int ch = k16 % C;
+              // chain k16 % C accumulates every C-th K step
               const int n = ((rows + 15) / 16) * 16;
               const uint64_t bdesc = sw128_desc(at + k16 * 32);
-              umma_bf16(tmem_base + ch * chain_cols, adesc, bdesc, idesc_bf16(n),
-                        (!first || k16 >= C) ? 1u : 0u);
+              umma_bf16(tmem_base + (k16 % C) * tok_layout, adesc, bdesc, idesc_bf16(n),
+                        (i > 0 || k16 >= C) ? 1u : 0u);
             } else {
               for (int sub = 0; sub * 256 < rows; ++sub) {
                 const int n = min(256, ((rows - sub * 256 + 15) / 16) * 16);
                 const uint64_t bdesc = sw128_desc(at + sub * 256 * 128 + k16 * 32);
-                umma_bf16(tmem_base + sub * 256, adesc, bdesc, idesc_bf16(n), (!first || k16 > 0) ? 1u : 0u);
+                umma_bf16(tmem_base + sub * 256, adesc, bdesc, idesc_bf16(n), (i > 0 || k16 > 0) ? 1u : 0u);
               }
             }
           }
@@ -267,7 +245,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         umma_commit(&acc_full);
-        u += ke - kb;
       }
       if (*abort) {
         // every MMA issued so far must finish before TMEM and the tiles go away
@@ -276,19 +253,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else {
-    // ---------------- epilogue: TMEM (+ other segments' partials) -> fp32 output ----------------
+    // ---------------- epilogue: TMEM -> fp32 partials ----------------
     const int q = warp & 3;  // TMEM lane quarter this warp may access
-    const int nl = q * 32 + lane;  // weight row within the tile
-    int seg = 0;
-    for (long long u = u_beg; u < u_end; ++seg) {
-      const int t = (int)(u / k_chunks), kb = (int)(u % k_chunks);
-      const int ke = (int)min((long long)k_chunks, kb + (u_end - u));
-      const int pass = t / n_tiles, tile = t - pass * n_tiles;
-      const int row0 = pass * kMaxTok, rows = min(M - row0, kMaxTok);
-      const long long t_beg = (long long)t * k_chunks, t_end = t_beg + k_chunks;
-      u += ke - kb;
+    const int n = n0 + q * 32 + lane;
+    float* dst = out + (size_t)blockIdx.y * split_stride;
+    for (int pass = 0; pass < n_pass; ++pass) {
+      const int row0 = pass * kMaxTok;
+      const int rows = min(M - row0, kMaxTok);
       bool ok = true;
-      if (lane == 0) ok = mbar_wait(&acc_full, (uint32_t)seg & 1u, wait_limit, abort);
+      if (lane == 0) ok = mbar_wait(&acc_full, (uint32_t)pass & 1u, wait_limit, abort);
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) {
         if (lane == 0) {
@@ -298,80 +271,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       fence_after();
-      const bool owner = kb == 0;
-      const bool complete = owner && ke == k_chunks;
-      // later segments of this tile: first segments of the CTAs starting inside it
-      int c_last = c;
-      if (owner && !complete) {
-        while (c_last + 1 < G && pl.start(c_last + 1) < t_end) ++c_last;
-        // wait for each of them (K order) before reading
-        for (int cc = c + 1; cc <= c_last; ++cc) {
-          if (pl.start(cc) >= pl.start(cc + 1)) continue;  // empty range
-          bool fine = true;
-          if (lane == 0) {
-            fine = false;
-            for (uint32_t i = 0; i < wait_limit && !*abort; ++i) {
-              int v;
-              asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(flags + cc) : "memory");
-              if (v != 0) {
-                fine = true;
-                break;
-              }
-            }
-          }
-          fine = __shfl_sync(0xffffffffu, fine, 0);
-          if (!fine) {
-            if (lane == 0) {
-              set_error(err, VLAC_ERR_TIMEOUT);
-              *abort = 1;
-            }
-            break;
-          }
-        }
-      }
-      float* slot = ws + (size_t)c * kBM * kMaxTok;  // this CTA's partial (token-major, 128 weights)
       for (int c0 = 0; c0 < rows; c0 += 16) {
         float v[16];
         tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, v);
-        if (C > 1) {
-          for (int ch = 1; ch < C; ++ch) {
-            float w[16];
-            tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ch * chain_cols + c0), w);
+        for (int ch = 1; ch < C; ++ch) {  // chains added in order
+          float w[16];
+          tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ch * tok_layout + c0), w);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) v[j] += w[j];
-          }
+          for (int j = 0; j < 16; ++j) v[j] += w[j];
         }
-        if (!owner) {
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
-            if (c0 + j < rows) slot[(size_t)(c0 + j) * kBM + nl] = v[j];
-        } else {
-          for (int cc = c + 1; cc <= c_last; ++cc) {
-            if (pl.start(cc) >= pl.start(cc + 1)) continue;
-            const float* ps = ws + (size_t)cc * kBM * kMaxTok;
-#pragma unroll
-            for (int j = 0; j < 16; ++j)
-              if (c0 + j < rows) v[j] += ps[(size_t)(c0 + j) * kBM + nl];
-          }
-#pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int m = row0 + c0 + j;
-            if (c0 + j < rows) out[(size_t)m * N + (size_t)tile * kBM + nl] = v[j];
-          }
+        for (int j = 0; j < 16; ++j) {
+          const int m = row0 + c0 + j;
+          if (m < M) dst[(size_t)m * N + n] = v[j];
         }
       }
       fence_before();
-      if (!owner) {
-        // publish the partial: all four epilogue warps' stores, then the flag
-        __threadfence();
-        asm volatile("bar.sync 2, 128;" ::: "memory");
-        if (warp == 2 && lane == 0) asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(flags + c), "r"(1) : "memory");
-      } else if (!complete) {
-        // consumed: clear the other segments' flags for the next launch
-        asm volatile("bar.sync 2, 128;" ::: "memory");
-        if (warp == 2 && lane == 0)
-          for (int cc = c + 1; cc <= c_last; ++cc) flags[cc] = 0;
-      }
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty);
     }
@@ -391,22 +306,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace tc
 
-// Stream-K: at most one CTA per SM, at least kMinUnits K chunks per CTA.
-constexpr int kMinUnits = 8;
-int gemm_tc_grid(int N, int K, int max_rows, int n_sm) {
-  const long long U = (long long)((max_rows + tc::kMaxTok - 1) / tc::kMaxTok) * (N / tc::kBM) * (K / tc::kBK);
-  return (int)std::max(1LL, std::min((long long)n_sm, (U + kMinUnits - 1) / kMinUnits));
-}
-
-void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K, int grid,
-                    float* out, float* ws, int* flags, int* err, uint32_t wait_limit, cudaStream_t st) {
+void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
+                    int splits, float* out, int* err, uint32_t wait_limit, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
     cudaFuncSetAttribute(tc::gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, tc::kSmemBytes);
     attr_set = true;
   }
-  launch_k(tc::gemm_tc_kernel, dim3(grid), dim3(tc::kThreads), tc::kSmemBytes, st, *tmA, *tmW, m_ptr, m_cap, N,
-           K / tc::kBK, out, ws, flags, err, wait_limit);
+  const int k_chunks = K / tc::kBK;
+  const int cps = (k_chunks + splits - 1) / splits;
+  dim3 grid(N / tc::kBM, splits);
+  launch_k(tc::gemm_tc_kernel, grid, dim3(tc::kThreads), tc::kSmemBytes, st, *tmA, *tmW, m_ptr, m_cap, N, k_chunks,
+           cps, out, (size_t)m_cap * N, err, wait_limit);
 }
 
 // =============================================================================

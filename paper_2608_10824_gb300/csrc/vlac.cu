@@ -2,6 +2,7 @@
 // caller-owned caches and the step of Algorithm 1.
 #include <algorithm>
 #include <cmath>
+#include <cstdio>
 #include <cstdlib>
 #include <cstring>
 #include <new>
@@ -67,8 +68,6 @@ struct vlac_ctx {
   uint8_t *mask, *full;
   int *idx, *M, *off, *emit_slot, *off_dec, *idx_dec, *err;
   float *logits_ws, *attn_part, *ssq_a, *ssq_b;
-  float* sk_ws;    // stream-K partial tiles, one per CTA
-  int* sk_flags;   // stream-K partial-ready flags, one per CTA
   // staged per-step inputs and outputs (fixed addresses, so a step can be a graph)
   uint8_t* in_frames;
   int32_t* in_prompt;
@@ -334,6 +333,40 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
       return fail(VLAC_ERR_CUDA);
   }
 
+  // ---- split-K of the prefix GEMMs: balance CTA waves (one CTA per SM)
+  // against the fp32 partial traffic of every extra split ----
+  if (c->bf16) {
+    auto pick = [&](int N, int K) {
+      const int tiles = N / 128, kch = K / 64;
+      const double chunk_us = c->rows_cap <= 128 ? 0.2 : c->rows_cap <= 256 ? 0.3 : 0.56;
+      const double slice_us = (double)c->rows_cap * N * 8.0 / 10e6;  // write + read of one fp32 slice (~10 TB/s)
+      int best = 1;
+      double best_t = 1e30;
+      for (int sp = 1; sp <= 8 && sp <= kch; ++sp) {
+        const int waves = (tiles * sp + c->n_sm - 1) / c->n_sm;
+        const double t = waves * ((kch + sp - 1) / sp) * chunk_us + (sp - 1) * slice_us;
+        if (t < best_t - 1e-9) {
+          best_t = t;
+          best = sp;
+        }
+      }
+      return best;
+    };
+    c->split_qkv = pick(3 * (int)Hd, (int)Hd);
+    c->split_o = pick((int)Hd, (int)Hd);
+    c->split_gu = pick(2 * (int)F, (int)Hd);
+    c->split_d = pick((int)Hd, (int)F);
+    if (const char* e = std::getenv("VLAC_SPLITS")) {  // "qkv,o,gu,down" override for sweeps
+      int a[4];
+      if (std::sscanf(e, "%d,%d,%d,%d", &a[0], &a[1], &a[2], &a[3]) == 4) {
+        c->split_qkv = a[0];
+        c->split_o = a[1];
+        c->split_gu = a[2];
+        c->split_d = a[3];
+      }
+    }
+  }
+
   // ---- workspace ----
   const size_t rc_ = c->rows_cap, Bm = d.max_batch;
   const size_t part_n = std::max({3 * Hd, 2 * F, (size_t)c->split_o * Hd, (size_t)c->split_d * Hd});
@@ -361,8 +394,6 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->err, 4, base);
     sc.take(c->logits_ws, Bm * (d.parallel ? d.n_action : 1) * d.n_bins * 4, base);
     sc.take(c->attn_part, Bm * d.n_heads * ((c->Tc + 31) / 32) * (d.head_dim + 2) * 4, base);
-    sc.take(c->sk_ws, c->bf16 ? (size_t)c->n_sm * 128 * 512 * 4 : 16, base);
-    sc.take(c->sk_flags, (size_t)c->n_sm * 4, base);
     sc.take(c->ssq_a, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
     sc.take(c->ssq_b, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
     const size_t fbytes = (size_t)d.n_views * d.img_h * d.img_w * 3;
@@ -544,9 +575,7 @@ void gemm(vlac_ctx* c, const ActMaps* tmA, const CUtensorMap* tmW, const T* A, c
           int N, int K, int splits, cudaStream_t st) {
   ProfScope ps(c, VLAC_PROF_PREFIX_GEMM, (double)N * K * sizeof(T), st);
   if constexpr (sizeof(T) == 2) {
-    (void)splits;
-    launch_gemm_tc(tmA, tmW, m_ptr, c->rows_cap, N, K, gemm_tc_grid(N, K, c->rows_cap, c->n_sm), c->part, c->sk_ws,
-                   c->sk_flags, c->err, c->wait_limit, st);
+    launch_gemm_tc(tmA, tmW, m_ptr, c->rows_cap, N, K, splits, c->part, c->err, c->wait_limit, st);
   } else {
     launch_gemm_simt<T>(A, static_cast<const T*>(W), m_ptr, c->rows_cap, N, K, c->part, st);
   }
