@@ -62,6 +62,7 @@ struct vlac_ctx {
   // workspace
   char* wsmem = nullptr;
   float *X, *Xd, *part;
+  size_t part_elems = 0;
   void *A, *Q, *AO, *G, *col;
   StepParams* prm;
   int3* stats;
@@ -80,6 +81,7 @@ struct vlac_ctx {
   int32_t *o_idx, *o_M;
   cudaStream_t cap_stream = nullptr;
   bool use_graph = true;
+  bool fatal = false;  // a launch was refused for exceeding a workspace buffer
   int* err_host = nullptr;  // pinned
   uint64_t launches = 0;
   uint32_t wait_limit = kDefaultWaitLimit;
@@ -369,7 +371,10 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
 
   // ---- workspace ----
   const size_t rc_ = c->rows_cap, Bm = d.max_batch;
-  const size_t part_n = std::max({3 * Hd, 2 * F, (size_t)c->split_o * Hd, (size_t)c->split_d * Hd});
+  // every GEMM writes splits x rows_cap x N fp32 partials into `part`
+  const size_t part_n = std::max({(size_t)c->split_qkv * 3 * Hd, (size_t)c->split_o * Hd, (size_t)c->split_gu * 2 * F,
+                                  (size_t)c->split_d * Hd, Hd});
+  c->part_elems = rc_ * part_n;
   Carve sc;
   auto plan_s = [&](char* base) {
     sc = Carve();
@@ -573,6 +578,10 @@ void dgemv(vlac_ctx* c, const DGemv& a_in, int epi, int nb, cudaStream_t st) {
 template <typename T>
 void gemm(vlac_ctx* c, const ActMaps* tmA, const CUtensorMap* tmW, const T* A, const void* W, const int* m_ptr,
           int N, int K, int splits, cudaStream_t st) {
+  if ((size_t)splits * c->rows_cap * N > c->part_elems) {  // never launch a GEMM whose partials do not fit
+    c->fatal = true;
+    return;
+  }
   ProfScope ps(c, VLAC_PROF_PREFIX_GEMM, (double)N * K * sizeof(T), st);
   if constexpr (sizeof(T) == 2) {
     launch_gemm_tc(tmA, tmW, m_ptr, c->rows_cap, N, K, splits, c->part, c->err, c->wait_limit, st);
@@ -780,7 +789,8 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
 }
 
 int run_body(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
-  return c->bf16 ? step_impl<bf16>(c, k, st) : step_impl<float>(c, k, st);
+  const int rc = c->bf16 ? step_impl<bf16>(c, k, st) : step_impl<float>(c, k, st);
+  return c->fatal ? VLAC_ERR_INVALID_ARG : rc;
 }
 
 // First step of a cache runs eagerly (lazy per-kernel set-up happens there);
