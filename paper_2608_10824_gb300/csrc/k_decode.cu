@@ -230,6 +230,21 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
           }
         }
       }
+      // the next GEMV's weights do not depend on anything: pull the start of
+      // the region its CTA of this index will stream into L2 now
+      if (a.pf_W && (int)blockIdx.x < a.pf_grid) {
+        const int Gn = (a.pf_pairs + kGP - 1) / kGP;
+        const long long n0 = ((long long)Gn * blockIdx.x) / a.pf_grid, n1 = ((long long)Gn * (blockIdx.x + 1)) / a.pf_grid;
+        const size_t gbytes = (size_t)TR * a.pf_K * sizeof(T);
+        const uint8_t* base = static_cast<const uint8_t*>(a.pf_W) + (size_t)n0 * gbytes;
+        size_t left = min((size_t)a.pf_bytes, (size_t)(n1 - n0) * gbytes);
+        for (size_t off = 0; left > 0;) {
+          const uint32_t piece = (uint32_t)min(left, (size_t)65536);
+          prefetch_l2(base + off, piece);
+          off += piece;
+          left -= piece;
+        }
+      }
     }
     pdl_wait();
     pdl_trigger();

@@ -338,21 +338,13 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   // ---- split-K of the prefix GEMMs: balance CTA waves (one CTA per SM)
   // against the fp32 partial traffic of every extra split ----
   if (c->bf16) {
+    // Every CTA re-reads the whole activation tile from L2, so extra splits of
+    // the wide projections cost more than their better wave fill gains; only
+    // the narrow ones (fewer tiles than half the SMs) are split.
     auto pick = [&](int N, int K) {
       const int tiles = N / 128, kch = K / 64;
-      const double chunk_us = c->rows_cap <= 128 ? 0.2 : c->rows_cap <= 256 ? 0.3 : 0.56;
-      const double slice_us = (double)c->rows_cap * N * 8.0 / 10e6;  // write + read of one fp32 slice (~10 TB/s)
-      int best = 1;
-      double best_t = 1e30;
-      for (int sp = 1; sp <= 8 && sp <= kch; ++sp) {
-        const int waves = (tiles * sp + c->n_sm - 1) / c->n_sm;
-        const double t = waves * ((kch + sp - 1) / sp) * chunk_us + (sp - 1) * slice_us;
-        if (t < best_t - 1e-9) {
-          best_t = t;
-          best = sp;
-        }
-      }
-      return best;
+      if (2 * tiles > c->n_sm) return 1;
+      return std::max(1, std::min({8, kch, c->n_sm / tiles}));
     };
     c->split_qkv = pick(3 * (int)Hd, (int)Hd);
     c->split_o = pick((int)Hd, (int)Hd);
@@ -702,6 +694,14 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
                                c->idx_dec, c->ssq_b, c->err, st);
       }
       c->launches += 1;
+      // prefetch chain: each GEMV pulls the start of the next one's weights into L2
+      auto set_pf = [&](DGemv& g, const void* Wn, int Kn, int pairs) {
+        g.pf_W = Wn;
+        g.pf_K = Kn;
+        g.pf_pairs = pairs;
+        g.pf_grid = dgemv_grid(pairs, c->n_sm);
+        g.pf_bytes = 128 * 1024;
+      };
       for (int l = 0; l < L; ++l) {
         DGemv g{};
         g.eps = eps;
@@ -724,6 +724,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         g.ssq_in = c->ssq_b;
         g.n_ssq = l == 0 ? Hd / kDecodeRowsPerCta : dgemv_grid(Hd / 2, c->n_sm);  // embedding or down-projection
         g.err = c->err;
+        set_pf(g, c->dwo[l], Hd, Hd / 2);
         dgemv<T>(c, g, kEpiQkvRope, B, st);
         {
           ProfScope ps_(c, VLAC_PROF_DECODE_ATTN, 0, st);
@@ -741,6 +742,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         o.n_out = Hd;
         o.ssq_out = c->ssq_a;
         o.err = c->err;
+        set_pf(o, c->dgu[l], Hd, F);
         dgemv<T>(c, o, kEpiResid, B, st);
         // gate/up with the MLP RMSNorm prologue and SwiGLU
         DGemv u{};
@@ -755,6 +757,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         u.ssq_in = c->ssq_a;
         u.n_ssq = dgemv_grid(Hd / 2, c->n_sm);  // o-projection
         u.err = c->err;
+        set_pf(u, c->dwd[l], F, Hd / 2);
         dgemv<T>(c, u, kEpiSwiglu, B, st);
         // down-projection + residual
         DGemv dn{};
@@ -766,6 +769,8 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         dn.n_out = Hd;
         dn.ssq_out = c->ssq_b;
         dn.err = c->err;
+        if (l + 1 < L) set_pf(dn, c->dqkv[l + 1], Hd, 3 * Hd / 2);
+        else if (a + 1 < D) set_pf(dn, c->dqkv[0], Hd, 3 * Hd / 2);
         dgemv<T>(c, dn, kEpiResid, B, st);
       }
       {
