@@ -344,7 +344,9 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     auto pick = [&](int N, int K) {
       const int tiles = N / 128, kch = K / 64;
       if (2 * tiles > c->n_sm) return 1;
-      return std::max(1, std::min({8, kch, c->n_sm / tiles}));
+      const int sp = std::max(1, std::min({8, kch, c->n_sm / tiles}));
+      const int cps = (kch + sp - 1) / sp;  // chunks per split; every split must get some
+      return (kch + cps - 1) / cps;
     };
     c->split_qkv = pick(3 * (int)Hd, (int)Hd);
     c->split_o = pick((int)Hd, (int)Hd);
@@ -570,7 +572,9 @@ void dgemv(vlac_ctx* c, const DGemv& a_in, int epi, int nb, cudaStream_t st) {
 template <typename T>
 void gemm(vlac_ctx* c, const ActMaps* tmA, const CUtensorMap* tmW, const T* A, const void* W, const int* m_ptr,
           int N, int K, int splits, cudaStream_t st) {
-  if ((size_t)splits * c->rows_cap * N > c->part_elems) {  // never launch a GEMM whose partials do not fit
+  const int kch = c->bf16 ? K / 64 : 1, cps = (kch + splits - 1) / splits;
+  if ((size_t)splits * c->rows_cap * N > c->part_elems ||  // never launch a GEMM whose partials do not fit,
+      (splits - 1) * cps >= kch) {                          // or one with a split that has no K range
     c->fatal = true;
     return;
   }
