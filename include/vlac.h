@@ -186,6 +186,33 @@ int vlac_selftest_wait(vlac_ctx* ctx, uint32_t spin_limit);
 int vlac_prof_enable(vlac_ctx* ctx, int on);
 int vlac_prof_read(vlac_ctx* ctx, int kind, double* total_ms, uint64_t* launches, double* bytes);
 
+/* Allocation-free selection step.  The paper has no counterpart of this call:
+ * it exists for callers that cannot allocate device memory when they run it
+ * -- code inside a CUDA stream capture, real-time control loops whose memory
+ * is fixed up front, host frameworks that own every device allocation.  It
+ * runs the same kernels as vlac_step's selection (Stage-1 exact patch
+ * similarity, the gate on m_prev < tau_margin or gate_override, the Stage-3
+ * recompute order) without a context and without allocating: its scratch is
+ * one fixed 256 KiB device array inside the library, which every call on a
+ * device shares and which keeps the last call's contents.  Calls whose GPU
+ * work overlaps (other streams, other host threads) therefore race; order
+ * them on one stream.  The first call on each device looks up that array's
+ * device address (make it before any stream capture).
+ *   d:              host; geometry as for vlac_create (d->max_batch bounds batch)
+ *   frames, prev_frames: device [batch][n_views][img_h][img_w][3] uint8
+ *   valid:          device [batch] uint8, 0 = no previous frame (full branch)
+ *   m_prev:         device [batch] fp32, the previous step's m_{t-1}
+ *   reuse_permille: host [n_layers], each <= 1000
+ *   gate_override:  device [batch] int8 (-1 gate, 0 cached, 1 full) or NULL
+ *   outputs (device): static_mask [batch][Nv], idx [batch][S], M [batch][n_layers],
+ *                     recomputed [batch]
+ * Returns VLAC_ERR_INVALID_ARG for bad arguments and when the call needs more
+ * than the fixed scratch: batch x visual patches must stay within 20,000. */
+int vlac_select_noalloc(const vlac_dims* d, int batch, const uint8_t* frames, const uint8_t* prev_frames,
+                        const uint8_t* valid, const float* m_prev, vlac_rational tau_sim, float tau_margin,
+                        const uint16_t* reuse_permille, const int8_t* gate_override, uint8_t* static_mask,
+                        int32_t* idx, int32_t* M, uint8_t* recomputed, void* stream);
+
 const char* vlac_strerror(int code);
 
 #ifdef __cplusplus

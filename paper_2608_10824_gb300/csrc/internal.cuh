@@ -197,6 +197,8 @@ inline void launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sme
 // ---- launchers (defined in the kernel translation units) -------------------
 namespace vlac {
 
+int check_dims(const vlac_dims* d);  // VLAC_OK or the error vlac_create would return
+
 void launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid,
                         const StepParams* prm, int B, int n_views, int img_h, int img_w, int patch,
                         int3* stats, uint8_t* mask, uint8_t* user_mask, cudaStream_t st);

@@ -120,7 +120,7 @@ struct vlac_cache {
 
 // ---- dims ------------------------------------------------------------------
 
-static int check_dims(const vlac_dims* d) {
+int vlac::check_dims(const vlac_dims* d) {
   if (!d) return VLAC_ERR_INVALID_ARG;
   if (d->n_layers < 1 || d->n_layers > kMaxLayers || d->n_heads < 1 || d->n_heads * d->head_dim != d->hidden ||
       d->ffn < 1 || d->vocab < 1 || d->n_bins < 2 || d->n_bins > d->vocab || d->n_bins > 4096 || d->patch < 1 ||

@@ -67,7 +67,7 @@ class StepOut(C.Structure):
 
 EXPORTS = ["vlac_create", "vlac_destroy", "vlac_cache_bytes", "vlac_cache_init", "vlac_cache_destroy",
            "vlac_step", "vlac_reset", "vlac_sync_error", "vlac_launch_count", "vlac_selftest_wait",
-           "vlac_prof_enable", "vlac_prof_read", "vlac_strerror"]
+           "vlac_prof_enable", "vlac_prof_read", "vlac_select_noalloc", "vlac_strerror"]
 
 
 def lib():
@@ -94,6 +94,8 @@ def lib():
             L.vlac_prof_enable.argtypes = [vp, i32]
             L.vlac_prof_read.argtypes = [vp, i32, C.POINTER(C.c_double), C.POINTER(C.c_uint64),
                                          C.POINTER(C.c_double)]
+            L.vlac_select_noalloc.argtypes = [C.POINTER(Dims), i32, vp, vp, vp, vp, Rational, C.c_float, vp, vp,
+                                              vp, vp, vp, vp, vp]
             L.vlac_strerror.argtypes = [i32]
             L.vlac_strerror.restype = C.c_char_p
             for name in EXPORTS:
@@ -227,6 +229,33 @@ class Context:
 
     def selftest_wait(self, spin_limit: int) -> int:
         return lib().vlac_selftest_wait(self._h, spin_limit)
+
+
+def select_noalloc(d, frames, prev_frames, valid, m_prev, tau_sim=(996, 1000), tau_margin: float = 0.0,
+                   permille=None, gate_override=None, out: Optional[Dict] = None, max_batch: Optional[int] = None,
+                   stream=None) -> Dict:
+    """Selection step without allocating device memory (see vlac_select_noalloc
+    in include/vlac.h).  Inputs are CUDA tensors; `out` may hold preallocated
+    outputs (static_mask, idx, M, recomputed), which this call then fills."""
+    import torch
+    B = frames.shape[0]
+    if permille is None:
+        permille = np.full(d.n_layers, 1000, dtype=np.uint16)
+    permille = np.ascontiguousarray(permille, dtype=np.uint16)
+    if out is None:
+        dev = frames.device
+        out = {"static_mask": torch.zeros((B, d.n_visual), dtype=torch.uint8, device=dev),
+               "idx": torch.zeros((B, d.pass_len), dtype=torch.int32, device=dev),
+               "M": torch.zeros((B, d.n_layers), dtype=torch.int32, device=dev),
+               "recomputed": torch.zeros((B,), dtype=torch.uint8, device=dev)}
+    dims = c_dims(d, max_batch if max_batch is not None else max(B, d.max_batch))
+    rc = lib().vlac_select_noalloc(C.byref(dims), B, frames.data_ptr(), prev_frames.data_ptr(), valid.data_ptr(),
+                                   m_prev.data_ptr(), Rational(int(tau_sim[0]), int(tau_sim[1])),
+                                   float(tau_margin), permille.ctypes.data, _ptr(gate_override),
+                                   out["static_mask"].data_ptr(), out["idx"].data_ptr(), out["M"].data_ptr(),
+                                   out["recomputed"].data_ptr(), _stream_ptr(stream))
+    _check(rc, "vlac_select_noalloc")
+    return out
 
 
 class Cache:
