@@ -116,11 +116,256 @@ __global__ void __launch_bounds__(256) attn_kernel(Rows rows, int n_heads, const
   }
 }
 
+// ---- bf16 path: tensor cores (mma.m16n8k16), flash-attention style ----------------
+//
+// One block of 4 warps per (64 query rows of one sequence, head); warp w owns
+// 16 rows.  Key tiles of 64 positions (aligned to absolute positions) are
+// double-buffered in shared memory by cp.async.  Per tile: S = Q K^T on the
+// tensor cores (fp32 accumulators), scale, causal mask by the row's absolute
+// position, online softmax in fp32, P rounded to bf16 and O += P V on the
+// tensor cores.  Masked keys contribute exact zeros and a fully masked tile
+// leaves a row's state unchanged, so a row's result does not depend on the
+// other rows of its block.
+namespace {
+
+constexpr int kAQ = 64;   // query rows per block
+constexpr int kAK = 64;   // keys per tile
+constexpr int kAW = 4;    // warps per block
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16(float* d, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+// 16 bytes global -> shared, zero-filled when !valid
+__device__ __forceinline__ void cp16(uint32_t dst, const void* src, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0) : "memory");
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+template <int HD>
+__global__ void __launch_bounds__(kAW * 32) attn_mma_kernel(Rows rows, int n_heads, const bf16* __restrict__ Q,
+                                                            const bf16* __restrict__ Kc, const bf16* __restrict__ Vc,
+                                                            size_t kv_seq_stride, int Tc, int P, int parallel,
+                                                            int n_action, float scale, bf16* __restrict__ O) {
+  pdl_wait();
+  pdl_trigger();
+  constexpr int LD = HD + 8;        // padded row (elements): conflict-free ldmatrix
+  constexpr int KS = HD / 16;       // k-steps of S = Q K^T
+  constexpr int ND = HD / 8;        // 8-column tiles of O
+  constexpr int CH = HD * 2 / 16;   // 16-byte chunks per key row
+  extern __shared__ __align__(16) uint8_t dsm[];
+  bf16* Ks = reinterpret_cast<bf16*>(dsm);             // [2][kAK][LD]
+  bf16* Vs = Ks + 2 * kAK * LD;                        // [2][kAK][LD]
+  __shared__ int lim_s[kAQ];
+  __shared__ int maxlim_s;
+  const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int cnt = rows.off[b + 1] - rows.off[b];
+  const int i0 = qt * kAQ;
+  if (i0 >= cnt) return;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t = lane & 3;
+  const int hidden = n_heads * HD, r0 = rows.off[b] + i0;
+  if (tid < kAQ) {
+    int lim = 0;
+    if (i0 + tid < cnt) {
+      const int pos = rows.idx[(size_t)b * rows.idx_stride + i0 + tid];
+      lim = (parallel && pos >= P) ? P + n_action : pos + 1;
+      lim = min(lim, Tc);
+    }
+    lim_s[tid] = lim;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int m = 0;
+    for (int q = 0; q < kAQ; ++q) m = max(m, lim_s[q]);
+    maxlim_s = m;
+  }
+  const bf16* Kh = Kc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
+  const bf16* Vh = Vc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
+  const uint32_t ks_base = smem_u32(Ks), vs_base = smem_u32(Vs);
+  auto load_tile = [&](int tile, int buf) {
+    const int t0 = tile * kAK;
+    for (int c = tid; c < kAK * CH; c += kAW * 32) {
+      const int j = c / CH, q = c - j * CH, key = t0 + j;
+      const bool ok = key < Tc;
+      const size_t off = (size_t)(ok ? key : 0) * HD + q * 8;
+      const uint32_t so = (uint32_t)(((buf * kAK + j) * LD + q * 8) * 2);
+      cp16(ks_base + so, Kh + off, ok);
+      cp16(vs_base + so, Vh + off, ok);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  load_tile(0, 0);
+  // this warp's Q rows as A fragments (rows past the block's rows are zero)
+  const int ra = warp * 16 + g, rb = ra + 8;  // rows of the block held by this thread
+  uint32_t qa[KS][4];
+  {
+    const bool va = i0 + ra < cnt, vb = i0 + rb < cnt;
+    const bf16* qpa = Q + (size_t)(r0 + (va ? ra : 0)) * hidden + (size_t)h * HD;
+    const bf16* qpb = Q + (size_t)(r0 + (vb ? rb : 0)) * hidden + (size_t)h * HD;
+#pragma unroll
+    for (int ks = 0; ks < KS; ++ks) {
+      const int e = 16 * ks + 2 * t;
+      qa[ks][0] = va ? *reinterpret_cast<const uint32_t*>(qpa + e) : 0u;
+      qa[ks][1] = vb ? *reinterpret_cast<const uint32_t*>(qpb + e) : 0u;
+      qa[ks][2] = va ? *reinterpret_cast<const uint32_t*>(qpa + e + 8) : 0u;
+      qa[ks][3] = vb ? *reinterpret_cast<const uint32_t*>(qpb + e + 8) : 0u;
+    }
+  }
+  __syncthreads();
+  const int lim_a = lim_s[ra], lim_b = lim_s[rb];
+  const int n_tiles = (maxlim_s + kAK - 1) / kAK;
+  float o[ND][4];
+#pragma unroll
+  for (int nd = 0; nd < ND; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
+  float m_a = -INFINITY, m_b = -INFINITY, l_a = 0.f, l_b = 0.f;  // per-thread partial row sums
+  for (int tile = 0; tile < n_tiles; ++tile) {
+    const int buf = tile & 1;
+    if (tile + 1 < n_tiles) {
+      load_tile(tile + 1, buf ^ 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+    }
+    __syncthreads();
+    // S = Q K^T for 64 keys: 8 n-tiles of 8 keys
+    float sc[8][4];
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < KS; ++ks) {
+#pragma unroll
+      for (int np = 0; np < 4; ++np) {  // n-tiles 2np, 2np + 1
+        // matrices: (keys 16np + 0..7, dims 16ks), (same keys, dims 16ks + 8), next 8 keys likewise
+        const int mi = lane >> 3, rr = lane & 7;
+        const int key = 16 * np + (mi >> 1) * 8 + rr, dim = 16 * ks + (mi & 1) * 8;
+        uint32_t k0, k1, k2, k3;
+        ldsm_x4(ks_base + (uint32_t)(((buf * kAK + key) * LD + dim) * 2), k0, k1, k2, k3);
+        mma_bf16(sc[2 * np], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], k0, k1);
+        mma_bf16(sc[2 * np + 1], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], k2, k3);
+      }
+    }
+    // scale, mask, online softmax (rows ra: elements 0, 1; rb: elements 2, 3)
+    const int t0 = tile * kAK;
+    float mx_a = m_a, mx_b = m_b;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      const int key = t0 + nt * 8 + 2 * t;
+      sc[nt][0] = key < lim_a ? sc[nt][0] * scale : -INFINITY;
+      sc[nt][1] = key + 1 < lim_a ? sc[nt][1] * scale : -INFINITY;
+      sc[nt][2] = key < lim_b ? sc[nt][2] * scale : -INFINITY;
+      sc[nt][3] = key + 1 < lim_b ? sc[nt][3] * scale : -INFINITY;
+      mx_a = fmaxf(mx_a, fmaxf(sc[nt][0], sc[nt][1]));
+      mx_b = fmaxf(mx_b, fmaxf(sc[nt][2], sc[nt][3]));
+    }
+    mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 1));
+    mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 2));
+    mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 1));
+    mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 2));
+    const float base_a = mx_a == -INFINITY ? 0.f : mx_a, base_b = mx_b == -INFINITY ? 0.f : mx_b;
+    const float corr_a = m_a == -INFINITY ? 0.f : expf(m_a - base_a);
+    const float corr_b = m_b == -INFINITY ? 0.f : expf(m_b - base_b);
+    m_a = mx_a;
+    m_b = mx_b;
+    l_a *= corr_a;
+    l_b *= corr_b;
+#pragma unroll
+    for (int nd = 0; nd < ND; ++nd) {
+      o[nd][0] *= corr_a;
+      o[nd][1] *= corr_a;
+      o[nd][2] *= corr_b;
+      o[nd][3] *= corr_b;
+    }
+    uint32_t pa[4][4];  // P as A fragments of the 4 key k-steps
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      const float p0 = expf(sc[nt][0] - base_a), p1 = expf(sc[nt][1] - base_a);
+      const float p2 = expf(sc[nt][2] - base_b), p3 = expf(sc[nt][3] - base_b);
+      l_a += p0 + p1;
+      l_b += p2 + p3;
+      pa[nt >> 1][(nt & 1) * 2 + 0] = pack_bf16(p0, p1);
+      pa[nt >> 1][(nt & 1) * 2 + 1] = pack_bf16(p2, p3);
+    }
+    // O += P V: k-steps of 16 keys, 8-column tiles of V (transposed loads)
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+#pragma unroll
+      for (int np = 0; np < ND / 2; ++np) {  // column tiles 2np, 2np + 1
+        const int mi = lane >> 3, rr = lane & 7;
+        const int key = 16 * kk + (mi & 1) * 8 + rr, dim = 16 * np + (mi >> 1) * 8;
+        uint32_t v0, v1, v2, v3;
+        ldsm_x4_t(vs_base + (uint32_t)(((buf * kAK + key) * LD + dim) * 2), v0, v1, v2, v3);
+        mma_bf16(o[2 * np], pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3], v0, v1);
+        mma_bf16(o[2 * np + 1], pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3], v2, v3);
+      }
+    }
+    __syncthreads();  // the buffer is refilled next
+  }
+  // full row sums over the quad, then O / l
+  l_a += __shfl_xor_sync(0xffffffffu, l_a, 1);
+  l_a += __shfl_xor_sync(0xffffffffu, l_a, 2);
+  l_b += __shfl_xor_sync(0xffffffffu, l_b, 1);
+  l_b += __shfl_xor_sync(0xffffffffu, l_b, 2);
+  const float ia = l_a > 0.f ? 1.0f / l_a : 0.f, ib = l_b > 0.f ? 1.0f / l_b : 0.f;
+  if (i0 + ra < cnt) {
+    bf16* op = O + (size_t)(r0 + ra) * hidden + (size_t)h * HD;
+#pragma unroll
+    for (int nd = 0; nd < ND; ++nd)
+      *reinterpret_cast<uint32_t*>(op + nd * 8 + 2 * t) = pack_bf16(o[nd][0] * ia, o[nd][1] * ia);
+  }
+  if (i0 + rb < cnt) {
+    bf16* op = O + (size_t)(r0 + rb) * hidden + (size_t)h * HD;
+#pragma unroll
+    for (int nd = 0; nd < ND; ++nd)
+      *reinterpret_cast<uint32_t*>(op + nd * 8 + 2 * t) = pack_bf16(o[nd][2] * ib, o[nd][3] * ib);
+  }
+}
+
+template <int HD>
+void attn_mma_launch(Rows rows, int B, int S, int n_heads, const bf16* Q, const bf16* Kc, const bf16* Vc,
+                     size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, float scale, bf16* O,
+                     cudaStream_t st) {
+  const size_t smem = (size_t)4 * kAK * (HD + 8) * sizeof(bf16);
+  static bool smem_set = false;  // raised once, before any graph capture of the kernel
+  if (!smem_set) {
+    cudaFuncSetAttribute(attn_mma_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    smem_set = true;
+  }
+  const dim3 grid((S + kAQ - 1) / kAQ, n_heads, B);
+  launch_k(attn_mma_kernel<HD>, grid, dim3(kAW * 32), smem, st, rows, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, P,
+           parallel, n_action, scale, O);
+}
+
+}  // namespace
+
 template <typename T>
 void launch_attention(Rows rows, int B, int S, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc,
                       size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, T* O, cudaStream_t st) {
-  dim3 grid((S + 15) / 16, n_heads, B);
   const float scale = 1.0f / sqrtf((float)head_dim);
+  if constexpr (sizeof(T) == 2) {
+    if (head_dim == 128)
+      attn_mma_launch<128>(rows, B, S, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, P, parallel, n_action, scale, O, st);
+    else
+      attn_mma_launch<64>(rows, B, S, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, P, parallel, n_action, scale, O, st);
+    return;
+  }
+  dim3 grid((S + 15) / 16, n_heads, B);
   if (head_dim == 128)
     launch_k(attn_kernel<T, 128>, grid, dim3(256), 0, st, rows, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, P, parallel,
              n_action, scale, O);
