@@ -83,17 +83,49 @@ __global__ void embed_kernel(Rows rows, int hidden, int Nv, int P, int has_propr
   }
 }
 
+// ---- vector helpers (4 consecutive elements; row lengths are multiples of 4) ----
+
+template <typename T> __device__ __forceinline__ float4 load4(const T* p);
+template <> __device__ __forceinline__ float4 load4<float>(const float* p) { return *reinterpret_cast<const float4*>(p); }
+template <> __device__ __forceinline__ float4 load4<bf16>(const bf16* p) {
+  const uint2 w = *reinterpret_cast<const uint2*>(p);
+  return make_float4(__uint_as_float(w.x << 16), __uint_as_float(w.x & 0xFFFF0000u), __uint_as_float(w.y << 16),
+                     __uint_as_float(w.y & 0xFFFF0000u));
+}
+template <typename T> __device__ __forceinline__ void store4(T* p, float4 v);
+template <> __device__ __forceinline__ void store4<float>(float* p, float4 v) { *reinterpret_cast<float4*>(p) = v; }
+template <> __device__ __forceinline__ void store4<bf16>(bf16* p, float4 v) {
+  const __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
+  *reinterpret_cast<uint2*>(p) =
+      make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+}
+__device__ __forceinline__ float4 add4(float4 a, float4 b) {
+  return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+}
+__device__ __forceinline__ float sq4(float4 a, float acc) {
+  return fmaf(a.w, a.w, fmaf(a.z, a.z, fmaf(a.y, a.y, fmaf(a.x, a.x, acc))));
+}
+// Sum over the GEMM's K splits (split s at part + s * stride), in split order.
+__device__ __forceinline__ float4 sum_splits4(const float* __restrict__ part, int splits, size_t stride, size_t o) {
+  float4 v = *reinterpret_cast<const float4*>(part + o);
+  for (int s = 1; s < splits; ++s) v = add4(v, *reinterpret_cast<const float4*>(part + o + (size_t)s * stride));
+  return v;
+}
+
 // ---- RMSNorm ----------------------------------------------------------------
 
-// y = T((x * r) * g), r = 1 / sqrt(mean(x^2) + eps).  One block per row.
+// y = T((x * r) * g), r = 1 / sqrt(mean(x^2) + eps); `ss` is this thread's part
+// of sum(x^2).  One block per row.
 template <typename T>
-__device__ __forceinline__ void rmsnorm_row(const float* __restrict__ x, const T* __restrict__ g, int hidden,
+__device__ __forceinline__ void rmsnorm_row(const float* __restrict__ x, float ss, const T* __restrict__ g, int hidden,
                                             float eps, T* __restrict__ y, float* red) {
-  float ss = 0.f;
-  for (int k = threadIdx.x; k < hidden; k += blockDim.x) ss = fmaf(x[k], x[k], ss);
   ss = block_sum(ss, red);
   const float r = 1.0f / sqrtf(ss / (float)hidden + eps);
-  for (int k = threadIdx.x; k < hidden; k += blockDim.x) y[k] = from_f<T>((x[k] * r) * to_f(g[k]));
+#pragma unroll 4
+  for (int c = threadIdx.x; c < hidden / 4; c += blockDim.x) {
+    const float4 xv = reinterpret_cast<const float4*>(x)[c], gv = load4<T>(g + 4 * c);
+    store4<T>(y + 4 * c, make_float4((xv.x * r) * gv.x, (xv.y * r) * gv.y, (xv.z * r) * gv.z, (xv.w * r) * gv.w));
+  }
 }
 
 // Layer input: rows computed at the previous layer record their layer-l input
@@ -111,28 +143,31 @@ __global__ void layer_in_kernel(Rows rows, const int* __restrict__ off_prev, int
   if (i >= cnt && (H == nullptr || i >= cnt_prev)) return;
   const int pos = rows.idx[(size_t)b * rows.idx_stride + i];
   float* x = rows.X + ((size_t)b * rows.idx_stride + i) * hidden;
+  float ss = 0.f;
   if (H) {
     float* h = H + (size_t)b * h_seq_stride + (size_t)pos * hidden;
     const float4* s4 = reinterpret_cast<const float4*>(i < cnt_prev ? x : h);
     float4* d4 = reinterpret_cast<float4*>(i < cnt_prev ? h : x);
-    for (int k = threadIdx.x; k < hidden / 4; k += blockDim.x) d4[k] = s4[k];
-    __syncthreads();
+#pragma unroll 4
+    for (int k = threadIdx.x; k < hidden / 4; k += blockDim.x) {
+      const float4 v = s4[k];
+      d4[k] = v;
+      ss = sq4(v, ss);
+    }
+  } else {
+#pragma unroll 4
+    for (int k = threadIdx.x; k < hidden / 4; k += blockDim.x) ss = sq4(reinterpret_cast<const float4*>(x)[k], ss);
   }
   if (i >= cnt) return;
-  rmsnorm_row<T>(x, gain, hidden, eps, A + (size_t)(rows.off[b] + i) * hidden, red);
+  rmsnorm_row<T>(x, ss, gain, hidden, eps, A + (size_t)(rows.off[b] + i) * hidden, red);
 }
 
 // ---- GEMM epilogues ------------------------------------------------------------
 
-__device__ __forceinline__ float sum_splits(const float* __restrict__ part, int splits, size_t stride, size_t o) {
-  float v = part[o];
-  for (int s = 1; s < splits; ++s) v += part[o + (size_t)s * stride];
-  return v;
-}
-
 // q, k, v from the fused projection [q | k | v]; RoPE (rotate-half) on q and k
 // at the row's absolute position; Q to its row, K and V scattered into the
-// cache at that position (layout [b][head][position][head_dim]).
+// cache at that position (layout [b][head][position][head_dim]).  A thread
+// takes four consecutive e of one head and their partners e + half.
 template <typename T>
 __global__ void qkv_epilogue_kernel(Rows rows, int n_heads, int head_dim, const float* __restrict__ part,
                                     int splits, size_t split_stride, const float* __restrict__ rope_cos,
@@ -145,26 +180,31 @@ __global__ void qkv_epilogue_kernel(Rows rows, int n_heads, int head_dim, const 
   if (i >= cnt) return;
   const int r = rows.off[b] + i;
   const int pos = rows.idx[(size_t)b * rows.idx_stride + i];
-  const int hidden = n_heads * head_dim, half = head_dim / 2, N = 3 * hidden;
+  const int hidden = n_heads * head_dim, half = head_dim / 2, N = 3 * hidden, q4 = half / 4;
   const float* pr = part + (size_t)r * N;
   T* q_out = Q + (size_t)r * hidden;
-  for (int t = threadIdx.x; t < n_heads * half; t += blockDim.x) {
-    const int h = t / half, e = t - h * half;
-    const float c = rope_cos[(size_t)pos * half + e], s = rope_sin[(size_t)pos * half + e];
+  for (int t = threadIdx.x; t < n_heads * q4; t += blockDim.x) {
+    const int h = t / q4, e = 4 * (t - h * q4);
+    const float4 c = *reinterpret_cast<const float4*>(rope_cos + (size_t)pos * half + e);
+    const float4 s = *reinterpret_cast<const float4*>(rope_sin + (size_t)pos * half + e);
     const size_t base = (size_t)h * head_dim + e;
-    const float q1 = sum_splits(pr, splits, split_stride, base);
-    const float q2 = sum_splits(pr, splits, split_stride, base + half);
-    const float k1 = sum_splits(pr, splits, split_stride, hidden + base);
-    const float k2 = sum_splits(pr, splits, split_stride, hidden + base + half);
-    const float v1 = sum_splits(pr, splits, split_stride, 2 * hidden + base);
-    const float v2 = sum_splits(pr, splits, split_stride, 2 * hidden + base + half);
-    q_out[base] = from_f<T>(q1 * c - q2 * s);
-    q_out[base + half] = from_f<T>(q2 * c + q1 * s);
+    const float4 q1 = sum_splits4(pr, splits, split_stride, base);
+    const float4 q2 = sum_splits4(pr, splits, split_stride, base + half);
+    const float4 k1 = sum_splits4(pr, splits, split_stride, hidden + base);
+    const float4 k2 = sum_splits4(pr, splits, split_stride, hidden + base + half);
+    const float4 v1 = sum_splits4(pr, splits, split_stride, 2 * hidden + base);
+    const float4 v2 = sum_splits4(pr, splits, split_stride, 2 * hidden + base + half);
+    store4<T>(q_out + base, make_float4(q1.x * c.x - q2.x * s.x, q1.y * c.y - q2.y * s.y, q1.z * c.z - q2.z * s.z,
+                                        q1.w * c.w - q2.w * s.w));
+    store4<T>(q_out + base + half, make_float4(q2.x * c.x + q1.x * s.x, q2.y * c.y + q1.y * s.y,
+                                               q2.z * c.z + q1.z * s.z, q2.w * c.w + q1.w * s.w));
     const size_t kv = (size_t)b * kv_seq_stride + ((size_t)h * Tc + pos) * head_dim + e;
-    Kc[kv] = from_f<T>(k1 * c - k2 * s);
-    Kc[kv + half] = from_f<T>(k2 * c + k1 * s);
-    Vc[kv] = from_f<T>(v1);
-    Vc[kv + half] = from_f<T>(v2);
+    store4<T>(Kc + kv, make_float4(k1.x * c.x - k2.x * s.x, k1.y * c.y - k2.y * s.y, k1.z * c.z - k2.z * s.z,
+                                   k1.w * c.w - k2.w * s.w));
+    store4<T>(Kc + kv + half, make_float4(k2.x * c.x + k1.x * s.x, k2.y * c.y + k1.y * s.y, k2.z * c.z + k1.z * s.z,
+                                          k2.w * c.w + k1.w * s.w));
+    store4<T>(Vc + kv, v1);
+    store4<T>(Vc + kv + half, v2);
   }
 }
 
@@ -181,9 +221,14 @@ __global__ void residual_norm_kernel(Rows rows, int hidden, const float* __restr
   const int r = rows.off[b] + i;
   float* x = rows.X + ((size_t)b * rows.idx_stride + i) * hidden;
   const float* pr = part + (size_t)r * hidden;
-  for (int k = threadIdx.x; k < hidden; k += blockDim.x) x[k] = x[k] + sum_splits(pr, splits, split_stride, k);
-  __syncthreads();
-  rmsnorm_row<T>(x, gain, hidden, eps, A + (size_t)r * hidden, red);
+  float ss = 0.f;
+#pragma unroll 4
+  for (int c = threadIdx.x; c < hidden / 4; c += blockDim.x) {
+    const float4 v = add4(reinterpret_cast<const float4*>(x)[c], sum_splits4(pr, splits, split_stride, 4 * (size_t)c));
+    reinterpret_cast<float4*>(x)[c] = v;
+    ss = sq4(v, ss);
+  }
+  rmsnorm_row<T>(x, ss, gain, hidden, eps, A + (size_t)r * hidden, red);
 }
 
 // G = T(silu(g) * u) from the fused projection [gate | up].
@@ -197,10 +242,13 @@ __global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part
   if (i >= cnt) return;
   const int r = rows.off[b] + i;
   const float* pr = part + (size_t)r * 2 * ffn;
-  for (int j = threadIdx.x; j < ffn; j += blockDim.x) {
-    const float g = sum_splits(pr, splits, split_stride, j);
-    const float u = sum_splits(pr, splits, split_stride, (size_t)ffn + j);
-    G[(size_t)r * ffn + j] = from_f<T>((g / (1.0f + expf(-g))) * u);
+#pragma unroll 4
+  for (int c = threadIdx.x; c < ffn / 4; c += blockDim.x) {
+    const float4 g = sum_splits4(pr, splits, split_stride, 4 * (size_t)c);
+    const float4 u = sum_splits4(pr, splits, split_stride, (size_t)ffn + 4 * c);
+    store4<T>(G + (size_t)r * ffn + 4 * c,
+              make_float4((g.x / (1.0f + expf(-g.x))) * u.x, (g.y / (1.0f + expf(-g.y))) * u.y,
+                          (g.z / (1.0f + expf(-g.z))) * u.z, (g.w / (1.0f + expf(-g.w))) * u.w));
   }
 }
 
@@ -215,7 +263,10 @@ __global__ void residual_kernel(Rows rows, int hidden, const float* __restrict__
   const int r = rows.off[b] + i;
   float* x = rows.X + ((size_t)b * rows.idx_stride + i) * hidden;
   const float* pr = part + (size_t)r * hidden;
-  for (int k = threadIdx.x; k < hidden; k += blockDim.x) x[k] = x[k] + sum_splits(pr, splits, split_stride, k);
+#pragma unroll 4
+  for (int c = threadIdx.x; c < hidden / 4; c += blockDim.x)
+    reinterpret_cast<float4*>(x)[c] =
+        add4(reinterpret_cast<const float4*>(x)[c], sum_splits4(pr, splits, split_stride, 4 * (size_t)c));
 }
 
 // Autoregressive decode input: the bin fed back (argmax, or the forced replay
