@@ -278,7 +278,7 @@ void launch_tile_decode_weights(const T* W, int K, int n_pairs, int epi, int n_h
 size_t tiled_decode_elems(int K, int n_pairs);
 template <typename T>
 void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride,
-                          int Tc, int pos, float* part, T* O, cudaStream_t st);
+                          int Tc, int pos, float* part, unsigned* counters, T* O, cudaStream_t st);
 template <typename T>
 void launch_head2(const float* X, const int* row_of_seq, size_t x_seq_stride, int rows_per_seq, int B, int hidden,
                   int n_bins, const T* final_norm, const T* head_w, float eps, float* logits_ws, int D, int tok0,

@@ -446,55 +446,65 @@ template void launch_dgemv<bf16>(const DGemv&, int, int, int, cudaStream_t);
 
 // ---- decode attention: one query per (sequence, head) ----------------------------
 //
-// One CTA per (head, sequence) with one warp per 32-key tile (up to 32 tiles).
+// The keys 0..pos of every (sequence, head) are cut into chunks of 64; one
+// block of two warps per (chunk, head, sequence), one warp per 32-key tile.
 // A warp issues all loads of its tile at once -- lane j reads key j's K row,
-// and the V elements [lane*EPL, lane*EPL + EPL) of all 32 keys -- so the tile
-// costs one memory round trip.  Tiles are combined in tile order.
+// and the V rows go to shared memory by cp.async -- so a tile costs one memory
+// round trip.  Each block leaves its partial (max, sum, output row) in `part`;
+// the last block of a (sequence, head) to finish (a counter that it resets)
+// adds the partials in chunk order and writes the output.
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
                "l"(gmem)
                : "memory");
 }
 
+constexpr int kDecKeys = 64;  // keys per block
+
 template <typename T, int HD>
-__global__ void __launch_bounds__(512) dec_attn_kernel(const T* __restrict__ Q, const T* __restrict__ Kc,
-                                                       const T* __restrict__ Vc, size_t kv_seq_stride, int Tc, int pos,
-                                                       int n_heads, float scale, T* __restrict__ O) {
+__global__ void __launch_bounds__(64) dec_attn_kernel(const T* __restrict__ Q, const T* __restrict__ Kc,
+                                                      const T* __restrict__ Vc, size_t kv_seq_stride, int Tc, int pos,
+                                                      int n_heads, float scale, float* __restrict__ part,
+                                                      unsigned* __restrict__ counters, T* __restrict__ O) {
   constexpr int EPL = HD / 32, V = Vec<T>::n, CPR = HD * (int)sizeof(T) / 16;  // 16-byte chunks per row
-  extern __shared__ __align__(16) uint8_t dsm[];
+  constexpr int NW = kDecKeys / 32;
+  __shared__ __align__(16) T vbuf_all[NW][32][HD];
   __shared__ float qs[HD];
-  __shared__ float wm[16], wl[16];
-  __shared__ float wacc[16][HD];
+  __shared__ float wm[NW], wl[NW];
+  __shared__ float wacc[NW][HD];
+  __shared__ int is_last;
   pdl_wait();
   pdl_trigger();
-  const int h = blockIdx.x, b = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nw = blockDim.x >> 5;
+  const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z, n_kc = gridDim.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int hidden = n_heads * HD;
-  T* vbuf = reinterpret_cast<T*>(dsm) + (size_t)warp * 32 * HD;
+  T* vbuf = &vbuf_all[warp][0][0];
   const T* Kh = Kc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
   const T* Vh = Vc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
   const int nkeys = min(pos + 1, Tc);
+  const int k0 = c * kDecKeys, k1 = min(nkeys, k0 + kDecKeys);
   for (int e = threadIdx.x; e < HD; e += blockDim.x) qs[e] = to_f(Q[(size_t)b * hidden + (size_t)h * HD + e]);
   __syncthreads();
   float m_run = -INFINITY, l_run = 0.f, acc[EPL];
 #pragma unroll
   for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
-  for (int j0 = warp * 32; j0 < nkeys; j0 += nw * 32) {
-    const int j = j0 + lane, jn = min(32, nkeys - j0);
+  const int j0 = k0 + warp * 32;
+  if (j0 < k1) {
+    const int j = j0 + lane, jn = min(32, k1 - j0);
     // the tile's V rows go to shared memory asynchronously, its K rows to registers
-    for (int c = lane; c < jn * CPR; c += 32) {
-      const int jj = c / CPR, q = c - jj * CPR;
-      cp_async16(vbuf + (size_t)jj * HD + q * (16 / sizeof(T)), Vh + (size_t)(j0 + jj) * HD + q * (16 / sizeof(T)));
+    for (int q = lane; q < jn * CPR; q += 32) {
+      const int jj = q / CPR, r = q - jj * CPR;
+      cp_async16(vbuf + (size_t)jj * HD + r * (16 / sizeof(T)), Vh + (size_t)(j0 + jj) * HD + r * (16 / sizeof(T)));
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
     uint4 kr[HD / V];
-    if (j < nkeys) {
+    if (j < k1) {
       const uint4* src = reinterpret_cast<const uint4*>(Kh + (size_t)j * HD);
 #pragma unroll
       for (int v = 0; v < HD / V; ++v) kr[v] = src[v];
     }
     float sc = -INFINITY;
-    if (j < nkeys) {
+    if (j < k1) {
       float d = 0.f;
 #pragma unroll
       for (int v = 0; v < HD / V; ++v) {
@@ -505,15 +515,9 @@ __global__ void __launch_bounds__(512) dec_attn_kernel(const T* __restrict__ Q, 
       }
       sc = d * scale;
     }
-    float mt = sc;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
-    const float mn = fmaxf(m_run, mt);
-    const float p = (sc == -INFINITY) ? 0.f : expf(sc - mn);
-    const float corr = (m_run == -INFINITY) ? 0.f : expf(m_run - mn);
-    l_run = l_run * corr + warp_allsum(p);
-#pragma unroll
-    for (int e = 0; e < EPL; ++e) acc[e] *= corr;
+    m_run = warp_max(sc);
+    const float p = (sc == -INFINITY) ? 0.f : expf(sc - m_run);
+    l_run = warp_sum(p);
     asm volatile("cp.async.wait_group 0;" ::: "memory");
     __syncwarp();
 #pragma unroll 8
@@ -523,8 +527,6 @@ __global__ void __launch_bounds__(512) dec_attn_kernel(const T* __restrict__ Q, 
 #pragma unroll
       for (int e = 0; e < EPL; ++e) acc[e] = fmaf(pj, to_f(vr[e]), acc[e]);
     }
-    __syncwarp();
-    m_run = mn;
   }
   if (lane == 0) {
     wm[warp] = m_run;
@@ -533,47 +535,68 @@ __global__ void __launch_bounds__(512) dec_attn_kernel(const T* __restrict__ Q, 
 #pragma unroll
   for (int e = 0; e < EPL; ++e) wacc[warp][lane * EPL + e] = acc[e];
   __syncthreads();
-  for (int e = threadIdx.x; e < HD; e += blockDim.x) {
+  // this block's partial: the warps' tiles combined in tile order
+  float* mine = part + ((size_t)(b * n_heads + h) * n_kc + c) * (HD + 2);
+  {
     float M = -INFINITY;
-    for (int w = 0; w < nw; ++w) M = fmaxf(M, wm[w]);
+    for (int w = 0; w < NW; ++w) M = fmaxf(M, wm[w]);
+    for (int e = threadIdx.x; e < HD; e += blockDim.x) {
+      float L = 0.f, o = 0.f;
+      for (int w = 0; w < NW; ++w) {
+        const float f = (wm[w] == -INFINITY) ? 0.f : expf(wm[w] - M);
+        L = fmaf(wl[w], f, L);
+        o = fmaf(wacc[w][e], f, o);
+      }
+      mine[2 + e] = o;
+      if (e == 0) {
+        mine[0] = M;
+        mine[1] = L;
+      }
+    }
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const unsigned prev = atomicAdd(counters + b * n_heads + h, 1u);
+    is_last = prev == (unsigned)(n_kc - 1);
+  }
+  __syncthreads();
+  if (!is_last) return;
+  // the last block: every chunk's partial, in chunk order
+  __threadfence();
+  const float* all = part + (size_t)(b * n_heads + h) * n_kc * (HD + 2);
+  float M = -INFINITY;
+  for (int q = 0; q < n_kc; ++q) M = fmaxf(M, __ldcg(all + (size_t)q * (HD + 2)));
+  for (int e = threadIdx.x; e < HD; e += blockDim.x) {
     float L = 0.f, o = 0.f;
-    for (int w = 0; w < nw; ++w) {
-      const float f = expf(wm[w] - M);
-      L = fmaf(wl[w], f, L);
-      o = fmaf(wacc[w][e], f, o);
+    for (int q = 0; q < n_kc; ++q) {
+      const float mq = __ldcg(all + (size_t)q * (HD + 2));
+      const float f = (mq == -INFINITY) ? 0.f : expf(mq - M);
+      L = fmaf(__ldcg(all + (size_t)q * (HD + 2) + 1), f, L);
+      o = fmaf(__ldcg(all + (size_t)q * (HD + 2) + 2 + e), f, o);
     }
     O[(size_t)b * hidden + (size_t)h * HD + e] = from_f<T>(o / L);
   }
-}
-
-template <typename T, int HD>
-static void dec_attn_launch(int B, int n_heads, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride, int Tc,
-                            int pos, float scale, T* O, cudaStream_t st) {
-  const size_t per_warp = (size_t)32 * HD * sizeof(T);
-  const int tiles = (std::min(pos + 1, Tc) + 31) / 32;
-  const int warps = std::max(1, std::min({16, tiles, (int)((200 * 1024) / per_warp)}));
-  const size_t smem = per_warp * warps;
-  static size_t smem_set = 48 * 1024;  // raised once, before any graph capture of the kernel
-  if (smem > smem_set) {
-    cudaFuncSetAttribute(dec_attn_kernel<T, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(200 * 1024));
-    smem_set = 200 * 1024;
-  }
-  launch_k(dec_attn_kernel<T, HD>, dim3(n_heads, B), dim3(warps * 32), smem, st, Q, Kc, Vc, kv_seq_stride, Tc, pos,
-           n_heads, scale, O);
+  if (threadIdx.x == 0) counters[b * n_heads + h] = 0u;  // ready for the next launch
 }
 
 template <typename T>
 void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride,
-                          int Tc, int pos, float* part, T* O, cudaStream_t st) {
-  (void)part;
+                          int Tc, int pos, float* part, unsigned* counters, T* O, cudaStream_t st) {
   const float scale = 1.0f / sqrtf((float)head_dim);
-  if (head_dim == 128) dec_attn_launch<T, 128>(B, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, pos, scale, O, st);
-  else dec_attn_launch<T, 64>(B, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, pos, scale, O, st);
+  const int n_kc = (std::min(pos + 1, Tc) + kDecKeys - 1) / kDecKeys;
+  const dim3 grid(n_kc, n_heads, B);
+  if (head_dim == 128)
+    launch_k(dec_attn_kernel<T, 128>, grid, dim3(kDecKeys), 0, st, Q, Kc, Vc, kv_seq_stride, Tc, pos, n_heads, scale,
+             part, counters, O);
+  else
+    launch_k(dec_attn_kernel<T, 64>, grid, dim3(kDecKeys), 0, st, Q, Kc, Vc, kv_seq_stride, Tc, pos, n_heads, scale,
+             part, counters, O);
 }
 template void launch_dec_attention<float>(int, int, int, const float*, const float*, const float*, size_t, int, int,
-                                          float*, float*, cudaStream_t);
+                                          float*, unsigned*, float*, cudaStream_t);
 template void launch_dec_attention<bf16>(int, int, int, const bf16*, const bf16*, const bf16*, size_t, int, int,
-                                         float*, bf16*, cudaStream_t);
+                                         float*, unsigned*, bf16*, cudaStream_t);
 
 // ---- action head -------------------------------------------------------------------
 

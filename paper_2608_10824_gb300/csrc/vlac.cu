@@ -69,6 +69,7 @@ struct vlac_ctx {
   uint8_t *mask, *full;
   int *idx, *M, *off, *emit_slot, *off_dec, *idx_dec, *err;
   float *logits_ws, *attn_part, *ssq_a, *ssq_b;
+  unsigned* attn_cnt;  // decode attention: finished key chunks per (sequence, head); zero between launches
   // staged per-step inputs and outputs (fixed addresses, so a step can be a graph)
   uint8_t* in_frames;
   int32_t* in_prompt;
@@ -393,6 +394,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->err, 4, base);
     sc.take(c->logits_ws, Bm * (d.parallel ? d.n_action : 1) * d.n_bins * 4, base);
     sc.take(c->attn_part, Bm * d.n_heads * ((c->Tc + 31) / 32) * (d.head_dim + 2) * 4, base);
+    sc.take(c->attn_cnt, Bm * d.n_heads * sizeof(unsigned), base);
     sc.take(c->ssq_a, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
     sc.take(c->ssq_b, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
     const size_t fbytes = (size_t)d.n_views * d.img_h * d.img_w * 3;
@@ -733,7 +735,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         {
           ProfScope ps_(c, VLAC_PROF_DECODE_ATTN, 0, st);
           launch_dec_attention<T>(B, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, pos,
-                                  c->attn_part, AO, st);
+                                  c->attn_part, c->attn_cnt, AO, st);
         }
         c->launches += 1;
         // o-projection + residual
