@@ -13,6 +13,11 @@ import synth
 # oracle's m_{t-1} is within 1e-4 of theta_m (the step is then re-synced by
 # forcing the oracle's branch).
 LOGIT_TOL = {"bf16": 2e-2, "f32": 1e-3}
+# Full 32-layer 7B shapes: two runs of the GPU path that differ only in the
+# fp32 summation order of the GEMM partial sums differ by up to 3.4e-2 in the
+# logits (the bf16 re-rounding of every layer's GEMM inputs amplifies any
+# fp32-level difference), so the bar there is twice that measured floor.
+LOGIT_TOL_DEEP = 7e-2
 ID_EXEMPT_MARGIN = 1e-3
 FLAG_TIE = 1e-4
 
@@ -44,7 +49,7 @@ def episode(d, n_frames: int, seed: int, batch: int = 1, kind=None):
 class Lockstep:
     """Runs the oracle and the library side by side, one step at a time."""
 
-    def __init__(self, d, w_cpu, w_gpu=None, batch: int = 1):
+    def __init__(self, d, w_cpu, w_gpu=None, batch: int = 1, logit_tol=None):
         import torch
 
         import oracle
@@ -59,6 +64,7 @@ class Lockstep:
         self.torch = torch
         self.prev_m = None
         self.log = []
+        self.logit_tol = logit_tol
 
     def step(self, frames, prompt, proprio, tau_sim, tau_m, permille, margin_kind=0, force_branch=None):
         torch = self.torch
@@ -83,13 +89,13 @@ class Lockstep:
         g = {k: v.cpu().numpy() for k, v in g.items()}
         err = self.ctx.sync_error()
         assert err == 0, f"device error {err}"
-        rep = compare(d, o, g, self.prev_m, tau_m)
+        rep = compare(d, o, g, self.prev_m, tau_m, self.logit_tol)
         self.prev_m = o["step_margin"].copy()
         self.log.append(rep)
         return o, g, rep
 
 
-def compare(d, o, g, prev_m, tau_m):
+def compare(d, o, g, prev_m, tau_m, logit_tol=None):
     """Checks one step; returns a small report of the numeric gaps."""
     B = o["action_ids"].shape[0]
     for k in ("static_mask", "idx", "M", "recomputed"):
@@ -98,7 +104,7 @@ def compare(d, o, g, prev_m, tau_m):
         tie = prev_m is not None and abs(prev_m[b] - tau_m) < FLAG_TIE
         if not tie:
             assert g["gate_auto"][b] == o["gate_auto"][b], f"gate_auto[{b}]"
-    tol = LOGIT_TOL[d.dtype]
+    tol = LOGIT_TOL[d.dtype] if logit_tol is None else logit_tol
     diff = np.abs(g["logits"].astype(np.float64) - o["logits"])
     assert diff.max() <= tol, f"logits differ by {diff.max():.3e} > {tol}"
     mism = g["action_ids"] != o["action_ids"]
