@@ -36,6 +36,11 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 EPISODE = 50
 TAU_SIM = (996, 1000)
 CPU_LAYERS = 2  # the CPU oracle sample runs this many of the 32 layers
+# dram__bytes_read.sum + dram__bytes_write.sum of one dgemv_kernel launch,
+# averaged over the four projections of a decode layer (one ncu capture of
+# the current kernel, profiles/dgemv_openvla7b_decode_layer.txt); None until
+# captured for a workload
+DGEMV_TRAFFIC_PER_LAUNCH = {}
 
 
 def peaks():
@@ -51,9 +56,10 @@ def peaks():
 # Algorithmic work of one step (2 FLOPs per multiply-add)
 # ---------------------------------------------------------------------------
 
-def step_work(d, M_seq, idx_seq, recomputed: bool):
+def step_work(d, M_seq, idx_seq):
     """FLOPs and bytes one sequence's step must move, from its per-layer row
-    counts M[l] and recompute order idx (what the method computes)."""
+    counts M[l] and recompute order idx (what the method computes), per pass:
+    a list of (flops, bytes other than weights, weight bytes)."""
     Hd, F, L, nb = d.hidden, d.ffn, d.n_layers, d.n_bins
     P, D = d.prefix_len, d.n_action
     M_seq = [int(m) for m in M_seq]
@@ -61,12 +67,10 @@ def step_work(d, M_seq, idx_seq, recomputed: bool):
     per_row = 2 * (4 * Hd * Hd + 3 * F * Hd)            # QKV + O + gate/up + down
     w_bytes = L * (4 * Hd * Hd + 3 * F * Hd) * 2        # bf16 weights of one pass
     head_bytes = nb * Hd * 2
-    flops = 0.0
-    byts = 0.0
     passes = []
     # prefix pass
     fp = 0.0
-    bp = float(w_bytes + head_bytes)
+    bp = 0.0
     for l in range(L):
         rows = idx_seq[:M_seq[l]]
         fp += M_seq[l] * per_row + 4 * Hd * float(np.sum(rows + 1))   # QK^T and PV over j <= pos
@@ -75,20 +79,29 @@ def step_work(d, M_seq, idx_seq, recomputed: bool):
         if l > 0:
             bp += max(M_seq[l - 1], M_seq[l]) * Hd * 4                  # record / reload layer inputs
     n_vis0 = int(np.sum((idx_seq[:M_seq[0]] >= 1) & (idx_seq[:M_seq[0]] <= d.n_visual)))
-    fp += 2 * n_vis0 * d.patch_dim * Hd + 2 * nb * Hd
-    bp += Hd * d.patch_dim * 2 + 2 * d.n_views * d.img_h * d.img_w * 3
-    passes.append((fp, bp))
+    fp += 2 * n_vis0 * d.patch_dim * Hd + 2 * nb * Hd * (D if d.parallel else 1)
+    bp += 2 * d.n_views * d.img_h * d.img_w * 3
+    passes.append((fp, bp, float(w_bytes + head_bytes + Hd * d.patch_dim * 2)))
     # autoregressive decode passes
     if not d.parallel:
         for a in range(1, D):
             pos = P + a - 1
             fd = L * (per_row + 4 * Hd * (pos + 1)) + 2 * nb * Hd
-            bd = w_bytes + head_bytes + L * (2 * (pos + 1) * Hd * 2 + 2 * Hd * 2) + Hd * 2
-            passes.append((fd, bd))
-    for f_, b_ in passes:
-        flops += f_
-        byts += b_
-    return flops, byts, passes
+            bd = L * (2 * (pos + 1) * Hd * 2 + 2 * Hd * 2) + Hd * 2
+            passes.append((fd, bd, float(w_bytes + head_bytes)))
+    return passes
+
+
+def batch_work(d, Ms, idxs):
+    """(flops, bytes, per-pass [(flops, bytes)]) of one step of a batch: the
+    sequences' own work adds up, the weights are read once per pass."""
+    per_seq = [step_work(d, Ms[b], idxs[b]) for b in range(len(Ms))]
+    passes = []
+    for i in range(len(per_seq[0])):
+        f = sum(ps[i][0] for ps in per_seq)
+        b = sum(ps[i][1] for ps in per_seq) + per_seq[0][i][2]
+        passes.append((f, b))
+    return sum(p[0] for p in passes), sum(p[1] for p in passes), passes
 
 
 # ---------------------------------------------------------------------------
@@ -140,13 +153,13 @@ class Clocks:
 # CPU oracle sample (the cpu_baseline leg and the reference arm)
 # ---------------------------------------------------------------------------
 
-def oracle_sample(d, frames, prompt, pm, tau_m, n_steps, seed, budget_s=None):
+def oracle_sample(d, frames, prompt, prop, pm, tau_m, n_steps, seed, budget_s=None):
     """Times the CPU oracle on the first CPU_LAYERS layers of each step of the
     same episode and scales the step time by n_layers / CPU_LAYERS."""
     import torch
 
     import oracle
-    ds = d.replace(n_layers=CPU_LAYERS)
+    ds = d.replace(n_layers=CPU_LAYERS, max_batch=1)
     dev = "cuda" if torch.cuda.is_available() else "cpu"
     w = synth.make_weights(ds, seed=seed, device=dev, lm_head_rows=d.n_bins)
     w = synth.weights_to(w, "cpu")
@@ -158,8 +171,8 @@ def oracle_sample(d, frames, prompt, pm, tau_m, n_steps, seed, budget_s=None):
         if t % EPISODE == 0:
             cache.reset()
         t0 = time.perf_counter()
-        orc.step(cache, frames[t % EPISODE], prompt, tau_sim=TAU_SIM, tau_margin=tau_m, permille=pm[:CPU_LAYERS],
-                 want_logits=False)
+        orc.step(cache, frames[t % EPISODE][:1], prompt[:1], None if prop is None else prop[t % EPISODE][:1],
+                 tau_sim=TAU_SIM, tau_margin=tau_m, permille=pm[:CPU_LAYERS], want_logits=False)
         times.append((time.perf_counter() - t0) * d.n_layers / CPU_LAYERS)
         if budget_s is not None and time.perf_counter() - t_begin > budget_s:
             break
@@ -171,10 +184,10 @@ def cores_used():
     return int(n) if n else (os.cpu_count() or 1)
 
 
-def run_reference(args, d, frames, prompt, pm, rank):
+def run_reference(args, d, frames, prompt, prop, pm, rank):
     if rank != 0:
         return
-    times = oracle_sample(d, frames, prompt, pm, args.tau_margin, args.warmup + args.steps, seed=args.seed)
+    times = oracle_sample(d, frames, prompt, prop, pm, args.tau_margin, args.warmup + args.steps, seed=args.seed)
     timed = times[args.warmup:]
     total = sum(timed)
     v = len(timed) / total
@@ -192,10 +205,14 @@ def run_reference(args, d, frames, prompt, pm, rank):
 
 
 def config_block(d, args):
-    return {"workload": f"{args.config}: OpenVLA-7B-shaped Llama-2 backbone (32 layers, hidden 4096, "
-                        f"32x128 heads, SwiGLU 11008, vocab 32000, 256 action bins), 224x224 frame -> "
-                        f"256 patches, 27 text tokens, 7 autoregressive action tokens, 50-frame scene episode",
-            "global_batch": 1 * args.gpus, "seq_len": d.pass_len, "parallelism": f"replicas x{args.gpus}",
+    vis = f"{d.n_views}x{d.img_h}x{d.img_w} frame(s) -> {d.n_visual} patches"
+    act = (f"{d.n_action} parallel action positions" if d.parallel else f"{d.n_action} autoregressive action tokens")
+    extra = f", {d.proprio_dim}-d proprio token" if d.proprio_dim else ""
+    batch = (f", batch of {d.max_batch} episodes with blob speeds U[0, 8] px/frame" if d.max_batch > 1 else "")
+    return {"workload": f"{args.config}: OpenVLA-7B-shaped Llama-2 backbone ({d.n_layers} layers, hidden {d.hidden}, "
+                        f"{d.n_heads}x{d.head_dim} heads, SwiGLU {d.ffn}, vocab {d.vocab}, {d.n_bins} action bins), "
+                        f"{vis}{extra}, {d.n_text} text tokens, {act}, {EPISODE}-frame scene episode{batch}",
+            "global_batch": d.max_batch * args.gpus, "seq_len": d.pass_len, "parallelism": f"replicas x{args.gpus}",
             "tau_sim": f"{TAU_SIM[0]}/{TAU_SIM[1]}", "tau_margin": args.tau_margin,
             "reuse_permille": "linear 900 -> 500", "l2": "inputs larger than L2 (13 GB of weights per pass)"}
 
@@ -223,12 +240,15 @@ def main():
     local = int(os.environ.get("LOCAL_RANK", "0"))
     d = synth.dims_for(args.config)
     seed = args.seed + rank
-    frames = synth.make_episode(d, EPISODE, seed=seed, kind="scene")
-    prompt = synth.make_prompt(d, seed=seed)
+    B = d.max_batch
+    frames = synth.make_episode(d, EPISODE, seed=seed, batch=B, kind="scene",
+                                speeds=synth.batch_speeds(B, seed=seed) if B > 1 else None)
+    prompt = synth.make_prompt(d, seed=seed, batch=B)
+    prop = synth.make_proprio(d, EPISODE, seed=seed, batch=B)   # None without a proprio token
     pm = synth.linear_schedule(d.n_layers)
 
     if args.impl == "reference":
-        run_reference(args, d, frames, prompt, pm, rank)
+        run_reference(args, d, frames, prompt, prop, pm, rank)
         return
 
     import torch
@@ -241,21 +261,22 @@ def main():
 
     dev = torch.device("cuda", local)
     w = synth.make_weights(d, seed=args.seed, device=dev)
-    ctx = Context(d, w, max_batch=1)
+    ctx = Context(d, w, max_batch=B)
     del w
     torch.cuda.empty_cache()
-    cache = ctx.new_cache(1)
-    fr_dev = torch.from_numpy(frames).to(dev)          # [T][1][1][H][W][3]
+    cache = ctx.new_cache(B)
+    fr_dev = torch.from_numpy(frames).to(dev)          # [T][B][views][H][W][3]
     pr_dev = torch.from_numpy(prompt).to(dev)
+    pp_dev = None if prop is None else torch.from_numpy(np.ascontiguousarray(prop, np.float32)).to(dev)
     K, W = args.steps, args.warmup
-    outs = ctx.alloc_outputs(1, want=("M", "idx", "gate_auto"))
+    outs = ctx.alloc_outputs(B, want=("M", "idx", "gate_auto"))
     hist = {k: torch.zeros((K,) + tuple(v.shape), dtype=v.dtype, device=dev) for k, v in outs.items()}
 
     def one_step(t, out):
         if t % EPISODE == 0:
             ctx.reset(cache)
-        ctx.step(cache, fr_dev[t % EPISODE], pr_dev, tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm,
-                 out=out)
+        ctx.step(cache, fr_dev[t % EPISODE], pr_dev, None if pp_dev is None else pp_dev[t % EPISODE],
+                 tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm, out=out)
 
     def barrier():
         torch.cuda.synchronize()
@@ -286,24 +307,26 @@ def main():
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
     assert ctx.sync_error() == 0
-    value = world * K / (ms / 1e3)
+    value = world * B * K / (ms / 1e3)   # sequence-steps per second
 
     # ---- algorithmic work of the timed steps ----
-    Ms = hist["M"].cpu().numpy()[:, 0]
-    idxs = hist["idx"].cpu().numpy()[:, 0]
-    rec = hist["recomputed"].cpu().numpy()[:, 0]
+    Ms = hist["M"].cpu().numpy()           # [K][B][L]
+    idxs = hist["idx"].cpu().numpy()       # [K][B][S]
+    rec = hist["recomputed"].cpu().numpy()  # [K][B]
     pk, src = peaks()
-    F_tot = B_tot = 0.0
+    F_tot = B_tot = gemm_flops = 0.0
     t_roof_step = t_roof_pass = 0.0
+    per_row = 2 * (4 * d.hidden * d.hidden + 3 * d.ffn * d.hidden)
     for k in range(K):
-        f_, b_, passes = step_work(d, Ms[k], idxs[k], bool(rec[k]))
+        f_, b_, passes = batch_work(d, Ms[k], idxs[k])
         F_tot += f_
         B_tot += b_
+        gemm_flops += float(Ms[k].sum()) * per_row
         t_roof_step += max(f_ / (pk["bf16_tflops"] * 1e12), b_ / (pk["hbm_gbs"] * 1e9))
         t_roof_pass += sum(max(fp / (pk["bf16_tflops"] * 1e12), bp / (pk["hbm_gbs"] * 1e9)) for fp, bp in passes)
     t_meas = ms / 1e3 / K
 
-    # ---- roofline of the dominant kernel (decode GEMV), second pass with per-launch events ----
+    # ---- per-kind device time, second pass with per-launch events ----
     ctx.prof_enable(True)
     for k in range(K):
         one_step(W + K + k, outs)
@@ -317,15 +340,32 @@ def main():
         breakdown[kinds[i]] = ctx.prof_read(i)[0] / K
     gemv_gbs = g_bytes / (g_ms / 1e3) / 1e9 if g_ms > 0 else None
     gemm_gbs = p_bytes / (p_ms / 1e3) / 1e9 if p_ms > 0 else None
+    gemm_tfs = gemm_flops / (p_ms / 1e3) / 1e12 if p_ms > 0 else None
+    if g_n:
+        # weight streaming of the decode passes dominates the step
+        roof = {"bound": "hbm", "achieved": gemv_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": gemv_gbs / pk["hbm_gbs"], "traffic": DGEMV_TRAFFIC_PER_LAUNCH.get(args.config),
+                "kernel": "dgemv_kernel (decode weight streaming)", "launches": g_n,
+                "avg_launch_us": 1e3 * g_ms / g_n, "peak_source": f"{src} hbm_gbs"}
+    else:
+        # no decode passes: the prefix GEMMs (tensor cores) dominate
+        roof = {"bound": "tensor", "achieved": gemm_tfs, "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s",
+                "frac": gemm_tfs / pk["bf16_tflops_sustained"], "traffic": None,
+                "kernel": "gemm_tc_kernel (tcgen05 prefix projections)", "launches": p_n,
+                "avg_launch_us": 1e3 * p_ms / max(p_n, 1), "peak_source": f"{src} bf16_tflops_sustained"}
 
     # ---- end to end through the public API with host buffers ----
     fr_host = torch.from_numpy(frames).pin_memory()
     pr_host = torch.from_numpy(prompt).pin_memory()
+    pp_host = None if pp_dev is None else pp_dev.cpu().pin_memory()
     f_buf = torch.empty_like(fr_dev[0])
     p_buf = torch.empty_like(pr_dev)
+    q_buf = None if pp_dev is None else torch.empty_like(pp_dev[0])
     res_host = {n: torch.empty(outs[n].shape, dtype=outs[n].dtype).pin_memory()
                 for n in ("action_ids", "margins", "recomputed", "step_margin")}
     h2d = f_buf.numel() * f_buf.element_size() + p_buf.numel() * p_buf.element_size()
+    if q_buf is not None:
+        h2d += q_buf.numel() * q_buf.element_size()
     d2h = sum(v.numel() * v.element_size() for v in res_host.values())
     barrier()
     t0 = time.perf_counter()
@@ -333,9 +373,11 @@ def main():
         t = W + 2 * K + k
         f_buf.copy_(fr_host[t % EPISODE], non_blocking=True)
         p_buf.copy_(pr_host, non_blocking=True)
+        if q_buf is not None:
+            q_buf.copy_(pp_host[t % EPISODE], non_blocking=True)
         if t % EPISODE == 0:
             ctx.reset(cache)
-        ctx.step(cache, f_buf, p_buf, tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm, out=outs)
+        ctx.step(cache, f_buf, p_buf, q_buf, tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm, out=outs)
         for n, hbuf in res_host.items():
             hbuf.copy_(outs[n], non_blocking=True)
         torch.cuda.current_stream().synchronize()  # the action is needed before the next frame
@@ -344,16 +386,17 @@ def main():
         t_ = torch.tensor([e2e_s], device=dev)
         dist.all_reduce(t_, op=dist.ReduceOp.MAX)
         e2e_s = float(t_.item())
-    e2e = world * K / e2e_s
+    e2e = world * B * K / e2e_s
 
     # ---- CPU oracle baseline (rank 0, N = 1 only) ----
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        times = oracle_sample(d, frames, prompt, pm, args.tau_margin, 10 ** 6, seed=args.seed,
+        times = oracle_sample(d, frames, prompt, prop, pm, args.tau_margin, 10 ** 6, seed=args.seed,
                               budget_s=args.cpu_budget)
         cpu = {"value": len(times) / sum(times), "unit": "steps/s", "cores": cores_used(), "kind": "oracle",
-               "sample": f"{len(times)} steps of the same episode; the oracle runs the first {CPU_LAYERS} of "
-                         f"{d.n_layers} layers of each step, time scaled by {d.n_layers}/{CPU_LAYERS}"}
+               "sample": f"{len(times)} steps of the first sequence's episode; the oracle runs the first "
+                         f"{CPU_LAYERS} of {d.n_layers} layers of each step, time scaled by "
+                         f"{d.n_layers}/{CPU_LAYERS}"}
 
     if rank != 0:
         return
@@ -366,19 +409,19 @@ def main():
                           "t_roof_ms": 1e3 * t_roof_step / K, "t_meas_ms": 1e3 * t_meas,
                           "alg_tflop_per_step": F_tot / K / 1e12, "alg_gb_per_step": B_tot / K / 1e9,
                           "peaks": src, "fire_rate": float(rec.mean())},
-        "roofline": {"bound": "hbm", "achieved": gemv_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                     "frac": (gemv_gbs / pk["hbm_gbs"]) if gemv_gbs else None, "traffic": None,
-                     "kernel": "gemv_kernel (decode weight streaming)", "launches": g_n,
-                     "avg_launch_us": 1e3 * g_ms / max(g_n, 1), "peak_source": f"{src} hbm_gbs"},
-        "prefix_gemm": {"weight_gbs": gemm_gbs, "launches": p_n, "avg_launch_us": 1e3 * p_ms / max(p_n, 1)},
+        "roofline": roof,
+        "prefix_gemm": {"weight_gbs": gemm_gbs, "tflops": gemm_tfs, "launches": p_n,
+                        "avg_launch_us": 1e3 * p_ms / max(p_n, 1)},
         "device_ms_per_step_by_kind": {k: round(v, 4) for k, v in breakdown.items()},
         "clocks": clocks,
         "e2e": {"value": e2e, "unit": "steps/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "note": "frame + prompt H2D from pinned memory, action ids/margins/flag D2H, synchronised "
-                        "every step (closed loop)"},
+                "note": "frames + prompt (+ proprio) H2D from pinned memory, action ids/margins/flags D2H, "
+                        "synchronised every step (closed loop)"},
         "gpu_launches": int(launches),
         "cpu_baseline": cpu,
     }
+    if B > 1:
+        line["unit_note"] = f"steps/s counts sequence-steps: {B} sequences per batched step"
     print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
