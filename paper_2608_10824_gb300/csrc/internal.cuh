@@ -65,6 +65,7 @@ struct DGemv {
   float* ssq_out;       // residual GEMV: this launch's per-CTA sums of squares [nb][grid]
   int* err;             // device error word (bounded waits)
   int ns;               // stages of the weight ring
+  int pre;              // stages streamed before the input vector is ready (0: no limit)
   // the next decode GEMV of the stream: this CTA pulls the start of that
   // kernel's CTA region into L2 once its own loads are issued
   const void* pf_W;
@@ -144,6 +145,21 @@ __device__ __forceinline__ void set_error(int* err, int code) {
   if (err) atomicCAS(err, 0, code);
 }
 
+// ldmatrix: four 8x8 b16 matrices; lane l gives the row address of row l%8 of matrix l/8
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+// D += A * B on the legacy tensor path, m16n8k16, bf16 operands, fp32 accumulators
+__device__ __forceinline__ void mma_bf16(float* d, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -276,6 +292,7 @@ template <typename T>
 void launch_tile_decode_weights(const T* W, int K, int n_pairs, int epi, int n_heads, int head_dim, int ffn, T* out,
                                 cudaStream_t st);
 size_t tiled_decode_elems(int K, int n_pairs);
+size_t dgemv_stage_bytes();  // bytes of one weight-ring stage of the decode GEMV
 template <typename T>
 void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride,
                           int Tc, int pos, float* part, unsigned* counters, T* O, cudaStream_t st);

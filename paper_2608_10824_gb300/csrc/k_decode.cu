@@ -7,6 +7,8 @@
 // Attention of the single query per head is split over key chunks and
 // combined in a fixed order.  The action head (final norm, bin logits) is a
 // multi-CTA GEMV followed by a one-warp top-2 / margin reduction per row.
+#include <cooperative_groups.h>
+
 #include <algorithm>
 #include <type_traits>
 
@@ -15,14 +17,6 @@
 namespace vlac {
 
 namespace {
-
-__device__ __forceinline__ uint4 ld_stream(const void* p) {
-  uint4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "l"(p));
-  return v;
-}
 
 template <typename T> struct Vec;
 template <> struct Vec<bf16> { static constexpr int n = 8; };
@@ -94,25 +88,42 @@ __device__ __forceinline__ void norm_rows_to_smem(const float* __restrict__ X, c
 //
 // Weight layout for decode streaming (built once at create time): output row
 // pairs are grouped 4 at a time (8 weight rows); a group's K range is cut into
-// chunks of kDecKC elements; the tile [8 rows][chunk] is contiguous, and the
-// tiles of a group follow each other, then the next group.  Pair p's rows:
+// chunks of kDecTileB bytes per row; the tile [8 rows][chunk] is contiguous,
+// and the tiles of a group follow each other, then the next group.  Pair p's
+// rows:
 //   QKV:     (i, i + head_dim/2) of one head of q, k or v;
 //   SwiGLU:  (gate j, up j);
 //   other:   (2p, 2p + 1).
+// Inside a bf16 tile the 8 rows are interleaved in steps of 8 elements
+// ([k/8][row][k%8]): the 8 rows of one 8-element K step are 128 contiguous
+// bytes, so one ldmatrix.x4 reads 8 rows x 32 K without bank conflicts and
+// hands every lane its B fragment of two m16n8k16 products.  fp32 tiles stay
+// row-major ([row][k]).
 //
 // Persistent GEMV: one CTA per SM owns a contiguous, balanced range of groups
 // and so one contiguous region of the tiled weights.  A producer warp streams
 // it tile by tile into a ring of shared-memory stages with 1-D bulk copies;
 // the producer starts before the dependency wait (weights are constant), so a
-// kernel's first stages stream in while its predecessor drains.  8 consumer
-// warps: warp w handles pair w/2 over half of each tile's K range; the halves
-// are added in order at the end of the group.
+// kernel's first stages stream in while its predecessor drains.
+//
+// bf16 consumers (8 warps): warp w takes the w-th eighth of every tile's K
+// range, for all 8 rows, on the tensor pipe: the weights are the B operand
+// (n = row), the input vectors the A operand (m = sequence, rows >= NB zero),
+// so D[b][row] accumulates y_b over the warp's K range in fp32.  The products
+// are exact and the adds are fp32, as in a scalar dot product; the tensor
+// path only removes the unpacking and multiply-add instructions that
+// otherwise bound the consumers below the stream rate.  At the end of a group
+// the 8 warps' partials are added in warp (K) order by one warp, which
+// rotates from group to group, and it runs the epilogue.  fp32 consumers run
+// the scalar loop: warp w handles pair w/2 over one half of each tile's K.
 //
 // RMSNorm without a second pass over the row: every residual-writing GEMV
 // (and the decode embedding) stores per CTA and sequence the sum of squares
 // of the residual elements it produced; a normalising GEMV sums those
 // partials in index order for the mean square and normalises the input
-// vector once into shared memory (x * r * g rounded to T).
+// vector once into shared memory (x * r * g rounded to T).  bf16 vectors are
+// kept in A-fragment order: per 32-element K step and lane t the elements
+// (2t, 2t+1, 2t+8, 2t+9, 2t+16, 2t+17, 2t+24, 2t+25), one 16-byte load.
 
 constexpr int kNC = 8;          // consumer warps
 constexpr int kGP = 4;          // row pairs per group
@@ -121,6 +132,13 @@ constexpr int kDecTileB = 4096; // bytes of one tile row (K chunk)
 
 __host__ __device__ inline size_t sgemv_xs_bytes(int nb, int K, int esz) {
   return ((size_t)nb * K * esz + 1023) / 1024 * 1024;
+}
+
+// position (in elements, within its row) of element k of a bf16 input vector
+// in A-fragment order
+__device__ __forceinline__ int afrag_pos(int k) {
+  const int i = k >> 5, w = k & 31, s = w >> 3, t = (w & 7) >> 1;
+  return ((i * 4 + t) * 8) + s * 2 + (w & 1);
 }
 
 template <int EPI>
@@ -144,16 +162,18 @@ __host__ __device__ __forceinline__ void dec_pair_rows(int p, int n_heads, int h
 template <typename T, int EPI>
 __global__ void tile_decode_weights_kernel(const T* __restrict__ W, int K, int n_pairs, int n_heads, int head_dim,
                                            int ffn, T* __restrict__ out) {
+  constexpr int TR = 2 * kGP;
   const int KC = kDecTileB / (int)sizeof(T);
-  const int g = blockIdx.x, r = blockIdx.y;  // r: 0..7
+  const int g = blockIdx.x, r = blockIdx.y;  // r: 0 .. TR-1
   const int p = g * kGP + r / 2;
   int r1 = 0, r2 = 0;
   if (p < n_pairs) dec_pair_rows<EPI>(p, n_heads, head_dim, ffn, r1, r2);
   const T* src = W + (size_t)((r & 1) ? r2 : r1) * K;
-  T* base = out + (size_t)g * 2 * kGP * K;
+  T* base = out + (size_t)g * TR * K;
   for (int k = threadIdx.x; k < K; k += blockDim.x) {
     const int c = k / KC, kk = k - c * KC, kn = min(KC, K - c * KC);
-    base[(size_t)2 * kGP * c * KC + (size_t)r * kn + kk] = p < n_pairs ? src[k] : from_f<T>(0.f);
+    const size_t at = sizeof(T) == 2 ? (size_t)((kk >> 3) * TR + r) * 8 + (kk & 7) : (size_t)r * kn + kk;
+    base[(size_t)TR * c * KC + at] = p < n_pairs ? src[k] : from_f<T>(0.f);
   }
 }
 
@@ -172,9 +192,62 @@ void launch_tile_decode_weights(const T* W, int K, int n_pairs, int epi, int n_h
 template void launch_tile_decode_weights<float>(const float*, int, int, int, int, int, int, float*, cudaStream_t);
 template void launch_tile_decode_weights<bf16>(const bf16*, int, int, int, int, int, int, bf16*, cudaStream_t);
 size_t tiled_decode_elems(int K, int n_pairs) { return (size_t)((n_pairs + kGP - 1) / kGP) * 2 * kGP * K; }
+size_t dgemv_stage_bytes() { return (size_t)2 * kGP * kDecTileB; }
+
+// Epilogue of one output row pair (p) of sequence b: y1, y2 are the two rows'
+// dot products; e1, e2 the operands loaded ahead (RoPE cos/sin, or the two
+// residual elements).  Returns the residual epilogue's sum of squares.
+template <typename T, int EPI>
+__device__ __forceinline__ float dgemv_epilogue(const DGemv& a, int p, int b, float y1, float y2, float e1, float e2) {
+  if constexpr (EPI == kEpiQkvRope) {
+    const int hd = a.head_dim, half = hd >> 1, hidden = a.n_heads * hd;
+    const int sec = p / (hidden / 2), within = p - sec * (hidden / 2);
+    const int h = within / half, e = within - h * half;
+    float o1 = y1, o2 = y2;
+    if (sec < 2) {
+      o1 = y1 * e1 - y2 * e2;  // (cos, sin) of the pair's RoPE angle
+      o2 = y2 * e1 + y1 * e2;
+    }
+    T* dst = sec == 0 ? static_cast<T*>(a.Q) + (size_t)b * hidden + (size_t)h * hd
+                      : static_cast<T*>(sec == 1 ? a.Kc : a.Vc) + (size_t)b * a.kv_seq_stride +
+                            ((size_t)h * a.Tc + a.pos) * hd;
+    dst[e] = from_f<T>(o1);
+    dst[e + half] = from_f<T>(o2);
+    return 0.f;
+  } else if constexpr (EPI == kEpiSwiglu) {
+    static_cast<T*>(a.G)[(size_t)b * a.ffn + p] = from_f<T>((y1 / (1.0f + expf(-y1))) * y2);
+    return 0.f;
+  } else {
+    float* x = a.Xres + (size_t)b * a.n_out;
+    const float n1 = e1 + y1, n2 = e2 + y2;
+    x[2 * p] = n1;
+    x[2 * p + 1] = n2;
+    return fmaf(n1, n1, n2 * n2);
+  }
+}
+
+template <typename T, int EPI>
+__device__ __forceinline__ void dgemv_epilogue_operands(const DGemv& a, int p, int b, float& e1, float& e2) {
+  e1 = e2 = 0.f;
+  if constexpr (EPI == kEpiQkvRope) {
+    const int hd = a.head_dim, half = hd >> 1, hidden = a.n_heads * hd;
+    const int sec = p / (hidden / 2), within = p - sec * (hidden / 2);
+    const int e = within - (within / half) * half;
+    if (sec < 2) {
+      e1 = a.rope_cos[(size_t)a.pos * half + e];
+      e2 = a.rope_sin[(size_t)a.pos * half + e];
+    }
+  } else if constexpr (EPI == kEpiResid) {
+    e1 = a.Xres[(size_t)b * a.n_out + 2 * p];
+    e2 = a.Xres[(size_t)b * a.n_out + 2 * p + 1];
+  }
+}
+
+__device__ __forceinline__ uint32_t ldg_u32(const void* p) { return __ldg(static_cast<const unsigned int*>(p)); }
 
 template <typename T, int NB, int EPI, bool NORM, bool XG>
 __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
+  constexpr bool kMma = sizeof(T) == 2;
   constexpr int V = Vec<T>::n;
   constexpr int KC = kDecTileB / (int)sizeof(T);
   constexpr int TR = 2 * kGP;  // tile rows
@@ -183,16 +256,17 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
   extern __shared__ __align__(1024) uint8_t dsm[];
   __shared__ __align__(8) uint64_t full_bar[kMaxNS];
   __shared__ __align__(8) uint64_t empty_bar[kMaxNS];
-  __shared__ float red[kNC][NB];
-  __shared__ float half_acc[kGP][2][NB];
+  __shared__ __align__(8) uint64_t ready_bar;  // the input vector is in place (limits the early stream)
+  __shared__ float red[kNC][32];
   __shared__ float rr[NB];
+  __shared__ __align__(8) float2 pacc[2][kNC][32];  // bf16 path: per-warp partials, two groups in flight
+  __shared__ float half_acc[kGP][2][NB];            // fp32 path: the second K half of every pair
   __shared__ int abort_flag;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int K = a.K, nchunk = (K + KC - 1) / KC;
   const int G = (a.n_pairs + kGP - 1) / kGP;
   const int g0 = (int)(((long long)G * blockIdx.x) / gridDim.x);
   const int g1 = (int)(((long long)G * (blockIdx.x + 1)) / gridDim.x);
-  const int hd = a.head_dim, half = hd >> 1;
   T* xs = reinterpret_cast<T*>(dsm);
   uint8_t* stages = dsm + (XG ? 0 : sgemv_xs_bytes(NB, K, (int)sizeof(T)));
   const T* Wt = static_cast<const T*>(a.W);
@@ -201,6 +275,7 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], kNC);
     }
+    mbar_init(&ready_bar, 1);
     abort_flag = 0;
     mbar_fence_init();
   }
@@ -210,12 +285,17 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
   if (warp == kNC) {
     // ---- producer: weights only, so it runs ahead of the dependency wait ----
     if (lane == 0) {
-      int stage = 0;
+      int stage = 0, issued = 0;
       uint32_t phase = 0;
       for (int g = g0; g < g1 && !*abort; ++g) {
         const T* gbase = Wt + (size_t)g * TR * K;
         for (int c = 0; c < nchunk; ++c) {
           const int kn = min(KC, K - c * KC);
+          if (issued++ == a.pre && a.pre > 0 && !mbar_wait(&ready_bar, 0, kWaitLimit, abort)) {
+            set_error(a.err, VLAC_ERR_TIMEOUT);
+            *abort = 1;
+            break;
+          }
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, kWaitLimit, abort)) {
             set_error(a.err, VLAC_ERR_TIMEOUT);
             *abort = 1;
@@ -256,6 +336,25 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
   pdl_trigger();
   const int tid = threadIdx.x;  // 0 .. kNC*32-1
   if constexpr (NORM) {
+    const T* gn = static_cast<const T*>(a.gain);
+    // bf16: the first items of the vector are loaded together with the
+    // sums-of-squares partials, so that the prologue costs one round trip
+    constexpr int kPre = 2;  // items (8 elements) per thread loaded ahead
+    const int n8 = K / 8;
+    uint4 pg[kPre];
+    float4 px0[kPre], px1[kPre];
+    if constexpr (kMma) {
+#pragma unroll
+      for (int j = 0; j < kPre; ++j) {
+        const int m = tid + j * kNC * 32;
+        if (m < NB * n8) {
+          const int b = m / n8, k = (m - b * n8) * 8;
+          pg[j] = *reinterpret_cast<const uint4*>(gn + k);
+          px0[j] = *reinterpret_cast<const float4*>(a.X + (size_t)b * K + k);
+          px1[j] = *reinterpret_cast<const float4*>(a.X + (size_t)b * K + k + 4);
+        }
+      }
+    }
     float sacc[NB];
 #pragma unroll
     for (int b = 0; b < NB; ++b) sacc[b] = 0.f;
@@ -274,129 +373,261 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
       rr[tid] = 1.0f / sqrtf(t / (float)K + a.eps);
     }
     asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
-    const T* g = static_cast<const T*>(a.gain);
-    for (int k = tid; k < K; k += kNC * 32) {
-      const float gk = to_f(g[k]);
+    if constexpr (kMma) {
+      // 8 elements per item; the first kPre items of a thread were loaded above
+#pragma unroll 4
+      for (int m = tid; m < NB * n8; m += kNC * 32) {
+        const int b = m / n8, k = (m - b * n8) * 8, j = (m - tid) / (kNC * 32);
+        uint4 gv;
+        float4 x0, x1;
+        if (j < kPre) {
+          gv = pg[0];
+          x0 = px0[0];
+          x1 = px1[0];
 #pragma unroll
-      for (int b = 0; b < NB; ++b) xs[(size_t)b * K + k] = from_f<T>((a.X[(size_t)b * K + k] * rr[b]) * gk);
+          for (int jj = 1; jj < kPre; ++jj)
+            if (jj == j) {
+              gv = pg[jj];
+              x0 = px0[jj];
+              x1 = px1[jj];
+            }
+        } else {
+          gv = *reinterpret_cast<const uint4*>(gn + k);
+          x0 = *reinterpret_cast<const float4*>(a.X + (size_t)b * K + k);
+          x1 = *reinterpret_cast<const float4*>(a.X + (size_t)b * K + k + 4);
+        }
+        float gf[8];
+        unpack<T>(gv, gf);
+        const float r = rr[b];
+        const float xv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+        uint32_t* row = reinterpret_cast<uint32_t*>(xs + (size_t)b * K);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const __nv_bfloat162 v = __floats2bfloat162_rn((xv[2 * j] * r) * gf[2 * j], (xv[2 * j + 1] * r) * gf[2 * j + 1]);
+          row[afrag_pos(k + 2 * j) >> 1] = *reinterpret_cast<const uint32_t*>(&v);
+        }
+      }
+    } else {
+      for (int k = tid; k < K; k += kNC * 32) {
+        const float gk = to_f(gn[k]);
+#pragma unroll
+        for (int b = 0; b < NB; ++b) xs[(size_t)b * K + k] = from_f<T>((a.X[(size_t)b * K + k] * rr[b]) * gk);
+      }
     }
   } else if constexpr (!XG) {
-    const uint4* src = reinterpret_cast<const uint4*>(static_cast<const T*>(a.xin));
-    uint4* dst = reinterpret_cast<uint4*>(xs);
-    for (int i = tid; i < NB * K / V; i += kNC * 32) dst[i] = src[i];
+    if constexpr (kMma) {
+      const int n8 = K / 8;
+#pragma unroll 4
+      for (int m = tid; m < NB * n8; m += kNC * 32) {
+        const int b = m / n8, k = (m - b * n8) * 8;
+        const uint4 v = *reinterpret_cast<const uint4*>(static_cast<const T*>(a.xin) + (size_t)b * K + k);
+        uint32_t* row = reinterpret_cast<uint32_t*>(xs + (size_t)b * K);
+        row[afrag_pos(k) >> 1] = v.x;
+        row[afrag_pos(k + 2) >> 1] = v.y;
+        row[afrag_pos(k + 4) >> 1] = v.z;
+        row[afrag_pos(k + 6) >> 1] = v.w;
+      }
+    } else {
+      const uint4* src = reinterpret_cast<const uint4*>(static_cast<const T*>(a.xin));
+      uint4* dst = reinterpret_cast<uint4*>(xs);
+      for (int i = tid; i < NB * K / V; i += kNC * 32) dst[i] = src[i];
+    }
   }
   asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
-  const T* xsrc = XG ? static_cast<const T*>(a.xin) : xs;
+  if (tid == 0) mbar_arrive(&ready_bar);
 
-  const int q = warp >> 1, hk = warp & 1;  // pair within the group, K half
-  float ssq[NB];
-#pragma unroll
-  for (int b = 0; b < NB; ++b) ssq[b] = 0.f;
+  float ssq = 0.f;  // residual epilogue: this thread's sum of squares (sequence per lane, see below)
   bool aborted = false;
   int stage = 0;
   uint32_t phase = 0;
-  for (int g = g0; g < g1; ++g) {
-    float acc1[NB], acc2[NB];
+  if constexpr (kMma) {
+    const int gq = lane >> 2, tq = lane & 3;  // fragment row (sequence) and column pair
+    const uint32_t st_lane = smem_u32(stages) + (uint32_t)lane * 16;
+    for (int g = g0; g < g1; ++g) {
+      const int pb = (g - g0) & 1, ew = (g - g0) % kNC;  // partial buffer, epilogue warp
+      const int p = g * kGP + tq;
+      const bool epi = warp == ew && gq < NB && p < a.n_pairs;
+      float e1 = 0.f, e2 = 0.f;
+      if (epi) dgemv_epilogue_operands<T, EPI>(a, p, gq, e1, e2);  // latency hidden by the tiles
+      // four accumulator sets, so that consecutive products do not wait on
+      // each other; added in a fixed order at the end of the group
+      float d[4][4];
 #pragma unroll
-    for (int b = 0; b < NB; ++b) acc1[b] = acc2[b] = 0.f;
-    for (int c = 0; c < nchunk; ++c) {
-      const int k0 = c * KC, kn = min(KC, K - k0), kh = kn >> 1;
-      bool ok = true;
-      if (lane == 0) ok = mbar_wait(&full_bar[stage], phase, kWaitLimit, abort);
-      ok = __shfl_sync(0xffffffffu, ok, 0);
-      if (!ok) {
-        if (lane == 0) {
-          set_error(a.err, VLAC_ERR_TIMEOUT);
-          *abort = 1;
+      for (int u = 0; u < 4; ++u) d[u][0] = d[u][1] = d[u][2] = d[u][3] = 0.f;
+      for (int c = 0; c < nchunk; ++c) {
+        const int k0 = c * KC, n32 = min(KC, K - k0) >> 5;
+        const int i0 = n32 * warp / kNC, i1 = n32 * (warp + 1) / kNC;
+        bool ok = true;
+        if (lane == 0) ok = mbar_wait(&full_bar[stage], phase, kWaitLimit, abort);
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) {
+          if (lane == 0) {
+            set_error(a.err, VLAC_ERR_TIMEOUT);
+            *abort = 1;
+          }
+          aborted = true;
+          break;
         }
-        aborted = true;
-        break;
-      }
-      const T* st = reinterpret_cast<const T*>(stages + (size_t)stage * stage_b);
-      const uint4* w1 = reinterpret_cast<const uint4*>(st + (size_t)(2 * q) * kn + hk * kh);
-      const uint4* w2 = reinterpret_cast<const uint4*>(st + (size_t)(2 * q + 1) * kn + hk * kh);
-      for (int v = lane; v < kh / V; v += 32) {
-        float f1[V], f2[V];
-        unpack<T>(w1[v], f1);
-        unpack<T>(w2[v], f2);
+        const uint32_t st = st_lane + (uint32_t)(stage * stage_b);
+        const T* xrow = XG ? static_cast<const T*>(a.xin) + (size_t)gq * K + k0 + 2 * tq : xs + (size_t)gq * K + k0 + tq * 8;
+        int i = i0;
+        // blocks of four 32-element K steps: all fragments are loaded before
+        // the first product, one accumulator set per step
+        for (; i + 4 <= i1; i += 4) {
+          uint32_t bf[4][4];
+          uint4 xa[4];
 #pragma unroll
-        for (int b = 0; b < NB; ++b) {
-          float xf[V];
-          const uint4* xp = reinterpret_cast<const uint4*>(xsrc + (size_t)b * K + k0 + hk * kh);
-          uint4 xu;
-          if constexpr (XG) xu = __ldg(xp + v);
-          else xu = xp[v];
-          unpack<T>(xu, xf);
+          for (int u = 0; u < 4; ++u) {
+            ldsm_x4(st + (uint32_t)(i + u) * 512u, bf[u][0], bf[u][1], bf[u][2], bf[u][3]);
+            xa[u] = make_uint4(0u, 0u, 0u, 0u);
+          }
+          if (gq < NB) {
 #pragma unroll
-          for (int i = 0; i < V; ++i) {
-            acc1[b] = fmaf(f1[i], xf[i], acc1[b]);
-            acc2[b] = fmaf(f2[i], xf[i], acc2[b]);
+            for (int u = 0; u < 4; ++u) {
+              if constexpr (XG) {
+                const T* xr = xrow + (i + u) * 32;
+                xa[u] = make_uint4(ldg_u32(xr), ldg_u32(xr + 8), ldg_u32(xr + 16), ldg_u32(xr + 24));
+              } else {
+                xa[u] = *reinterpret_cast<const uint4*>(xrow + (i + u) * 32);
+              }
+            }
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            mma_bf16(d[u], xa[u].x, 0u, xa[u].y, 0u, bf[u][0], bf[u][1]);
+            mma_bf16(d[u], xa[u].z, 0u, xa[u].w, 0u, bf[u][2], bf[u][3]);
           }
         }
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&empty_bar[stage]);
-      if (++stage == NS) {
-        stage = 0;
-        phase ^= 1u;
-      }
-    }
-    if (aborted) break;
-    // add the two K halves of every pair in order, then the epilogue
-#pragma unroll
-    for (int b = 0; b < NB; ++b) {
-      const float t1 = warp_allsum(acc1[b]), t2 = warp_allsum(acc2[b]);
-      if (hk == 1 && lane == 0) {
-        half_acc[q][0][b] = t1;
-        half_acc[q][1][b] = t2;
-      }
-      acc1[b] = t1;
-      acc2[b] = t2;
-    }
-    asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
-    const int p = g * kGP + q;
-    if (hk == 0 && lane < NB && p < a.n_pairs) {
-      const int b = lane;
-      float y1 = 0.f, y2 = 0.f;
-#pragma unroll
-      for (int bb = 0; bb < NB; ++bb)
-        if (bb == b) {
-          y1 = acc1[bb] + half_acc[q][0][bb];
-          y2 = acc2[bb] + half_acc[q][1][bb];
+        for (; i < i1; ++i) {
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(st + (uint32_t)i * 512u, b0, b1, b2, b3);
+          uint4 xv = make_uint4(0u, 0u, 0u, 0u);
+          if (gq < NB) {
+            if constexpr (XG) {
+              const T* xr = xrow + i * 32;
+              xv = make_uint4(ldg_u32(xr), ldg_u32(xr + 8), ldg_u32(xr + 16), ldg_u32(xr + 24));
+            } else {
+              xv = *reinterpret_cast<const uint4*>(xrow + i * 32);
+            }
+          }
+          mma_bf16(d[0], xv.x, 0u, xv.y, 0u, b0, b1);
+          mma_bf16(d[0], xv.z, 0u, xv.w, 0u, b2, b3);
         }
-      if constexpr (EPI == kEpiQkvRope) {
-        const int hidden = a.n_heads * hd;
-        const int sec = p / (hidden / 2), within = p - sec * (hidden / 2);
-        const int h = within / half, e = within - h * half;
-        float o1 = y1, o2 = y2;
-        if (sec < 2) {
-          const float cs = a.rope_cos[(size_t)a.pos * half + e], sn = a.rope_sin[(size_t)a.pos * half + e];
-          o1 = y1 * cs - y2 * sn;
-          o2 = y2 * cs + y1 * sn;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty_bar[stage]);
+        if (++stage == NS) {
+          stage = 0;
+          phase ^= 1u;
         }
-        T* dst = sec == 0 ? static_cast<T*>(a.Q) + (size_t)b * hidden + (size_t)h * hd
-                          : static_cast<T*>(sec == 1 ? a.Kc : a.Vc) + (size_t)b * a.kv_seq_stride +
-                                ((size_t)h * a.Tc + a.pos) * hd;
-        dst[e] = from_f<T>(o1);
-        dst[e + half] = from_f<T>(o2);
-      } else if constexpr (EPI == kEpiSwiglu) {
-        static_cast<T*>(a.G)[(size_t)b * a.ffn + p] = from_f<T>((y1 / (1.0f + expf(-y1))) * y2);
-      } else {
-        float* x = a.Xres + (size_t)b * a.n_out;
-        const float n1 = x[2 * p] + y1, n2 = x[2 * p + 1] + y2;
-        x[2 * p] = n1;
-        x[2 * p + 1] = n2;
-        ssq[0] = fmaf(n1, n1, fmaf(n2, n2, ssq[0]));  // lane b keeps sequence b's sum in ssq[0]
+      }
+      if (aborted) break;
+      // D[gq][2tq], D[gq][2tq+1]: this warp's share of pair tq of sequence gq
+      if (gq < NB)
+        pacc[pb][warp][lane] = make_float2(((d[0][0] + d[1][0]) + d[2][0]) + d[3][0], ((d[0][1] + d[1][1]) + d[2][1]) + d[3][1]);
+      // after this barrier every warp has also finished the previous group's
+      // epilogue, so the other buffer is free for the next group
+      asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
+      if (epi) {
+        float y1 = 0.f, y2 = 0.f;
+#pragma unroll
+        for (int w = 0; w < kNC; ++w) {
+          const float2 v = pacc[pb][w][lane];
+          y1 += v.x;
+          y2 += v.y;
+        }
+        ssq += dgemv_epilogue<T, EPI>(a, p, gq, y1, y2, e1, e2);
       }
     }
-    asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));  // half_acc is reused by the next group
+  } else {
+    const int q = warp >> 1, hk = warp & 1;  // pair within the group, K half
+    const T* xsrc = XG ? static_cast<const T*>(a.xin) : xs;
+    for (int g = g0; g < g1; ++g) {
+      const int p = g * kGP + q;
+      const bool epi = hk == 0 && lane < NB && p < a.n_pairs;
+      float e1 = 0.f, e2 = 0.f;
+      if (epi) dgemv_epilogue_operands<T, EPI>(a, p, lane, e1, e2);
+      float acc1[NB], acc2[NB];
+#pragma unroll
+      for (int b = 0; b < NB; ++b) acc1[b] = acc2[b] = 0.f;
+      for (int c = 0; c < nchunk; ++c) {
+        const int k0 = c * KC, kn = min(KC, K - k0), nv = kn / V;
+        const int v0 = hk ? nv / 2 : 0, v1 = hk ? nv : nv / 2;  // this warp's 16-byte vectors of the rows
+        bool ok = true;
+        if (lane == 0) ok = mbar_wait(&full_bar[stage], phase, kWaitLimit, abort);
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) {
+          if (lane == 0) {
+            set_error(a.err, VLAC_ERR_TIMEOUT);
+            *abort = 1;
+          }
+          aborted = true;
+          break;
+        }
+        const T* st = reinterpret_cast<const T*>(stages + (size_t)stage * stage_b);
+        const uint4* w1 = reinterpret_cast<const uint4*>(st + (size_t)(2 * q) * kn);
+        const uint4* w2 = reinterpret_cast<const uint4*>(st + (size_t)(2 * q + 1) * kn);
+        for (int v = v0 + lane; v < v1; v += 32) {
+          float f1[V], f2[V];
+          unpack<T>(w1[v], f1);
+          unpack<T>(w2[v], f2);
+#pragma unroll
+          for (int b = 0; b < NB; ++b) {
+            float xf[V];
+            unpack<T>(reinterpret_cast<const uint4*>(xsrc + (size_t)b * K + k0)[v], xf);
+#pragma unroll
+            for (int i = 0; i < V; ++i) {
+              acc1[b] = fmaf(f1[i], xf[i], acc1[b]);
+              acc2[b] = fmaf(f2[i], xf[i], acc2[b]);
+            }
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty_bar[stage]);
+        if (++stage == NS) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (aborted) break;
+      // add the two K halves of every pair in order, then the epilogue
+#pragma unroll
+      for (int b = 0; b < NB; ++b) {
+        const float t1 = warp_allsum(acc1[b]), t2 = warp_allsum(acc2[b]);
+        if (hk == 1 && lane == 0) {
+          half_acc[q][0][b] = t1;
+          half_acc[q][1][b] = t2;
+        }
+        acc1[b] = t1;
+        acc2[b] = t2;
+      }
+      asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
+      if (epi) {
+        float y1 = 0.f, y2 = 0.f;
+#pragma unroll
+        for (int bb = 0; bb < NB; ++bb)
+          if (bb == lane) {
+            y1 = acc1[bb] + half_acc[q][0][bb];
+            y2 = acc2[bb] + half_acc[q][1][bb];
+          }
+        ssq += dgemv_epilogue<T, EPI>(a, p, lane, y1, y2, e1, e2);
+      }
+      asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));  // half_acc is reused by the next group
+    }
   }
   if constexpr (EPI == kEpiResid) {
-    if (lane < NB) red[warp][lane] = (hk == 0) ? ssq[0] : 0.f;
+    // per thread: sequence gq = lane/4 (bf16) or lane (fp32); summed over the
+    // warps and then the lanes of a sequence in a fixed order
+    red[warp][lane] = ssq;
     asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
     if (tid < NB) {
       float t = 0.f;
-      for (int w = 0; w < kNC; ++w) t += red[w][tid];
+      for (int w = 0; w < kNC; ++w) {
+        if constexpr (kMma) {
+          for (int j = 0; j < 4; ++j) t += red[w][tid * 4 + j];
+        } else {
+          t += red[w][tid];
+        }
+      }
       a.ssq_out[(size_t)tid * gridDim.x + blockIdx.x] = t;
     }
   }
@@ -580,11 +811,175 @@ __global__ void __launch_bounds__(64) dec_attn_kernel(const T* __restrict__ Q, c
   if (threadIdx.x == 0) counters[b * n_heads + h] = 0u;  // ready for the next launch
 }
 
+// Cluster variant (bf16, up to 8 blocks of 128 keys): the blocks of one
+// (sequence, head) form a thread-block cluster.  K and V rows of the keys
+// before `pos` were written by earlier passes, so they are requested before
+// the dependency wait and arrive while the preceding QKV projection drains;
+// only Q and the new key's row wait for it.  Each block leaves its partial
+// in its own shared memory; block 0 of the cluster reads them over
+// distributed shared memory in chunk order and writes the output.
+constexpr int kDcW = 4;             // warps per block, 32 keys each
+constexpr int kDcKeys = kDcW * 32;  // keys per block
+constexpr int kDcMaxCluster = 8;    // portable cluster size
+
+template <int HD>
+__global__ void __launch_bounds__(kDcW * 32) dec_attn_cluster_kernel(const bf16* __restrict__ Q,
+                                                                     const bf16* __restrict__ Kc,
+                                                                     const bf16* __restrict__ Vc,
+                                                                     size_t kv_seq_stride, int Tc, int pos,
+                                                                     int n_heads, float scale, bf16* __restrict__ O) {
+  using T = bf16;
+  constexpr int EPL = HD / 32, V = Vec<T>::n, CPR = HD * (int)sizeof(T) / 16;  // 16-byte chunks per row
+  __shared__ __align__(16) T vbuf_all[kDcW][32][HD];
+  __shared__ float qs[HD];
+  __shared__ float wm[kDcW], wl[kDcW];
+  __shared__ float wacc[kDcW][HD];
+  __shared__ float cpart[HD + 2];  // this block's (max, sum, output row)
+  namespace cg = cooperative_groups;
+  cg::cluster_group cluster = cg::this_cluster();
+  const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z, n_kc = gridDim.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int hidden = n_heads * HD;
+  T* vbuf = &vbuf_all[warp][0][0];
+  const T* Kh = Kc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
+  const T* Vh = Vc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
+  const int nkeys = min(pos + 1, Tc);
+  const int k1 = min(nkeys, (c + 1) * kDcKeys);
+  const int j0 = c * kDcKeys + warp * 32, jn = max(0, min(32, k1 - j0)), j = j0 + lane;
+  // ---- before the dependency wait: the rows of the older keys ----
+  for (int q = lane; q < jn * CPR; q += 32) {
+    const int jj = q / CPR, r = q - jj * CPR;
+    if (j0 + jj != pos)
+      cp_async16(vbuf + (size_t)jj * HD + r * (16 / sizeof(T)), Vh + (size_t)(j0 + jj) * HD + r * (16 / sizeof(T)));
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+  uint4 kr[HD / V];
+  if (lane < jn && j != pos) {
+    const uint4* src = reinterpret_cast<const uint4*>(Kh + (size_t)j * HD);
+#pragma unroll
+    for (int v = 0; v < HD / V; ++v) kr[v] = src[v];
+  }
+  pdl_wait();
+  pdl_trigger();
+  // ---- the query and the new key's row ----
+  if (lane < jn && j == pos) {
+    const uint4* src = reinterpret_cast<const uint4*>(Kh + (size_t)j * HD);
+#pragma unroll
+    for (int v = 0; v < HD / V; ++v) kr[v] = src[v];
+  }
+  if (pos >= j0 && pos < j0 + jn)
+    for (int r = lane; r < CPR; r += 32)
+      cp_async16(vbuf + (size_t)(pos - j0) * HD + r * (16 / sizeof(T)), Vh + (size_t)pos * HD + r * (16 / sizeof(T)));
+  asm volatile("cp.async.commit_group;" ::: "memory");
+  for (int e = threadIdx.x; e < HD; e += blockDim.x) qs[e] = to_f(Q[(size_t)b * hidden + (size_t)h * HD + e]);
+  __syncthreads();
+  float m_run = -INFINITY, l_run = 0.f, acc[EPL];
+#pragma unroll
+  for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
+  if (jn > 0) {
+    float sc = -INFINITY;
+    if (lane < jn) {
+      float d = 0.f;
+#pragma unroll
+      for (int v = 0; v < HD / V; ++v) {
+        float f[V];
+        unpack<T>(kr[v], f);
+#pragma unroll
+        for (int i = 0; i < V; ++i) d = fmaf(f[i], qs[v * V + i], d);
+      }
+      sc = d * scale;
+    }
+    m_run = warp_max(sc);
+    const float p = (sc == -INFINITY) ? 0.f : expf(sc - m_run);
+    l_run = warp_sum(p);
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncwarp();
+#pragma unroll 8
+    for (int jj = 0; jj < jn; ++jj) {
+      const float pj = __shfl_sync(0xffffffffu, p, jj);
+      const T* vr = vbuf + (size_t)jj * HD + lane * EPL;
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) acc[e] = fmaf(pj, to_f(vr[e]), acc[e]);
+    }
+  }
+  if (lane == 0) {
+    wm[warp] = m_run;
+    wl[warp] = l_run;
+  }
+#pragma unroll
+  for (int e = 0; e < EPL; ++e) wacc[warp][lane * EPL + e] = acc[e];
+  __syncthreads();
+  {
+    float M = -INFINITY;
+    for (int w = 0; w < kDcW; ++w) M = fmaxf(M, wm[w]);
+    for (int e = threadIdx.x; e < HD; e += blockDim.x) {
+      float L = 0.f, o = 0.f;
+      for (int w = 0; w < kDcW; ++w) {
+        const float f = (wm[w] == -INFINITY) ? 0.f : expf(wm[w] - M);
+        L = fmaf(wl[w], f, L);
+        o = fmaf(wacc[w][e], f, o);
+      }
+      cpart[2 + e] = o;
+      if (e == 0) {
+        cpart[0] = M;
+        cpart[1] = L;
+      }
+    }
+  }
+  cluster.sync();
+  if (cluster.block_rank() == 0) {
+    float M = -INFINITY;
+    for (int q = 0; q < n_kc; ++q) M = fmaxf(M, *cluster.map_shared_rank(&cpart[0], q));
+    for (int e = threadIdx.x; e < HD; e += blockDim.x) {
+      float L = 0.f, o = 0.f;
+      for (int q = 0; q < n_kc; ++q) {
+        const float* rp = cluster.map_shared_rank(&cpart[0], q);
+        const float f = (rp[0] == -INFINITY) ? 0.f : expf(rp[0] - M);
+        L = fmaf(rp[1], f, L);
+        o = fmaf(rp[2 + e], f, o);
+      }
+      O[(size_t)b * hidden + (size_t)h * HD + e] = from_f<T>(o / L);
+    }
+  }
+  cluster.sync();  // every block's partial stays in place until block 0 has read it
+}
+
+template <int HD>
+void launch_dec_attn_cluster(int B, int n_heads, int n_kc, const bf16* Q, const bf16* Kc, const bf16* Vc,
+                             size_t kv_seq_stride, int Tc, int pos, float scale, bf16* O, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(n_kc, n_heads, B);
+  cfg.blockDim = dim3(kDcW * 32);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = n_kc;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = g_pdl ? 2 : 1;
+  cudaLaunchKernelEx(&cfg, dec_attn_cluster_kernel<HD>, Q, Kc, Vc, kv_seq_stride, Tc, pos, n_heads, scale, O);
+}
+
 template <typename T>
 void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride,
                           int Tc, int pos, float* part, unsigned* counters, T* O, cudaStream_t st) {
   const float scale = 1.0f / sqrtf((float)head_dim);
-  const int n_kc = (std::min(pos + 1, Tc) + kDecKeys - 1) / kDecKeys;
+  const int nkeys = std::min(pos + 1, Tc);
+  if constexpr (sizeof(T) == 2) {
+    const int n_kc = (nkeys + kDcKeys - 1) / kDcKeys;
+    if (n_kc <= kDcMaxCluster && (head_dim == 128 || head_dim == 64)) {
+      if (head_dim == 128)
+        launch_dec_attn_cluster<128>(B, n_heads, n_kc, Q, Kc, Vc, kv_seq_stride, Tc, pos, scale, O, st);
+      else
+        launch_dec_attn_cluster<64>(B, n_heads, n_kc, Q, Kc, Vc, kv_seq_stride, Tc, pos, scale, O, st);
+      return;
+    }
+  }
+  const int n_kc = (nkeys + kDecKeys - 1) / kDecKeys;
   const dim3 grid(n_kc, n_heads, B);
   if (head_dim == 128)
     launch_k(dec_attn_kernel<T, 128>, grid, dim3(kDecKeys), 0, st, Q, Kc, Vc, kv_seq_stride, Tc, pos, n_heads, scale,
@@ -611,7 +1006,7 @@ __global__ void __launch_bounds__(256) head_logits_kernel(const float* __restric
                                                           float* __restrict__ logits_ws) {
   pdl_wait();
   pdl_trigger();
-  extern __shared__ __align__(16) uint8_t dsm[];
+  extern __shared__ __align__(1024) uint8_t dsm[];
   T* xs = reinterpret_cast<T*>(dsm);
   const int j = blockIdx.y, b = blockIdx.z;
   const int row = row_of_seq ? row_of_seq[b] + j : j;

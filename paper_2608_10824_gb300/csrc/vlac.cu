@@ -46,7 +46,9 @@ struct vlac_ctx {
   size_t esz;
   int dev;
   int n_sm = 1;
-  int gemv_ns = 6;  // decode-GEMV weight ring stages (32 KB each)
+  int gemv_ns = 4;  // decode-GEMV weight ring stages (32 KB each)
+  int gemv_pre = 0;  // decode-GEMV stages streamed ahead of the input-vector prologue (0: the whole ring)
+  int gemv_pf_kb = 128;  // decode-GEMV L2 prefetch of the next projection, KB per CTA
   char* dmem = nullptr;  // decode-streaming copies of the projections
   std::vector<void*> dqkv, dwo, dgu, dwd;
   // weights
@@ -204,6 +206,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (const char* e = std::getenv("VLAC_PDL")) g_pdl = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_GRAPH")) c->use_graph = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_GEMV_NS")) c->gemv_ns = std::max(2, std::min(24, std::atoi(e)));
+  if (const char* e = std::getenv("VLAC_GEMV_PRE")) c->gemv_pre = std::max(0, std::atoi(e));
+  if (const char* e = std::getenv("VLAC_GEMV_PF_KB")) c->gemv_pf_kb = std::max(0, std::atoi(e));
   c->d = *dims;
   const vlac_dims& d = c->d;
   c->bf16 = d.dtype == VLAC_BF16;
@@ -561,9 +565,10 @@ template <typename T>
 void dgemv(vlac_ctx* c, const DGemv& a_in, int epi, int nb, cudaStream_t st) {
   DGemv a = a_in;
   a.ns = c->gemv_ns;
-  // the stage ring (32 KB stages) must fit next to the input vector in shared memory
+  a.pre = c->gemv_pre;
+  // the stage ring must fit next to the input vector in shared memory
   const size_t xs = ((size_t)nb * a.K * sizeof(T) + 1023) / 1024 * 1024;
-  while (a.ns > 2 && (size_t)a.ns * 32 * 1024 + (xs > 64 * 1024 ? 0 : xs) > 200 * 1024) --a.ns;
+  while (a.ns > 2 && (size_t)a.ns * dgemv_stage_bytes() + (xs > 64 * 1024 ? 0 : xs) > 200 * 1024) --a.ns;
   ProfScope ps(c, VLAC_PROF_DECODE_GEMV,
                (double)2 * a.n_pairs * a.K * sizeof(T) + (double)nb * a.K * sizeof(T) + (double)nb * 2 * a.n_pairs * 4,
                st);
@@ -706,7 +711,8 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         g.pf_K = Kn;
         g.pf_pairs = pairs;
         g.pf_grid = dgemv_grid(pairs, c->n_sm);
-        g.pf_bytes = 128 * 1024;
+        g.pf_bytes = (uint32_t)c->gemv_pf_kb * 1024;
+        if (!g.pf_bytes) g.pf_W = nullptr;
       };
       for (int l = 0; l < L; ++l) {
         DGemv g{};

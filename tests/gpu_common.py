@@ -14,11 +14,19 @@ import synth
 # forcing the oracle's branch).
 LOGIT_TOL = {"bf16": 2e-2, "f32": 1e-3}
 # Full 32-layer 7B shapes: two runs of the GPU path that differ only in the
-# fp32 summation order of the GEMM partial sums differ by up to 3.4e-2 in the
+# fp32 summation order of the GEMM partial sums differ by up to 4.2e-2 in the
 # logits (the bf16 re-rounding of every layer's GEMM inputs amplifies any
-# fp32-level difference), so the bar there is twice that measured floor.
-LOGIT_TOL_DEEP = 7e-2
+# fp32-level difference; the figure moves with every change of summation
+# order, 3.4e-2 to 4.2e-2 so far), so the bar there is about twice the
+# largest measured floor.
+LOGIT_TOL_DEEP = 1e-1
 ID_EXEMPT_MARGIN = 1e-3
+# At that depth an argmax flips wherever the oracle's two candidate logits
+# are closer than the logit error can move them apart: with every logit
+# within LOGIT_TOL_DEEP, a differing id is only possible where the oracle's
+# logit for its own bin exceeds its logit for the GPU's bin by less than
+# twice the bar.  The deep tests exempt exactly those ids, and require the
+# GPU's id to be the first maximum of the GPU's own logits.
 FLAG_TIE = 1e-4
 
 SMALL = {
@@ -109,8 +117,15 @@ def compare(d, o, g, prev_m, tau_m, logit_tol=None):
     assert diff.max() <= tol, f"logits differ by {diff.max():.3e} > {tol}"
     mism = g["action_ids"] != o["action_ids"]
     exempt = o["margins"] < ID_EXEMPT_MARGIN
+    if logit_tol is not None:
+        gl = g["logits"].astype(np.float64)
+        np.testing.assert_array_equal(np.argmax(gl, axis=-1), g["action_ids"], err_msg="GPU id vs GPU logits")
+        o_own = np.take_along_axis(o["logits"], o["action_ids"][..., None].astype(np.int64), -1)[..., 0]
+        o_gpu = np.take_along_axis(o["logits"], g["action_ids"][..., None].astype(np.int64), -1)[..., 0]
+        exempt = exempt | (o_own - o_gpu < 2 * logit_tol)
     bad = mism & ~exempt
-    assert not bad.any(), f"action ids differ outside the exemption: {np.argwhere(bad)}"
+    assert not bad.any(), (f"action ids differ outside the exemption: {np.argwhere(bad)}, "
+                           f"oracle margins {o['margins'][bad]}")
     np.testing.assert_allclose(g["margins"], o["margins"], atol=max(tol * 0.05, 1e-6), rtol=0.05)
     return {"max_logit_diff": float(diff.max()), "id_mismatch": int(mism.sum()),
             "id_exempt": int(exempt.sum()), "recomputed": o["recomputed"].tolist()}

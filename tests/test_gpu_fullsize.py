@@ -137,6 +137,7 @@ def test_summation_order_floor(cuda_device):
             os.environ["VLAC_SPLITS"] = old
     floor = np.abs(logits[0] - logits[1]).max()
     dist = max(np.abs(lg - o["logits"]).max() for lg in logits)
+    print(f"summation-order floor {floor:.4e}, oracle distance {dist:.4e}")
     assert 2e-3 < floor <= LOGIT_TOL_DEEP / 2, floor
     assert dist <= LOGIT_TOL_DEEP, (dist, floor)
     del w_gpu
