@@ -20,7 +20,8 @@ namespace tc {
 constexpr int kBM = 128;        // weight rows per CTA (MMA M)
 constexpr int kBK = 64;         // K elements per stage = one 128-byte swizzle row
 constexpr int kBoxRows = 32;    // granularity of the activation operand's token rows (boxes of 32..256 rows)
-constexpr int kMaxTok = 512;    // token columns per pass (TMEM has 512 fp32 columns)
+constexpr int kMaxTok = 256;    // token columns per pass when several passes are needed
+constexpr int kOnePass = 384;   // up to this many tokens run in one pass (split accumulator chains)
 constexpr int kMaxStages = 8;
 constexpr int kWTileBytes = kBM * kBK * 2;  // 16 KB
 constexpr int kSmemBytes = 212 * 1024;      // dynamic shared memory (tiles only)
@@ -127,13 +128,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int kc1 = min(kc0 + chunks_per_split, k_chunks);
   const int nk = kc1 - kc0;
   if (nk <= 0) return;
-  const int tok_layout = ((min(M, kMaxTok) + kBoxRows - 1) / kBoxRows) * kBoxRows;
+  // token passes: one pass up to kOnePass tokens, else passes of kMaxTok
+  // (every pass streams the weight tile again)
+  const int pass_tok = M <= kOnePass ? M : kMaxTok;
+  const int tok_layout = ((min(M, pass_tok) + kBoxRows - 1) / kBoxRows) * kBoxRows;
   const uint32_t stage_bytes = kWTileBytes + (uint32_t)tok_layout * 128u;
   const int n_stages = min(kMaxStages, (int)((kSmemBytes - 1024) / stage_bytes));
-  const int n_pass = (M + kMaxTok - 1) / kMaxTok;
-  // independent accumulator chains: MMAs into one accumulator serialise, so
-  // short token sets spread the K steps over 2 or 4 accumulators
+  const int n_pass = (M + pass_tok - 1) / pass_tok;
+  // independent accumulator chains: consecutive MMAs into one accumulator
+  // serialise, so the K steps alternate between C accumulators (4 for up to
+  // 128 tokens, 2 for up to 256).  Above 256 tokens the 512 TMEM columns do
+  // not hold two chains of every token: the first `split` tokens get two
+  // chains and the rest one (split + tok_layout <= 512 columns).
   const int C = tok_layout <= 128 ? 4 : tok_layout <= 256 ? 2 : 1;
+  const int split = C == 1 ? ((512 - tok_layout) / kBoxRows) * kBoxRows : 0;
   const uint32_t ncols = 512;
 
   if (threadIdx.x == 0) {
@@ -168,8 +176,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0;
       uint32_t phase = 0;
       for (int pass = 0; pass < n_pass && !*abort; ++pass) {
-        const int row0 = pass * kMaxTok;
-        const int rows = min(M - row0, kMaxTok);
+        const int row0 = pass * pass_tok;
+        const int rows = min(M - row0, pass_tok);
         const int nbox = (rows + kBoxRows - 1) / kBoxRows;
         for (int kc = kc0; kc < kc1; ++kc) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, wait_limit, abort)) {
@@ -204,7 +212,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0;
       uint32_t phase = 0;
       for (int pass = 0; pass < n_pass && !*abort; ++pass) {
-        const int rows = min(M - pass * kMaxTok, kMaxTok);
+        const int rows = min(M - pass * pass_tok, pass_tok);
         if (pass > 0 && !mbar_wait(&acc_empty, (uint32_t)(pass - 1) & 1u, wait_limit, abort)) {
           set_error(err, VLAC_ERR_TIMEOUT);
           *abort = 1;
@@ -224,7 +232,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k16 = 0; k16 < kBK / 16; ++k16) {
             const uint64_t adesc = sw128_desc(wt + k16 * 32);
-            if (C > 1) {
+            if (split > 0) {
+              // tokens [0, split): chain k16 % 2; tokens [split, rows): one chain
+              umma_bf16(tmem_base + (k16 & 1) * split, adesc, sw128_desc(at + k16 * 32), idesc_bf16(split),
+                        (i > 0 || k16 >= 2) ? 1u : 0u);
+              const int nr = ((rows - split + 15) / 16) * 16;
+              umma_bf16(tmem_base + 2 * split, adesc, sw128_desc(at + split * 128 + k16 * 32), idesc_bf16(nr),
+                        (i > 0 || k16 > 0) ? 1u : 0u);
+            } else if (C > 1) {
               // chain k16 % C accumulates every C-th K step
               const int n = ((rows + 15) / 16) * 16;
               const uint64_t bdesc = sw128_desc(at + k16 * 32);
@@ -258,8 +273,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int n = n0 + q * 32 + lane;
     float* dst = out + (size_t)blockIdx.y * split_stride;
     for (int pass = 0; pass < n_pass; ++pass) {
-      const int row0 = pass * kMaxTok;
-      const int rows = min(M - row0, kMaxTok);
+      const int row0 = pass * pass_tok;
+      const int rows = min(M - row0, pass_tok);
       bool ok = true;
       if (lane == 0) ok = mbar_wait(&acc_full, (uint32_t)pass & 1u, wait_limit, abort);
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -273,7 +288,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_after();
       for (int c0 = 0; c0 < rows; c0 += 16) {
         float v[16];
-        tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, v);
+        const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16);
+        if (split > 0) {
+          if (c0 < split) {  // the two chains, in order
+            float w[16];
+            tmem_ld16(lane_base + (uint32_t)c0, v);
+            tmem_ld16(lane_base + (uint32_t)(split + c0), w);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) v[j] += w[j];
+          } else {
+            tmem_ld16(lane_base + (uint32_t)(2 * split + (c0 - split)), v);
+          }
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int m = row0 + c0 + j;
+            if (m < M) dst[(size_t)m * N + n] = v[j];
+          }
+          continue;
+        }
+        tmem_ld16(lane_base + (uint32_t)c0, v);
         for (int ch = 1; ch < C; ++ch) {  // chains added in order
           float w[16];
           tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ch * tok_layout + c0), w);

@@ -42,6 +42,11 @@ SMALL = {
     "small_batch": synth.Dims(n_layers=2, hidden=256, n_heads=2, head_dim=128, ffn=768, vocab=1024, n_bins=256,
                               img_h=112, img_w=112, patch=14, n_views=1, n_text=8, proprio_dim=0, n_action=7,
                               parallel=0, dtype="bf16", max_batch=3),
+    # bf16, MLP width 4160: the down-projection's K (4160) spans three
+    # 2048-element decode-GEMV chunks (the last one 64 elements); two sequences
+    "small_wide": synth.Dims(n_layers=2, hidden=256, n_heads=2, head_dim=128, ffn=4160, vocab=1024, n_bins=256,
+                             img_h=112, img_w=112, patch=14, n_views=1, n_text=8, proprio_dim=0, n_action=7,
+                             parallel=0, dtype="bf16", max_batch=2),
     # fp32 tiny model (SIMT path)
     "tiny": synth.dims_for("tiny"),
 }

@@ -42,6 +42,19 @@ def test_scene_frames_parity(cuda_device):
     assert g["static_mask"].sum() > d.n_visual // 2
 
 
+def test_multi_chunk_parity(cuda_device):
+    """Decode GEMV over a K of several chunks with a ragged last chunk, one
+    and two sequences."""
+    d = SMALL["small_wide"]
+    w = synth.make_weights(d, seed=10)
+    for B in (1, 2):
+        ls = Lockstep(d, w, batch=B)
+        frames, prompt, _ = episode(d, 3, seed=6, batch=B)
+        pm = synth.linear_schedule(d.n_layers)
+        for t in range(3):
+            ls.step(frames[t], prompt, None, (95, 100), 0.0, pm)
+
+
 def test_batch_parity(cuda_device):
     d = SMALL["small_batch"]
     w = synth.make_weights(d, seed=9)
