@@ -40,7 +40,7 @@ CPU_LAYERS = 2  # the CPU oracle sample runs this many of the 32 layers
 # averaged over the four projections of a decode layer, from one ncu capture
 # of the current kernel (profiles/dgemv_openvla7b_decode_layer.txt; it counts
 # the L2 prefetch of the next projection twice, as ncu flushes the caches)
-DGEMV_TRAFFIC_PER_LAUNCH = {}  # none yet for the tensor-pipe consumer version of the kernel
+DGEMV_TRAFFIC_PER_LAUNCH = {"openvla7b": 120.6e6, "layer7b": 120.6e6}
 
 
 def peaks():
