@@ -114,6 +114,10 @@ __device__ __forceinline__ float4 sum_splits4(const float* __restrict__ part, in
 
 // ---- RMSNorm ----------------------------------------------------------------
 
+// Threads of a row-normalising block: one float4 of a 4096-wide row each, so
+// that all of a row's loads are in flight at once.
+constexpr int kNormThreads = 1024;
+
 // y = T((x * r) * g), r = 1 / sqrt(mean(x^2) + eps); `ss` is this thread's part
 // of sum(x^2).  One block per row.
 template <typename T>
@@ -183,7 +187,10 @@ __global__ void qkv_epilogue_kernel(Rows rows, int n_heads, int head_dim, const 
   const int hidden = n_heads * head_dim, half = head_dim / 2, N = 3 * hidden, q4 = half / 4;
   const float* pr = part + (size_t)r * N;
   T* q_out = Q + (size_t)r * hidden;
-  for (int t = threadIdx.x; t < n_heads * q4; t += blockDim.x) {
+  // gridDim.z blocks share a row
+  const int nt = n_heads * q4, t0 = (int)(((long long)nt * blockIdx.z) / gridDim.z);
+  const int t1 = (int)(((long long)nt * (blockIdx.z + 1)) / gridDim.z);
+  for (int t = t0 + threadIdx.x; t < t1; t += blockDim.x) {
     const int h = t / q4, e = 4 * (t - h * q4);
     const float4 c = *reinterpret_cast<const float4*>(rope_cos + (size_t)pos * half + e);
     const float4 s = *reinterpret_cast<const float4*>(rope_sin + (size_t)pos * half + e);
@@ -242,8 +249,11 @@ __global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part
   if (i >= cnt) return;
   const int r = rows.off[b] + i;
   const float* pr = part + (size_t)r * 2 * ffn;
+  // gridDim.z blocks share a row, so that enough loads are in flight
+  const int n4 = ffn / 4, c0 = (int)(((long long)n4 * blockIdx.z) / gridDim.z);
+  const int c1 = (int)(((long long)n4 * (blockIdx.z + 1)) / gridDim.z);
 #pragma unroll 4
-  for (int c = threadIdx.x; c < ffn / 4; c += blockDim.x) {
+  for (int c = c0 + threadIdx.x; c < c1; c += blockDim.x) {
     const float4 g = sum_splits4(pr, splits, split_stride, 4 * (size_t)c);
     const float4 u = sum_splits4(pr, splits, split_stride, (size_t)ffn + 4 * c);
     store4<T>(G + (size_t)r * ffn + 4 * c,
@@ -263,8 +273,11 @@ __global__ void residual_kernel(Rows rows, int hidden, const float* __restrict__
   const int r = rows.off[b] + i;
   float* x = rows.X + ((size_t)b * rows.idx_stride + i) * hidden;
   const float* pr = part + (size_t)r * hidden;
+  // gridDim.z blocks share a row, so that enough loads are in flight
+  const int n4 = hidden / 4, c0 = (int)(((long long)n4 * blockIdx.z) / gridDim.z);
+  const int c1 = (int)(((long long)n4 * (blockIdx.z + 1)) / gridDim.z);
 #pragma unroll 4
-  for (int c = threadIdx.x; c < hidden / 4; c += blockDim.x)
+  for (int c = c0 + threadIdx.x; c < c1; c += blockDim.x)
     reinterpret_cast<float4*>(x)[c] =
         add4(reinterpret_cast<const float4*>(x)[c], sum_splits4(pr, splits, split_stride, 4 * (size_t)c));
 }
@@ -373,29 +386,29 @@ void launch_embed(Rows rows, int B, int S, int hidden, int Nv, int P, int has_pr
 template <typename T>
 void launch_layer_in(Rows rows, const int* off_prev, int B, int S, int hidden, float* H, size_t h_seq_stride,
                      const T* gain, float eps, T* A, cudaStream_t st) {
-  launch_k(layer_in_kernel<T>, dim3(S, B), dim3(256), 0, st, rows, off_prev, hidden, H, h_seq_stride, gain, eps, A);
+  launch_k(layer_in_kernel<T>, dim3(S, B), dim3(kNormThreads), 0, st, rows, off_prev, hidden, H, h_seq_stride, gain, eps, A);
 }
 template <typename T>
 void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, int splits,
                          size_t split_stride, const float* rope_cos, const float* rope_sin, T* Q, T* Kc, T* Vc,
                          size_t kv_seq_stride, int Tc, cudaStream_t st) {
-  launch_k(qkv_epilogue_kernel<T>, dim3(S, B), dim3(256), 0, st, rows, n_heads, head_dim, part, splits, split_stride,
+  launch_k(qkv_epilogue_kernel<T>, dim3(S, B, 2), dim3(256), 0, st, rows, n_heads, head_dim, part, splits, split_stride,
            rope_cos, rope_sin, Q, Kc, Vc, kv_seq_stride, Tc);
 }
 template <typename T>
 void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part, int splits, size_t split_stride,
                           const T* gain, float eps, T* A, cudaStream_t st) {
-  launch_k(residual_norm_kernel<T>, dim3(S, B), dim3(256), 0, st, rows, hidden, part, splits, split_stride, gain, eps,
+  launch_k(residual_norm_kernel<T>, dim3(S, B), dim3(kNormThreads), 0, st, rows, hidden, part, splits, split_stride, gain, eps,
            A);
 }
 template <typename T>
 void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, int splits, size_t split_stride, T* G,
                    cudaStream_t st) {
-  launch_k(swiglu_kernel<T>, dim3(S, B), dim3(256), 0, st, rows, ffn, part, splits, split_stride, G);
+  launch_k(swiglu_kernel<T>, dim3(S, B, 4), dim3(256), 0, st, rows, ffn, part, splits, split_stride, G);
 }
 void launch_residual(Rows rows, int B, int S, int hidden, const float* part, int splits, size_t split_stride,
                      cudaStream_t st) {
-  launch_k(residual_kernel, dim3(S, B), dim3(256), 0, st, rows, hidden, part, splits, split_stride);
+  launch_k(residual_kernel, dim3(S, B, 4), dim3(256), 0, st, rows, hidden, part, splits, split_stride);
 }
 template <typename T>
 void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
