@@ -48,7 +48,7 @@ struct vlac_ctx {
   int n_sm = 1;
   int gemv_ns = 4;  // decode-GEMV weight ring stages (32 KB each)
   int gemv_pre = 0;  // decode-GEMV stages streamed ahead of the input-vector prologue (0: the whole ring)
-  int gemv_pf_kb = 128;  // decode-GEMV L2 prefetch of the next projection, KB per CTA
+  int gemv_pf_kb = 0;  // decode-GEMV L2 prefetch of the next projection, KB per CTA (measured: off is best)
   char* dmem = nullptr;  // decode-streaming copies of the projections
   std::vector<void*> dqkv, dwo, dgu, dwd;
   // weights
