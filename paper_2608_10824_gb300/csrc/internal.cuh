@@ -65,7 +65,6 @@ struct DGemv {
   float* ssq_out;       // residual GEMV: this launch's per-CTA sums of squares [nb][grid]
   int* err;             // device error word (bounded waits)
   int ns;               // stages of the weight ring
-  int pre;              // stages streamed before the input vector is ready (0: no limit)
   // the next decode GEMV of the stream: this CTA pulls the start of that
   // kernel's CTA region into L2 once its own loads are issued
   const void* pf_W;

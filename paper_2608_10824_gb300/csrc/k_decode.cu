@@ -256,7 +256,6 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
   extern __shared__ __align__(1024) uint8_t dsm[];
   __shared__ __align__(8) uint64_t full_bar[kMaxNS];
   __shared__ __align__(8) uint64_t empty_bar[kMaxNS];
-  __shared__ __align__(8) uint64_t ready_bar;  // the input vector is in place (limits the early stream)
   __shared__ float red[kNC][32];
   __shared__ float rr[NB];
   __shared__ __align__(8) float2 pacc[2][kNC][32];  // bf16 path: per-warp partials, two groups in flight
@@ -275,7 +274,6 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], kNC);
     }
-    mbar_init(&ready_bar, 1);
     abort_flag = 0;
     mbar_fence_init();
   }
@@ -285,17 +283,12 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
   if (warp == kNC) {
     // ---- producer: weights only, so it runs ahead of the dependency wait ----
     if (lane == 0) {
-      int stage = 0, issued = 0;
+      int stage = 0;
       uint32_t phase = 0;
       for (int g = g0; g < g1 && !*abort; ++g) {
         const T* gbase = Wt + (size_t)g * TR * K;
         for (int c = 0; c < nchunk; ++c) {
           const int kn = min(KC, K - c * KC);
-          if (issued++ == a.pre && a.pre > 0 && !mbar_wait(&ready_bar, 0, kWaitLimit, abort)) {
-            set_error(a.err, VLAC_ERR_TIMEOUT);
-            *abort = 1;
-            break;
-          }
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, kWaitLimit, abort)) {
             set_error(a.err, VLAC_ERR_TIMEOUT);
             *abort = 1;
@@ -434,7 +427,6 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
     }
   }
   asm volatile("bar.sync 1, %0;" ::"r"(kNC * 32));
-  if (tid == 0) mbar_arrive(&ready_bar);
 
   float ssq = 0.f;  // residual epilogue: this thread's sum of squares (sequence per lane, see below)
   bool aborted = false;

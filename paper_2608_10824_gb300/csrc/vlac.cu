@@ -47,7 +47,6 @@ struct vlac_ctx {
   int dev;
   int n_sm = 1;
   int gemv_ns = 4;  // decode-GEMV weight ring stages (32 KB each)
-  int gemv_pre = 0;  // decode-GEMV stages streamed ahead of the input-vector prologue (0: the whole ring)
   int gemv_pf_kb = 0;  // decode-GEMV L2 prefetch of the next projection, KB per CTA (measured: off is best)
   char* dmem = nullptr;  // decode-streaming copies of the projections
   std::vector<void*> dqkv, dwo, dgu, dwd;
@@ -206,7 +205,6 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (const char* e = std::getenv("VLAC_PDL")) g_pdl = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_GRAPH")) c->use_graph = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_GEMV_NS")) c->gemv_ns = std::max(2, std::min(24, std::atoi(e)));
-  if (const char* e = std::getenv("VLAC_GEMV_PRE")) c->gemv_pre = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("VLAC_GEMV_PF_KB")) c->gemv_pf_kb = std::max(0, std::atoi(e));
   c->d = *dims;
   const vlac_dims& d = c->d;
@@ -565,7 +563,6 @@ template <typename T>
 void dgemv(vlac_ctx* c, const DGemv& a_in, int epi, int nb, cudaStream_t st) {
   DGemv a = a_in;
   a.ns = c->gemv_ns;
-  a.pre = c->gemv_pre;
   // the stage ring must fit next to the input vector in shared memory
   const size_t xs = ((size_t)nb * a.K * sizeof(T) + 1023) / 1024 * 1024;
   while (a.ns > 2 && (size_t)a.ns * dgemv_stage_bytes() + (xs > 64 * 1024 ? 0 : xs) > 200 * 1024) --a.ns;
