@@ -65,8 +65,9 @@ struct DGemv {
   float* ssq_out;       // residual GEMV: this launch's per-CTA sums of squares [nb][grid]
   int* err;             // device error word (bounded waits)
   int ns;               // stages of the weight ring
-  // the next decode GEMV of the stream: this CTA pulls the start of that
-  // kernel's CTA region into L2 once its own loads are issued
+  // optional (pf_W null: off): the next decode GEMV of the stream; this CTA
+  // pulls the start of that kernel's CTA region into L2 once its own loads
+  // are issued
   const void* pf_W;
   int pf_K, pf_pairs, pf_grid;
   uint32_t pf_bytes;

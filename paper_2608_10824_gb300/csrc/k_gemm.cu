@@ -1,13 +1,13 @@
-// Projections of the layer loop: out[s][m][n] = sum_k A[m][k] * W[n][k] over
-// the k range of split s.  Three kernels, one per regime:
-//   - gemm_tc:   bf16 prefix pass (M = recomputed rows, device-resident),
-//                tcgen05 MMA with fp32 accumulators in TMEM, operands staged
-//                by TMA into 128B-swizzled shared memory.  The weight tile is
-//                the 128-row MMA operand and the token rows are the N side
-//                ("swap-AB"), so one weight tile feeds every recomputed row.
-//   - gemv:      decode passes (M = batch <= 8): HBM-bound weight streaming
-//                with 16-byte non-allocating loads and fp32 FMAs.
+// Projections of the prefix pass: out[s][m][n] = sum_k A[m][k] * W[n][k] over
+// the k range of split s.  Two kernels:
+//   - gemm_tc:   bf16 (M = recomputed rows, device-resident), tcgen05 MMA
+//                with fp32 accumulators in TMEM, operands staged by TMA into
+//                128B-swizzled shared memory.  The weight tile is the 128-row
+//                MMA operand and the token rows are the N side ("swap-AB"), so
+//                one weight tile feeds every recomputed row.
 //   - gemm_simt: the fp32 tiny model.
+// The decode passes (M = batch <= 8) use the fused weight-streaming GEMV in
+// k_decode.cu.
 #include "internal.cuh"
 
 namespace vlac {

@@ -702,7 +702,8 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
                                c->idx_dec, c->ssq_b, c->err, st);
       }
       c->launches += 1;
-      // prefetch chain: each GEMV pulls the start of the next one's weights into L2
+      // optional prefetch chain (VLAC_GEMV_PF_KB, off by default): each GEMV
+      // pulls the start of the next one's weights into L2
       auto set_pf = [&](DGemv& g, const void* Wn, int Kn, int pairs) {
         g.pf_W = Wn;
         g.pf_K = Kn;
