@@ -130,6 +130,16 @@ constexpr int kGP = 4;          // row pairs per group
 constexpr int kMaxNS = 24;      // stage ring capacity
 constexpr int kDecTileB = 4096; // bytes of one tile row (K chunk)
 
+// Groups [g0, g1) of CTA b when G groups are cut over n CTAs: the first
+// G mod n CTAs take one group more.  CTAs are placed on SMs in index order as
+// the previous kernel's CTAs leave, so the low indices start first and fill
+// their weight ring earliest; they are the ones given the extra group.
+__host__ __device__ inline void dgemv_group_range(int G, int n, int b, int& g0, int& g1) {
+  const int q = G / n, r = G - q * n;
+  g0 = b * q + min(b, r);
+  g1 = g0 + q + (b < r ? 1 : 0);
+}
+
 __host__ __device__ inline size_t sgemv_xs_bytes(int nb, int K, int esz) {
   return ((size_t)nb * K * esz + 1023) / 1024 * 1024;
 }
@@ -264,8 +274,8 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int K = a.K, nchunk = (K + KC - 1) / KC;
   const int G = (a.n_pairs + kGP - 1) / kGP;
-  const int g0 = (int)(((long long)G * blockIdx.x) / gridDim.x);
-  const int g1 = (int)(((long long)G * (blockIdx.x + 1)) / gridDim.x);
+  int g0, g1;
+  dgemv_group_range(G, gridDim.x, blockIdx.x, g0, g1);
   T* xs = reinterpret_cast<T*>(dsm);
   uint8_t* stages = dsm + (XG ? 0 : sgemv_xs_bytes(NB, K, (int)sizeof(T)));
   const T* Wt = static_cast<const T*>(a.W);
@@ -307,7 +317,8 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
       // the region its CTA of this index will stream into L2 now
       if (a.pf_W && (int)blockIdx.x < a.pf_grid) {
         const int Gn = (a.pf_pairs + kGP - 1) / kGP;
-        const long long n0 = ((long long)Gn * blockIdx.x) / a.pf_grid, n1 = ((long long)Gn * (blockIdx.x + 1)) / a.pf_grid;
+        int n0, n1;
+        dgemv_group_range(Gn, a.pf_grid, blockIdx.x, n0, n1);
         const size_t gbytes = (size_t)TR * a.pf_K * sizeof(T);
         const uint8_t* base = static_cast<const uint8_t*>(a.pf_W) + (size_t)n0 * gbytes;
         size_t left = min((size_t)a.pf_bytes, (size_t)(n1 - n0) * gbytes);
