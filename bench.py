@@ -39,7 +39,7 @@ CPU_LAYERS = 2  # the CPU oracle sample runs this many of the 32 layers
 # dram__bytes_read.sum + dram__bytes_write.sum of one dgemv_kernel launch,
 # averaged over the four projections of a decode layer, from one ncu capture
 # of the current kernel (profiles/dgemv_openvla7b_decode_layer.txt)
-DGEMV_TRAFFIC_PER_LAUNCH = {"openvla7b": 101.9e6, "layer7b": 101.9e6}
+DGEMV_TRAFFIC_PER_LAUNCH = {"openvla7b": 102.0e6, "layer7b": 102.0e6}
 
 
 def peaks():
