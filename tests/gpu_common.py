@@ -34,7 +34,7 @@ SMALL = {
     "small": synth.Dims(n_layers=2, hidden=256, n_heads=2, head_dim=128, ffn=768, vocab=1024, n_bins=256,
                         img_h=112, img_w=112, patch=14, n_views=1, n_text=8, proprio_dim=0, n_action=7,
                         parallel=0, dtype="bf16"),
-    # bf16, two 224x224 views + proprio + 56-position parallel block: 596 rows (> 512, two GEMM passes)
+    # bf16, two 224x224 views + proprio + 56-position parallel block: 596 rows (> 384: three GEMM passes)
     "small_oft": synth.Dims(n_layers=2, hidden=256, n_heads=4, head_dim=64, ffn=512, vocab=512, n_bins=256,
                             img_h=224, img_w=224, patch=14, n_views=2, n_text=27, proprio_dim=8, n_action=56,
                             parallel=1, dtype="bf16"),

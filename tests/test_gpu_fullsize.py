@@ -1,6 +1,6 @@
 """Parity at the full workload sizes: the OpenVLA-7B shape (32 layers, hidden
 4096, 283-token prefix, 7 autoregressive action tokens), the OpenVLA-OFT shape
-(two views, proprio, 56 parallel action positions: 596 rows, two GEMM passes)
+(two views, proprio, 56 parallel action positions: 596 rows, three GEMM passes)
 and the batch of 8 sequences, against the fp64 oracle on the host.
 
 The steps run in the launch configuration the benchmark times.  Selection,
