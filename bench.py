@@ -203,6 +203,31 @@ def run_reference(args, d, frames, prompt, prop, pm, rank):
     }), flush=True)
 
 
+# ---------------------------------------------------------------------------
+# Replicas (N > 1): one process per GPU, each with its own episode; no
+# collective on the data path, only the timing reduction
+# ---------------------------------------------------------------------------
+
+def replica_seed(seed: int, rank: int) -> int:
+    """Each rank replays its own seeded episode."""
+    return seed + rank
+
+
+def reduce_max(value: float, dist, device) -> float:
+    """The slowest rank's time (MAX over ranks); `dist` None means one rank."""
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate_rate(world: int, B: int, K: int, seconds: float) -> float:
+    """Whole-job sequence-steps per second: every rank ran K steps of B sequences."""
+    return world * B * K / seconds
+
+
 def config_block(d, args):
     vis = f"{d.n_views}x{d.img_h}x{d.img_w} frame(s) -> {d.n_visual} patches"
     act = (f"{d.n_action} parallel action positions" if d.parallel else f"{d.n_action} autoregressive action tokens")
@@ -238,7 +263,7 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     d = synth.dims_for(args.config)
-    seed = args.seed + rank
+    seed = replica_seed(args.seed, rank)
     B = d.max_batch
     frames = synth.make_episode(d, EPISODE, seed=seed, batch=B, kind="scene",
                                 speeds=synth.batch_speeds(B, seed=seed) if B > 1 else None)
@@ -300,13 +325,9 @@ def main():
     barrier()
     clocks = clk.stop()
     launches = ctx.launch_count() - n0
-    ms = e0.elapsed_time(e1)
-    if dist is not None:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = reduce_max(e0.elapsed_time(e1), dist, dev)
     assert ctx.sync_error() == 0
-    value = world * B * K / (ms / 1e3)   # sequence-steps per second
+    value = aggregate_rate(world, B, K, ms / 1e3)   # sequence-steps per second
 
     # ---- algorithmic work of the timed steps ----
     Ms = hist["M"].cpu().numpy()           # [K][B][L]
@@ -380,12 +401,8 @@ def main():
         for n, hbuf in res_host.items():
             hbuf.copy_(outs[n], non_blocking=True)
         torch.cuda.current_stream().synchronize()  # the action is needed before the next frame
-    e2e_s = time.perf_counter() - t0
-    if dist is not None:
-        t_ = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(t_, op=dist.ReduceOp.MAX)
-        e2e_s = float(t_.item())
-    e2e = world * B * K / e2e_s
+    e2e_s = reduce_max(time.perf_counter() - t0, dist, dev)
+    e2e = aggregate_rate(world, B, K, e2e_s)
 
     # ---- CPU oracle baseline (rank 0, N = 1 only) ----
     cpu = None
