@@ -141,6 +141,25 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
 }
 constexpr uint32_t kWaitLimit = 1u << 24;
 
+// Give-up path of a bulk-copy ring: before its CTA exits, wait (bounded, deaf
+// to any give-up flag) until the producer's last min(issued, ns) copies have
+// landed.  A stage is refilled only after every consumer waited for its
+// previous copy, so these are the only copies that can still be in flight;
+// (stage, phase) is the producer's ring position after its last issue.
+__device__ __forceinline__ void ring_drain(uint64_t* full, int ns, int stage, uint32_t phase, uint32_t issued) {
+  const int n_last = (int)min(issued, (uint32_t)ns);
+  for (int q = 0; q < n_last; ++q) {
+    int s = stage - 1 - q;
+    uint32_t ph = phase;
+    if (s < 0) {
+      s += ns;
+      ph ^= 1u;
+    }
+    for (uint32_t it = 0; it < kWaitLimit && !mbar_test(&full[s], ph); ++it) {
+    }
+  }
+}
+
 __device__ __forceinline__ void set_error(int* err, int code) {
   if (err) atomicCAS(err, 0, code);
 }

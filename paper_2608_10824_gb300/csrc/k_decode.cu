@@ -271,6 +271,8 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
   __shared__ __align__(8) float2 pacc[2][kNC][32];  // bf16 path: per-warp partials, two groups in flight
   __shared__ float half_acc[kGP][2][NB];            // fp32 path: the second K half of every pair
   __shared__ int abort_flag;
+  __shared__ __align__(8) uint64_t done_bar;  // the producer has issued its last copy
+  __shared__ uint32_t prod_end[3];             // its ring stage, phase and copy count at that point
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int K = a.K, nchunk = (K + KC - 1) / KC;
   const int G = (a.n_pairs + kGP - 1) / kGP;
@@ -284,6 +286,7 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], kNC);
     }
+    mbar_init(&done_bar, 1);
     abort_flag = 0;
     mbar_fence_init();
   }
@@ -294,7 +297,7 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
     // ---- producer: weights only, so it runs ahead of the dependency wait ----
     if (lane == 0) {
       int stage = 0;
-      uint32_t phase = 0;
+      uint32_t phase = 0, issued = 0;
       for (int g = g0; g < g1 && !*abort; ++g) {
         const T* gbase = Wt + (size_t)g * TR * K;
         for (int c = 0; c < nchunk; ++c) {
@@ -307,12 +310,17 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
           const uint32_t bytes = (uint32_t)(TR * kn * sizeof(T));
           mbar_expect_tx(&full_bar[stage], bytes);
           bulk_g2s(stages + (size_t)stage * stage_b, gbase + (size_t)TR * c * KC, bytes, &full_bar[stage]);
+          ++issued;
           if (++stage == NS) {
             stage = 0;
             phase ^= 1u;
           }
         }
       }
+      prod_end[0] = (uint32_t)stage;
+      prod_end[1] = phase;
+      prod_end[2] = issued;
+      mbar_arrive(&done_bar);  // release: the consumers that gave up read prod_end after it
       // the next GEMV's weights do not depend on anything: pull the start of
       // the region its CTA of this index will stream into L2 now
       if (a.pf_W && (int)blockIdx.x < a.pf_grid) {
@@ -468,8 +476,14 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
             set_error(a.err, VLAC_ERR_TIMEOUT);
             *abort = 1;
           }
+          // the warp stays in the group loop, in step with the others' named
+          // barriers; the stage is not handed back, so it is never refilled
           aborted = true;
-          break;
+          if (++stage == NS) {
+            stage = 0;
+            phase ^= 1u;
+          }
+          continue;
         }
         const uint32_t st = st_lane + (uint32_t)(stage * stage_b);
         const T* xrow = XG ? static_cast<const T*>(a.xin) + (size_t)gq * K + k0 + 2 * tq : xs + (size_t)gq * K + k0 + tq * 8;
@@ -523,7 +537,6 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
           phase ^= 1u;
         }
       }
-      if (aborted) break;
       // D[gq][2tq], D[gq][2tq+1]: this warp's share of pair tq of sequence gq
       if (gq < NB)
         pacc[pb][warp][lane] = make_float2(((d[0][0] + d[1][0]) + d[2][0]) + d[3][0], ((d[0][1] + d[1][1]) + d[2][1]) + d[3][1]);
@@ -563,8 +576,14 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
             set_error(a.err, VLAC_ERR_TIMEOUT);
             *abort = 1;
           }
+          // the warp stays in the group loop, in step with the others' named
+          // barriers; the stage is not handed back, so it is never refilled
           aborted = true;
-          break;
+          if (++stage == NS) {
+            stage = 0;
+            phase ^= 1u;
+          }
+          continue;
         }
         const T* st = reinterpret_cast<const T*>(stages + (size_t)stage * stage_b);
         const uint4* w1 = reinterpret_cast<const uint4*>(st + (size_t)(2 * q) * kn);
@@ -591,7 +610,6 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
           phase ^= 1u;
         }
       }
-      if (aborted) break;
       // add the two K halves of every pair in order, then the epilogue
 #pragma unroll
       for (int b = 0; b < NB; ++b) {
@@ -633,6 +651,13 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
       }
       a.ssq_out[(size_t)tid * gridDim.x + blockIdx.x] = t;
     }
+  }
+  // A warp that gave up skipped waits, so copies may still be landing in this
+  // CTA's shared memory; a warp that did not saw every copy land.
+  if (aborted && lane == 0) {
+    bool ended = false;
+    for (uint32_t it = 0; it < kWaitLimit && !ended; ++it) ended = mbar_test(&done_bar, 0);
+    if (ended) ring_drain(full_bar, NS, (int)prod_end[0], prod_end[1], prod_end[2]);
   }
 }
 
