@@ -53,14 +53,15 @@ class _Weights(C.Structure):
 
 class _Opts(C.Structure):
     _fields_ = [("margin_kind", C.c_int32), ("reduction", C.c_int32),
-                ("gate_override", C.c_void_p), ("forced_ids", C.c_void_p)]
+                ("gate_override", C.c_void_p), ("forced_ids", C.c_void_p),
+                ("s2_top_k", C.c_int32), ("s2_layer", C.c_int32)]
 
 
 class _Out(C.Structure):
     _fields_ = [("action_ids", C.c_void_p), ("margins", C.c_void_p), ("logit_gap", C.c_void_p),
                 ("logits", C.c_void_p), ("recomputed", C.c_void_p), ("gate_auto", C.c_void_p),
                 ("step_margin", C.c_void_p), ("static_mask", C.c_void_p), ("idx", C.c_void_p),
-                ("M", C.c_void_p)]
+                ("M", C.c_void_p), ("relevance", C.c_void_p), ("relevant", C.c_void_p)]
 
 
 def lib():
@@ -86,6 +87,9 @@ def lib():
                                            C.c_int64, C.c_int64, C.c_int64, C.c_int]
             L.orc_select.argtypes = [C.POINTER(_Dims), vp, vp, C.c_int, u32, u32, vp, C.c_int,
                                      vp, vp, vp]
+            L.orc_select2.argtypes = [C.POINTER(_Dims), vp, vp, C.c_int, u32, u32, vp, C.c_int,
+                                      vp, C.c_int, vp, vp, vp, vp]
+            L.orc_top_k.argtypes = [vp, C.c_int, C.c_int, vp]
             L.orc_margin.argtypes = [vp, C.c_int, C.POINTER(i32), C.POINTER(C.c_double),
                                      C.POINTER(C.c_double)]
             L.orc_round_bf16.argtypes = [C.c_double]
@@ -126,7 +130,9 @@ def more_similar(ki, i, kj, j) -> bool:
     return bool(lib().orc_more_similar(ki[0], ki[1], ki[2], i, kj[0], kj[1], kj[2], j))
 
 
-def select(d, frame, prev, have_prev: bool, tau, permille, full: bool):
+def select(d, frame, prev, have_prev: bool, tau, permille, full: bool, relevance=None, top_k: int = 0):
+    """Stages 1-3; with `relevance` and top_k > 0 also Stage 2.  Returns
+    (|reusable|, Stage-1 mask, idx, M) and, with Stage 2, the relevant set."""
     frame = np.ascontiguousarray(frame, dtype=np.uint8)
     prev = np.ascontiguousarray(prev, dtype=np.uint8)
     permille = np.ascontiguousarray(permille, dtype=np.uint16)
@@ -134,11 +140,28 @@ def select(d, frame, prev, have_prev: bool, tau, permille, full: bool):
     idx = np.zeros(d.pass_len, dtype=np.int32)
     M = np.zeros(d.n_layers, dtype=np.int32)
     dd = c_dims(d)
-    n = lib().orc_select(C.byref(dd), _ptr(frame), _ptr(prev), int(have_prev), tau[0], tau[1],
-                         _ptr(permille), int(full), _ptr(mask), _ptr(idx), _ptr(M))
+    if relevance is None and top_k == 0:
+        n = lib().orc_select(C.byref(dd), _ptr(frame), _ptr(prev), int(have_prev), tau[0], tau[1],
+                             _ptr(permille), int(full), _ptr(mask), _ptr(idx), _ptr(M))
+        if n < 0:
+            raise ValueError("orc_select rejected its arguments")
+        return n, mask, idx, M
+    rel = None if relevance is None else np.ascontiguousarray(relevance, dtype=np.float64)
+    relevant = np.zeros(d.n_visual, dtype=np.uint8)
+    n = lib().orc_select2(C.byref(dd), _ptr(frame), _ptr(prev), int(have_prev), tau[0], tau[1],
+                          _ptr(permille), int(full), _ptr(rel), int(top_k), _ptr(mask), _ptr(relevant),
+                          _ptr(idx), _ptr(M))
     if n < 0:
-        raise ValueError("orc_select rejected its arguments")
-    return n, mask, idx, M
+        raise ValueError("orc_select2 rejected its arguments")
+    return n, mask, idx, M, relevant
+
+
+def top_k(rel: np.ndarray, k: int) -> np.ndarray:
+    """Stage 2's removal set of a relevance vector (1 = among the top k)."""
+    r = np.ascontiguousarray(rel, dtype=np.float64)
+    out = np.zeros(r.size, dtype=np.uint8)
+    lib().orc_top_k(_ptr(r), r.size, int(k), _ptr(out))
+    return out
 
 
 def margin(logits: np.ndarray):
@@ -208,7 +231,8 @@ class Oracle:
 
     def step(self, cache: "OracleCache", frames, prompt, proprio=None, tau_sim=(996, 1000),
              tau_margin: float = 0.0, permille=None, margin_kind: int = 0, reduction: Optional[int] = None,
-             gate_override=None, forced_ids=None, want_logits: bool = True):
+             gate_override=None, forced_ids=None, want_logits: bool = True, s2_top_k: int = 0,
+             s2_layer: Optional[int] = None):
         d, B = self.d, cache.batch
         D, S, L = d.n_action, d.pass_len, d.n_layers
         frames = np.ascontiguousarray(frames, dtype=np.uint8).reshape(B, d.n_views, d.img_h, d.img_w, 3)
@@ -229,10 +253,14 @@ class Oracle:
             "recomputed": np.zeros(B, np.uint8), "gate_auto": np.zeros(B, np.uint8),
             "step_margin": np.zeros(B, np.float64), "static_mask": np.zeros((B, d.n_visual), np.uint8),
             "idx": np.zeros((B, S), np.int32), "M": np.zeros((B, L), np.int32),
+            "relevance": np.zeros((B, d.n_visual), np.float64), "relevant": np.zeros((B, d.n_visual), np.uint8),
         }
         co = _Out(*[_ptr(out[k]) for k in ("action_ids", "margins", "logit_gap", "logits", "recomputed",
-                                           "gate_auto", "step_margin", "static_mask", "idx", "M")])
-        opts = _Opts(margin_kind, reduction, _ptr(go), _ptr(fi))
+                                           "gate_auto", "step_margin", "static_mask", "idx", "M",
+                                           "relevance", "relevant")])
+        if s2_layer is None:
+            s2_layer = L // 2
+        opts = _Opts(margin_kind, reduction, _ptr(go), _ptr(fi), int(s2_top_k), int(s2_layer))
         r = lib().orc_step(self._h, cache._h, _ptr(frames), _ptr(prompt), _ptr(proprio), tau_sim[0],
                            tau_sim[1], float(tau_margin), _ptr(permille), C.byref(opts), C.byref(co))
         if r != 0:

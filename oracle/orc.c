@@ -33,6 +33,8 @@ struct orc_cache {
   uint8_t* prev; /* [B][frame bytes] */
   double* m_prev;
   uint8_t* valid;
+  double* rel;        /* [B][Nv]: Stage-2 relevance from the previous step */
+  uint8_t* rel_valid; /* [B]: rel holds the previous step's relevance */
 };
 
 /* ------------------------------------------------------------------------ */
@@ -197,25 +199,46 @@ int orc_more_similar(int64_t d_i, int64_t na_i, int64_t nb_i, int i,
 }
 
 static int pos_is_visual(const orc_ctx* c, int pos) { return pos >= 1 && pos <= c->Nv; }
+/* Prompt tokens: BOS at 0 and the text after the visual (and proprio) tokens. */
+static int pos_is_text(const orc_ctx* c, int pos) {
+  return pos == 0 || (pos > c->Nv + (c->d.proprio_dim > 0 ? 1 : 0) && pos < c->P);
+}
 
-/* Stage 1 + Stage 3 applied: the recompute order idx[0..S) and per-layer row
- * counts M[l] such that the rows recomputed at layer l are idx[0 .. M[l]).
- *   idx = [every position that is not a static patch, ascending]
- *         ++ [static patches, least similar first].
- *   k_l = floor(permille[l] * |S| / 1000) static patches (the most similar)
- *   are reused at layer l, so M[l] = S - k_l.
- * The full branch recomputes everything: idx = 0 .. S-1 and M[l] = S. */
-int orc_select(const orc_dims* d, const uint8_t* frame, const uint8_t* prev, int have_prev,
-               uint32_t num, uint32_t den, const uint16_t* permille, int full,
-               uint8_t* mask, int32_t* idx, int32_t* M) {
+/* Stage 2's removal set: the top_k entries of rel, ranked by value (higher
+ * first), equal values by index (lower first). */
+void orc_top_k(const double* rel, int n, int top_k, uint8_t* out) {
+  for (int v = 0; v < n; ++v) {
+    int before = 0;
+    for (int u = 0; u < n; ++u)
+      if (rel[u] > rel[v] || (rel[u] == rel[v] && u < v)) ++before;
+    out[v] = (uint8_t)(before < top_k);
+  }
+}
+
+/* Stages 1-3 applied: the recompute order idx[0..S) and per-layer row counts
+ * M[l] such that the rows recomputed at layer l are idx[0 .. M[l]).
+ *   reusable = static patches (Stage 1) that Stage 2 did not mark relevant.
+ *   idx = [every position that is not a reusable patch, ascending]
+ *         ++ [reusable patches, least similar first].
+ *   k_l = floor(permille[l] * |reusable| / 1000) reusable patches (the most
+ *   similar) are reused at layer l, so M[l] = S - k_l.
+ * The full branch recomputes everything: idx = 0 .. S-1 and M[l] = S.
+ * Returns |reusable|. */
+int orc_select2(const orc_dims* d, const uint8_t* frame, const uint8_t* prev, int have_prev,
+                uint32_t num, uint32_t den, const uint16_t* permille, int full,
+                const double* relevance, int top_k, uint8_t* mask, uint8_t* relevant,
+                int32_t* idx, int32_t* M) {
   const int Nv = d->n_views * (d->img_h / d->patch) * (d->img_w / d->patch);
   const int P = d->n_text + Nv + (d->proprio_dim > 0 ? 1 : 0);
   const int S = P + (d->parallel ? d->n_action : 0);
   const int L = d->n_layers;
   for (int l = 0; l < L; ++l)
     if (permille[l] > 1000) return ORC_ERR_ARG;
+  if (top_k < 0) return ORC_ERR_ARG;
   int64_t* st = (int64_t*)malloc(sizeof(int64_t) * 3 * (size_t)(Nv > 0 ? Nv : 1));
   int* stat = (int*)malloc(sizeof(int) * (size_t)(Nv > 0 ? Nv : 1));
+  uint8_t* rel = (uint8_t*)calloc((size_t)(Nv > 0 ? Nv : 1), 1);
+  if (relevance && top_k > 0) orc_top_k(relevance, Nv, top_k, rel);
   int nS = 0;
   for (int v = 0; v < Nv; ++v) {
     int s = 0;
@@ -224,13 +247,14 @@ int orc_select(const orc_dims* d, const uint8_t* frame, const uint8_t* prev, int
       s = orc_is_static(st[3 * v], st[3 * v + 1], st[3 * v + 2], num, den);
     }
     if (mask) mask[v] = (uint8_t)s;
-    if (s) stat[nS++] = v;
+    if (relevant) relevant[v] = rel[v];
+    if (s && !rel[v]) stat[nS++] = v;
   }
   if (full) {
     for (int i = 0; i < S; ++i) idx[i] = i;
     for (int l = 0; l < L; ++l) M[l] = S;
   } else {
-    /* insertion sort of the static patches into reuse order */
+    /* insertion sort of the reusable patches into reuse order */
     for (int a = 1; a < nS; ++a) {
       int key = stat[a], b = a - 1;
       while (b >= 0 && orc_more_similar(st[3 * key], st[3 * key + 1], st[3 * key + 2], key,
@@ -242,19 +266,26 @@ int orc_select(const orc_dims* d, const uint8_t* frame, const uint8_t* prev, int
     }
     int n = 0;
     for (int pos = 0; pos < S; ++pos) {
-      int is_static = 0;
+      int reusable = 0;
       if (pos >= 1 && pos <= Nv) {
         for (int q = 0; q < nS; ++q)
-          if (stat[q] == pos - 1) { is_static = 1; break; }
+          if (stat[q] == pos - 1) { reusable = 1; break; }
       }
-      if (!is_static) idx[n++] = pos;
+      if (!reusable) idx[n++] = pos;
     }
     for (int q = nS - 1; q >= 0; --q) idx[n++] = 1 + stat[q];
     for (int l = 0; l < L; ++l) M[l] = S - (int)(((int64_t)permille[l] * nS) / 1000);
   }
   free(st);
   free(stat);
+  free(rel);
   return nS;
+}
+
+int orc_select(const orc_dims* d, const uint8_t* frame, const uint8_t* prev, int have_prev,
+               uint32_t num, uint32_t den, const uint16_t* permille, int full,
+               uint8_t* mask, int32_t* idx, int32_t* M) {
+  return orc_select2(d, frame, prev, have_prev, num, den, permille, full, NULL, 0, mask, NULL, idx, M);
 }
 
 /* ------------------------------------------------------------------------ */
@@ -342,7 +373,9 @@ int orc_cache_new(const orc_ctx* c, int batch, orc_cache** out) {
   k->prev = (uint8_t*)calloc((size_t)batch * frame_bytes(&c->d), 1);
   k->m_prev = (double*)calloc((size_t)batch, sizeof(double));
   k->valid = (uint8_t*)calloc((size_t)batch, 1);
-  if (!k->K || !k->V || !k->H || !k->prev || !k->m_prev || !k->valid) {
+  k->rel = (double*)calloc((size_t)batch * (c->Nv > 0 ? c->Nv : 1), sizeof(double));
+  k->rel_valid = (uint8_t*)calloc((size_t)batch, 1);
+  if (!k->K || !k->V || !k->H || !k->prev || !k->m_prev || !k->valid || !k->rel || !k->rel_valid) {
     orc_cache_free(k);
     return ORC_ERR_OOM;
   }
@@ -358,6 +391,8 @@ void orc_cache_free(orc_cache* k) {
   free(k->prev);
   free(k->m_prev);
   free(k->valid);
+  free(k->rel);
+  free(k->rel_valid);
   free(k);
 }
 
@@ -365,7 +400,7 @@ void orc_cache_free(orc_cache* k) {
 int orc_reset(orc_cache* k, int seq) {
   if (!k || seq < -1 || seq >= k->B) return ORC_ERR_ARG;
   for (int b = 0; b < k->B; ++b)
-    if (seq == -1 || seq == b) k->valid[b] = 0;
+    if (seq == -1 || seq == b) k->valid[b] = k->rel_valid[b] = 0;
   return ORC_OK;
 }
 
@@ -403,8 +438,12 @@ static int key_limit(const orc_ctx* c, int pos) {
 
 /* One decoder layer for n rows at positions pos[i]; x holds their fp32
  * residual rows.  Fresh K/V of every row are written to the cache before any
- * row attends, and attention reads the cache (reused + fresh entries). */
-static void layer_rows(const orc_ctx* c, orc_cache* k, int b, int l, int n, const int32_t* pos, float* x) {
+ * row attends, and attention reads the cache (reused + fresh entries).
+ * rel (Stage 2, NULL = not wanted) receives, per visual patch v, the softmax
+ * probability of key 1 + v summed over the text rows among the n (in row
+ * order) and, within a row, over the heads in order. */
+static void layer_rows(const orc_ctx* c, orc_cache* k, int b, int l, int n, const int32_t* pos, float* x,
+                       double* rel) {
   const int Hd = c->d.hidden, nh = c->d.n_heads, hd = c->d.head_dim, F = c->d.ffn;
   const size_t T = c->T, L = c->d.n_layers;
   float* Kl = k->K + (((size_t)b * L + l) * T) * Hd;
@@ -435,6 +474,9 @@ static void layer_rows(const orc_ctx* c, orc_cache* k, int b, int l, int n, cons
     }
   }
   const double scale = 1.0 / sqrt((double)hd);
+  const int Nv = c->Nv;
+  /* per (row, head): probability of each visual key (text rows only) */
+  double* pv = rel ? (double*)calloc((size_t)n * nh * (Nv > 0 ? Nv : 1), sizeof(double)) : NULL;
 #pragma omp parallel for schedule(dynamic)
   for (int ih = 0; ih < n * nh; ++ih) {
     const int i = ih / nh, hh = ih % nh;
@@ -453,12 +495,21 @@ static void layer_rows(const orc_ctx* c, orc_cache* k, int b, int l, int n, cons
       sc[j] = exp(sc[j] - mx);
       z += sc[j];
     }
+    if (pv && pos_is_text(c, pos[i]))
+      for (int j = 1; j < nk && j <= Nv; ++j) pv[((size_t)i * nh + hh) * Nv + (j - 1)] = sc[j] / z;
     for (int e = 0; e < hd; ++e) {
       double o = 0.0;
       for (int j = 0; j < nk; ++j) o += sc[j] * (double)Vl[(size_t)j * Hd + (size_t)hh * hd + e];
       att[(size_t)i * Hd + (size_t)hh * hd + e] = store_act(c, o / z);
     }
     free(sc);
+  }
+  if (pv) {
+    for (int v = 0; v < Nv; ++v) rel[v] = 0.0;
+    for (int i = 0; i < n; ++i)
+      for (int hh = 0; hh < nh; ++hh)
+        for (int v = 0; v < Nv; ++v) rel[v] += pv[((size_t)i * nh + hh) * Nv + v];
+    free(pv);
   }
   linear(c, c->w.wo[l], Hd, Hd, n, att, y);
   for (size_t e = 0; e < (size_t)n * Hd; ++e) x[e] = (float)((double)x[e] + y[e]);
@@ -550,9 +601,16 @@ static int step_seq(orc_ctx* c, orc_cache* k, int b, const uint8_t* frame, const
   int32_t* idx = (int32_t*)malloc(sizeof(int32_t) * S);
   int32_t* M = (int32_t*)malloc(sizeof(int32_t) * L);
   uint8_t* mask = (uint8_t*)malloc((size_t)(c->Nv > 0 ? c->Nv : 1));
-  int nS = orc_select(&c->d, frame, prev, k->valid[b], num, den, permille, full, mask, idx, M);
-  if (nS < 0) { free(idx); free(M); free(mask); return ORC_ERR_ARG; }
+  uint8_t* relevant = (uint8_t*)malloc((size_t)(c->Nv > 0 ? c->Nv : 1));
+  /* Stage 2 uses the relevance the previous step measured */
+  const int s2 = o && o->s2_top_k > 0;
+  const double* rel_prev = (s2 && k->rel_valid[b]) ? k->rel + (size_t)b * c->Nv : NULL;
+  int nS = orc_select2(&c->d, frame, prev, k->valid[b], num, den, permille, full, rel_prev, s2 ? o->s2_top_k : 0,
+                       mask, relevant, idx, M);
+  if (nS < 0) { free(idx); free(M); free(mask); free(relevant); return ORC_ERR_ARG; }
   if (out->static_mask) memcpy(out->static_mask + (size_t)b * c->Nv, mask, (size_t)c->Nv);
+  if (out->relevant) memcpy(out->relevant + (size_t)b * c->Nv, relevant, (size_t)c->Nv);
+  free(relevant);
   if (out->idx) memcpy(out->idx + (size_t)b * S, idx, sizeof(int32_t) * S);
   if (out->M) memcpy(out->M + (size_t)b * L, M, sizeof(int32_t) * L);
 
@@ -560,6 +618,7 @@ static int step_seq(orc_ctx* c, orc_cache* k, int b, const uint8_t* frame, const
   float* x = (float*)malloc(sizeof(float) * (size_t)S * Hd);
   for (int i = 0; i < M[0]; ++i) embed_row(c, idx[i], frame, prompt, proprio, x + (size_t)i * Hd);
   float* Hb = k->H + (size_t)b * L * S * Hd;
+  double* rel_now = s2 ? (double*)calloc((size_t)(c->Nv > 0 ? c->Nv : 1), sizeof(double)) : NULL;
   for (int l = 0; l < L; ++l) {
     if (l > 0) {
       /* rows computed at layer l-1 record their layer-l input; rows that join
@@ -569,8 +628,15 @@ static int step_seq(orc_ctx* c, orc_cache* k, int b, const uint8_t* frame, const
       for (int i = M[l - 1]; i < M[l]; ++i)
         memcpy(x + (size_t)i * Hd, Hb + ((size_t)l * S + idx[i]) * Hd, sizeof(float) * Hd);
     }
-    layer_rows(c, k, b, l, M[l], idx, x);
+    layer_rows(c, k, b, l, M[l], idx, x, (s2 && l == o->s2_layer) ? rel_now : NULL);
   }
+  /* every text row is recomputed at every layer, so this step's relevance is
+   * complete; it is what the next step's Stage 2 reads */
+  if (out->relevance)
+    for (int v = 0; v < c->Nv; ++v) out->relevance[(size_t)b * c->Nv + v] = s2 ? rel_now[v] : 0.0;
+  if (s2) memcpy(k->rel + (size_t)b * c->Nv, rel_now, sizeof(double) * c->Nv);
+  k->rel_valid[b] = (uint8_t)s2;
+  free(rel_now);
 
   /* Action tokens. */
   double* lg = (double*)malloc(sizeof(double) * nb);
@@ -599,7 +665,7 @@ static int step_seq(orc_ctx* c, orc_cache* k, int b, const uint8_t* frame, const
       int32_t p = c->P + a - 1;
       xdec = (float*)malloc(sizeof(float) * Hd);
       for (int e = 0; e < Hd; ++e) xdec[e] = (float)wget(c, c->w.tok_emb, (size_t)tok * Hd + e);
-      for (int l = 0; l < L; ++l) layer_rows(c, k, b, l, 1, &p, xdec);
+      for (int l = 0; l < L; ++l) layer_rows(c, k, b, l, 1, &p, xdec, NULL);
       xr = xdec;
     }
     double pm, gap;
@@ -628,6 +694,8 @@ int orc_step(orc_ctx* c, orc_cache* k, const uint8_t* frames, const int32_t* pro
       !out->margins || !out->logit_gap || !out->recomputed || !out->gate_auto || !out->step_margin || tau_den == 0)
     return ORC_ERR_ARG;
   if (c->d.proprio_dim > 0 && !proprio) return ORC_ERR_ARG;
+  if (opts && (opts->s2_top_k < 0 || (opts->s2_top_k > 0 && (opts->s2_layer < 0 || opts->s2_layer >= c->d.n_layers))))
+    return ORC_ERR_ARG;
   const size_t fb = frame_bytes(&c->d);
   for (int b = 0; b < k->B; ++b) {
     int r = step_seq(c, k, b, frames + (size_t)b * fb, prompt_ids + (size_t)b * c->d.n_text,

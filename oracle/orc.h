@@ -11,6 +11,12 @@
  *     embeddings, concatenated with the language tokens.
  *   - Sec. III-B Stage 1: cosine similarity between corresponding patches
  *     of I_t and I_{t-1}; similarity above tau marks a patch static.
+ *   - Sec. III-B Stage 2 (optional): static patches that drew the most
+ *     text-to-vision attention are taken out of the reusable set.  The
+ *     relevance of a patch is the softmax probability that the text queries
+ *     put on its key, summed over text rows and heads, at one caller-chosen
+ *     layer of the previous step; the top_k patches by relevance are
+ *     removed.
  *   - Sec. III-B Stage 3: a per-layer proportion of the static patches is
  *     reused (here a caller-given per-mille schedule).
  *   - Sec. IV-A Eq. (1): mean top-1/top-2 probability margin over the D
@@ -69,6 +75,8 @@ typedef struct orc_opts {
   int32_t reduction;            /* 0 = mean over the action tokens (Eq. 1), 1 = minimum */
   const int8_t* gate_override;  /* [B]: -1 gate, 0 force cached, 1 force full; NULL = gate */
   const int32_t* forced_ids;    /* [B][n_action] bins fed back in decode; NULL = argmax */
+  int32_t s2_top_k;             /* Stage 2: patches removed per step; 0 = Stage 2 off */
+  int32_t s2_layer;             /* Stage 2: the layer whose attention gives the relevance */
 } orc_opts;
 
 typedef struct orc_out {
@@ -82,6 +90,8 @@ typedef struct orc_out {
   uint8_t* static_mask; /* [B][n_visual] or NULL */
   int32_t* idx;         /* [B][S] recompute order or NULL */
   int32_t* M;           /* [B][n_layers] rows recomputed per layer or NULL */
+  double* relevance;    /* [B][n_visual] this step's Stage-2 relevance (0 when off) or NULL */
+  uint8_t* relevant;    /* [B][n_visual] patches Stage 2 removed this step or NULL */
 } orc_out;
 
 typedef struct orc_ctx orc_ctx;
@@ -111,6 +121,16 @@ int orc_more_similar(int64_t d_i, int64_t na_i, int64_t nb_i, int i,
 int orc_select(const orc_dims* d, const uint8_t* frame, const uint8_t* prev, int have_prev,
                uint32_t num, uint32_t den, const uint16_t* permille, int full,
                uint8_t* mask, int32_t* idx, int32_t* M);
+/* orc_select with Stage 2: `relevance` ([n_visual], NULL = none) marks its
+ * top_k patches relevant (written to `relevant` if not NULL); a relevant
+ * patch is never reused. */
+int orc_select2(const orc_dims* d, const uint8_t* frame, const uint8_t* prev, int have_prev,
+                uint32_t num, uint32_t den, const uint16_t* permille, int full,
+                const double* relevance, int top_k, uint8_t* mask, uint8_t* relevant,
+                int32_t* idx, int32_t* M);
+/* out[v] = 1 for the top_k entries of rel[0..n): v is in iff fewer than top_k
+ * entries rank before it (higher value, or equal value and lower index). */
+void orc_top_k(const double* rel, int n, int top_k, uint8_t* out);
 void orc_margin(const double* logits, int n, int32_t* argmax, double* pmargin, double* lgap);
 double orc_round_bf16(double v);
 void orc_rope_table(const orc_dims* d, int n_pos, float* cos_t, float* sin_t);
