@@ -61,7 +61,8 @@ class _Out(C.Structure):
     _fields_ = [("action_ids", C.c_void_p), ("margins", C.c_void_p), ("logit_gap", C.c_void_p),
                 ("logits", C.c_void_p), ("recomputed", C.c_void_p), ("gate_auto", C.c_void_p),
                 ("step_margin", C.c_void_p), ("static_mask", C.c_void_p), ("idx", C.c_void_p),
-                ("M", C.c_void_p), ("relevance", C.c_void_p), ("relevant", C.c_void_p)]
+                ("M", C.c_void_p), ("relevance", C.c_void_p), ("relevant", C.c_void_p),
+                ("entropy", C.c_void_p), ("vocab_margin", C.c_void_p), ("action_delta", C.c_void_p)]
 
 
 def lib():
@@ -92,6 +93,8 @@ def lib():
             L.orc_top_k.argtypes = [vp, C.c_int, C.c_int, vp]
             L.orc_margin.argtypes = [vp, C.c_int, C.POINTER(i32), C.POINTER(C.c_double),
                                      C.POINTER(C.c_double)]
+            L.orc_entropy.argtypes = [vp, C.c_int]
+            L.orc_entropy.restype = C.c_double
             L.orc_round_bf16.argtypes = [C.c_double]
             L.orc_round_bf16.restype = C.c_double
             L.orc_rope_table.argtypes = [C.POINTER(_Dims), C.c_int, vp, vp]
@@ -171,6 +174,11 @@ def margin(logits: np.ndarray):
     return a.value, pm.value, gap.value
 
 
+def entropy(logits: np.ndarray) -> float:
+    lg = np.ascontiguousarray(logits, dtype=np.float64)
+    return lib().orc_entropy(_ptr(lg), lg.size)
+
+
 def round_bf16(v: float) -> float:
     return lib().orc_round_bf16(float(v))
 
@@ -232,7 +240,7 @@ class Oracle:
     def step(self, cache: "OracleCache", frames, prompt, proprio=None, tau_sim=(996, 1000),
              tau_margin: float = 0.0, permille=None, margin_kind: int = 0, reduction: Optional[int] = None,
              gate_override=None, forced_ids=None, want_logits: bool = True, s2_top_k: int = 0,
-             s2_layer: Optional[int] = None):
+             s2_layer: Optional[int] = None, want_vocab_margin: bool = False):
         d, B = self.d, cache.batch
         D, S, L = d.n_action, d.pass_len, d.n_layers
         frames = np.ascontiguousarray(frames, dtype=np.uint8).reshape(B, d.n_views, d.img_h, d.img_w, 3)
@@ -254,10 +262,13 @@ class Oracle:
             "step_margin": np.zeros(B, np.float64), "static_mask": np.zeros((B, d.n_visual), np.uint8),
             "idx": np.zeros((B, S), np.int32), "M": np.zeros((B, L), np.int32),
             "relevance": np.zeros((B, d.n_visual), np.float64), "relevant": np.zeros((B, d.n_visual), np.uint8),
+            "entropy": np.zeros((B, D), np.float64),
+            "vocab_margin": np.zeros((B, D), np.float64) if want_vocab_margin else None,
+            "action_delta": np.zeros(B, np.int32),
         }
         co = _Out(*[_ptr(out[k]) for k in ("action_ids", "margins", "logit_gap", "logits", "recomputed",
                                            "gate_auto", "step_margin", "static_mask", "idx", "M",
-                                           "relevance", "relevant")])
+                                           "relevance", "relevant", "entropy", "vocab_margin", "action_delta")])
         if s2_layer is None:
             s2_layer = L // 2
         opts = _Opts(margin_kind, reduction, _ptr(go), _ptr(fi), int(s2_top_k), int(s2_layer))
@@ -267,6 +278,8 @@ class Oracle:
             raise ValueError(f"orc_step failed ({r})")
         if not want_logits:
             del out["logits"]
+        if not want_vocab_margin:
+            del out["vocab_margin"]
         return out
 
 

@@ -35,6 +35,8 @@ struct orc_cache {
   uint8_t* valid;
   double* rel;        /* [B][Nv]: Stage-2 relevance from the previous step */
   uint8_t* rel_valid; /* [B]: rel holds the previous step's relevance */
+  int32_t* prev_ids;  /* [B][n_action]: the previous step's action bins */
+  uint8_t* ids_valid; /* [B]: prev_ids holds them */
 };
 
 /* ------------------------------------------------------------------------ */
@@ -308,6 +310,21 @@ void orc_margin(const double* lg, int n, int32_t* argmax, double* pmargin, doubl
   *lgap = l1 - l2;
 }
 
+/* Entropy of the softmax p_j = exp(l_j - l1) / z:  -sum p_j ln p_j
+ * = ln z - sum p_j (l_j - l1). */
+double orc_entropy(const double* lg, int n) {
+  double l1 = lg[0];
+  for (int j = 1; j < n; ++j)
+    if (lg[j] > l1) l1 = lg[j];
+  double z = 0.0, s = 0.0;
+  for (int j = 0; j < n; ++j) {
+    const double e = exp(lg[j] - l1);
+    z += e;
+    s += e * (lg[j] - l1);
+  }
+  return log(z) - s / z;
+}
+
 /* ------------------------------------------------------------------------ */
 /* Context and cache                                                        */
 /* ------------------------------------------------------------------------ */
@@ -375,7 +392,10 @@ int orc_cache_new(const orc_ctx* c, int batch, orc_cache** out) {
   k->valid = (uint8_t*)calloc((size_t)batch, 1);
   k->rel = (double*)calloc((size_t)batch * (c->Nv > 0 ? c->Nv : 1), sizeof(double));
   k->rel_valid = (uint8_t*)calloc((size_t)batch, 1);
-  if (!k->K || !k->V || !k->H || !k->prev || !k->m_prev || !k->valid || !k->rel || !k->rel_valid) {
+  k->prev_ids = (int32_t*)calloc((size_t)batch * c->d.n_action, sizeof(int32_t));
+  k->ids_valid = (uint8_t*)calloc((size_t)batch, 1);
+  if (!k->K || !k->V || !k->H || !k->prev || !k->m_prev || !k->valid || !k->rel || !k->rel_valid || !k->prev_ids ||
+      !k->ids_valid) {
     orc_cache_free(k);
     return ORC_ERR_OOM;
   }
@@ -393,6 +413,8 @@ void orc_cache_free(orc_cache* k) {
   free(k->valid);
   free(k->rel);
   free(k->rel_valid);
+  free(k->prev_ids);
+  free(k->ids_valid);
   free(k);
 }
 
@@ -400,7 +422,7 @@ void orc_cache_free(orc_cache* k) {
 int orc_reset(orc_cache* k, int seq) {
   if (!k || seq < -1 || seq >= k->B) return ORC_ERR_ARG;
   for (int b = 0; b < k->B; ++b)
-    if (seq == -1 || seq == b) k->valid[b] = k->rel_valid[b] = 0;
+    if (seq == -1 || seq == b) k->valid[b] = k->rel_valid[b] = k->ids_valid[b] = 0;
   return ORC_OK;
 }
 
@@ -563,18 +585,35 @@ static void embed_row(const orc_ctx* c, int pos, const uint8_t* frame, const int
   }
 }
 
-/* Final norm and the action-bin rows of the LM head -> logits, argmax, margins. */
-static void head_row(const orc_ctx* c, const float* x, double* logits, int32_t* id, double* pm, double* lg) {
-  const int Hd = c->d.hidden, nb = c->d.n_bins;
+/* Final norm and the action-bin rows of the LM head -> logits, argmax,
+ * margins, and the entropy of the bin softmax.  With vm != NULL also every
+ * other row of the LM head: p1 - p2 of the softmax over the whole
+ * vocabulary (the two largest probabilities of any tokens). */
+static void head_row(const orc_ctx* c, const float* x, double* logits, int32_t* id, double* pm, double* lg,
+                     double* ent, double* vm) {
+  const int Hd = c->d.hidden, nb = c->d.n_bins, V = c->d.vocab;
   double* h = (double*)malloc(sizeof(double) * Hd);
   double* wr = (double*)malloc(sizeof(double) * Hd);
   rmsnorm_row(c, x, c->w.final_norm, h);
   for (int j = 0; j < nb; ++j) {
-    const size_t row = (size_t)(c->d.vocab - nb + j);
+    const size_t row = (size_t)(V - nb + j);
     for (int e = 0; e < Hd; ++e) wr[e] = wget(c, c->w.lm_head, row * Hd + e);
     logits[j] = dot(h, wr, Hd);
   }
   orc_margin(logits, nb, id, pm, lg);
+  *ent = orc_entropy(logits, nb);
+  if (vm) {
+    double* all = (double*)malloc(sizeof(double) * V);
+    for (int r = 0; r < V - nb; ++r) {
+      for (int e = 0; e < Hd; ++e) wr[e] = wget(c, c->w.lm_head, (size_t)r * Hd + e);
+      all[r] = dot(h, wr, Hd);
+    }
+    memcpy(all + (V - nb), logits, sizeof(double) * nb);
+    int32_t top;
+    double gap;
+    orc_margin(all, V, &top, vm, &gap);
+    free(all);
+  }
   free(h);
   free(wr);
 }
@@ -668,18 +707,29 @@ static int step_seq(orc_ctx* c, orc_cache* k, int b, const uint8_t* frame, const
       for (int l = 0; l < L; ++l) layer_rows(c, k, b, l, 1, &p, xdec, NULL);
       xr = xdec;
     }
-    double pm, gap;
-    head_row(c, xr, lg, &ids[a], &pm, &gap);
+    double pm, gap, ent, vm = 0.0;
+    const int want_vm = (o && o->margin_kind == 2) || out->vocab_margin;
+    head_row(c, xr, lg, &ids[a], &pm, &gap, &ent, want_vm ? &vm : NULL);
     if (out->logits) memcpy(out->logits + ((size_t)b * D + a) * nb, lg, sizeof(double) * nb);
     out->margins[(size_t)b * D + a] = pm;
     out->logit_gap[(size_t)b * D + a] = gap;
-    const double sig = (o && o->margin_kind == 1) ? gap : pm;
+    if (out->entropy) out->entropy[(size_t)b * D + a] = ent;
+    if (out->vocab_margin) out->vocab_margin[(size_t)b * D + a] = vm;
+    const double sig = (o && o->margin_kind == 1) ? gap : (o && o->margin_kind == 2) ? vm : pm;
     sig_sum += sig;
     if (sig < sig_min) sig_min = sig;
     free(xdec);
   }
   const double m_t = (o && o->reduction == 1) ? sig_min : sig_sum / D;
   out->step_margin[b] = m_t;
+  /* action delta against the previous step's bins (Sec. VI) */
+  int32_t* pid = k->prev_ids + (size_t)b * D;
+  int32_t delta = 0;
+  if (k->ids_valid[b])
+    for (int a = 0; a < D; ++a) delta += abs(ids[a] - pid[a]);
+  if (out->action_delta) out->action_delta[b] = delta;
+  memcpy(pid, ids, sizeof(int32_t) * D);
+  k->ids_valid[b] = 1;
   k->m_prev[b] = m_t;
   k->valid[b] = 1;
   memcpy(prev, frame, fb);
@@ -694,6 +744,7 @@ int orc_step(orc_ctx* c, orc_cache* k, const uint8_t* frames, const int32_t* pro
       !out->margins || !out->logit_gap || !out->recomputed || !out->gate_auto || !out->step_margin || tau_den == 0)
     return ORC_ERR_ARG;
   if (c->d.proprio_dim > 0 && !proprio) return ORC_ERR_ARG;
+  if (opts && (opts->margin_kind < 0 || opts->margin_kind > 2)) return ORC_ERR_ARG;
   if (opts && (opts->s2_top_k < 0 || (opts->s2_top_k > 0 && (opts->s2_layer < 0 || opts->s2_layer >= c->d.n_layers))))
     return ORC_ERR_ARG;
   const size_t fb = frame_bytes(&c->d);

@@ -20,7 +20,11 @@
  *   - Sec. III-B Stage 3: a per-layer proportion of the static patches is
  *     reused (here a caller-given per-mille schedule).
  *   - Sec. IV-A Eq. (1): mean top-1/top-2 probability margin over the D
- *     action tokens.
+ *     action tokens, with the softmax over the action bins or (margin kind
+ *     2) over the whole vocabulary.
+ *   - Sec. VI: the alternative signals the paper evaluated, as outputs: the
+ *     entropy of each action token's distribution and the action delta
+ *     between consecutive steps.
  *   - Algorithm 1: gate on m_{t-1} < theta_m -> invalidate and run a full
  *     pass; otherwise reuse the cache and recompute only the rest; then
  *     decode the action tokens.
@@ -71,7 +75,8 @@ typedef struct orc_weights {
 } orc_weights;
 
 typedef struct orc_opts {
-  int32_t margin_kind;          /* 0 = probability p1 - p2 (Eq. 1), 1 = logit gap l1 - l2 */
+  int32_t margin_kind;          /* 0 = probability p1 - p2 over the bins (Eq. 1), 1 = logit gap
+                                   l1 - l2, 2 = probability p1 - p2 over the whole vocabulary */
   int32_t reduction;            /* 0 = mean over the action tokens (Eq. 1), 1 = minimum */
   const int8_t* gate_override;  /* [B]: -1 gate, 0 force cached, 1 force full; NULL = gate */
   const int32_t* forced_ids;    /* [B][n_action] bins fed back in decode; NULL = argmax */
@@ -92,6 +97,9 @@ typedef struct orc_out {
   int32_t* M;           /* [B][n_layers] rows recomputed per layer or NULL */
   double* relevance;    /* [B][n_visual] this step's Stage-2 relevance (0 when off) or NULL */
   uint8_t* relevant;    /* [B][n_visual] patches Stage 2 removed this step or NULL */
+  double* entropy;      /* [B][n_action] entropy (nats) of the bin softmax or NULL */
+  double* vocab_margin; /* [B][n_action] p1 - p2 of the softmax over the whole vocabulary or NULL */
+  int32_t* action_delta; /* [B] sum over d of |a_t^d - a_{t-1}^d| in bins (0 without a previous step) or NULL */
 } orc_out;
 
 typedef struct orc_ctx orc_ctx;
@@ -132,6 +140,8 @@ int orc_select2(const orc_dims* d, const uint8_t* frame, const uint8_t* prev, in
  * entries rank before it (higher value, or equal value and lower index). */
 void orc_top_k(const double* rel, int n, int top_k, uint8_t* out);
 void orc_margin(const double* logits, int n, int32_t* argmax, double* pmargin, double* lgap);
+/* -sum_j p_j ln p_j of the softmax of logits[0..n), in nats. */
+double orc_entropy(const double* logits, int n);
 double orc_round_bf16(double v);
 void orc_rope_table(const orc_dims* d, int n_pos, float* cos_t, float* sin_t);
 
