@@ -124,6 +124,13 @@ __device__ __forceinline__ void norm_rows_to_smem(const float* __restrict__ X, c
 // vector once into shared memory (x * r * g rounded to T).  bf16 vectors are
 // kept in A-fragment order: per 32-element K step and lane t the elements
 // (2t, 2t+1, 2t+8, 2t+9, 2t+16, 2t+17, 2t+24, 2t+25), one 16-byte load.
+//
+// Every ring wait is bounded (kWaitLimit polls).  A wait that gives up
+// latches VLAC_ERR_TIMEOUT and raises the CTA's give-up flag: the producer
+// stops issuing; the consumers run out their loops without computing or
+// handing stages back, so they stay in step at the named barriers; and a
+// consumer that gave up waits (bounded) for the producer's copies still
+// landing before the CTA exits.
 
 constexpr int kNC = 8;          // consumer warps
 constexpr int kGP = 4;          // row pairs per group
