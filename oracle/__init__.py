@@ -80,6 +80,8 @@ def lib():
             L.orc_step.argtypes = [vp, vp, vp, vp, vp, u32, u32, C.c_double, vp,
                                    C.POINTER(_Opts), C.POINTER(_Out)]
             L.orc_cache_read.argtypes = [vp, C.c_int, C.c_int, C.c_int, vp]
+            L.orc_cache_write.argtypes = [vp, C.c_int, C.c_int, C.c_int, vp]
+            L.orc_layer.argtypes = [vp, vp, C.c_int, C.c_int, C.c_int, vp, vp]
             L.orc_cache_state.argtypes = [vp, C.c_int, C.POINTER(C.c_double), C.POINTER(C.c_int)]
             L.orc_patch_stats.argtypes = [C.POINTER(_Dims), vp, vp, C.c_int, C.POINTER(C.c_int64),
                                           C.POINTER(C.c_int64), C.POINTER(C.c_int64)]
@@ -237,6 +239,17 @@ class Oracle:
     def new_cache(self, batch: int = 1) -> "OracleCache":
         return OracleCache(self, batch)
 
+    def layer(self, cache: "OracleCache", seq: int, layer: int, pos, x) -> np.ndarray:
+        """One decoder layer for the rows at positions `pos` with inputs x
+        [n][hidden]; returns their outputs (the cache's K/V at those positions
+        are written)."""
+        pos = np.ascontiguousarray(pos, dtype=np.int32)
+        out = np.array(x, dtype=np.float32, copy=True, order="C")
+        r = lib().orc_layer(self._h, cache._h, seq, layer, pos.size, _ptr(pos), _ptr(out))
+        if r != 0:
+            raise ValueError(f"orc_layer failed ({r})")
+        return out
+
     def step(self, cache: "OracleCache", frames, prompt, proprio=None, tau_sim=(996, 1000),
              tau_margin: float = 0.0, permille=None, margin_kind: int = 0, reduction: Optional[int] = None,
              gate_override=None, forced_ids=None, want_logits: bool = True, s2_top_k: int = 0,
@@ -310,6 +323,12 @@ class OracleCache:
         if lib().orc_cache_read(self._h, seq, k, layer, _ptr(dst)) != 0:
             raise ValueError("bad cache read")
         return dst
+
+    def write(self, seq: int, kind: str, layer: int, values: np.ndarray):
+        d = self.orc.d
+        src = np.ascontiguousarray(values, dtype=np.float32).reshape(d.cache_len, d.hidden)
+        if lib().orc_cache_write(self._h, seq, {"K": 0, "V": 1}[kind], layer, _ptr(src)) != 0:
+            raise ValueError("bad cache write")
 
     def state(self, seq: int):
         m, v = C.c_double(), C.c_int()

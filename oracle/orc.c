@@ -439,6 +439,16 @@ int orc_cache_read(const orc_cache* k, int seq, int kind, int layer, float* dst)
   return ORC_OK;
 }
 
+int orc_cache_write(orc_cache* k, int seq, int kind, int layer, const float* src) {
+  if (!k || !src) return ORC_ERR_ARG;
+  const orc_ctx* c = k->c;
+  if (seq < 0 || seq >= k->B || layer < 0 || layer >= c->d.n_layers || kind < 0 || kind > 1) return ORC_ERR_ARG;
+  const size_t Hd = c->d.hidden, L = c->d.n_layers;
+  float* dst = (kind == 0 ? k->K : k->V) + (((size_t)seq * L + layer) * c->T) * Hd;
+  memcpy(dst, src, sizeof(float) * c->T * Hd);
+  return ORC_OK;
+}
+
 int orc_cache_state(const orc_cache* k, int seq, double* m_prev, int* valid) {
   if (!k || seq < 0 || seq >= k->B) return ORC_ERR_ARG;
   *m_prev = k->m_prev[seq];
@@ -548,6 +558,19 @@ static void layer_rows(const orc_ctx* c, orc_cache* k, int b, int l, int n, cons
   for (size_t e = 0; e < (size_t)n * Hd; ++e) x[e] = (float)((double)x[e] + y[e]);
 
   free(h); free(q); free(kk); free(vv); free(att); free(y); free(g); free(u);
+}
+
+int orc_layer(orc_ctx* c, orc_cache* k, int seq, int layer, int n, const int32_t* pos, float* x) {
+  if (!c || !k || k->c != c || !pos || !x || seq < 0 || seq >= k->B || layer < 0 || layer >= c->d.n_layers ||
+      n < 1 || n > c->S)
+    return ORC_ERR_ARG;
+  for (int i = 0; i < n; ++i) {
+    if (pos[i] < 0 || pos[i] >= c->S) return ORC_ERR_ARG;
+    for (int j = 0; j < i; ++j)
+      if (pos[j] == pos[i]) return ORC_ERR_ARG;
+  }
+  layer_rows(c, k, seq, layer, n, pos, x, NULL);
+  return ORC_OK;
 }
 
 /* Layer-0 input of the token at `pos` (Sec. III-A layout: BOS, visual

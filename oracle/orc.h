@@ -118,6 +118,15 @@ int orc_step(orc_ctx* c, orc_cache* k, const uint8_t* frames, const int32_t* pro
 /* Copies one layer of sequence `seq`'s cache: kind 0 = K, 1 = V ([cache_len][hidden]),
  * 2 = H (layer inputs, [S][hidden]).  Values as stored (float). */
 int orc_cache_read(const orc_cache* k, int seq, int kind, int layer, float* dst);
+/* The reverse of orc_cache_read for K (kind 0) and V (kind 1): the values are
+ * stored as given. */
+int orc_cache_write(orc_cache* k, int seq, int kind, int layer, const float* src);
+/* One decoder layer (the Llama-2 block of Sec. III-A as the prefix pass runs
+ * it) for n rows of sequence `seq` at distinct positions pos[i] < the prefix
+ * pass length: x [n][hidden] holds the rows' layer inputs and receives their
+ * outputs; the rows' K/V are written into the cache at their positions before
+ * any row attends; attention is causal by position over the cache. */
+int orc_layer(orc_ctx* c, orc_cache* k, int seq, int layer, int n, const int32_t* pos, float* x);
 int orc_cache_state(const orc_cache* k, int seq, double* m_prev, int* valid);
 
 /* Pieces exposed for pin tests. */

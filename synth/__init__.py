@@ -206,6 +206,21 @@ def make_proprio(d: Dims, n_frames: int, seed: int = 0, batch: int = 1) -> Optio
     return np.cumsum(steps, axis=0).astype(np.float32)
 
 
+def make_layer_case(d: Dims, M: int, seed: int = 0):
+    """The one-layer workload: a seeded sample of M distinct prefix positions
+    (sorted), the rows' layer inputs N(0, 1) in float32 [M][hidden], and the
+    layer's cache K and V, each [cache_len][hidden] N(0, 1) stored in the
+    model's dtype (returned as float32 arrays holding those values)."""
+    rng = np.random.default_rng(seed * 7919 + M)
+    pos = np.sort(rng.choice(d.pass_len, size=M, replace=False)).astype(np.int32)
+    x = rng.normal(size=(M, d.hidden)).astype(np.float32)
+    kv = []
+    for key in (11, 12):
+        t = _normal((d.cache_len, d.hidden), seed, key, "cpu", _torch_dtype(d), std=1.0)
+        kv.append(t.float().numpy())
+    return pos, x, kv[0], kv[1]
+
+
 def linear_schedule(n_layers: int, first: int = 900, last: int = 500) -> np.ndarray:
     """Per-layer reuse proportion in per-mille, linear from `first` to `last`."""
     if n_layers == 1:
