@@ -54,7 +54,7 @@ class _Weights(C.Structure):
 class _Opts(C.Structure):
     _fields_ = [("margin_kind", C.c_int32), ("reduction", C.c_int32),
                 ("gate_override", C.c_void_p), ("forced_ids", C.c_void_p),
-                ("s2_top_k", C.c_int32), ("s2_layer", C.c_int32)]
+                ("s2_top_k", C.c_int32), ("s2_layer", C.c_int32), ("active", C.c_void_p)]
 
 
 class _Out(C.Structure):
@@ -253,7 +253,7 @@ class Oracle:
     def step(self, cache: "OracleCache", frames, prompt, proprio=None, tau_sim=(996, 1000),
              tau_margin: float = 0.0, permille=None, margin_kind: int = 0, reduction: Optional[int] = None,
              gate_override=None, forced_ids=None, want_logits: bool = True, s2_top_k: int = 0,
-             s2_layer: Optional[int] = None, want_vocab_margin: bool = False):
+             s2_layer: Optional[int] = None, want_vocab_margin: bool = False, active=None):
         d, B = self.d, cache.batch
         D, S, L = d.n_action, d.pass_len, d.n_layers
         frames = np.ascontiguousarray(frames, dtype=np.uint8).reshape(B, d.n_views, d.img_h, d.img_w, 3)
@@ -284,7 +284,8 @@ class Oracle:
                                            "relevance", "relevant", "entropy", "vocab_margin", "action_delta")])
         if s2_layer is None:
             s2_layer = L // 2
-        opts = _Opts(margin_kind, reduction, _ptr(go), _ptr(fi), int(s2_top_k), int(s2_layer))
+        act = None if active is None else np.ascontiguousarray(active, dtype=np.uint8).reshape(B)
+        opts = _Opts(margin_kind, reduction, _ptr(go), _ptr(fi), int(s2_top_k), int(s2_layer), _ptr(act))
         r = lib().orc_step(self._h, cache._h, _ptr(frames), _ptr(prompt), _ptr(proprio), tau_sim[0],
                            tau_sim[1], float(tau_margin), _ptr(permille), C.byref(opts), C.byref(co))
         if r != 0:

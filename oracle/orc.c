@@ -772,6 +772,26 @@ int orc_step(orc_ctx* c, orc_cache* k, const uint8_t* frames, const int32_t* pro
     return ORC_ERR_ARG;
   const size_t fb = frame_bytes(&c->d);
   for (int b = 0; b < k->B; ++b) {
+    if (opts && opts->active && !opts->active[b]) {
+      /* a sequence that sits the step out: nothing of it changes */
+      const size_t D = c->d.n_action, nb = c->d.n_bins, Nv = c->Nv, S = c->S, L = c->d.n_layers;
+      memset(out->action_ids + b * D, 0, sizeof(int32_t) * D);
+      memset(out->margins + b * D, 0, sizeof(double) * D);
+      memset(out->logit_gap + b * D, 0, sizeof(double) * D);
+      if (out->logits) memset(out->logits + b * D * nb, 0, sizeof(double) * D * nb);
+      out->recomputed[b] = 0;
+      out->gate_auto[b] = 0;
+      out->step_margin[b] = 0.0;
+      if (out->static_mask) memset(out->static_mask + b * Nv, 0, Nv);
+      if (out->idx) memset(out->idx + b * S, 0, sizeof(int32_t) * S);
+      if (out->M) memset(out->M + b * L, 0, sizeof(int32_t) * L);
+      if (out->relevance) memset(out->relevance + b * Nv, 0, sizeof(double) * Nv);
+      if (out->relevant) memset(out->relevant + b * Nv, 0, Nv);
+      if (out->entropy) memset(out->entropy + b * D, 0, sizeof(double) * D);
+      if (out->vocab_margin) memset(out->vocab_margin + b * D, 0, sizeof(double) * D);
+      if (out->action_delta) out->action_delta[b] = 0;
+      continue;
+    }
     int r = step_seq(c, k, b, frames + (size_t)b * fb, prompt_ids + (size_t)b * c->d.n_text,
                      proprio ? proprio + (size_t)b * c->d.proprio_dim : NULL, tau_num, tau_den, tau_margin,
                      reuse_permille, opts, out);

@@ -82,6 +82,8 @@ typedef struct orc_opts {
   const int32_t* forced_ids;    /* [B][n_action] bins fed back in decode; NULL = argmax */
   int32_t s2_top_k;             /* Stage 2: patches removed per step; 0 = Stage 2 off */
   int32_t s2_layer;             /* Stage 2: the layer whose attention gives the relevance */
+  const uint8_t* active;        /* [B]: 0 = this sequence sits the step out (its cache and state
+                                   stay as they are, its outputs are zero); NULL = all step */
 } orc_opts;
 
 typedef struct orc_out {
