@@ -1,0 +1,61 @@
+"""The benchmark's step work model (the roofline denominators it reports)
+against hand counts for the OpenVLA-7B shape: 6,476,005,376 backbone
+parameters (12.95 GB of bf16 weights per pass), seven passes per step (the
+prefix pass and six single-token decode passes), 2 FLOPs per multiply-add."""
+import os
+import sys
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+import synth  # noqa: E402
+
+D = synth.dims_for("openvla7b")
+PER_LAYER = 4 * 4096 * 4096 + 3 * 11008 * 4096
+W_PASS = 32 * PER_LAYER * 2  # bytes of bf16 backbone weights read by one pass
+
+
+def _full():
+    S = D.pass_len
+    return [S] * D.n_layers, np.arange(S)
+
+
+def test_backbone_size():
+    assert 32 * PER_LAYER == 6_476_005_376
+    assert W_PASS == pytest.approx(12.95e9, rel=1e-3)
+
+
+def test_full_step_counts():
+    M, idx = _full()
+    passes = bench.step_work(D, M, idx)
+    assert len(passes) == D.n_action  # prefix + 6 decode passes
+    # every pass reads the backbone once (plus the head rows; the prefix pass also the patch projection)
+    for f, b, w in passes:
+        assert W_PASS <= w < W_PASS * 1.01
+    f0 = passes[0][0]
+    gemm = D.pass_len * 2 * 32 * PER_LAYER
+    assert gemm <= f0 < gemm * 1.05  # attention, patch embedding and head are a few per cent
+    F, B, _ = bench.batch_work(D, [M], [idx])
+    assert F == pytest.approx(sum(p[0] for p in passes))
+    assert B == pytest.approx(sum(p[1] + p[2] for p in passes))
+    # the step is HBM-bound at the measured peaks: about 13.6 ms of 91-92 GB
+    t = max(F / 1891.6e12, B / 6754.1e9)
+    assert B == pytest.approx(92.0e9, rel=0.01)
+    assert t == pytest.approx(13.6e-3, rel=0.01)
+
+
+def test_cached_rows_cut_only_the_prefix_flops():
+    S = D.pass_len
+    M_full, idx = _full()
+    M_cached = [S - (int(p) * 230) // 1000 for p in synth.linear_schedule(D.n_layers)]
+    full = bench.step_work(D, M_full, idx)
+    cached = bench.step_work(D, M_cached, idx)
+    assert cached[0][0] < full[0][0]
+    # decode passes and weight bytes do not depend on the reuse
+    for a, b in zip(full[1:], cached[1:]):
+        assert a == b
+    assert cached[0][2] == full[0][2]
