@@ -59,3 +59,31 @@ def test_cached_rows_cut_only_the_prefix_flops():
     for a, b in zip(full[1:], cached[1:]):
         assert a == b
     assert cached[0][2] == full[0][2]
+
+
+class _FakeSmi:
+    def __init__(self, text):
+        self.text = text
+
+    def terminate(self):
+        pass
+
+    def communicate(self, timeout=None):
+        return self.text, ""
+
+
+def test_clock_samples_are_parsed():
+    """The clocks line of the bench: median SM clock under load, the maximum,
+    and every throttle reason seen Active in any sample."""
+    rows = ["0, 2070, 2070, 900.5, 0x0, Not Active, Not Active, Not Active, Not Active",
+            "0, 1980, 2070, 1390.0, 0x4, Not Active, Not Active, Not Active, Active",
+            "0, 2070, 2070, 1100.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+            "garbage line",
+            "0, [N/A], 2070, 0, 0x0, Not Active, Not Active, Not Active, Not Active"]
+    c = bench.Clocks.__new__(bench.Clocks)
+    c.p = _FakeSmi("\n".join(rows))
+    got = c.stop()
+    assert got["sm_mhz"] == 2070.0 and got["sm_max_mhz"] == 2070.0 and got["samples"] == 3
+    assert got["reasons"] == ["sw_power_cap"]
+    c.p = None
+    assert c.stop()["reasons"] == ["nvidia-smi unavailable"]
