@@ -45,7 +45,7 @@ def test_strerror_names_every_code(lib):
 
 
 def test_invalid_dims_rejected_without_a_device(lib):
-    from paper_2608_10824_gb300.vlac import Dims, Weights, c_dims
+    from paper_2608_10824_gb300.vlac import Weights, c_dims
     h = C.c_void_p()
     w = Weights()
     bad = [

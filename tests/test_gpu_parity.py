@@ -2,7 +2,6 @@
 span several GEMM tiles and ragged tails: selection indices, per-layer row
 counts, static masks and recompute flags bit-exact; logits within the stated
 tolerance; action ids exact outside the small-margin exemption."""
-import numpy as np
 import pytest
 
 import synth
