@@ -8,6 +8,8 @@
 //   - gemm_simt: the fp32 tiny model.
 // The decode passes (M = batch <= 8) use the fused weight-streaming GEMV in
 // k_decode.cu.
+#include <cstdlib>
+
 #include "internal.cuh"
 
 namespace vlac {
@@ -141,8 +143,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   pdl_wait();
   pdl_trigger();
-  const int M = min(*m_ptr, m_cap);
-  if (M <= 0) return;
+  const int M_all = min(*m_ptr, m_cap);
+  if (M_all <= 0) return;
+  // token blocks (gridDim.y > 1): above kOnePass rows every CTA takes one
+  // block of kMaxTok rows, so the blocks of a tile run side by side instead
+  // of as passes of one CTA; at or below it block 0 takes every row
+  int row_base = 0, M = M_all;
+  if (gridDim.y > 1) {
+    if (M_all <= kOnePass) {
+      if (blockIdx.y > 0) return;
+    } else {
+      row_base = (int)blockIdx.y * kMaxTok;
+      if (row_base >= M_all) return;
+      M = min(M_all - row_base, kMaxTok);
+    }
+  }
   const int nk = kc1 - kc0;
   if (nk <= 0) return;
   // token passes: one pass up to kOnePass tokens, else passes of kMaxTok
@@ -209,7 +224,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // the token rows in as few boxes as possible: 256, 128, 64 and 32 rows
           for (int done = 0, left = nbox; left > 0;) {
             const int lg = left >= 8 ? 3 : left >= 4 ? 2 : left >= 2 ? 1 : 0;
-            tma_load_2d(at + (size_t)done * kBoxRows * 128, &tmA.m[lg], kc * kBK, row0 + done * kBoxRows,
+            tma_load_2d(at + (size_t)done * kBoxRows * 128, &tmA.m[lg], kc * kBK, row_base + row0 + done * kBoxRows,
                         &full_bar[stage]);
             done += 1 << lg;
             left -= 1 << lg;
@@ -330,7 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
             const int m = row0 + c0 + j;
-            if (m < M) dst[(size_t)m * ld + n] = v[j];
+            if (m < M) dst[(size_t)(row_base + m) * ld + n] = v[j];
           }
           continue;
         }
@@ -344,7 +359,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
           const int m = row0 + c0 + j;
-          if (m < M) dst[(size_t)m * ld + n] = v[j];
+          if (m < M) dst[(size_t)(row_base + m) * ld + n] = v[j];
         }
       }
       fence_before();
@@ -377,7 +392,14 @@ void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr
   const int k_chunks = K / tc::kBK;
   const int cps = (k_chunks + sp.tail - 1) / sp.tail;
   const int full_tiles = sp.full_cols / tc::kBM, n_tiles = N / tc::kBM;
-  dim3 grid(full_tiles + (n_tiles - full_tiles) * sp.tail);
+  // token blocks side by side when the rows can exceed one pass (the CTAs of
+  // blocks a step does not need return at once)
+  static const bool token_blocks = [] {
+    const char* e = std::getenv("VLAC_GEMM_TOKEN_BLOCKS");
+    return !e || std::atoi(e) != 0;
+  }();
+  const int tb = (token_blocks && m_cap > tc::kOnePass) ? (m_cap + tc::kMaxTok - 1) / tc::kMaxTok : 1;
+  dim3 grid(full_tiles + (n_tiles - full_tiles) * sp.tail, tb);
   launch_k(tc::gemm_tc_kernel, grid, dim3(tc::kThreads), tc::kSmemBytes, st, *tmA, *tmW, m_ptr, m_cap, N, k_chunks,
            cps, out, sp.stride, full_tiles, sp.tail, sp.tail_p, sp.tail_stride, sp.tail_ld, err, wait_limit);
 }
