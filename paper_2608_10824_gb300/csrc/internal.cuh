@@ -26,6 +26,22 @@ struct StepParams {
   uint16_t permille[kMaxLayers];
 };
 
+// Where the K-split partial sums of a prefix GEMM live (out[s][m][n] of
+// launch_gemm_tc).  Columns below full_cols come from CTAs that ran the whole
+// K range: one partial, at part.  The other columns have `tail` partials: the
+// first at part, split s >= 1 either at part + s * stride (the uniform
+// layout, tail_ld == 0) or compactly at
+// tail_p + (s - 1) * tail_stride + row * tail_ld + (col - full_cols).
+struct SplitPlan {
+  int full_cols;
+  int tail;
+  size_t stride;
+  float* tail_p;
+  size_t tail_stride;
+  int tail_ld;
+};
+inline SplitPlan uniform_splits(int splits, size_t stride) { return SplitPlan{0, splits, stride, nullptr, 0, 0}; }
+
 // A set of rows processed by one layer: per sequence b, rows i < count_b with
 // count_b = off[b+1] - off[b]; the compacted row index is off[b] + i, the
 // token position is idx[b * idx_stride + i], and the fp32 residual row lives at
@@ -255,17 +271,15 @@ template <typename T>
 void launch_layer_in(Rows rows, const int* off_prev, int B, int S, int hidden, float* H, size_t h_seq_stride,
                      const T* gain, float eps, T* A, cudaStream_t st);
 template <typename T>
-void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, int splits,
-                         size_t split_stride, const float* rope_cos, const float* rope_sin, T* Q, T* Kc,
-                         T* Vc, size_t kv_seq_stride, int Tc, cudaStream_t st);
+void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, const SplitPlan& sp,
+                         const float* rope_cos, const float* rope_sin, T* Q, T* Kc, T* Vc, size_t kv_seq_stride,
+                         int Tc, cudaStream_t st);
 template <typename T>
-void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part, int splits,
-                          size_t split_stride, const T* gain, float eps, T* A, cudaStream_t st);
+void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part, const SplitPlan& sp, const T* gain,
+                          float eps, T* A, cudaStream_t st);
 template <typename T>
-void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, int splits, size_t split_stride, T* G,
-                   cudaStream_t st);
-void launch_residual(Rows rows, int B, int S, int hidden, const float* part, int splits, size_t split_stride,
-                     cudaStream_t st);
+void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, const SplitPlan& sp, T* G, cudaStream_t st);
+void launch_residual(Rows rows, int B, int S, int hidden, const float* part, const SplitPlan& sp, cudaStream_t st);
 template <typename T>
 void launch_attention(Rows rows, int B, int S, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc,
                       size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, T* O, cudaStream_t st);
@@ -297,8 +311,11 @@ struct ActMaps {
   CUtensorMap m[4];
 };
 // GEMMs: out[s][m][n] = sum over split s of A[m][k] * W[n][k]; rows m < *m_ptr.
+// Split plan sp: CTAs for the first sp.full_cols / 128 weight tiles run the
+// whole K range; every other tile is cut into sp.tail K ranges (see SplitPlan
+// for where each partial goes).
 void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
-                    int splits, float* out, int* err, uint32_t wait_limit, cudaStream_t st);
+                    const SplitPlan& sp, float* out, int* err, uint32_t wait_limit, cudaStream_t st);
 template <typename T>
 void launch_gemm_simt(const T* A, const T* W, const int* m_ptr, int m_cap, int N, int K, float* out,
                       cudaStream_t st);

@@ -8,6 +8,8 @@
 //   - gemm_simt: the fp32 tiny model.
 // The decode passes (M = batch <= 8) use the fused weight-streaming GEMV in
 // k_decode.cu.
+#include <cstdlib>
+
 #include "internal.cuh"
 
 namespace vlac {
@@ -95,7 +97,9 @@ __device__ __forceinline__ uint32_t idesc_bf16(int n) {
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ ActMaps tmA, const __grid_constant__ CUtensorMap tmW,
                    const int* __restrict__ m_ptr, int m_cap, int N, int k_chunks, int chunks_per_split,
-                   float* __restrict__ out, size_t split_stride, int* __restrict__ err, uint32_t wait_limit) {
+                   float* __restrict__ out, size_t split_stride, int full_tiles, int tail,
+                   float* __restrict__ tail_out, size_t tail_stride, int tail_ld, int* __restrict__ err,
+                   uint32_t wait_limit) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kMaxStages];
   __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
@@ -108,24 +112,52 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   uint8_t* tiles = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // this CTA's weight tile and K range: the first full_tiles CTAs run a whole
+  // tile; the rest cut the remaining tiles into `tail` K ranges each (with
+  // full_tiles == 0 in the order of a (tiles x splits) grid)
+  const int n_tiles = N / kBM;
+  int tile, sidx;  // sidx -1: the whole K range
+  if ((int)blockIdx.x < full_tiles) {
+    tile = blockIdx.x;
+    sidx = -1;
+  } else if (full_tiles == 0) {
+    tile = blockIdx.x % n_tiles;
+    sidx = blockIdx.x / n_tiles;
+  } else {
+    const int j = blockIdx.x - full_tiles;
+    tile = full_tiles + j / tail;
+    sidx = j - (j / tail) * tail;
+  }
+  const int n0 = tile * kBM;
+  const int kc0 = sidx < 0 ? 0 : sidx * chunks_per_split;
+  const int kc1 = sidx < 0 ? k_chunks : min(kc0 + chunks_per_split, k_chunks);
   if (threadIdx.x == 0) {
     // the weight tiles do not depend on earlier kernels: start pulling the
     // first ones into L2 while the previous kernel drains
-    const int k0 = blockIdx.y * chunks_per_split;
-    const int k1 = min(min(k0 + chunks_per_split, k_chunks), k0 + kPrefetchChunks);
-    for (int kc = k0; kc < k1; ++kc)
+    const int k1 = min(kc1, kc0 + kPrefetchChunks);
+    for (int kc = kc0; kc < k1; ++kc)
       asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
                        reinterpret_cast<uint64_t>(&tmW)),
-                   "r"(kc * kBK), "r"((int)blockIdx.x * kBM)
+                   "r"(kc * kBK), "r"(n0)
                    : "memory");
   }
   pdl_wait();
   pdl_trigger();
-  const int M = min(*m_ptr, m_cap);
-  if (M <= 0) return;
-  const int n0 = blockIdx.x * kBM;
-  const int kc0 = blockIdx.y * chunks_per_split;
-  const int kc1 = min(kc0 + chunks_per_split, k_chunks);
+  const int M_all = min(*m_ptr, m_cap);
+  if (M_all <= 0) return;
+  // token blocks (gridDim.y > 1): above kOnePass rows every CTA takes one
+  // block of kMaxTok rows, so the blocks of a tile run side by side instead
+  // of as passes of one CTA; at or below it block 0 takes every row
+  int row_base = 0, M = M_all;
+  if (gridDim.y > 1) {
+    if (M_all <= kOnePass) {
+      if (blockIdx.y > 0) return;
+    } else {
+      row_base = (int)blockIdx.y * kMaxTok;
+      if (row_base >= M_all) return;
+      M = min(M_all - row_base, kMaxTok);
+    }
+  }
   const int nk = kc1 - kc0;
   if (nk <= 0) return;
   // token passes: one pass up to kOnePass tokens, else passes of kMaxTok
@@ -192,7 +224,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // the token rows in as few boxes as possible: 256, 128, 64 and 32 rows
           for (int done = 0, left = nbox; left > 0;) {
             const int lg = left >= 8 ? 3 : left >= 4 ? 2 : left >= 2 ? 1 : 0;
-            tma_load_2d(at + (size_t)done * kBoxRows * 128, &tmA.m[lg], kc * kBK, row0 + done * kBoxRows,
+            tma_load_2d(at + (size_t)done * kBoxRows * 128, &tmA.m[lg], kc * kBK, row_base + row0 + done * kBoxRows,
                         &full_bar[stage]);
             done += 1 << lg;
             left -= 1 << lg;
@@ -270,8 +302,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // ---------------- epilogue: TMEM -> fp32 partials ----------------
     const int q = warp & 3;  // TMEM lane quarter this warp may access
-    const int n = n0 + q * 32 + lane;
-    float* dst = out + (size_t)blockIdx.y * split_stride;
+    // where this CTA's partial goes: split 0 (or a whole tile) into out, a
+    // later split into its uniform slot or the compact tail slots
+    float* dst = out;
+    int ld = N, n = n0 + q * 32 + lane;
+    if (sidx > 0) {
+      if (tail_ld) {
+        dst = tail_out + (size_t)(sidx - 1) * tail_stride;
+        ld = tail_ld;
+        n -= full_tiles * kBM;
+      } else {
+        dst = out + (size_t)sidx * split_stride;
+      }
+    }
     for (int pass = 0; pass < n_pass; ++pass) {
       const int row0 = pass * pass_tok;
       const int rows = min(M - row0, pass_tok);
@@ -302,7 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
             const int m = row0 + c0 + j;
-            if (m < M) dst[(size_t)m * N + n] = v[j];
+            if (m < M) dst[(size_t)(row_base + m) * ld + n] = v[j];
           }
           continue;
         }
@@ -316,7 +359,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
           const int m = row0 + c0 + j;
-          if (m < M) dst[(size_t)m * N + n] = v[j];
+          if (m < M) dst[(size_t)(row_base + m) * ld + n] = v[j];
         }
       }
       fence_before();
@@ -340,17 +383,25 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace tc
 
 void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
-                    int splits, float* out, int* err, uint32_t wait_limit, cudaStream_t st) {
+                    const SplitPlan& sp, float* out, int* err, uint32_t wait_limit, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
     cudaFuncSetAttribute(tc::gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, tc::kSmemBytes);
     attr_set = true;
   }
   const int k_chunks = K / tc::kBK;
-  const int cps = (k_chunks + splits - 1) / splits;
-  dim3 grid(N / tc::kBM, splits);
+  const int cps = (k_chunks + sp.tail - 1) / sp.tail;
+  const int full_tiles = sp.full_cols / tc::kBM, n_tiles = N / tc::kBM;
+  // token blocks side by side when the rows can exceed one pass (the CTAs of
+  // blocks a step does not need return at once)
+  static const bool token_blocks = [] {
+    const char* e = std::getenv("VLAC_GEMM_TOKEN_BLOCKS");
+    return !e || std::atoi(e) != 0;
+  }();
+  const int tb = (token_blocks && m_cap > tc::kOnePass) ? (m_cap + tc::kMaxTok - 1) / tc::kMaxTok : 1;
+  dim3 grid(full_tiles + (n_tiles - full_tiles) * sp.tail, tb);
   launch_k(tc::gemm_tc_kernel, grid, dim3(tc::kThreads), tc::kSmemBytes, st, *tmA, *tmW, m_ptr, m_cap, N, k_chunks,
-           cps, out, (size_t)m_cap * N, err, wait_limit);
+           cps, out, sp.stride, full_tiles, sp.tail, sp.tail_p, sp.tail_stride, sp.tail_ld, err, wait_limit);
 }
 
 // =============================================================================

@@ -105,10 +105,17 @@ __device__ __forceinline__ float4 add4(float4 a, float4 b) {
 __device__ __forceinline__ float sq4(float4 a, float acc) {
   return fmaf(a.w, a.w, fmaf(a.z, a.z, fmaf(a.y, a.y, fmaf(a.x, a.x, acc))));
 }
-// Sum over the GEMM's K splits (split s at part + s * stride), in split order.
-__device__ __forceinline__ float4 sum_splits4(const float* __restrict__ part, int splits, size_t stride, size_t o) {
-  float4 v = *reinterpret_cast<const float4*>(part + o);
-  for (int s = 1; s < splits; ++s) v = add4(v, *reinterpret_cast<const float4*>(part + o + (size_t)s * stride));
+// Sum over the GEMM's K splits of column o of compacted row r (pr = that
+// row of split 0), in split order; see SplitPlan for the layout.
+__device__ __forceinline__ float4 sum_splits4(const float* __restrict__ pr, const SplitPlan& sp, int r, size_t o) {
+  float4 v = *reinterpret_cast<const float4*>(pr + o);
+  if ((long long)o < sp.full_cols) return v;
+  if (sp.tail_ld) {
+    const float* t = sp.tail_p + (size_t)r * sp.tail_ld + (o - sp.full_cols);
+    for (int s = 1; s < sp.tail; ++s) v = add4(v, *reinterpret_cast<const float4*>(t + (size_t)(s - 1) * sp.tail_stride));
+  } else {
+    for (int s = 1; s < sp.tail; ++s) v = add4(v, *reinterpret_cast<const float4*>(pr + o + (size_t)s * sp.stride));
+  }
   return v;
 }
 
@@ -174,7 +181,7 @@ __global__ void layer_in_kernel(Rows rows, const int* __restrict__ off_prev, int
 // takes four consecutive e of one head and their partners e + half.
 template <typename T>
 __global__ void qkv_epilogue_kernel(Rows rows, int n_heads, int head_dim, const float* __restrict__ part,
-                                    int splits, size_t split_stride, const float* __restrict__ rope_cos,
+                                    SplitPlan sp, const float* __restrict__ rope_cos,
                                     const float* __restrict__ rope_sin, T* __restrict__ Q, T* __restrict__ Kc,
                                     T* __restrict__ Vc, size_t kv_seq_stride, int Tc) {
   pdl_wait();
@@ -195,12 +202,12 @@ __global__ void qkv_epilogue_kernel(Rows rows, int n_heads, int head_dim, const 
     const float4 c = *reinterpret_cast<const float4*>(rope_cos + (size_t)pos * half + e);
     const float4 s = *reinterpret_cast<const float4*>(rope_sin + (size_t)pos * half + e);
     const size_t base = (size_t)h * head_dim + e;
-    const float4 q1 = sum_splits4(pr, splits, split_stride, base);
-    const float4 q2 = sum_splits4(pr, splits, split_stride, base + half);
-    const float4 k1 = sum_splits4(pr, splits, split_stride, hidden + base);
-    const float4 k2 = sum_splits4(pr, splits, split_stride, hidden + base + half);
-    const float4 v1 = sum_splits4(pr, splits, split_stride, 2 * hidden + base);
-    const float4 v2 = sum_splits4(pr, splits, split_stride, 2 * hidden + base + half);
+    const float4 q1 = sum_splits4(pr, sp, r, base);
+    const float4 q2 = sum_splits4(pr, sp, r, base + half);
+    const float4 k1 = sum_splits4(pr, sp, r, hidden + base);
+    const float4 k2 = sum_splits4(pr, sp, r, hidden + base + half);
+    const float4 v1 = sum_splits4(pr, sp, r, 2 * hidden + base);
+    const float4 v2 = sum_splits4(pr, sp, r, 2 * hidden + base + half);
     store4<T>(q_out + base, make_float4(q1.x * c.x - q2.x * s.x, q1.y * c.y - q2.y * s.y, q1.z * c.z - q2.z * s.z,
                                         q1.w * c.w - q2.w * s.w));
     store4<T>(q_out + base + half, make_float4(q2.x * c.x + q1.x * s.x, q2.y * c.y + q1.y * s.y,
@@ -217,8 +224,8 @@ __global__ void qkv_epilogue_kernel(Rows rows, int n_heads, int head_dim, const 
 
 // x += o-projection (summed over splits), then A = T(RMSNorm(x) * g).
 template <typename T>
-__global__ void residual_norm_kernel(Rows rows, int hidden, const float* __restrict__ part, int splits,
-                                     size_t split_stride, const T* __restrict__ gain, float eps, T* __restrict__ A) {
+__global__ void residual_norm_kernel(Rows rows, int hidden, const float* __restrict__ part, SplitPlan sp,
+                                     const T* __restrict__ gain, float eps, T* __restrict__ A) {
   pdl_wait();
   pdl_trigger();
   __shared__ float red[32];
@@ -231,7 +238,7 @@ __global__ void residual_norm_kernel(Rows rows, int hidden, const float* __restr
   float ss = 0.f;
 #pragma unroll 4
   for (int c = threadIdx.x; c < hidden / 4; c += blockDim.x) {
-    const float4 v = add4(reinterpret_cast<const float4*>(x)[c], sum_splits4(pr, splits, split_stride, 4 * (size_t)c));
+    const float4 v = add4(reinterpret_cast<const float4*>(x)[c], sum_splits4(pr, sp, r, 4 * (size_t)c));
     reinterpret_cast<float4*>(x)[c] = v;
     ss = sq4(v, ss);
   }
@@ -240,8 +247,7 @@ __global__ void residual_norm_kernel(Rows rows, int hidden, const float* __restr
 
 // G = T(silu(g) * u) from the fused projection [gate | up].
 template <typename T>
-__global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part, int splits, size_t split_stride,
-                              T* __restrict__ G) {
+__global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part, SplitPlan sp, T* __restrict__ G) {
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.y, i = blockIdx.x;
@@ -254,8 +260,8 @@ __global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part
   const int c1 = (int)(((long long)n4 * (blockIdx.z + 1)) / gridDim.z);
 #pragma unroll 4
   for (int c = c0 + threadIdx.x; c < c1; c += blockDim.x) {
-    const float4 g = sum_splits4(pr, splits, split_stride, 4 * (size_t)c);
-    const float4 u = sum_splits4(pr, splits, split_stride, (size_t)ffn + 4 * c);
+    const float4 g = sum_splits4(pr, sp, r, 4 * (size_t)c);
+    const float4 u = sum_splits4(pr, sp, r, (size_t)ffn + 4 * c);
     store4<T>(G + (size_t)r * ffn + 4 * c,
               make_float4((g.x / (1.0f + expf(-g.x))) * u.x, (g.y / (1.0f + expf(-g.y))) * u.y,
                           (g.z / (1.0f + expf(-g.z))) * u.z, (g.w / (1.0f + expf(-g.w))) * u.w));
@@ -263,8 +269,7 @@ __global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part
 }
 
 // x += down-projection (summed over splits).
-__global__ void residual_kernel(Rows rows, int hidden, const float* __restrict__ part, int splits,
-                                size_t split_stride) {
+__global__ void residual_kernel(Rows rows, int hidden, const float* __restrict__ part, SplitPlan sp) {
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.y, i = blockIdx.x;
@@ -279,7 +284,7 @@ __global__ void residual_kernel(Rows rows, int hidden, const float* __restrict__
 #pragma unroll 4
   for (int c = c0 + threadIdx.x; c < c1; c += blockDim.x)
     reinterpret_cast<float4*>(x)[c] =
-        add4(reinterpret_cast<const float4*>(x)[c], sum_splits4(pr, splits, split_stride, 4 * (size_t)c));
+        add4(reinterpret_cast<const float4*>(x)[c], sum_splits4(pr, sp, r, 4 * (size_t)c));
 }
 
 // Autoregressive decode input: the bin fed back (argmax, or the forced replay
@@ -389,26 +394,23 @@ void launch_layer_in(Rows rows, const int* off_prev, int B, int S, int hidden, f
   launch_k(layer_in_kernel<T>, dim3(S, B), dim3(kNormThreads), 0, st, rows, off_prev, hidden, H, h_seq_stride, gain, eps, A);
 }
 template <typename T>
-void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, int splits,
-                         size_t split_stride, const float* rope_cos, const float* rope_sin, T* Q, T* Kc, T* Vc,
-                         size_t kv_seq_stride, int Tc, cudaStream_t st) {
-  launch_k(qkv_epilogue_kernel<T>, dim3(S, B, 2), dim3(256), 0, st, rows, n_heads, head_dim, part, splits, split_stride,
-           rope_cos, rope_sin, Q, Kc, Vc, kv_seq_stride, Tc);
+void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, const SplitPlan& sp,
+                         const float* rope_cos, const float* rope_sin, T* Q, T* Kc, T* Vc, size_t kv_seq_stride,
+                         int Tc, cudaStream_t st) {
+  launch_k(qkv_epilogue_kernel<T>, dim3(S, B, 2), dim3(256), 0, st, rows, n_heads, head_dim, part, sp, rope_cos,
+           rope_sin, Q, Kc, Vc, kv_seq_stride, Tc);
 }
 template <typename T>
-void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part, int splits, size_t split_stride,
-                          const T* gain, float eps, T* A, cudaStream_t st) {
-  launch_k(residual_norm_kernel<T>, dim3(S, B), dim3(kNormThreads), 0, st, rows, hidden, part, splits, split_stride, gain, eps,
-           A);
+void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part, const SplitPlan& sp, const T* gain,
+                          float eps, T* A, cudaStream_t st) {
+  launch_k(residual_norm_kernel<T>, dim3(S, B), dim3(kNormThreads), 0, st, rows, hidden, part, sp, gain, eps, A);
 }
 template <typename T>
-void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, int splits, size_t split_stride, T* G,
-                   cudaStream_t st) {
-  launch_k(swiglu_kernel<T>, dim3(S, B, 4), dim3(256), 0, st, rows, ffn, part, splits, split_stride, G);
+void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, const SplitPlan& sp, T* G, cudaStream_t st) {
+  launch_k(swiglu_kernel<T>, dim3(S, B, 4), dim3(256), 0, st, rows, ffn, part, sp, G);
 }
-void launch_residual(Rows rows, int B, int S, int hidden, const float* part, int splits, size_t split_stride,
-                     cudaStream_t st) {
-  launch_k(residual_kernel, dim3(S, B, 4), dim3(256), 0, st, rows, hidden, part, splits, split_stride);
+void launch_residual(Rows rows, int B, int S, int hidden, const float* part, const SplitPlan& sp, cudaStream_t st) {
+  launch_k(residual_kernel, dim3(S, B, 4), dim3(256), 0, st, rows, hidden, part, sp);
 }
 template <typename T>
 void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
@@ -429,11 +431,11 @@ void launch_finish(int B, int D, const StepParams* prm, const float* margins, co
                                 const T*, const float*, const T*, const T*, int*, cudaStream_t);                 \
   template void launch_layer_in<T>(Rows, const int*, int, int, int, float*, size_t, const T*, float, T*,          \
                                    cudaStream_t);                                                                 \
-  template void launch_qkv_epilogue<T>(Rows, int, int, int, int, const float*, int, size_t, const float*,         \
+  template void launch_qkv_epilogue<T>(Rows, int, int, int, int, const float*, const SplitPlan&, const float*,  \
                                        const float*, T*, T*, T*, size_t, int, cudaStream_t);                      \
-  template void launch_residual_norm<T>(Rows, int, int, int, const float*, int, size_t, const T*, float, T*,      \
+  template void launch_residual_norm<T>(Rows, int, int, int, const float*, const SplitPlan&, const T*, float, T*, \
                                         cudaStream_t);                                                            \
-  template void launch_swiglu<T>(Rows, int, int, int, const float*, int, size_t, T*, cudaStream_t);               \
+  template void launch_swiglu<T>(Rows, int, int, int, const float*, const SplitPlan&, T*, cudaStream_t);          \
   template void launch_decode_embed<T>(int, int, int, int, int, int, int, const T*, const int32_t*,               \
                                        const int32_t*, const StepParams*, float*, int*, float*, int*, cudaStream_t);
 VLAC_INST(float)

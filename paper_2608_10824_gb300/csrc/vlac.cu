@@ -60,6 +60,11 @@ struct vlac_ctx {
   CUtensorMap tm_patch;
   ActMaps tm_A, tm_AO, tm_G, tm_col;
   int split_qkv = 1, split_o = 1, split_gu = 1, split_d = 1;
+  // where each projection's K-split partials go (uniform splits, or whole
+  // tiles plus K-split tail tiles when the tiles exceed one wave of SMs)
+  SplitPlan sp_qkv{}, sp_o{}, sp_gu{}, sp_d{};
+  float* part_tail = nullptr;  // compact partials of the tail tiles' later splits
+  size_t part_tail_elems = 0;
   // workspace
   char* wsmem = nullptr;
   float *X, *Xd, *part;
@@ -366,6 +371,37 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     }
   }
 
+  // ---- tail tiles: a projection with more weight tiles than one wave of
+  // CTAs (one per SM) runs whole tiles for every full wave and cuts each
+  // remaining tile's K range over the SMs the last wave would leave idle;
+  // only those tiles have more than one partial ----
+  {
+    int plan_sms = c->n_sm;
+    if (const char* e = std::getenv("VLAC_PLAN_SMS")) plan_sms = std::max(1, std::atoi(e));  // tests and sweeps
+    bool tail_on = c->bf16;
+    if (const char* e = std::getenv("VLAC_GEMM_TAIL")) tail_on = tail_on && std::atoi(e) != 0;
+    const size_t rcap = c->rows_cap;
+    auto plan = [&](int N, int K, int split) {
+      const int tiles = N / 128, kch = K / 64;
+      if (tail_on && tiles > plan_sms) {
+        const int full = (tiles / plan_sms) * plan_sms, rem = tiles - full;
+        int tail = rem ? std::min({8, kch, plan_sms / rem}) : 1;
+        if (tail >= 2) {
+          const int cps = (kch + tail - 1) / tail;
+          tail = (kch + cps - 1) / cps;  // every split gets some K
+          const int ld = rem * 128;
+          c->part_tail_elems = std::max(c->part_tail_elems, (size_t)(tail - 1) * rcap * ld);
+          return SplitPlan{full * 128, tail, rcap * (size_t)N, nullptr, rcap * (size_t)ld, ld};
+        }
+      }
+      return uniform_splits(split, rcap * (size_t)N);
+    };
+    c->sp_qkv = plan(3 * (int)Hd, (int)Hd, c->split_qkv);
+    c->sp_o = plan((int)Hd, (int)Hd, c->split_o);
+    c->sp_gu = plan(2 * (int)F, (int)Hd, c->split_gu);
+    c->sp_d = plan((int)Hd, (int)F, c->split_d);
+  }
+
   // ---- workspace ----
   const size_t rc_ = c->rows_cap, Bm = d.max_batch;
   // every GEMM writes splits x rows_cap x N fp32 partials into `part`
@@ -378,6 +414,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->X, rc_ * Hd * 4, base);
     sc.take(c->Xd, Bm * Hd * 4, base);
     sc.take(c->part, rc_ * part_n * 4, base);
+    sc.take(c->part_tail, std::max(c->part_tail_elems, (size_t)4) * 4, base);
     sc.take(c->A, rc_ * Hd * E, base);
     sc.take(c->Q, rc_ * Hd * E, base);
     sc.take(c->AO, rc_ * Hd * E, base);
@@ -575,16 +612,19 @@ void dgemv(vlac_ctx* c, const DGemv& a_in, int epi, int nb, cudaStream_t st) {
 
 template <typename T>
 void gemm(vlac_ctx* c, const ActMaps* tmA, const CUtensorMap* tmW, const T* A, const void* W, const int* m_ptr,
-          int N, int K, int splits, cudaStream_t st) {
-  const int kch = c->bf16 ? K / 64 : 1, cps = (kch + splits - 1) / splits;
-  if ((size_t)splits * c->rows_cap * N > c->part_elems ||  // never launch a GEMM whose partials do not fit,
-      (splits - 1) * cps >= kch) {                          // or one with a split that has no K range
+          int N, int K, const SplitPlan& sp, cudaStream_t st) {
+  const int kch = c->bf16 ? K / 64 : 1, cps = (kch + sp.tail - 1) / sp.tail;
+  const bool compact = sp.tail_ld != 0;
+  const size_t slots = compact ? 1 : (size_t)sp.tail;
+  if (slots * c->rows_cap * N > c->part_elems ||  // never launch a GEMM whose partials do not fit,
+      (compact && (size_t)(sp.tail - 1) * c->rows_cap * sp.tail_ld > c->part_tail_elems) ||
+      (sp.tail - 1) * cps >= kch || (!c->bf16 && (sp.tail != 1 || sp.full_cols))) {  // or a split without K
     c->fatal = true;
     return;
   }
   ProfScope ps(c, VLAC_PROF_PREFIX_GEMM, (double)N * K * sizeof(T), st);
   if constexpr (sizeof(T) == 2) {
-    launch_gemm_tc(tmA, tmW, m_ptr, c->rows_cap, N, K, splits, c->part, c->err, c->wait_limit, st);
+    launch_gemm_tc(tmA, tmW, m_ptr, c->rows_cap, N, K, sp, c->part, c->err, c->wait_limit, st);
   } else {
     launch_gemm_simt<T>(A, static_cast<const T*>(W), m_ptr, c->rows_cap, N, K, c->part, st);
   }
@@ -637,7 +677,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
     ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
     launch_im2col<T>(r0, B, S, frames, d.n_views, d.img_h, d.img_w, d.patch, c->kpad, col, st);
   }
-  gemm<T>(c, &c->tm_col, &c->tm_patch, col, c->patch_w, m0, Hd, c->kpad, 1, st);
+  gemm<T>(c, &c->tm_col, &c->tm_patch, col, c->patch_w, m0, Hd, c->kpad, uniform_splits(1, c->rows_cap * Hd), st);
   {
     ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
     launch_embed<T>(r0, B, S, Hd, c->Nv, c->P, c->has_p, d.proprio_dim, d.n_text, d.vocab, prompt, proprio,
@@ -645,7 +685,11 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   }
   c->launches += 2;
 
-  const size_t rs = (size_t)c->rows_cap;
+  auto with_tail = [&](SplitPlan p) {
+    p.tail_p = c->part_tail;
+    return p;
+  };
+  const SplitPlan sq = with_tail(c->sp_qkv), so = with_tail(c->sp_o), sg = with_tail(c->sp_gu), sd = with_tail(c->sp_d);
   for (int l = 0; l < L; ++l) {
     Rows rl{c->off + (size_t)l * (B + 1), c->idx, S, c->X};
     const int* ml = rl.off + B;
@@ -655,10 +699,10 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
       launch_layer_in<T>(rl, off_prev, B, S, Hd, l == 0 ? nullptr : k->H + (size_t)l * S * Hd, k->h_seq_stride,
                          W(c->attn_norm[l]), eps, A, st);
     }
-    gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_qkv[l] : nullptr, A, c->wqkv[l], ml, 3 * Hd, Hd, c->split_qkv, st);
+    gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_qkv[l] : nullptr, A, c->wqkv[l], ml, 3 * Hd, Hd, sq, st);
     {
       ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_qkv_epilogue<T>(rl, B, S, nh, hd, c->part, c->split_qkv, rs * 3 * Hd, c->rope_cos, c->rope_sin, Q,
+      launch_qkv_epilogue<T>(rl, B, S, nh, hd, c->part, sq, c->rope_cos, c->rope_sin, Q,
                              Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, st);
     }
     {
@@ -666,20 +710,20 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
       launch_attention<T>(rl, B, S, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, c->P,
                           d.parallel, D, AO, st);
     }
-    gemm<T>(c, &c->tm_AO, c->bf16 ? &c->tm_o[l] : nullptr, AO, c->wo[l], ml, Hd, Hd, c->split_o, st);
+    gemm<T>(c, &c->tm_AO, c->bf16 ? &c->tm_o[l] : nullptr, AO, c->wo[l], ml, Hd, Hd, so, st);
     {
       ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_residual_norm<T>(rl, B, S, Hd, c->part, c->split_o, rs * Hd, W(c->ffn_norm[l]), eps, A, st);
+      launch_residual_norm<T>(rl, B, S, Hd, c->part, so, W(c->ffn_norm[l]), eps, A, st);
     }
-    gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_gu[l] : nullptr, A, c->wgu[l], ml, 2 * F, Hd, c->split_gu, st);
+    gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_gu[l] : nullptr, A, c->wgu[l], ml, 2 * F, Hd, sg, st);
     {
       ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_swiglu<T>(rl, B, S, F, c->part, c->split_gu, rs * 2 * F, G, st);
+      launch_swiglu<T>(rl, B, S, F, c->part, sg, G, st);
     }
-    gemm<T>(c, &c->tm_G, c->bf16 ? &c->tm_d[l] : nullptr, G, c->wd[l], ml, Hd, F, c->split_d, st);
+    gemm<T>(c, &c->tm_G, c->bf16 ? &c->tm_d[l] : nullptr, G, c->wd[l], ml, Hd, F, sd, st);
     {
       ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_residual(rl, B, S, Hd, c->part, c->split_d, rs * Hd, st);
+      launch_residual(rl, B, S, Hd, c->part, sd, st);
     }
     c->launches += 6;
   }
