@@ -435,6 +435,19 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
     // q/k/v: RMSNorm of the residual rows (sums of squares from the decode
     // embedding for layer 0, else from the previous down-projection)
     if (l > 0) grid_sync(a, ++epoch, abort);
+    if (threadIdx.x == 0) {
+      // this CTA's attention items: their older K/V rows (written by earlier
+      // passes) start on their way into L2 while the q/k/v projection runs
+      for (int item = blockIdx.x; item < NB * a.n_heads; item += gridDim.x) {
+        const int b = item / a.n_heads, h = item - b * a.n_heads;
+        const size_t off = (size_t)l * a.kv_layer + (size_t)b * a.kv_seq_stride + (size_t)h * a.Tc * kPHD;
+        const uint32_t bytes = (uint32_t)(min(a.pos, a.Tc) * kPHD * 2);
+        if (bytes >= 16) {
+          prefetch_l2(a.Kc + off, bytes & ~15u);
+          prefetch_l2(a.Vc + off, bytes & ~15u);
+        }
+      }
+    }
     {
       const Proj P = proj_of(a, l, 0);
       prologue_norm<NB>(a, l == 0 ? a.ssq0 : a.ssq, l == 0 ? a.n_ssq0 : (int)gridDim.x, a.g_attn[l], P.K, xs, red, rr);
