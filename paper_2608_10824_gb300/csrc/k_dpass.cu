@@ -400,30 +400,52 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
   if (warp == kPC) {
     // ---- producer: every projection of every layer, in consumption order ----
     if (lane == 0) {
-      for (int l = 0; l < a.L; ++l)
-        for (int j = 0; j < 4; ++j) {
+      uint32_t issued = 0;
+      bool dead = false;
+      for (int l = 0; l < a.L && !dead; ++l)
+        for (int j = 0; j < 4 && !dead; ++j) {
           const Proj P = proj_of(a, l, j);
           const int G = (P.n_pairs + kDecGroupPairs - 1) / kDecGroupPairs, nchunk = (P.K + kPKC - 1) / kPKC;
           int g0, g1;
           dgemv_group_range(G, gridDim.x, blockIdx.x, g0, g1);
-          for (int g = g0; g < g1; ++g)
+          for (int g = g0; g < g1 && !dead; ++g)
             for (int c = 0; c < nchunk; ++c) {
               const int kn = min(kPKC, P.K - c * kPKC);
               if (!mbar_wait(&R.empty[R.stage], R.phase ^ 1u, kWaitLimit, ring_dead)) {
+                // the consumers stopped releasing stages: nothing more is issued
                 set_error(a.err, VLAC_ERR_TIMEOUT);
                 *ring_dead = 1;
-                return;  // the consumers stopped releasing stages: nothing more is issued
+                dead = true;
+                break;
               }
               const uint32_t bytes = (uint32_t)(kPTR * kn * 2);
               mbar_expect_tx(&R.full[R.stage], bytes);
               bulk_g2s(R.stages + (size_t)R.stage * kPStage, P.W + (size_t)g * kPTR * P.K + (size_t)kPTR * c * kPKC,
                        bytes, &R.full[R.stage]);
+              ++issued;
               if (++R.stage == R.ns) {
                 R.stage = 0;
                 R.phase ^= 1u;
               }
             }
         }
+      // No bulk copy may still be landing in this CTA's shared memory when it
+      // exits.  The last min(issued, ns) copies went to the stages just
+      // before R.stage; each has landed once its full barrier completed the
+      // phase it was issued in.  On the normal path the consumers waited for
+      // all of them already; after a give-up this wait (bounded, and deaf to
+      // the give-up flags) is the one that holds the CTA until they land.
+      const int n_last = (int)min(issued, (uint32_t)R.ns);
+      for (int q = 0; q < n_last; ++q) {
+        int s = R.stage - 1 - q;
+        uint32_t ph = R.phase;
+        if (s < 0) {
+          s += R.ns;
+          ph ^= 1u;
+        }
+        for (uint32_t it = 0; it < kWaitLimit && !mbar_test(&R.full[s], ph); ++it) {
+        }
+      }
     }
     return;
   }

@@ -768,12 +768,19 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
           p.ssq = c->ssq_a;
           p.bar = c->dp_bar;
           p.err = c->err;
+          int rc_dp;
           {
             ProfScope ps_(c, VLAC_PROF_DECODE_GEMV, (double)L * (4.0 * Hd * Hd + 3.0 * F * Hd) * 2, st);
-            if (launch_dpass(p, B, c->n_sm, st) != VLAC_OK) c->fatal = true;
+            rc_dp = launch_dpass(p, B, c->n_sm, st);
           }
-          c->launches += 1;
-          dp_done = true;
+          if (rc_dp == VLAC_OK) {
+            c->launches += 1;
+            dp_done = true;
+          } else if (rc_dp == VLAC_ERR_UNSUPPORTED) {
+            (void)cudaGetLastError();  // one CTA per SM does not fit: the per-projection chain runs instead
+          } else {
+            c->fatal = true;
+          }
         }
       }
       for (int l = 0; l < L && !dp_done; ++l) {
