@@ -198,10 +198,9 @@ __device__ float consume(const DPass& a, int l, const Proj& P, int g0, int g1, c
     for (int c = 0; c < nchunk; ++c) {
       const int k0 = c * kPKC, n32 = min(kPKC, K - k0) >> 5;
       const int i0 = n32 * warp / kPC, i1 = n32 * (warp + 1) / kPC;
-      // ring waits ignore the grid barrier's give-up flag, so that every bulk
-      // copy in flight is waited for before its stage is handed back (and
-      // before the CTA exits); once one ring wait times out the ring is dead
-      // and the others return at once
+      // ring waits ignore the grid barrier's give-up flag: a stage is handed
+      // back only after its copy landed; once one ring wait times out the
+      // ring is dead and the others return at once
       bool ok = true;
       if (lane == 0) ok = mbar_wait(&R.full[R.stage], R.phase, kWaitLimit, ring_dead);
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -230,14 +229,14 @@ __device__ float consume(const DPass& a, int l, const Proj& P, int g0, int g1, c
           mma_bf16(d[0], xv.x, 0u, xv.y, 0u, b0, b1);
           mma_bf16(d[0], xv.z, 0u, xv.w, 0u, b2, b3);
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&R.empty[R.stage]);
       } else if (lane == 0) {
+        // a stage whose wait failed is not handed back, so it is never
+        // refilled; the producer sees the flag and stops
         set_error(a.err, VLAC_ERR_TIMEOUT);
         *ring_dead = 1;
       }
-      // the stage is released either way, so that the producer never waits
-      // on a consumer that gave up
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&R.empty[R.stage]);
       if (++R.stage == R.ns) {
         R.stage = 0;
         R.phase ^= 1u;
@@ -429,23 +428,9 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
               }
             }
         }
-      // No bulk copy may still be landing in this CTA's shared memory when it
-      // exits.  The last min(issued, ns) copies went to the stages just
-      // before R.stage; each has landed once its full barrier completed the
-      // phase it was issued in.  On the normal path the consumers waited for
-      // all of them already; after a give-up this wait (bounded, and deaf to
-      // the give-up flags) is the one that holds the CTA until they land.
-      const int n_last = (int)min(issued, (uint32_t)R.ns);
-      for (int q = 0; q < n_last; ++q) {
-        int s = R.stage - 1 - q;
-        uint32_t ph = R.phase;
-        if (s < 0) {
-          s += R.ns;
-          ph ^= 1u;
-        }
-        for (uint32_t it = 0; it < kWaitLimit && !mbar_test(&R.full[s], ph); ++it) {
-        }
-      }
+      // no bulk copy may still be landing in this CTA's shared memory when it
+      // exits; on the normal path the consumers waited for every one already
+      ring_drain(R.full, R.ns, R.stage, R.phase, issued);
     }
     return;
   }
