@@ -360,6 +360,14 @@ struct DPass {
   float* ssq;
   unsigned* bar;
   int* err;
+  // attention: each (sequence, head) cut into attn_chunks key ranges; with
+  // more than one, every range's partial (max, sum, unnormalised output) goes
+  // to attn_part + (b * n_heads + h) * part_stride + chunk * (head_dim + 2) and
+  // the last range to finish (counted in attn_cnt, zero between uses) combines
+  int attn_chunks;
+  size_t part_stride;
+  float* attn_part;
+  unsigned* attn_cnt;
 };
 bool dpass_supported(int hidden, int ffn, int n_heads, int head_dim, int nb, int ns);
 int launch_dpass(const DPass& a, int nb, int n_sm, cudaStream_t st);

@@ -296,22 +296,28 @@ __device__ void write_ssq(const DPass& a, float ssq, float (*red)[32]) {
   consumers_sync();
 }
 
-// Single-query attention of layer l for (sequence, head) items spread over the
-// CTAs: warp w takes keys w*32 + 256t + lane (online softmax per warp), the
-// eight warps are combined in order.
+// Single-query attention of layer l: items (sequence, head, key range) spread
+// over the CTAs.  Warp w takes keys k0 + w*32 + 256t + lane of the item's range
+// (online softmax per warp) and the eight warps are combined in order.  With
+// one range per head the CTA writes the output row; with several, it writes
+// its range's partial and the last range to finish combines the ranges in
+// order (no CTA waits for another).
 template <int NB>
-__device__ void attention(const DPass& a, int l, float* qs, float* wm, float* wl, float (*wacc)[kPHD]) {
+__device__ void attention(const DPass& a, int l, float* qs, float* wm, float* wl, float (*wacc)[kPHD],
+                          volatile int* s_last) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int hidden = a.hidden, nkeys = min(a.pos + 1, a.Tc);
-  for (int item = blockIdx.x; item < NB * a.n_heads; item += gridDim.x) {
-    const int b = item / a.n_heads, h = item - b * a.n_heads;
+  const int hidden = a.hidden, nkeys = min(a.pos + 1, a.Tc), nch = a.attn_chunks;
+  for (int item = blockIdx.x; item < NB * a.n_heads * nch; item += gridDim.x) {
+    const int bh = item / nch, ch = item - bh * nch;
+    const int b = bh / a.n_heads, h = bh - b * a.n_heads;
+    const int k0 = (int)(((long long)nkeys * ch) / nch), k1 = (int)(((long long)nkeys * (ch + 1)) / nch);
     const bf16* Kh = a.Kc + (size_t)l * a.kv_layer + (size_t)b * a.kv_seq_stride + (size_t)h * a.Tc * kPHD;
     const bf16* Vh = a.Vc + (size_t)l * a.kv_layer + (size_t)b * a.kv_seq_stride + (size_t)h * a.Tc * kPHD;
     if (tid < kPHD) qs[tid] = __bfloat162float(__ldcg(a.Q + (size_t)b * hidden + (size_t)h * kPHD + tid));
     consumers_sync();
     float m_run = -INFINITY, l_run = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
-    for (int j0 = warp * 32; j0 < nkeys; j0 += kPC * 32) {
-      const int jn = min(32, nkeys - j0), j = j0 + lane;
+    for (int j0 = k0 + warp * 32; j0 < k1; j0 += kPC * 32) {
+      const int jn = min(32, k1 - j0), j = j0 + lane;
       float s = -INFINITY;
       if (lane < jn) {
         const uint4* kr = reinterpret_cast<const uint4*>(Kh + (size_t)j * kPHD);
@@ -352,16 +358,48 @@ __device__ void attention(const DPass& a, int l, float* qs, float* wm, float* wl
 #pragma unroll
     for (int e = 0; e < 4; ++e) wacc[warp][lane * 4 + e] = acc[e];
     consumers_sync();
+    // this item's (max, sum, unnormalised output), warps in order
+    float M = -INFINITY, L = 0.f, o = 0.f;
     if (tid < kPHD) {
-      float M = -INFINITY;
       for (int w = 0; w < kPC; ++w) M = fmaxf(M, wm[w]);
-      float L = 0.f, o = 0.f;
       for (int w = 0; w < kPC; ++w) {
         const float f = wm[w] == -INFINITY ? 0.f : expf(wm[w] - M);
         L = fmaf(wl[w], f, L);
         o = fmaf(wacc[w][tid], f, o);
       }
-      a.AO[(size_t)b * hidden + (size_t)h * kPHD + tid] = __float2bfloat16_rn(o / L);
+    }
+    if (nch == 1) {
+      if (tid < kPHD) a.AO[(size_t)b * hidden + (size_t)h * kPHD + tid] = __float2bfloat16_rn(o / L);
+      consumers_sync();
+      continue;
+    }
+    float* part = a.attn_part + (size_t)bh * a.part_stride;
+    if (tid < kPHD) {
+      part[(size_t)ch * (kPHD + 2) + 2 + tid] = o;
+      if (tid == 0) {
+        part[(size_t)ch * (kPHD + 2)] = M;
+        part[(size_t)ch * (kPHD + 2) + 1] = L;
+      }
+    }
+    __threadfence();
+    consumers_sync();
+    if (tid == 0) *s_last = atomicAdd(a.attn_cnt + bh, 1u) == (unsigned)(nch - 1);
+    consumers_sync();
+    if (*s_last) {
+      __threadfence();
+      if (tid < kPHD) {
+        float Mx = -INFINITY;
+        for (int c = 0; c < nch; ++c) Mx = fmaxf(Mx, __ldcg(part + (size_t)c * (kPHD + 2)));
+        float Lt = 0.f, ot = 0.f;
+        for (int c = 0; c < nch; ++c) {
+          const float mc = __ldcg(part + (size_t)c * (kPHD + 2));
+          const float f = mc == -INFINITY ? 0.f : expf(mc - Mx);
+          Lt = fmaf(__ldcg(part + (size_t)c * (kPHD + 2) + 1), f, Lt);
+          ot = fmaf(__ldcg(part + (size_t)c * (kPHD + 2) + 2 + tid), f, ot);
+        }
+        a.AO[(size_t)b * hidden + (size_t)h * kPHD + tid] = __float2bfloat16_rn(ot / Lt);
+      }
+      if (tid == 0) a.attn_cnt[bh] = 0u;  // ready for the next layer (after the grid barriers)
     }
     consumers_sync();
   }
@@ -377,7 +415,7 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
   __shared__ __align__(8) float2 pacc[2][kPC][32];
   __shared__ float qs[kPHD], wm[kPC], wl[kPC];
   __shared__ float wacc[kPC][kPHD];
-  __shared__ int abort_flag, ring_flag;
+  __shared__ int abort_flag, ring_flag, last_flag;
   uint8_t* dsm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int xs_bytes = ((NB * max(a.hidden, a.ffn) * 2 + 1023) / 1024) * 1024;
@@ -462,7 +500,7 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
       consume<NB, 0>(a, l, P, g0, g1, xs, R, pacc, ring_dead);
     }
     grid_sync(a, ++epoch, abort);
-    attention<NB>(a, l, qs, wm, wl, wacc);
+    attention<NB>(a, l, qs, wm, wl, wacc, &last_flag);
     grid_sync(a, ++epoch, abort);
     {  // o-projection + residual
       const Proj P = proj_of(a, l, 1);
@@ -501,6 +539,8 @@ int dpass_launch(const DPass& a, int n_sm, cudaStream_t st) {
       per_sm < 1)
     return VLAC_ERR_UNSUPPORTED;
   if (cudaMemsetAsync(a.bar, 0, sizeof(unsigned), st) != cudaSuccess) return VLAC_ERR_CUDA;
+  if (a.attn_chunks > 1 && cudaMemsetAsync(a.attn_cnt, 0, (size_t)NB * a.n_heads * sizeof(unsigned), st) != cudaSuccess)
+    return VLAC_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(n_sm);
   cfg.blockDim = dim3((kPC + 1) * 32);

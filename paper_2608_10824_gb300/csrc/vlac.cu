@@ -49,6 +49,7 @@ struct vlac_ctx {
   int gemv_ns = 4;  // decode-GEMV weight ring stages (32 KB each)
   int gemv_pf_kb = 0;  // decode-GEMV L2 prefetch of the next projection, KB per CTA (measured: off is best)
   bool use_dpass = false;  // decode passes as one persistent cooperative launch (k_dpass.cu) where supported
+  int dpass_attn_chunks = 0;  // its key ranges per (sequence, head); 0 = chosen from the SM count
   void** dp_ptrs = nullptr;  // device: per-layer pointers [w_qkv | w_o | w_gu | w_d | g_attn | g_ffn][L]
   unsigned* dp_bar = nullptr;  // device: the persistent pass's grid-barrier counter
   char* dmem = nullptr;  // decode-streaming copies of the projections
@@ -210,6 +211,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (const char* e = std::getenv("VLAC_GEMV_NS")) c->gemv_ns = std::max(2, std::min(24, std::atoi(e)));
   if (const char* e = std::getenv("VLAC_GEMV_PF_KB")) c->gemv_pf_kb = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("VLAC_DPASS")) c->use_dpass = std::atoi(e) != 0;
+  if (const char* e = std::getenv("VLAC_DPASS_ATTN_CHUNKS")) c->dpass_attn_chunks = std::max(0, std::atoi(e));
   c->d = *dims;
   const vlac_dims& d = c->d;
   c->bf16 = d.dtype == VLAC_BF16;
@@ -768,6 +770,17 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
           p.ssq = c->ssq_a;
           p.bar = c->dp_bar;
           p.err = c->err;
+          {
+            // key ranges per (sequence, head): enough items for the SMs, at
+            // most one per 32 keys (the partial buffer's capacity) and 8
+            const int cap = std::min(8, (c->Tc + 31) / 32);
+            int chunks = std::max(1, std::min(cap, c->n_sm / std::max(1, B * nh)));
+            if (c->dpass_attn_chunks > 0) chunks = std::min(cap, c->dpass_attn_chunks);
+            p.attn_chunks = chunks;
+            p.part_stride = (size_t)((c->Tc + 31) / 32) * (hd + 2);
+            p.attn_part = c->attn_part;
+            p.attn_cnt = c->attn_cnt;
+          }
           int rc_dp;
           {
             ProfScope ps_(c, VLAC_PROF_DECODE_GEMV, (double)L * (4.0 * Hd * Hd + 3.0 * F * Hd) * 2, st);

@@ -23,8 +23,13 @@ def dpass_on():
         os.environ["VLAC_DPASS"] = old
 
 
+@pytest.mark.parametrize("chunks", ["auto", "1", "3"])
 @pytest.mark.parametrize("name,batch", [("small", 1), ("small_wide", 1), ("small_wide", 2)])
-def test_dpass_parity(name, batch, dpass_on, cuda_device):
+def test_dpass_parity(name, batch, chunks, dpass_on, cuda_device, monkeypatch):
+    """chunks: key ranges per (sequence, head) in the attention phase (1: one
+    CTA per head; otherwise the ranges' partials are combined by the last)."""
+    if chunks != "auto":
+        monkeypatch.setenv("VLAC_DPASS_ATTN_CHUNKS", chunks)
     d = SMALL[name]
     w = synth.make_weights(d, seed=21)
     ls = Lockstep(d, w, batch=batch)
