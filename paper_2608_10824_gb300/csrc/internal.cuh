@@ -90,6 +90,31 @@ struct DGemv {
 };
 constexpr int kDecodeRowsPerCta = 4;  // residual rows per decode-GEMV CTA (2 row pairs)
 
+// Tiled decode weights (built at create, streamed by the decode GEMV and the
+// persistent decode pass): groups of kDecGroupPairs output row pairs, K cut
+// into chunks of kDecTileBytes per row, bf16 tiles interleaved in 8-element K
+// steps ([k/8][row][k%8]).
+constexpr int kDecGroupPairs = 4;
+constexpr int kDecTileBytes = 4096;
+
+// Groups [g0, g1) of CTA b when G groups are cut over n CTAs: the first
+// G mod n CTAs take one group more.  CTAs are placed on SMs in index order as
+// the previous kernel's CTAs leave, so the low indices start first and fill
+// their weight ring earliest; they are the ones given the extra group.
+__host__ __device__ inline void dgemv_group_range(int G, int n, int b, int& g0, int& g1) {
+  const int q = G / n, r = G - q * n;
+  g0 = b * q + (b < r ? b : r);
+  g1 = g0 + q + (b < r ? 1 : 0);
+}
+
+// Position (in elements, within its row) of element k of a bf16 input vector
+// in the A-fragment order of mma.m16n8k16: per 32-element K step and lane t
+// the elements 2t, 2t+1, 2t+8, 2t+9, 2t+16, 2t+17, 2t+24, 2t+25.
+__device__ __forceinline__ int afrag_pos(int k) {
+  const int i = k >> 5, w = k & 31, s = w >> 3, t = (w & 7) >> 1;
+  return ((i * 4 + t) * 8) + s * 2 + (w & 1);
+}
+
 // ---- scalar helpers --------------------------------------------------------
 template <typename T> __device__ __forceinline__ float to_f(T v);
 template <> __device__ __forceinline__ float to_f<float>(float v) { return v; }
@@ -323,6 +348,46 @@ int launch_wait_selftest(int* err, uint32_t spin_limit, cudaStream_t st);
 template <typename T>
 void launch_dgemv(const DGemv& a, int epi, int nb, int n_sm, cudaStream_t st);
 int dgemv_grid(int n_pairs, int n_sm);  // CTAs (and sum-of-squares partials) of one decode GEMV
+
+// Persistent decode pass (k_dpass.cu): all layers of one decode token in one
+// cooperative launch, one CTA per SM.  Per-layer arrays are device arrays of L
+// pointers (tiled decode weights, RMSNorm gains); K/V of layer l at
+// Kc/Vc + l * kv_layer.  `ssq0` holds the decode embedding's sums of squares
+// ([nb][n_ssq0]); `ssq` ([nb][grid]) and `bar` (zeroed by the launcher) are
+// the launch's own workspace.
+struct DPass {
+  const bf16* const* w_qkv;
+  const bf16* const* w_o;
+  const bf16* const* w_gu;
+  const bf16* const* w_d;
+  const bf16* const* g_attn;
+  const bf16* const* g_ffn;
+  int L, hidden, ffn, n_heads, Tc, pos, ns, n_ssq0;
+  float eps, scale;
+  const float* rope_cos;
+  const float* rope_sin;
+  float* X;
+  bf16* Q;
+  bf16* AO;
+  bf16* G;
+  bf16* Kc;
+  bf16* Vc;
+  size_t kv_layer, kv_seq_stride;
+  const float* ssq0;
+  float* ssq;
+  unsigned* bar;
+  int* err;
+  // attention: each (sequence, head) cut into attn_chunks key ranges; with
+  // more than one, every range's partial (max, sum, unnormalised output) goes
+  // to attn_part + (b * n_heads + h) * part_stride + chunk * (head_dim + 2) and
+  // the last range to finish (counted in attn_cnt, zero between uses) combines
+  int attn_chunks;
+  size_t part_stride;
+  float* attn_part;
+  unsigned* attn_cnt;
+};
+bool dpass_supported(int hidden, int ffn, int n_heads, int head_dim, int nb, int ns);
+int launch_dpass(const DPass& a, int nb, int n_sm, cudaStream_t st);
 // Decode-streaming copy of a projection (W: [rows][K]); see k_decode.cu for the layout.
 template <typename T>
 void launch_tile_decode_weights(const T* W, int K, int n_pairs, int epi, int n_heads, int head_dim, int ffn, T* out,

@@ -133,30 +133,14 @@ __device__ __forceinline__ void norm_rows_to_smem(const float* __restrict__ X, c
 // landing before the CTA exits.
 
 constexpr int kNC = 8;          // consumer warps
-constexpr int kGP = 4;          // row pairs per group
-constexpr int kMaxNS = 24;      // stage ring capacity
-constexpr int kDecTileB = 4096; // bytes of one tile row (K chunk)
-
-// Groups [g0, g1) of CTA b when G groups are cut over n CTAs: the first
-// G mod n CTAs take one group more.  CTAs are placed on SMs in index order as
-// the previous kernel's CTAs leave, so the low indices start first and fill
-// their weight ring earliest; they are the ones given the extra group.
-__host__ __device__ inline void dgemv_group_range(int G, int n, int b, int& g0, int& g1) {
-  const int q = G / n, r = G - q * n;
-  g0 = b * q + min(b, r);
-  g1 = g0 + q + (b < r ? 1 : 0);
-}
+constexpr int kGP = kDecGroupPairs;      // row pairs per group
+constexpr int kMaxNS = 24;               // stage ring capacity
+constexpr int kDecTileB = kDecTileBytes; // bytes of one tile row (K chunk)
 
 __host__ __device__ inline size_t sgemv_xs_bytes(int nb, int K, int esz) {
   return ((size_t)nb * K * esz + 1023) / 1024 * 1024;
 }
 
-// position (in elements, within its row) of element k of a bf16 input vector
-// in A-fragment order
-__device__ __forceinline__ int afrag_pos(int k) {
-  const int i = k >> 5, w = k & 31, s = w >> 3, t = (w & 7) >> 1;
-  return ((i * 4 + t) * 8) + s * 2 + (w & 1);
-}
 
 template <int EPI>
 __host__ __device__ __forceinline__ void dec_pair_rows(int p, int n_heads, int head_dim, int ffn, int& r1, int& r2) {

@@ -48,6 +48,10 @@ struct vlac_ctx {
   int n_sm = 1;
   int gemv_ns = 4;  // decode-GEMV weight ring stages (32 KB each)
   int gemv_pf_kb = 0;  // decode-GEMV L2 prefetch of the next projection, KB per CTA (measured: off is best)
+  bool use_dpass = false;  // decode passes as one persistent cooperative launch (k_dpass.cu) where supported
+  int dpass_attn_chunks = 0;  // its key ranges per (sequence, head); 0 = chosen from the SM count
+  void** dp_ptrs = nullptr;  // device: per-layer pointers [w_qkv | w_o | w_gu | w_d | g_attn | g_ffn][L]
+  unsigned* dp_bar = nullptr;  // device: the persistent pass's grid-barrier counter
   char* dmem = nullptr;  // decode-streaming copies of the projections
   std::vector<void*> dqkv, dwo, dgu, dwd;
   // weights
@@ -211,6 +215,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (const char* e = std::getenv("VLAC_GRAPH")) c->use_graph = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_GEMV_NS")) c->gemv_ns = std::max(2, std::min(24, std::atoi(e)));
   if (const char* e = std::getenv("VLAC_GEMV_PF_KB")) c->gemv_pf_kb = std::max(0, std::atoi(e));
+  if (const char* e = std::getenv("VLAC_DPASS")) c->use_dpass = std::atoi(e) != 0;
+  if (const char* e = std::getenv("VLAC_DPASS_ATTN_CHUNKS")) c->dpass_attn_chunks = std::max(0, std::atoi(e));
   c->d = *dims;
   const vlac_dims& d = c->d;
   c->bf16 = d.dtype == VLAC_BF16;
@@ -436,6 +442,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->attn_cnt, Bm * d.n_heads * sizeof(unsigned), base);
     sc.take(c->ssq_a, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
     sc.take(c->ssq_b, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
+    sc.take(c->dp_ptrs, 6 * L * sizeof(void*), base);
+    sc.take(c->dp_bar, sizeof(unsigned), base);
     const size_t fbytes = (size_t)d.n_views * d.img_h * d.img_w * 3;
     sc.take(c->in_frames, Bm * fbytes, base);
     sc.take(c->in_prompt, Bm * d.n_text * 4, base);
@@ -464,6 +472,19 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     std::vector<int> od(Bm + 1);
     for (size_t b = 0; b <= Bm; ++b) od[b] = (int)b;
     if (cudaMemcpy(c->off_dec, od.data(), od.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(VLAC_ERR_CUDA);
+  }
+  if (c->bf16 && !c->dqkv.empty()) {  // per-layer pointers of the persistent decode pass
+    std::vector<void*> pp(6 * L);
+    for (size_t l = 0; l < L; ++l) {
+      pp[l] = c->dqkv[l];
+      pp[L + l] = c->dwo[l];
+      pp[2 * L + l] = c->dgu[l];
+      pp[3 * L + l] = c->dwd[l];
+      pp[4 * L + l] = c->attn_norm[l];
+      pp[5 * L + l] = c->ffn_norm[l];
+    }
+    if (cudaMemcpy(c->dp_ptrs, pp.data(), pp.size() * sizeof(void*), cudaMemcpyHostToDevice) != cudaSuccess)
       return fail(VLAC_ERR_CUDA);
   }
   if (cudaMallocHost(&c->err_host, sizeof(int)) != cudaSuccess) {
@@ -756,7 +777,70 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         g.pf_bytes = (uint32_t)c->gemv_pf_kb * 1024;
         if (!g.pf_bytes) g.pf_W = nullptr;
       };
-      for (int l = 0; l < L; ++l) {
+      // all layers as one persistent cooperative launch (VLAC_DPASS=1, bf16,
+      // head_dim 128, up to two sequences); else one launch per projection
+      bool dp_done = false;
+      if constexpr (sizeof(T) == 2) {
+        if (c->use_dpass && dpass_supported((int)Hd, (int)F, nh, hd, B, c->gemv_ns)) {
+          DPass p{};
+          const bf16* const* pp = reinterpret_cast<const bf16* const*>(c->dp_ptrs);
+          p.w_qkv = pp;
+          p.w_o = pp + L;
+          p.w_gu = pp + 2 * L;
+          p.w_d = pp + 3 * L;
+          p.g_attn = pp + 4 * L;
+          p.g_ffn = pp + 5 * L;
+          p.L = L;
+          p.hidden = (int)Hd;
+          p.ffn = (int)F;
+          p.n_heads = nh;
+          p.Tc = c->Tc;
+          p.pos = pos;
+          p.ns = c->gemv_ns;
+          p.n_ssq0 = (int)Hd / kDecodeRowsPerCta;
+          p.eps = eps;
+          p.scale = 1.0f / sqrtf((float)hd);
+          p.rope_cos = c->rope_cos;
+          p.rope_sin = c->rope_sin;
+          p.X = c->Xd;
+          p.Q = Q;
+          p.AO = AO;
+          p.G = G;
+          p.Kc = Kc;
+          p.Vc = Vc;
+          p.kv_layer = kv_layer;
+          p.kv_seq_stride = k->kv_seq_stride;
+          p.ssq0 = c->ssq_b;
+          p.ssq = c->ssq_a;
+          p.bar = c->dp_bar;
+          p.err = c->err;
+          {
+            // key ranges per (sequence, head): enough items for the SMs, at
+            // most one per 32 keys (the partial buffer's capacity) and 8
+            const int cap = std::min(8, (c->Tc + 31) / 32);
+            int chunks = std::max(1, std::min(cap, c->n_sm / std::max(1, B * nh)));
+            if (c->dpass_attn_chunks > 0) chunks = std::min(cap, c->dpass_attn_chunks);
+            p.attn_chunks = chunks;
+            p.part_stride = (size_t)((c->Tc + 31) / 32) * (hd + 2);
+            p.attn_part = c->attn_part;
+            p.attn_cnt = c->attn_cnt;
+          }
+          int rc_dp;
+          {
+            ProfScope ps_(c, VLAC_PROF_DECODE_GEMV, (double)L * (4.0 * Hd * Hd + 3.0 * F * Hd) * 2, st);
+            rc_dp = launch_dpass(p, B, c->n_sm, st);
+          }
+          if (rc_dp == VLAC_OK) {
+            c->launches += 1;
+            dp_done = true;
+          } else if (rc_dp == VLAC_ERR_UNSUPPORTED) {
+            (void)cudaGetLastError();  // one CTA per SM does not fit: the per-projection chain runs instead
+          } else {
+            c->fatal = true;
+          }
+        }
+      }
+      for (int l = 0; l < L && !dp_done; ++l) {
         DGemv g{};
         g.eps = eps;
         g.n_heads = nh;
