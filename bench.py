@@ -95,6 +95,67 @@ def step_work(d, M_seq, idx_seq):
     return passes
 
 
+def layer_work(d, pos):
+    """FLOPs and bytes of one decoder layer for rows at positions `pos` over
+    a cache of d.cache_len positions (the one-layer workload): the layer's
+    weights, the cache's K and V read, the rows' fresh K/V written and their
+    fp32 inputs read and outputs written."""
+    Hd, F = d.hidden, d.ffn
+    pos = np.asarray(pos, dtype=np.int64)
+    M = int(pos.size)
+    flops = M * 2 * (4 * Hd * Hd + 3 * F * Hd) + 4 * Hd * float(np.sum(pos + 1))
+    nbytes = (4 * Hd * Hd + 3 * F * Hd) * 2 + 2 * d.cache_len * Hd * 2 + M * 2 * Hd * 2 + 2 * M * Hd * 4
+    return flops, nbytes
+
+
+def run_layer_sweep(args, d):
+    """The one-layer workload: per recomputed-row count M, the device time of
+    one decoder layer (vlac_layer_bench) over a cache pre-filled with N(0, 1)
+    values, averaged over --steps calls after --warmup, against the layer's
+    roofline.  Prints one JSON line."""
+    import torch
+
+    from paper_2608_10824_gb300 import Context
+    dev = torch.device("cuda", 0)
+    w = synth.make_weights(d, seed=args.seed, device=dev, lm_head_rows=d.n_bins)
+    ctx = Context(d, w, max_batch=1)
+    del w
+    torch.cuda.empty_cache()
+    cache = ctx.new_cache(1)
+    dt = torch.bfloat16 if d.dtype == "bf16" else torch.float32
+    pk, src = peaks()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)   # 256 MB > L2, written between calls
+    results = []
+    for M in [m for m in (d.pass_len, 200, 120, 60, 30) if m <= d.pass_len]:
+        pos, x, k0, v0 = synth.make_layer_case(d, M, seed=args.seed)
+        ctx.cache_load(cache, 0, 0, torch.from_numpy(k0).to(dt).to(dev), torch.from_numpy(v0).to(dt).to(dev))
+        pos_d = torch.from_numpy(pos).to(dev)
+        x0 = torch.from_numpy(x).to(dev)
+        xb = torch.empty_like(x0)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        for i in range(args.warmup + args.steps):
+            xb.copy_(x0)
+            flush.fill_(i & 255)
+            if i >= args.warmup:
+                ev[i - args.warmup][0].record()
+            ctx.layer_bench(cache, 0, 0, pos_d, xb)
+            if i >= args.warmup:
+                ev[i - args.warmup][1].record()
+        torch.cuda.synchronize()
+        assert ctx.sync_error() == 0
+        ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+        f, b = layer_work(d, pos)
+        t_roof = max(f / (pk["bf16_tflops"] * 1e12), b / (pk["hbm_gbs"] * 1e9))
+        results.append({"M": M, "ms": ms, "roofline_ms": t_roof * 1e3, "frac": t_roof * 1e3 / ms,
+                        "tflops": f / (ms / 1e3) / 1e12, "gbs": b / (ms / 1e3) / 1e9})
+    print(json.dumps({"metric": "one decoder layer (7B shape) per recomputed-row count", "unit": "ms",
+                      "workload": f"{args.config}: 1 layer, hidden {d.hidden}, {d.n_heads}x{d.head_dim} heads, "
+                                  f"SwiGLU {d.ffn}, {d.pass_len}-position prefix pass, cache of {d.cache_len} "
+                                  f"positions pre-filled N(0, 1), seeded sorted positions, inputs N(0, 1)",
+                      "steps": args.steps, "warmup": args.warmup, "peaks": src, "l2": "256 MB written between calls",
+                      "results": results}))
+
+
 def batch_work(d, Ms, idxs):
     """(flops, bytes, per-pass [(flops, bytes)]) of one step of a batch: the
     sequences' own work adds up, the weights are read once per pass."""
@@ -260,6 +321,8 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-budget", type=float, default=25.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layer-sweep", action="store_true",
+                    help="time one decoder layer per recomputed-row count (the one-layer workload) instead")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -267,6 +330,9 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     d = synth.dims_for(args.config)
+    if args.layer_sweep:
+        run_layer_sweep(args, synth.dims_for("layer7b") if args.config == "openvla7b" else d)
+        return
     seed = replica_seed(args.seed, rank)
     B = d.max_batch
     frames = synth.make_episode(d, EPISODE, seed=seed, batch=B, kind="scene",

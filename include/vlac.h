@@ -154,6 +154,37 @@ int vlac_step(vlac_ctx* ctx, vlac_cache* cache, const uint8_t* frames, const int
  * no cache existed (Algorithm 1, cache invalidation). */
 int vlac_reset(vlac_cache* cache, int seq, void* stream);
 
+/* One decoder layer of the prefix pass on its own (the one-layer workload:
+ * gather, q/k/v + RoPE + K/V scatter, mixed-cache attention, o-projection,
+ * MLP, as vlac_step runs them for each layer).
+ *   seq, layer:  the cache sequence (< batch) and layer (< n_layers)
+ *   pos:         device int32 [M], distinct positions of the rows, each below
+ *                the prefix pass length S (n_text + visual + proprio, plus the
+ *                parallel action block); an index outside [0, S) latches
+ *                VLAC_ERR_DEVICE_CHECK in the context's error word and is
+ *                replaced by 0, so that no access leaves the cache
+ *   M:           1 .. S rows
+ *   x:           device fp32 [M][hidden]: the rows' layer inputs on entry,
+ *                their layer outputs on return
+ * The rows' K/V are written into the cache at their positions before any row
+ * attends; each row attends causally by position to that layer of the cache
+ * (rows of a parallel action block see the whole block).  Asynchronous on
+ * `stream`; the context's workspace is used, so calls on one context do not
+ * overlap.  VLAC_ERR_INVALID_ARG for NULL pointers or out-of-range seq,
+ * layer or M. */
+int vlac_layer_bench(vlac_ctx* ctx, vlac_cache* cache, int seq, int layer, const int32_t* pos, int M, float* x,
+                     void* stream);
+
+/* K and V of one layer of sequence `seq` as device arrays [T][hidden] in the
+ * model's element type (bf16 or fp32), row t the key (value) vector of
+ * position t, heads side by side; T = the cache's positions: S + n_action - 1
+ * for autoregressive decode, S for a parallel action block.
+ * vlac_cache_load copies them into the cache, vlac_cache_store out of it.
+ * Asynchronous on `stream`.  VLAC_ERR_INVALID_ARG for NULL or unaligned
+ * (4-byte) pointers or out-of-range seq or layer. */
+int vlac_cache_load(vlac_cache* cache, int seq, int layer, const void* K, const void* V, void* stream);
+int vlac_cache_store(const vlac_cache* cache, int seq, int layer, void* K, void* V, void* stream);
+
 /* Waits for the context's device work and returns (and clears) the latched
  * device error word. */
 int vlac_sync_error(vlac_ctx* ctx);

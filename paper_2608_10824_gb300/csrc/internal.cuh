@@ -329,6 +329,15 @@ struct CopyList {
   int n;
 };
 void launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st);
+// One-layer entry: idx[i] = pos[i] for i < M (an index outside [0, S) latches
+// VLAC_ERR_DEVICE_CHECK and is replaced by 0, so no access leaves the cache),
+// off = {0, M}.
+void launch_layer_setup(const int32_t* pos, int M, int S, int* idx, int* off, int* err, cudaStream_t st);
+// K or V of one layer of one sequence between the cache layout
+// [head][position][head_dim] (cache) and [position][head * head_dim] (flat),
+// elements of esz bytes; to_cache selects the direction.
+void launch_kv_copy(void* cache, void* flat, int n_heads, int Tc, int head_dim, int esz, bool to_cache,
+                    cudaStream_t st);
 void launch_copies(const CopyList& list, cudaStream_t st);
 
 // Tensor maps of one activation buffer with boxes of 32, 64, 128 and 256 rows.

@@ -366,6 +366,51 @@ __global__ void copy_spans_kernel(CopyList list, StepParams p, StepParams* prm) 
   }
 }
 
+// ---- the one-layer entry ----------------------------------------------------------
+
+__global__ void layer_setup_kernel(const int32_t* __restrict__ pos, int M, int S, int* __restrict__ idx,
+                                   int* __restrict__ off, int* err) {
+  pdl_wait();
+  pdl_trigger();
+  for (int i = threadIdx.x; i < M; i += blockDim.x) {
+    int p = pos[i];
+    if (p < 0 || p >= S) {
+      set_error(err, VLAC_ERR_DEVICE_CHECK);
+      p = 0;
+    }
+    idx[i] = p;
+  }
+  if (threadIdx.x == 0) {
+    off[0] = 0;
+    off[1] = M;
+  }
+}
+
+// One block per (position, head): head_dim elements, copied as 4-byte words.
+__global__ void kv_copy_kernel(uint8_t* __restrict__ cache, uint8_t* __restrict__ flat, int n_heads, int Tc,
+                               int row_bytes, bool to_cache) {
+  pdl_wait();
+  pdl_trigger();
+  const int t = blockIdx.x, h = blockIdx.y;
+  uint32_t* cw = reinterpret_cast<uint32_t*>(cache + ((size_t)h * Tc + t) * row_bytes);
+  uint32_t* fw = reinterpret_cast<uint32_t*>(flat + ((size_t)t * n_heads + h) * row_bytes);
+  for (int w = threadIdx.x; w < row_bytes / 4; w += blockDim.x) {
+    if (to_cache)
+      cw[w] = fw[w];
+    else
+      fw[w] = cw[w];
+  }
+}
+
+void launch_layer_setup(const int32_t* pos, int M, int S, int* idx, int* off, int* err, cudaStream_t st) {
+  launch_k(layer_setup_kernel, dim3(1), dim3(256), 0, st, pos, M, S, idx, off, err);
+}
+void launch_kv_copy(void* cache, void* flat, int n_heads, int Tc, int head_dim, int esz, bool to_cache,
+                    cudaStream_t st) {
+  launch_k(kv_copy_kernel, dim3(Tc, n_heads), dim3(64), 0, st, static_cast<uint8_t*>(cache),
+           static_cast<uint8_t*>(flat), n_heads, Tc, head_dim * esz, to_cache);
+}
+
 void launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st) {
   launch_k(copy_spans_kernel, dim3(64), dim3(256), 0, st, list, p, prm);
 }

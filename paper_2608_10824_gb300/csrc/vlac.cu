@@ -652,6 +652,61 @@ void gemm(vlac_ctx* c, const ActMaps* tmA, const CUtensorMap* tmW, const T* A, c
   c->launches += 1;
 }
 
+// One decoder layer of the prefix pass for the rows `rl` of B sequences:
+// the input norm (rows joining at this layer start from H, rows computed at
+// the previous layer record their input there; H NULL at layer 0), q/k/v
+// with RoPE and the K/V scatter into Kc_l / Vc_l (this layer of the cache),
+// the mixed-cache attention, o-projection + residual, the MLP norm, gate/up +
+// SwiGLU and down + residual.
+template <typename T>
+void prefix_layer(vlac_ctx* c, const Rows& rl, const int* off_prev, int B, int l, float* H, size_t h_seq_stride,
+                  T* Kc_l, T* Vc_l, size_t kv_seq_stride, cudaStream_t st) {
+  const vlac_dims& d = c->d;
+  const int S = c->S, Hd = d.hidden, F = d.ffn, nh = d.n_heads, hd = d.head_dim;
+  const float eps = d.rms_eps;
+  T* A = static_cast<T*>(c->A);
+  T* Q = static_cast<T*>(c->Q);
+  T* AO = static_cast<T*>(c->AO);
+  T* G = static_cast<T*>(c->G);
+  auto W = [](void* p) { return static_cast<const T*>(p); };
+  auto with_tail = [&](SplitPlan p) {
+    p.tail_p = c->part_tail;
+    return p;
+  };
+  const SplitPlan sq = with_tail(c->sp_qkv), so = with_tail(c->sp_o), sg = with_tail(c->sp_gu), sd = with_tail(c->sp_d);
+  const int* ml = rl.off + B;
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_layer_in<T>(rl, off_prev, B, S, Hd, H, h_seq_stride, W(c->attn_norm[l]), eps, A, st);
+  }
+  gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_qkv[l] : nullptr, A, c->wqkv[l], ml, 3 * Hd, Hd, sq, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_qkv_epilogue<T>(rl, B, S, nh, hd, c->part, sq, c->rope_cos, c->rope_sin, Q, Kc_l, Vc_l, kv_seq_stride,
+                           c->Tc, st);
+  }
+  {
+    ProfScope ps_(c, VLAC_PROF_PREFIX_ATTN, 0, st);
+    launch_attention<T>(rl, B, S, nh, hd, Q, Kc_l, Vc_l, kv_seq_stride, c->Tc, c->P, d.parallel, d.n_action, AO, st);
+  }
+  gemm<T>(c, &c->tm_AO, c->bf16 ? &c->tm_o[l] : nullptr, AO, c->wo[l], ml, Hd, Hd, so, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_residual_norm<T>(rl, B, S, Hd, c->part, so, W(c->ffn_norm[l]), eps, A, st);
+  }
+  gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_gu[l] : nullptr, A, c->wgu[l], ml, 2 * F, Hd, sg, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_swiglu<T>(rl, B, S, F, c->part, sg, G, st);
+  }
+  gemm<T>(c, &c->tm_G, c->bf16 ? &c->tm_d[l] : nullptr, G, c->wd[l], ml, Hd, F, sd, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_residual(rl, B, S, Hd, c->part, sd, st);
+  }
+  c->launches += 6;
+}
+
 // The step body: reads only the staged inputs and writes only the context's
 // output buffers, so its launches can be captured once and replayed.
 template <typename T>
@@ -706,47 +761,11 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   }
   c->launches += 2;
 
-  auto with_tail = [&](SplitPlan p) {
-    p.tail_p = c->part_tail;
-    return p;
-  };
-  const SplitPlan sq = with_tail(c->sp_qkv), so = with_tail(c->sp_o), sg = with_tail(c->sp_gu), sd = with_tail(c->sp_d);
   for (int l = 0; l < L; ++l) {
     Rows rl{c->off + (size_t)l * (B + 1), c->idx, S, c->X};
-    const int* ml = rl.off + B;
     const int* off_prev = l == 0 ? rl.off : c->off + (size_t)(l - 1) * (B + 1);
-    {
-      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_layer_in<T>(rl, off_prev, B, S, Hd, l == 0 ? nullptr : k->H + (size_t)l * S * Hd, k->h_seq_stride,
-                         W(c->attn_norm[l]), eps, A, st);
-    }
-    gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_qkv[l] : nullptr, A, c->wqkv[l], ml, 3 * Hd, Hd, sq, st);
-    {
-      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_qkv_epilogue<T>(rl, B, S, nh, hd, c->part, sq, c->rope_cos, c->rope_sin, Q,
-                             Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, st);
-    }
-    {
-      ProfScope ps_(c, VLAC_PROF_PREFIX_ATTN, 0, st);
-      launch_attention<T>(rl, B, S, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, c->P,
-                          d.parallel, D, AO, st);
-    }
-    gemm<T>(c, &c->tm_AO, c->bf16 ? &c->tm_o[l] : nullptr, AO, c->wo[l], ml, Hd, Hd, so, st);
-    {
-      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_residual_norm<T>(rl, B, S, Hd, c->part, so, W(c->ffn_norm[l]), eps, A, st);
-    }
-    gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_gu[l] : nullptr, A, c->wgu[l], ml, 2 * F, Hd, sg, st);
-    {
-      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_swiglu<T>(rl, B, S, F, c->part, sg, G, st);
-    }
-    gemm<T>(c, &c->tm_G, c->bf16 ? &c->tm_d[l] : nullptr, G, c->wd[l], ml, Hd, F, sd, st);
-    {
-      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_residual(rl, B, S, Hd, c->part, sd, st);
-    }
-    c->launches += 6;
+    prefix_layer<T>(c, rl, off_prev, B, l, l == 0 ? nullptr : k->H + (size_t)l * S * Hd, k->h_seq_stride,
+                    Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, st);
   }
   // action head on the prefix pass: the last text row, or the parallel action block
   {
@@ -1042,6 +1061,61 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   c->launches += 1;
   CK(cudaGetLastError());
   return VLAC_OK;
+}
+
+// ---- the one-layer workload -----------------------------------------------------
+
+namespace {
+template <typename T>
+int layer_bench_impl(vlac_ctx* c, vlac_cache* k, int seq, int layer, const int32_t* pos, int M, float* x,
+                     cudaStream_t st) {
+  const vlac_dims& d = c->d;
+  const size_t Hd = d.hidden, kv_layer = (size_t)d.n_heads * c->Tc * d.head_dim;
+  launch_layer_setup(pos, M, c->S, c->idx, c->off, c->err, st);
+  c->launches += 1;
+  CK(cudaMemcpyAsync(c->X, x, (size_t)M * Hd * sizeof(float), cudaMemcpyDeviceToDevice, st));
+  Rows rl{c->off, c->idx, c->S, c->X};
+  T* Kc = static_cast<T*>(k->K) + (size_t)seq * k->kv_seq_stride + (size_t)layer * kv_layer;
+  T* Vc = static_cast<T*>(k->V) + (size_t)seq * k->kv_seq_stride + (size_t)layer * kv_layer;
+  prefix_layer<T>(c, rl, rl.off, 1, layer, nullptr, 0, Kc, Vc, k->kv_seq_stride, st);
+  CK(cudaMemcpyAsync(x, c->X, (size_t)M * Hd * sizeof(float), cudaMemcpyDeviceToDevice, st));
+  CK(cudaGetLastError());
+  return c->fatal ? VLAC_ERR_INVALID_ARG : VLAC_OK;
+}
+}  // namespace
+
+extern "C" int vlac_layer_bench(vlac_ctx* c, vlac_cache* k, int seq, int layer, const int32_t* pos, int M, float* x,
+                                void* stream) {
+  if (!c || !k || !pos || !x || k->ctx != c || seq < 0 || seq >= k->B || layer < 0 || layer >= c->d.n_layers ||
+      M < 1 || M > c->S)
+    return VLAC_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  return c->bf16 ? layer_bench_impl<bf16>(c, k, seq, layer, pos, M, x, st)
+                 : layer_bench_impl<float>(c, k, seq, layer, pos, M, x, st);
+}
+
+namespace {
+int kv_move(const vlac_cache* k, int seq, int layer, void* K, void* V, bool to_cache, void* stream) {
+  if (!k || !K || !V || seq < 0 || seq >= k->B || layer < 0 || layer >= k->ctx->d.n_layers ||
+      (reinterpret_cast<uintptr_t>(K) | reinterpret_cast<uintptr_t>(V)) % 4)
+    return VLAC_ERR_INVALID_ARG;
+  const vlac_ctx* c = k->ctx;
+  const vlac_dims& d = c->d;
+  const size_t kv_layer = (size_t)d.n_heads * c->Tc * d.head_dim;
+  const size_t off = ((size_t)seq * k->kv_seq_stride + (size_t)layer * kv_layer) * c->esz;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  launch_kv_copy(static_cast<char*>(k->K) + off, K, d.n_heads, c->Tc, d.head_dim, (int)c->esz, to_cache, st);
+  launch_kv_copy(static_cast<char*>(k->V) + off, V, d.n_heads, c->Tc, d.head_dim, (int)c->esz, to_cache, st);
+  CK(cudaGetLastError());
+  return VLAC_OK;
+}
+}  // namespace
+
+extern "C" int vlac_cache_load(vlac_cache* k, int seq, int layer, const void* K, const void* V, void* stream) {
+  return kv_move(k, seq, layer, const_cast<void*>(K), const_cast<void*>(V), true, stream);
+}
+extern "C" int vlac_cache_store(const vlac_cache* k, int seq, int layer, void* K, void* V, void* stream) {
+  return kv_move(k, seq, layer, K, V, false, stream);
 }
 
 extern "C" int vlac_sync_error(vlac_ctx* c) {

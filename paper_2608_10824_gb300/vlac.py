@@ -67,7 +67,8 @@ class StepOut(C.Structure):
 
 EXPORTS = ["vlac_create", "vlac_destroy", "vlac_cache_bytes", "vlac_cache_init", "vlac_cache_destroy",
            "vlac_step", "vlac_reset", "vlac_sync_error", "vlac_launch_count", "vlac_selftest_wait",
-           "vlac_prof_enable", "vlac_prof_read", "vlac_select_noalloc", "vlac_strerror"]
+           "vlac_prof_enable", "vlac_prof_read", "vlac_select_noalloc", "vlac_strerror", "vlac_layer_bench",
+           "vlac_cache_load", "vlac_cache_store"]
 
 
 def lib():
@@ -96,6 +97,9 @@ def lib():
                                          C.POINTER(C.c_double)]
             L.vlac_select_noalloc.argtypes = [C.POINTER(Dims), i32, vp, vp, vp, vp, Rational, C.c_float, vp, vp,
                                               vp, vp, vp, vp, vp]
+            L.vlac_layer_bench.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp]
+            L.vlac_cache_load.argtypes = [vp, i32, i32, vp, vp, vp]
+            L.vlac_cache_store.argtypes = [vp, i32, i32, vp, vp, vp]
             L.vlac_strerror.argtypes = [i32]
             L.vlac_strerror.restype = C.c_char_p
             for name in EXPORTS:
@@ -208,6 +212,23 @@ class Context:
                              permille.ctypes.data, C.byref(opts), C.byref(so), _stream_ptr(stream))
         _check(rc, "vlac_step")
         return out
+
+    def layer_bench(self, cache: "Cache", seq: int, layer: int, pos, x, stream=None):
+        """One decoder layer for the rows at positions `pos` (CUDA int32 [M]);
+        x (CUDA fp32 [M][hidden]) holds their inputs and receives their outputs."""
+        assert pos.dtype.itemsize == 4 and x.is_contiguous() and x.shape[0] == pos.shape[0]
+        _check(lib().vlac_layer_bench(self._h, cache._h, seq, layer, pos.data_ptr(), int(pos.shape[0]),
+                                      x.data_ptr(), _stream_ptr(stream)), "vlac_layer_bench")
+
+    def cache_load(self, cache: "Cache", seq: int, layer: int, K, V, stream=None):
+        """K, V: CUDA [cache_len][hidden] in the model's dtype, into the cache."""
+        _check(lib().vlac_cache_load(cache._h, seq, layer, K.data_ptr(), V.data_ptr(), _stream_ptr(stream)),
+               "vlac_cache_load")
+
+    def cache_store(self, cache: "Cache", seq: int, layer: int, K, V, stream=None):
+        """K, V: CUDA [cache_len][hidden] in the model's dtype, filled from the cache."""
+        _check(lib().vlac_cache_store(cache._h, seq, layer, K.data_ptr(), V.data_ptr(), _stream_ptr(stream)),
+               "vlac_cache_store")
 
     def reset(self, cache: "Cache", seq: int = -1, stream=None):
         _check(lib().vlac_reset(cache._h, seq, _stream_ptr(stream)), "vlac_reset")
