@@ -98,6 +98,12 @@ typedef struct vlac_step_opts {
                                   cache always runs the full branch. */
   const int32_t* forced_ids;   /* device [B][n_action]: bins fed back during autoregressive
                                   decode instead of the argmax (lock-step replay); NULL = argmax */
+  const uint8_t* active;       /* device [B]: 0 = the sequence sits this step out (a running batch
+                                  that episodes join and leave): its prefix cache, gate state and
+                                  previous frame stay as they are and its outputs are zero (the
+                                  batch's decode rows still run, so its decode positions, which
+                                  its next step rewrites before reading them, may change);
+                                  NULL = all step */
 } vlac_step_opts;
 
 /* Device output buffers of one step (B = the cache's batch, D = n_action,

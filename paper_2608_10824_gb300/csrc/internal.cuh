@@ -22,7 +22,7 @@ struct StepParams {
   int32_t reduction;  // resolved: 0 mean, 1 min
   int32_t has_override;
   int32_t has_forced;
-  int32_t pad;
+  int32_t has_active;
   uint16_t permille[kMaxLayers];
 };
 
@@ -282,7 +282,7 @@ void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid,
                    const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
                    int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
                    uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
-                   cudaStream_t st);
+                   const uint8_t* active, cudaStream_t st);
 
 template <typename T>
 void launch_im2col(Rows rows, int B, int S, const uint8_t* frames, int n_views, int img_h, int img_w,
@@ -313,7 +313,19 @@ void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int 
                          const int32_t* ids, const int32_t* forced, const StepParams* prm, float* Xd,
                          int* idx_dec, float* ssq_out, int* err, cudaStream_t st);
 void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps,
-                   float* m_prev, uint8_t* valid, float* user_step_margin, cudaStream_t st);
+                   float* m_prev, uint8_t* valid, float* user_step_margin, const uint8_t* active, cudaStream_t st);
+// End of a step: the previous frame of every sequence that stepped becomes
+// this step's frame, and the outputs of the sequences that sat the step out
+// are zeroed (with prm->has_active; active NULL = all stepped).
+struct StepOutputs {
+  int32_t* ids;
+  float *margins, *gaps, *logits, *step_margin;
+  uint8_t *recomputed, *gate_auto, *mask;
+  int32_t *idx, *M;
+};
+void launch_commit(int B, int D, int n_bins, int Nv, int S, int L, size_t frame_bytes, const uint8_t* frames,
+                   uint8_t* prev, const StepParams* prm, const uint8_t* active, const StepOutputs& o,
+                   cudaStream_t st);
 
 // Copies of the caller's per-step inputs into the context's staging buffers
 // (and the step scalars into device memory), and of the step's outputs back

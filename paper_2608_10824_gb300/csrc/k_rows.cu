@@ -322,11 +322,15 @@ __global__ void decode_embed_kernel(int d, int D, int P, int hidden, int vocab, 
 // the next step's gate and becomes valid.
 __global__ void finish_kernel(int B, int D, const StepParams* __restrict__ prm, const float* __restrict__ margins,
                               const float* __restrict__ gaps, float* __restrict__ m_prev, uint8_t* __restrict__ valid,
-                              float* __restrict__ user_step_margin) {
+                              float* __restrict__ user_step_margin, const uint8_t* __restrict__ active) {
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
+  if (prm->has_active && active && !active[b]) {  // sat the step out: the gate state stays
+    user_step_margin[b] = 0.f;
+    return;
+  }
   const float* sig = (prm->margin_kind == VLAC_MARGIN_LOGIT ? gaps : margins) + (size_t)b * D;
   float m;
   if (prm->reduction == VLAC_REDUCE_MIN) {
@@ -465,9 +469,54 @@ void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int 
            prm, Xd, idx_dec, ssq_out, err);
 }
 void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps, float* m_prev,
-                   uint8_t* valid, float* user_step_margin, cudaStream_t st) {
+                   uint8_t* valid, float* user_step_margin, const uint8_t* active, cudaStream_t st) {
   launch_k(finish_kernel, dim3((B + 63) / 64), dim3(64), 0, st, B, D, prm, margins, gaps, m_prev, valid,
-           user_step_margin);
+           user_step_margin, active);
+}
+
+// Grid (chunks, B): sequence b's previous frame becomes this step's frame (16-byte
+// words where both ends allow, bytes otherwise), or, for a sequence that sat
+// the step out, its outputs are zeroed.
+__global__ void commit_kernel(int D, int n_bins, int Nv, int S, int L, size_t frame_bytes,
+                              const uint8_t* __restrict__ frames, uint8_t* __restrict__ prev,
+                              const StepParams* __restrict__ prm, const uint8_t* __restrict__ active, StepOutputs o) {
+  pdl_wait();
+  pdl_trigger();
+  const int b = blockIdx.y;
+  const size_t tid = (size_t)blockIdx.x * blockDim.x + threadIdx.x, nth = (size_t)gridDim.x * blockDim.x;
+  if (!(prm->has_active && active && !active[b])) {
+    const uint8_t* src = frames + (size_t)b * frame_bytes;
+    uint8_t* dst = prev + (size_t)b * frame_bytes;
+    if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0) {
+      const size_t nv = frame_bytes / 16;
+      for (size_t i = tid; i < nv; i += nth) reinterpret_cast<uint4*>(dst)[i] = reinterpret_cast<const uint4*>(src)[i];
+      for (size_t i = nv * 16 + tid; i < frame_bytes; i += nth) dst[i] = src[i];
+    } else {
+      for (size_t i = tid; i < frame_bytes; i += nth) dst[i] = src[i];
+    }
+    return;
+  }
+  for (size_t i = tid; i < (size_t)D; i += nth) {
+    o.ids[(size_t)b * D + i] = 0;
+    o.margins[(size_t)b * D + i] = 0.f;
+    o.gaps[(size_t)b * D + i] = 0.f;
+  }
+  for (size_t i = tid; i < (size_t)D * n_bins; i += nth) o.logits[(size_t)b * D * n_bins + i] = 0.f;
+  for (size_t i = tid; i < (size_t)Nv; i += nth) o.mask[(size_t)b * Nv + i] = 0;
+  for (size_t i = tid; i < (size_t)S; i += nth) o.idx[(size_t)b * S + i] = 0;
+  for (size_t i = tid; i < (size_t)L; i += nth) o.M[(size_t)b * L + i] = 0;
+  if (tid == 0) {
+    o.recomputed[b] = 0;
+    o.gate_auto[b] = 0;
+    o.step_margin[b] = 0.f;
+  }
+}
+
+void launch_commit(int B, int D, int n_bins, int Nv, int S, int L, size_t frame_bytes, const uint8_t* frames,
+                   uint8_t* prev, const StepParams* prm, const uint8_t* active, const StepOutputs& o,
+                   cudaStream_t st) {
+  launch_k(commit_kernel, dim3(16, B), dim3(256), 0, st, D, n_bins, Nv, S, L, frame_bytes, frames, prev, prm, active,
+           o);
 }
 
 #define VLAC_INST(T)                                                                                              \

@@ -88,7 +88,8 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
                               int Nv, int S, int L, int P, int parallel, int n_action, uint8_t* __restrict__ full_out,
                               int* __restrict__ idx, int* __restrict__ M, int* __restrict__ emit_slot,
                               uint8_t* __restrict__ user_recomputed, uint8_t* __restrict__ user_gate_auto,
-                              int* __restrict__ user_idx, int* __restrict__ user_M) {
+                              int* __restrict__ user_idx, int* __restrict__ user_M,
+                              const uint8_t* __restrict__ active) {
   pdl_wait();
   pdl_trigger();
   extern __shared__ uint8_t smem[];
@@ -98,6 +99,17 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
   __shared__ int s_full;
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
+  if (prm->has_active && active && !active[b]) {
+    // the sequence sits this step out: no rows at any layer
+    if (tid == 0) {
+      full_out[b] = 0;
+      emit_slot[b] = 0;
+      if (user_recomputed) user_recomputed[b] = 0;
+      if (user_gate_auto) user_gate_auto[b] = 0;
+    }
+    for (int l = tid; l < L; l += blockDim.x) M[(size_t)b * L + l] = 0;
+    return;
+  }
   if (tid == 0) {
     const bool ok = valid[b] != 0;
     const bool gate = !ok || m_prev[b] < prm->tau_margin;
@@ -190,10 +202,10 @@ void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid,
                    const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
                    int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
                    uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
-                   cudaStream_t st) {
+                   const uint8_t* active, cudaStream_t st) {
   const size_t smem = (size_t)Nv * (sizeof(int3) + sizeof(int) + 1) + 16;
   launch_k(select_kernel, dim3(B), dim3(512), smem, st, stats, mask, valid, m_prev, prm, override_, Nv, S, L, P,
-           parallel, n_action, full, idx, M, emit_slot, user_recomputed, user_gate_auto, user_idx, user_M);
+           parallel, n_action, full, idx, M, emit_slot, user_recomputed, user_gate_auto, user_idx, user_M, active);
   launch_k(plan_kernel, dim3(1), dim3(256), 0, st, M, B, L, off);
 }
 

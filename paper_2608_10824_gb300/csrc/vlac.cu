@@ -86,6 +86,7 @@ struct vlac_ctx {
   float* in_proprio;
   int8_t* in_override;
   int32_t* in_forced;
+  uint8_t* in_active;
   int32_t* o_ids;
   float *o_margins, *o_gaps, *o_step_margin, *o_logits;
   uint8_t *o_recomputed, *o_gate_auto, *o_mask;
@@ -450,6 +451,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->in_proprio, Bm * std::max(d.proprio_dim, 1) * 4, base);
     sc.take(c->in_override, Bm, base);
     sc.take(c->in_forced, Bm * d.n_action * 4, base);
+    sc.take(c->in_active, Bm, base);
     sc.take(c->o_ids, Bm * d.n_action * 4, base);
     sc.take(c->o_margins, Bm * d.n_action * 4, base);
     sc.take(c->o_gaps, Bm * d.n_action * 4, base);
@@ -742,7 +744,8 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_select(c->stats, c->mask, k->valid, k->m_prev, c->prm, ovr, B, c->Nv, S, L, c->P, d.parallel, D, c->full,
-                  c->idx, c->M, c->off, c->emit_slot, out->recomputed, out->gate_auto, out->idx, out->M, st);
+                  c->idx, c->M, c->off, c->emit_slot, out->recomputed, out->gate_auto, out->idx, out->M,
+                  c->in_active, st);
   }
   c->launches += 3;
 
@@ -940,11 +943,17 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   }
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
-    launch_finish(B, D, c->prm, out->margins, out->logit_gap, k->m_prev, k->valid, out->step_margin, st);
+    launch_finish(B, D, c->prm, out->margins, out->logit_gap, k->m_prev, k->valid, out->step_margin, c->in_active,
+                  st);
   }
-  c->launches += 1;
-  const size_t fb = (size_t)d.n_views * d.img_h * d.img_w * 3;
-  CK(cudaMemcpyAsync(k->prev, frames, (size_t)B * fb, cudaMemcpyDeviceToDevice, st));
+  {
+    ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
+    const StepOutputs so{out->action_ids, out->margins,     out->logit_gap, out->logits, out->step_margin,
+                         out->recomputed, out->gate_auto,   out->static_mask, out->idx,  out->M};
+    launch_commit(B, D, nb, c->Nv, S, L, (size_t)d.n_views * d.img_h * d.img_w * 3, frames, k->prev, c->prm,
+                  c->in_active, so, st);
+  }
+  c->launches += 2;
   CK(cudaMemcpyAsync(c->err_host, c->err, sizeof(int), cudaMemcpyDeviceToHost, st));
   CK(cudaGetLastError());
   return VLAC_OK;
@@ -1016,6 +1025,7 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   p.reduction = red;
   p.has_override = (opts && opts->gate_override) ? 1 : 0;
   p.has_forced = (opts && opts->forced_ids) ? 1 : 0;
+  p.has_active = (opts && opts->active) ? 1 : 0;
   // an error latched by an earlier step on this context is reported first
   if (*c->err_host) {
     const int e = *c->err_host;
@@ -1036,6 +1046,7 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   if (d.proprio_dim) add(in, proprio, c->in_proprio, (size_t)B * d.proprio_dim * 4);
   if (p.has_override) add(in, opts->gate_override, c->in_override, (size_t)B);
   if (p.has_forced) add(in, opts->forced_ids, c->in_forced, (size_t)B * D * 4);
+  if (p.has_active) add(in, opts->active, c->in_active, (size_t)B);
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_stage(p, c->prm, in, st);

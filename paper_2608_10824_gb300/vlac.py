@@ -56,7 +56,7 @@ class Rational(C.Structure):
 
 class StepOpts(C.Structure):
     _fields_ = [("margin_kind", C.c_int32), ("reduction", C.c_int32), ("gate_override", C.c_void_p),
-                ("forced_ids", C.c_void_p)]
+                ("forced_ids", C.c_void_p), ("active", C.c_void_p)]
 
 
 class StepOut(C.Structure):
@@ -194,7 +194,8 @@ class Context:
 
     def step(self, cache: "Cache", frames, prompt, proprio=None, tau_sim=(996, 1000), tau_margin: float = 0.0,
              permille=None, margin_kind: int = MARGIN_PROB, reduction: int = REDUCE_DEFAULT, gate_override=None,
-             forced_ids=None, out: Optional[Dict] = None, want: Sequence[str] = (), stream=None) -> Dict:
+             forced_ids=None, out: Optional[Dict] = None, want: Sequence[str] = (), stream=None,
+             active=None) -> Dict:
         """One step for every sequence of `cache`; inputs are CUDA tensors.
         Returns the dict of device output tensors (allocated unless given)."""
         d = self.d
@@ -206,7 +207,7 @@ class Context:
         so = StepOut(*[_ptr(out.get(k)) for k in (
             "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
             "static_mask", "idx", "M")])
-        opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids))
+        opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids), _ptr(active))
         rc = lib().vlac_step(self._h, cache._h, frames.data_ptr(), prompt.data_ptr(), _ptr(proprio),
                              Rational(int(tau_sim[0]), int(tau_sim[1])), float(tau_margin),
                              permille.ctypes.data, C.byref(opts), C.byref(so), _stream_ptr(stream))

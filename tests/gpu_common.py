@@ -79,12 +79,16 @@ class Lockstep:
         self.log = []
         self.logit_tol = logit_tol
 
-    def step(self, frames, prompt, proprio, tau_sim, tau_m, permille, margin_kind=0, force_branch=None):
+    def step(self, frames, prompt, proprio, tau_sim, tau_m, permille, margin_kind=0, force_branch=None,
+             active=None):
+        """active: uint8 [B], 0 = the sequence sits the step out (both sides)."""
         torch = self.torch
         d, B = self.d, self.B
+        act = None if active is None else np.ascontiguousarray(active, np.uint8)
         o = self.orc.step(self.oc, frames, prompt, proprio, tau_sim=tau_sim, tau_margin=tau_m,
                           permille=permille, margin_kind=margin_kind,
-                          gate_override=None if force_branch is None else np.full(B, force_branch, np.int8))
+                          gate_override=None if force_branch is None else np.full(B, force_branch, np.int8),
+                          active=act)
         # branch: free-running, except where the oracle's m_{t-1} sits in the tie zone
         ovr = np.full(B, -1, np.int8) if force_branch is None else np.full(B, force_branch, np.int8)
         if self.prev_m is not None and force_branch is None:
@@ -97,13 +101,17 @@ class Lockstep:
             tau_sim=tau_sim, tau_margin=tau_m, permille=permille, margin_kind=margin_kind,
             gate_override=torch.from_numpy(ovr).cuda(),
             forced_ids=torch.from_numpy(o["action_ids"].astype(np.int32)).cuda(),
-            want=("gate_auto", "logits", "static_mask", "idx", "M"))
+            want=("gate_auto", "logits", "static_mask", "idx", "M"),
+            active=None if act is None else torch.from_numpy(act).cuda())
         torch.cuda.synchronize()
         g = {k: v.cpu().numpy() for k, v in g.items()}
         err = self.ctx.sync_error()
         assert err == 0, f"device error {err}"
         rep = compare(d, o, g, self.prev_m, tau_m, self.logit_tol)
-        self.prev_m = o["step_margin"].copy()
+        m = o["step_margin"].copy()
+        if act is not None and self.prev_m is not None:  # a paused sequence keeps its m_{t-1}
+            m = np.where(act != 0, m, self.prev_m)
+        self.prev_m = m
         self.log.append(rep)
         return o, g, rep
 
