@@ -104,6 +104,9 @@ typedef struct vlac_step_opts {
   int32_t s2_layer;            /* Stage 2: the layer (0 .. n_layers-1) whose attention gives the
                                   relevance: per visual patch, the softmax probability the text
                                   queries put on its key, summed over text rows and heads */
+  const uint8_t* s2_forced;    /* device [B][Nv]: the Stage-2 removal set to apply instead of the
+                                  library's own (lock-step replay; `relevant` still reports the
+                                  library's own set); NULL = the library's own */
 } vlac_step_opts;
 
 /* Device output buffers of one step (B = the cache's batch, D = n_action,

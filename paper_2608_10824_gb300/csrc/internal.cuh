@@ -24,7 +24,7 @@ struct StepParams {
   int32_t has_forced;
   int32_t s2_top_k;  // Stage 2: 0 = off
   int32_t s2_layer;
-  int32_t pad;
+  int32_t has_s2_forced;
   uint16_t permille[kMaxLayers];
 };
 
@@ -241,13 +241,15 @@ void launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_
                         int3* stats, uint8_t* mask, uint8_t* user_mask, cudaStream_t st);
 // Stage 2 state (all NULL = Stage 2 unavailable): rel [B][Nv] the previous
 // step's relevance and rel_valid [B] whether it holds one (cleared here on a
-// step with Stage 2 off); relevant [B][Nv] receives the removal set and
-// rel_out [B][Nv] is zeroed on a step with Stage 2 off.
+// step with Stage 2 off); s2_forced [B][Nv] (with prm->has_s2_forced) is
+// applied instead of the kernel's own removal set; relevant [B][Nv] receives
+// the own set and rel_out [B][Nv] is zeroed on a step with Stage 2 off.
 void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
                    const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
                    int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
                    uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
-                   const float* rel, uint8_t* rel_valid, uint8_t* relevant, float* rel_out, cudaStream_t st);
+                   const float* rel, uint8_t* rel_valid, const uint8_t* s2_forced, uint8_t* relevant,
+                   float* rel_out, cudaStream_t st);
 
 template <typename T>
 void launch_im2col(Rows rows, int B, int S, const uint8_t* frames, int n_views, int img_h, int img_w,

@@ -93,8 +93,8 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
                               int* __restrict__ idx, int* __restrict__ M, int* __restrict__ emit_slot,
                               uint8_t* __restrict__ user_recomputed, uint8_t* __restrict__ user_gate_auto,
                               int* __restrict__ user_idx, int* __restrict__ user_M, const float* __restrict__ rel,
-                              uint8_t* __restrict__ rel_valid, uint8_t* __restrict__ relevant,
-                              float* __restrict__ rel_out) {
+                              uint8_t* __restrict__ rel_valid, const uint8_t* __restrict__ s2_forced,
+                              uint8_t* __restrict__ relevant, float* __restrict__ rel_out) {
   pdl_wait();
   pdl_trigger();
   extern __shared__ uint8_t smem[];
@@ -135,7 +135,9 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
       }
       r = before < top_k;
     }
-    if (r) s_stat[v] = 0;
+    // lock-step replay: the caller's set is applied, the own one reported
+    const bool apply = (top_k > 0 && prm->has_s2_forced && s2_forced) ? s2_forced[(size_t)b * Nv + v] != 0 : r;
+    if (apply) s_stat[v] = 0;
     if (relevant) relevant[(size_t)b * Nv + v] = r;
     if (top_k == 0 && rel_out) rel_out[(size_t)b * Nv + v] = 0.f;
   }
@@ -217,11 +219,12 @@ void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid,
                    const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
                    int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
                    uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
-                   const float* rel, uint8_t* rel_valid, uint8_t* relevant, float* rel_out, cudaStream_t st) {
+                   const float* rel, uint8_t* rel_valid, const uint8_t* s2_forced, uint8_t* relevant,
+                   float* rel_out, cudaStream_t st) {
   const size_t smem = (size_t)Nv * (sizeof(int3) + sizeof(int) + 1) + 16;
   launch_k(select_kernel, dim3(B), dim3(512), smem, st, stats, mask, valid, m_prev, prm, override_, Nv, S, L, P,
            parallel, n_action, full, idx, M, emit_slot, user_recomputed, user_gate_auto, user_idx, user_M, rel,
-           rel_valid, relevant, rel_out);
+           rel_valid, s2_forced, relevant, rel_out);
   launch_k(plan_kernel, dim3(1), dim3(256), 0, st, M, B, L, off);
 }
 

@@ -100,7 +100,7 @@ extern "C" int vlac_select_noalloc(const vlac_dims* d, int batch, const uint8_t*
                      static_mask, nullptr, st);
   launch_select(stats, static_mask, valid, m_prev, prm, gate_override, batch, Nv, S, L, P, d->parallel,
                 d->n_action, full, idx, M, off, emit, recomputed, nullptr, nullptr, nullptr, nullptr, nullptr,
-                nullptr, nullptr, st);
+                nullptr, nullptr, nullptr, st);
   if (cudaGetLastError() != cudaSuccess) return VLAC_ERR_CUDA;
   return VLAC_OK;
 }

@@ -77,6 +77,7 @@ struct vlac_ctx {
   float* in_proprio;
   int8_t* in_override;
   int32_t* in_forced;
+  uint8_t* in_s2_forced;
   int32_t* o_ids;
   float *o_margins, *o_gaps, *o_step_margin, *o_logits;
   uint8_t *o_recomputed, *o_gate_auto, *o_mask;
@@ -413,6 +414,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->in_proprio, Bm * std::max(d.proprio_dim, 1) * 4, base);
     sc.take(c->in_override, Bm, base);
     sc.take(c->in_forced, Bm * d.n_action * 4, base);
+    sc.take(c->in_s2_forced, Bm * c->Nv, base);
     sc.take(c->o_ids, Bm * d.n_action * 4, base);
     sc.take(c->o_margins, Bm * d.n_action * 4, base);
     sc.take(c->o_gaps, Bm * d.n_action * 4, base);
@@ -646,7 +648,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_select(c->stats, c->mask, k->valid, k->m_prev, c->prm, ovr, B, c->Nv, S, L, c->P, d.parallel, D, c->full,
                   c->idx, c->M, c->off, c->emit_slot, out->recomputed, out->gate_auto, out->idx, out->M, k->rel,
-                  k->rel_valid, out->relevant, out->relevance, st);
+                  k->rel_valid, c->in_s2_forced, out->relevant, out->relevance, st);
   }
   c->launches += 3;
 
@@ -912,6 +914,7 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   if (s2_k < 0 || (s2_k > 0 && (s2_l < 0 || s2_l >= c->d.n_layers))) return VLAC_ERR_INVALID_ARG;
   p.s2_top_k = s2_k;
   p.s2_layer = s2_k > 0 ? s2_l : 0;
+  p.has_s2_forced = (s2_k > 0 && opts->s2_forced) ? 1 : 0;
   // an error latched by an earlier step on this context is reported first
   if (*c->err_host) {
     const int e = *c->err_host;
@@ -932,6 +935,7 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   if (d.proprio_dim) add(in, proprio, c->in_proprio, (size_t)B * d.proprio_dim * 4);
   if (p.has_override) add(in, opts->gate_override, c->in_override, (size_t)B);
   if (p.has_forced) add(in, opts->forced_ids, c->in_forced, (size_t)B * D * 4);
+  if (p.has_s2_forced) add(in, opts->s2_forced, c->in_s2_forced, (size_t)B * c->Nv);
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_stage(p, c->prm, in, st);

@@ -56,7 +56,8 @@ class Rational(C.Structure):
 
 class StepOpts(C.Structure):
     _fields_ = [("margin_kind", C.c_int32), ("reduction", C.c_int32), ("gate_override", C.c_void_p),
-                ("forced_ids", C.c_void_p), ("s2_top_k", C.c_int32), ("s2_layer", C.c_int32)]
+                ("forced_ids", C.c_void_p), ("s2_top_k", C.c_int32), ("s2_layer", C.c_int32),
+                ("s2_forced", C.c_void_p)]
 
 
 class StepOut(C.Structure):
@@ -193,11 +194,12 @@ class Context:
     def step(self, cache: "Cache", frames, prompt, proprio=None, tau_sim=(996, 1000), tau_margin: float = 0.0,
              permille=None, margin_kind: int = MARGIN_PROB, reduction: int = REDUCE_DEFAULT, gate_override=None,
              forced_ids=None, out: Optional[Dict] = None, want: Sequence[str] = (), stream=None,
-             s2_top_k: int = 0, s2_layer: Optional[int] = None) -> Dict:
+             s2_top_k: int = 0, s2_layer: Optional[int] = None, s2_forced=None) -> Dict:
         """One step for every sequence of `cache`; inputs are CUDA tensors.
         Returns the dict of device output tensors (allocated unless given).
         s2_top_k > 0 turns on Stage 2 with the relevance of layer s2_layer
-        (default: the middle layer)."""
+        (default: the middle layer); s2_forced (CUDA uint8 [B][Nv]) replaces
+        its removal set (lock-step replay)."""
         d = self.d
         if permille is None:
             permille = np.full(d.n_layers, 1000, dtype=np.uint16)
@@ -209,7 +211,8 @@ class Context:
             "static_mask", "idx", "M", "relevance", "relevant")])
         if s2_layer is None:
             s2_layer = d.n_layers // 2
-        opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids), int(s2_top_k), int(s2_layer))
+        opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids), int(s2_top_k), int(s2_layer),
+                        _ptr(s2_forced))
         rc = lib().vlac_step(self._h, cache._h, frames.data_ptr(), prompt.data_ptr(), _ptr(proprio),
                              Rational(int(tau_sim[0]), int(tau_sim[1])), float(tau_margin),
                              permille.ctypes.data, C.byref(opts), C.byref(so), _stream_ptr(stream))
