@@ -303,7 +303,14 @@ def config_block(d, args):
                         f"{vis}{extra}, {d.n_text} text tokens, {act}, {EPISODE}-frame scene episode{batch}",
             "global_batch": d.max_batch * args.gpus, "seq_len": d.pass_len, "parallelism": f"replicas x{args.gpus}",
             "tau_sim": f"{TAU_SIM[0]}/{TAU_SIM[1]}", "tau_margin": args.tau_margin,
-            "reuse_permille": "linear 900 -> 500", "l2": "inputs larger than L2 (13 GB of weights per pass)"}
+            "reuse_permille": "linear 900 -> 500", "l2": "inputs larger than L2 (13 GB of weights per pass)",
+            "stage2": (f"top_k {args.stage2_top_k} by the text-to-vision relevance of layer {stage2_layer(d, args)}"
+                       if getattr(args, "stage2_top_k", 0) > 0 else "off")}
+
+
+def stage2_layer(d, args) -> int:
+    layer = getattr(args, "stage2_layer", None)
+    return d.n_layers // 2 if layer is None else layer
 
 
 # ---------------------------------------------------------------------------
@@ -323,6 +330,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layer-sweep", action="store_true",
                     help="time one decoder layer per recomputed-row count (the one-layer workload) instead")
+    ap.add_argument("--stage2-top-k", type=int, default=0,
+                    help="Stage 2 (task-relevant filtering): patches kept out of the reuse set; 0 = off")
+    ap.add_argument("--stage2-layer", type=int, default=None, help="layer whose attention gives the relevance")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -370,7 +380,8 @@ def main():
         if t % EPISODE == 0:
             ctx.reset(cache)
         ctx.step(cache, fr_dev[t % EPISODE], pr_dev, None if pp_dev is None else pp_dev[t % EPISODE],
-                 tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm, out=out)
+                 tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm, out=out,
+                 s2_top_k=args.stage2_top_k, s2_layer=stage2_layer(d, args))
 
     def barrier():
         torch.cuda.synchronize()
@@ -468,7 +479,8 @@ def main():
             q_buf.copy_(pp_host[t % EPISODE], non_blocking=True)
         if t % EPISODE == 0:
             ctx.reset(cache)
-        ctx.step(cache, f_buf, p_buf, q_buf, tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm, out=outs)
+        ctx.step(cache, f_buf, p_buf, q_buf, tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm, out=outs,
+                 s2_top_k=args.stage2_top_k, s2_layer=stage2_layer(d, args))
         for n, hbuf in res_host.items():
             hbuf.copy_(outs[n], non_blocking=True)
         torch.cuda.current_stream().synchronize()  # the action is needed before the next frame

@@ -104,6 +104,15 @@ typedef struct vlac_step_opts {
                                   batch's decode rows still run, so its decode positions, which
                                   its next step rewrites before reading them, may change);
                                   NULL = all step */
+  int32_t s2_top_k;            /* Stage 2 (Sec. III-B task-relevant filtering): the top_k visual
+                                  patches by the previous step's relevance are never reused;
+                                  0 = Stage 2 off (default) */
+  int32_t s2_layer;            /* Stage 2: the layer (0 .. n_layers-1) whose attention gives the
+                                  relevance: per visual patch, the softmax probability the text
+                                  queries put on its key, summed over text rows and heads */
+  const uint8_t* s2_forced;    /* device [B][Nv]: the Stage-2 removal set to apply instead of the
+                                  library's own (lock-step replay; `relevant` still reports the
+                                  library's own set); NULL = the library's own */
 } vlac_step_opts;
 
 /* Device output buffers of one step (B = the cache's batch, D = n_action,
@@ -119,6 +128,8 @@ typedef struct vlac_step_out {
   uint8_t* static_mask; /* optional [B][Nv] Stage-1 result (0 without a previous frame) */
   int32_t* idx;         /* optional [B][S] recompute order: rows of layer l are idx[0..M[l]) */
   int32_t* M;           /* optional [B][L] rows recomputed at each layer */
+  float* relevance;     /* optional [B][Nv] this step's Stage-2 relevance (0 when Stage 2 is off) */
+  uint8_t* relevant;    /* optional [B][Nv] patches Stage 2 kept out of the reusable set this step */
 } vlac_step_out;
 
 typedef struct vlac_ctx vlac_ctx;
@@ -133,7 +144,8 @@ int vlac_destroy(vlac_ctx* ctx);
 /* Bytes of device memory a cache for `batch` (1 .. max_batch) sequences needs:
  * per sequence the K/V of every layer and position, the fp32 input of every
  * layer for the prefix positions (tokens that rejoin at a deeper layer start
- * from it), the previous frame, m_{t-1} and a valid flag. */
+ * from it), the previous frame, m_{t-1}, a valid flag and the last step's
+ * Stage-2 relevance. */
 int vlac_cache_bytes(const vlac_ctx* ctx, int batch, size_t* bytes);
 /* Formats caller-owned device memory (>= vlac_cache_bytes, 256-byte aligned)
  * as an empty cache; the memory must outlive the cache handle.  Synchronous. */
@@ -146,9 +158,11 @@ int vlac_cache_destroy(vlac_cache* cache);
  *   proprio:         device [B][proprio_dim] fp32, NULL when proprio_dim == 0
  *   tau_sim:         Stage-1 threshold (static iff cos > num/den)
  *   tau_margin:      the gate fires iff m_{t-1} < tau_margin (strict)
- *   reuse_permille:  host [n_layers]: k_l = floor(permille[l] * |static| / 1000)
- *                    static patches (the most similar) are reused at layer l; each <= 1000
- *   opts:            NULL = defaults
+ *   reuse_permille:  host [n_layers]: k_l = floor(permille[l] * |reusable| / 1000)
+ *                    reusable patches (the most similar) are reused at layer l; each
+ *                    <= 1000.  Reusable = static and, with Stage 2, not relevant.
+ *   opts:            NULL = defaults; VLAC_ERR_INVALID_ARG if s2_top_k < 0, or if
+ *                    s2_top_k > 0 and s2_layer is not a layer
  *   out:             device output buffers (required members non-NULL)
  * Returns VLAC_ERR_STATE if the cache belongs to another context. */
 int vlac_step(vlac_ctx* ctx, vlac_cache* cache, const uint8_t* frames, const int32_t* prompt_ids,
@@ -157,7 +171,8 @@ int vlac_step(vlac_ctx* ctx, vlac_cache* cache, const uint8_t* frames, const int
               void* stream);
 
 /* Invalidates sequence `seq` (-1 = all): its next step runs the full pass as if
- * no cache existed (Algorithm 1, cache invalidation). */
+ * no cache existed (Algorithm 1, cache invalidation), and Stage 2 has no
+ * previous relevance to use. */
 int vlac_reset(vlac_cache* cache, int seq, void* stream);
 
 /* One decoder layer of the prefix pass on its own (the one-layer workload:

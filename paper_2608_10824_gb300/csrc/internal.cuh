@@ -23,6 +23,9 @@ struct StepParams {
   int32_t has_override;
   int32_t has_forced;
   int32_t has_active;
+  int32_t s2_top_k;  // Stage 2: 0 = off
+  int32_t s2_layer;
+  int32_t has_s2_forced;
   uint16_t permille[kMaxLayers];
 };
 
@@ -278,11 +281,17 @@ int check_dims(const vlac_dims* d);  // VLAC_OK or the error vlac_create would r
 void launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid,
                         const StepParams* prm, int B, int n_views, int img_h, int img_w, int patch,
                         int3* stats, uint8_t* mask, uint8_t* user_mask, cudaStream_t st);
+// Stage 2 state (all NULL = Stage 2 unavailable): rel [B][Nv] the previous
+// step's relevance and rel_valid [B] whether it holds one (cleared here on a
+// step with Stage 2 off); s2_forced [B][Nv] (with prm->has_s2_forced) is
+// applied instead of the kernel's own removal set; relevant [B][Nv] receives
+// the own set and rel_out [B][Nv] is zeroed on a step with Stage 2 off.
 void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
                    const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
                    int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
                    uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
-                   const uint8_t* active, cudaStream_t st);
+                   const uint8_t* active, const float* rel, uint8_t* rel_valid, const uint8_t* s2_forced,
+                   uint8_t* relevant, float* rel_out, cudaStream_t st);
 
 template <typename T>
 void launch_im2col(Rows rows, int B, int S, const uint8_t* frames, int n_views, int img_h, int img_w,
@@ -308,6 +317,14 @@ void launch_residual(Rows rows, int B, int S, int hidden, const float* part, con
 template <typename T>
 void launch_attention(Rows rows, int B, int S, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc,
                       size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, T* O, cudaStream_t st);
+// Stage 2 relevance of one layer (rows as for launch_attention; text rows are
+// positions text_lo .. P-1): part [B][n_heads][Nv] per head, then rel and
+// rel_out [B][Nv] summed over the heads in order, and rel_valid[b] = 1.
+// Returns nonzero if the shared-memory need exceeds a block's.
+template <typename T>
+int launch_relevance(Rows rows, int B, int n_heads, int head_dim, const T* Q, const T* Kc, size_t kv_seq_stride,
+                     int Tc, int Nv, int text_lo, int P, float* part, float* rel, float* rel_out, uint8_t* rel_valid,
+                     const StepParams* prm, const uint8_t* active, cudaStream_t st);
 template <typename T>
 void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
                          const int32_t* ids, const int32_t* forced, const StepParams* prm, float* Xd,
@@ -322,6 +339,8 @@ struct StepOutputs {
   float *margins, *gaps, *logits, *step_margin;
   uint8_t *recomputed, *gate_auto, *mask;
   int32_t *idx, *M;
+  float* relevance;   // Stage 2 outputs [B][Nv]
+  uint8_t* relevant;
 };
 void launch_commit(int B, int D, int n_bins, int Nv, int S, int L, size_t frame_bytes, const uint8_t* frames,
                    uint8_t* prev, const StepParams* prm, const uint8_t* active, const StepOutputs& o,
@@ -335,7 +354,7 @@ struct CopySpan {
   void* dst;
   size_t bytes;
 };
-constexpr int kMaxSpans = 12;
+constexpr int kMaxSpans = 16;
 struct CopyList {
   CopySpan span[kMaxSpans];
   int n;

@@ -505,6 +505,10 @@ __global__ void commit_kernel(int D, int n_bins, int Nv, int S, int L, size_t fr
   for (size_t i = tid; i < (size_t)Nv; i += nth) o.mask[(size_t)b * Nv + i] = 0;
   for (size_t i = tid; i < (size_t)S; i += nth) o.idx[(size_t)b * S + i] = 0;
   for (size_t i = tid; i < (size_t)L; i += nth) o.M[(size_t)b * L + i] = 0;
+  for (size_t i = tid; i < (size_t)Nv; i += nth) {
+    if (o.relevance) o.relevance[(size_t)b * Nv + i] = 0.f;
+    if (o.relevant) o.relevant[(size_t)b * Nv + i] = 0;
+  }
   if (tid == 0) {
     o.recomputed[b] = 0;
     o.gate_auto[b] = 0;

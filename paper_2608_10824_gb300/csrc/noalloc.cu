@@ -99,7 +99,8 @@ extern "C" int vlac_select_noalloc(const vlac_dims* d, int batch, const uint8_t*
   launch_patch_stats(frames, prev_frames, valid, prm, batch, d->n_views, d->img_h, d->img_w, d->patch, stats,
                      static_mask, nullptr, st);
   launch_select(stats, static_mask, valid, m_prev, prm, gate_override, batch, Nv, S, L, P, d->parallel,
-                d->n_action, full, idx, M, off, emit, recomputed, nullptr, nullptr, nullptr, nullptr, st);
+                d->n_action, full, idx, M, off, emit, recomputed, nullptr, nullptr, nullptr, nullptr, nullptr,
+                nullptr, nullptr, nullptr, nullptr, st);
   if (cudaGetLastError() != cudaSuccess) return VLAC_ERR_CUDA;
   return VLAC_OK;
 }

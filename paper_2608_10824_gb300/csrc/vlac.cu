@@ -87,10 +87,16 @@ struct vlac_ctx {
   int8_t* in_override;
   int32_t* in_forced;
   uint8_t* in_active;
+  uint8_t* in_s2_forced;
   int32_t* o_ids;
   float *o_margins, *o_gaps, *o_step_margin, *o_logits;
   uint8_t *o_recomputed, *o_gate_auto, *o_mask;
   int32_t *o_idx, *o_M;
+  float* o_rel;         // Stage-2 relevance of the step [B][Nv]
+  uint8_t* o_relevant;  // Stage-2 removal set of the step [B][Nv]
+  float* rel_part;      // Stage-2 relevance per (sequence, head) [B][n_heads][Nv]
+  bool s2_on = false;   // this step measures and applies Stage 2
+  int s2_layer = 0;
   cudaStream_t cap_stream = nullptr;
   bool use_graph = true;
   bool fatal = false;  // a launch was refused for exceeding a workspace buffer
@@ -115,10 +121,13 @@ struct vlac_cache {
   cudaGraphExec_t gexec = nullptr;
   int eager_steps = 0;
   uint64_t graph_launches = 0;
+  int graph_sig = 0;  // the Stage-2 layout the graph was captured with (0 = off, 1 + layer)
   void *K, *V;
   float* H;
   uint8_t *prev, *valid;
   float* m_prev;
+  float* rel;          // [B][Nv] the last step's Stage-2 relevance
+  uint8_t* rel_valid;  // [B] rel holds one
   size_t kv_seq_stride, h_seq_stride;  // elements per sequence
 };
 
@@ -452,6 +461,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->in_override, Bm, base);
     sc.take(c->in_forced, Bm * d.n_action * 4, base);
     sc.take(c->in_active, Bm, base);
+    sc.take(c->in_s2_forced, Bm * c->Nv, base);
     sc.take(c->o_ids, Bm * d.n_action * 4, base);
     sc.take(c->o_margins, Bm * d.n_action * 4, base);
     sc.take(c->o_gaps, Bm * d.n_action * 4, base);
@@ -462,6 +472,9 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->o_mask, Bm * c->Nv, base);
     sc.take(c->o_idx, Bm * c->S * 4, base);
     sc.take(c->o_M, Bm * L * 4, base);
+    sc.take(c->o_rel, Bm * c->Nv * 4, base);
+    sc.take(c->o_relevant, Bm * c->Nv, base);
+    sc.take(c->rel_part, Bm * d.n_heads * c->Nv * 4, base);
   };
   plan_s(nullptr);
   if (cudaMalloc(&c->wsmem, sc.off) != cudaSuccess) {
@@ -525,8 +538,8 @@ static size_t cache_layout(const vlac_ctx* c, int B, char* base, vlac_cache* k) 
   void* K;
   void* V;
   float* H;
-  uint8_t *prev, *valid;
-  float* m_prev;
+  uint8_t *prev, *valid, *rel_valid;
+  float *m_prev, *rel;
   const size_t kv = (size_t)d.n_layers * d.n_heads * c->Tc * d.head_dim;
   const size_t hs = (size_t)d.n_layers * c->S * d.hidden;
   cv.take(K, B * kv * c->esz, base);
@@ -535,8 +548,11 @@ static size_t cache_layout(const vlac_ctx* c, int B, char* base, vlac_cache* k) 
   cv.take(prev, (size_t)B * d.n_views * d.img_h * d.img_w * 3, base);
   cv.take(m_prev, (size_t)B * 4, base);
   cv.take(valid, (size_t)B, base);
+  cv.take(rel, (size_t)B * c->Nv * 4, base);
+  cv.take(rel_valid, (size_t)B, base);
   if (k) {
     k->K = K; k->V = V; k->H = H; k->prev = prev; k->m_prev = m_prev; k->valid = valid;
+    k->rel = rel; k->rel_valid = rel_valid;
     k->kv_seq_stride = kv;
     k->h_seq_stride = hs;
   }
@@ -579,8 +595,13 @@ extern "C" int vlac_cache_destroy(vlac_cache* k) {
 extern "C" int vlac_reset(vlac_cache* k, int seq, void* stream) {
   if (!k || seq < -1 || seq >= k->B) return VLAC_ERR_INVALID_ARG;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (seq < 0) CK(cudaMemsetAsync(k->valid, 0, (size_t)k->B, st));
-  else CK(cudaMemsetAsync(k->valid + seq, 0, 1, st));
+  if (seq < 0) {
+    CK(cudaMemsetAsync(k->valid, 0, (size_t)k->B, st));
+    CK(cudaMemsetAsync(k->rel_valid, 0, (size_t)k->B, st));
+  } else {
+    CK(cudaMemsetAsync(k->valid + seq, 0, 1, st));
+    CK(cudaMemsetAsync(k->rel_valid + seq, 0, 1, st));
+  }
   return VLAC_OK;
 }
 
@@ -713,8 +734,8 @@ void prefix_layer(vlac_ctx* c, const Rows& rl, const int* off_prev, int B, int l
 // output buffers, so its launches can be captured once and replayed.
 template <typename T>
 int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
-  vlac_step_out outv{c->o_ids, c->o_margins, c->o_gaps, c->o_recomputed, c->o_step_margin, c->o_gate_auto,
-                     c->o_logits, c->o_mask, c->o_idx, c->o_M};
+  vlac_step_out outv{c->o_ids,   c->o_margins, c->o_gaps, c->o_recomputed, c->o_step_margin, c->o_gate_auto,
+                     c->o_logits, c->o_mask,    c->o_idx,  c->o_M,         c->o_rel,         c->o_relevant};
   const vlac_step_out* out = &outv;
   const uint8_t* frames = c->in_frames;
   const int32_t* prompt = c->in_prompt;
@@ -745,7 +766,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_select(c->stats, c->mask, k->valid, k->m_prev, c->prm, ovr, B, c->Nv, S, L, c->P, d.parallel, D, c->full,
                   c->idx, c->M, c->off, c->emit_slot, out->recomputed, out->gate_auto, out->idx, out->M,
-                  c->in_active, st);
+                  c->in_active, k->rel, k->rel_valid, c->in_s2_forced, out->relevant, out->relevance, st);
   }
   c->launches += 3;
 
@@ -769,6 +790,16 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
     const int* off_prev = l == 0 ? rl.off : c->off + (size_t)(l - 1) * (B + 1);
     prefix_layer<T>(c, rl, off_prev, B, l, l == 0 ? nullptr : k->H + (size_t)l * S * Hd, k->h_seq_stride,
                     Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, st);
+    if (c->s2_on && l == c->s2_layer) {
+      // Stage 2: the text rows' attention on the visual keys of this layer (Q
+      // still holds this layer's rows)
+      ProfScope ps_(c, VLAC_PROF_PREFIX_ATTN, 0, st);
+      if (launch_relevance<T>(rl, B, nh, hd, Q, Kc + l * kv_layer, k->kv_seq_stride, c->Tc, c->Nv,
+                              1 + c->Nv + c->has_p, c->P, c->rel_part, k->rel, out->relevance, k->rel_valid,
+                              c->prm, c->in_active, st))
+        c->fatal = true;
+      c->launches += 2;
+    }
   }
   // action head on the prefix pass: the last text row, or the parallel action block
   {
@@ -948,8 +979,9 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   }
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
-    const StepOutputs so{out->action_ids, out->margins,     out->logit_gap, out->logits, out->step_margin,
-                         out->recomputed, out->gate_auto,   out->static_mask, out->idx,  out->M};
+    const StepOutputs so{out->action_ids, out->margins,   out->logit_gap,   out->logits, out->step_margin,
+                         out->recomputed, out->gate_auto, out->static_mask, out->idx,    out->M,
+                         out->relevance,  out->relevant};
     launch_commit(B, D, nb, c->Nv, S, L, (size_t)d.n_views * d.img_h * d.img_w * 3, frames, k->prev, c->prm,
                   c->in_active, so, st);
   }
@@ -968,6 +1000,16 @@ int run_body(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
 // the second captures the body into a graph, which every later step replays.
 int run_step(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   if (!c->use_graph || c->prof_on) return run_body(c, k, st);
+  const int sig = c->s2_on ? 1 + c->s2_layer : 0;
+  if (k->gexec && k->graph_sig != sig) {
+    // Stage 2 switched on or off, or moved to another layer: the launch list
+    // differs, so the graph is captured again (after one eager step)
+    cudaGraphExecDestroy(k->gexec);
+    cudaGraphDestroy(k->graph);
+    k->gexec = nullptr;
+    k->graph = nullptr;
+    k->eager_steps = 0;
+  }
   if (!k->gexec) {
     if (k->eager_steps++ == 0) return run_body(c, k, st);
     const uint64_t n0 = c->launches;
@@ -987,6 +1029,7 @@ int run_step(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
       return VLAC_ERR_CUDA;
     }
     k->graph = g;
+    k->graph_sig = sig;
     k->graph_launches = c->launches - n0;
     c->launches = n0;
   }
@@ -1026,6 +1069,11 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   p.has_override = (opts && opts->gate_override) ? 1 : 0;
   p.has_forced = (opts && opts->forced_ids) ? 1 : 0;
   p.has_active = (opts && opts->active) ? 1 : 0;
+  const int s2_k = opts ? opts->s2_top_k : 0, s2_l = opts ? opts->s2_layer : 0;
+  if (s2_k < 0 || (s2_k > 0 && (s2_l < 0 || s2_l >= c->d.n_layers))) return VLAC_ERR_INVALID_ARG;
+  p.s2_top_k = s2_k;
+  p.s2_layer = s2_k > 0 ? s2_l : 0;
+  p.has_s2_forced = (s2_k > 0 && opts->s2_forced) ? 1 : 0;
   // an error latched by an earlier step on this context is reported first
   if (*c->err_host) {
     const int e = *c->err_host;
@@ -1047,11 +1095,14 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   if (p.has_override) add(in, opts->gate_override, c->in_override, (size_t)B);
   if (p.has_forced) add(in, opts->forced_ids, c->in_forced, (size_t)B * D * 4);
   if (p.has_active) add(in, opts->active, c->in_active, (size_t)B);
+  if (p.has_s2_forced) add(in, opts->s2_forced, c->in_s2_forced, (size_t)B * c->Nv);
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_stage(p, c->prm, in, st);
   }
   c->launches += 1;
+  c->s2_on = p.s2_top_k > 0;
+  c->s2_layer = p.s2_layer;
   int rc = run_step(c, k, st);
   if (rc) return rc;
   CopyList o{};
@@ -1065,6 +1116,8 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   add(o, c->o_mask, out->static_mask, (size_t)B * c->Nv);
   add(o, c->o_idx, out->idx, (size_t)B * c->S * 4);
   add(o, c->o_M, out->M, (size_t)B * d.n_layers * 4);
+  add(o, c->o_rel, out->relevance, (size_t)B * c->Nv * 4);
+  add(o, c->o_relevant, out->relevant, (size_t)B * c->Nv);
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_copies(o, st);

@@ -56,13 +56,14 @@ class Rational(C.Structure):
 
 class StepOpts(C.Structure):
     _fields_ = [("margin_kind", C.c_int32), ("reduction", C.c_int32), ("gate_override", C.c_void_p),
-                ("forced_ids", C.c_void_p), ("active", C.c_void_p)]
+                ("forced_ids", C.c_void_p), ("active", C.c_void_p), ("s2_top_k", C.c_int32), ("s2_layer", C.c_int32),
+                ("s2_forced", C.c_void_p)]
 
 
 class StepOut(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in (
         "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
-        "static_mask", "idx", "M")]
+        "static_mask", "idx", "M", "relevance", "relevant")]
 
 
 EXPORTS = ["vlac_create", "vlac_destroy", "vlac_cache_bytes", "vlac_cache_init", "vlac_cache_destroy",
@@ -186,7 +187,9 @@ class Context:
         }
         shapes = {"gate_auto": ((batch,), torch.uint8), "logits": ((batch, D, d.n_bins), torch.float32),
                   "static_mask": ((batch, d.n_visual), torch.uint8), "idx": ((batch, d.pass_len), torch.int32),
-                  "M": ((batch, d.n_layers), torch.int32)}
+                  "M": ((batch, d.n_layers), torch.int32),
+                  "relevance": ((batch, d.n_visual), torch.float32),
+                  "relevant": ((batch, d.n_visual), torch.uint8)}
         for k in want:
             shp, dt = shapes[k]
             out[k] = torch.zeros(shp, dtype=dt, device=dev)
@@ -195,9 +198,12 @@ class Context:
     def step(self, cache: "Cache", frames, prompt, proprio=None, tau_sim=(996, 1000), tau_margin: float = 0.0,
              permille=None, margin_kind: int = MARGIN_PROB, reduction: int = REDUCE_DEFAULT, gate_override=None,
              forced_ids=None, out: Optional[Dict] = None, want: Sequence[str] = (), stream=None,
-             active=None) -> Dict:
+             active=None, s2_top_k: int = 0, s2_layer: Optional[int] = None, s2_forced=None) -> Dict:
         """One step for every sequence of `cache`; inputs are CUDA tensors.
-        Returns the dict of device output tensors (allocated unless given)."""
+        Returns the dict of device output tensors (allocated unless given).
+        s2_top_k > 0 turns on Stage 2 with the relevance of layer s2_layer
+        (default: the middle layer); s2_forced (CUDA uint8 [B][Nv]) replaces
+        its removal set (lock-step replay)."""
         d = self.d
         if permille is None:
             permille = np.full(d.n_layers, 1000, dtype=np.uint16)
@@ -206,8 +212,11 @@ class Context:
             out = self.alloc_outputs(cache.batch, want)
         so = StepOut(*[_ptr(out.get(k)) for k in (
             "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
-            "static_mask", "idx", "M")])
-        opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids), _ptr(active))
+            "static_mask", "idx", "M", "relevance", "relevant")])
+        if s2_layer is None:
+            s2_layer = d.n_layers // 2
+        opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids), _ptr(active), int(s2_top_k),
+                        int(s2_layer), _ptr(s2_forced))
         rc = lib().vlac_step(self._h, cache._h, frames.data_ptr(), prompt.data_ptr(), _ptr(proprio),
                              Rational(int(tau_sim[0]), int(tau_sim[1])), float(tau_margin),
                              permille.ctypes.data, C.byref(opts), C.byref(so), _stream_ptr(stream))

@@ -28,6 +28,11 @@ ID_EXEMPT_MARGIN = 1e-3
 # twice the bar.  The deep tests exempt exactly those ids, and require the
 # GPU's id to be the first maximum of the GPU's own logits.
 FLAG_TIE = 1e-4
+# Stage 2 relevance, relative to the sequence's largest relevance: the kernel
+# sums fp32 probabilities of the same bf16 (or fp32) Q and K the oracle sums
+# in fp64.  A removal-set difference is allowed only for patches whose oracle
+# relevance lies within twice this of the oracle's k-th / (k+1)-th midpoint.
+REL_TOL = {"bf16": 1e-4, "f32": 1e-5}
 
 SMALL = {
     # bf16 path (tcgen05 GEMMs), head_dim 128, autoregressive decode
@@ -76,19 +81,24 @@ class Lockstep:
         self.gc = self.ctx.new_cache(batch)
         self.torch = torch
         self.prev_m = None
+        self.prev_rel = None
         self.log = []
         self.logit_tol = logit_tol
 
     def step(self, frames, prompt, proprio, tau_sim, tau_m, permille, margin_kind=0, force_branch=None,
-             active=None):
-        """active: uint8 [B], 0 = the sequence sits the step out (both sides)."""
+             active=None, s2_top_k=0, s2_layer=None, s2_lockstep=True):
+        """active: uint8 [B], 0 = the sequence sits the step out (both sides).
+        s2_top_k > 0: Stage 2 on both sides; with s2_lockstep the library
+        applies the oracle's removal set (its own is still compared)."""
         torch = self.torch
         d, B = self.d, self.B
         act = None if active is None else np.ascontiguousarray(active, np.uint8)
+        if s2_layer is None:
+            s2_layer = d.n_layers // 2
         o = self.orc.step(self.oc, frames, prompt, proprio, tau_sim=tau_sim, tau_margin=tau_m,
                           permille=permille, margin_kind=margin_kind,
                           gate_override=None if force_branch is None else np.full(B, force_branch, np.int8),
-                          active=act)
+                          active=act, s2_top_k=s2_top_k, s2_layer=s2_layer)
         # branch: free-running, except where the oracle's m_{t-1} sits in the tie zone
         ovr = np.full(B, -1, np.int8) if force_branch is None else np.full(B, force_branch, np.int8)
         if self.prev_m is not None and force_branch is None:
@@ -101,17 +111,25 @@ class Lockstep:
             tau_sim=tau_sim, tau_margin=tau_m, permille=permille, margin_kind=margin_kind,
             gate_override=torch.from_numpy(ovr).cuda(),
             forced_ids=torch.from_numpy(o["action_ids"].astype(np.int32)).cuda(),
-            want=("gate_auto", "logits", "static_mask", "idx", "M"),
-            active=None if act is None else torch.from_numpy(act).cuda())
+            want=("gate_auto", "logits", "static_mask", "idx", "M", "relevance", "relevant"),
+            active=None if act is None else torch.from_numpy(act).cuda(),
+            s2_top_k=s2_top_k, s2_layer=s2_layer,
+            s2_forced=(torch.from_numpy(np.ascontiguousarray(o["relevant"])).cuda()
+                       if s2_top_k > 0 and s2_lockstep else None))
         torch.cuda.synchronize()
         g = {k: v.cpu().numpy() for k, v in g.items()}
         err = self.ctx.sync_error()
         assert err == 0, f"device error {err}"
         rep = compare(d, o, g, self.prev_m, tau_m, self.logit_tol)
+        rep.update(compare_stage2(d, o, g, s2_top_k, self.prev_rel))
+        rel = o["relevance"].copy() if s2_top_k > 0 else None
         m = o["step_margin"].copy()
         if act is not None and self.prev_m is not None:  # a paused sequence keeps its m_{t-1}
             m = np.where(act != 0, m, self.prev_m)
+            if rel is not None and self.prev_rel is not None:  # and its relevance
+                rel = np.where(act[:, None] != 0, rel, self.prev_rel)
         self.prev_m = m
+        self.prev_rel = rel
         self.log.append(rep)
         return o, g, rep
 
@@ -142,3 +160,30 @@ def compare(d, o, g, prev_m, tau_m, logit_tol=None):
     np.testing.assert_allclose(g["margins"], o["margins"], atol=max(tol * 0.05, 1e-6), rtol=0.05)
     return {"max_logit_diff": float(diff.max()), "id_mismatch": int(mism.sum()),
             "id_exempt": int(exempt.sum()), "recomputed": o["recomputed"].tolist()}
+
+
+def compare_stage2(d, o, g, top_k, prev_rel):
+    """Stage 2: this step's relevance within REL_TOL of the oracle's (relative
+    to the sequence's largest), and the removal set the library decided from
+    its previous relevance equal to the oracle's except inside the tie band
+    around the oracle's k-th / (k+1)-th midpoint."""
+    if top_k == 0:
+        assert not g["relevance"].any() and not g["relevant"].any(), "Stage 2 off: nothing measured or removed"
+        return {"rel_diff": 0.0, "removal_diffs": 0}
+    tol = REL_TOL[d.dtype]
+    worst, diffs = 0.0, 0
+    for b in range(o["relevance"].shape[0]):
+        scale = float(np.max(o["relevance"][b]))
+        err = float(np.max(np.abs(g["relevance"][b].astype(np.float64) - o["relevance"][b]))) / scale
+        assert err <= tol, f"relevance of sequence {b} differs by {err:.3e} (relative) > {tol}"
+        worst = max(worst, err)
+        bad = g["relevant"][b] != o["relevant"][b]
+        if bad.any():
+            assert prev_rel is not None, "a removal set without a previous relevance"
+            r = np.sort(prev_rel[b])[::-1]
+            mid = 0.5 * (r[top_k - 1] + r[top_k]) if top_k < r.size else -np.inf
+            band = 2 * tol * float(np.max(prev_rel[b]))
+            outside = bad & (np.abs(prev_rel[b] - mid) > band)
+            assert not outside.any(), f"removal set differs outside the tie band: {np.flatnonzero(outside)}"
+            diffs += int(bad.sum())
+    return {"rel_diff": worst, "removal_diffs": diffs}
