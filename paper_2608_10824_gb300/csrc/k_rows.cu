@@ -314,15 +314,30 @@ __global__ void decode_embed_kernel(int d, int D, int P, int hidden, int vocab, 
 }
 
 // m_t = mean (Eq. 1) or min of the per-token signals; the cache keeps it for
-// the next step's gate and becomes valid.
+// the next step's gate and becomes valid.  The action delta (Sec. VI) is the
+// L1 distance in bins to the previous step's ids on the sequence.
 __global__ void finish_kernel(int B, int D, const StepParams* __restrict__ prm, const float* __restrict__ margins,
-                              const float* __restrict__ gaps, float* __restrict__ m_prev, uint8_t* __restrict__ valid,
-                              float* __restrict__ user_step_margin) {
+                              const float* __restrict__ gaps, const float* __restrict__ vms,
+                              float* __restrict__ m_prev, uint8_t* __restrict__ valid,
+                              float* __restrict__ user_step_margin, const int32_t* __restrict__ ids,
+                              int32_t* __restrict__ prev_ids, uint8_t* __restrict__ ids_valid,
+                              int32_t* __restrict__ delta) {
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
-  const float* sig = (prm->margin_kind == VLAC_MARGIN_LOGIT ? gaps : margins) + (size_t)b * D;
+  const float* sig = (prm->margin_kind == VLAC_MARGIN_LOGIT   ? gaps
+                      : prm->margin_kind == VLAC_MARGIN_VOCAB ? vms
+                                                              : margins) +
+                     (size_t)b * D;
+  int dl = 0;
+  for (int a = 0; a < D; ++a) {
+    const int v = ids[(size_t)b * D + a];
+    if (ids_valid[b]) dl += abs(v - prev_ids[(size_t)b * D + a]);
+    prev_ids[(size_t)b * D + a] = v;
+  }
+  ids_valid[b] = 1;
+  delta[b] = dl;
   float m;
   if (prm->reduction == VLAC_REDUCE_MIN) {
     m = sig[0];
@@ -417,10 +432,11 @@ void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int 
   launch_k(decode_embed_kernel<T>, dim3(B), dim3(256), 0, st, d, D, P, hidden, vocab, n_bins, tok_emb, ids, forced,
            prm, Xd, idx_dec, ssq_out, err);
 }
-void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps, float* m_prev,
-                   uint8_t* valid, float* user_step_margin, cudaStream_t st) {
-  launch_k(finish_kernel, dim3((B + 63) / 64), dim3(64), 0, st, B, D, prm, margins, gaps, m_prev, valid,
-           user_step_margin);
+void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps, const float* vms,
+                   float* m_prev, uint8_t* valid, float* user_step_margin, const int32_t* ids, int32_t* prev_ids,
+                   uint8_t* ids_valid, int32_t* delta, cudaStream_t st) {
+  launch_k(finish_kernel, dim3((B + 63) / 64), dim3(64), 0, st, B, D, prm, margins, gaps, vms, m_prev, valid,
+           user_step_margin, ids, prev_ids, ids_valid, delta);
 }
 
 #define VLAC_INST(T)                                                                                              \

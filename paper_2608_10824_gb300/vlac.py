@@ -23,7 +23,7 @@ VLAC_OK = 0
 ERRORS = {-1: "VLAC_ERR_INVALID_ARG", -2: "VLAC_ERR_CUDA", -3: "VLAC_ERR_OOM", -4: "VLAC_ERR_TIMEOUT",
           -5: "VLAC_ERR_DEVICE_CHECK", -6: "VLAC_ERR_STATE", -7: "VLAC_ERR_UNSUPPORTED"}
 F32, BF16 = 0, 1
-MARGIN_PROB, MARGIN_LOGIT = 0, 1
+MARGIN_PROB, MARGIN_LOGIT, MARGIN_VOCAB = 0, 1, 2
 REDUCE_DEFAULT, REDUCE_MEAN, REDUCE_MIN = -1, 0, 1
 
 
@@ -62,7 +62,7 @@ class StepOpts(C.Structure):
 class StepOut(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in (
         "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
-        "static_mask", "idx", "M")]
+        "static_mask", "idx", "M", "entropy", "vocab_margin", "action_delta")]
 
 
 EXPORTS = ["vlac_create", "vlac_destroy", "vlac_cache_bytes", "vlac_cache_init", "vlac_cache_destroy",
@@ -182,7 +182,9 @@ class Context:
         }
         shapes = {"gate_auto": ((batch,), torch.uint8), "logits": ((batch, D, d.n_bins), torch.float32),
                   "static_mask": ((batch, d.n_visual), torch.uint8), "idx": ((batch, d.pass_len), torch.int32),
-                  "M": ((batch, d.n_layers), torch.int32)}
+                  "M": ((batch, d.n_layers), torch.int32),
+                  "entropy": ((batch, D), torch.float32), "vocab_margin": ((batch, D), torch.float32),
+                  "action_delta": ((batch,), torch.int32)}
         for k in want:
             shp, dt = shapes[k]
             out[k] = torch.zeros(shp, dtype=dt, device=dev)
@@ -201,7 +203,7 @@ class Context:
             out = self.alloc_outputs(cache.batch, want)
         so = StepOut(*[_ptr(out.get(k)) for k in (
             "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
-            "static_mask", "idx", "M")])
+            "static_mask", "idx", "M", "entropy", "vocab_margin", "action_delta")])
         opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids))
         rc = lib().vlac_step(self._h, cache._h, frames.data_ptr(), prompt.data_ptr(), _ptr(proprio),
                              Rational(int(tau_sim[0]), int(tau_sim[1])), float(tau_margin),

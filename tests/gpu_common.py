@@ -28,6 +28,11 @@ ID_EXEMPT_MARGIN = 1e-3
 # twice the bar.  The deep tests exempt exactly those ids, and require the
 # GPU's id to be the first maximum of the GPU's own logits.
 FLAG_TIE = 1e-4
+# Entropy of the bin softmax: H moves by at most max_j |l_j - E_p[l]| per unit
+# of logit error, about 5 for these models' logit spread, so the bar is five
+# times the logit bar; the library's entropy must also match the entropy of
+# its own logits to fp32 rounding.
+ENTROPY_FACTOR = 5.0
 
 SMALL = {
     # bf16 path (tcgen05 GEMMs), head_dim 128, autoregressive decode
@@ -76,15 +81,20 @@ class Lockstep:
         self.gc = self.ctx.new_cache(batch)
         self.torch = torch
         self.prev_m = None
+        self.prev_ids = None
         self.log = []
         self.logit_tol = logit_tol
 
-    def step(self, frames, prompt, proprio, tau_sim, tau_m, permille, margin_kind=0, force_branch=None):
+    def step(self, frames, prompt, proprio, tau_sim, tau_m, permille, margin_kind=0, force_branch=None,
+             want_vocab=False):
+        """want_vocab: also the whole-vocabulary margin (always with margin kind 2)."""
         torch = self.torch
         d, B = self.d, self.B
+        vocab = want_vocab or margin_kind == 2
         o = self.orc.step(self.oc, frames, prompt, proprio, tau_sim=tau_sim, tau_margin=tau_m,
                           permille=permille, margin_kind=margin_kind,
-                          gate_override=None if force_branch is None else np.full(B, force_branch, np.int8))
+                          gate_override=None if force_branch is None else np.full(B, force_branch, np.int8),
+                          want_vocab_margin=vocab)
         # branch: free-running, except where the oracle's m_{t-1} sits in the tie zone
         ovr = np.full(B, -1, np.int8) if force_branch is None else np.full(B, force_branch, np.int8)
         if self.prev_m is not None and force_branch is None:
@@ -97,12 +107,15 @@ class Lockstep:
             tau_sim=tau_sim, tau_margin=tau_m, permille=permille, margin_kind=margin_kind,
             gate_override=torch.from_numpy(ovr).cuda(),
             forced_ids=torch.from_numpy(o["action_ids"].astype(np.int32)).cuda(),
-            want=("gate_auto", "logits", "static_mask", "idx", "M"))
+            want=("gate_auto", "logits", "static_mask", "idx", "M", "entropy", "action_delta")
+            + (("vocab_margin",) if vocab else ()))
         torch.cuda.synchronize()
         g = {k: v.cpu().numpy() for k, v in g.items()}
         err = self.ctx.sync_error()
         assert err == 0, f"device error {err}"
         rep = compare(d, o, g, self.prev_m, tau_m, self.logit_tol)
+        rep.update(compare_signals(d, o, g, self.prev_ids, self.logit_tol))
+        self.prev_ids = (o["action_ids"].copy(), g["action_ids"].copy())
         self.prev_m = o["step_margin"].copy()
         self.log.append(rep)
         return o, g, rep
@@ -134,3 +147,27 @@ def compare(d, o, g, prev_m, tau_m, logit_tol=None):
     np.testing.assert_allclose(g["margins"], o["margins"], atol=max(tol * 0.05, 1e-6), rtol=0.05)
     return {"max_logit_diff": float(diff.max()), "id_mismatch": int(mism.sum()),
             "id_exempt": int(exempt.sum()), "recomputed": o["recomputed"].tolist()}
+
+
+def compare_signals(d, o, g, prev_ids, logit_tol=None):
+    """Entropy within ENTROPY_FACTOR x the logit bar of the oracle's (and
+    within fp32 rounding of the entropy of the library's own logits); the
+    whole-vocabulary margin like the bin margin; the action delta exact for
+    every sequence whose ids agree with the oracle's on this and the
+    previous step."""
+    tol = LOGIT_TOL[d.dtype] if logit_tol is None else logit_tol
+    gl = g["logits"].astype(np.float64)
+    p = np.exp(gl - gl.max(-1, keepdims=True))
+    z = p.sum(-1, keepdims=True)
+    own = np.log(z[..., 0]) - (p * (gl - gl.max(-1, keepdims=True))).sum(-1) / z[..., 0]
+    np.testing.assert_allclose(g["entropy"], own, atol=1e-4, rtol=1e-5, err_msg="entropy vs own logits")
+    ediff = float(np.max(np.abs(g["entropy"] - o["entropy"])))
+    assert ediff <= ENTROPY_FACTOR * tol, f"entropy differs by {ediff:.3e}"
+    if "vocab_margin" in g and "vocab_margin" in o:
+        np.testing.assert_allclose(g["vocab_margin"], o["vocab_margin"], atol=max(tol * 0.05, 1e-6), rtol=0.05,
+                                   err_msg="vocabulary margin")
+    same = (g["action_ids"] == o["action_ids"]).all(-1)
+    if prev_ids is not None:
+        same &= (prev_ids[0] == prev_ids[1]).all(-1)
+    np.testing.assert_array_equal(g["action_delta"][same], o["action_delta"][same], err_msg="action delta")
+    return {"entropy_diff": ediff, "delta_compared": int(same.sum())}
