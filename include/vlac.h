@@ -44,6 +44,8 @@ extern "C" {
 
 #define VLAC_MARGIN_PROB 0  /* gate signal p1 - p2 of the softmax over the action bins (Eq. 1) */
 #define VLAC_MARGIN_LOGIT 1 /* gate signal l1 - l2, the top-2 logit gap */
+#define VLAC_MARGIN_VOCAB 2 /* gate signal p1 - p2 of the softmax over the whole vocabulary (Sec. IV-A);
+                               reads every LM-head row per action token */
 #define VLAC_REDUCE_DEFAULT (-1) /* mean for autoregressive decode (Eq. 1), min for a parallel block */
 #define VLAC_REDUCE_MEAN 0
 #define VLAC_REDUCE_MIN 1
@@ -82,7 +84,8 @@ typedef struct vlac_weights {
   const void* const* w_up;      /* [ffn][hidden] */
   const void* const* w_down;    /* [hidden][ffn] */
   const void* final_norm;       /* [hidden] */
-  const void* lm_head;          /* [vocab][hidden]; only rows vocab-n_bins .. vocab-1 are read */
+  const void* lm_head;          /* [vocab][hidden]; rows vocab-n_bins .. vocab-1 give the action
+                                   bins, the others only the whole-vocabulary margin */
 } vlac_weights;
 
 /* Stage-1 threshold as an exact fraction: a patch is static iff cos > num/den. */
@@ -91,7 +94,7 @@ typedef struct vlac_rational {
 } vlac_rational;
 
 typedef struct vlac_step_opts {
-  int32_t margin_kind;         /* VLAC_MARGIN_PROB (default) or VLAC_MARGIN_LOGIT */
+  int32_t margin_kind;         /* VLAC_MARGIN_PROB (default), VLAC_MARGIN_LOGIT or VLAC_MARGIN_VOCAB */
   int32_t reduction;           /* VLAC_REDUCE_* */
   const int8_t* gate_override; /* device [B]: -1 gate decides, 0 force the cached branch,
                                   1 force the full branch; NULL = gate decides.  An empty
@@ -130,6 +133,11 @@ typedef struct vlac_step_out {
   int32_t* M;           /* optional [B][L] rows recomputed at each layer */
   float* relevance;     /* optional [B][Nv] this step's Stage-2 relevance (0 when Stage 2 is off) */
   uint8_t* relevant;    /* optional [B][Nv] patches Stage 2 kept out of the reusable set this step */
+  float* entropy;       /* optional [B][D] entropy (nats) of each action token's bin softmax (Sec. VI) */
+  float* vocab_margin;  /* optional [B][D] p1 - p2 of the softmax over the whole vocabulary; asking
+                           for it (or for VLAC_MARGIN_VOCAB) reads every LM-head row per token */
+  int32_t* action_delta; /* optional [B] sum over d of |a_t^d - a_{t-1}^d| in bins, 0 on a sequence's
+                            first step and after a reset (Sec. VI) */
 } vlac_step_out;
 
 typedef struct vlac_ctx vlac_ctx;

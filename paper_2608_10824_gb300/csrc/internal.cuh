@@ -329,8 +329,13 @@ template <typename T>
 void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
                          const int32_t* ids, const int32_t* forced, const StepParams* prm, float* Xd,
                          int* idx_dec, float* ssq_out, int* err, cudaStream_t st);
-void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps,
-                   float* m_prev, uint8_t* valid, float* user_step_margin, const uint8_t* active, cudaStream_t st);
+// m_t from the per-token signals (margins, gaps or vocabulary margins vms by
+// prm->margin_kind); also the action delta against prev_ids (kept in the
+// cache, with ids_valid) into delta.  A sequence that sat the step out
+// (prm->has_active, active[b] == 0) keeps its gate state and previous ids.
+void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps, const float* vms,
+                   float* m_prev, uint8_t* valid, float* user_step_margin, const int32_t* ids, int32_t* prev_ids,
+                   uint8_t* ids_valid, int32_t* delta, const uint8_t* active, cudaStream_t st);
 // End of a step: the previous frame of every sequence that stepped becomes
 // this step's frame, and the outputs of the sequences that sat the step out
 // are zeroed (with prm->has_active; active NULL = all stepped).
@@ -341,6 +346,8 @@ struct StepOutputs {
   int32_t *idx, *M;
   float* relevance;   // Stage 2 outputs [B][Nv]
   uint8_t* relevant;
+  float *entropy, *vocab_margin;  // [B][D]
+  int32_t* action_delta;          // [B]
 };
 void launch_commit(int B, int D, int n_bins, int Nv, int S, int L, size_t frame_bytes, const uint8_t* frames,
                    uint8_t* prev, const StepParams* prm, const uint8_t* active, const StepOutputs& o,
@@ -437,9 +444,22 @@ size_t dgemv_stage_bytes();  // bytes of one weight-ring stage of the decode GEM
 template <typename T>
 void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride,
                           int Tc, int pos, float* part, unsigned* counters, T* O, cudaStream_t st);
+// Margin over the whole vocabulary: W the LM-head rows outside the bins
+// ([n_rows][hidden], T), xh scratch for the normed action rows ([rows][hidden],
+// T), vl scratch for their logits ([rows][n_rows] fp32), vm the margins [B][D].
+struct VocabHead {
+  const void* W;
+  int n_rows;
+  void* xh;
+  float* vl;
+  float* vm;
+};
+// Action head of rows_per_seq rows per sequence: bin logits, ids, margins,
+// gaps, entropy (may be NULL) and, with vh, the whole-vocabulary margin.
 template <typename T>
 void launch_head2(const float* X, const int* row_of_seq, size_t x_seq_stride, int rows_per_seq, int B, int hidden,
                   int n_bins, const T* final_norm, const T* head_w, float eps, float* logits_ws, int D, int tok0,
-                  int32_t* ids, float* margins, float* gaps, float* logits, cudaStream_t st);
+                  int32_t* ids, float* margins, float* gaps, float* logits, float* entropy, const VocabHead* vh,
+                  cudaStream_t st);
 
 }  // namespace vlac

@@ -319,19 +319,35 @@ __global__ void decode_embed_kernel(int d, int D, int P, int hidden, int vocab, 
 }
 
 // m_t = mean (Eq. 1) or min of the per-token signals; the cache keeps it for
-// the next step's gate and becomes valid.
+// the next step's gate and becomes valid.  The action delta (Sec. VI) is the
+// L1 distance in bins to the previous step's ids on the sequence.
 __global__ void finish_kernel(int B, int D, const StepParams* __restrict__ prm, const float* __restrict__ margins,
-                              const float* __restrict__ gaps, float* __restrict__ m_prev, uint8_t* __restrict__ valid,
-                              float* __restrict__ user_step_margin, const uint8_t* __restrict__ active) {
+                              const float* __restrict__ gaps, const float* __restrict__ vms,
+                              float* __restrict__ m_prev, uint8_t* __restrict__ valid,
+                              float* __restrict__ user_step_margin, const int32_t* __restrict__ ids,
+                              int32_t* __restrict__ prev_ids, uint8_t* __restrict__ ids_valid,
+                              int32_t* __restrict__ delta, const uint8_t* __restrict__ active) {
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
-  if (prm->has_active && active && !active[b]) {  // sat the step out: the gate state stays
+  if (prm->has_active && active && !active[b]) {  // sat the step out: the gate state and ids stay
     user_step_margin[b] = 0.f;
+    delta[b] = 0;
     return;
   }
-  const float* sig = (prm->margin_kind == VLAC_MARGIN_LOGIT ? gaps : margins) + (size_t)b * D;
+  const float* sig = (prm->margin_kind == VLAC_MARGIN_LOGIT   ? gaps
+                      : prm->margin_kind == VLAC_MARGIN_VOCAB ? vms
+                                                              : margins) +
+                     (size_t)b * D;
+  int dl = 0;
+  for (int a = 0; a < D; ++a) {
+    const int v = ids[(size_t)b * D + a];
+    if (ids_valid[b]) dl += abs(v - prev_ids[(size_t)b * D + a]);
+    prev_ids[(size_t)b * D + a] = v;
+  }
+  ids_valid[b] = 1;
+  delta[b] = dl;
   float m;
   if (prm->reduction == VLAC_REDUCE_MIN) {
     m = sig[0];
@@ -468,10 +484,11 @@ void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int 
   launch_k(decode_embed_kernel<T>, dim3(B), dim3(256), 0, st, d, D, P, hidden, vocab, n_bins, tok_emb, ids, forced,
            prm, Xd, idx_dec, ssq_out, err);
 }
-void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps, float* m_prev,
-                   uint8_t* valid, float* user_step_margin, const uint8_t* active, cudaStream_t st) {
-  launch_k(finish_kernel, dim3((B + 63) / 64), dim3(64), 0, st, B, D, prm, margins, gaps, m_prev, valid,
-           user_step_margin, active);
+void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps, const float* vms,
+                   float* m_prev, uint8_t* valid, float* user_step_margin, const int32_t* ids, int32_t* prev_ids,
+                   uint8_t* ids_valid, int32_t* delta, const uint8_t* active, cudaStream_t st) {
+  launch_k(finish_kernel, dim3((B + 63) / 64), dim3(64), 0, st, B, D, prm, margins, gaps, vms, m_prev, valid,
+           user_step_margin, ids, prev_ids, ids_valid, delta, active);
 }
 
 // Grid (chunks, B): sequence b's previous frame becomes this step's frame (16-byte
@@ -500,6 +517,8 @@ __global__ void commit_kernel(int D, int n_bins, int Nv, int S, int L, size_t fr
     o.ids[(size_t)b * D + i] = 0;
     o.margins[(size_t)b * D + i] = 0.f;
     o.gaps[(size_t)b * D + i] = 0.f;
+    if (o.entropy) o.entropy[(size_t)b * D + i] = 0.f;
+    if (o.vocab_margin) o.vocab_margin[(size_t)b * D + i] = 0.f;
   }
   for (size_t i = tid; i < (size_t)D * n_bins; i += nth) o.logits[(size_t)b * D * n_bins + i] = 0.f;
   for (size_t i = tid; i < (size_t)Nv; i += nth) o.mask[(size_t)b * Nv + i] = 0;

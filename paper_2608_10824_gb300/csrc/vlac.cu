@@ -57,6 +57,7 @@ struct vlac_ctx {
   // weights
   char* wmem = nullptr;
   void *tok_emb, *patch_w, *proprio_w, *action_emb, *final_norm, *head_w;
+  void* head_full;  // the whole LM head [vocab][hidden]; head_w is its last n_bins rows
   std::vector<void*> attn_norm, ffn_norm, wqkv, wo, wgu, wd;
   float *rope_cos, *rope_sin;
   // TMA descriptors (bf16 only)
@@ -97,6 +98,11 @@ struct vlac_ctx {
   float* rel_part;      // Stage-2 relevance per (sequence, head) [B][n_heads][Nv]
   bool s2_on = false;   // this step measures and applies Stage 2
   int s2_layer = 0;
+  float *o_entropy, *o_vm;  // per action token: bin-softmax entropy, whole-vocabulary margin
+  int32_t* o_delta;         // per sequence: action delta
+  void* vh_rows;            // whole-vocabulary margin: normed action rows [rows][hidden] (T)
+  float* vh_logits;         // and their logits over the non-bin rows [rows][vocab - n_bins]
+  bool vm_on = false;       // this step computes the whole-vocabulary margin
   cudaStream_t cap_stream = nullptr;
   bool use_graph = true;
   bool fatal = false;  // a launch was refused for exceeding a workspace buffer
@@ -121,13 +127,15 @@ struct vlac_cache {
   cudaGraphExec_t gexec = nullptr;
   int eager_steps = 0;
   uint64_t graph_launches = 0;
-  int graph_sig = 0;  // the Stage-2 layout the graph was captured with (0 = off, 1 + layer)
+  int graph_sig = 0;  // what the graph was captured with: Stage 2 (0 off, 1 + layer) * 2 + the vocabulary margin
   void *K, *V;
   float* H;
   uint8_t *prev, *valid;
   float* m_prev;
   float* rel;          // [B][Nv] the last step's Stage-2 relevance
   uint8_t* rel_valid;  // [B] rel holds one
+  int32_t* prev_ids;   // [B][n_action] the previous step's action bins
+  uint8_t* ids_valid;  // [B] prev_ids holds them
   size_t kv_seq_stride, h_seq_stride;  // elements per sequence
 };
 
@@ -255,7 +263,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     wc.take(c->proprio_w, Hd * std::max(d.proprio_dim, 1) * E, base);
     wc.take(c->action_emb, (size_t)d.n_action * Hd * E, base);
     wc.take(c->final_norm, Hd * E, base);
-    wc.take(c->head_w, (size_t)d.n_bins * Hd * E, base);
+    wc.take(c->head_full, (size_t)d.vocab * Hd * E, base);
+    if (base) c->head_w = static_cast<char*>(c->head_full) + (size_t)(d.vocab - d.n_bins) * Hd * E;
     c->attn_norm.resize(L); c->ffn_norm.resize(L); c->wqkv.resize(L); c->wo.resize(L); c->wgu.resize(L); c->wd.resize(L);
     for (size_t l = 0; l < L; ++l) {
       wc.take(c->attn_norm[l], Hd * E, base);
@@ -290,8 +299,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (d.proprio_dim) ok = ok && cp(c->proprio_w, w->proprio_w, Hd * d.proprio_dim * E);
   if (d.parallel) ok = ok && cp(c->action_emb, w->action_emb, (size_t)d.n_action * Hd * E);
   ok = ok && cp(c->final_norm, w->final_norm, Hd * E);
-  ok = ok && cp(c->head_w, static_cast<const char*>(w->lm_head) + (size_t)(d.vocab - d.n_bins) * Hd * E,
-                (size_t)d.n_bins * Hd * E);
+  ok = ok && cp(c->head_full, w->lm_head, (size_t)d.vocab * Hd * E);
   for (size_t l = 0; l < L && ok; ++l) {
     char* qkv = static_cast<char*>(c->wqkv[l]);
     char* gu = static_cast<char*>(c->wgu[l]);
@@ -475,6 +483,12 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->o_rel, Bm * c->Nv * 4, base);
     sc.take(c->o_relevant, Bm * c->Nv, base);
     sc.take(c->rel_part, Bm * d.n_heads * c->Nv * 4, base);
+    sc.take(c->o_entropy, Bm * d.n_action * 4, base);
+    sc.take(c->o_vm, Bm * d.n_action * 4, base);
+    sc.take(c->o_delta, Bm * 4, base);
+    const size_t head_rows = Bm * (d.parallel ? d.n_action : 1);
+    sc.take(c->vh_rows, head_rows * Hd * E, base);
+    sc.take(c->vh_logits, head_rows * std::max(d.vocab - d.n_bins, 1) * 4, base);
   };
   plan_s(nullptr);
   if (cudaMalloc(&c->wsmem, sc.off) != cudaSuccess) {
@@ -538,8 +552,9 @@ static size_t cache_layout(const vlac_ctx* c, int B, char* base, vlac_cache* k) 
   void* K;
   void* V;
   float* H;
-  uint8_t *prev, *valid, *rel_valid;
+  uint8_t *prev, *valid, *rel_valid, *ids_valid;
   float *m_prev, *rel;
+  int32_t* prev_ids;
   const size_t kv = (size_t)d.n_layers * d.n_heads * c->Tc * d.head_dim;
   const size_t hs = (size_t)d.n_layers * c->S * d.hidden;
   cv.take(K, B * kv * c->esz, base);
@@ -550,9 +565,12 @@ static size_t cache_layout(const vlac_ctx* c, int B, char* base, vlac_cache* k) 
   cv.take(valid, (size_t)B, base);
   cv.take(rel, (size_t)B * c->Nv * 4, base);
   cv.take(rel_valid, (size_t)B, base);
+  cv.take(prev_ids, (size_t)B * d.n_action * 4, base);
+  cv.take(ids_valid, (size_t)B, base);
   if (k) {
     k->K = K; k->V = V; k->H = H; k->prev = prev; k->m_prev = m_prev; k->valid = valid;
     k->rel = rel; k->rel_valid = rel_valid;
+    k->prev_ids = prev_ids; k->ids_valid = ids_valid;
     k->kv_seq_stride = kv;
     k->h_seq_stride = hs;
   }
@@ -598,9 +616,11 @@ extern "C" int vlac_reset(vlac_cache* k, int seq, void* stream) {
   if (seq < 0) {
     CK(cudaMemsetAsync(k->valid, 0, (size_t)k->B, st));
     CK(cudaMemsetAsync(k->rel_valid, 0, (size_t)k->B, st));
+    CK(cudaMemsetAsync(k->ids_valid, 0, (size_t)k->B, st));
   } else {
     CK(cudaMemsetAsync(k->valid + seq, 0, 1, st));
     CK(cudaMemsetAsync(k->rel_valid + seq, 0, 1, st));
+    CK(cudaMemsetAsync(k->ids_valid + seq, 0, 1, st));
   }
   return VLAC_OK;
 }
@@ -735,7 +755,11 @@ void prefix_layer(vlac_ctx* c, const Rows& rl, const int* off_prev, int B, int l
 template <typename T>
 int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   vlac_step_out outv{c->o_ids,   c->o_margins, c->o_gaps, c->o_recomputed, c->o_step_margin, c->o_gate_auto,
-                     c->o_logits, c->o_mask,    c->o_idx,  c->o_M,         c->o_rel,         c->o_relevant};
+                     c->o_logits, c->o_mask,    c->o_idx,  c->o_M,         c->o_rel,         c->o_relevant,
+                     c->o_entropy, c->o_vm,    c->o_delta};
+  VocabHead vh{c->head_full, c->d.vocab - c->d.n_bins, c->vh_rows, c->vh_logits, c->o_vm};
+  const VocabHead* vhp = c->vm_on ? &vh : nullptr;
+  const int head_launches = c->vm_on ? (vh.n_rows ? 5 : 4) : 2;
   const vlac_step_out* out = &outv;
   const uint8_t* frames = c->in_frames;
   const int32_t* prompt = c->in_prompt;
@@ -806,9 +830,9 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
     ProfScope ps_(c, VLAC_PROF_HEAD, 0, st);
     launch_head2<T>(c->X, c->emit_slot, (size_t)S * Hd, d.parallel ? D : 1, B, Hd, nb, W(c->final_norm),
                     W(c->head_w), eps, c->logits_ws, D, 0, out->action_ids, out->margins, out->logit_gap, out->logits,
-                    st);
+                    out->entropy, vhp, st);
   }
-  c->launches += 2;
+  c->launches += head_launches;
 
   if (!d.parallel) {
     // autoregressive decode: one row per sequence, fused GEMVs
@@ -967,21 +991,22 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
       {
         ProfScope ps_(c, VLAC_PROF_HEAD, 0, st);
         launch_head2<T>(c->Xd, nullptr, Hd, 1, B, Hd, nb, W(c->final_norm), W(c->head_w), eps, c->logits_ws, D, a,
-                        out->action_ids, out->margins, out->logit_gap, out->logits, st);
+                        out->action_ids, out->margins, out->logit_gap, out->logits, out->entropy, vhp, st);
       }
-      c->launches += 2;
+      c->launches += head_launches;
     }
   }
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
-    launch_finish(B, D, c->prm, out->margins, out->logit_gap, k->m_prev, k->valid, out->step_margin, c->in_active,
-                  st);
+    launch_finish(B, D, c->prm, out->margins, out->logit_gap, out->vocab_margin, k->m_prev, k->valid, out->step_margin,
+                  out->action_ids, k->prev_ids, k->ids_valid, out->action_delta, c->in_active, st);
   }
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     const StepOutputs so{out->action_ids, out->margins,   out->logit_gap,   out->logits, out->step_margin,
                          out->recomputed, out->gate_auto, out->static_mask, out->idx,    out->M,
-                         out->relevance,  out->relevant};
+                         out->relevance,  out->relevant,  out->entropy,     out->vocab_margin,
+                         out->action_delta};
     launch_commit(B, D, nb, c->Nv, S, L, (size_t)d.n_views * d.img_h * d.img_w * 3, frames, k->prev, c->prm,
                   c->in_active, so, st);
   }
@@ -1000,9 +1025,10 @@ int run_body(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
 // the second captures the body into a graph, which every later step replays.
 int run_step(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   if (!c->use_graph || c->prof_on) return run_body(c, k, st);
-  const int sig = c->s2_on ? 1 + c->s2_layer : 0;
+  const int sig = (c->s2_on ? 1 + c->s2_layer : 0) * 2 + (c->vm_on ? 1 : 0);
   if (k->gexec && k->graph_sig != sig) {
-    // Stage 2 switched on or off, or moved to another layer: the launch list
+    // Stage 2 or the whole-vocabulary margin switched on or off, or Stage 2
+    // moved to another layer: the launch list
     // differs, so the graph is captured again (after one eager step)
     cudaGraphExecDestroy(k->gexec);
     cudaGraphDestroy(k->graph);
@@ -1058,7 +1084,7 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   }
   int mk = opts ? opts->margin_kind : VLAC_MARGIN_PROB;
   int red = opts ? opts->reduction : VLAC_REDUCE_DEFAULT;
-  if (mk != VLAC_MARGIN_PROB && mk != VLAC_MARGIN_LOGIT) return VLAC_ERR_INVALID_ARG;
+  if (mk != VLAC_MARGIN_PROB && mk != VLAC_MARGIN_LOGIT && mk != VLAC_MARGIN_VOCAB) return VLAC_ERR_INVALID_ARG;
   if (red == VLAC_REDUCE_DEFAULT) red = c->d.parallel ? VLAC_REDUCE_MIN : VLAC_REDUCE_MEAN;
   if (red != VLAC_REDUCE_MEAN && red != VLAC_REDUCE_MIN) return VLAC_ERR_INVALID_ARG;
   p.tau_num = tau_sim.num;
@@ -1103,6 +1129,7 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   c->launches += 1;
   c->s2_on = p.s2_top_k > 0;
   c->s2_layer = p.s2_layer;
+  c->vm_on = mk == VLAC_MARGIN_VOCAB || out->vocab_margin != nullptr;
   int rc = run_step(c, k, st);
   if (rc) return rc;
   CopyList o{};
@@ -1118,6 +1145,9 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   add(o, c->o_M, out->M, (size_t)B * d.n_layers * 4);
   add(o, c->o_rel, out->relevance, (size_t)B * c->Nv * 4);
   add(o, c->o_relevant, out->relevant, (size_t)B * c->Nv);
+  add(o, c->o_entropy, out->entropy, (size_t)B * D * 4);
+  if (c->vm_on) add(o, c->o_vm, out->vocab_margin, (size_t)B * D * 4);
+  add(o, c->o_delta, out->action_delta, (size_t)B * 4);
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_copies(o, st);

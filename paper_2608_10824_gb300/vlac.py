@@ -23,7 +23,7 @@ VLAC_OK = 0
 ERRORS = {-1: "VLAC_ERR_INVALID_ARG", -2: "VLAC_ERR_CUDA", -3: "VLAC_ERR_OOM", -4: "VLAC_ERR_TIMEOUT",
           -5: "VLAC_ERR_DEVICE_CHECK", -6: "VLAC_ERR_STATE", -7: "VLAC_ERR_UNSUPPORTED"}
 F32, BF16 = 0, 1
-MARGIN_PROB, MARGIN_LOGIT = 0, 1
+MARGIN_PROB, MARGIN_LOGIT, MARGIN_VOCAB = 0, 1, 2
 REDUCE_DEFAULT, REDUCE_MEAN, REDUCE_MIN = -1, 0, 1
 
 
@@ -63,7 +63,7 @@ class StepOpts(C.Structure):
 class StepOut(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in (
         "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
-        "static_mask", "idx", "M", "relevance", "relevant")]
+        "static_mask", "idx", "M", "relevance", "relevant", "entropy", "vocab_margin", "action_delta")]
 
 
 EXPORTS = ["vlac_create", "vlac_destroy", "vlac_cache_bytes", "vlac_cache_init", "vlac_cache_destroy",
@@ -189,7 +189,9 @@ class Context:
                   "static_mask": ((batch, d.n_visual), torch.uint8), "idx": ((batch, d.pass_len), torch.int32),
                   "M": ((batch, d.n_layers), torch.int32),
                   "relevance": ((batch, d.n_visual), torch.float32),
-                  "relevant": ((batch, d.n_visual), torch.uint8)}
+                  "relevant": ((batch, d.n_visual), torch.uint8),
+                  "entropy": ((batch, D), torch.float32), "vocab_margin": ((batch, D), torch.float32),
+                  "action_delta": ((batch,), torch.int32)}
         for k in want:
             shp, dt = shapes[k]
             out[k] = torch.zeros(shp, dtype=dt, device=dev)
@@ -212,7 +214,7 @@ class Context:
             out = self.alloc_outputs(cache.batch, want)
         so = StepOut(*[_ptr(out.get(k)) for k in (
             "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
-            "static_mask", "idx", "M", "relevance", "relevant")])
+            "static_mask", "idx", "M", "relevance", "relevant", "entropy", "vocab_margin", "action_delta")])
         if s2_layer is None:
             s2_layer = d.n_layers // 2
         opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids), _ptr(active), int(s2_top_k),

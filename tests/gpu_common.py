@@ -33,6 +33,11 @@ FLAG_TIE = 1e-4
 # in fp64.  A removal-set difference is allowed only for patches whose oracle
 # relevance lies within twice this of the oracle's k-th / (k+1)-th midpoint.
 REL_TOL = {"bf16": 1e-4, "f32": 1e-5}
+# Entropy of the bin softmax: H moves by at most max_j |l_j - E_p[l]| per unit
+# of logit error, about 5 for these models' logit spread, so the bar is five
+# times the logit bar; the library's entropy must also match the entropy of
+# its own logits to fp32 rounding.
+ENTROPY_FACTOR = 5.0
 
 SMALL = {
     # bf16 path (tcgen05 GEMMs), head_dim 128, autoregressive decode
@@ -82,23 +87,26 @@ class Lockstep:
         self.torch = torch
         self.prev_m = None
         self.prev_rel = None
+        self.prev_ids = None
         self.log = []
         self.logit_tol = logit_tol
 
     def step(self, frames, prompt, proprio, tau_sim, tau_m, permille, margin_kind=0, force_branch=None,
-             active=None, s2_top_k=0, s2_layer=None, s2_lockstep=True):
+             active=None, s2_top_k=0, s2_layer=None, s2_lockstep=True, want_vocab=False):
         """active: uint8 [B], 0 = the sequence sits the step out (both sides).
         s2_top_k > 0: Stage 2 on both sides; with s2_lockstep the library
-        applies the oracle's removal set (its own is still compared)."""
+        applies the oracle's removal set (its own is still compared).
+        want_vocab: also the whole-vocabulary margin (always with margin kind 2)."""
         torch = self.torch
         d, B = self.d, self.B
         act = None if active is None else np.ascontiguousarray(active, np.uint8)
+        vocab = want_vocab or margin_kind == 2
         if s2_layer is None:
             s2_layer = d.n_layers // 2
         o = self.orc.step(self.oc, frames, prompt, proprio, tau_sim=tau_sim, tau_margin=tau_m,
                           permille=permille, margin_kind=margin_kind,
                           gate_override=None if force_branch is None else np.full(B, force_branch, np.int8),
-                          active=act, s2_top_k=s2_top_k, s2_layer=s2_layer)
+                          active=act, s2_top_k=s2_top_k, s2_layer=s2_layer, want_vocab_margin=vocab)
         # branch: free-running, except where the oracle's m_{t-1} sits in the tie zone
         ovr = np.full(B, -1, np.int8) if force_branch is None else np.full(B, force_branch, np.int8)
         if self.prev_m is not None and force_branch is None:
@@ -111,7 +119,8 @@ class Lockstep:
             tau_sim=tau_sim, tau_margin=tau_m, permille=permille, margin_kind=margin_kind,
             gate_override=torch.from_numpy(ovr).cuda(),
             forced_ids=torch.from_numpy(o["action_ids"].astype(np.int32)).cuda(),
-            want=("gate_auto", "logits", "static_mask", "idx", "M", "relevance", "relevant"),
+            want=("gate_auto", "logits", "static_mask", "idx", "M", "relevance", "relevant", "entropy", "action_delta")
+            + (("vocab_margin",) if vocab else ()),
             active=None if act is None else torch.from_numpy(act).cuda(),
             s2_top_k=s2_top_k, s2_layer=s2_layer,
             s2_forced=(torch.from_numpy(np.ascontiguousarray(o["relevant"])).cuda()
@@ -121,7 +130,10 @@ class Lockstep:
         err = self.ctx.sync_error()
         assert err == 0, f"device error {err}"
         rep = compare(d, o, g, self.prev_m, tau_m, self.logit_tol)
-        rep.update(compare_stage2(d, o, g, s2_top_k, self.prev_rel))
+        stepped = np.ones(B, bool) if act is None else act != 0
+        rep.update(compare_stage2(d, o, g, s2_top_k, self.prev_rel, stepped))
+        rep.update(compare_signals(d, o, g, self.prev_ids, self.logit_tol, stepped))
+        self.prev_ids = (o["action_ids"].copy(), g["action_ids"].copy())
         rel = o["relevance"].copy() if s2_top_k > 0 else None
         m = o["step_margin"].copy()
         if act is not None and self.prev_m is not None:  # a paused sequence keeps its m_{t-1}
@@ -162,7 +174,7 @@ def compare(d, o, g, prev_m, tau_m, logit_tol=None):
             "id_exempt": int(exempt.sum()), "recomputed": o["recomputed"].tolist()}
 
 
-def compare_stage2(d, o, g, top_k, prev_rel):
+def compare_stage2(d, o, g, top_k, prev_rel, stepped=None):
     """Stage 2: this step's relevance within REL_TOL of the oracle's (relative
     to the sequence's largest), and the removal set the library decided from
     its previous relevance equal to the oracle's except inside the tie band
@@ -173,6 +185,9 @@ def compare_stage2(d, o, g, top_k, prev_rel):
     tol = REL_TOL[d.dtype]
     worst, diffs = 0.0, 0
     for b in range(o["relevance"].shape[0]):
+        if stepped is not None and not stepped[b]:  # sat the step out: both sides return zeros
+            assert not g["relevance"][b].any() and not g["relevant"][b].any()
+            continue
         scale = float(np.max(o["relevance"][b]))
         err = float(np.max(np.abs(g["relevance"][b].astype(np.float64) - o["relevance"][b]))) / scale
         assert err <= tol, f"relevance of sequence {b} differs by {err:.3e} (relative) > {tol}"
@@ -187,3 +202,33 @@ def compare_stage2(d, o, g, top_k, prev_rel):
             assert not outside.any(), f"removal set differs outside the tie band: {np.flatnonzero(outside)}"
             diffs += int(bad.sum())
     return {"rel_diff": worst, "removal_diffs": diffs}
+def compare_signals(d, o, g, prev_ids, logit_tol=None, stepped=None):
+    """Entropy within ENTROPY_FACTOR x the logit bar of the oracle's (and
+    within fp32 rounding of the entropy of the library's own logits); the
+    whole-vocabulary margin like the bin margin; the action delta exact for
+    every sequence whose ids agree with the oracle's on this and the
+    previous step."""
+    tol = LOGIT_TOL[d.dtype] if logit_tol is None else logit_tol
+    if stepped is not None and not stepped.all():  # sequences that sat the step out return zeros
+        assert not g["entropy"][~stepped].any() and not g["action_delta"][~stepped].any()
+        if not stepped.any():
+            return {"entropy_diff": 0.0, "delta_compared": 0}
+        o = {k: (v[stepped] if isinstance(v, np.ndarray) and v.shape[:1] == stepped.shape else v) for k, v in o.items()}
+        g = {k: (v[stepped] if isinstance(v, np.ndarray) and v.shape[:1] == stepped.shape else v) for k, v in g.items()}
+        if prev_ids is not None:
+            prev_ids = (prev_ids[0][stepped], prev_ids[1][stepped])
+    gl = g["logits"].astype(np.float64)
+    p = np.exp(gl - gl.max(-1, keepdims=True))
+    z = p.sum(-1, keepdims=True)
+    own = np.log(z[..., 0]) - (p * (gl - gl.max(-1, keepdims=True))).sum(-1) / z[..., 0]
+    np.testing.assert_allclose(g["entropy"], own, atol=1e-4, rtol=1e-5, err_msg="entropy vs own logits")
+    ediff = float(np.max(np.abs(g["entropy"] - o["entropy"])))
+    assert ediff <= ENTROPY_FACTOR * tol, f"entropy differs by {ediff:.3e}"
+    if "vocab_margin" in g and "vocab_margin" in o:
+        np.testing.assert_allclose(g["vocab_margin"], o["vocab_margin"], atol=max(tol * 0.05, 1e-6), rtol=0.05,
+                                   err_msg="vocabulary margin")
+    same = (g["action_ids"] == o["action_ids"]).all(-1)
+    if prev_ids is not None:
+        same &= (prev_ids[0] == prev_ids[1]).all(-1)
+    np.testing.assert_array_equal(g["action_delta"][same], o["action_delta"][same], err_msg="action delta")
+    return {"entropy_diff": ediff, "delta_compared": int(same.sum())}
