@@ -248,8 +248,8 @@ int vlac_prof_read(vlac_ctx* ctx, int kind, double* total_ms, uint64_t* launches
 
 /* Allocation-free selection step.  The paper has no counterpart of this call:
  * it exists for callers that cannot allocate device memory when they run it
- * -- code inside a CUDA stream capture, real-time control loops whose memory
- * is fixed up front, host frameworks that own every device allocation.  It
+ * -- real-time control loops whose memory is fixed up front, host frameworks
+ * that own every device allocation and forbid a library its own.  It
  * runs the same kernels as vlac_step's selection (Stage-1 exact patch
  * similarity, the gate on m_prev < tau_margin or gate_override, the Stage-3
  * recompute order) without a context and without allocating: its scratch is
@@ -266,8 +266,10 @@ int vlac_prof_read(vlac_ctx* ctx, int kind, double* total_ms, uint64_t* launches
  *   gate_override:  device [batch] int8 (-1 gate, 0 cached, 1 full) or NULL
  *   outputs (device): static_mask [batch][Nv], idx [batch][S], M [batch][n_layers],
  *                     recomputed [batch]
- * Returns VLAC_ERR_INVALID_ARG for bad arguments and when the call needs more
- * than the fixed scratch: batch x visual patches must stay within 20,000. */
+ * Returns VLAC_ERR_INVALID_ARG for bad arguments and VLAC_ERR_UNSUPPORTED
+ * when valid dims need more than the fixed scratch: batch x visual patches
+ * must stay within 20,000.  VLAC_ERR_CUDA when a launch fails (only this
+ * call's launches are checked). */
 int vlac_select_noalloc(const vlac_dims* d, int batch, const uint8_t* frames, const uint8_t* prev_frames,
                         const uint8_t* valid, const float* m_prev, vlac_rational tau_sim, float tau_margin,
                         const uint16_t* reuse_permille, const int8_t* gate_override, uint8_t* static_mask,

@@ -254,10 +254,11 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 }
 
 // Launch with optional programmatic stream serialization (the kernel may
-// start while its predecessor drains; it must call pdl_wait()).
+// start while its predecessor drains; it must call pdl_wait()).  Returns the
+// launch's own status.
 extern bool g_pdl;
 template <typename... KArgs, typename... Args>
-inline void launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args) {
+inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;
@@ -268,7 +269,7 @@ inline void launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sme
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = g_pdl ? 1 : 0;
-  cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
 }  // namespace vlac
@@ -278,7 +279,7 @@ namespace vlac {
 
 int check_dims(const vlac_dims* d);  // VLAC_OK or the error vlac_create would return
 
-void launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid,
+cudaError_t launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid,
                         const StepParams* prm, int B, int n_views, int img_h, int img_w, int patch,
                         int3* stats, uint8_t* mask, uint8_t* user_mask, cudaStream_t st);
 // Stage 2 state (all NULL = Stage 2 unavailable): rel [B][Nv] the previous
@@ -286,7 +287,7 @@ void launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_
 // step with Stage 2 off); s2_forced [B][Nv] (with prm->has_s2_forced) is
 // applied instead of the kernel's own removal set; relevant [B][Nv] receives
 // the own set and rel_out [B][Nv] is zeroed on a step with Stage 2 off.
-void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
+cudaError_t launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
                    const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
                    int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
                    uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
@@ -366,7 +367,7 @@ struct CopyList {
   CopySpan span[kMaxSpans];
   int n;
 };
-void launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st);
+cudaError_t launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st);
 // One-layer entry: idx[i] = pos[i] for i < M (an index outside [0, S) latches
 // VLAC_ERR_DEVICE_CHECK and is replaced by 0, so no access leaves the cache),
 // off = {0, M}.

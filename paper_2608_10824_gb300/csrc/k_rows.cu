@@ -431,8 +431,8 @@ void launch_kv_copy(void* cache, void* flat, int n_heads, int Tc, int head_dim, 
            static_cast<uint8_t*>(flat), n_heads, Tc, head_dim * esz, to_cache);
 }
 
-void launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st) {
-  launch_k(copy_spans_kernel, dim3(64), dim3(256), 0, st, list, p, prm);
+cudaError_t launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st) {
+  return launch_k(copy_spans_kernel, dim3(64), dim3(256), 0, st, list, p, prm);
 }
 void launch_copies(const CopyList& list, cudaStream_t st) {
   StepParams none{};

@@ -10,11 +10,15 @@
 // Algorithm 1: m_{t-1} < theta_m (strict) invalidates the cache and runs the
 // full pass; otherwise Stage 3 reuses, at layer l, the floor(s_l * |R| / 1000)
 // most similar reusable patches and recomputes the rest.
+#include <mutex>
+
 #include "internal.cuh"
 
 namespace vlac {
 
 typedef unsigned __int128 u128;
+
+constexpr int kMaxSelectDevices = 64;
 
 // cos > num/den, exact.  Both patches all-zero: cos = 1; exactly one: cos = 0.
 __device__ __forceinline__ bool cos_above(uint32_t d, uint32_t na, uint32_t nb, uint32_t num, uint32_t den) {
@@ -218,26 +222,51 @@ __global__ void plan_kernel(const int* __restrict__ M, int B, int L, int* __rest
   }
 }
 
-void launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid, const StepParams* prm,
-                        int B, int n_views, int img_h, int img_w, int patch, int3* stats, uint8_t* mask,
-                        uint8_t* user_mask, cudaStream_t st) {
+cudaError_t launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid,
+                               const StepParams* prm, int B, int n_views, int img_h, int img_w, int patch,
+                               int3* stats, uint8_t* mask, uint8_t* user_mask, cudaStream_t st) {
   const int Nv = n_views * (img_h / patch) * (img_w / patch);
   dim3 grid((Nv + 7) / 8, B);
-  launch_k(patch_stats_kernel, grid, dim3(256), 0, st, frames, prev, valid, prm, n_views, img_h, img_w, patch, Nv,
+  return launch_k(patch_stats_kernel, grid, dim3(256), 0, st, frames, prev, valid, prm, n_views, img_h, img_w, patch, Nv,
            stats, mask, user_mask);
 }
 
-void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
-                   const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
-                   int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
-                   uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
-                   const uint8_t* active, const float* rel, uint8_t* rel_valid, const uint8_t* s2_forced,
-                   uint8_t* relevant, float* rel_out, cudaStream_t st) {
-  const size_t smem = (size_t)Nv * (sizeof(int3) + sizeof(int) + 1) + 16;
-  launch_k(select_kernel, dim3(B), dim3(512), smem, st, stats, mask, valid, m_prev, prm, override_, Nv, S, L, P,
+// Shared memory of select_kernel for Nv patches: the int3 statistics, the
+// reuse ranks and the static flags.  Above 48 KB (Nv > 2890) the kernel needs
+// the opt-in limit, raised once per device for the largest Nv the dims
+// accept (4096 patches).
+static size_t select_smem(int Nv) { return (size_t)Nv * (sizeof(int3) + sizeof(int) + 1) + 16; }
+static cudaError_t select_smem_attr(size_t smem) {
+  if (smem <= 48u * 1024u) return cudaSuccess;
+  static std::mutex mu;
+  static bool done[kMaxSelectDevices] = {};
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxSelectDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!done[dev]) {
+    e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)select_smem(4096));
+    if (e != cudaSuccess) return e;
+    done[dev] = true;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
+                          const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
+                          int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
+                          uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
+                          const uint8_t* active, const float* rel, uint8_t* rel_valid, const uint8_t* s2_forced,
+                          uint8_t* relevant, float* rel_out, cudaStream_t st) {
+  const size_t smem = select_smem(Nv);
+  cudaError_t e = select_smem_attr(smem);
+  if (e != cudaSuccess) return e;
+  e = launch_k(select_kernel, dim3(B), dim3(512), smem, st, stats, mask, valid, m_prev, prm, override_, Nv, S, L, P,
            parallel, n_action, full, idx, M, emit_slot, user_recomputed, user_gate_auto, user_idx, user_M, active, rel,
            rel_valid, s2_forced, relevant, rel_out);
-  launch_k(plan_kernel, dim3(1), dim3(256), 0, st, M, B, L, off);
+  if (e != cudaSuccess) return e;
+  return launch_k(plan_kernel, dim3(1), dim3(256), 0, st, M, B, L, off);
 }
 
 }  // namespace vlac
