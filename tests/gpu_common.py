@@ -28,11 +28,17 @@ ID_EXEMPT_MARGIN = 1e-3
 # twice the bar.  The deep tests exempt exactly those ids, and require the
 # GPU's id to be the first maximum of the GPU's own logits.
 FLAG_TIE = 1e-4
-# Stage 2 relevance, relative to the sequence's largest relevance: the kernel
-# sums fp32 probabilities of the same bf16 (or fp32) Q and K the oracle sums
-# in fp64.  A removal-set difference is allowed only for patches whose oracle
-# relevance lies within twice this of the oracle's k-th / (k+1)-th midpoint.
+# Stage 2 relevance, relative to the sequence's largest relevance.  At layer
+# 0 the kernel sums fp32 probabilities of the same bf16 (or fp32) Q and K the
+# oracle sums in fp64 (REL_TOL).  At a deeper layer of a bf16 model Q and K
+# also carry the earlier layers' GEMM-input roundings (a bf16 flip moves a
+# score by up to 2^-8 of one of its terms), so the probabilities move by the
+# score error rather than by fp32 rounding: REL_TOL_DEEP, about three times
+# the largest distance measured on the small models (6.1e-4 at layer 1).
+# A removal-set difference is allowed only for patches whose oracle relevance
+# lies within twice the bar of the oracle's k-th / (k+1)-th midpoint.
 REL_TOL = {"bf16": 1e-4, "f32": 1e-5}
+REL_TOL_DEEP = {"bf16": 2e-3, "f32": 1e-5}
 # Entropy of the bin softmax: H moves by at most max_j |l_j - E_p[l]| per unit
 # of logit error, about 5 for these models' logit spread, so the bar is five
 # times the logit bar; the library's entropy must also match the entropy of
@@ -131,9 +137,14 @@ class Lockstep:
         assert err == 0, f"device error {err}"
         rep = compare(d, o, g, self.prev_m, tau_m, self.logit_tol)
         stepped = np.ones(B, bool) if act is None else act != 0
-        rep.update(compare_stage2(d, o, g, s2_top_k, self.prev_rel, stepped))
+        rep.update(compare_stage2(d, o, g, s2_top_k, self.prev_rel, stepped, s2_layer))
         rep.update(compare_signals(d, o, g, self.prev_ids, self.logit_tol, stepped))
-        self.prev_ids = (o["action_ids"].copy(), g["action_ids"].copy())
+        # the ids a sequence's next action delta is measured against: a sequence
+        # that sat the step out keeps those of the last step it ran
+        po, pg = o["action_ids"].copy(), g["action_ids"].copy()
+        if act is not None and self.prev_ids is not None:
+            po[~stepped], pg[~stepped] = self.prev_ids[0][~stepped], self.prev_ids[1][~stepped]
+        self.prev_ids = (po, pg)
         rel = o["relevance"].copy() if s2_top_k > 0 else None
         m = o["step_margin"].copy()
         if act is not None and self.prev_m is not None:  # a paused sequence keeps its m_{t-1}
@@ -174,7 +185,7 @@ def compare(d, o, g, prev_m, tau_m, logit_tol=None):
             "id_exempt": int(exempt.sum()), "recomputed": o["recomputed"].tolist()}
 
 
-def compare_stage2(d, o, g, top_k, prev_rel, stepped=None):
+def compare_stage2(d, o, g, top_k, prev_rel, stepped=None, s2_layer=0):
     """Stage 2: this step's relevance within REL_TOL of the oracle's (relative
     to the sequence's largest), and the removal set the library decided from
     its previous relevance equal to the oracle's except inside the tie band
@@ -182,7 +193,7 @@ def compare_stage2(d, o, g, top_k, prev_rel, stepped=None):
     if top_k == 0:
         assert not g["relevance"].any() and not g["relevant"].any(), "Stage 2 off: nothing measured or removed"
         return {"rel_diff": 0.0, "removal_diffs": 0}
-    tol = REL_TOL[d.dtype]
+    tol = (REL_TOL if s2_layer == 0 else REL_TOL_DEEP)[d.dtype]
     worst, diffs = 0.0, 0
     for b in range(o["relevance"].shape[0]):
         if stepped is not None and not stepped[b]:  # sat the step out: both sides return zeros
