@@ -98,8 +98,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ ActMaps tmA, const __grid_constant__ CUtensorMap tmW,
                    const int* __restrict__ m_ptr, int m_cap, int N, int k_chunks, int chunks_per_split,
                    float* __restrict__ out, size_t split_stride, int full_tiles, int tail,
-                   float* __restrict__ tail_out, size_t tail_stride, int tail_ld, int* __restrict__ err,
-                   uint32_t wait_limit) {
+                   float* __restrict__ tail_out, size_t tail_stride, int tail_ld, int chain_mode,
+                   int* __restrict__ err, uint32_t wait_limit) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kMaxStages];
   __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
@@ -116,15 +116,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   // tile; the rest cut the remaining tiles into `tail` K ranges each (with
   // full_tiles == 0 in the order of a (tiles x splits) grid)
   const int n_tiles = N / kBM;
+  const int bx = blockIdx.x, by = blockIdx.y, ny = gridDim.y;
   int tile, sidx;  // sidx -1: the whole K range
-  if ((int)blockIdx.x < full_tiles) {
-    tile = blockIdx.x;
+  if (bx < full_tiles) {
+    tile = bx;
     sidx = -1;
   } else if (full_tiles == 0) {
-    tile = blockIdx.x % n_tiles;
-    sidx = blockIdx.x / n_tiles;
+    tile = bx % n_tiles;
+    sidx = bx / n_tiles;
   } else {
-    const int j = blockIdx.x - full_tiles;
+    const int j = bx - full_tiles;
     tile = full_tiles + j / tail;
     sidx = j - (j / tail) * tail;
   }
@@ -145,35 +146,39 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_trigger();
   const int M_all = min(*m_ptr, m_cap);
   if (M_all <= 0) return;
-  // token blocks (gridDim.y > 1): above kOnePass rows every CTA takes one
+  // token blocks (gridDim.y > 1): above one pass of rows every CTA takes one
   // block of kMaxTok rows, so the blocks of a tile run side by side instead
   // of as passes of one CTA; at or below it block 0 takes every row
+  const int one_pass = chain_mode == 1 ? kMaxTok : kOnePass;
   int row_base = 0, M = M_all;
-  if (gridDim.y > 1) {
-    if (M_all <= kOnePass) {
-      if (blockIdx.y > 0) return;
+  if (ny > 1) {
+    if (M_all <= one_pass) {
+      if (by > 0) return;
     } else {
-      row_base = (int)blockIdx.y * kMaxTok;
+      row_base = by * kMaxTok;
       if (row_base >= M_all) return;
       M = min(M_all - row_base, kMaxTok);
     }
   }
   const int nk = kc1 - kc0;
   if (nk <= 0) return;
-  // token passes: one pass up to kOnePass tokens, else passes of kMaxTok
+  // token passes: one pass up to one_pass tokens, else passes of kMaxTok
   // (every pass streams the weight tile again)
-  const int pass_tok = M <= kOnePass ? M : kMaxTok;
+  const int pass_tok = M <= one_pass ? M : kMaxTok;
   const int tok_layout = ((min(M, pass_tok) + kBoxRows - 1) / kBoxRows) * kBoxRows;
   const uint32_t stage_bytes = kWTileBytes + (uint32_t)tok_layout * 128u;
   const int n_stages = min(kMaxStages, (int)((kSmemBytes - 1024) / stage_bytes));
   const int n_pass = (M + pass_tok - 1) / pass_tok;
-  // independent accumulator chains: consecutive MMAs into one accumulator
-  // serialise, so the K steps alternate between C accumulators (4 for up to
-  // 128 tokens, 2 for up to 256).  Above 256 tokens the 512 TMEM columns do
-  // not hold two chains of every token: the first `split` tokens get two
-  // chains and the rest one (split + tok_layout <= 512 columns).
-  const int C = tok_layout <= 128 ? 4 : tok_layout <= 256 ? 2 : 1;
-  const int split = C == 1 ? ((512 - tok_layout) / kBoxRows) * kBoxRows : 0;
+  // Independent accumulator chains: consecutive MMAs into one accumulator
+  // serialise, so the K steps of 16 alternate between C accumulators, added
+  // in order by the epilogue.  chain_mode 1 (the default): always C = 2, at
+  // most 256 tokens per pass (2 x 256 TMEM columns), so a token's fp32
+  // summation order does not depend on which other tokens share the pass.
+  // chain_mode 0: C = 4 for up to 128 tokens, 2 for up to 256, and above 256
+  // the first `split` tokens get two chains and the rest one (split +
+  // tok_layout <= 512 columns): one pass up to 384 tokens, not row-invariant.
+  const int C = chain_mode == 1 ? 2 : tok_layout <= 128 ? 4 : tok_layout <= 256 ? 2 : 1;
+  const int split = (C == 1 && chain_mode == 0) ? ((512 - tok_layout) / kBoxRows) * kBoxRows : 0;
   const uint32_t ncols = 512;
 
   if (threadIdx.x == 0) {
@@ -394,14 +399,29 @@ void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr
   const int full_tiles = sp.full_cols / tc::kBM, n_tiles = N / tc::kBM;
   // token blocks side by side when the rows can exceed one pass (the CTAs of
   // blocks a step does not need return at once)
-  static const bool token_blocks = [] {
+  // VLAC_GEMM_TOKEN_BLOCKS: 0 never, 1 whenever the rows exceed one pass;
+  // unset: above two passes of rows (at two passes the second block's CTAs
+  // re-read the weights from DRAM a wave later, where passes inside one CTA
+  // find them in L2)
+  static const int token_blocks = [] {
     const char* e = std::getenv("VLAC_GEMM_TOKEN_BLOCKS");
-    return !e || std::atoi(e) != 0;
+    return e ? (std::atoi(e) != 0 ? 1 : 0) : -1;
   }();
-  const int tb = (token_blocks && m_cap > tc::kOnePass) ? (m_cap + tc::kMaxTok - 1) / tc::kMaxTok : 1;
+  // accumulator chains (see gemm_tc_kernel): 1 (default) keeps every row's
+  // summation order independent of the row count; VLAC_GEMM_CHAINS=0 selects
+  // the row-count-dependent chains (faster for 257-384 rows, not
+  // row-invariant), kept for measurement
+  static const int chain_mode = [] {
+    const char* e = std::getenv("VLAC_GEMM_CHAINS");
+    return (e && std::atoi(e) == 0) ? 0 : 1;
+  }();
+  const int one_pass = chain_mode == 1 ? tc::kMaxTok : tc::kOnePass;
+  const bool tb_on = token_blocks == 1 ? m_cap > one_pass : token_blocks == 0 ? false : m_cap > 2 * tc::kMaxTok;
+  const int tb = tb_on ? (m_cap + tc::kMaxTok - 1) / tc::kMaxTok : 1;
   dim3 grid(full_tiles + (n_tiles - full_tiles) * sp.tail, tb);
   launch_k(tc::gemm_tc_kernel, grid, dim3(tc::kThreads), tc::kSmemBytes, st, *tmA, *tmW, m_ptr, m_cap, N, k_chunks,
-           cps, out, sp.stride, full_tiles, sp.tail, sp.tail_p, sp.tail_stride, sp.tail_ld, err, wait_limit);
+           cps, out, sp.stride, full_tiles, sp.tail, sp.tail_p, sp.tail_stride, sp.tail_ld, chain_mode, err,
+           wait_limit);
 }
 
 // =============================================================================
