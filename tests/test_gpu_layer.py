@@ -19,6 +19,19 @@ from tests.gpu_common import LOGIT_TOL, SMALL
 
 pytestmark = [pytest.mark.gpu, pytest.mark.timeout(1800)]
 
+# The 7B-shaped layer is fed N(0, 1) rows, about fifty times a real step's
+# hidden state, and its SwiGLU product then reaches |G| ~ 40, where one bf16
+# step is 0.25: wherever fp32 (GPU) and fp64 (oracle) sums fall on opposite
+# sides of a rounding midpoint, the down projection moves every output of
+# that row by 0.25 * W_down[i][j].  A plain fp32 restatement of the layer on
+# the CPU sits 3.9e-2 from the oracle on these inputs (tests/test_layer_floor.py),
+# (every row 2.9e-3 to 3.5e-3 off, relative L2), so the element bar at that
+# width is LAYER_TOL_WIDE; every row must also stay
+# within ROW_REL_TOL of the oracle's row (relative L2), which a wrong term,
+# index or operand would break by orders of magnitude.
+LAYER_TOL_WIDE = 1e-1
+ROW_REL_TOL = 2.0 ** -7
+
 
 def _run(d, w_cpu, w_gpu, Ms, seed, layer=0):
     import torch
@@ -28,7 +41,7 @@ def _run(d, w_cpu, w_gpu, Ms, seed, layer=0):
     orc = oracle.Oracle(d, w_cpu)
     ctx = Context(d, w_gpu, max_batch=1)
     dt = torch.bfloat16 if d.dtype == "bf16" else torch.float32
-    tol = LOGIT_TOL[d.dtype]
+    tol = LOGIT_TOL[d.dtype] if d.hidden < 4096 else LAYER_TOL_WIDE
     kv_rel = 2.0 ** -7 if d.dtype == "bf16" else 1e-5
     report = []
     for M in Ms:
@@ -47,8 +60,12 @@ def _run(d, w_cpu, w_gpu, Ms, seed, layer=0):
         torch.cuda.synchronize()
         assert ctx.sync_error() == 0
         got = xg.cpu().numpy()
-        diff = float(np.max(np.abs(got.astype(np.float64) - want)))
+        err = np.abs(got.astype(np.float64) - want)
+        diff = float(err.max())
+        row_rel = float(np.max(np.linalg.norm(got - want, axis=1) / np.linalg.norm(want, axis=1)))
+        print(f"M={M}: max {diff:.3e} mean {float(err.mean()):.3e} row-relative L2 {row_rel:.3e}")
         assert diff <= tol, f"M={M}: layer outputs differ by {diff:.3e} > {tol}"
+        assert row_rel <= ROW_REL_TOL, f"M={M}: a row differs by {row_rel:.3e} (relative L2)"
         for name, g_kv, o_kv in (("K", kg, oc.read(0, "K", layer)), ("V", vg, oc.read(0, "V", layer))):
             g_kv = g_kv.float().cpu().numpy()
             rows = np.zeros(d.cache_len, bool)
