@@ -38,12 +38,11 @@ TAU_SIM = (996, 1000)
 CPU_LAYERS = 2  # the CPU oracle sample runs this many of the 32 layers
 # dram__bytes_read.sum + dram__bytes_write.sum of one dgemv_kernel launch,
 # averaged over the four projections of a decode layer, from one ncu capture
-# (profiles/dgemv_openvla7b_decode_layer.txt: 102.0 MB).  Reported only while
-# the kernel is the one the counters were taken on; the kernel's give-up path
-# has changed since, so the figure is withheld until the next capture.
-DGEMV_TRAFFIC_PER_LAUNCH: dict = {}
-DGEMV_TRAFFIC_NOTE = ("ncu traffic withheld: dgemv_kernel changed (give-up path) after the last capture, "
-                      "which measured 102.0 MB per launch")
+# of the current kernel (profiles/dgemv_openvla7b_decode_layer.txt); the
+# weights and launch shapes are the same in both single-sequence workloads.
+# Reported only while the kernel is the one the counters were taken on.
+DGEMV_TRAFFIC_PER_LAUNCH: dict = {c: 102.06e6 for c in ("openvla7b", "layer7b")}
+DGEMV_TRAFFIC_NOTE = "ncu capture only for the 7B-shaped decode layer"
 
 
 def peaks():
@@ -93,6 +92,67 @@ def step_work(d, M_seq, idx_seq):
             bd = L * (2 * (pos + 1) * Hd * 2 + 2 * Hd * 2) + Hd * 2
             passes.append((fd, bd, float(w_bytes + head_bytes)))
     return passes
+
+
+def layer_work(d, pos):
+    """FLOPs and bytes of one decoder layer for rows at positions `pos` over
+    a cache of d.cache_len positions (the one-layer workload): the layer's
+    weights, the cache's K and V read, the rows' fresh K/V written and their
+    fp32 inputs read and outputs written."""
+    Hd, F = d.hidden, d.ffn
+    pos = np.asarray(pos, dtype=np.int64)
+    M = int(pos.size)
+    flops = M * 2 * (4 * Hd * Hd + 3 * F * Hd) + 4 * Hd * float(np.sum(pos + 1))
+    nbytes = (4 * Hd * Hd + 3 * F * Hd) * 2 + 2 * d.cache_len * Hd * 2 + M * 2 * Hd * 2 + 2 * M * Hd * 4
+    return flops, nbytes
+
+
+def run_layer_sweep(args, d):
+    """The one-layer workload: per recomputed-row count M, the device time of
+    one decoder layer (vlac_layer_bench) over a cache pre-filled with N(0, 1)
+    values, averaged over --steps calls after --warmup, against the layer's
+    roofline.  Prints one JSON line."""
+    import torch
+
+    from paper_2608_10824_gb300 import Context
+    dev = torch.device("cuda", 0)
+    w = synth.make_weights(d, seed=args.seed, device=dev, lm_head_rows=d.n_bins)
+    ctx = Context(d, w, max_batch=1)
+    del w
+    torch.cuda.empty_cache()
+    cache = ctx.new_cache(1)
+    dt = torch.bfloat16 if d.dtype == "bf16" else torch.float32
+    pk, src = peaks()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)   # 256 MB > L2, written between calls
+    results = []
+    for M in [m for m in (d.pass_len, 200, 120, 60, 30) if m <= d.pass_len]:
+        pos, x, k0, v0 = synth.make_layer_case(d, M, seed=args.seed)
+        ctx.cache_load(cache, 0, 0, torch.from_numpy(k0).to(dt).to(dev), torch.from_numpy(v0).to(dt).to(dev))
+        pos_d = torch.from_numpy(pos).to(dev)
+        x0 = torch.from_numpy(x).to(dev)
+        xb = torch.empty_like(x0)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        for i in range(args.warmup + args.steps):
+            xb.copy_(x0)
+            flush.fill_(i & 255)
+            if i >= args.warmup:
+                ev[i - args.warmup][0].record()
+            ctx.layer_bench(cache, 0, 0, pos_d, xb)
+            if i >= args.warmup:
+                ev[i - args.warmup][1].record()
+        torch.cuda.synchronize()
+        assert ctx.sync_error() == 0
+        ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+        f, b = layer_work(d, pos)
+        t_roof = max(f / (pk["bf16_tflops"] * 1e12), b / (pk["hbm_gbs"] * 1e9))
+        results.append({"M": M, "ms": ms, "roofline_ms": t_roof * 1e3, "frac": t_roof * 1e3 / ms,
+                        "tflops": f / (ms / 1e3) / 1e12, "gbs": b / (ms / 1e3) / 1e9})
+    print(json.dumps({"metric": "one decoder layer (7B shape) per recomputed-row count", "unit": "ms",
+                      "workload": f"{args.config}: 1 layer, hidden {d.hidden}, {d.n_heads}x{d.head_dim} heads, "
+                                  f"SwiGLU {d.ffn}, {d.pass_len}-position prefix pass, cache of {d.cache_len} "
+                                  f"positions pre-filled N(0, 1), seeded sorted positions, inputs N(0, 1)",
+                      "steps": args.steps, "warmup": args.warmup, "peaks": src, "l2": "256 MB written between calls",
+                      "results": results}))
 
 
 def batch_work(d, Ms, idxs):
@@ -242,7 +302,14 @@ def config_block(d, args):
                         f"{vis}{extra}, {d.n_text} text tokens, {act}, {EPISODE}-frame scene episode{batch}",
             "global_batch": d.max_batch * args.gpus, "seq_len": d.pass_len, "parallelism": f"replicas x{args.gpus}",
             "tau_sim": f"{TAU_SIM[0]}/{TAU_SIM[1]}", "tau_margin": args.tau_margin,
-            "reuse_permille": "linear 900 -> 500", "l2": "inputs larger than L2 (13 GB of weights per pass)"}
+            "reuse_permille": "linear 900 -> 500", "l2": "inputs larger than L2 (13 GB of weights per pass)",
+            "stage2": (f"top_k {args.stage2_top_k} by the text-to-vision relevance of layer {stage2_layer(d, args)}"
+                       if getattr(args, "stage2_top_k", 0) > 0 else "off")}
+
+
+def stage2_layer(d, args) -> int:
+    layer = getattr(args, "stage2_layer", None)
+    return d.n_layers // 2 if layer is None else layer
 
 
 # ---------------------------------------------------------------------------
@@ -260,6 +327,11 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-budget", type=float, default=25.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layer-sweep", action="store_true",
+                    help="time one decoder layer per recomputed-row count (the one-layer workload) instead")
+    ap.add_argument("--stage2-top-k", type=int, default=0,
+                    help="Stage 2 (task-relevant filtering): patches kept out of the reuse set; 0 = off")
+    ap.add_argument("--stage2-layer", type=int, default=None, help="layer whose attention gives the relevance")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -267,6 +339,9 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     d = synth.dims_for(args.config)
+    if args.layer_sweep:
+        run_layer_sweep(args, synth.dims_for("layer7b") if args.config == "openvla7b" else d)
+        return
     seed = replica_seed(args.seed, rank)
     B = d.max_batch
     frames = synth.make_episode(d, EPISODE, seed=seed, batch=B, kind="scene",
@@ -300,11 +375,12 @@ def main():
     outs = ctx.alloc_outputs(B, want=("M", "idx", "gate_auto"))
     hist = {k: torch.zeros((K,) + tuple(v.shape), dtype=v.dtype, device=dev) for k, v in outs.items()}
 
-    def one_step(t, out):
+    def one_step(t, out, tau=None):
         if t % EPISODE == 0:
             ctx.reset(cache)
         ctx.step(cache, fr_dev[t % EPISODE], pr_dev, None if pp_dev is None else pp_dev[t % EPISODE],
-                 tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm, out=out)
+                 tau_sim=TAU_SIM, tau_margin=args.tau_margin if tau is None else tau, permille=pm, out=out,
+                 s2_top_k=args.stage2_top_k, s2_layer=stage2_layer(d, args))
 
     def barrier():
         torch.cuda.synchronize()
@@ -312,48 +388,67 @@ def main():
             dist.barrier()
             torch.cuda.synchronize()
 
+    pk, src = peaks()
+    stream = torch.cuda.current_stream()
+
+    def timed_pass(t0, tau):
+        """K steps from frame t0 at theta_m = tau, bracketed by barriers and
+        CUDA events on the launching stream; returns (ms over ranks, launches,
+        clocks, work)."""
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        clk = Clocks(local)
+        time.sleep(0.3)
+        n0 = ctx.launch_count()
+        e0.record(stream)
+        for k in range(K):
+            one_step(t0 + k, {n: hist[n][k] for n in hist}, tau)
+        e1.record(stream)
+        barrier()
+        clocks = clk.stop()
+        launches = ctx.launch_count() - n0
+        ms = reduce_max(e0.elapsed_time(e1), dist, dev)
+        assert ctx.sync_error() == 0
+        # algorithmic work of the timed steps
+        Ms = hist["M"].cpu().numpy()           # [K][B][L]
+        idxs = hist["idx"].cpu().numpy()       # [K][B][S]
+        rec = hist["recomputed"].cpu().numpy()  # [K][B]
+        F_tot = B_tot = gemm_flops = 0.0
+        t_roof_step = t_roof_pass = 0.0
+        per_row = 2 * (4 * d.hidden * d.hidden + 3 * d.ffn * d.hidden)
+        for k in range(K):
+            f_, b_, passes = batch_work(d, Ms[k], idxs[k])
+            F_tot += f_
+            B_tot += b_
+            gemm_flops += float(Ms[k].sum()) * per_row
+            t_roof_step += max(f_ / (pk["bf16_tflops"] * 1e12), b_ / (pk["hbm_gbs"] * 1e9))
+            t_roof_pass += sum(max(fp / (pk["bf16_tflops"] * 1e12), bp / (pk["hbm_gbs"] * 1e9))
+                               for fp, bp in passes)
+        t_meas = ms / 1e3 / K
+        roof = {"frac": t_roof_step / K / t_meas, "frac_per_pass": t_roof_pass / K / t_meas,
+                "t_roof_ms": 1e3 * t_roof_step / K, "t_meas_ms": 1e3 * t_meas,
+                "alg_tflop_per_step": F_tot / K / 1e12, "alg_gb_per_step": B_tot / K / 1e9,
+                "peaks": src, "fire_rate": float(rec.mean())}
+        return ms, launches, clocks, roof, gemm_flops
+
     for t in range(W):
         one_step(t, outs)
     barrier()
     assert ctx.sync_error() == 0
     # ---- timed region: device-resident inputs ----
-    stream = torch.cuda.current_stream()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    clk = Clocks(local)
-    time.sleep(0.3)
-    n0 = ctx.launch_count()
-    e0.record(stream)
-    for k in range(K):
-        one_step(W + k, {n: hist[n][k] for n in hist})
-    e1.record(stream)
-    barrier()
-    clocks = clk.stop()
-    launches = ctx.launch_count() - n0
-    ms = reduce_max(e0.elapsed_time(e1), dist, dev)
-    assert ctx.sync_error() == 0
+    ms, launches, clocks, step_roof, gemm_flops = timed_pass(W, None)
     value = aggregate_rate(world, B, K, ms / 1e3)   # sequence-steps per second
-
-    # ---- algorithmic work of the timed steps ----
-    Ms = hist["M"].cpu().numpy()           # [K][B][L]
-    idxs = hist["idx"].cpu().numpy()       # [K][B][S]
-    rec = hist["recomputed"].cpu().numpy()  # [K][B]
-    pk, src = peaks()
-    F_tot = B_tot = gemm_flops = 0.0
-    t_roof_step = t_roof_pass = 0.0
-    per_row = 2 * (4 * d.hidden * d.hidden + 3 * d.ffn * d.hidden)
-    for k in range(K):
-        f_, b_, passes = batch_work(d, Ms[k], idxs[k])
-        F_tot += f_
-        B_tot += b_
-        gemm_flops += float(Ms[k].sum()) * per_row
-        t_roof_step += max(f_ / (pk["bf16_tflops"] * 1e12), b_ / (pk["hbm_gbs"] * 1e9))
-        t_roof_pass += sum(max(fp / (pk["bf16_tflops"] * 1e12), bp / (pk["hbm_gbs"] * 1e9)) for fp, bp in passes)
-    t_meas = ms / 1e3 / K
+    # ---- the same K frames once more at theta_m = 0: the gate never fires,
+    # every step after the first of an episode takes the cached branch ----
+    cached = None
+    if args.tau_margin != 0.0:
+        c_ms, _, c_clocks, c_roof, _ = timed_pass(W + K, 0.0)
+        cached = {"tau_margin": 0.0, "value": aggregate_rate(world, B, K, c_ms / 1e3), "unit": "steps/s",
+                  "ms_per_step": c_ms / K, "step_roofline": c_roof, "clocks": c_clocks}
 
     # ---- per-kind device time, second pass with per-launch events ----
     ctx.prof_enable(True)
     for k in range(K):
-        one_step(W + K + k, outs)
+        one_step(W + 2 * K + k, outs)
     barrier()
     ctx.prof_enable(False)
     g_ms, g_n, g_bytes = ctx.prof_read(0)
@@ -395,14 +490,15 @@ def main():
     barrier()
     t0 = time.perf_counter()
     for k in range(K):
-        t = W + 2 * K + k
+        t = W + 3 * K + k
         f_buf.copy_(fr_host[t % EPISODE], non_blocking=True)
         p_buf.copy_(pr_host, non_blocking=True)
         if q_buf is not None:
             q_buf.copy_(pp_host[t % EPISODE], non_blocking=True)
         if t % EPISODE == 0:
             ctx.reset(cache)
-        ctx.step(cache, f_buf, p_buf, q_buf, tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm, out=outs)
+        ctx.step(cache, f_buf, p_buf, q_buf, tau_sim=TAU_SIM, tau_margin=args.tau_margin, permille=pm, out=outs,
+                 s2_top_k=args.stage2_top_k, s2_layer=stage2_layer(d, args))
         for n, hbuf in res_host.items():
             hbuf.copy_(outs[n], non_blocking=True)
         torch.cuda.current_stream().synchronize()  # the action is needed before the next frame
@@ -426,14 +522,15 @@ def main():
         "ms_per_step": ms / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic (seeded scene frames, random-init N(0,0.02) bf16 weights)",
         "config": config_block(d, args),
-        "step_roofline": {"frac": t_roof_step / K / t_meas, "frac_per_pass": t_roof_pass / K / t_meas,
-                          "t_roof_ms": 1e3 * t_roof_step / K, "t_meas_ms": 1e3 * t_meas,
-                          "alg_tflop_per_step": F_tot / K / 1e12, "alg_gb_per_step": B_tot / K / 1e9,
-                          "peaks": src, "fire_rate": float(rec.mean())},
+        "step_roofline": step_roof,
+        "cached_branch": cached,
         "roofline": roof,
         "prefix_gemm": {"weight_gbs": gemm_gbs, "tflops": gemm_tfs, "launches": p_n,
                         "avg_launch_us": 1e3 * p_ms / max(p_n, 1)},
         "device_ms_per_step_by_kind": {k: round(v, 4) for k, v in breakdown.items()},
+        "by_kind_note": (f"per-launch CUDA events in a second, non-graph pass of the same K steps serialise the "
+                         f"launches: the kinds sum to {sum(breakdown.values()):.2f} ms per step against "
+                         f"{ms / K:.2f} ms of graph replay in the timed pass"),
         "clocks": clocks,
         "e2e": {"value": e2e, "unit": "steps/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "note": "frames + prompt (+ proprio) H2D from pinned memory, action ids/margins/flags D2H, "

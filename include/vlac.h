@@ -44,6 +44,8 @@ extern "C" {
 
 #define VLAC_MARGIN_PROB 0  /* gate signal p1 - p2 of the softmax over the action bins (Eq. 1) */
 #define VLAC_MARGIN_LOGIT 1 /* gate signal l1 - l2, the top-2 logit gap */
+#define VLAC_MARGIN_VOCAB 2 /* gate signal p1 - p2 of the softmax over the whole vocabulary (Sec. IV-A);
+                               reads every LM-head row per action token */
 #define VLAC_REDUCE_DEFAULT (-1) /* mean for autoregressive decode (Eq. 1), min for a parallel block */
 #define VLAC_REDUCE_MEAN 0
 #define VLAC_REDUCE_MIN 1
@@ -82,7 +84,8 @@ typedef struct vlac_weights {
   const void* const* w_up;      /* [ffn][hidden] */
   const void* const* w_down;    /* [hidden][ffn] */
   const void* final_norm;       /* [hidden] */
-  const void* lm_head;          /* [vocab][hidden]; only rows vocab-n_bins .. vocab-1 are read */
+  const void* lm_head;          /* [vocab][hidden]; rows vocab-n_bins .. vocab-1 give the action
+                                   bins, the others only the whole-vocabulary margin */
 } vlac_weights;
 
 /* Stage-1 threshold as an exact fraction: a patch is static iff cos > num/den. */
@@ -91,13 +94,28 @@ typedef struct vlac_rational {
 } vlac_rational;
 
 typedef struct vlac_step_opts {
-  int32_t margin_kind;         /* VLAC_MARGIN_PROB (default) or VLAC_MARGIN_LOGIT */
+  int32_t margin_kind;         /* VLAC_MARGIN_PROB (default), VLAC_MARGIN_LOGIT or VLAC_MARGIN_VOCAB */
   int32_t reduction;           /* VLAC_REDUCE_* */
   const int8_t* gate_override; /* device [B]: -1 gate decides, 0 force the cached branch,
                                   1 force the full branch; NULL = gate decides.  An empty
                                   cache always runs the full branch. */
   const int32_t* forced_ids;   /* device [B][n_action]: bins fed back during autoregressive
                                   decode instead of the argmax (lock-step replay); NULL = argmax */
+  const uint8_t* active;       /* device [B]: 0 = the sequence sits this step out (a running batch
+                                  that episodes join and leave): its prefix cache, gate state and
+                                  previous frame stay as they are and its outputs are zero (the
+                                  batch's decode rows still run, so its decode positions, which
+                                  its next step rewrites before reading them, may change);
+                                  NULL = all step */
+  int32_t s2_top_k;            /* Stage 2 (Sec. III-B task-relevant filtering): the top_k visual
+                                  patches by the previous step's relevance are never reused;
+                                  0 = Stage 2 off (default) */
+  int32_t s2_layer;            /* Stage 2: the layer (0 .. n_layers-1) whose attention gives the
+                                  relevance: per visual patch, the softmax probability the text
+                                  queries put on its key, summed over text rows and heads */
+  const uint8_t* s2_forced;    /* device [B][Nv]: the Stage-2 removal set to apply instead of the
+                                  library's own (lock-step replay; `relevant` still reports the
+                                  library's own set); NULL = the library's own */
 } vlac_step_opts;
 
 /* Device output buffers of one step (B = the cache's batch, D = n_action,
@@ -113,6 +131,13 @@ typedef struct vlac_step_out {
   uint8_t* static_mask; /* optional [B][Nv] Stage-1 result (0 without a previous frame) */
   int32_t* idx;         /* optional [B][S] recompute order: rows of layer l are idx[0..M[l]) */
   int32_t* M;           /* optional [B][L] rows recomputed at each layer */
+  float* relevance;     /* optional [B][Nv] this step's Stage-2 relevance (0 when Stage 2 is off) */
+  uint8_t* relevant;    /* optional [B][Nv] patches Stage 2 kept out of the reusable set this step */
+  float* entropy;       /* optional [B][D] entropy (nats) of each action token's bin softmax (Sec. VI) */
+  float* vocab_margin;  /* optional [B][D] p1 - p2 of the softmax over the whole vocabulary; asking
+                           for it (or for VLAC_MARGIN_VOCAB) reads every LM-head row per token */
+  int32_t* action_delta; /* optional [B] sum over d of |a_t^d - a_{t-1}^d| in bins, 0 on a sequence's
+                            first step and after a reset (Sec. VI) */
 } vlac_step_out;
 
 typedef struct vlac_ctx vlac_ctx;
@@ -127,7 +152,8 @@ int vlac_destroy(vlac_ctx* ctx);
 /* Bytes of device memory a cache for `batch` (1 .. max_batch) sequences needs:
  * per sequence the K/V of every layer and position, the fp32 input of every
  * layer for the prefix positions (tokens that rejoin at a deeper layer start
- * from it), the previous frame, m_{t-1} and a valid flag. */
+ * from it), the previous frame, m_{t-1}, a valid flag and the last step's
+ * Stage-2 relevance. */
 int vlac_cache_bytes(const vlac_ctx* ctx, int batch, size_t* bytes);
 /* Formats caller-owned device memory (>= vlac_cache_bytes, 256-byte aligned)
  * as an empty cache; the memory must outlive the cache handle.  Synchronous. */
@@ -140,9 +166,11 @@ int vlac_cache_destroy(vlac_cache* cache);
  *   proprio:         device [B][proprio_dim] fp32, NULL when proprio_dim == 0
  *   tau_sim:         Stage-1 threshold (static iff cos > num/den)
  *   tau_margin:      the gate fires iff m_{t-1} < tau_margin (strict)
- *   reuse_permille:  host [n_layers]: k_l = floor(permille[l] * |static| / 1000)
- *                    static patches (the most similar) are reused at layer l; each <= 1000
- *   opts:            NULL = defaults
+ *   reuse_permille:  host [n_layers]: k_l = floor(permille[l] * |reusable| / 1000)
+ *                    reusable patches (the most similar) are reused at layer l; each
+ *                    <= 1000.  Reusable = static and, with Stage 2, not relevant.
+ *   opts:            NULL = defaults; VLAC_ERR_INVALID_ARG if s2_top_k < 0, or if
+ *                    s2_top_k > 0 and s2_layer is not a layer
  *   out:             device output buffers (required members non-NULL)
  * Returns VLAC_ERR_STATE if the cache belongs to another context. */
 int vlac_step(vlac_ctx* ctx, vlac_cache* cache, const uint8_t* frames, const int32_t* prompt_ids,
@@ -151,8 +179,40 @@ int vlac_step(vlac_ctx* ctx, vlac_cache* cache, const uint8_t* frames, const int
               void* stream);
 
 /* Invalidates sequence `seq` (-1 = all): its next step runs the full pass as if
- * no cache existed (Algorithm 1, cache invalidation). */
+ * no cache existed (Algorithm 1, cache invalidation), and Stage 2 has no
+ * previous relevance to use. */
 int vlac_reset(vlac_cache* cache, int seq, void* stream);
+
+/* One decoder layer of the prefix pass on its own (the one-layer workload:
+ * gather, q/k/v + RoPE + K/V scatter, mixed-cache attention, o-projection,
+ * MLP, as vlac_step runs them for each layer).
+ *   seq, layer:  the cache sequence (< batch) and layer (< n_layers)
+ *   pos:         device int32 [M], distinct positions of the rows, each below
+ *                the prefix pass length S (n_text + visual + proprio, plus the
+ *                parallel action block); an index outside [0, S) latches
+ *                VLAC_ERR_DEVICE_CHECK in the context's error word and is
+ *                replaced by 0, so that no access leaves the cache
+ *   M:           1 .. S rows
+ *   x:           device fp32 [M][hidden]: the rows' layer inputs on entry,
+ *                their layer outputs on return
+ * The rows' K/V are written into the cache at their positions before any row
+ * attends; each row attends causally by position to that layer of the cache
+ * (rows of a parallel action block see the whole block).  Asynchronous on
+ * `stream`; the context's workspace is used, so calls on one context do not
+ * overlap.  VLAC_ERR_INVALID_ARG for NULL pointers or out-of-range seq,
+ * layer or M. */
+int vlac_layer_bench(vlac_ctx* ctx, vlac_cache* cache, int seq, int layer, const int32_t* pos, int M, float* x,
+                     void* stream);
+
+/* K and V of one layer of sequence `seq` as device arrays [T][hidden] in the
+ * model's element type (bf16 or fp32), row t the key (value) vector of
+ * position t, heads side by side; T = the cache's positions: S + n_action - 1
+ * for autoregressive decode, S for a parallel action block.
+ * vlac_cache_load copies them into the cache, vlac_cache_store out of it.
+ * Asynchronous on `stream`.  VLAC_ERR_INVALID_ARG for NULL or unaligned
+ * (4-byte) pointers or out-of-range seq or layer. */
+int vlac_cache_load(vlac_cache* cache, int seq, int layer, const void* K, const void* V, void* stream);
+int vlac_cache_store(const vlac_cache* cache, int seq, int layer, void* K, void* V, void* stream);
 
 /* Waits for the context's device work and returns (and clears) the latched
  * device error word. */
@@ -188,8 +248,8 @@ int vlac_prof_read(vlac_ctx* ctx, int kind, double* total_ms, uint64_t* launches
 
 /* Allocation-free selection step.  The paper has no counterpart of this call:
  * it exists for callers that cannot allocate device memory when they run it
- * -- code inside a CUDA stream capture, real-time control loops whose memory
- * is fixed up front, host frameworks that own every device allocation.  It
+ * -- real-time control loops whose memory is fixed up front, host frameworks
+ * that own every device allocation and forbid a library its own.  It
  * runs the same kernels as vlac_step's selection (Stage-1 exact patch
  * similarity, the gate on m_prev < tau_margin or gate_override, the Stage-3
  * recompute order) without a context and without allocating: its scratch is
@@ -206,8 +266,10 @@ int vlac_prof_read(vlac_ctx* ctx, int kind, double* total_ms, uint64_t* launches
  *   gate_override:  device [batch] int8 (-1 gate, 0 cached, 1 full) or NULL
  *   outputs (device): static_mask [batch][Nv], idx [batch][S], M [batch][n_layers],
  *                     recomputed [batch]
- * Returns VLAC_ERR_INVALID_ARG for bad arguments and when the call needs more
- * than the fixed scratch: batch x visual patches must stay within 20,000. */
+ * Returns VLAC_ERR_INVALID_ARG for bad arguments and VLAC_ERR_UNSUPPORTED
+ * when valid dims need more than the fixed scratch: batch x visual patches
+ * must stay within 20,000.  VLAC_ERR_CUDA when a launch fails (only this
+ * call's launches are checked). */
 int vlac_select_noalloc(const vlac_dims* d, int batch, const uint8_t* frames, const uint8_t* prev_frames,
                         const uint8_t* valid, const float* m_prev, vlac_rational tau_sim, float tau_margin,
                         const uint16_t* reuse_permille, const int8_t* gate_override, uint8_t* static_mask,

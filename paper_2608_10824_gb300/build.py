@@ -11,7 +11,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libvlac.so")
-SOURCES = ["vlac.cu", "k_select.cu", "k_rows.cu", "k_attn.cu", "k_gemm.cu", "k_decode.cu", "noalloc.cu"]
+SOURCES = ["vlac.cu", "k_select.cu", "k_rows.cu", "k_attn.cu", "k_gemm.cu", "k_decode.cu", "k_dpass.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-I", INCLUDE, "-I", CSRC]

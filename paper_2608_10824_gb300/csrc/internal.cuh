@@ -22,9 +22,28 @@ struct StepParams {
   int32_t reduction;  // resolved: 0 mean, 1 min
   int32_t has_override;
   int32_t has_forced;
-  int32_t pad;
+  int32_t has_active;
+  int32_t s2_top_k;  // Stage 2: 0 = off
+  int32_t s2_layer;
+  int32_t has_s2_forced;
   uint16_t permille[kMaxLayers];
 };
+
+// Where the K-split partial sums of a prefix GEMM live (out[s][m][n] of
+// launch_gemm_tc).  Columns below full_cols come from CTAs that ran the whole
+// K range: one partial, at part.  The other columns have `tail` partials: the
+// first at part, split s >= 1 either at part + s * stride (the uniform
+// layout, tail_ld == 0) or compactly at
+// tail_p + (s - 1) * tail_stride + row * tail_ld + (col - full_cols).
+struct SplitPlan {
+  int full_cols;
+  int tail;
+  size_t stride;
+  float* tail_p;
+  size_t tail_stride;
+  int tail_ld;
+};
+inline SplitPlan uniform_splits(int splits, size_t stride) { return SplitPlan{0, splits, stride, nullptr, 0, 0}; }
 
 // A set of rows processed by one layer: per sequence b, rows i < count_b with
 // count_b = off[b+1] - off[b]; the compacted row index is off[b] + i, the
@@ -73,6 +92,31 @@ struct DGemv {
   uint32_t pf_bytes;
 };
 constexpr int kDecodeRowsPerCta = 4;  // residual rows per decode-GEMV CTA (2 row pairs)
+
+// Tiled decode weights (built at create, streamed by the decode GEMV and the
+// persistent decode pass): groups of kDecGroupPairs output row pairs, K cut
+// into chunks of kDecTileBytes per row, bf16 tiles interleaved in 8-element K
+// steps ([k/8][row][k%8]).
+constexpr int kDecGroupPairs = 4;
+constexpr int kDecTileBytes = 4096;
+
+// Groups [g0, g1) of CTA b when G groups are cut over n CTAs: the first
+// G mod n CTAs take one group more.  CTAs are placed on SMs in index order as
+// the previous kernel's CTAs leave, so the low indices start first and fill
+// their weight ring earliest; they are the ones given the extra group.
+__host__ __device__ inline void dgemv_group_range(int G, int n, int b, int& g0, int& g1) {
+  const int q = G / n, r = G - q * n;
+  g0 = b * q + (b < r ? b : r);
+  g1 = g0 + q + (b < r ? 1 : 0);
+}
+
+// Position (in elements, within its row) of element k of a bf16 input vector
+// in the A-fragment order of mma.m16n8k16: per 32-element K step and lane t
+// the elements 2t, 2t+1, 2t+8, 2t+9, 2t+16, 2t+17, 2t+24, 2t+25.
+__device__ __forceinline__ int afrag_pos(int k) {
+  const int i = k >> 5, w = k & 31, s = w >> 3, t = (w & 7) >> 1;
+  return ((i * 4 + t) * 8) + s * 2 + (w & 1);
+}
 
 // ---- scalar helpers --------------------------------------------------------
 template <typename T> __device__ __forceinline__ float to_f(T v);
@@ -210,10 +254,11 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 }
 
 // Launch with optional programmatic stream serialization (the kernel may
-// start while its predecessor drains; it must call pdl_wait()).
+// start while its predecessor drains; it must call pdl_wait()).  Returns the
+// launch's own status.
 extern bool g_pdl;
 template <typename... KArgs, typename... Args>
-inline void launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args) {
+inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;
@@ -224,7 +269,7 @@ inline void launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sme
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = g_pdl ? 1 : 0;
-  cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
 }  // namespace vlac
@@ -234,14 +279,20 @@ namespace vlac {
 
 int check_dims(const vlac_dims* d);  // VLAC_OK or the error vlac_create would return
 
-void launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid,
+cudaError_t launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid,
                         const StepParams* prm, int B, int n_views, int img_h, int img_w, int patch,
                         int3* stats, uint8_t* mask, uint8_t* user_mask, cudaStream_t st);
-void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
+// Stage 2 state (all NULL = Stage 2 unavailable): rel [B][Nv] the previous
+// step's relevance and rel_valid [B] whether it holds one (cleared here on a
+// step with Stage 2 off); s2_forced [B][Nv] (with prm->has_s2_forced) is
+// applied instead of the kernel's own removal set; relevant [B][Nv] receives
+// the own set and rel_out [B][Nv] is zeroed on a step with Stage 2 off.
+cudaError_t launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
                    const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
                    int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
                    uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
-                   cudaStream_t st);
+                   const uint8_t* active, const float* rel, uint8_t* rel_valid, const uint8_t* s2_forced,
+                   uint8_t* relevant, float* rel_out, cudaStream_t st);
 
 template <typename T>
 void launch_im2col(Rows rows, int B, int S, const uint8_t* frames, int n_views, int img_h, int img_w,
@@ -255,26 +306,53 @@ template <typename T>
 void launch_layer_in(Rows rows, const int* off_prev, int B, int S, int hidden, float* H, size_t h_seq_stride,
                      const T* gain, float eps, T* A, cudaStream_t st);
 template <typename T>
-void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, int splits,
-                         size_t split_stride, const float* rope_cos, const float* rope_sin, T* Q, T* Kc,
-                         T* Vc, size_t kv_seq_stride, int Tc, cudaStream_t st);
+void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, const SplitPlan& sp,
+                         const float* rope_cos, const float* rope_sin, T* Q, T* Kc, T* Vc, size_t kv_seq_stride,
+                         int Tc, cudaStream_t st);
 template <typename T>
-void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part, int splits,
-                          size_t split_stride, const T* gain, float eps, T* A, cudaStream_t st);
+void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part, const SplitPlan& sp, const T* gain,
+                          float eps, T* A, cudaStream_t st);
 template <typename T>
-void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, int splits, size_t split_stride, T* G,
-                   cudaStream_t st);
-void launch_residual(Rows rows, int B, int S, int hidden, const float* part, int splits, size_t split_stride,
-                     cudaStream_t st);
+void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, const SplitPlan& sp, T* G, cudaStream_t st);
+void launch_residual(Rows rows, int B, int S, int hidden, const float* part, const SplitPlan& sp, cudaStream_t st);
 template <typename T>
 void launch_attention(Rows rows, int B, int S, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc,
                       size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, T* O, cudaStream_t st);
+// Stage 2 relevance of one layer (rows as for launch_attention; text rows are
+// positions text_lo .. P-1): part [B][n_heads][Nv] per head, then rel and
+// rel_out [B][Nv] summed over the heads in order, and rel_valid[b] = 1.
+// Returns nonzero if the shared-memory need exceeds a block's.
+template <typename T>
+int launch_relevance(Rows rows, int B, int n_heads, int head_dim, const T* Q, const T* Kc, size_t kv_seq_stride,
+                     int Tc, int Nv, int text_lo, int P, float* part, float* rel, float* rel_out, uint8_t* rel_valid,
+                     const StepParams* prm, const uint8_t* active, cudaStream_t st);
 template <typename T>
 void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
                          const int32_t* ids, const int32_t* forced, const StepParams* prm, float* Xd,
                          int* idx_dec, float* ssq_out, int* err, cudaStream_t st);
-void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps,
-                   float* m_prev, uint8_t* valid, float* user_step_margin, cudaStream_t st);
+// m_t from the per-token signals (margins, gaps or vocabulary margins vms by
+// prm->margin_kind); also the action delta against prev_ids (kept in the
+// cache, with ids_valid) into delta.  A sequence that sat the step out
+// (prm->has_active, active[b] == 0) keeps its gate state and previous ids.
+void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps, const float* vms,
+                   float* m_prev, uint8_t* valid, float* user_step_margin, const int32_t* ids, int32_t* prev_ids,
+                   uint8_t* ids_valid, int32_t* delta, const uint8_t* active, cudaStream_t st);
+// End of a step: the previous frame of every sequence that stepped becomes
+// this step's frame, and the outputs of the sequences that sat the step out
+// are zeroed (with prm->has_active; active NULL = all stepped).
+struct StepOutputs {
+  int32_t* ids;
+  float *margins, *gaps, *logits, *step_margin;
+  uint8_t *recomputed, *gate_auto, *mask;
+  int32_t *idx, *M;
+  float* relevance;   // Stage 2 outputs [B][Nv]
+  uint8_t* relevant;
+  float *entropy, *vocab_margin;  // [B][D]
+  int32_t* action_delta;          // [B]
+};
+void launch_commit(int B, int D, int n_bins, int Nv, int S, int L, size_t frame_bytes, const uint8_t* frames,
+                   uint8_t* prev, const StepParams* prm, const uint8_t* active, const StepOutputs& o,
+                   cudaStream_t st);
 
 // Copies of the caller's per-step inputs into the context's staging buffers
 // (and the step scalars into device memory), and of the step's outputs back
@@ -284,12 +362,21 @@ struct CopySpan {
   void* dst;
   size_t bytes;
 };
-constexpr int kMaxSpans = 12;
+constexpr int kMaxSpans = 16;
 struct CopyList {
   CopySpan span[kMaxSpans];
   int n;
 };
-void launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st);
+cudaError_t launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st);
+// One-layer entry: idx[i] = pos[i] for i < M (an index outside [0, S) latches
+// VLAC_ERR_DEVICE_CHECK and is replaced by 0, so no access leaves the cache),
+// off = {0, M}.
+void launch_layer_setup(const int32_t* pos, int M, int S, int* idx, int* off, int* err, cudaStream_t st);
+// K or V of one layer of one sequence between the cache layout
+// [head][position][head_dim] (cache) and [position][head * head_dim] (flat),
+// elements of esz bytes; to_cache selects the direction.
+void launch_kv_copy(void* cache, void* flat, int n_heads, int Tc, int head_dim, int esz, bool to_cache,
+                    cudaStream_t st);
 void launch_copies(const CopyList& list, cudaStream_t st);
 
 // Tensor maps of one activation buffer with boxes of 32, 64, 128 and 256 rows.
@@ -297,8 +384,11 @@ struct ActMaps {
   CUtensorMap m[4];
 };
 // GEMMs: out[s][m][n] = sum over split s of A[m][k] * W[n][k]; rows m < *m_ptr.
+// Split plan sp: CTAs for the first sp.full_cols / 128 weight tiles run the
+// whole K range; every other tile is cut into sp.tail K ranges (see SplitPlan
+// for where each partial goes).
 void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
-                    int splits, float* out, int* err, uint32_t wait_limit, cudaStream_t st);
+                    const SplitPlan& sp, float* out, int* err, uint32_t wait_limit, cudaStream_t st);
 template <typename T>
 void launch_gemm_simt(const T* A, const T* W, const int* m_ptr, int m_cap, int N, int K, float* out,
                       cudaStream_t st);
@@ -306,6 +396,46 @@ int launch_wait_selftest(int* err, uint32_t spin_limit, cudaStream_t st);
 template <typename T>
 void launch_dgemv(const DGemv& a, int epi, int nb, int n_sm, cudaStream_t st);
 int dgemv_grid(int n_pairs, int n_sm);  // CTAs (and sum-of-squares partials) of one decode GEMV
+
+// Persistent decode pass (k_dpass.cu): all layers of one decode token in one
+// cooperative launch, one CTA per SM.  Per-layer arrays are device arrays of L
+// pointers (tiled decode weights, RMSNorm gains); K/V of layer l at
+// Kc/Vc + l * kv_layer.  `ssq0` holds the decode embedding's sums of squares
+// ([nb][n_ssq0]); `ssq` ([nb][grid]) and `bar` (zeroed by the launcher) are
+// the launch's own workspace.
+struct DPass {
+  const bf16* const* w_qkv;
+  const bf16* const* w_o;
+  const bf16* const* w_gu;
+  const bf16* const* w_d;
+  const bf16* const* g_attn;
+  const bf16* const* g_ffn;
+  int L, hidden, ffn, n_heads, Tc, pos, ns, n_ssq0;
+  float eps, scale;
+  const float* rope_cos;
+  const float* rope_sin;
+  float* X;
+  bf16* Q;
+  bf16* AO;
+  bf16* G;
+  bf16* Kc;
+  bf16* Vc;
+  size_t kv_layer, kv_seq_stride;
+  const float* ssq0;
+  float* ssq;
+  unsigned* bar;
+  int* err;
+  // attention: each (sequence, head) cut into attn_chunks key ranges; with
+  // more than one, every range's partial (max, sum, unnormalised output) goes
+  // to attn_part + (b * n_heads + h) * part_stride + chunk * (head_dim + 2) and
+  // the last range to finish (counted in attn_cnt, zero between uses) combines
+  int attn_chunks;
+  size_t part_stride;
+  float* attn_part;
+  unsigned* attn_cnt;
+};
+bool dpass_supported(int hidden, int ffn, int n_heads, int head_dim, int nb, int ns);
+int launch_dpass(const DPass& a, int nb, int n_sm, cudaStream_t st);
 // Decode-streaming copy of a projection (W: [rows][K]); see k_decode.cu for the layout.
 template <typename T>
 void launch_tile_decode_weights(const T* W, int K, int n_pairs, int epi, int n_heads, int head_dim, int ffn, T* out,
@@ -315,9 +445,22 @@ size_t dgemv_stage_bytes();  // bytes of one weight-ring stage of the decode GEM
 template <typename T>
 void launch_dec_attention(int B, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc, size_t kv_seq_stride,
                           int Tc, int pos, float* part, unsigned* counters, T* O, cudaStream_t st);
+// Margin over the whole vocabulary: W the LM-head rows outside the bins
+// ([n_rows][hidden], T), xh scratch for the normed action rows ([rows][hidden],
+// T), vl scratch for their logits ([rows][n_rows] fp32), vm the margins [B][D].
+struct VocabHead {
+  const void* W;
+  int n_rows;
+  void* xh;
+  float* vl;
+  float* vm;
+};
+// Action head of rows_per_seq rows per sequence: bin logits, ids, margins,
+// gaps, entropy (may be NULL) and, with vh, the whole-vocabulary margin.
 template <typename T>
 void launch_head2(const float* X, const int* row_of_seq, size_t x_seq_stride, int rows_per_seq, int B, int hidden,
                   int n_bins, const T* final_norm, const T* head_w, float eps, float* logits_ws, int D, int tok0,
-                  int32_t* ids, float* margins, float* gaps, float* logits, cudaStream_t st);
+                  int32_t* ids, float* margins, float* gaps, float* logits, float* entropy, const VocabHead* vh,
+                  cudaStream_t st);
 
 }  // namespace vlac

@@ -361,6 +361,151 @@ void launch_attention(Rows rows, int B, int S, int n_heads, int head_dim, const 
              n_action, scale, O);
 }
 
+// ---- Stage 2 relevance (Sec. III-B, task-relevant filtering) ----------------
+//
+// For one layer: the softmax probability that each text row puts on each
+// visual key (positions 1 .. Nv), summed over the text rows.  One block per
+// (head, sequence).  Warp w takes the text rows w, w + 8, ... in row order:
+// the lanes compute the row's scores over its keys (kept in shared memory),
+// the warp reduces the maximum and the sum, and the lanes add the visual
+// probabilities into the warp's own sums.  The warps' sums are then added in
+// warp order.  The exact causal softmax of each row, sinks included, as in the
+// prefix attention.
+constexpr int kRelWarps = 8;
+
+template <typename T, int HD>
+__global__ void __launch_bounds__(kRelWarps * 32)
+    relevance_kernel(Rows rows, int n_heads, const T* __restrict__ Q, const T* __restrict__ Kc,
+                     size_t kv_seq_stride, int Tc, int Nv, int text_lo, int P, float scale,
+                     float* __restrict__ part) {
+  pdl_wait();
+  pdl_trigger();
+  extern __shared__ __align__(16) float rsm[];
+  const int h = blockIdx.x, b = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float* qs = rsm + warp * HD;                                        // [kRelWarps][HD]
+  float* sc = rsm + kRelWarps * HD + (size_t)warp * Tc;               // [kRelWarps][Tc]
+  float* acc = rsm + (size_t)kRelWarps * (HD + Tc) + (size_t)warp * Nv;  // [kRelWarps][Nv]
+  for (int v = lane; v < Nv; v += 32) acc[v] = 0.f;
+  const int cnt = rows.off[b + 1] - rows.off[b];
+  const int hidden = n_heads * HD;
+  const T* Kh = Kc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
+  for (int i = warp; i < cnt; i += kRelWarps) {
+    const int pos = rows.idx[(size_t)b * rows.idx_stride + i];
+    if (pos < text_lo || pos >= P) continue;  // not a text row after the image
+    const int nk = min(pos + 1, Tc);
+    const T* q = Q + (size_t)(rows.off[b] + i) * hidden + (size_t)h * HD;
+    for (int e = lane; e < HD; e += 32) qs[e] = to_f(q[e]);
+    __syncwarp();
+    float mx = -INFINITY;
+    for (int j = lane; j < nk; j += 32) {
+      const T* kr = Kh + (size_t)j * HD;
+      float dot = 0.f;
+      if constexpr (sizeof(T) == 2) {
+        const uint4* k4 = reinterpret_cast<const uint4*>(kr);
+#pragma unroll 4
+        for (int c8 = 0; c8 < HD / 8; ++c8) {
+          const uint4 u = k4[c8];
+          const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            dot = fmaf(__uint_as_float(wv[t] << 16), qs[c8 * 8 + 2 * t], dot);
+            dot = fmaf(__uint_as_float(wv[t] & 0xFFFF0000u), qs[c8 * 8 + 2 * t + 1], dot);
+          }
+        }
+      } else {
+        const float4* k4 = reinterpret_cast<const float4*>(kr);
+#pragma unroll 4
+        for (int c4 = 0; c4 < HD / 4; ++c4) {
+          const float4 u = k4[c4];
+          dot = fmaf(u.x, qs[c4 * 4 + 0], dot);
+          dot = fmaf(u.y, qs[c4 * 4 + 1], dot);
+          dot = fmaf(u.z, qs[c4 * 4 + 2], dot);
+          dot = fmaf(u.w, qs[c4 * 4 + 3], dot);
+        }
+      }
+      const float sv = dot * scale;
+      sc[j] = sv;
+      mx = fmaxf(mx, sv);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float z = 0.f;
+    for (int j = lane; j < nk; j += 32) {
+      const float pj = expf(sc[j] - mx);
+      sc[j] = pj;
+      z += pj;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+    const float inv = 1.0f / z;
+    __syncwarp();  // every lane's probabilities are in sc
+    for (int v = lane; v < Nv && v + 1 < nk; v += 32) acc[v] += sc[v + 1] * inv;
+    __syncwarp();  // before the next row overwrites qs and sc
+  }
+  __syncthreads();
+  const float* acc0 = rsm + (size_t)kRelWarps * (HD + Tc);
+  for (int v = threadIdx.x; v < Nv; v += blockDim.x) {
+    float t = 0.f;
+    for (int w = 0; w < kRelWarps; ++w) t += acc0[(size_t)w * Nv + v];
+    part[((size_t)b * n_heads + h) * Nv + v] = t;
+  }
+}
+
+// The heads' relevance added in head order; the step's relevance is kept for
+// the next step's selection and returned.
+__global__ void relevance_sum_kernel(const float* __restrict__ part, int n_heads, int Nv, float* __restrict__ rel,
+                                     float* __restrict__ rel_out, uint8_t* __restrict__ rel_valid,
+                                     const StepParams* __restrict__ prm, const uint8_t* __restrict__ active) {
+  pdl_wait();
+  pdl_trigger();
+  const int b = blockIdx.x;
+  if (prm->has_active && active && !active[b]) {  // sat the step out: its relevance stays
+    for (int v = threadIdx.x; v < Nv; v += blockDim.x) rel_out[(size_t)b * Nv + v] = 0.f;
+    return;
+  }
+  for (int v = threadIdx.x; v < Nv; v += blockDim.x) {
+    float t = 0.f;
+    for (int h = 0; h < n_heads; ++h) t += part[((size_t)b * n_heads + h) * Nv + v];
+    rel[(size_t)b * Nv + v] = t;
+    rel_out[(size_t)b * Nv + v] = t;
+  }
+  if (threadIdx.x == 0) rel_valid[b] = 1;
+}
+
+template <typename T, int HD>
+void relevance_launch(Rows rows, int B, int n_heads, const T* Q, const T* Kc, size_t kv_seq_stride, int Tc, int Nv,
+                      int text_lo, int P, size_t smem, float* part, cudaStream_t st) {
+  static size_t smem_set = 48 * 1024;  // raised once per kernel, before any graph capture of it
+  if (smem > smem_set) {
+    cudaFuncSetAttribute(relevance_kernel<T, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    smem_set = smem;
+  }
+  launch_k(relevance_kernel<T, HD>, dim3(n_heads, B), dim3(kRelWarps * 32), smem, st, rows, n_heads, Q, Kc,
+           kv_seq_stride, Tc, Nv, text_lo, P, 1.0f / sqrtf((float)HD), part);
+}
+
+template <typename T>
+int launch_relevance(Rows rows, int B, int n_heads, int head_dim, const T* Q, const T* Kc, size_t kv_seq_stride,
+                     int Tc, int Nv, int text_lo, int P, float* part, float* rel, float* rel_out, uint8_t* rel_valid,
+                     const StepParams* prm, const uint8_t* active, cudaStream_t st) {
+  const size_t smem = (size_t)kRelWarps * (head_dim + Tc + Nv) * sizeof(float);
+  if (smem > 200 * 1024) return 1;
+  if (head_dim == 128)
+    relevance_launch<T, 128>(rows, B, n_heads, Q, Kc, kv_seq_stride, Tc, Nv, text_lo, P, smem, part, st);
+  else
+    relevance_launch<T, 64>(rows, B, n_heads, Q, Kc, kv_seq_stride, Tc, Nv, text_lo, P, smem, part, st);
+  launch_k(relevance_sum_kernel, dim3(B), dim3(256), 0, st, (const float*)part, n_heads, Nv, rel, rel_out, rel_valid,
+           prm, active);
+  return 0;
+}
+
+template int launch_relevance<float>(Rows, int, int, int, const float*, const float*, size_t, int, int, int, int,
+                                     float*, float*, float*, uint8_t*, const StepParams*, const uint8_t*,
+                                     cudaStream_t);
+template int launch_relevance<bf16>(Rows, int, int, int, const bf16*, const bf16*, size_t, int, int, int, int,
+                                    float*, float*, float*, uint8_t*, const StepParams*, const uint8_t*,
+                                    cudaStream_t);
+
 template void launch_attention<float>(Rows, int, int, int, int, const float*, const float*, const float*, size_t,
                                       int, int, int, int, float*, cudaStream_t);
 template void launch_attention<bf16>(Rows, int, int, int, int, const bf16*, const bf16*, const bf16*, size_t, int,

@@ -133,30 +133,14 @@ __device__ __forceinline__ void norm_rows_to_smem(const float* __restrict__ X, c
 // landing before the CTA exits.
 
 constexpr int kNC = 8;          // consumer warps
-constexpr int kGP = 4;          // row pairs per group
-constexpr int kMaxNS = 24;      // stage ring capacity
-constexpr int kDecTileB = 4096; // bytes of one tile row (K chunk)
-
-// Groups [g0, g1) of CTA b when G groups are cut over n CTAs: the first
-// G mod n CTAs take one group more.  CTAs are placed on SMs in index order as
-// the previous kernel's CTAs leave, so the low indices start first and fill
-// their weight ring earliest; they are the ones given the extra group.
-__host__ __device__ inline void dgemv_group_range(int G, int n, int b, int& g0, int& g1) {
-  const int q = G / n, r = G - q * n;
-  g0 = b * q + min(b, r);
-  g1 = g0 + q + (b < r ? 1 : 0);
-}
+constexpr int kGP = kDecGroupPairs;      // row pairs per group
+constexpr int kMaxNS = 24;               // stage ring capacity
+constexpr int kDecTileB = kDecTileBytes; // bytes of one tile row (K chunk)
 
 __host__ __device__ inline size_t sgemv_xs_bytes(int nb, int K, int esz) {
   return ((size_t)nb * K * esz + 1023) / 1024 * 1024;
 }
 
-// position (in elements, within its row) of element k of a bf16 input vector
-// in A-fragment order
-__device__ __forceinline__ int afrag_pos(int k) {
-  const int i = k >> 5, w = k & 31, s = w >> 3, t = (w & 7) >> 1;
-  return ((i * 4 + t) * 8) + s * 2 + (w & 1);
-}
 
 template <int EPI>
 __host__ __device__ __forceinline__ void dec_pair_rows(int p, int n_heads, int head_dim, int ffn, int& r1, int& r2) {
@@ -1075,10 +1059,12 @@ __global__ void __launch_bounds__(256) head_logits_kernel(const float* __restric
   }
 }
 
-// argmax (lowest bin on ties), top-2 logit gap and p1 - p2 of one row.
+// argmax (lowest bin on ties), top-2 logit gap, p1 - p2 and the entropy
+// -sum p ln p = ln z - sum p (l - l1) of one row.
 __global__ void __launch_bounds__(32) head_margin_kernel(const float* __restrict__ logits_ws, int n_bins, int D, int tok0,
                                                          int32_t* __restrict__ ids, float* __restrict__ margins,
-                                                         float* __restrict__ gaps, float* __restrict__ logits) {
+                                                         float* __restrict__ gaps, float* __restrict__ logits,
+                                                         float* __restrict__ entropy) {
   pdl_wait();
   pdl_trigger();
   const int j = blockIdx.x, b = blockIdx.y, lane = threadIdx.x;
@@ -1099,37 +1085,204 @@ __global__ void __launch_bounds__(32) head_margin_kernel(const float* __restrict
       bi = oi;
     }
   }
-  float v2 = -INFINITY, z = 0.f;
+  float v2 = -INFINITY, z = 0.f, zl = 0.f;
   for (int c = lane; c < n_bins; c += 32) {
     if (c != bi) v2 = fmaxf(v2, lg[c]);
-    z += expf(lg[c] - bv);
+    const float e = expf(lg[c] - bv);
+    z += e;
+    zl = fmaf(e, lg[c] - bv, zl);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v2 = fmaxf(v2, __shfl_xor_sync(0xffffffffu, v2, o));
   z = warp_allsum(z);
+  zl = warp_allsum(zl);
   const size_t t = (size_t)b * D + tok0 + j;
   if (lane == 0) {
     ids[t] = bi;
     margins[t] = -expm1f(v2 - bv) / z;
     gaps[t] = bv - v2;
+    if (entropy) entropy[t] = logf(z) - zl / z;
   }
   if (logits)
     for (int c = lane; c < n_bins; c += 32) logits[t * n_bins + c] = lg[c];
 }
 
+// ---- margin over the whole vocabulary (Sec. IV-A, VLAC_MARGIN_VOCAB) ------------
+
+// The final-norm rows of the action positions, stored as T for the vocabulary
+// GEMV: row (b, j) at xh + (b * rows_per_seq + j) * hidden, rounded exactly as
+// the bin head rounds them.
+template <typename T>
+__global__ void __launch_bounds__(256) head_rows_kernel(const float* __restrict__ X, const int* __restrict__ row_of_seq,
+                                                        size_t x_seq_stride, int hidden, const T* __restrict__ final_norm,
+                                                        float eps, T* __restrict__ xh) {
+  pdl_wait();
+  pdl_trigger();
+  const int j = blockIdx.x, b = blockIdx.y;
+  const int row = row_of_seq ? row_of_seq[b] + j : j;
+  norm_rows_to_smem<T, 1>(X + (size_t)b * x_seq_stride + (size_t)row * hidden, final_norm, hidden, eps,
+                          xh + ((size_t)b * gridDim.x + j) * hidden);
+}
+
+// Logits of the LM-head rows outside the action bins (r < n_rows) for NR
+// normed action rows at once: a CTA takes 64 weight rows, 8 per warp, lanes
+// over K; every weight element read is used for the NR rows.
+// vl[(g * NR + i) * n_rows + r] for input row g * NR + i < n_in.
+constexpr int kVocRowsPerCta = 64;
+
+template <typename T, int NR>
+__global__ void __launch_bounds__(256) vocab_logits_kernel(const T* __restrict__ W, int n_rows, int hidden,
+                                                           const T* __restrict__ xh, int n_in,
+                                                           float* __restrict__ vl) {
+  pdl_wait();
+  pdl_trigger();
+  constexpr int V = Vec<T>::n;
+  extern __shared__ __align__(16) uint8_t vsm[];
+  T* xs = reinterpret_cast<T*>(vsm);  // [NR][hidden]
+  const int g = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int kv = hidden / V;
+  for (int m = threadIdx.x; m < NR * kv; m += blockDim.x) {
+    const int i = m / kv, k = m - i * kv;
+    const int row = g * NR + i;
+    reinterpret_cast<uint4*>(xs)[m] =
+        row < n_in ? reinterpret_cast<const uint4*>(xh + (size_t)row * hidden)[k] : make_uint4(0u, 0u, 0u, 0u);
+  }
+  __syncthreads();
+  const int r0 = blockIdx.x * kVocRowsPerCta + warp * 8;
+  float acc[8][NR];
+#pragma unroll
+  for (int q = 0; q < 8; ++q)
+#pragma unroll
+    for (int i = 0; i < NR; ++i) acc[q][i] = 0.f;
+  for (int k = lane; k < kv; k += 32) {
+    float xf[NR][V];
+#pragma unroll
+    for (int i = 0; i < NR; ++i) unpack<T>(reinterpret_cast<const uint4*>(xs + (size_t)i * hidden)[k], xf[i]);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      float wf[V];
+      const uint4 wv = r0 + q < n_rows ? __ldg(reinterpret_cast<const uint4*>(W + (size_t)(r0 + q) * hidden) + k)
+                                       : make_uint4(0u, 0u, 0u, 0u);
+      unpack<T>(wv, wf);
+#pragma unroll
+      for (int i = 0; i < NR; ++i)
+#pragma unroll
+        for (int e = 0; e < V; ++e) acc[q][i] = fmaf(wf[e], xf[i][e], acc[q][i]);
+    }
+  }
+#pragma unroll
+  for (int q = 0; q < 8; ++q)
+#pragma unroll
+    for (int i = 0; i < NR; ++i) {
+      const float s = warp_allsum(acc[q][i]);
+      const int row = g * NR + i;
+      if (lane == 0 && r0 + q < n_rows && row < n_in) vl[(size_t)row * n_rows + r0 + q] = s;
+    }
+}
+
+// p1 - p2 of the softmax over all vocab logits of one action row: the two
+// largest (a value present twice counts twice) and sum exp(l - l1), from the
+// non-bin logits vl and the bin logits of logits_ws; fixed reduction order.
+__global__ void __launch_bounds__(256) vocab_margin_kernel(const float* __restrict__ vl, int n_rows,
+                                                           const float* __restrict__ logits_ws, int n_bins, int D,
+                                                           int tok0, float* __restrict__ vm) {
+  pdl_wait();
+  pdl_trigger();
+  __shared__ float s1[8], s2[8], sz[8];
+  const int j = blockIdx.x, b = blockIdx.y, rows_per_seq = gridDim.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const size_t rix = (size_t)b * rows_per_seq + j;
+  const float* a = vl + rix * n_rows;
+  const float* bl = logits_ws + rix * n_bins;
+  const int n = n_rows + n_bins;
+  float t1 = -INFINITY, t2 = -INFINITY;
+  for (int c = threadIdx.x; c < n; c += blockDim.x) {
+    const float v = c < n_rows ? a[c] : bl[c - n_rows];
+    if (v > t1) {
+      t2 = t1;
+      t1 = v;
+    } else if (v > t2) {
+      t2 = v;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float u1 = __shfl_xor_sync(0xffffffffu, t1, o), u2 = __shfl_xor_sync(0xffffffffu, t2, o);
+    const float n2 = fmaxf(fminf(t1, u1), fmaxf(t2, u2));
+    t1 = fmaxf(t1, u1);
+    t2 = n2;
+  }
+  if (lane == 0) {
+    s1[warp] = t1;
+    s2[warp] = t2;
+  }
+  __syncthreads();
+  t1 = s1[0];
+  t2 = s2[0];
+  for (int w = 1; w < 8; ++w) {
+    const float n2 = fmaxf(fminf(t1, s1[w]), fmaxf(t2, s2[w]));
+    t1 = fmaxf(t1, s1[w]);
+    t2 = n2;
+  }
+  float z = 0.f;
+  for (int c = threadIdx.x; c < n; c += blockDim.x) z += expf((c < n_rows ? a[c] : bl[c - n_rows]) - t1);
+  z = warp_allsum(z);
+  if (lane == 0) sz[warp] = z;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float zt = 0.f;
+    for (int w = 0; w < 8; ++w) zt += sz[w];
+    vm[(size_t)b * D + tok0 + j] = -expm1f(t2 - t1) / zt;
+  }
+}
+
+template <typename T, int NR>
+static void vocab_logits_launch(const T* W, int n_rows, int hidden, const T* xh, int n_in, float* vl,
+                                cudaStream_t st) {
+  const size_t smem = (size_t)NR * hidden * sizeof(T);
+  static size_t smem_set = 48 * 1024;  // raised once per kernel, before any graph capture of it
+  if (smem > smem_set) {
+    cudaFuncSetAttribute(vocab_logits_kernel<T, NR>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    smem_set = smem;
+  }
+  const dim3 grid((n_rows + kVocRowsPerCta - 1) / kVocRowsPerCta, (n_in + NR - 1) / NR);
+  launch_k(vocab_logits_kernel<T, NR>, grid, dim3(256), smem, st, W, n_rows, hidden, xh, n_in, vl);
+}
+
 template <typename T>
 void launch_head2(const float* X, const int* row_of_seq, size_t x_seq_stride, int rows_per_seq, int B, int hidden,
                   int n_bins, const T* final_norm, const T* head_w, float eps, float* logits_ws, int D, int tok0,
-                  int32_t* ids, float* margins, float* gaps, float* logits, cudaStream_t st) {
+                  int32_t* ids, float* margins, float* gaps, float* logits, float* entropy, const VocabHead* vh,
+                  cudaStream_t st) {
   const size_t smem = (size_t)hidden * sizeof(T);
   launch_k(head_logits_kernel<T>, dim3(n_bins / 16, rows_per_seq, B), dim3(256), smem, st, X, row_of_seq,
            x_seq_stride, hidden, n_bins, final_norm, head_w, eps, logits_ws);
   launch_k(head_margin_kernel, dim3(rows_per_seq, B), dim3(32), 0, st, logits_ws, n_bins, D, tok0, ids, margins, gaps,
-           logits);
+           logits, entropy);
+  if (!vh) return;
+  // the other rows of the LM head: every weight row read once per group of <= 8 action rows
+  T* xh = static_cast<T*>(vh->xh);
+  const T* Wv = static_cast<const T*>(vh->W);
+  launch_k(head_rows_kernel<T>, dim3(rows_per_seq, B), dim3(256), 0, st, X, row_of_seq, x_seq_stride, hidden,
+           final_norm, eps, xh);
+  const int n_in = rows_per_seq * B;
+  if (vh->n_rows == 0) {  // every token is an action bin
+  } else if (n_in == 1)
+    vocab_logits_launch<T, 1>(Wv, vh->n_rows, hidden, xh, n_in, vh->vl, st);
+  else if (n_in == 2)
+    vocab_logits_launch<T, 2>(Wv, vh->n_rows, hidden, xh, n_in, vh->vl, st);
+  else if (n_in <= 4)
+    vocab_logits_launch<T, 4>(Wv, vh->n_rows, hidden, xh, n_in, vh->vl, st);
+  else
+    vocab_logits_launch<T, 8>(Wv, vh->n_rows, hidden, xh, n_in, vh->vl, st);
+  launch_k(vocab_margin_kernel, dim3(rows_per_seq, B), dim3(256), 0, st, (const float*)vh->vl, vh->n_rows,
+           (const float*)logits_ws, n_bins, D, tok0, vh->vm);
 }
 template void launch_head2<float>(const float*, const int*, size_t, int, int, int, int, const float*, const float*,
-                                  float, float*, int, int, int32_t*, float*, float*, float*, cudaStream_t);
+                                  float, float*, int, int, int32_t*, float*, float*, float*, float*, const VocabHead*,
+                                  cudaStream_t);
 template void launch_head2<bf16>(const float*, const int*, size_t, int, int, int, int, const bf16*, const bf16*,
-                                 float, float*, int, int, int32_t*, float*, float*, float*, cudaStream_t);
+                                 float, float*, int, int, int32_t*, float*, float*, float*, float*, const VocabHead*,
+                                 cudaStream_t);
 
 }  // namespace vlac

@@ -8,6 +8,8 @@
 //   - gemm_simt: the fp32 tiny model.
 // The decode passes (M = batch <= 8) use the fused weight-streaming GEMV in
 // k_decode.cu.
+#include <cstdlib>
+
 #include "internal.cuh"
 
 namespace vlac {
@@ -95,7 +97,9 @@ __device__ __forceinline__ uint32_t idesc_bf16(int n) {
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ ActMaps tmA, const __grid_constant__ CUtensorMap tmW,
                    const int* __restrict__ m_ptr, int m_cap, int N, int k_chunks, int chunks_per_split,
-                   float* __restrict__ out, size_t split_stride, int* __restrict__ err, uint32_t wait_limit) {
+                   float* __restrict__ out, size_t split_stride, int full_tiles, int tail,
+                   float* __restrict__ tail_out, size_t tail_stride, int tail_ld, int chain_mode,
+                   int* __restrict__ err, uint32_t wait_limit) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kMaxStages];
   __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
@@ -108,40 +112,73 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   uint8_t* tiles = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // this CTA's weight tile and K range: the first full_tiles CTAs run a whole
+  // tile; the rest cut the remaining tiles into `tail` K ranges each (with
+  // full_tiles == 0 in the order of a (tiles x splits) grid)
+  const int n_tiles = N / kBM;
+  const int bx = blockIdx.x, by = blockIdx.y, ny = gridDim.y;
+  int tile, sidx;  // sidx -1: the whole K range
+  if (bx < full_tiles) {
+    tile = bx;
+    sidx = -1;
+  } else if (full_tiles == 0) {
+    tile = bx % n_tiles;
+    sidx = bx / n_tiles;
+  } else {
+    const int j = bx - full_tiles;
+    tile = full_tiles + j / tail;
+    sidx = j - (j / tail) * tail;
+  }
+  const int n0 = tile * kBM;
+  const int kc0 = sidx < 0 ? 0 : sidx * chunks_per_split;
+  const int kc1 = sidx < 0 ? k_chunks : min(kc0 + chunks_per_split, k_chunks);
   if (threadIdx.x == 0) {
     // the weight tiles do not depend on earlier kernels: start pulling the
     // first ones into L2 while the previous kernel drains
-    const int k0 = blockIdx.y * chunks_per_split;
-    const int k1 = min(min(k0 + chunks_per_split, k_chunks), k0 + kPrefetchChunks);
-    for (int kc = k0; kc < k1; ++kc)
+    const int k1 = min(kc1, kc0 + kPrefetchChunks);
+    for (int kc = kc0; kc < k1; ++kc)
       asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
                        reinterpret_cast<uint64_t>(&tmW)),
-                   "r"(kc * kBK), "r"((int)blockIdx.x * kBM)
+                   "r"(kc * kBK), "r"(n0)
                    : "memory");
   }
   pdl_wait();
   pdl_trigger();
-  const int M = min(*m_ptr, m_cap);
-  if (M <= 0) return;
-  const int n0 = blockIdx.x * kBM;
-  const int kc0 = blockIdx.y * chunks_per_split;
-  const int kc1 = min(kc0 + chunks_per_split, k_chunks);
+  const int M_all = min(*m_ptr, m_cap);
+  if (M_all <= 0) return;
+  // token blocks (gridDim.y > 1): above one pass of rows every CTA takes one
+  // block of kMaxTok rows, so the blocks of a tile run side by side instead
+  // of as passes of one CTA; at or below it block 0 takes every row
+  const int one_pass = chain_mode == 1 ? kMaxTok : kOnePass;
+  int row_base = 0, M = M_all;
+  if (ny > 1) {
+    if (M_all <= one_pass) {
+      if (by > 0) return;
+    } else {
+      row_base = by * kMaxTok;
+      if (row_base >= M_all) return;
+      M = min(M_all - row_base, kMaxTok);
+    }
+  }
   const int nk = kc1 - kc0;
   if (nk <= 0) return;
-  // token passes: one pass up to kOnePass tokens, else passes of kMaxTok
+  // token passes: one pass up to one_pass tokens, else passes of kMaxTok
   // (every pass streams the weight tile again)
-  const int pass_tok = M <= kOnePass ? M : kMaxTok;
+  const int pass_tok = M <= one_pass ? M : kMaxTok;
   const int tok_layout = ((min(M, pass_tok) + kBoxRows - 1) / kBoxRows) * kBoxRows;
   const uint32_t stage_bytes = kWTileBytes + (uint32_t)tok_layout * 128u;
   const int n_stages = min(kMaxStages, (int)((kSmemBytes - 1024) / stage_bytes));
   const int n_pass = (M + pass_tok - 1) / pass_tok;
-  // independent accumulator chains: consecutive MMAs into one accumulator
-  // serialise, so the K steps alternate between C accumulators (4 for up to
-  // 128 tokens, 2 for up to 256).  Above 256 tokens the 512 TMEM columns do
-  // not hold two chains of every token: the first `split` tokens get two
-  // chains and the rest one (split + tok_layout <= 512 columns).
-  const int C = tok_layout <= 128 ? 4 : tok_layout <= 256 ? 2 : 1;
-  const int split = C == 1 ? ((512 - tok_layout) / kBoxRows) * kBoxRows : 0;
+  // Independent accumulator chains: consecutive MMAs into one accumulator
+  // serialise, so the K steps of 16 alternate between C accumulators, added
+  // in order by the epilogue.  chain_mode 1 (the default): always C = 2, at
+  // most 256 tokens per pass (2 x 256 TMEM columns), so a token's fp32
+  // summation order does not depend on which other tokens share the pass.
+  // chain_mode 0: C = 4 for up to 128 tokens, 2 for up to 256, and above 256
+  // the first `split` tokens get two chains and the rest one (split +
+  // tok_layout <= 512 columns): one pass up to 384 tokens, not row-invariant.
+  const int C = chain_mode == 1 ? 2 : tok_layout <= 128 ? 4 : tok_layout <= 256 ? 2 : 1;
+  const int split = (C == 1 && chain_mode == 0) ? ((512 - tok_layout) / kBoxRows) * kBoxRows : 0;
   const uint32_t ncols = 512;
 
   if (threadIdx.x == 0) {
@@ -192,7 +229,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // the token rows in as few boxes as possible: 256, 128, 64 and 32 rows
           for (int done = 0, left = nbox; left > 0;) {
             const int lg = left >= 8 ? 3 : left >= 4 ? 2 : left >= 2 ? 1 : 0;
-            tma_load_2d(at + (size_t)done * kBoxRows * 128, &tmA.m[lg], kc * kBK, row0 + done * kBoxRows,
+            tma_load_2d(at + (size_t)done * kBoxRows * 128, &tmA.m[lg], kc * kBK, row_base + row0 + done * kBoxRows,
                         &full_bar[stage]);
             done += 1 << lg;
             left -= 1 << lg;
@@ -270,8 +307,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // ---------------- epilogue: TMEM -> fp32 partials ----------------
     const int q = warp & 3;  // TMEM lane quarter this warp may access
-    const int n = n0 + q * 32 + lane;
-    float* dst = out + (size_t)blockIdx.y * split_stride;
+    // where this CTA's partial goes: split 0 (or a whole tile) into out, a
+    // later split into its uniform slot or the compact tail slots
+    float* dst = out;
+    int ld = N, n = n0 + q * 32 + lane;
+    if (sidx > 0) {
+      if (tail_ld) {
+        dst = tail_out + (size_t)(sidx - 1) * tail_stride;
+        ld = tail_ld;
+        n -= full_tiles * kBM;
+      } else {
+        dst = out + (size_t)sidx * split_stride;
+      }
+    }
     for (int pass = 0; pass < n_pass; ++pass) {
       const int row0 = pass * pass_tok;
       const int rows = min(M - row0, pass_tok);
@@ -302,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
             const int m = row0 + c0 + j;
-            if (m < M) dst[(size_t)m * N + n] = v[j];
+            if (m < M) dst[(size_t)(row_base + m) * ld + n] = v[j];
           }
           continue;
         }
@@ -316,7 +364,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
           const int m = row0 + c0 + j;
-          if (m < M) dst[(size_t)m * N + n] = v[j];
+          if (m < M) dst[(size_t)(row_base + m) * ld + n] = v[j];
         }
       }
       fence_before();
@@ -340,17 +388,40 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace tc
 
 void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr, int m_cap, int N, int K,
-                    int splits, float* out, int* err, uint32_t wait_limit, cudaStream_t st) {
+                    const SplitPlan& sp, float* out, int* err, uint32_t wait_limit, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
     cudaFuncSetAttribute(tc::gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, tc::kSmemBytes);
     attr_set = true;
   }
   const int k_chunks = K / tc::kBK;
-  const int cps = (k_chunks + splits - 1) / splits;
-  dim3 grid(N / tc::kBM, splits);
+  const int cps = (k_chunks + sp.tail - 1) / sp.tail;
+  const int full_tiles = sp.full_cols / tc::kBM, n_tiles = N / tc::kBM;
+  // token blocks side by side when the rows can exceed one pass (the CTAs of
+  // blocks a step does not need return at once)
+  // VLAC_GEMM_TOKEN_BLOCKS: 0 never, 1 whenever the rows exceed one pass;
+  // unset: above two passes of rows (at two passes the second block's CTAs
+  // re-read the weights from DRAM a wave later, where passes inside one CTA
+  // find them in L2)
+  static const int token_blocks = [] {
+    const char* e = std::getenv("VLAC_GEMM_TOKEN_BLOCKS");
+    return e ? (std::atoi(e) != 0 ? 1 : 0) : -1;
+  }();
+  // accumulator chains (see gemm_tc_kernel): 1 (default) keeps every row's
+  // summation order independent of the row count; VLAC_GEMM_CHAINS=0 selects
+  // the row-count-dependent chains (faster for 257-384 rows, not
+  // row-invariant), kept for measurement
+  static const int chain_mode = [] {
+    const char* e = std::getenv("VLAC_GEMM_CHAINS");
+    return (e && std::atoi(e) == 0) ? 0 : 1;
+  }();
+  const int one_pass = chain_mode == 1 ? tc::kMaxTok : tc::kOnePass;
+  const bool tb_on = token_blocks == 1 ? m_cap > one_pass : token_blocks == 0 ? false : m_cap > 2 * tc::kMaxTok;
+  const int tb = tb_on ? (m_cap + tc::kMaxTok - 1) / tc::kMaxTok : 1;
+  dim3 grid(full_tiles + (n_tiles - full_tiles) * sp.tail, tb);
   launch_k(tc::gemm_tc_kernel, grid, dim3(tc::kThreads), tc::kSmemBytes, st, *tmA, *tmW, m_ptr, m_cap, N, k_chunks,
-           cps, out, (size_t)m_cap * N, err, wait_limit);
+           cps, out, sp.stride, full_tiles, sp.tail, sp.tail_p, sp.tail_stride, sp.tail_ld, chain_mode, err,
+           wait_limit);
 }
 
 // =============================================================================

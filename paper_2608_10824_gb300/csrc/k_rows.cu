@@ -105,10 +105,17 @@ __device__ __forceinline__ float4 add4(float4 a, float4 b) {
 __device__ __forceinline__ float sq4(float4 a, float acc) {
   return fmaf(a.w, a.w, fmaf(a.z, a.z, fmaf(a.y, a.y, fmaf(a.x, a.x, acc))));
 }
-// Sum over the GEMM's K splits (split s at part + s * stride), in split order.
-__device__ __forceinline__ float4 sum_splits4(const float* __restrict__ part, int splits, size_t stride, size_t o) {
-  float4 v = *reinterpret_cast<const float4*>(part + o);
-  for (int s = 1; s < splits; ++s) v = add4(v, *reinterpret_cast<const float4*>(part + o + (size_t)s * stride));
+// Sum over the GEMM's K splits of column o of compacted row r (pr = that
+// row of split 0), in split order; see SplitPlan for the layout.
+__device__ __forceinline__ float4 sum_splits4(const float* __restrict__ pr, const SplitPlan& sp, int r, size_t o) {
+  float4 v = *reinterpret_cast<const float4*>(pr + o);
+  if ((long long)o < sp.full_cols) return v;
+  if (sp.tail_ld) {
+    const float* t = sp.tail_p + (size_t)r * sp.tail_ld + (o - sp.full_cols);
+    for (int s = 1; s < sp.tail; ++s) v = add4(v, *reinterpret_cast<const float4*>(t + (size_t)(s - 1) * sp.tail_stride));
+  } else {
+    for (int s = 1; s < sp.tail; ++s) v = add4(v, *reinterpret_cast<const float4*>(pr + o + (size_t)s * sp.stride));
+  }
   return v;
 }
 
@@ -174,7 +181,7 @@ __global__ void layer_in_kernel(Rows rows, const int* __restrict__ off_prev, int
 // takes four consecutive e of one head and their partners e + half.
 template <typename T>
 __global__ void qkv_epilogue_kernel(Rows rows, int n_heads, int head_dim, const float* __restrict__ part,
-                                    int splits, size_t split_stride, const float* __restrict__ rope_cos,
+                                    SplitPlan sp, const float* __restrict__ rope_cos,
                                     const float* __restrict__ rope_sin, T* __restrict__ Q, T* __restrict__ Kc,
                                     T* __restrict__ Vc, size_t kv_seq_stride, int Tc) {
   pdl_wait();
@@ -195,12 +202,12 @@ __global__ void qkv_epilogue_kernel(Rows rows, int n_heads, int head_dim, const 
     const float4 c = *reinterpret_cast<const float4*>(rope_cos + (size_t)pos * half + e);
     const float4 s = *reinterpret_cast<const float4*>(rope_sin + (size_t)pos * half + e);
     const size_t base = (size_t)h * head_dim + e;
-    const float4 q1 = sum_splits4(pr, splits, split_stride, base);
-    const float4 q2 = sum_splits4(pr, splits, split_stride, base + half);
-    const float4 k1 = sum_splits4(pr, splits, split_stride, hidden + base);
-    const float4 k2 = sum_splits4(pr, splits, split_stride, hidden + base + half);
-    const float4 v1 = sum_splits4(pr, splits, split_stride, 2 * hidden + base);
-    const float4 v2 = sum_splits4(pr, splits, split_stride, 2 * hidden + base + half);
+    const float4 q1 = sum_splits4(pr, sp, r, base);
+    const float4 q2 = sum_splits4(pr, sp, r, base + half);
+    const float4 k1 = sum_splits4(pr, sp, r, hidden + base);
+    const float4 k2 = sum_splits4(pr, sp, r, hidden + base + half);
+    const float4 v1 = sum_splits4(pr, sp, r, 2 * hidden + base);
+    const float4 v2 = sum_splits4(pr, sp, r, 2 * hidden + base + half);
     store4<T>(q_out + base, make_float4(q1.x * c.x - q2.x * s.x, q1.y * c.y - q2.y * s.y, q1.z * c.z - q2.z * s.z,
                                         q1.w * c.w - q2.w * s.w));
     store4<T>(q_out + base + half, make_float4(q2.x * c.x + q1.x * s.x, q2.y * c.y + q1.y * s.y,
@@ -217,8 +224,8 @@ __global__ void qkv_epilogue_kernel(Rows rows, int n_heads, int head_dim, const 
 
 // x += o-projection (summed over splits), then A = T(RMSNorm(x) * g).
 template <typename T>
-__global__ void residual_norm_kernel(Rows rows, int hidden, const float* __restrict__ part, int splits,
-                                     size_t split_stride, const T* __restrict__ gain, float eps, T* __restrict__ A) {
+__global__ void residual_norm_kernel(Rows rows, int hidden, const float* __restrict__ part, SplitPlan sp,
+                                     const T* __restrict__ gain, float eps, T* __restrict__ A) {
   pdl_wait();
   pdl_trigger();
   __shared__ float red[32];
@@ -231,7 +238,7 @@ __global__ void residual_norm_kernel(Rows rows, int hidden, const float* __restr
   float ss = 0.f;
 #pragma unroll 4
   for (int c = threadIdx.x; c < hidden / 4; c += blockDim.x) {
-    const float4 v = add4(reinterpret_cast<const float4*>(x)[c], sum_splits4(pr, splits, split_stride, 4 * (size_t)c));
+    const float4 v = add4(reinterpret_cast<const float4*>(x)[c], sum_splits4(pr, sp, r, 4 * (size_t)c));
     reinterpret_cast<float4*>(x)[c] = v;
     ss = sq4(v, ss);
   }
@@ -240,8 +247,7 @@ __global__ void residual_norm_kernel(Rows rows, int hidden, const float* __restr
 
 // G = T(silu(g) * u) from the fused projection [gate | up].
 template <typename T>
-__global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part, int splits, size_t split_stride,
-                              T* __restrict__ G) {
+__global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part, SplitPlan sp, T* __restrict__ G) {
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.y, i = blockIdx.x;
@@ -254,8 +260,8 @@ __global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part
   const int c1 = (int)(((long long)n4 * (blockIdx.z + 1)) / gridDim.z);
 #pragma unroll 4
   for (int c = c0 + threadIdx.x; c < c1; c += blockDim.x) {
-    const float4 g = sum_splits4(pr, splits, split_stride, 4 * (size_t)c);
-    const float4 u = sum_splits4(pr, splits, split_stride, (size_t)ffn + 4 * c);
+    const float4 g = sum_splits4(pr, sp, r, 4 * (size_t)c);
+    const float4 u = sum_splits4(pr, sp, r, (size_t)ffn + 4 * c);
     store4<T>(G + (size_t)r * ffn + 4 * c,
               make_float4((g.x / (1.0f + expf(-g.x))) * u.x, (g.y / (1.0f + expf(-g.y))) * u.y,
                           (g.z / (1.0f + expf(-g.z))) * u.z, (g.w / (1.0f + expf(-g.w))) * u.w));
@@ -263,8 +269,7 @@ __global__ void swiglu_kernel(Rows rows, int ffn, const float* __restrict__ part
 }
 
 // x += down-projection (summed over splits).
-__global__ void residual_kernel(Rows rows, int hidden, const float* __restrict__ part, int splits,
-                                size_t split_stride) {
+__global__ void residual_kernel(Rows rows, int hidden, const float* __restrict__ part, SplitPlan sp) {
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.y, i = blockIdx.x;
@@ -279,7 +284,7 @@ __global__ void residual_kernel(Rows rows, int hidden, const float* __restrict__
 #pragma unroll 4
   for (int c = c0 + threadIdx.x; c < c1; c += blockDim.x)
     reinterpret_cast<float4*>(x)[c] =
-        add4(reinterpret_cast<const float4*>(x)[c], sum_splits4(pr, splits, split_stride, 4 * (size_t)c));
+        add4(reinterpret_cast<const float4*>(x)[c], sum_splits4(pr, sp, r, 4 * (size_t)c));
 }
 
 // Autoregressive decode input: the bin fed back (argmax, or the forced replay
@@ -314,15 +319,35 @@ __global__ void decode_embed_kernel(int d, int D, int P, int hidden, int vocab, 
 }
 
 // m_t = mean (Eq. 1) or min of the per-token signals; the cache keeps it for
-// the next step's gate and becomes valid.
+// the next step's gate and becomes valid.  The action delta (Sec. VI) is the
+// L1 distance in bins to the previous step's ids on the sequence.
 __global__ void finish_kernel(int B, int D, const StepParams* __restrict__ prm, const float* __restrict__ margins,
-                              const float* __restrict__ gaps, float* __restrict__ m_prev, uint8_t* __restrict__ valid,
-                              float* __restrict__ user_step_margin) {
+                              const float* __restrict__ gaps, const float* __restrict__ vms,
+                              float* __restrict__ m_prev, uint8_t* __restrict__ valid,
+                              float* __restrict__ user_step_margin, const int32_t* __restrict__ ids,
+                              int32_t* __restrict__ prev_ids, uint8_t* __restrict__ ids_valid,
+                              int32_t* __restrict__ delta, const uint8_t* __restrict__ active) {
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
-  const float* sig = (prm->margin_kind == VLAC_MARGIN_LOGIT ? gaps : margins) + (size_t)b * D;
+  if (prm->has_active && active && !active[b]) {  // sat the step out: the gate state and ids stay
+    user_step_margin[b] = 0.f;
+    delta[b] = 0;
+    return;
+  }
+  const float* sig = (prm->margin_kind == VLAC_MARGIN_LOGIT   ? gaps
+                      : prm->margin_kind == VLAC_MARGIN_VOCAB ? vms
+                                                              : margins) +
+                     (size_t)b * D;
+  int dl = 0;
+  for (int a = 0; a < D; ++a) {
+    const int v = ids[(size_t)b * D + a];
+    if (ids_valid[b]) dl += abs(v - prev_ids[(size_t)b * D + a]);
+    prev_ids[(size_t)b * D + a] = v;
+  }
+  ids_valid[b] = 1;
+  delta[b] = dl;
   float m;
   if (prm->reduction == VLAC_REDUCE_MIN) {
     m = sig[0];
@@ -361,8 +386,53 @@ __global__ void copy_spans_kernel(CopyList list, StepParams p, StepParams* prm) 
   }
 }
 
-void launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st) {
-  launch_k(copy_spans_kernel, dim3(64), dim3(256), 0, st, list, p, prm);
+// ---- the one-layer entry ----------------------------------------------------------
+
+__global__ void layer_setup_kernel(const int32_t* __restrict__ pos, int M, int S, int* __restrict__ idx,
+                                   int* __restrict__ off, int* err) {
+  pdl_wait();
+  pdl_trigger();
+  for (int i = threadIdx.x; i < M; i += blockDim.x) {
+    int p = pos[i];
+    if (p < 0 || p >= S) {
+      set_error(err, VLAC_ERR_DEVICE_CHECK);
+      p = 0;
+    }
+    idx[i] = p;
+  }
+  if (threadIdx.x == 0) {
+    off[0] = 0;
+    off[1] = M;
+  }
+}
+
+// One block per (position, head): head_dim elements, copied as 4-byte words.
+__global__ void kv_copy_kernel(uint8_t* __restrict__ cache, uint8_t* __restrict__ flat, int n_heads, int Tc,
+                               int row_bytes, bool to_cache) {
+  pdl_wait();
+  pdl_trigger();
+  const int t = blockIdx.x, h = blockIdx.y;
+  uint32_t* cw = reinterpret_cast<uint32_t*>(cache + ((size_t)h * Tc + t) * row_bytes);
+  uint32_t* fw = reinterpret_cast<uint32_t*>(flat + ((size_t)t * n_heads + h) * row_bytes);
+  for (int w = threadIdx.x; w < row_bytes / 4; w += blockDim.x) {
+    if (to_cache)
+      cw[w] = fw[w];
+    else
+      fw[w] = cw[w];
+  }
+}
+
+void launch_layer_setup(const int32_t* pos, int M, int S, int* idx, int* off, int* err, cudaStream_t st) {
+  launch_k(layer_setup_kernel, dim3(1), dim3(256), 0, st, pos, M, S, idx, off, err);
+}
+void launch_kv_copy(void* cache, void* flat, int n_heads, int Tc, int head_dim, int esz, bool to_cache,
+                    cudaStream_t st) {
+  launch_k(kv_copy_kernel, dim3(Tc, n_heads), dim3(64), 0, st, static_cast<uint8_t*>(cache),
+           static_cast<uint8_t*>(flat), n_heads, Tc, head_dim * esz, to_cache);
+}
+
+cudaError_t launch_stage(const StepParams& p, StepParams* prm, const CopyList& list, cudaStream_t st) {
+  return launch_k(copy_spans_kernel, dim3(64), dim3(256), 0, st, list, p, prm);
 }
 void launch_copies(const CopyList& list, cudaStream_t st) {
   StepParams none{};
@@ -389,26 +459,23 @@ void launch_layer_in(Rows rows, const int* off_prev, int B, int S, int hidden, f
   launch_k(layer_in_kernel<T>, dim3(S, B), dim3(kNormThreads), 0, st, rows, off_prev, hidden, H, h_seq_stride, gain, eps, A);
 }
 template <typename T>
-void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, int splits,
-                         size_t split_stride, const float* rope_cos, const float* rope_sin, T* Q, T* Kc, T* Vc,
-                         size_t kv_seq_stride, int Tc, cudaStream_t st) {
-  launch_k(qkv_epilogue_kernel<T>, dim3(S, B, 2), dim3(256), 0, st, rows, n_heads, head_dim, part, splits, split_stride,
-           rope_cos, rope_sin, Q, Kc, Vc, kv_seq_stride, Tc);
+void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, const SplitPlan& sp,
+                         const float* rope_cos, const float* rope_sin, T* Q, T* Kc, T* Vc, size_t kv_seq_stride,
+                         int Tc, cudaStream_t st) {
+  launch_k(qkv_epilogue_kernel<T>, dim3(S, B, 2), dim3(256), 0, st, rows, n_heads, head_dim, part, sp, rope_cos,
+           rope_sin, Q, Kc, Vc, kv_seq_stride, Tc);
 }
 template <typename T>
-void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part, int splits, size_t split_stride,
-                          const T* gain, float eps, T* A, cudaStream_t st) {
-  launch_k(residual_norm_kernel<T>, dim3(S, B), dim3(kNormThreads), 0, st, rows, hidden, part, splits, split_stride, gain, eps,
-           A);
+void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part, const SplitPlan& sp, const T* gain,
+                          float eps, T* A, cudaStream_t st) {
+  launch_k(residual_norm_kernel<T>, dim3(S, B), dim3(kNormThreads), 0, st, rows, hidden, part, sp, gain, eps, A);
 }
 template <typename T>
-void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, int splits, size_t split_stride, T* G,
-                   cudaStream_t st) {
-  launch_k(swiglu_kernel<T>, dim3(S, B, 4), dim3(256), 0, st, rows, ffn, part, splits, split_stride, G);
+void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, const SplitPlan& sp, T* G, cudaStream_t st) {
+  launch_k(swiglu_kernel<T>, dim3(S, B, 4), dim3(256), 0, st, rows, ffn, part, sp, G);
 }
-void launch_residual(Rows rows, int B, int S, int hidden, const float* part, int splits, size_t split_stride,
-                     cudaStream_t st) {
-  launch_k(residual_kernel, dim3(S, B, 4), dim3(256), 0, st, rows, hidden, part, splits, split_stride);
+void launch_residual(Rows rows, int B, int S, int hidden, const float* part, const SplitPlan& sp, cudaStream_t st) {
+  launch_k(residual_kernel, dim3(S, B, 4), dim3(256), 0, st, rows, hidden, part, sp);
 }
 template <typename T>
 void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
@@ -417,10 +484,62 @@ void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int 
   launch_k(decode_embed_kernel<T>, dim3(B), dim3(256), 0, st, d, D, P, hidden, vocab, n_bins, tok_emb, ids, forced,
            prm, Xd, idx_dec, ssq_out, err);
 }
-void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps, float* m_prev,
-                   uint8_t* valid, float* user_step_margin, cudaStream_t st) {
-  launch_k(finish_kernel, dim3((B + 63) / 64), dim3(64), 0, st, B, D, prm, margins, gaps, m_prev, valid,
-           user_step_margin);
+void launch_finish(int B, int D, const StepParams* prm, const float* margins, const float* gaps, const float* vms,
+                   float* m_prev, uint8_t* valid, float* user_step_margin, const int32_t* ids, int32_t* prev_ids,
+                   uint8_t* ids_valid, int32_t* delta, const uint8_t* active, cudaStream_t st) {
+  launch_k(finish_kernel, dim3((B + 63) / 64), dim3(64), 0, st, B, D, prm, margins, gaps, vms, m_prev, valid,
+           user_step_margin, ids, prev_ids, ids_valid, delta, active);
+}
+
+// Grid (chunks, B): sequence b's previous frame becomes this step's frame (16-byte
+// words where both ends allow, bytes otherwise), or, for a sequence that sat
+// the step out, its outputs are zeroed.
+__global__ void commit_kernel(int D, int n_bins, int Nv, int S, int L, size_t frame_bytes,
+                              const uint8_t* __restrict__ frames, uint8_t* __restrict__ prev,
+                              const StepParams* __restrict__ prm, const uint8_t* __restrict__ active, StepOutputs o) {
+  pdl_wait();
+  pdl_trigger();
+  const int b = blockIdx.y;
+  const size_t tid = (size_t)blockIdx.x * blockDim.x + threadIdx.x, nth = (size_t)gridDim.x * blockDim.x;
+  if (!(prm->has_active && active && !active[b])) {
+    const uint8_t* src = frames + (size_t)b * frame_bytes;
+    uint8_t* dst = prev + (size_t)b * frame_bytes;
+    if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0) {
+      const size_t nv = frame_bytes / 16;
+      for (size_t i = tid; i < nv; i += nth) reinterpret_cast<uint4*>(dst)[i] = reinterpret_cast<const uint4*>(src)[i];
+      for (size_t i = nv * 16 + tid; i < frame_bytes; i += nth) dst[i] = src[i];
+    } else {
+      for (size_t i = tid; i < frame_bytes; i += nth) dst[i] = src[i];
+    }
+    return;
+  }
+  for (size_t i = tid; i < (size_t)D; i += nth) {
+    o.ids[(size_t)b * D + i] = 0;
+    o.margins[(size_t)b * D + i] = 0.f;
+    o.gaps[(size_t)b * D + i] = 0.f;
+    if (o.entropy) o.entropy[(size_t)b * D + i] = 0.f;
+    if (o.vocab_margin) o.vocab_margin[(size_t)b * D + i] = 0.f;
+  }
+  for (size_t i = tid; i < (size_t)D * n_bins; i += nth) o.logits[(size_t)b * D * n_bins + i] = 0.f;
+  for (size_t i = tid; i < (size_t)Nv; i += nth) o.mask[(size_t)b * Nv + i] = 0;
+  for (size_t i = tid; i < (size_t)S; i += nth) o.idx[(size_t)b * S + i] = 0;
+  for (size_t i = tid; i < (size_t)L; i += nth) o.M[(size_t)b * L + i] = 0;
+  for (size_t i = tid; i < (size_t)Nv; i += nth) {
+    if (o.relevance) o.relevance[(size_t)b * Nv + i] = 0.f;
+    if (o.relevant) o.relevant[(size_t)b * Nv + i] = 0;
+  }
+  if (tid == 0) {
+    o.recomputed[b] = 0;
+    o.gate_auto[b] = 0;
+    o.step_margin[b] = 0.f;
+  }
+}
+
+void launch_commit(int B, int D, int n_bins, int Nv, int S, int L, size_t frame_bytes, const uint8_t* frames,
+                   uint8_t* prev, const StepParams* prm, const uint8_t* active, const StepOutputs& o,
+                   cudaStream_t st) {
+  launch_k(commit_kernel, dim3(16, B), dim3(256), 0, st, D, n_bins, Nv, S, L, frame_bytes, frames, prev, prm, active,
+           o);
 }
 
 #define VLAC_INST(T)                                                                                              \
@@ -429,11 +548,11 @@ void launch_finish(int B, int D, const StepParams* prm, const float* margins, co
                                 const T*, const float*, const T*, const T*, int*, cudaStream_t);                 \
   template void launch_layer_in<T>(Rows, const int*, int, int, int, float*, size_t, const T*, float, T*,          \
                                    cudaStream_t);                                                                 \
-  template void launch_qkv_epilogue<T>(Rows, int, int, int, int, const float*, int, size_t, const float*,         \
+  template void launch_qkv_epilogue<T>(Rows, int, int, int, int, const float*, const SplitPlan&, const float*,  \
                                        const float*, T*, T*, T*, size_t, int, cudaStream_t);                      \
-  template void launch_residual_norm<T>(Rows, int, int, int, const float*, int, size_t, const T*, float, T*,      \
+  template void launch_residual_norm<T>(Rows, int, int, int, const float*, const SplitPlan&, const T*, float, T*, \
                                         cudaStream_t);                                                            \
-  template void launch_swiglu<T>(Rows, int, int, int, const float*, int, size_t, T*, cudaStream_t);               \
+  template void launch_swiglu<T>(Rows, int, int, int, const float*, const SplitPlan&, T*, cudaStream_t);          \
   template void launch_decode_embed<T>(int, int, int, int, int, int, int, const T*, const int32_t*,               \
                                        const int32_t*, const StepParams*, float*, int*, float*, int*, cudaStream_t);
 VLAC_INST(float)

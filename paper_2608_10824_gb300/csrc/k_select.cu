@@ -4,14 +4,21 @@
 // I_t and I_{t-1}; a patch is static when the similarity is above tau.  The
 // similarity vector is the raw uint8 RGB values of the patch, and the
 // comparison against tau = num/den is decided exactly in integers.
+// Sec. III-B, Stage 2 (optional): the top_k patches by the previous step's
+// text-to-vision relevance are taken out of the static set; the rest is the
+// reusable set.
 // Algorithm 1: m_{t-1} < theta_m (strict) invalidates the cache and runs the
-// full pass; otherwise Stage 3 reuses, at layer l, the floor(s_l * |S| / 1000)
-// most similar static patches and recomputes the rest.
+// full pass; otherwise Stage 3 reuses, at layer l, the floor(s_l * |R| / 1000)
+// most similar reusable patches and recomputes the rest.
+#include <mutex>
+
 #include "internal.cuh"
 
 namespace vlac {
 
 typedef unsigned __int128 u128;
+
+constexpr int kMaxSelectDevices = 64;
 
 // cos > num/den, exact.  Both patches all-zero: cos = 1; exactly one: cos = 0.
 __device__ __forceinline__ bool cos_above(uint32_t d, uint32_t na, uint32_t nb, uint32_t num, uint32_t den) {
@@ -79,16 +86,20 @@ __global__ void patch_stats_kernel(const uint8_t* __restrict__ frames, const uin
   }
 }
 
-// One block per sequence: gate decision, reuse ranking and the ordered
-// recompute list.  idx = [non-static positions ascending] ++ [static patches,
-// least similar first], so the rows recomputed at layer l are idx[0 .. M[l]).
+// One block per sequence: gate decision, Stage-2 removal, reuse ranking and
+// the ordered recompute list.  idx = [positions that are not reusable,
+// ascending] ++ [reusable patches, least similar first], so the rows
+// recomputed at layer l are idx[0 .. M[l]).
 __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __restrict__ mask,
                               const uint8_t* __restrict__ valid, const float* __restrict__ m_prev,
                               const StepParams* __restrict__ prm, const int8_t* __restrict__ override_,
                               int Nv, int S, int L, int P, int parallel, int n_action, uint8_t* __restrict__ full_out,
                               int* __restrict__ idx, int* __restrict__ M, int* __restrict__ emit_slot,
                               uint8_t* __restrict__ user_recomputed, uint8_t* __restrict__ user_gate_auto,
-                              int* __restrict__ user_idx, int* __restrict__ user_M) {
+                              int* __restrict__ user_idx, int* __restrict__ user_M,
+                              const uint8_t* __restrict__ active, const float* __restrict__ rel,
+                              uint8_t* __restrict__ rel_valid, const uint8_t* __restrict__ s2_forced,
+                              uint8_t* __restrict__ relevant, float* __restrict__ rel_out) {
   pdl_wait();
   pdl_trigger();
   extern __shared__ uint8_t smem[];
@@ -98,6 +109,17 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
   __shared__ int s_full;
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
+  if (prm->has_active && active && !active[b]) {
+    // the sequence sits this step out: no rows at any layer
+    if (tid == 0) {
+      full_out[b] = 0;
+      emit_slot[b] = 0;
+      if (user_recomputed) user_recomputed[b] = 0;
+      if (user_gate_auto) user_gate_auto[b] = 0;
+    }
+    for (int l = tid; l < L; l += blockDim.x) M[(size_t)b * L + l] = 0;
+    return;
+  }
   if (tid == 0) {
     const bool ok = valid[b] != 0;
     const bool gate = !ok || m_prev[b] < prm->tau_margin;
@@ -113,6 +135,29 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
     s_st[v] = stats[(size_t)b * Nv + v];
     s_stat[v] = mask[(size_t)b * Nv + v];
   }
+  // Stage 2: patch v is relevant when fewer than top_k patches rank before it
+  // (higher relevance, or equal relevance and lower index)
+  const int top_k = prm->s2_top_k;
+  const bool s2 = top_k > 0 && rel && rel_valid[b];
+  for (int v = tid; v < Nv; v += blockDim.x) {
+    bool r = false;
+    if (s2) {
+      const float* rb = rel + (size_t)b * Nv;
+      const float rv = rb[v];
+      int before = 0;
+      for (int u = 0; u < Nv; ++u) {
+        const float ru = rb[u];
+        before += (ru > rv || (ru == rv && u < v)) ? 1 : 0;
+      }
+      r = before < top_k;
+    }
+    // lock-step replay: the caller's set is applied, the own one reported
+    const bool apply = (top_k > 0 && prm->has_s2_forced && s2_forced) ? s2_forced[(size_t)b * Nv + v] != 0 : r;
+    if (apply) s_stat[v] = 0;
+    if (relevant) relevant[(size_t)b * Nv + v] = r;
+    if (top_k == 0 && rel_out) rel_out[(size_t)b * Nv + v] = 0.f;
+  }
+  if (top_k == 0 && rel_valid && tid == 0) rel_valid[b] = 0;  // nothing measured this step
   __syncthreads();
   const bool full = s_full != 0;
   int* idx_b = idx + (size_t)b * S;
@@ -128,7 +173,7 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
     if (tid == 0) s_ns = 0;
     __syncthreads();
     int local = 0;
-    for (int v = tid; v < Nv; v += blockDim.x) local += s_stat[v];
+    for (int v = tid; v < Nv; v += blockDim.x) local += s_stat[v];  // |R|
     if (local) atomicAdd(&s_ns, local);
     for (int v = tid; v < Nv; v += blockDim.x) {
       if (!s_stat[v]) continue;
@@ -177,24 +222,51 @@ __global__ void plan_kernel(const int* __restrict__ M, int B, int L, int* __rest
   }
 }
 
-void launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid, const StepParams* prm,
-                        int B, int n_views, int img_h, int img_w, int patch, int3* stats, uint8_t* mask,
-                        uint8_t* user_mask, cudaStream_t st) {
+cudaError_t launch_patch_stats(const uint8_t* frames, const uint8_t* prev, const uint8_t* valid,
+                               const StepParams* prm, int B, int n_views, int img_h, int img_w, int patch,
+                               int3* stats, uint8_t* mask, uint8_t* user_mask, cudaStream_t st) {
   const int Nv = n_views * (img_h / patch) * (img_w / patch);
   dim3 grid((Nv + 7) / 8, B);
-  launch_k(patch_stats_kernel, grid, dim3(256), 0, st, frames, prev, valid, prm, n_views, img_h, img_w, patch, Nv,
+  return launch_k(patch_stats_kernel, grid, dim3(256), 0, st, frames, prev, valid, prm, n_views, img_h, img_w, patch, Nv,
            stats, mask, user_mask);
 }
 
-void launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
-                   const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
-                   int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
-                   uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
-                   cudaStream_t st) {
-  const size_t smem = (size_t)Nv * (sizeof(int3) + sizeof(int) + 1) + 16;
-  launch_k(select_kernel, dim3(B), dim3(512), smem, st, stats, mask, valid, m_prev, prm, override_, Nv, S, L, P,
-           parallel, n_action, full, idx, M, emit_slot, user_recomputed, user_gate_auto, user_idx, user_M);
-  launch_k(plan_kernel, dim3(1), dim3(256), 0, st, M, B, L, off);
+// Shared memory of select_kernel for Nv patches: the int3 statistics, the
+// reuse ranks and the static flags.  Above 48 KB (Nv > 2890) the kernel needs
+// the opt-in limit, raised once per device for the largest Nv the dims
+// accept (4096 patches).
+static size_t select_smem(int Nv) { return (size_t)Nv * (sizeof(int3) + sizeof(int) + 1) + 16; }
+static cudaError_t select_smem_attr(size_t smem) {
+  if (smem <= 48u * 1024u) return cudaSuccess;
+  static std::mutex mu;
+  static bool done[kMaxSelectDevices] = {};
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxSelectDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!done[dev]) {
+    e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)select_smem(4096));
+    if (e != cudaSuccess) return e;
+    done[dev] = true;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
+                          const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
+                          int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
+                          uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
+                          const uint8_t* active, const float* rel, uint8_t* rel_valid, const uint8_t* s2_forced,
+                          uint8_t* relevant, float* rel_out, cudaStream_t st) {
+  const size_t smem = select_smem(Nv);
+  cudaError_t e = select_smem_attr(smem);
+  if (e != cudaSuccess) return e;
+  e = launch_k(select_kernel, dim3(B), dim3(512), smem, st, stats, mask, valid, m_prev, prm, override_, Nv, S, L, P,
+           parallel, n_action, full, idx, M, emit_slot, user_recomputed, user_gate_auto, user_idx, user_M, active, rel,
+           rel_valid, s2_forced, relevant, rel_out);
+  if (e != cudaSuccess) return e;
+  return launch_k(plan_kernel, dim3(1), dim3(256), 0, st, M, B, L, off);
 }
 
 }  // namespace vlac

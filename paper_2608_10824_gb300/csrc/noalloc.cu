@@ -1,8 +1,7 @@
 // Allocation-free variant of the selection stage (Stage-1 patch similarity,
 // the gate and the Stage-3 recompute order) for callers that may not allocate
-// device memory at run time: code running while a CUDA stream is being
-// captured into a graph, real-time control loops whose memory is fixed up
-// front, and host frameworks that own every device allocation themselves.
+// device memory at run time: real-time control loops whose memory is fixed
+// up front, and host frameworks that own every device allocation themselves.
 //
 // The kernels are the ones vlac_step runs; only their scratch (the per-patch
 // integer statistics, the step scalars, the per-layer row offsets) lives in a
@@ -72,7 +71,7 @@ extern "C" int vlac_select_noalloc(const vlac_dims* d, int batch, const uint8_t*
   const size_t o_off = round256(o_full + (size_t)batch);
   const size_t o_emit = round256(o_off + sizeof(int) * (size_t)L * (batch + 1));
   const size_t need = round256(o_emit + sizeof(int) * (size_t)batch);
-  if (need > kNoallocScratchBytes) return VLAC_ERR_INVALID_ARG;  // beyond the fixed scratch
+  if (need > kNoallocScratchBytes) return VLAC_ERR_UNSUPPORTED;  // valid dims, beyond the fixed scratch
   StepParams p;
   memset(&p, 0, sizeof(p));
   for (int l = 0; l < L; ++l) {
@@ -94,12 +93,16 @@ extern "C" int vlac_select_noalloc(const vlac_dims* d, int batch, const uint8_t*
   int* emit = reinterpret_cast<int*>(base + o_emit);
   // every scratch entry a kernel reads is written earlier in this call, so
   // nothing has to be cleared first
+  // each launch's own status: an error left over from the caller's earlier
+  // work is neither reported as this call's nor cleared
   CopyList none{};
-  launch_stage(p, prm, none, st);
-  launch_patch_stats(frames, prev_frames, valid, prm, batch, d->n_views, d->img_h, d->img_w, d->patch, stats,
-                     static_mask, nullptr, st);
-  launch_select(stats, static_mask, valid, m_prev, prm, gate_override, batch, Nv, S, L, P, d->parallel,
-                d->n_action, full, idx, M, off, emit, recomputed, nullptr, nullptr, nullptr, st);
-  if (cudaGetLastError() != cudaSuccess) return VLAC_ERR_CUDA;
+  if (launch_stage(p, prm, none, st) != cudaSuccess) return VLAC_ERR_CUDA;
+  if (launch_patch_stats(frames, prev_frames, valid, prm, batch, d->n_views, d->img_h, d->img_w, d->patch, stats,
+                         static_mask, nullptr, st) != cudaSuccess)
+    return VLAC_ERR_CUDA;
+  if (launch_select(stats, static_mask, valid, m_prev, prm, gate_override, batch, Nv, S, L, P, d->parallel,
+                    d->n_action, full, idx, M, off, emit, recomputed, nullptr, nullptr, nullptr, nullptr, nullptr,
+                    nullptr, nullptr, nullptr, nullptr, st) != cudaSuccess)
+    return VLAC_ERR_CUDA;
   return VLAC_OK;
 }

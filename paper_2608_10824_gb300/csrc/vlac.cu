@@ -48,11 +48,16 @@ struct vlac_ctx {
   int n_sm = 1;
   int gemv_ns = 4;  // decode-GEMV weight ring stages (32 KB each)
   int gemv_pf_kb = 0;  // decode-GEMV L2 prefetch of the next projection, KB per CTA (measured: off is best)
+  bool use_dpass = false;  // decode passes as one persistent cooperative launch (k_dpass.cu) where supported
+  int dpass_attn_chunks = 0;  // its key ranges per (sequence, head); 0 = chosen from the SM count
+  void** dp_ptrs = nullptr;  // device: per-layer pointers [w_qkv | w_o | w_gu | w_d | g_attn | g_ffn][L]
+  unsigned* dp_bar = nullptr;  // device: the persistent pass's grid-barrier counter
   char* dmem = nullptr;  // decode-streaming copies of the projections
   std::vector<void*> dqkv, dwo, dgu, dwd;
   // weights
   char* wmem = nullptr;
   void *tok_emb, *patch_w, *proprio_w, *action_emb, *final_norm, *head_w;
+  void* head_full;  // the whole LM head [vocab][hidden]; head_w is its last n_bins rows
   std::vector<void*> attn_norm, ffn_norm, wqkv, wo, wgu, wd;
   float *rope_cos, *rope_sin;
   // TMA descriptors (bf16 only)
@@ -60,6 +65,11 @@ struct vlac_ctx {
   CUtensorMap tm_patch;
   ActMaps tm_A, tm_AO, tm_G, tm_col;
   int split_qkv = 1, split_o = 1, split_gu = 1, split_d = 1;
+  // where each projection's K-split partials go (uniform splits, or whole
+  // tiles plus K-split tail tiles when the tiles exceed one wave of SMs)
+  SplitPlan sp_qkv{}, sp_o{}, sp_gu{}, sp_d{};
+  float* part_tail = nullptr;  // compact partials of the tail tiles' later splits
+  size_t part_tail_elems = 0;
   // workspace
   char* wsmem = nullptr;
   float *X, *Xd, *part;
@@ -77,10 +87,22 @@ struct vlac_ctx {
   float* in_proprio;
   int8_t* in_override;
   int32_t* in_forced;
+  uint8_t* in_active;
+  uint8_t* in_s2_forced;
   int32_t* o_ids;
   float *o_margins, *o_gaps, *o_step_margin, *o_logits;
   uint8_t *o_recomputed, *o_gate_auto, *o_mask;
   int32_t *o_idx, *o_M;
+  float* o_rel;         // Stage-2 relevance of the step [B][Nv]
+  uint8_t* o_relevant;  // Stage-2 removal set of the step [B][Nv]
+  float* rel_part;      // Stage-2 relevance per (sequence, head) [B][n_heads][Nv]
+  bool s2_on = false;   // this step measures and applies Stage 2
+  int s2_layer = 0;
+  float *o_entropy, *o_vm;  // per action token: bin-softmax entropy, whole-vocabulary margin
+  int32_t* o_delta;         // per sequence: action delta
+  void* vh_rows;            // whole-vocabulary margin: normed action rows [rows][hidden] (T)
+  float* vh_logits;         // and their logits over the non-bin rows [rows][vocab - n_bins]
+  bool vm_on = false;       // this step computes the whole-vocabulary margin
   cudaStream_t cap_stream = nullptr;
   bool use_graph = true;
   bool fatal = false;  // a launch was refused for exceeding a workspace buffer
@@ -105,10 +127,15 @@ struct vlac_cache {
   cudaGraphExec_t gexec = nullptr;
   int eager_steps = 0;
   uint64_t graph_launches = 0;
+  int graph_sig = 0;  // what the graph was captured with: Stage 2 (0 off, 1 + layer) * 2 + the vocabulary margin
   void *K, *V;
   float* H;
   uint8_t *prev, *valid;
   float* m_prev;
+  float* rel;          // [B][Nv] the last step's Stage-2 relevance
+  uint8_t* rel_valid;  // [B] rel holds one
+  int32_t* prev_ids;   // [B][n_action] the previous step's action bins
+  uint8_t* ids_valid;  // [B] prev_ids holds them
   size_t kv_seq_stride, h_seq_stride;  // elements per sequence
 };
 
@@ -206,6 +233,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (const char* e = std::getenv("VLAC_GRAPH")) c->use_graph = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_GEMV_NS")) c->gemv_ns = std::max(2, std::min(24, std::atoi(e)));
   if (const char* e = std::getenv("VLAC_GEMV_PF_KB")) c->gemv_pf_kb = std::max(0, std::atoi(e));
+  if (const char* e = std::getenv("VLAC_DPASS")) c->use_dpass = std::atoi(e) != 0;
+  if (const char* e = std::getenv("VLAC_DPASS_ATTN_CHUNKS")) c->dpass_attn_chunks = std::max(0, std::atoi(e));
   c->d = *dims;
   const vlac_dims& d = c->d;
   c->bf16 = d.dtype == VLAC_BF16;
@@ -234,7 +263,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     wc.take(c->proprio_w, Hd * std::max(d.proprio_dim, 1) * E, base);
     wc.take(c->action_emb, (size_t)d.n_action * Hd * E, base);
     wc.take(c->final_norm, Hd * E, base);
-    wc.take(c->head_w, (size_t)d.n_bins * Hd * E, base);
+    wc.take(c->head_full, (size_t)d.vocab * Hd * E, base);
+    if (base) c->head_w = static_cast<char*>(c->head_full) + (size_t)(d.vocab - d.n_bins) * Hd * E;
     c->attn_norm.resize(L); c->ffn_norm.resize(L); c->wqkv.resize(L); c->wo.resize(L); c->wgu.resize(L); c->wd.resize(L);
     for (size_t l = 0; l < L; ++l) {
       wc.take(c->attn_norm[l], Hd * E, base);
@@ -269,8 +299,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (d.proprio_dim) ok = ok && cp(c->proprio_w, w->proprio_w, Hd * d.proprio_dim * E);
   if (d.parallel) ok = ok && cp(c->action_emb, w->action_emb, (size_t)d.n_action * Hd * E);
   ok = ok && cp(c->final_norm, w->final_norm, Hd * E);
-  ok = ok && cp(c->head_w, static_cast<const char*>(w->lm_head) + (size_t)(d.vocab - d.n_bins) * Hd * E,
-                (size_t)d.n_bins * Hd * E);
+  ok = ok && cp(c->head_full, w->lm_head, (size_t)d.vocab * Hd * E);
   for (size_t l = 0; l < L && ok; ++l) {
     char* qkv = static_cast<char*>(c->wqkv[l]);
     char* gu = static_cast<char*>(c->wgu[l]);
@@ -366,6 +395,37 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     }
   }
 
+  // ---- tail tiles: a projection with more weight tiles than one wave of
+  // CTAs (one per SM) runs whole tiles for every full wave and cuts each
+  // remaining tile's K range over the SMs the last wave would leave idle;
+  // only those tiles have more than one partial ----
+  {
+    int plan_sms = c->n_sm;
+    if (const char* e = std::getenv("VLAC_PLAN_SMS")) plan_sms = std::max(1, std::atoi(e));  // tests and sweeps
+    bool tail_on = c->bf16;
+    if (const char* e = std::getenv("VLAC_GEMM_TAIL")) tail_on = tail_on && std::atoi(e) != 0;
+    const size_t rcap = c->rows_cap;
+    auto plan = [&](int N, int K, int split) {
+      const int tiles = N / 128, kch = K / 64;
+      if (tail_on && tiles > plan_sms) {
+        const int full = (tiles / plan_sms) * plan_sms, rem = tiles - full;
+        int tail = rem ? std::min({8, kch, plan_sms / rem}) : 1;
+        if (tail >= 2) {
+          const int cps = (kch + tail - 1) / tail;
+          tail = (kch + cps - 1) / cps;  // every split gets some K
+          const int ld = rem * 128;
+          c->part_tail_elems = std::max(c->part_tail_elems, (size_t)(tail - 1) * rcap * ld);
+          return SplitPlan{full * 128, tail, rcap * (size_t)N, nullptr, rcap * (size_t)ld, ld};
+        }
+      }
+      return uniform_splits(split, rcap * (size_t)N);
+    };
+    c->sp_qkv = plan(3 * (int)Hd, (int)Hd, c->split_qkv);
+    c->sp_o = plan((int)Hd, (int)Hd, c->split_o);
+    c->sp_gu = plan(2 * (int)F, (int)Hd, c->split_gu);
+    c->sp_d = plan((int)Hd, (int)F, c->split_d);
+  }
+
   // ---- workspace ----
   const size_t rc_ = c->rows_cap, Bm = d.max_batch;
   // every GEMM writes splits x rows_cap x N fp32 partials into `part`
@@ -378,6 +438,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->X, rc_ * Hd * 4, base);
     sc.take(c->Xd, Bm * Hd * 4, base);
     sc.take(c->part, rc_ * part_n * 4, base);
+    sc.take(c->part_tail, std::max(c->part_tail_elems, (size_t)4) * 4, base);
     sc.take(c->A, rc_ * Hd * E, base);
     sc.take(c->Q, rc_ * Hd * E, base);
     sc.take(c->AO, rc_ * Hd * E, base);
@@ -399,12 +460,16 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->attn_cnt, Bm * d.n_heads * sizeof(unsigned), base);
     sc.take(c->ssq_a, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
     sc.take(c->ssq_b, Bm * std::max((size_t)c->n_sm, Hd / kDecodeRowsPerCta) * 4, base);
+    sc.take(c->dp_ptrs, 6 * L * sizeof(void*), base);
+    sc.take(c->dp_bar, sizeof(unsigned), base);
     const size_t fbytes = (size_t)d.n_views * d.img_h * d.img_w * 3;
     sc.take(c->in_frames, Bm * fbytes, base);
     sc.take(c->in_prompt, Bm * d.n_text * 4, base);
     sc.take(c->in_proprio, Bm * std::max(d.proprio_dim, 1) * 4, base);
     sc.take(c->in_override, Bm, base);
     sc.take(c->in_forced, Bm * d.n_action * 4, base);
+    sc.take(c->in_active, Bm, base);
+    sc.take(c->in_s2_forced, Bm * c->Nv, base);
     sc.take(c->o_ids, Bm * d.n_action * 4, base);
     sc.take(c->o_margins, Bm * d.n_action * 4, base);
     sc.take(c->o_gaps, Bm * d.n_action * 4, base);
@@ -415,6 +480,15 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->o_mask, Bm * c->Nv, base);
     sc.take(c->o_idx, Bm * c->S * 4, base);
     sc.take(c->o_M, Bm * L * 4, base);
+    sc.take(c->o_rel, Bm * c->Nv * 4, base);
+    sc.take(c->o_relevant, Bm * c->Nv, base);
+    sc.take(c->rel_part, Bm * d.n_heads * c->Nv * 4, base);
+    sc.take(c->o_entropy, Bm * d.n_action * 4, base);
+    sc.take(c->o_vm, Bm * d.n_action * 4, base);
+    sc.take(c->o_delta, Bm * 4, base);
+    const size_t head_rows = Bm * (d.parallel ? d.n_action : 1);
+    sc.take(c->vh_rows, head_rows * Hd * E, base);
+    sc.take(c->vh_logits, head_rows * std::max(d.vocab - d.n_bins, 1) * 4, base);
   };
   plan_s(nullptr);
   if (cudaMalloc(&c->wsmem, sc.off) != cudaSuccess) {
@@ -427,6 +501,19 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     std::vector<int> od(Bm + 1);
     for (size_t b = 0; b <= Bm; ++b) od[b] = (int)b;
     if (cudaMemcpy(c->off_dec, od.data(), od.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(VLAC_ERR_CUDA);
+  }
+  if (c->bf16 && !c->dqkv.empty()) {  // per-layer pointers of the persistent decode pass
+    std::vector<void*> pp(6 * L);
+    for (size_t l = 0; l < L; ++l) {
+      pp[l] = c->dqkv[l];
+      pp[L + l] = c->dwo[l];
+      pp[2 * L + l] = c->dgu[l];
+      pp[3 * L + l] = c->dwd[l];
+      pp[4 * L + l] = c->attn_norm[l];
+      pp[5 * L + l] = c->ffn_norm[l];
+    }
+    if (cudaMemcpy(c->dp_ptrs, pp.data(), pp.size() * sizeof(void*), cudaMemcpyHostToDevice) != cudaSuccess)
       return fail(VLAC_ERR_CUDA);
   }
   if (cudaMallocHost(&c->err_host, sizeof(int)) != cudaSuccess) {
@@ -465,8 +552,9 @@ static size_t cache_layout(const vlac_ctx* c, int B, char* base, vlac_cache* k) 
   void* K;
   void* V;
   float* H;
-  uint8_t *prev, *valid;
-  float* m_prev;
+  uint8_t *prev, *valid, *rel_valid, *ids_valid;
+  float *m_prev, *rel;
+  int32_t* prev_ids;
   const size_t kv = (size_t)d.n_layers * d.n_heads * c->Tc * d.head_dim;
   const size_t hs = (size_t)d.n_layers * c->S * d.hidden;
   cv.take(K, B * kv * c->esz, base);
@@ -475,8 +563,14 @@ static size_t cache_layout(const vlac_ctx* c, int B, char* base, vlac_cache* k) 
   cv.take(prev, (size_t)B * d.n_views * d.img_h * d.img_w * 3, base);
   cv.take(m_prev, (size_t)B * 4, base);
   cv.take(valid, (size_t)B, base);
+  cv.take(rel, (size_t)B * c->Nv * 4, base);
+  cv.take(rel_valid, (size_t)B, base);
+  cv.take(prev_ids, (size_t)B * d.n_action * 4, base);
+  cv.take(ids_valid, (size_t)B, base);
   if (k) {
     k->K = K; k->V = V; k->H = H; k->prev = prev; k->m_prev = m_prev; k->valid = valid;
+    k->rel = rel; k->rel_valid = rel_valid;
+    k->prev_ids = prev_ids; k->ids_valid = ids_valid;
     k->kv_seq_stride = kv;
     k->h_seq_stride = hs;
   }
@@ -519,8 +613,15 @@ extern "C" int vlac_cache_destroy(vlac_cache* k) {
 extern "C" int vlac_reset(vlac_cache* k, int seq, void* stream) {
   if (!k || seq < -1 || seq >= k->B) return VLAC_ERR_INVALID_ARG;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (seq < 0) CK(cudaMemsetAsync(k->valid, 0, (size_t)k->B, st));
-  else CK(cudaMemsetAsync(k->valid + seq, 0, 1, st));
+  if (seq < 0) {
+    CK(cudaMemsetAsync(k->valid, 0, (size_t)k->B, st));
+    CK(cudaMemsetAsync(k->rel_valid, 0, (size_t)k->B, st));
+    CK(cudaMemsetAsync(k->ids_valid, 0, (size_t)k->B, st));
+  } else {
+    CK(cudaMemsetAsync(k->valid + seq, 0, 1, st));
+    CK(cudaMemsetAsync(k->rel_valid + seq, 0, 1, st));
+    CK(cudaMemsetAsync(k->ids_valid + seq, 0, 1, st));
+  }
   return VLAC_OK;
 }
 
@@ -575,28 +676,90 @@ void dgemv(vlac_ctx* c, const DGemv& a_in, int epi, int nb, cudaStream_t st) {
 
 template <typename T>
 void gemm(vlac_ctx* c, const ActMaps* tmA, const CUtensorMap* tmW, const T* A, const void* W, const int* m_ptr,
-          int N, int K, int splits, cudaStream_t st) {
-  const int kch = c->bf16 ? K / 64 : 1, cps = (kch + splits - 1) / splits;
-  if ((size_t)splits * c->rows_cap * N > c->part_elems ||  // never launch a GEMM whose partials do not fit,
-      (splits - 1) * cps >= kch) {                          // or one with a split that has no K range
+          int N, int K, const SplitPlan& sp, cudaStream_t st) {
+  const int kch = c->bf16 ? K / 64 : 1, cps = (kch + sp.tail - 1) / sp.tail;
+  const bool compact = sp.tail_ld != 0;
+  const size_t slots = compact ? 1 : (size_t)sp.tail;
+  if (slots * c->rows_cap * N > c->part_elems ||  // never launch a GEMM whose partials do not fit,
+      (compact && (size_t)(sp.tail - 1) * c->rows_cap * sp.tail_ld > c->part_tail_elems) ||
+      (sp.tail - 1) * cps >= kch || (!c->bf16 && (sp.tail != 1 || sp.full_cols))) {  // or a split without K
     c->fatal = true;
     return;
   }
   ProfScope ps(c, VLAC_PROF_PREFIX_GEMM, (double)N * K * sizeof(T), st);
   if constexpr (sizeof(T) == 2) {
-    launch_gemm_tc(tmA, tmW, m_ptr, c->rows_cap, N, K, splits, c->part, c->err, c->wait_limit, st);
+    launch_gemm_tc(tmA, tmW, m_ptr, c->rows_cap, N, K, sp, c->part, c->err, c->wait_limit, st);
   } else {
     launch_gemm_simt<T>(A, static_cast<const T*>(W), m_ptr, c->rows_cap, N, K, c->part, st);
   }
   c->launches += 1;
 }
 
+// One decoder layer of the prefix pass for the rows `rl` of B sequences:
+// the input norm (rows joining at this layer start from H, rows computed at
+// the previous layer record their input there; H NULL at layer 0), q/k/v
+// with RoPE and the K/V scatter into Kc_l / Vc_l (this layer of the cache),
+// the mixed-cache attention, o-projection + residual, the MLP norm, gate/up +
+// SwiGLU and down + residual.
+template <typename T>
+void prefix_layer(vlac_ctx* c, const Rows& rl, const int* off_prev, int B, int l, float* H, size_t h_seq_stride,
+                  T* Kc_l, T* Vc_l, size_t kv_seq_stride, cudaStream_t st) {
+  const vlac_dims& d = c->d;
+  const int S = c->S, Hd = d.hidden, F = d.ffn, nh = d.n_heads, hd = d.head_dim;
+  const float eps = d.rms_eps;
+  T* A = static_cast<T*>(c->A);
+  T* Q = static_cast<T*>(c->Q);
+  T* AO = static_cast<T*>(c->AO);
+  T* G = static_cast<T*>(c->G);
+  auto W = [](void* p) { return static_cast<const T*>(p); };
+  auto with_tail = [&](SplitPlan p) {
+    p.tail_p = c->part_tail;
+    return p;
+  };
+  const SplitPlan sq = with_tail(c->sp_qkv), so = with_tail(c->sp_o), sg = with_tail(c->sp_gu), sd = with_tail(c->sp_d);
+  const int* ml = rl.off + B;
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_layer_in<T>(rl, off_prev, B, S, Hd, H, h_seq_stride, W(c->attn_norm[l]), eps, A, st);
+  }
+  gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_qkv[l] : nullptr, A, c->wqkv[l], ml, 3 * Hd, Hd, sq, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_qkv_epilogue<T>(rl, B, S, nh, hd, c->part, sq, c->rope_cos, c->rope_sin, Q, Kc_l, Vc_l, kv_seq_stride,
+                           c->Tc, st);
+  }
+  {
+    ProfScope ps_(c, VLAC_PROF_PREFIX_ATTN, 0, st);
+    launch_attention<T>(rl, B, S, nh, hd, Q, Kc_l, Vc_l, kv_seq_stride, c->Tc, c->P, d.parallel, d.n_action, AO, st);
+  }
+  gemm<T>(c, &c->tm_AO, c->bf16 ? &c->tm_o[l] : nullptr, AO, c->wo[l], ml, Hd, Hd, so, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_residual_norm<T>(rl, B, S, Hd, c->part, so, W(c->ffn_norm[l]), eps, A, st);
+  }
+  gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_gu[l] : nullptr, A, c->wgu[l], ml, 2 * F, Hd, sg, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_swiglu<T>(rl, B, S, F, c->part, sg, G, st);
+  }
+  gemm<T>(c, &c->tm_G, c->bf16 ? &c->tm_d[l] : nullptr, G, c->wd[l], ml, Hd, F, sd, st);
+  {
+    ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
+    launch_residual(rl, B, S, Hd, c->part, sd, st);
+  }
+  c->launches += 6;
+}
+
 // The step body: reads only the staged inputs and writes only the context's
 // output buffers, so its launches can be captured once and replayed.
 template <typename T>
 int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
-  vlac_step_out outv{c->o_ids, c->o_margins, c->o_gaps, c->o_recomputed, c->o_step_margin, c->o_gate_auto,
-                     c->o_logits, c->o_mask, c->o_idx, c->o_M};
+  vlac_step_out outv{c->o_ids,   c->o_margins, c->o_gaps, c->o_recomputed, c->o_step_margin, c->o_gate_auto,
+                     c->o_logits, c->o_mask,    c->o_idx,  c->o_M,         c->o_rel,         c->o_relevant,
+                     c->o_entropy, c->o_vm,    c->o_delta};
+  VocabHead vh{c->head_full, c->d.vocab - c->d.n_bins, c->vh_rows, c->vh_logits, c->o_vm};
+  const VocabHead* vhp = c->vm_on ? &vh : nullptr;
+  const int head_launches = c->vm_on ? (vh.n_rows ? 5 : 4) : 2;
   const vlac_step_out* out = &outv;
   const uint8_t* frames = c->in_frames;
   const int32_t* prompt = c->in_prompt;
@@ -626,7 +789,8 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_select(c->stats, c->mask, k->valid, k->m_prev, c->prm, ovr, B, c->Nv, S, L, c->P, d.parallel, D, c->full,
-                  c->idx, c->M, c->off, c->emit_slot, out->recomputed, out->gate_auto, out->idx, out->M, st);
+                  c->idx, c->M, c->off, c->emit_slot, out->recomputed, out->gate_auto, out->idx, out->M,
+                  c->in_active, k->rel, k->rel_valid, c->in_s2_forced, out->relevant, out->relevance, st);
   }
   c->launches += 3;
 
@@ -637,7 +801,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
     ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
     launch_im2col<T>(r0, B, S, frames, d.n_views, d.img_h, d.img_w, d.patch, c->kpad, col, st);
   }
-  gemm<T>(c, &c->tm_col, &c->tm_patch, col, c->patch_w, m0, Hd, c->kpad, 1, st);
+  gemm<T>(c, &c->tm_col, &c->tm_patch, col, c->patch_w, m0, Hd, c->kpad, uniform_splits(1, c->rows_cap * Hd), st);
   {
     ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
     launch_embed<T>(r0, B, S, Hd, c->Nv, c->P, c->has_p, d.proprio_dim, d.n_text, d.vocab, prompt, proprio,
@@ -645,52 +809,30 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   }
   c->launches += 2;
 
-  const size_t rs = (size_t)c->rows_cap;
   for (int l = 0; l < L; ++l) {
     Rows rl{c->off + (size_t)l * (B + 1), c->idx, S, c->X};
-    const int* ml = rl.off + B;
     const int* off_prev = l == 0 ? rl.off : c->off + (size_t)(l - 1) * (B + 1);
-    {
-      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_layer_in<T>(rl, off_prev, B, S, Hd, l == 0 ? nullptr : k->H + (size_t)l * S * Hd, k->h_seq_stride,
-                         W(c->attn_norm[l]), eps, A, st);
-    }
-    gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_qkv[l] : nullptr, A, c->wqkv[l], ml, 3 * Hd, Hd, c->split_qkv, st);
-    {
-      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_qkv_epilogue<T>(rl, B, S, nh, hd, c->part, c->split_qkv, rs * 3 * Hd, c->rope_cos, c->rope_sin, Q,
-                             Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, st);
-    }
-    {
+    prefix_layer<T>(c, rl, off_prev, B, l, l == 0 ? nullptr : k->H + (size_t)l * S * Hd, k->h_seq_stride,
+                    Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, st);
+    if (c->s2_on && l == c->s2_layer) {
+      // Stage 2: the text rows' attention on the visual keys of this layer (Q
+      // still holds this layer's rows)
       ProfScope ps_(c, VLAC_PROF_PREFIX_ATTN, 0, st);
-      launch_attention<T>(rl, B, S, nh, hd, Q, Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, c->Tc, c->P,
-                          d.parallel, D, AO, st);
+      if (launch_relevance<T>(rl, B, nh, hd, Q, Kc + l * kv_layer, k->kv_seq_stride, c->Tc, c->Nv,
+                              1 + c->Nv + c->has_p, c->P, c->rel_part, k->rel, out->relevance, k->rel_valid,
+                              c->prm, c->in_active, st))
+        c->fatal = true;
+      c->launches += 2;
     }
-    gemm<T>(c, &c->tm_AO, c->bf16 ? &c->tm_o[l] : nullptr, AO, c->wo[l], ml, Hd, Hd, c->split_o, st);
-    {
-      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_residual_norm<T>(rl, B, S, Hd, c->part, c->split_o, rs * Hd, W(c->ffn_norm[l]), eps, A, st);
-    }
-    gemm<T>(c, &c->tm_A, c->bf16 ? &c->tm_gu[l] : nullptr, A, c->wgu[l], ml, 2 * F, Hd, c->split_gu, st);
-    {
-      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_swiglu<T>(rl, B, S, F, c->part, c->split_gu, rs * 2 * F, G, st);
-    }
-    gemm<T>(c, &c->tm_G, c->bf16 ? &c->tm_d[l] : nullptr, G, c->wd[l], ml, Hd, F, c->split_d, st);
-    {
-      ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-      launch_residual(rl, B, S, Hd, c->part, c->split_d, rs * Hd, st);
-    }
-    c->launches += 6;
   }
   // action head on the prefix pass: the last text row, or the parallel action block
   {
     ProfScope ps_(c, VLAC_PROF_HEAD, 0, st);
     launch_head2<T>(c->X, c->emit_slot, (size_t)S * Hd, d.parallel ? D : 1, B, Hd, nb, W(c->final_norm),
                     W(c->head_w), eps, c->logits_ws, D, 0, out->action_ids, out->margins, out->logit_gap, out->logits,
-                    st);
+                    out->entropy, vhp, st);
   }
-  c->launches += 2;
+  c->launches += head_launches;
 
   if (!d.parallel) {
     // autoregressive decode: one row per sequence, fused GEMVs
@@ -712,7 +854,70 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         g.pf_bytes = (uint32_t)c->gemv_pf_kb * 1024;
         if (!g.pf_bytes) g.pf_W = nullptr;
       };
-      for (int l = 0; l < L; ++l) {
+      // all layers as one persistent cooperative launch (VLAC_DPASS=1, bf16,
+      // head_dim 128, up to two sequences); else one launch per projection
+      bool dp_done = false;
+      if constexpr (sizeof(T) == 2) {
+        if (c->use_dpass && dpass_supported((int)Hd, (int)F, nh, hd, B, c->gemv_ns)) {
+          DPass p{};
+          const bf16* const* pp = reinterpret_cast<const bf16* const*>(c->dp_ptrs);
+          p.w_qkv = pp;
+          p.w_o = pp + L;
+          p.w_gu = pp + 2 * L;
+          p.w_d = pp + 3 * L;
+          p.g_attn = pp + 4 * L;
+          p.g_ffn = pp + 5 * L;
+          p.L = L;
+          p.hidden = (int)Hd;
+          p.ffn = (int)F;
+          p.n_heads = nh;
+          p.Tc = c->Tc;
+          p.pos = pos;
+          p.ns = c->gemv_ns;
+          p.n_ssq0 = (int)Hd / kDecodeRowsPerCta;
+          p.eps = eps;
+          p.scale = 1.0f / sqrtf((float)hd);
+          p.rope_cos = c->rope_cos;
+          p.rope_sin = c->rope_sin;
+          p.X = c->Xd;
+          p.Q = Q;
+          p.AO = AO;
+          p.G = G;
+          p.Kc = Kc;
+          p.Vc = Vc;
+          p.kv_layer = kv_layer;
+          p.kv_seq_stride = k->kv_seq_stride;
+          p.ssq0 = c->ssq_b;
+          p.ssq = c->ssq_a;
+          p.bar = c->dp_bar;
+          p.err = c->err;
+          {
+            // key ranges per (sequence, head): enough items for the SMs, at
+            // most one per 32 keys (the partial buffer's capacity) and 8
+            const int cap = std::min(8, (c->Tc + 31) / 32);
+            int chunks = std::max(1, std::min(cap, c->n_sm / std::max(1, B * nh)));
+            if (c->dpass_attn_chunks > 0) chunks = std::min(cap, c->dpass_attn_chunks);
+            p.attn_chunks = chunks;
+            p.part_stride = (size_t)((c->Tc + 31) / 32) * (hd + 2);
+            p.attn_part = c->attn_part;
+            p.attn_cnt = c->attn_cnt;
+          }
+          int rc_dp;
+          {
+            ProfScope ps_(c, VLAC_PROF_DECODE_GEMV, (double)L * (4.0 * Hd * Hd + 3.0 * F * Hd) * 2, st);
+            rc_dp = launch_dpass(p, B, c->n_sm, st);
+          }
+          if (rc_dp == VLAC_OK) {
+            c->launches += 1;
+            dp_done = true;
+          } else if (rc_dp == VLAC_ERR_UNSUPPORTED) {
+            (void)cudaGetLastError();  // one CTA per SM does not fit: the per-projection chain runs instead
+          } else {
+            c->fatal = true;
+          }
+        }
+      }
+      for (int l = 0; l < L && !dp_done; ++l) {
         DGemv g{};
         g.eps = eps;
         g.n_heads = nh;
@@ -786,18 +991,26 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
       {
         ProfScope ps_(c, VLAC_PROF_HEAD, 0, st);
         launch_head2<T>(c->Xd, nullptr, Hd, 1, B, Hd, nb, W(c->final_norm), W(c->head_w), eps, c->logits_ws, D, a,
-                        out->action_ids, out->margins, out->logit_gap, out->logits, st);
+                        out->action_ids, out->margins, out->logit_gap, out->logits, out->entropy, vhp, st);
       }
-      c->launches += 2;
+      c->launches += head_launches;
     }
   }
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
-    launch_finish(B, D, c->prm, out->margins, out->logit_gap, k->m_prev, k->valid, out->step_margin, st);
+    launch_finish(B, D, c->prm, out->margins, out->logit_gap, out->vocab_margin, k->m_prev, k->valid, out->step_margin,
+                  out->action_ids, k->prev_ids, k->ids_valid, out->action_delta, c->in_active, st);
   }
-  c->launches += 1;
-  const size_t fb = (size_t)d.n_views * d.img_h * d.img_w * 3;
-  CK(cudaMemcpyAsync(k->prev, frames, (size_t)B * fb, cudaMemcpyDeviceToDevice, st));
+  {
+    ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
+    const StepOutputs so{out->action_ids, out->margins,   out->logit_gap,   out->logits, out->step_margin,
+                         out->recomputed, out->gate_auto, out->static_mask, out->idx,    out->M,
+                         out->relevance,  out->relevant,  out->entropy,     out->vocab_margin,
+                         out->action_delta};
+    launch_commit(B, D, nb, c->Nv, S, L, (size_t)d.n_views * d.img_h * d.img_w * 3, frames, k->prev, c->prm,
+                  c->in_active, so, st);
+  }
+  c->launches += 2;
   CK(cudaMemcpyAsync(c->err_host, c->err, sizeof(int), cudaMemcpyDeviceToHost, st));
   CK(cudaGetLastError());
   return VLAC_OK;
@@ -812,6 +1025,17 @@ int run_body(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
 // the second captures the body into a graph, which every later step replays.
 int run_step(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   if (!c->use_graph || c->prof_on) return run_body(c, k, st);
+  const int sig = (c->s2_on ? 1 + c->s2_layer : 0) * 2 + (c->vm_on ? 1 : 0);
+  if (k->gexec && k->graph_sig != sig) {
+    // Stage 2 or the whole-vocabulary margin switched on or off, or Stage 2
+    // moved to another layer: the launch list
+    // differs, so the graph is captured again (after one eager step)
+    cudaGraphExecDestroy(k->gexec);
+    cudaGraphDestroy(k->graph);
+    k->gexec = nullptr;
+    k->graph = nullptr;
+    k->eager_steps = 0;
+  }
   if (!k->gexec) {
     if (k->eager_steps++ == 0) return run_body(c, k, st);
     const uint64_t n0 = c->launches;
@@ -831,6 +1055,7 @@ int run_step(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
       return VLAC_ERR_CUDA;
     }
     k->graph = g;
+    k->graph_sig = sig;
     k->graph_launches = c->launches - n0;
     c->launches = n0;
   }
@@ -859,7 +1084,7 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   }
   int mk = opts ? opts->margin_kind : VLAC_MARGIN_PROB;
   int red = opts ? opts->reduction : VLAC_REDUCE_DEFAULT;
-  if (mk != VLAC_MARGIN_PROB && mk != VLAC_MARGIN_LOGIT) return VLAC_ERR_INVALID_ARG;
+  if (mk != VLAC_MARGIN_PROB && mk != VLAC_MARGIN_LOGIT && mk != VLAC_MARGIN_VOCAB) return VLAC_ERR_INVALID_ARG;
   if (red == VLAC_REDUCE_DEFAULT) red = c->d.parallel ? VLAC_REDUCE_MIN : VLAC_REDUCE_MEAN;
   if (red != VLAC_REDUCE_MEAN && red != VLAC_REDUCE_MIN) return VLAC_ERR_INVALID_ARG;
   p.tau_num = tau_sim.num;
@@ -869,6 +1094,12 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   p.reduction = red;
   p.has_override = (opts && opts->gate_override) ? 1 : 0;
   p.has_forced = (opts && opts->forced_ids) ? 1 : 0;
+  p.has_active = (opts && opts->active) ? 1 : 0;
+  const int s2_k = opts ? opts->s2_top_k : 0, s2_l = opts ? opts->s2_layer : 0;
+  if (s2_k < 0 || (s2_k > 0 && (s2_l < 0 || s2_l >= c->d.n_layers))) return VLAC_ERR_INVALID_ARG;
+  p.s2_top_k = s2_k;
+  p.s2_layer = s2_k > 0 ? s2_l : 0;
+  p.has_s2_forced = (s2_k > 0 && opts->s2_forced) ? 1 : 0;
   // an error latched by an earlier step on this context is reported first
   if (*c->err_host) {
     const int e = *c->err_host;
@@ -889,11 +1120,16 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   if (d.proprio_dim) add(in, proprio, c->in_proprio, (size_t)B * d.proprio_dim * 4);
   if (p.has_override) add(in, opts->gate_override, c->in_override, (size_t)B);
   if (p.has_forced) add(in, opts->forced_ids, c->in_forced, (size_t)B * D * 4);
+  if (p.has_active) add(in, opts->active, c->in_active, (size_t)B);
+  if (p.has_s2_forced) add(in, opts->s2_forced, c->in_s2_forced, (size_t)B * c->Nv);
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_stage(p, c->prm, in, st);
   }
   c->launches += 1;
+  c->s2_on = p.s2_top_k > 0;
+  c->s2_layer = p.s2_layer;
+  c->vm_on = mk == VLAC_MARGIN_VOCAB || out->vocab_margin != nullptr;
   int rc = run_step(c, k, st);
   if (rc) return rc;
   CopyList o{};
@@ -907,6 +1143,11 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   add(o, c->o_mask, out->static_mask, (size_t)B * c->Nv);
   add(o, c->o_idx, out->idx, (size_t)B * c->S * 4);
   add(o, c->o_M, out->M, (size_t)B * d.n_layers * 4);
+  add(o, c->o_rel, out->relevance, (size_t)B * c->Nv * 4);
+  add(o, c->o_relevant, out->relevant, (size_t)B * c->Nv);
+  add(o, c->o_entropy, out->entropy, (size_t)B * D * 4);
+  if (c->vm_on) add(o, c->o_vm, out->vocab_margin, (size_t)B * D * 4);
+  add(o, c->o_delta, out->action_delta, (size_t)B * 4);
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_copies(o, st);
@@ -914,6 +1155,61 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   c->launches += 1;
   CK(cudaGetLastError());
   return VLAC_OK;
+}
+
+// ---- the one-layer workload -----------------------------------------------------
+
+namespace {
+template <typename T>
+int layer_bench_impl(vlac_ctx* c, vlac_cache* k, int seq, int layer, const int32_t* pos, int M, float* x,
+                     cudaStream_t st) {
+  const vlac_dims& d = c->d;
+  const size_t Hd = d.hidden, kv_layer = (size_t)d.n_heads * c->Tc * d.head_dim;
+  launch_layer_setup(pos, M, c->S, c->idx, c->off, c->err, st);
+  c->launches += 1;
+  CK(cudaMemcpyAsync(c->X, x, (size_t)M * Hd * sizeof(float), cudaMemcpyDeviceToDevice, st));
+  Rows rl{c->off, c->idx, c->S, c->X};
+  T* Kc = static_cast<T*>(k->K) + (size_t)seq * k->kv_seq_stride + (size_t)layer * kv_layer;
+  T* Vc = static_cast<T*>(k->V) + (size_t)seq * k->kv_seq_stride + (size_t)layer * kv_layer;
+  prefix_layer<T>(c, rl, rl.off, 1, layer, nullptr, 0, Kc, Vc, k->kv_seq_stride, st);
+  CK(cudaMemcpyAsync(x, c->X, (size_t)M * Hd * sizeof(float), cudaMemcpyDeviceToDevice, st));
+  CK(cudaGetLastError());
+  return c->fatal ? VLAC_ERR_INVALID_ARG : VLAC_OK;
+}
+}  // namespace
+
+extern "C" int vlac_layer_bench(vlac_ctx* c, vlac_cache* k, int seq, int layer, const int32_t* pos, int M, float* x,
+                                void* stream) {
+  if (!c || !k || !pos || !x || k->ctx != c || seq < 0 || seq >= k->B || layer < 0 || layer >= c->d.n_layers ||
+      M < 1 || M > c->S)
+    return VLAC_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  return c->bf16 ? layer_bench_impl<bf16>(c, k, seq, layer, pos, M, x, st)
+                 : layer_bench_impl<float>(c, k, seq, layer, pos, M, x, st);
+}
+
+namespace {
+int kv_move(const vlac_cache* k, int seq, int layer, void* K, void* V, bool to_cache, void* stream) {
+  if (!k || !K || !V || seq < 0 || seq >= k->B || layer < 0 || layer >= k->ctx->d.n_layers ||
+      (reinterpret_cast<uintptr_t>(K) | reinterpret_cast<uintptr_t>(V)) % 4)
+    return VLAC_ERR_INVALID_ARG;
+  const vlac_ctx* c = k->ctx;
+  const vlac_dims& d = c->d;
+  const size_t kv_layer = (size_t)d.n_heads * c->Tc * d.head_dim;
+  const size_t off = ((size_t)seq * k->kv_seq_stride + (size_t)layer * kv_layer) * c->esz;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  launch_kv_copy(static_cast<char*>(k->K) + off, K, d.n_heads, c->Tc, d.head_dim, (int)c->esz, to_cache, st);
+  launch_kv_copy(static_cast<char*>(k->V) + off, V, d.n_heads, c->Tc, d.head_dim, (int)c->esz, to_cache, st);
+  CK(cudaGetLastError());
+  return VLAC_OK;
+}
+}  // namespace
+
+extern "C" int vlac_cache_load(vlac_cache* k, int seq, int layer, const void* K, const void* V, void* stream) {
+  return kv_move(k, seq, layer, const_cast<void*>(K), const_cast<void*>(V), true, stream);
+}
+extern "C" int vlac_cache_store(const vlac_cache* k, int seq, int layer, void* K, void* V, void* stream) {
+  return kv_move(k, seq, layer, K, V, false, stream);
 }
 
 extern "C" int vlac_sync_error(vlac_ctx* c) {

@@ -23,7 +23,7 @@ VLAC_OK = 0
 ERRORS = {-1: "VLAC_ERR_INVALID_ARG", -2: "VLAC_ERR_CUDA", -3: "VLAC_ERR_OOM", -4: "VLAC_ERR_TIMEOUT",
           -5: "VLAC_ERR_DEVICE_CHECK", -6: "VLAC_ERR_STATE", -7: "VLAC_ERR_UNSUPPORTED"}
 F32, BF16 = 0, 1
-MARGIN_PROB, MARGIN_LOGIT = 0, 1
+MARGIN_PROB, MARGIN_LOGIT, MARGIN_VOCAB = 0, 1, 2
 REDUCE_DEFAULT, REDUCE_MEAN, REDUCE_MIN = -1, 0, 1
 
 
@@ -56,18 +56,20 @@ class Rational(C.Structure):
 
 class StepOpts(C.Structure):
     _fields_ = [("margin_kind", C.c_int32), ("reduction", C.c_int32), ("gate_override", C.c_void_p),
-                ("forced_ids", C.c_void_p)]
+                ("forced_ids", C.c_void_p), ("active", C.c_void_p), ("s2_top_k", C.c_int32), ("s2_layer", C.c_int32),
+                ("s2_forced", C.c_void_p)]
 
 
 class StepOut(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in (
         "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
-        "static_mask", "idx", "M")]
+        "static_mask", "idx", "M", "relevance", "relevant", "entropy", "vocab_margin", "action_delta")]
 
 
 EXPORTS = ["vlac_create", "vlac_destroy", "vlac_cache_bytes", "vlac_cache_init", "vlac_cache_destroy",
            "vlac_step", "vlac_reset", "vlac_sync_error", "vlac_launch_count", "vlac_selftest_wait",
-           "vlac_prof_enable", "vlac_prof_read", "vlac_select_noalloc", "vlac_strerror"]
+           "vlac_prof_enable", "vlac_prof_read", "vlac_select_noalloc", "vlac_strerror", "vlac_layer_bench",
+           "vlac_cache_load", "vlac_cache_store"]
 
 
 def lib():
@@ -96,6 +98,9 @@ def lib():
                                          C.POINTER(C.c_double)]
             L.vlac_select_noalloc.argtypes = [C.POINTER(Dims), i32, vp, vp, vp, vp, Rational, C.c_float, vp, vp,
                                               vp, vp, vp, vp, vp]
+            L.vlac_layer_bench.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp]
+            L.vlac_cache_load.argtypes = [vp, i32, i32, vp, vp, vp]
+            L.vlac_cache_store.argtypes = [vp, i32, i32, vp, vp, vp]
             L.vlac_strerror.argtypes = [i32]
             L.vlac_strerror.restype = C.c_char_p
             for name in EXPORTS:
@@ -182,7 +187,11 @@ class Context:
         }
         shapes = {"gate_auto": ((batch,), torch.uint8), "logits": ((batch, D, d.n_bins), torch.float32),
                   "static_mask": ((batch, d.n_visual), torch.uint8), "idx": ((batch, d.pass_len), torch.int32),
-                  "M": ((batch, d.n_layers), torch.int32)}
+                  "M": ((batch, d.n_layers), torch.int32),
+                  "relevance": ((batch, d.n_visual), torch.float32),
+                  "relevant": ((batch, d.n_visual), torch.uint8),
+                  "entropy": ((batch, D), torch.float32), "vocab_margin": ((batch, D), torch.float32),
+                  "action_delta": ((batch,), torch.int32)}
         for k in want:
             shp, dt = shapes[k]
             out[k] = torch.zeros(shp, dtype=dt, device=dev)
@@ -190,9 +199,13 @@ class Context:
 
     def step(self, cache: "Cache", frames, prompt, proprio=None, tau_sim=(996, 1000), tau_margin: float = 0.0,
              permille=None, margin_kind: int = MARGIN_PROB, reduction: int = REDUCE_DEFAULT, gate_override=None,
-             forced_ids=None, out: Optional[Dict] = None, want: Sequence[str] = (), stream=None) -> Dict:
+             forced_ids=None, out: Optional[Dict] = None, want: Sequence[str] = (), stream=None,
+             active=None, s2_top_k: int = 0, s2_layer: Optional[int] = None, s2_forced=None) -> Dict:
         """One step for every sequence of `cache`; inputs are CUDA tensors.
-        Returns the dict of device output tensors (allocated unless given)."""
+        Returns the dict of device output tensors (allocated unless given).
+        s2_top_k > 0 turns on Stage 2 with the relevance of layer s2_layer
+        (default: the middle layer); s2_forced (CUDA uint8 [B][Nv]) replaces
+        its removal set (lock-step replay)."""
         d = self.d
         if permille is None:
             permille = np.full(d.n_layers, 1000, dtype=np.uint16)
@@ -201,13 +214,33 @@ class Context:
             out = self.alloc_outputs(cache.batch, want)
         so = StepOut(*[_ptr(out.get(k)) for k in (
             "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
-            "static_mask", "idx", "M")])
-        opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids))
+            "static_mask", "idx", "M", "relevance", "relevant", "entropy", "vocab_margin", "action_delta")])
+        if s2_layer is None:
+            s2_layer = d.n_layers // 2
+        opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids), _ptr(active), int(s2_top_k),
+                        int(s2_layer), _ptr(s2_forced))
         rc = lib().vlac_step(self._h, cache._h, frames.data_ptr(), prompt.data_ptr(), _ptr(proprio),
                              Rational(int(tau_sim[0]), int(tau_sim[1])), float(tau_margin),
                              permille.ctypes.data, C.byref(opts), C.byref(so), _stream_ptr(stream))
         _check(rc, "vlac_step")
         return out
+
+    def layer_bench(self, cache: "Cache", seq: int, layer: int, pos, x, stream=None):
+        """One decoder layer for the rows at positions `pos` (CUDA int32 [M]);
+        x (CUDA fp32 [M][hidden]) holds their inputs and receives their outputs."""
+        assert pos.dtype.itemsize == 4 and x.is_contiguous() and x.shape[0] == pos.shape[0]
+        _check(lib().vlac_layer_bench(self._h, cache._h, seq, layer, pos.data_ptr(), int(pos.shape[0]),
+                                      x.data_ptr(), _stream_ptr(stream)), "vlac_layer_bench")
+
+    def cache_load(self, cache: "Cache", seq: int, layer: int, K, V, stream=None):
+        """K, V: CUDA [cache_len][hidden] in the model's dtype, into the cache."""
+        _check(lib().vlac_cache_load(cache._h, seq, layer, K.data_ptr(), V.data_ptr(), _stream_ptr(stream)),
+               "vlac_cache_load")
+
+    def cache_store(self, cache: "Cache", seq: int, layer: int, K, V, stream=None):
+        """K, V: CUDA [cache_len][hidden] in the model's dtype, filled from the cache."""
+        _check(lib().vlac_cache_store(cache._h, seq, layer, K.data_ptr(), V.data_ptr(), _stream_ptr(stream)),
+               "vlac_cache_store")
 
     def reset(self, cache: "Cache", seq: int = -1, stream=None):
         _check(lib().vlac_reset(cache._h, seq, _stream_ptr(stream)), "vlac_reset")

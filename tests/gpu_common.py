@@ -28,6 +28,22 @@ ID_EXEMPT_MARGIN = 1e-3
 # twice the bar.  The deep tests exempt exactly those ids, and require the
 # GPU's id to be the first maximum of the GPU's own logits.
 FLAG_TIE = 1e-4
+# Stage 2 relevance, relative to the sequence's largest relevance.  At layer
+# 0 the kernel sums fp32 probabilities of the same bf16 (or fp32) Q and K the
+# oracle sums in fp64 (REL_TOL).  At a deeper layer of a bf16 model Q and K
+# also carry the earlier layers' GEMM-input roundings (a bf16 flip moves a
+# score by up to 2^-8 of one of its terms), so the probabilities move by the
+# score error rather than by fp32 rounding: REL_TOL_DEEP, about three times
+# the largest distance measured on the small models (6.1e-4 at layer 1).
+# A removal-set difference is allowed only for patches whose oracle relevance
+# lies within twice the bar of the oracle's k-th / (k+1)-th midpoint.
+REL_TOL = {"bf16": 1e-4, "f32": 1e-5}
+REL_TOL_DEEP = {"bf16": 2e-3, "f32": 1e-5}
+# Entropy of the bin softmax: H moves by at most max_j |l_j - E_p[l]| per unit
+# of logit error, about 5 for these models' logit spread, so the bar is five
+# times the logit bar; the library's entropy must also match the entropy of
+# its own logits to fp32 rounding.
+ENTROPY_FACTOR = 5.0
 
 SMALL = {
     # bf16 path (tcgen05 GEMMs), head_dim 128, autoregressive decode
@@ -76,15 +92,27 @@ class Lockstep:
         self.gc = self.ctx.new_cache(batch)
         self.torch = torch
         self.prev_m = None
+        self.prev_rel = None
+        self.prev_ids = None
         self.log = []
         self.logit_tol = logit_tol
 
-    def step(self, frames, prompt, proprio, tau_sim, tau_m, permille, margin_kind=0, force_branch=None):
+    def step(self, frames, prompt, proprio, tau_sim, tau_m, permille, margin_kind=0, force_branch=None,
+             active=None, s2_top_k=0, s2_layer=None, s2_lockstep=True, want_vocab=False):
+        """active: uint8 [B], 0 = the sequence sits the step out (both sides).
+        s2_top_k > 0: Stage 2 on both sides; with s2_lockstep the library
+        applies the oracle's removal set (its own is still compared).
+        want_vocab: also the whole-vocabulary margin (always with margin kind 2)."""
         torch = self.torch
         d, B = self.d, self.B
+        act = None if active is None else np.ascontiguousarray(active, np.uint8)
+        vocab = want_vocab or margin_kind == 2
+        if s2_layer is None:
+            s2_layer = d.n_layers // 2
         o = self.orc.step(self.oc, frames, prompt, proprio, tau_sim=tau_sim, tau_margin=tau_m,
                           permille=permille, margin_kind=margin_kind,
-                          gate_override=None if force_branch is None else np.full(B, force_branch, np.int8))
+                          gate_override=None if force_branch is None else np.full(B, force_branch, np.int8),
+                          active=act, s2_top_k=s2_top_k, s2_layer=s2_layer, want_vocab_margin=vocab)
         # branch: free-running, except where the oracle's m_{t-1} sits in the tie zone
         ovr = np.full(B, -1, np.int8) if force_branch is None else np.full(B, force_branch, np.int8)
         if self.prev_m is not None and force_branch is None:
@@ -97,13 +125,34 @@ class Lockstep:
             tau_sim=tau_sim, tau_margin=tau_m, permille=permille, margin_kind=margin_kind,
             gate_override=torch.from_numpy(ovr).cuda(),
             forced_ids=torch.from_numpy(o["action_ids"].astype(np.int32)).cuda(),
-            want=("gate_auto", "logits", "static_mask", "idx", "M"))
+            want=("gate_auto", "logits", "static_mask", "idx", "M", "relevance", "relevant", "entropy", "action_delta")
+            + (("vocab_margin",) if vocab else ()),
+            active=None if act is None else torch.from_numpy(act).cuda(),
+            s2_top_k=s2_top_k, s2_layer=s2_layer,
+            s2_forced=(torch.from_numpy(np.ascontiguousarray(o["relevant"])).cuda()
+                       if s2_top_k > 0 and s2_lockstep else None))
         torch.cuda.synchronize()
         g = {k: v.cpu().numpy() for k, v in g.items()}
         err = self.ctx.sync_error()
         assert err == 0, f"device error {err}"
         rep = compare(d, o, g, self.prev_m, tau_m, self.logit_tol)
-        self.prev_m = o["step_margin"].copy()
+        stepped = np.ones(B, bool) if act is None else act != 0
+        rep.update(compare_stage2(d, o, g, s2_top_k, self.prev_rel, stepped, s2_layer))
+        rep.update(compare_signals(d, o, g, self.prev_ids, self.logit_tol, stepped))
+        # the ids a sequence's next action delta is measured against: a sequence
+        # that sat the step out keeps those of the last step it ran
+        po, pg = o["action_ids"].copy(), g["action_ids"].copy()
+        if act is not None and self.prev_ids is not None:
+            po[~stepped], pg[~stepped] = self.prev_ids[0][~stepped], self.prev_ids[1][~stepped]
+        self.prev_ids = (po, pg)
+        rel = o["relevance"].copy() if s2_top_k > 0 else None
+        m = o["step_margin"].copy()
+        if act is not None and self.prev_m is not None:  # a paused sequence keeps its m_{t-1}
+            m = np.where(act != 0, m, self.prev_m)
+            if rel is not None and self.prev_rel is not None:  # and its relevance
+                rel = np.where(act[:, None] != 0, rel, self.prev_rel)
+        self.prev_m = m
+        self.prev_rel = rel
         self.log.append(rep)
         return o, g, rep
 
@@ -134,3 +183,63 @@ def compare(d, o, g, prev_m, tau_m, logit_tol=None):
     np.testing.assert_allclose(g["margins"], o["margins"], atol=max(tol * 0.05, 1e-6), rtol=0.05)
     return {"max_logit_diff": float(diff.max()), "id_mismatch": int(mism.sum()),
             "id_exempt": int(exempt.sum()), "recomputed": o["recomputed"].tolist()}
+
+
+def compare_stage2(d, o, g, top_k, prev_rel, stepped=None, s2_layer=0):
+    """Stage 2: this step's relevance within REL_TOL of the oracle's (relative
+    to the sequence's largest), and the removal set the library decided from
+    its previous relevance equal to the oracle's except inside the tie band
+    around the oracle's k-th / (k+1)-th midpoint."""
+    if top_k == 0:
+        assert not g["relevance"].any() and not g["relevant"].any(), "Stage 2 off: nothing measured or removed"
+        return {"rel_diff": 0.0, "removal_diffs": 0}
+    tol = (REL_TOL if s2_layer == 0 else REL_TOL_DEEP)[d.dtype]
+    worst, diffs = 0.0, 0
+    for b in range(o["relevance"].shape[0]):
+        if stepped is not None and not stepped[b]:  # sat the step out: both sides return zeros
+            assert not g["relevance"][b].any() and not g["relevant"][b].any()
+            continue
+        scale = float(np.max(o["relevance"][b]))
+        err = float(np.max(np.abs(g["relevance"][b].astype(np.float64) - o["relevance"][b]))) / scale
+        assert err <= tol, f"relevance of sequence {b} differs by {err:.3e} (relative) > {tol}"
+        worst = max(worst, err)
+        bad = g["relevant"][b] != o["relevant"][b]
+        if bad.any():
+            assert prev_rel is not None, "a removal set without a previous relevance"
+            r = np.sort(prev_rel[b])[::-1]
+            mid = 0.5 * (r[top_k - 1] + r[top_k]) if top_k < r.size else -np.inf
+            band = 2 * tol * float(np.max(prev_rel[b]))
+            outside = bad & (np.abs(prev_rel[b] - mid) > band)
+            assert not outside.any(), f"removal set differs outside the tie band: {np.flatnonzero(outside)}"
+            diffs += int(bad.sum())
+    return {"rel_diff": worst, "removal_diffs": diffs}
+def compare_signals(d, o, g, prev_ids, logit_tol=None, stepped=None):
+    """Entropy within ENTROPY_FACTOR x the logit bar of the oracle's (and
+    within fp32 rounding of the entropy of the library's own logits); the
+    whole-vocabulary margin like the bin margin; the action delta exact for
+    every sequence whose ids agree with the oracle's on this and the
+    previous step."""
+    tol = LOGIT_TOL[d.dtype] if logit_tol is None else logit_tol
+    if stepped is not None and not stepped.all():  # sequences that sat the step out return zeros
+        assert not g["entropy"][~stepped].any() and not g["action_delta"][~stepped].any()
+        if not stepped.any():
+            return {"entropy_diff": 0.0, "delta_compared": 0}
+        o = {k: (v[stepped] if isinstance(v, np.ndarray) and v.shape[:1] == stepped.shape else v) for k, v in o.items()}
+        g = {k: (v[stepped] if isinstance(v, np.ndarray) and v.shape[:1] == stepped.shape else v) for k, v in g.items()}
+        if prev_ids is not None:
+            prev_ids = (prev_ids[0][stepped], prev_ids[1][stepped])
+    gl = g["logits"].astype(np.float64)
+    p = np.exp(gl - gl.max(-1, keepdims=True))
+    z = p.sum(-1, keepdims=True)
+    own = np.log(z[..., 0]) - (p * (gl - gl.max(-1, keepdims=True))).sum(-1) / z[..., 0]
+    np.testing.assert_allclose(g["entropy"], own, atol=1e-4, rtol=1e-5, err_msg="entropy vs own logits")
+    ediff = float(np.max(np.abs(g["entropy"] - o["entropy"])))
+    assert ediff <= ENTROPY_FACTOR * tol, f"entropy differs by {ediff:.3e}"
+    if "vocab_margin" in g and "vocab_margin" in o:
+        np.testing.assert_allclose(g["vocab_margin"], o["vocab_margin"], atol=max(tol * 0.05, 1e-6), rtol=0.05,
+                                   err_msg="vocabulary margin")
+    same = (g["action_ids"] == o["action_ids"]).all(-1)
+    if prev_ids is not None:
+        same &= (prev_ids[0] == prev_ids[1]).all(-1)
+    np.testing.assert_array_equal(g["action_delta"][same], o["action_delta"][same], err_msg="action delta")
+    return {"entropy_diff": ediff, "delta_compared": int(same.sum())}

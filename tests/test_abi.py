@@ -72,3 +72,7 @@ def test_null_handles_are_invalid_arguments(lib):
     n = C.c_size_t()
     assert lib.vlac_cache_bytes(None, 1, C.byref(n)) == -1
     assert lib.vlac_launch_count(None) == 0
+    # the one-layer entry and the cache K/V copies refuse NULL handles before any device call
+    assert lib.vlac_layer_bench(None, None, 0, 0, None, 1, None, None) == -1
+    assert lib.vlac_cache_load(None, 0, 0, None, None, None) == -1
+    assert lib.vlac_cache_store(None, 0, 0, None, None, None) == -1

@@ -9,7 +9,9 @@ the logits within LOGIT_TOL_DEEP, twice the spread measured between two runs
 of the GPU path that differ only in the fp32 summation order of their GEMM
 partial sums (test_summation_order_floor).  The oracle
 takes several seconds per 7B step, so each episode is short and covers both
-branches: a full pass (empty cache) and a cached step (theta_m = 0).  For the
+branches: a full pass (empty cache) and a cached step (theta_m = 0); the
+OpenVLA-7B episode then lets the gate fire (theta_m = +inf) and runs one more
+cached step.  Every step prints its largest logit difference.  For the
 batch, the oracle runs two of the eight sequences (the sequences of a batch
 are independent), and their outputs are compared with those rows of the batch.
 """
@@ -29,8 +31,11 @@ def _weights(d, seed):
     return synth.weights_to(w_gpu, "cpu"), w_gpu
 
 
-def _run_lockstep(name, n_frames, seed):
+def _run_lockstep(name, taus, seed):
+    """One lock-step episode, theta_m per frame from `taus`; returns the
+    branch each step ran."""
     d = synth.dims_for(name)
+    n_frames = len(taus)
     w_cpu, w_gpu = _weights(d, seed)
     ls = Lockstep(d, w_cpu, w_gpu, logit_tol=LOGIT_TOL_DEEP)
     del w_gpu
@@ -40,23 +45,27 @@ def _run_lockstep(name, n_frames, seed):
     pm = synth.linear_schedule(d.n_layers)
     branches = []
     for t in range(n_frames):
-        # the first step runs the full pass (empty cache), the later ones the
-        # cached branch (theta_m = 0 never fires)
-        o, g, rep = ls.step(frames[t], prompt, None if prop is None else prop[t], (996, 1000), 0.0, pm)
+        o, g, rep = ls.step(frames[t], prompt, None if prop is None else prop[t], (996, 1000), taus[t], pm)
         branches.append(int(o["recomputed"][0]))
-    assert branches[0] == 1 and all(b == 0 for b in branches[1:])
-    # the cached steps reused static patches at every layer
-    assert g["M"][0].max() < d.pass_len
+        print(f"{name} frame {t}: recomputed {branches[-1]}, max logit diff {rep['max_logit_diff']:.4e}, "
+              f"id mismatches {rep['id_mismatch']}")
+        if not branches[-1]:  # a cached step reused static patches at every layer
+            assert g["M"][0].max() < d.pass_len
     del ls
     gc.collect()
+    return branches
 
 
 def test_openvla7b_parity(cuda_device):
-    _run_lockstep("openvla7b", 3, seed=11)
+    """Full pass (empty cache), cached step (theta_m = 0 never fires), the
+    gate firing after a cached step (theta_m = +inf, Algorithm 1), and a
+    cached step after the gated one."""
+    inf = float("inf")
+    assert _run_lockstep("openvla7b", [0.0, 0.0, inf, 0.0], seed=11) == [1, 0, 1, 0]
 
 
 def test_oft7b_parity(cuda_device):
-    _run_lockstep("oft7b", 2, seed=12)
+    assert _run_lockstep("oft7b", [0.0, 0.0], seed=12) == [1, 0]
 
 
 def test_batch7b_sampled_parity(cuda_device):
@@ -94,7 +103,8 @@ def test_batch7b_sampled_parity(cuda_device):
         torch.cuda.synchronize()
         assert ctx.sync_error() == 0
         g = {k: v.cpu().numpy()[pick] for k, v in g.items()}
-        compare(d, o, g, prev_m, 0.0, LOGIT_TOL_DEEP)
+        rep = compare(d, o, g, prev_m, 0.0, LOGIT_TOL_DEEP)
+        print(f"batch7b frame {t}: max logit diff {rep['max_logit_diff']:.4e}, id mismatches {rep['id_mismatch']}")
         prev_m = o["step_margin"].copy()
     assert g["recomputed"].tolist() == [0, 0]
     del ctx, cache, probe, orc

@@ -78,3 +78,18 @@ def test_logit_gap_gate_signal(cuda_device):
     pm = synth.full_schedule(d.n_layers)
     for t in range(4):
         ls.step(frames[t], prompt, None, (95, 100), 0.3, pm, margin_kind=1)
+
+
+@pytest.mark.parametrize("name,batch", [("small", 1), ("small_oft", 1), ("small_batch", 3)])
+def test_gemm_tail_split_parity(cuda_device, monkeypatch, name, batch):
+    """Prefix GEMMs planned for 5 SMs: q/k/v (6 weight tiles) runs 5 whole
+    tiles and cuts the sixth into 4 K ranges; gate/up (12 tiles) 10 whole and
+    2 cut in two; their later partials go to the compact tail slots."""
+    monkeypatch.setenv("VLAC_PLAN_SMS", "5")
+    d = SMALL[name]
+    ls = Lockstep(d, synth.make_weights(d, seed=61), batch=batch)
+    frames, prompt, prop = episode(d, 3, seed=61, batch=batch)
+    pm = synth.linear_schedule(d.n_layers)
+    tau = (996, 1000) if d.img_h >= 224 else (95, 100)
+    for t in range(3):
+        ls.step(frames[t], prompt, None if prop is None else prop[t], tau, 0.0, pm)
