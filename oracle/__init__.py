@@ -54,7 +54,9 @@ class _Weights(C.Structure):
 class _Opts(C.Structure):
     _fields_ = [("margin_kind", C.c_int32), ("reduction", C.c_int32),
                 ("gate_override", C.c_void_p), ("forced_ids", C.c_void_p),
-                ("s2_top_k", C.c_int32), ("s2_layer", C.c_int32), ("active", C.c_void_p)]
+                ("s2_top_k", C.c_int32), ("s2_layer", C.c_int32), ("active", C.c_void_p),
+                ("s3_adaptive", C.c_int32), ("s3_lo", C.c_int32), ("s3_hi", C.c_int32), ("s3_weight", C.c_int32),
+                ("s3_forced", C.c_void_p)]
 
 
 class _Out(C.Structure):
@@ -62,7 +64,8 @@ class _Out(C.Structure):
                 ("logits", C.c_void_p), ("recomputed", C.c_void_p), ("gate_auto", C.c_void_p),
                 ("step_margin", C.c_void_p), ("static_mask", C.c_void_p), ("idx", C.c_void_p),
                 ("M", C.c_void_p), ("relevance", C.c_void_p), ("relevant", C.c_void_p),
-                ("entropy", C.c_void_p), ("vocab_margin", C.c_void_p), ("action_delta", C.c_void_p)]
+                ("entropy", C.c_void_p), ("vocab_margin", C.c_void_p), ("action_delta", C.c_void_p),
+                ("layer_entropy", C.c_void_p), ("schedule", C.c_void_p)]
 
 
 def lib():
@@ -77,6 +80,7 @@ def lib():
             L.orc_cache_new.argtypes = [vp, C.c_int, C.POINTER(vp)]
             L.orc_cache_free.argtypes = [vp]
             L.orc_reset.argtypes = [vp, C.c_int]
+            L.orc_entropy_schedule.argtypes = [vp, C.c_int, C.c_int, C.c_int, C.c_int, vp]
             L.orc_step.argtypes = [vp, vp, vp, vp, vp, u32, u32, C.c_double, vp,
                                    C.POINTER(_Opts), C.POINTER(_Out)]
             L.orc_cache_read.argtypes = [vp, C.c_int, C.c_int, C.c_int, vp]
@@ -169,6 +173,14 @@ def top_k(rel: np.ndarray, k: int) -> np.ndarray:
     return out
 
 
+def entropy_schedule(ent, lo: int, hi: int, weight: int) -> np.ndarray:
+    """Stage 3's per-mille schedule from per-layer normalized entropies."""
+    e = np.ascontiguousarray(ent, dtype=np.float64)
+    out = np.zeros(e.size, dtype=np.uint16)
+    lib().orc_entropy_schedule(_ptr(e), e.size, int(lo), int(hi), int(weight), _ptr(out))
+    return out
+
+
 def margin(logits: np.ndarray):
     lg = np.ascontiguousarray(logits, dtype=np.float64)
     a, pm, gap = C.c_int32(), C.c_double(), C.c_double()
@@ -253,7 +265,10 @@ class Oracle:
     def step(self, cache: "OracleCache", frames, prompt, proprio=None, tau_sim=(996, 1000),
              tau_margin: float = 0.0, permille=None, margin_kind: int = 0, reduction: Optional[int] = None,
              gate_override=None, forced_ids=None, want_logits: bool = True, s2_top_k: int = 0,
-             s2_layer: Optional[int] = None, want_vocab_margin: bool = False, active=None):
+             s2_layer: Optional[int] = None, want_vocab_margin: bool = False, active=None,
+             s3_adaptive=None, s3_forced=None):
+        """s3_adaptive: None (the caller's schedule) or (lo, hi, weight) per mille
+        for the entropy-adaptive Stage 3; s3_forced [B][L] replays a schedule."""
         d, B = self.d, cache.batch
         D, S, L = d.n_action, d.pass_len, d.n_layers
         frames = np.ascontiguousarray(frames, dtype=np.uint8).reshape(B, d.n_views, d.img_h, d.img_w, 3)
@@ -278,14 +293,19 @@ class Oracle:
             "entropy": np.zeros((B, D), np.float64),
             "vocab_margin": np.zeros((B, D), np.float64) if want_vocab_margin else None,
             "action_delta": np.zeros(B, np.int32),
+            "layer_entropy": np.zeros((B, L), np.float64), "schedule": np.zeros((B, L), np.uint16),
         }
         co = _Out(*[_ptr(out[k]) for k in ("action_ids", "margins", "logit_gap", "logits", "recomputed",
                                            "gate_auto", "step_margin", "static_mask", "idx", "M",
-                                           "relevance", "relevant", "entropy", "vocab_margin", "action_delta")])
+                                           "relevance", "relevant", "entropy", "vocab_margin", "action_delta",
+                                           "layer_entropy", "schedule")])
         if s2_layer is None:
             s2_layer = L // 2
         act = None if active is None else np.ascontiguousarray(active, dtype=np.uint8).reshape(B)
-        opts = _Opts(margin_kind, reduction, _ptr(go), _ptr(fi), int(s2_top_k), int(s2_layer), _ptr(act))
+        s3 = (0, 0, 0) if s3_adaptive is None else tuple(int(v) for v in s3_adaptive)
+        sf = None if s3_forced is None else np.ascontiguousarray(s3_forced, dtype=np.uint16).reshape(B, L)
+        opts = _Opts(margin_kind, reduction, _ptr(go), _ptr(fi), int(s2_top_k), int(s2_layer), _ptr(act),
+                     int(s3_adaptive is not None), s3[0], s3[1], s3[2], _ptr(sf))
         r = lib().orc_step(self._h, cache._h, _ptr(frames), _ptr(prompt), _ptr(proprio), tau_sim[0],
                            tau_sim[1], float(tau_margin), _ptr(permille), C.byref(opts), C.byref(co))
         if r != 0:

@@ -37,6 +37,8 @@ struct orc_cache {
   uint8_t* rel_valid; /* [B]: rel holds the previous step's relevance */
   int32_t* prev_ids;  /* [B][n_action]: the previous step's action bins */
   uint8_t* ids_valid; /* [B]: prev_ids holds them */
+  double* ent;        /* [B][L]: per-layer normalized attention entropy from the previous step */
+  uint8_t* ent_valid; /* [B]: ent holds it */
 };
 
 /* ------------------------------------------------------------------------ */
@@ -208,6 +210,23 @@ static int pos_is_text(const orc_ctx* c, int pos) {
 
 /* Stage 2's removal set: the top_k entries of rel, ranked by value (higher
  * first), equal values by index (lower first). */
+/* Stage 3 from the layers' normalized attention entropy (a reading: the paper
+ * names the idea, not the formula).  Low entropy, more reuse: the target of
+ * layer l is hi - (hi - lo) * ent[l] per mille; the targets are smoothed over
+ * depth, each layer moving `weight` per mille of the way from the previous
+ * layer's value to its own target; the result is floored and clamped. */
+void orc_entropy_schedule(const double* ent, int n_layers, int lo, int hi, int weight, uint16_t* permille) {
+  double r = 0.0;
+  for (int l = 0; l < n_layers; ++l) {
+    const double t = (double)hi - (double)(hi - lo) * ent[l];
+    r = l == 0 ? t : r + ((double)weight / 1000.0) * (t - r);
+    double f = floor(r);
+    if (f < 0.0) f = 0.0;
+    if (f > 1000.0) f = 1000.0;
+    permille[l] = (uint16_t)f;
+  }
+}
+
 void orc_top_k(const double* rel, int n, int top_k, uint8_t* out) {
   for (int v = 0; v < n; ++v) {
     int before = 0;
@@ -394,8 +413,10 @@ int orc_cache_new(const orc_ctx* c, int batch, orc_cache** out) {
   k->rel_valid = (uint8_t*)calloc((size_t)batch, 1);
   k->prev_ids = (int32_t*)calloc((size_t)batch * c->d.n_action, sizeof(int32_t));
   k->ids_valid = (uint8_t*)calloc((size_t)batch, 1);
+  k->ent = (double*)calloc((size_t)batch * L, sizeof(double));
+  k->ent_valid = (uint8_t*)calloc((size_t)batch, 1);
   if (!k->K || !k->V || !k->H || !k->prev || !k->m_prev || !k->valid || !k->rel || !k->rel_valid || !k->prev_ids ||
-      !k->ids_valid) {
+      !k->ids_valid || !k->ent || !k->ent_valid) {
     orc_cache_free(k);
     return ORC_ERR_OOM;
   }
@@ -415,6 +436,8 @@ void orc_cache_free(orc_cache* k) {
   free(k->rel_valid);
   free(k->prev_ids);
   free(k->ids_valid);
+  free(k->ent);
+  free(k->ent_valid);
   free(k);
 }
 
@@ -422,7 +445,7 @@ void orc_cache_free(orc_cache* k) {
 int orc_reset(orc_cache* k, int seq) {
   if (!k || seq < -1 || seq >= k->B) return ORC_ERR_ARG;
   for (int b = 0; b < k->B; ++b)
-    if (seq == -1 || seq == b) k->valid[b] = k->rel_valid[b] = k->ids_valid[b] = 0;
+    if (seq == -1 || seq == b) k->valid[b] = k->rel_valid[b] = k->ids_valid[b] = k->ent_valid[b] = 0;
   return ORC_OK;
 }
 
@@ -473,9 +496,13 @@ static int key_limit(const orc_ctx* c, int pos) {
  * row attends, and attention reads the cache (reused + fresh entries).
  * rel (Stage 2, NULL = not wanted) receives, per visual patch v, the softmax
  * probability of key 1 + v summed over the text rows among the n (in row
- * order) and, within a row, over the heads in order. */
+ * order) and, within a row, over the heads in order.
+ * ent (Stage 3 adaptive, NULL = not wanted) receives the layer's normalized
+ * attention entropy: over the text rows among the n that attend to two or
+ * more keys, and every head, the mean of H / ln(keys), H = -sum_j p_j ln p_j
+ * of the row's causal softmax (rows in order, heads in order within a row). */
 static void layer_rows(const orc_ctx* c, orc_cache* k, int b, int l, int n, const int32_t* pos, float* x,
-                       double* rel) {
+                       double* rel, double* ent) {
   const int Hd = c->d.hidden, nh = c->d.n_heads, hd = c->d.head_dim, F = c->d.ffn;
   const size_t T = c->T, L = c->d.n_layers;
   float* Kl = k->K + (((size_t)b * L + l) * T) * Hd;
@@ -509,6 +536,8 @@ static void layer_rows(const orc_ctx* c, orc_cache* k, int b, int l, int n, cons
   const int Nv = c->Nv;
   /* per (row, head): probability of each visual key (text rows only) */
   double* pv = rel ? (double*)calloc((size_t)n * nh * (Nv > 0 ? Nv : 1), sizeof(double)) : NULL;
+  /* per (row, head): normalized entropy, or -1 where the row does not count */
+  double* hv = ent ? (double*)malloc(sizeof(double) * (size_t)n * nh) : NULL;
 #pragma omp parallel for schedule(dynamic)
   for (int ih = 0; ih < n * nh; ++ih) {
     const int i = ih / nh, hh = ih % nh;
@@ -522,11 +551,15 @@ static void layer_rows(const orc_ctx* c, orc_cache* k, int b, int l, int n, cons
       sc[j] = dot(qi, kd, hd) * scale;
       if (sc[j] > mx) mx = sc[j];
     }
-    double z = 0.0;
+    double z = 0.0, zu = 0.0;
     for (int j = 0; j < nk; ++j) {
-      sc[j] = exp(sc[j] - mx);
+      const double u = sc[j] - mx;
+      sc[j] = exp(u);
       z += sc[j];
+      zu += sc[j] * u;
     }
+    /* H = -sum p ln p with p = e^u / z: ln z - sum e^u u / z */
+    if (hv) hv[ih] = (pos_is_text(c, pos[i]) && nk >= 2) ? (log(z) - zu / z) / log((double)nk) : -1.0;
     if (pv && pos_is_text(c, pos[i]))
       for (int j = 1; j < nk && j <= Nv; ++j) pv[((size_t)i * nh + hh) * Nv + (j - 1)] = sc[j] / z;
     for (int e = 0; e < hd; ++e) {
@@ -535,6 +568,17 @@ static void layer_rows(const orc_ctx* c, orc_cache* k, int b, int l, int n, cons
       att[(size_t)i * Hd + (size_t)hh * hd + e] = store_act(c, o / z);
     }
     free(sc);
+  }
+  if (hv) {
+    double sum = 0.0;
+    int cnt = 0;
+    for (int q = 0; q < n * nh; ++q)
+      if (hv[q] >= 0.0) {
+        sum += hv[q];
+        ++cnt;
+      }
+    *ent = cnt ? sum / cnt : 0.0;
+    free(hv);
   }
   if (pv) {
     for (int v = 0; v < Nv; ++v) rel[v] = 0.0;
@@ -569,7 +613,7 @@ int orc_layer(orc_ctx* c, orc_cache* k, int seq, int layer, int n, const int32_t
     for (int j = 0; j < i; ++j)
       if (pos[j] == pos[i]) return ORC_ERR_ARG;
   }
-  layer_rows(c, k, seq, layer, n, pos, x, NULL);
+  layer_rows(c, k, seq, layer, n, pos, x, NULL, NULL);
   return ORC_OK;
 }
 
@@ -667,8 +711,19 @@ static int step_seq(orc_ctx* c, orc_cache* k, int b, const uint8_t* frame, const
   /* Stage 2 uses the relevance the previous step measured */
   const int s2 = o && o->s2_top_k > 0;
   const double* rel_prev = (s2 && k->rel_valid[b]) ? k->rel + (size_t)b * c->Nv : NULL;
-  int nS = orc_select2(&c->d, frame, prev, k->valid[b], num, den, permille, full, rel_prev, s2 ? o->s2_top_k : 0,
+  /* Stage 3: the caller's schedule, or the one the previous step's layer
+   * entropies give (a lock-step replay may impose the other side's) */
+  const int s3 = o && o->s3_adaptive;
+  uint16_t* sched = (uint16_t*)malloc(sizeof(uint16_t) * L);
+  if (s3 && k->ent_valid[b])
+    orc_entropy_schedule(k->ent + (size_t)b * L, L, o->s3_lo, o->s3_hi, o->s3_weight, sched);
+  else
+    memcpy(sched, permille, sizeof(uint16_t) * L);
+  if (out->schedule) memcpy(out->schedule + (size_t)b * L, sched, sizeof(uint16_t) * L);
+  const uint16_t* use = (s3 && o->s3_forced) ? o->s3_forced + (size_t)b * L : sched;
+  int nS = orc_select2(&c->d, frame, prev, k->valid[b], num, den, use, full, rel_prev, s2 ? o->s2_top_k : 0,
                        mask, relevant, idx, M);
+  free(sched);
   if (nS < 0) { free(idx); free(M); free(mask); free(relevant); return ORC_ERR_ARG; }
   if (out->static_mask) memcpy(out->static_mask + (size_t)b * c->Nv, mask, (size_t)c->Nv);
   if (out->relevant) memcpy(out->relevant + (size_t)b * c->Nv, relevant, (size_t)c->Nv);
@@ -681,6 +736,7 @@ static int step_seq(orc_ctx* c, orc_cache* k, int b, const uint8_t* frame, const
   for (int i = 0; i < M[0]; ++i) embed_row(c, idx[i], frame, prompt, proprio, x + (size_t)i * Hd);
   float* Hb = k->H + (size_t)b * L * S * Hd;
   double* rel_now = s2 ? (double*)calloc((size_t)(c->Nv > 0 ? c->Nv : 1), sizeof(double)) : NULL;
+  double* ent_now = s3 ? (double*)calloc((size_t)L, sizeof(double)) : NULL;
   for (int l = 0; l < L; ++l) {
     if (l > 0) {
       /* rows computed at layer l-1 record their layer-l input; rows that join
@@ -690,8 +746,15 @@ static int step_seq(orc_ctx* c, orc_cache* k, int b, const uint8_t* frame, const
       for (int i = M[l - 1]; i < M[l]; ++i)
         memcpy(x + (size_t)i * Hd, Hb + ((size_t)l * S + idx[i]) * Hd, sizeof(float) * Hd);
     }
-    layer_rows(c, k, b, l, M[l], idx, x, (s2 && l == o->s2_layer) ? rel_now : NULL);
+    layer_rows(c, k, b, l, M[l], idx, x, (s2 && l == o->s2_layer) ? rel_now : NULL, s3 ? ent_now + l : NULL);
   }
+  /* every text row is recomputed at every layer, so the layer entropies are
+   * complete too; the next step's Stage 3 reads them */
+  if (out->layer_entropy)
+    for (int l = 0; l < L; ++l) out->layer_entropy[(size_t)b * L + l] = s3 ? ent_now[l] : 0.0;
+  if (s3) memcpy(k->ent + (size_t)b * L, ent_now, sizeof(double) * L);
+  k->ent_valid[b] = (uint8_t)s3;
+  free(ent_now);
   /* every text row is recomputed at every layer, so this step's relevance is
    * complete; it is what the next step's Stage 2 reads */
   if (out->relevance)
@@ -727,7 +790,7 @@ static int step_seq(orc_ctx* c, orc_cache* k, int b, const uint8_t* frame, const
       int32_t p = c->P + a - 1;
       xdec = (float*)malloc(sizeof(float) * Hd);
       for (int e = 0; e < Hd; ++e) xdec[e] = (float)wget(c, c->w.tok_emb, (size_t)tok * Hd + e);
-      for (int l = 0; l < L; ++l) layer_rows(c, k, b, l, 1, &p, xdec, NULL);
+      for (int l = 0; l < L; ++l) layer_rows(c, k, b, l, 1, &p, xdec, NULL, NULL);
       xr = xdec;
     }
     double pm, gap, ent, vm = 0.0;
@@ -770,6 +833,13 @@ int orc_step(orc_ctx* c, orc_cache* k, const uint8_t* frames, const int32_t* pro
   if (opts && (opts->margin_kind < 0 || opts->margin_kind > 2)) return ORC_ERR_ARG;
   if (opts && (opts->s2_top_k < 0 || (opts->s2_top_k > 0 && (opts->s2_layer < 0 || opts->s2_layer >= c->d.n_layers))))
     return ORC_ERR_ARG;
+  if (opts && opts->s3_adaptive &&
+      (opts->s3_lo < 0 || opts->s3_lo > opts->s3_hi || opts->s3_hi > 1000 || opts->s3_weight < 0 ||
+       opts->s3_weight > 1000))
+    return ORC_ERR_ARG;
+  if (opts && opts->s3_forced)
+    for (int q = 0; q < k->B * c->d.n_layers; ++q)
+      if (opts->s3_forced[q] > 1000) return ORC_ERR_ARG;
   const size_t fb = frame_bytes(&c->d);
   for (int b = 0; b < k->B; ++b) {
     if (opts && opts->active && !opts->active[b]) {
@@ -790,6 +860,8 @@ int orc_step(orc_ctx* c, orc_cache* k, const uint8_t* frames, const int32_t* pro
       if (out->entropy) memset(out->entropy + b * D, 0, sizeof(double) * D);
       if (out->vocab_margin) memset(out->vocab_margin + b * D, 0, sizeof(double) * D);
       if (out->action_delta) out->action_delta[b] = 0;
+      if (out->layer_entropy) memset(out->layer_entropy + b * L, 0, sizeof(double) * L);
+      if (out->schedule) memset(out->schedule + b * L, 0, sizeof(uint16_t) * L);
       continue;
     }
     int r = step_seq(c, k, b, frames + (size_t)b * fb, prompt_ids + (size_t)b * c->d.n_text,

@@ -18,7 +18,11 @@
  *     layer of the previous step; the top_k patches by relevance are
  *     removed.
  *   - Sec. III-B Stage 3: a per-layer proportion of the static patches is
- *     reused (here a caller-given per-mille schedule).
+ *     reused: a caller-given per-mille schedule, or (optional) one derived
+ *     from each layer's normalized attention entropy measured in the
+ *     previous step -- lower entropy, more reuse -- smoothed over depth.
+ *     The paper names the idea but gives no formula: the mapping and the
+ *     smoothing are this library's reading (parity unpinned).
  *   - Sec. IV-A Eq. (1): mean top-1/top-2 probability margin over the D
  *     action tokens, with the softmax over the action bins or (margin kind
  *     2) over the whole vocabulary.
@@ -84,6 +88,11 @@ typedef struct orc_opts {
   int32_t s2_layer;             /* Stage 2: the layer whose attention gives the relevance */
   const uint8_t* active;        /* [B]: 0 = this sequence sits the step out (its cache and state
                                    stay as they are, its outputs are zero); NULL = all step */
+  int32_t s3_adaptive;          /* Stage 3 from attention entropy: 0 = the caller's schedule */
+  int32_t s3_lo, s3_hi;         /* per-mille reuse of a layer of normalized entropy 1 / 0 */
+  int32_t s3_weight;            /* per-mille weight of a layer's own target in the smoothing over depth */
+  const uint16_t* s3_forced;    /* [B][n_layers]: lock-step replay, applied instead of the schedule this
+                                   step derives (its own is still reported); NULL = none */
 } orc_opts;
 
 typedef struct orc_out {
@@ -102,6 +111,10 @@ typedef struct orc_out {
   double* entropy;      /* [B][n_action] entropy (nats) of the bin softmax or NULL */
   double* vocab_margin; /* [B][n_action] p1 - p2 of the softmax over the whole vocabulary or NULL */
   int32_t* action_delta; /* [B] sum over d of |a_t^d - a_{t-1}^d| in bins (0 without a previous step) or NULL */
+  double* layer_entropy; /* [B][n_layers] normalized attention entropy of the text rows measured this
+                            step (0 with Stage 3 adaptive off) or NULL */
+  uint16_t* schedule;    /* [B][n_layers] the per-mille reuse schedule Stage 3 derived for this step
+                            (the caller's when adaptive is off or nothing was measured) or NULL */
 } orc_out;
 
 typedef struct orc_ctx orc_ctx;
@@ -153,6 +166,11 @@ void orc_top_k(const double* rel, int n, int top_k, uint8_t* out);
 void orc_margin(const double* logits, int n, int32_t* argmax, double* pmargin, double* lgap);
 /* -sum_j p_j ln p_j of the softmax of logits[0..n), in nats. */
 double orc_entropy(const double* logits, int n);
+/* Entropy-adaptive Stage 3 (this library's reading): layer l's target
+ * t_l = hi - (hi - lo) * ent[l] (per mille; ent in [0, 1]), smoothed over
+ * depth r_0 = t_0, r_l = r_{l-1} + (weight / 1000) * (t_l - r_{l-1}), and
+ * permille[l] = floor(r_l) clamped to [0, 1000]. */
+void orc_entropy_schedule(const double* ent, int n_layers, int lo, int hi, int weight, uint16_t* permille);
 double orc_round_bf16(double v);
 void orc_rope_table(const orc_dims* d, int n_pos, float* cos_t, float* sin_t);
 

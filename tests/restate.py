@@ -79,6 +79,7 @@ class Restated:
         self.prev = None
         self.m_prev = 0.0
         self.valid = False
+        self.ent_sum = None  # per layer: [sum of normalized entropies, count] while a prefix pass runs
 
     # -- storage roundings --------------------------------------------------
     def act_r(self, x):
@@ -167,13 +168,20 @@ class Restated:
         self.V[l, pos] = self.act_r(v)
         hd, nh = d.head_dim, d.n_heads
         out = np.zeros_like(q)
+        hp = 1 if d.proprio_dim else 0
         for i, p in enumerate(pos):
             nk = self.key_limit(int(p))
+            text = int(p) == 0 or self.Nv + hp < int(p) < self.P
             for hh in range(nh):
                 sl = slice(hh * hd, (hh + 1) * hd)
                 sc = self.K[l, :nk, sl] @ q[i, sl] / np.sqrt(hd)
                 e = np.exp(sc - sc.max())
-                out[i, sl] = (e / e.sum()) @ self.V[l, :nk, sl]
+                prob = e / e.sum()
+                out[i, sl] = prob @ self.V[l, :nk, sl]
+                if self.ent_sum is not None and text and nk >= 2:
+                    nz = prob[prob > 0]
+                    self.ent_sum[l][0] += float(-(nz * np.log(nz)).sum() / np.log(nk))
+                    self.ent_sum[l][1] += 1
         x = self.f32(x + self.act_r(out) @ W["wo"].T)
         h2 = self.rmsnorm(x, W["ffn_norm"])
         g = h2 @ W["w_gate"].T
@@ -219,6 +227,7 @@ class Restated:
             idx = [p for p in range(S) if p not in stat_pos] + [1 + v for v in reversed(order)]
             M = [S - (int(permille[l]) * len(stat)) // 1000 for l in range(L)]
         x = np.stack([self.embed(idx[i], frame, prompt, proprio) for i in range(M[0])])
+        self.ent_sum = [[0.0, 0] for _ in range(L)]
         for l in range(L):
             if l > 0:
                 for i in range(M[l - 1]):
@@ -228,6 +237,8 @@ class Restated:
                 else:
                     x = x[:M[l]]
             x = self.layer(l, x, idx[:M[l]])
+        layer_entropy = np.array([e / n if n else 0.0 for e, n in self.ent_sum])
+        self.ent_sum = None
         ids, margins, gaps, logits = [], [], [], []
         for a in range(D):
             if d.parallel:
@@ -251,7 +262,8 @@ class Restated:
         self.m_prev, self.valid, self.prev = m_t, True, frame.copy()
         return dict(action_ids=np.array(ids), margins=np.array(margins), logit_gap=np.array(gaps),
                     logits=np.stack(logits), recomputed=int(full), gate_auto=int(gate),
-                    step_margin=m_t, static_mask=mask, idx=np.array(idx), M=np.array(M))
+                    step_margin=m_t, static_mask=mask, idx=np.array(idx), M=np.array(M),
+                    layer_entropy=layer_entropy)
 
 
 def _bf16_fast(x: np.ndarray) -> np.ndarray:
