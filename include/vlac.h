@@ -116,6 +116,21 @@ typedef struct vlac_step_opts {
   const uint8_t* s2_forced;    /* device [B][Nv]: the Stage-2 removal set to apply instead of the
                                   library's own (lock-step replay; `relevant` still reports the
                                   library's own set); NULL = the library's own */
+  int32_t s3_adaptive;         /* Stage 3 (Sec. III-B, entropy-adaptive layer-wise reuse): 0 = the
+                                  caller's reuse_permille (default); 1 = per sequence, the schedule
+                                  the previous step's layer entropies give (the caller's on a
+                                  sequence's first step and after a reset).  The paper names the
+                                  idea, not a formula; this library's reading: layer l's normalized
+                                  attention entropy e_l (the mean over the text rows that see two or
+                                  more keys, and the heads, of H / ln(keys)) sets the target
+                                  t_l = s3_hi - (s3_hi - s3_lo) * e_l per mille, smoothed over depth
+                                  (r_0 = t_0, r_l = r_{l-1} + s3_weight / 1000 * (t_l - r_{l-1}))
+                                  and floored */
+  int32_t s3_lo, s3_hi;        /* 0 <= s3_lo <= s3_hi <= 1000 */
+  int32_t s3_weight;           /* 0 .. 1000 */
+  const uint16_t* s3_forced;   /* device [B][L]: the schedule to apply instead of the derived one
+                                  (lock-step replay; `schedule` still reports the derived one);
+                                  NULL = the derived one */
 } vlac_step_opts;
 
 /* Device output buffers of one step (B = the cache's batch, D = n_action,
@@ -138,6 +153,9 @@ typedef struct vlac_step_out {
                            for it (or for VLAC_MARGIN_VOCAB) reads every LM-head row per token */
   int32_t* action_delta; /* optional [B] sum over d of |a_t^d - a_{t-1}^d| in bins, 0 on a sequence's
                             first step and after a reset (Sec. VI) */
+  float* layer_entropy;  /* optional [B][L] normalized attention entropy of each layer measured this
+                            step (0 when Stage 3 adaptive is off) */
+  uint16_t* schedule;    /* optional [B][L] the per-mille reuse schedule Stage 3 derived for this step */
 } vlac_step_out;
 
 typedef struct vlac_ctx vlac_ctx;
@@ -226,6 +244,17 @@ uint64_t vlac_launch_count(const vlac_ctx* ctx);
  * VLAC_ERR_TIMEOUT in the error word and returns.  Synchronous; returns the
  * recorded status (VLAC_ERR_TIMEOUT when the wait gave up). */
 int vlac_selftest_wait(vlac_ctx* ctx, uint32_t spin_limit);
+
+/* Test hook: the number of polls after which the bounded waits of the step's
+ * kernels give up (the prefix GEMM's pipeline waits, the decode GEMV's ring
+ * waits, the prefix attention's tile waits); 0 makes every such wait give up
+ * at once.  A block that gave up latches VLAC_ERR_TIMEOUT, stops, and still
+ * lets the copies it issued land (those waits keep their own limit) before it
+ * exits, so the context stays usable.  Takes effect for launches made after
+ * the call: eager steps and step graphs captured later; a cache's existing
+ * step graph keeps the limit it was captured with.  Default 2^24.
+ * VLAC_ERR_INVALID_ARG for a NULL context. */
+int vlac_set_wait_limit(vlac_ctx* ctx, uint32_t polls);
 
 /* Per-launch timing, for roofline reports and time breakdowns.  While
  * enabled (steps then run without graph replay), each kernel launch of the

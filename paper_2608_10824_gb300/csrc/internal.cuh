@@ -26,6 +26,9 @@ struct StepParams {
   int32_t s2_top_k;  // Stage 2: 0 = off
   int32_t s2_layer;
   int32_t has_s2_forced;
+  int32_t s3_adaptive;  // Stage 3 from the previous step's layer entropies: 0 = the permille below
+  int32_t s3_lo, s3_hi, s3_weight;
+  int32_t has_s3_forced;
   uint16_t permille[kMaxLayers];
 };
 
@@ -83,6 +86,7 @@ struct DGemv {
   int n_ssq;
   float* ssq_out;       // residual GEMV: this launch's per-CTA sums of squares [nb][grid]
   int* err;             // device error word (bounded waits)
+  uint32_t wait_limit;  // polls of a ring wait before it gives up (drains keep kWaitLimit)
   int ns;               // stages of the weight ring
   // optional (pf_W null: off): the next decode GEMV of the stream; this CTA
   // pulls the start of that kernel's CTA region into L2 once its own loads
@@ -292,7 +296,14 @@ cudaError_t launch_select(const int3* stats, const uint8_t* mask, const uint8_t*
                    int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
                    uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
                    const uint8_t* active, const float* rel, uint8_t* rel_valid, const uint8_t* s2_forced,
-                   uint8_t* relevant, float* rel_out, cudaStream_t st);
+                   uint8_t* relevant, float* rel_out, const uint16_t* sched, cudaStream_t st);
+// Stage 3's schedule per sequence ([B][L]): own = derived (or the caller's),
+// use = what the selection applies (sched of launch_select).  With Stage 3
+// adaptive off it clears ent_valid and zeroes ent_out; a sequence that sits
+// the step out keeps its state and gets zero outputs.
+void launch_schedule(const StepParams* prm, const float* ent, uint8_t* ent_valid, const uint16_t* forced,
+                     const uint8_t* active, int B, int L, uint16_t* own, uint16_t* use, float* ent_out,
+                     cudaStream_t st);
 
 template <typename T>
 void launch_im2col(Rows rows, int B, int S, const uint8_t* frames, int n_views, int img_h, int img_w,
@@ -315,9 +326,20 @@ void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part
 template <typename T>
 void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, const SplitPlan& sp, T* G, cudaStream_t st);
 void launch_residual(Rows rows, int B, int S, int hidden, const float* part, const SplitPlan& sp, cudaStream_t st);
+// TMA maps of a cache's K and V (bf16 caches): 3-D {head_dim, Tc, batch x
+// layers x heads}, boxes of 64 dimensions x 64 positions, 128-byte swizzle,
+// positions past Tc read as zeros.  The box of (sequence b, layer l, head h)
+// is at z = b * layers * heads + l * heads + h.
+struct KvMaps {
+  CUtensorMap k, v;
+};
+// Mixed-cache attention of one layer.  bf16: the K/V tiles come through kvm
+// (z_seq = layers x heads, z_layer = l x heads); fp32: from Kc / Vc (this
+// layer's slice, kv_seq_stride elements per sequence).
 template <typename T>
 void launch_attention(Rows rows, int B, int S, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc,
-                      size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, T* O, cudaStream_t st);
+                      size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, T* O, const KvMaps* kvm,
+                      int z_seq, int z_layer, int* err, uint32_t wait_limit, cudaStream_t st);
 // Stage 2 relevance of one layer (rows as for launch_attention; text rows are
 // positions text_lo .. P-1): part [B][n_heads][Nv] per head, then rel and
 // rel_out [B][Nv] summed over the heads in order, and rel_valid[b] = 1.
@@ -326,6 +348,15 @@ template <typename T>
 int launch_relevance(Rows rows, int B, int n_heads, int head_dim, const T* Q, const T* Kc, size_t kv_seq_stride,
                      int Tc, int Nv, int text_lo, int P, float* part, float* rel, float* rel_out, uint8_t* rel_valid,
                      const StepParams* prm, const uint8_t* active, cudaStream_t st);
+// Stage 3: one layer's normalized attention entropy per (sequence, head, text
+// row) into part [B][n_heads][P - text_lo] (returns 1 if it cannot run);
+// then, after the prefix pass, the per-layer means from part [L][B][...]
+// into the cache (ent [B][L], ent_valid [B]) and ent_out.
+template <typename T>
+int launch_layer_entropy(Rows rows, int B, int n_heads, int head_dim, const T* Q, const T* Kc, size_t kv_seq_stride,
+                         int Tc, int text_lo, int P, float* part, cudaStream_t st);
+void launch_entropy_finish(const float* part, int L, int B, int n_heads, int nt, float* ent, uint8_t* ent_valid,
+                           float* ent_out, const StepParams* prm, const uint8_t* active, cudaStream_t st);
 template <typename T>
 void launch_decode_embed(int B, int d, int D, int P, int hidden, int vocab, int n_bins, const T* tok_emb,
                          const int32_t* ids, const int32_t* forced, const StepParams* prm, float* Xd,
@@ -362,7 +393,7 @@ struct CopySpan {
   void* dst;
   size_t bytes;
 };
-constexpr int kMaxSpans = 16;
+constexpr int kMaxSpans = 24;
 struct CopyList {
   CopySpan span[kMaxSpans];
   int n;

@@ -120,12 +120,17 @@ __global__ void __launch_bounds__(256) attn_kernel(Rows rows, int n_heads, const
 //
 // One block of 4 warps per (64 query rows of one sequence, head); warp w owns
 // 16 rows.  Key tiles of 64 positions (aligned to absolute positions) are
-// double-buffered in shared memory by cp.async.  Per tile: S = Q K^T on the
-// tensor cores (fp32 accumulators), scale, causal mask by the row's absolute
-// position, online softmax in fp32, P rounded to bf16 and O += P V on the
-// tensor cores.  Masked keys contribute exact zeros and a fully masked tile
-// leaves a row's state unchanged, so a row's result does not depend on the
-// other rows of its block.
+// double-buffered in shared memory by TMA (cp.async.bulk.tensor) from the
+// cache's 3-D tensor maps {head_dim, position, sequence x layer x head}: one
+// 64 x 64 box per 64 dimensions of K and of V, 128-byte swizzled, completing
+// on the buffer's mbarrier; keys at or past Tc lie outside the map and arrive
+// as zeros.  Per tile: S = Q K^T on the tensor cores (fp32 accumulators),
+// scale, causal mask by the row's absolute position, online softmax in fp32,
+// P rounded to bf16 and O += P V on the tensor cores.  Masked keys contribute
+// exact zeros and a fully masked tile leaves a row's state unchanged, so a
+// row's result does not depend on the other rows of its block.  The waits
+// are bounded: a wait that gives up latches VLAC_ERR_TIMEOUT, the block
+// stops, and thread 0 lets the copies still in flight land before it exits.
 namespace {
 
 constexpr int kAQ = 64;   // query rows per block
@@ -137,31 +142,40 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t&
                : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                : "r"(addr));
 }
-// 16 bytes global -> shared, zero-filled when !valid
-__device__ __forceinline__ void cp16(uint32_t dst, const void* src, bool valid) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0) : "memory");
-}
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&v);
 }
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* tm, int x, int y, int z, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+      "[%5];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
+// Byte offset of (key r, dimension e) in a tile of 64-dimension boxes, each
+// box 64 rows of 128 bytes with the 16-byte chunks of row r XOR-ed by r % 8.
+__device__ __forceinline__ uint32_t sw_off(int r, int e) {
+  return (uint32_t)((e >> 6) * (kAK * 128) + r * 128 + ((((e & 63) >> 3) ^ (r & 7)) << 4));
+}
 
 template <int HD>
 __global__ void __launch_bounds__(kAW * 32) attn_mma_kernel(Rows rows, int n_heads, const bf16* __restrict__ Q,
-                                                            const bf16* __restrict__ Kc, const bf16* __restrict__ Vc,
-                                                            size_t kv_seq_stride, int Tc, int P, int parallel,
-                                                            int n_action, float scale, bf16* __restrict__ O) {
+                                                            const __grid_constant__ KvMaps kvm, int z_seq,
+                                                            int z_layer, int Tc, int P, int parallel, int n_action,
+                                                            float scale, bf16* __restrict__ O,
+                                                            int* __restrict__ err, uint32_t wait_limit) {
   pdl_wait();
   pdl_trigger();
-  constexpr int LD = HD + 8;        // padded row (elements): conflict-free ldmatrix
   constexpr int KS = HD / 16;       // k-steps of S = Q K^T
   constexpr int ND = HD / 8;        // 8-column tiles of O
-  constexpr int CH = HD * 2 / 16;   // 16-byte chunks per key row
-  extern __shared__ __align__(16) uint8_t dsm[];
-  bf16* Ks = reinterpret_cast<bf16*>(dsm);             // [2][kAK][LD]
-  bf16* Vs = Ks + 2 * kAK * LD;                        // [2][kAK][LD]
+  constexpr uint32_t kTile = (uint32_t)kAK * HD * 2;  // bytes of one K (or V) tile
+  extern __shared__ __align__(1024) uint8_t dsm[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsm) + 1023) & ~uintptr_t(1023));
+  // [buf][K | V][tile]
+  __shared__ __align__(8) uint64_t full[2];
   __shared__ int lim_s[kAQ];
-  __shared__ int maxlim_s;
+  __shared__ int maxlim_s, abort_s, never_s;
   const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int cnt = rows.off[b + 1] - rows.off[b];
   const int i0 = qt * kAQ;
@@ -177,28 +191,35 @@ __global__ void __launch_bounds__(kAW * 32) attn_mma_kernel(Rows rows, int n_hea
     }
     lim_s[tid] = lim;
   }
+  if (tid == 0) {
+    mbar_init(&full[0], 1);
+    mbar_init(&full[1], 1);
+    abort_s = 0;
+    never_s = 0;
+    mbar_fence_init();
+  }
   __syncthreads();
   if (tid == 0) {
     int m = 0;
     for (int q = 0; q < kAQ; ++q) m = max(m, lim_s[q]);
     maxlim_s = m;
   }
-  const bf16* Kh = Kc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
-  const bf16* Vh = Vc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
-  const uint32_t ks_base = smem_u32(Ks), vs_base = smem_u32(Vs);
+  const int z = b * z_seq + z_layer + h;
+  const uint32_t sm_base = smem_u32(sm);
+  auto ks_of = [&](int buf) { return sm_base + (uint32_t)(2 * buf) * kTile; };
+  auto vs_of = [&](int buf) { return sm_base + (uint32_t)(2 * buf + 1) * kTile; };
+  // issued by thread 0 only
   auto load_tile = [&](int tile, int buf) {
-    const int t0 = tile * kAK;
-    for (int c = tid; c < kAK * CH; c += kAW * 32) {
-      const int j = c / CH, q = c - j * CH, key = t0 + j;
-      const bool ok = key < Tc;
-      const size_t off = (size_t)(ok ? key : 0) * HD + q * 8;
-      const uint32_t so = (uint32_t)(((buf * kAK + j) * LD + q * 8) * 2);
-      cp16(ks_base + so, Kh + off, ok);
-      cp16(vs_base + so, Vh + off, ok);
+    mbar_expect_tx(&full[buf], 2 * kTile);
+#pragma unroll
+    for (int hh = 0; hh < HD / 64; ++hh) {
+      tma_load_3d(ks_of(buf) + (uint32_t)hh * (kAK * 128), &kvm.k, hh * 64, tile * kAK, z, &full[buf]);
+      tma_load_3d(vs_of(buf) + (uint32_t)hh * (kAK * 128), &kvm.v, hh * 64, tile * kAK, z, &full[buf]);
     }
-    asm volatile("cp.async.commit_group;" ::: "memory");
   };
-  load_tile(0, 0);
+  __syncthreads();
+  const int n_tiles = (maxlim_s + kAK - 1) / kAK;
+  if (tid == 0 && n_tiles > 0) load_tile(0, 0);
   // this warp's Q rows as A fragments (rows past the block's rows are zero)
   const int ra = warp * 16 + g, rb = ra + 8;  // rows of the block held by this thread
   uint32_t qa[KS][4];
@@ -215,22 +236,22 @@ __global__ void __launch_bounds__(kAW * 32) attn_mma_kernel(Rows rows, int n_hea
       qa[ks][3] = vb ? *reinterpret_cast<const uint32_t*>(qpb + e + 8) : 0u;
     }
   }
-  __syncthreads();
   const int lim_a = lim_s[ra], lim_b = lim_s[rb];
-  const int n_tiles = (maxlim_s + kAK - 1) / kAK;
   float o[ND][4];
 #pragma unroll
   for (int nd = 0; nd < ND; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
   float m_a = -INFINITY, m_b = -INFINITY, l_a = 0.f, l_b = 0.f;  // per-thread partial row sums
-  for (int tile = 0; tile < n_tiles; ++tile) {
+  int tile = 0;
+  for (; tile < n_tiles; ++tile) {
     const int buf = tile & 1;
-    if (tile + 1 < n_tiles) {
-      load_tile(tile + 1, buf ^ 1);
-      asm volatile("cp.async.wait_group 1;" ::: "memory");
-    } else {
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
+    // buffer buf ^ 1 was released by the previous tile's closing barrier
+    if (tid == 0 && tile + 1 < n_tiles) load_tile(tile + 1, buf ^ 1);
+    if (!mbar_wait(&full[buf], (uint32_t)(tile >> 1) & 1u, wait_limit, &abort_s)) {
+      set_error(err, VLAC_ERR_TIMEOUT);
+      abort_s = 1;
     }
     __syncthreads();
+    if (abort_s) break;
     // S = Q K^T for 64 keys: 8 n-tiles of 8 keys
     float sc[8][4];
 #pragma unroll
@@ -243,7 +264,7 @@ __global__ void __launch_bounds__(kAW * 32) attn_mma_kernel(Rows rows, int n_hea
         const int mi = lane >> 3, rr = lane & 7;
         const int key = 16 * np + (mi >> 1) * 8 + rr, dim = 16 * ks + (mi & 1) * 8;
         uint32_t k0, k1, k2, k3;
-        ldsm_x4(ks_base + (uint32_t)(((buf * kAK + key) * LD + dim) * 2), k0, k1, k2, k3);
+        ldsm_x4(ks_of(buf) + sw_off(key, dim), k0, k1, k2, k3);
         mma_bf16(sc[2 * np], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], k0, k1);
         mma_bf16(sc[2 * np + 1], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], k2, k3);
       }
@@ -297,12 +318,20 @@ __global__ void __launch_bounds__(kAW * 32) attn_mma_kernel(Rows rows, int n_hea
         const int mi = lane >> 3, rr = lane & 7;
         const int key = 16 * kk + (mi & 1) * 8 + rr, dim = 16 * np + (mi >> 1) * 8;
         uint32_t v0, v1, v2, v3;
-        ldsm_x4_t(vs_base + (uint32_t)(((buf * kAK + key) * LD + dim) * 2), v0, v1, v2, v3);
+        ldsm_x4_t(vs_of(buf) + sw_off(key, dim), v0, v1, v2, v3);
         mma_bf16(o[2 * np], pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3], v0, v1);
         mma_bf16(o[2 * np + 1], pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3], v2, v3);
       }
     }
     __syncthreads();  // the buffer is refilled next
+  }
+  if (abort_s) {
+    // tiles tile and tile + 1 may have been issued and not consumed: let
+    // their copies land (bounded, deaf to the give-up flag) before exit
+    if (tid == 0)
+      for (int u = tile; u < min(tile + 2, n_tiles); ++u)
+        (void)mbar_wait(&full[u & 1], (uint32_t)(u >> 1) & 1u, kWaitLimit, &never_s);
+    return;
   }
   // full row sums over the quad, then O / l
   l_a += __shfl_xor_sync(0xffffffffu, l_a, 1);
@@ -325,31 +354,34 @@ __global__ void __launch_bounds__(kAW * 32) attn_mma_kernel(Rows rows, int n_hea
 }
 
 template <int HD>
-void attn_mma_launch(Rows rows, int B, int S, int n_heads, const bf16* Q, const bf16* Kc, const bf16* Vc,
-                     size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, float scale, bf16* O,
+void attn_mma_launch(Rows rows, int B, int S, int n_heads, const bf16* Q, const KvMaps& kvm, int z_seq, int z_layer,
+                     int Tc, int P, int parallel, int n_action, float scale, bf16* O, int* err, uint32_t wait_limit,
                      cudaStream_t st) {
-  const size_t smem = (size_t)4 * kAK * (HD + 8) * sizeof(bf16);
+  const size_t smem = (size_t)4 * kAK * HD * sizeof(bf16) + 1024;  // K and V, two buffers, 1024-byte aligned
   static bool smem_set = false;  // raised once, before any graph capture of the kernel
   if (!smem_set) {
     cudaFuncSetAttribute(attn_mma_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     smem_set = true;
   }
   const dim3 grid((S + kAQ - 1) / kAQ, n_heads, B);
-  launch_k(attn_mma_kernel<HD>, grid, dim3(kAW * 32), smem, st, rows, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, P,
-           parallel, n_action, scale, O);
+  launch_k(attn_mma_kernel<HD>, grid, dim3(kAW * 32), smem, st, rows, n_heads, Q, kvm, z_seq, z_layer, Tc, P,
+           parallel, n_action, scale, O, err, wait_limit);
 }
 
 }  // namespace
 
 template <typename T>
 void launch_attention(Rows rows, int B, int S, int n_heads, int head_dim, const T* Q, const T* Kc, const T* Vc,
-                      size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, T* O, cudaStream_t st) {
+                      size_t kv_seq_stride, int Tc, int P, int parallel, int n_action, T* O, const KvMaps* kvm,
+                      int z_seq, int z_layer, int* err, uint32_t wait_limit, cudaStream_t st) {
   const float scale = 1.0f / sqrtf((float)head_dim);
   if constexpr (sizeof(T) == 2) {
     if (head_dim == 128)
-      attn_mma_launch<128>(rows, B, S, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, P, parallel, n_action, scale, O, st);
+      attn_mma_launch<128>(rows, B, S, n_heads, Q, *kvm, z_seq, z_layer, Tc, P, parallel, n_action, scale, O, err,
+                           wait_limit, st);
     else
-      attn_mma_launch<64>(rows, B, S, n_heads, Q, Kc, Vc, kv_seq_stride, Tc, P, parallel, n_action, scale, O, st);
+      attn_mma_launch<64>(rows, B, S, n_heads, Q, *kvm, z_seq, z_layer, Tc, P, parallel, n_action, scale, O, err,
+                          wait_limit, st);
     return;
   }
   dim3 grid((S + 15) / 16, n_heads, B);
@@ -499,6 +531,123 @@ int launch_relevance(Rows rows, int B, int n_heads, int head_dim, const T* Q, co
   return 0;
 }
 
+// ---- Stage 3 layer entropy (Sec. III-B, entropy-adaptive layer-wise reuse) --
+//
+// For one layer: per text row that sees two or more keys (positions
+// text_lo .. P-1; BOS sees one) and head, the normalized entropy
+// H / ln(keys) of the row's exact causal softmax, H = ln z - sum_j e^u_j u_j / z
+// with u_j = s_j - max_j s_j and z = sum_j e^u_j.  One block per (head,
+// sequence), warp w taking the text rows w, w + 8, ...; part[b][h][pos -
+// text_lo].
+template <typename T, int HD>
+__global__ void __launch_bounds__(kRelWarps * 32)
+    entropy_kernel(Rows rows, int n_heads, const T* __restrict__ Q, const T* __restrict__ Kc, size_t kv_seq_stride,
+                   int Tc, int text_lo, int P, float scale, float* __restrict__ part) {
+  pdl_wait();
+  pdl_trigger();
+  extern __shared__ __align__(16) float esm[];
+  const int h = blockIdx.x, b = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float* qs = esm + warp * HD;                           // [kRelWarps][HD]
+  float* sc = esm + kRelWarps * HD + (size_t)warp * Tc;  // [kRelWarps][Tc]
+  const int cnt = rows.off[b + 1] - rows.off[b];
+  const int hidden = n_heads * HD, nt = P - text_lo;
+  const T* Kh = Kc + (size_t)b * kv_seq_stride + (size_t)h * Tc * HD;
+  for (int i = warp; i < cnt; i += kRelWarps) {
+    const int pos = rows.idx[(size_t)b * rows.idx_stride + i];
+    if (pos < text_lo || pos >= P) continue;
+    const int nk = min(pos + 1, Tc);
+    const T* q = Q + (size_t)(rows.off[b] + i) * hidden + (size_t)h * HD;
+    for (int e = lane; e < HD; e += 32) qs[e] = to_f(q[e]);
+    __syncwarp();
+    float mx = -INFINITY;
+    for (int j = lane; j < nk; j += 32) {
+      const T* kr = Kh + (size_t)j * HD;
+      float dot = 0.f;
+#pragma unroll 8
+      for (int e = 0; e < HD; ++e) dot = fmaf(to_f(kr[e]), qs[e], dot);
+      sc[j] = dot * scale;
+      mx = fmaxf(mx, sc[j]);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float z = 0.f, zu = 0.f;
+    for (int j = lane; j < nk; j += 32) {
+      const float u = sc[j] - mx, e = expf(u);
+      z += e;
+      zu = fmaf(e, u, zu);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      z += __shfl_xor_sync(0xffffffffu, z, o);
+      zu += __shfl_xor_sync(0xffffffffu, zu, o);
+    }
+    if (lane == 0) part[((size_t)b * n_heads + h) * nt + (pos - text_lo)] = (logf(z) - zu / z) / logf((float)nk);
+    __syncwarp();  // before the next row overwrites qs and sc
+  }
+}
+
+// Per sequence and layer: the mean of the layer's normalized entropies over
+// text rows (in position order) and heads, summed in fp64; kept in the cache
+// for the next step's schedule and returned.  A sequence that sat the step
+// out keeps its entropies.
+__global__ void entropy_finish_kernel(const float* __restrict__ part, int L, int B, int n_heads, int nt,
+                                      float* __restrict__ ent, uint8_t* __restrict__ ent_valid,
+                                      float* __restrict__ ent_out, const StepParams* __restrict__ prm,
+                                      const uint8_t* __restrict__ active) {
+  pdl_wait();
+  pdl_trigger();
+  const int b = blockIdx.x;
+  const bool sat_out = prm->has_active && active && !active[b];
+  for (int l = threadIdx.x; l < L; l += blockDim.x) {
+    if (sat_out) {
+      ent_out[(size_t)b * L + l] = 0.f;
+      continue;
+    }
+    const float* pl = part + ((size_t)l * B + b) * n_heads * nt;
+    double sum = 0.0;
+    for (int r = 0; r < nt; ++r)
+      for (int h = 0; h < n_heads; ++h) sum += (double)pl[(size_t)h * nt + r];
+    const float e = (float)(sum / (double)(nt * n_heads));
+    ent[(size_t)b * L + l] = e;
+    ent_out[(size_t)b * L + l] = e;
+  }
+  if (threadIdx.x == 0 && !sat_out) ent_valid[b] = 1;
+}
+
+template <typename T>
+int launch_layer_entropy(Rows rows, int B, int n_heads, int head_dim, const T* Q, const T* Kc, size_t kv_seq_stride,
+                         int Tc, int text_lo, int P, float* part, cudaStream_t st) {
+  const size_t smem = (size_t)kRelWarps * (head_dim + Tc) * sizeof(float);
+  if (smem > 200 * 1024 || P <= text_lo) return 1;
+  static size_t smem_set[2] = {48 * 1024, 48 * 1024};  // raised once per kernel, before any graph capture of it
+  const float scale = 1.0f / sqrtf((float)head_dim);
+  if (head_dim == 128) {
+    if (smem > smem_set[0]) {
+      cudaFuncSetAttribute(entropy_kernel<T, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      smem_set[0] = smem;
+    }
+    launch_k(entropy_kernel<T, 128>, dim3(n_heads, B), dim3(kRelWarps * 32), smem, st, rows, n_heads, Q, Kc,
+             kv_seq_stride, Tc, text_lo, P, scale, part);
+  } else {
+    if (smem > smem_set[1]) {
+      cudaFuncSetAttribute(entropy_kernel<T, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      smem_set[1] = smem;
+    }
+    launch_k(entropy_kernel<T, 64>, dim3(n_heads, B), dim3(kRelWarps * 32), smem, st, rows, n_heads, Q, Kc,
+             kv_seq_stride, Tc, text_lo, P, scale, part);
+  }
+  return 0;
+}
+void launch_entropy_finish(const float* part, int L, int B, int n_heads, int nt, float* ent, uint8_t* ent_valid,
+                           float* ent_out, const StepParams* prm, const uint8_t* active, cudaStream_t st) {
+  launch_k(entropy_finish_kernel, dim3(B), dim3(64), 0, st, part, L, B, n_heads, nt, ent, ent_valid, ent_out, prm,
+           active);
+}
+template int launch_layer_entropy<float>(Rows, int, int, int, const float*, const float*, size_t, int, int, int,
+                                         float*, cudaStream_t);
+template int launch_layer_entropy<bf16>(Rows, int, int, int, const bf16*, const bf16*, size_t, int, int, int, float*,
+                                        cudaStream_t);
+
 template int launch_relevance<float>(Rows, int, int, int, const float*, const float*, size_t, int, int, int, int,
                                      float*, float*, float*, uint8_t*, const StepParams*, const uint8_t*,
                                      cudaStream_t);
@@ -507,8 +656,9 @@ template int launch_relevance<bf16>(Rows, int, int, int, const bf16*, const bf16
                                     cudaStream_t);
 
 template void launch_attention<float>(Rows, int, int, int, int, const float*, const float*, const float*, size_t,
-                                      int, int, int, int, float*, cudaStream_t);
+                                      int, int, int, int, float*, const KvMaps*, int, int, int*, uint32_t,
+                                      cudaStream_t);
 template void launch_attention<bf16>(Rows, int, int, int, int, const bf16*, const bf16*, const bf16*, size_t, int,
-                                     int, int, int, bf16*, cudaStream_t);
+                                     int, int, int, bf16*, const KvMaps*, int, int, int*, uint32_t, cudaStream_t);
 
 }  // namespace vlac

@@ -125,7 +125,7 @@ __device__ __forceinline__ void norm_rows_to_smem(const float* __restrict__ X, c
 // kept in A-fragment order: per 32-element K step and lane t the elements
 // (2t, 2t+1, 2t+8, 2t+9, 2t+16, 2t+17, 2t+24, 2t+25), one 16-byte load.
 //
-// Every ring wait is bounded (kWaitLimit polls).  A wait that gives up
+// Every ring wait is bounded (a.wait_limit polls).  A wait that gives up
 // latches VLAC_ERR_TIMEOUT and raises the CTA's give-up flag: the producer
 // stops issuing; the consumers run out their loops without computing or
 // handing stages back, so they stay in step at the named barriers; and a
@@ -293,7 +293,7 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
         const T* gbase = Wt + (size_t)g * TR * K;
         for (int c = 0; c < nchunk; ++c) {
           const int kn = min(KC, K - c * KC);
-          if (!mbar_wait(&empty_bar[stage], phase ^ 1u, kWaitLimit, abort)) {
+          if (!mbar_wait(&empty_bar[stage], phase ^ 1u, a.wait_limit, abort)) {
             set_error(a.err, VLAC_ERR_TIMEOUT);
             *abort = 1;
             break;
@@ -460,7 +460,7 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
         const int k0 = c * KC, n32 = min(KC, K - k0) >> 5;
         const int i0 = n32 * warp / kNC, i1 = n32 * (warp + 1) / kNC;
         bool ok = true;
-        if (lane == 0) ok = mbar_wait(&full_bar[stage], phase, kWaitLimit, abort);
+        if (lane == 0) ok = mbar_wait(&full_bar[stage], phase, a.wait_limit, abort);
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) {
           if (lane == 0) {
@@ -560,7 +560,7 @@ __global__ void __launch_bounds__((kNC + 1) * 32, 1) dgemv_kernel(DGemv a) {
         const int k0 = c * KC, kn = min(KC, K - k0), nv = kn / V;
         const int v0 = hk ? nv / 2 : 0, v1 = hk ? nv : nv / 2;  // this warp's 16-byte vectors of the rows
         bool ok = true;
-        if (lane == 0) ok = mbar_wait(&full_bar[stage], phase, kWaitLimit, abort);
+        if (lane == 0) ok = mbar_wait(&full_bar[stage], phase, a.wait_limit, abort);
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) {
           if (lane == 0) {
@@ -1014,97 +1014,128 @@ template void launch_dec_attention<bf16>(int, int, int, const bf16*, const bf16*
 
 // ---- action head -------------------------------------------------------------------
 
-// Bin logits of one action row: final RMSNorm (into shared memory as T), then
-// 16 bins per CTA, two per warp.  Rows of sequence b are
-// X + b * x_seq_stride + (row_of_seq[b] + j) * hidden (row_of_seq NULL = row j).
+// Action head of one action row, fused (Eq. 1): the final RMSNorm, the
+// logits of the n_bins action-bin rows of the LM head, and the top-2 / margin
+// reduction.  One thread-block cluster of kHeadCluster blocks per (row,
+// sequence) splits the bins: each block norms the row into its shared memory
+// as T and computes n_bins / kHeadCluster logits, four bins per warp at a time
+// (lanes over K, fp32 FMA, warp sum); block 0 then collects every logit over
+// distributed shared memory and one warp reduces them: argmax (lowest bin on
+// ties), l1 - l2, p1 - p2 = (1 - exp(l2 - l1)) / z and the entropy
+// ln z - sum_c p_c (l_c - l1), z = sum_c exp(l_c - l1).  The cluster
+// barriers are the hardware's; no block waits on a flag.
+constexpr int kHeadCluster = 8;
 template <typename T>
-__global__ void __launch_bounds__(256) head_logits_kernel(const float* __restrict__ X, const int* __restrict__ row_of_seq,
-                                                          size_t x_seq_stride, int hidden, int n_bins,
-                                                          const T* __restrict__ final_norm,
-                                                          const T* __restrict__ head_w, float eps,
-                                                          float* __restrict__ logits_ws) {
+__global__ void __launch_bounds__(256) head_fused_kernel(const float* __restrict__ X, const int* __restrict__ row_of_seq,
+                                                         size_t x_seq_stride, int hidden, int n_bins,
+                                                         const T* __restrict__ final_norm,
+                                                         const T* __restrict__ head_w, float eps,
+                                                         float* __restrict__ logits_ws, int D, int tok0,
+                                                         int32_t* __restrict__ ids, float* __restrict__ margins,
+                                                         float* __restrict__ gaps, float* __restrict__ logits,
+                                                         float* __restrict__ entropy) {
+  namespace cg = cooperative_groups;
+  cg::cluster_group cluster = cg::this_cluster();
   pdl_wait();
   pdl_trigger();
   extern __shared__ __align__(1024) uint8_t dsm[];
-  T* xs = reinterpret_cast<T*>(dsm);
+  T* xs = reinterpret_cast<T*>(dsm);                                     // [hidden]
+  const int per = n_bins / kHeadCluster;
+  float* lg_own = reinterpret_cast<float*>(dsm + (size_t)hidden * sizeof(T));  // [per]
+  float* lg_all = lg_own + per;                                          // [n_bins], block 0 only
+  const int rank = (int)cluster.block_rank();
   const int j = blockIdx.y, b = blockIdx.z;
   const int row = row_of_seq ? row_of_seq[b] + j : j;
   const float* x = X + (size_t)b * x_seq_stride + (size_t)row * hidden;
   norm_rows_to_smem<T, 1>(x, final_norm, hidden, eps, xs);
   constexpr int V = Vec<T>::n;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int c1 = blockIdx.x * 16 + warp * 2, c2 = c1 + 1;
   const int kv = hidden / V;
-  const uint4* w1 = reinterpret_cast<const uint4*>(head_w + (size_t)c1 * hidden);
-  const uint4* w2 = reinterpret_cast<const uint4*>(head_w + (size_t)c2 * hidden);
   const uint4* xv = reinterpret_cast<const uint4*>(xs);
-  float a1 = 0.f, a2 = 0.f;
-  for (int k = lane; k < kv; k += 32) {
-    float f1[V], f2[V], xf[V];
-    unpack<T>(__ldg(w1 + k), f1);
-    unpack<T>(__ldg(w2 + k), f2);
-    unpack<T>(xv[k], xf);
+  // four bins per warp at a time (their weight rows streamed side by side);
+  // per bin the same order: lanes over K, fp32 FMA, then the warp sum
+  for (int c = 4 * warp; c < per; c += 32) {
+    const uint4* w[4];
+    float a[4];
 #pragma unroll
-    for (int i = 0; i < V; ++i) {
-      a1 = fmaf(f1[i], xf[i], a1);
-      a2 = fmaf(f2[i], xf[i], a2);
+    for (int q = 0; q < 4; ++q) {
+      w[q] = reinterpret_cast<const uint4*>(head_w + (size_t)(rank * per + min(c + q, per - 1)) * hidden);
+      a[q] = 0.f;
     }
-  }
-  a1 = warp_allsum(a1);
-  a2 = warp_allsum(a2);
-  if (lane == 0) {
-    float* lg = logits_ws + ((size_t)b * gridDim.y + j) * n_bins;
-    lg[c1] = a1;
-    lg[c2] = a2;
-  }
-}
-
-// argmax (lowest bin on ties), top-2 logit gap, p1 - p2 and the entropy
-// -sum p ln p = ln z - sum p (l - l1) of one row.
-__global__ void __launch_bounds__(32) head_margin_kernel(const float* __restrict__ logits_ws, int n_bins, int D, int tok0,
-                                                         int32_t* __restrict__ ids, float* __restrict__ margins,
-                                                         float* __restrict__ gaps, float* __restrict__ logits,
-                                                         float* __restrict__ entropy) {
-  pdl_wait();
-  pdl_trigger();
-  const int j = blockIdx.x, b = blockIdx.y, lane = threadIdx.x;
-  const float* lg = logits_ws + ((size_t)b * gridDim.x + j) * n_bins;
-  float bv = -INFINITY;
-  int bi = 0x7fffffff;
-  for (int c = lane; c < n_bins; c += 32)
-    if (lg[c] > bv) {
-      bv = lg[c];
-      bi = c;
+    // a lane's K steps k = lane, lane + 32, ... in order; the loads of four
+    // steps are issued before their products
+    for (int k0 = lane; k0 < kv; k0 += 128) {
+      uint4 wr[4][4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) wr[u][q] = k0 + 32 * u < kv ? __ldg(w[q] + k0 + 32 * u) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (k0 + 32 * u >= kv) break;
+        float xf[V];
+        unpack<T>(xv[k0 + 32 * u], xf);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          float f[V];
+          unpack<T>(wr[u][q], f);
+#pragma unroll
+          for (int i = 0; i < V; ++i) a[q] = fmaf(f[i], xf[i], a[q]);
+        }
+      }
     }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-    if (ov > bv || (ov == bv && oi < bi)) {
-      bv = ov;
-      bi = oi;
+    for (int q = 0; q < 4; ++q) {
+      a[q] = warp_allsum(a[q]);
+      if (lane == 0 && c + q < per) lg_own[c + q] = a[q];
     }
   }
-  float v2 = -INFINITY, z = 0.f, zl = 0.f;
-  for (int c = lane; c < n_bins; c += 32) {
-    if (c != bi) v2 = fmaxf(v2, lg[c]);
-    const float e = expf(lg[c] - bv);
-    z += e;
-    zl = fmaf(e, lg[c] - bv, zl);
-  }
+  cluster.sync();
+  if (rank == 0 && warp == 0) {
+    for (int c = lane; c < n_bins; c += 32) lg_all[c] = *cluster.map_shared_rank(&lg_own[c % per], c / per);
+    __syncwarp();
+    const float* lg = lg_all;
+    float bv = -INFINITY;
+    int bi = 0x7fffffff;
+    for (int c = lane; c < n_bins; c += 32)
+      if (lg[c] > bv) {
+        bv = lg[c];
+        bi = c;
+      }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v2 = fmaxf(v2, __shfl_xor_sync(0xffffffffu, v2, o));
-  z = warp_allsum(z);
-  zl = warp_allsum(zl);
-  const size_t t = (size_t)b * D + tok0 + j;
-  if (lane == 0) {
-    ids[t] = bi;
-    margins[t] = -expm1f(v2 - bv) / z;
-    gaps[t] = bv - v2;
-    if (entropy) entropy[t] = logf(z) - zl / z;
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (ov > bv || (ov == bv && oi < bi)) {
+        bv = ov;
+        bi = oi;
+      }
+    }
+    float v2 = -INFINITY, z = 0.f, zl = 0.f;
+    for (int c = lane; c < n_bins; c += 32) {
+      if (c != bi) v2 = fmaxf(v2, lg[c]);
+      const float e = expf(lg[c] - bv);
+      z += e;
+      zl = fmaf(e, lg[c] - bv, zl);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v2 = fmaxf(v2, __shfl_xor_sync(0xffffffffu, v2, o));
+    z = warp_allsum(z);
+    zl = warp_allsum(zl);
+    const size_t t = (size_t)b * D + tok0 + j;
+    if (lane == 0) {
+      ids[t] = bi;
+      margins[t] = -expm1f(v2 - bv) / z;
+      gaps[t] = bv - v2;
+      if (entropy) entropy[t] = logf(z) - zl / z;
+    }
+    float* ws = logits_ws + ((size_t)b * gridDim.y + j) * n_bins;  // the vocabulary margin reads them
+    for (int c = lane; c < n_bins; c += 32) {
+      ws[c] = lg[c];
+      if (logits) logits[t * n_bins + c] = lg[c];
+    }
   }
-  if (logits)
-    for (int c = lane; c < n_bins; c += 32) logits[t * n_bins + c] = lg[c];
+  cluster.sync();  // every block's logits stay in place until block 0 has read them
 }
 
 // ---- margin over the whole vocabulary (Sec. IV-A, VLAC_MARGIN_VOCAB) ------------
@@ -1254,11 +1285,28 @@ void launch_head2(const float* X, const int* row_of_seq, size_t x_seq_stride, in
                   int n_bins, const T* final_norm, const T* head_w, float eps, float* logits_ws, int D, int tok0,
                   int32_t* ids, float* margins, float* gaps, float* logits, float* entropy, const VocabHead* vh,
                   cudaStream_t st) {
-  const size_t smem = (size_t)hidden * sizeof(T);
-  launch_k(head_logits_kernel<T>, dim3(n_bins / 16, rows_per_seq, B), dim3(256), smem, st, X, row_of_seq,
-           x_seq_stride, hidden, n_bins, final_norm, head_w, eps, logits_ws);
-  launch_k(head_margin_kernel, dim3(rows_per_seq, B), dim3(32), 0, st, logits_ws, n_bins, D, tok0, ids, margins, gaps,
-           logits, entropy);
+  const size_t smem = (size_t)hidden * sizeof(T) + (size_t)(n_bins / kHeadCluster + n_bins) * sizeof(float);
+  static size_t smem_set = 48 * 1024;  // raised once per kernel, before any graph capture of it
+  if (smem > smem_set) {
+    cudaFuncSetAttribute(head_fused_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    smem_set = smem;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(kHeadCluster, rows_per_seq, B);
+  cfg.blockDim = dim3(256);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kHeadCluster;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = g_pdl ? 2 : 1;
+  cudaLaunchKernelEx(&cfg, head_fused_kernel<T>, X, row_of_seq, x_seq_stride, hidden, n_bins, final_norm, head_w, eps,
+                     logits_ws, D, tok0, ids, margins, gaps, logits, entropy);
   if (!vh) return;
   // the other rows of the LM head: every weight row read once per group of <= 8 action rows
   T* xh = static_cast<T*>(vh->xh);

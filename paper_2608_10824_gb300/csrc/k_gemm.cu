@@ -301,7 +301,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (*abort) {
         // every MMA issued so far must finish before TMEM and the tiles go away
         umma_commit(&drain_bar);
-        mbar_wait(&drain_bar, 0, wait_limit, &never);
+        mbar_wait(&drain_bar, 0, kWaitLimit, &never);
       }
     }
   } else {
@@ -377,7 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0 && abort_flag) {
     // let every bulk copy that was issued but not consumed land before exit
     for (int s = 0; s < n_stages; ++s)
-      if (prod_cnt[s] > cons_cnt[s]) mbar_wait(&full_bar[s], last_par[s], wait_limit, &never);
+      if (prod_cnt[s] > cons_cnt[s]) mbar_wait(&full_bar[s], last_par[s], kWaitLimit, &never);
   }
   fence_before();
   __syncthreads();
@@ -399,10 +399,10 @@ void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr
   const int full_tiles = sp.full_cols / tc::kBM, n_tiles = N / tc::kBM;
   // token blocks side by side when the rows can exceed one pass (the CTAs of
   // blocks a step does not need return at once)
-  // VLAC_GEMM_TOKEN_BLOCKS: 0 never, 1 whenever the rows exceed one pass;
-  // unset: above two passes of rows (at two passes the second block's CTAs
-  // re-read the weights from DRAM a wave later, where passes inside one CTA
-  // find them in L2)
+  // VLAC_GEMM_TOKEN_BLOCKS: 0 never, 1 whenever the rows exceed one pass.
+  // Two passes inside one CTA stream the weight tile twice; blocks side by
+  // side run the second pass on another SM at the same time, which pays off
+  // where the extra CTAs find idle SMs and costs a wave where they do not.
   static const int token_blocks = [] {
     const char* e = std::getenv("VLAC_GEMM_TOKEN_BLOCKS");
     return e ? (std::atoi(e) != 0 ? 1 : 0) : -1;
@@ -416,9 +416,19 @@ void launch_gemm_tc(const ActMaps* tmA, const CUtensorMap* tmW, const int* m_ptr
     return (e && std::atoi(e) == 0) ? 0 : 1;
   }();
   const int one_pass = chain_mode == 1 ? tc::kMaxTok : tc::kOnePass;
-  const bool tb_on = token_blocks == 1 ? m_cap > one_pass : token_blocks == 0 ? false : m_cap > 2 * tc::kMaxTok;
-  const int tb = tb_on ? (m_cap + tc::kMaxTok - 1) / tc::kMaxTok : 1;
-  dim3 grid(full_tiles + (n_tiles - full_tiles) * sp.tail, tb);
+  const int nx = full_tiles + (n_tiles - full_tiles) * sp.tail;
+  const int nb = (m_cap + tc::kMaxTok - 1) / tc::kMaxTok;
+  // unset: side by side above two passes, or where all the blocks' CTAs fit
+  // in about one and a third waves of SMs
+  static const int n_sm = [] {
+    int dev = 0, v = 152;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+    return v;
+  }();
+  const bool tb_on = m_cap > one_pass && (token_blocks == 1 ||
+                                          (token_blocks < 0 && (m_cap > 2 * tc::kMaxTok || 3 * nx * nb <= 4 * n_sm)));
+  const int tb = tb_on ? nb : 1;
+  dim3 grid(nx, tb);
   launch_k(tc::gemm_tc_kernel, grid, dim3(tc::kThreads), tc::kSmemBytes, st, *tmA, *tmW, m_ptr, m_cap, N, k_chunks,
            cps, out, sp.stride, full_tiles, sp.tail, sp.tail_p, sp.tail_stride, sp.tail_ld, chain_mode, err,
            wait_limit);

@@ -99,7 +99,8 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
                               int* __restrict__ user_idx, int* __restrict__ user_M,
                               const uint8_t* __restrict__ active, const float* __restrict__ rel,
                               uint8_t* __restrict__ rel_valid, const uint8_t* __restrict__ s2_forced,
-                              uint8_t* __restrict__ relevant, float* __restrict__ rel_out) {
+                              uint8_t* __restrict__ relevant, float* __restrict__ rel_out,
+                              const uint16_t* __restrict__ sched) {
   pdl_wait();
   pdl_trigger();
   extern __shared__ uint8_t smem[];
@@ -198,7 +199,8 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
     for (int v = tid; v < Nv; v += blockDim.x)
       if (s_stat[v]) idx_b[n_always + (nS - 1 - s_rank[v])] = 1 + v;
     for (int l = tid; l < L; l += blockDim.x)
-      M[(size_t)b * L + l] = S - (int)(((uint32_t)prm->permille[l] * (uint32_t)nS) / 1000u);
+      M[(size_t)b * L + l] =
+          S - (int)(((uint32_t)(sched ? sched[(size_t)b * L + l] : prm->permille[l]) * (uint32_t)nS) / 1000u);
     if (tid == 0) emit_slot[b] = parallel ? n_always - n_action : n_always - 1;
   }
   __syncthreads();
@@ -206,6 +208,46 @@ __global__ void select_kernel(const int3* __restrict__ stats, const uint8_t* __r
     for (int i = tid; i < S; i += blockDim.x) user_idx[(size_t)b * S + i] = idx_b[i];
   if (user_M)
     for (int l = tid; l < L; l += blockDim.x) user_M[(size_t)b * L + l] = M[(size_t)b * L + l];
+}
+
+// Stage 3's per-sequence schedule (Sec. III-B, entropy-adaptive layer-wise
+// reuse, this library's reading): with the option on and the previous step's
+// layer entropies e_l in the cache, t_l = hi - (hi - lo) * e_l per mille,
+// smoothed over depth (r_0 = t_0, r_l = r_{l-1} + weight/1000 * (t_l - r_{l-1}),
+// in fp64) and floored; otherwise the caller's schedule.  `own` receives the
+// derived schedule, `use` the one the selection applies (a lock-step replay
+// may impose another).
+__global__ void schedule_kernel(const StepParams* __restrict__ prm, const float* __restrict__ ent,
+                                uint8_t* __restrict__ ent_valid, const uint16_t* __restrict__ forced, int L,
+                                const uint8_t* __restrict__ active, uint16_t* __restrict__ own,
+                                uint16_t* __restrict__ use, float* __restrict__ ent_out) {
+  pdl_wait();
+  pdl_trigger();
+  const int b = blockIdx.x;
+  if (threadIdx.x != 0) return;
+  if (prm->has_active && active && !active[b]) {  // sat the step out: its state stays, its outputs are zero
+    for (int l = 0; l < L; ++l) {
+      own[(size_t)b * L + l] = 0;
+      use[(size_t)b * L + l] = prm->permille[l];
+      ent_out[(size_t)b * L + l] = 0.f;
+    }
+    return;
+  }
+  const bool adaptive = prm->s3_adaptive && ent_valid[b];
+  const double lo = prm->s3_lo, hi = prm->s3_hi, w = prm->s3_weight / 1000.0;
+  double r = 0.0;
+  for (int l = 0; l < L; ++l) {
+    uint16_t v = prm->permille[l];
+    if (adaptive) {
+      const double t = hi - (hi - lo) * (double)ent[(size_t)b * L + l];
+      r = l == 0 ? t : r + w * (t - r);
+      v = (uint16_t)fmin(1000.0, fmax(0.0, floor(r)));
+    }
+    own[(size_t)b * L + l] = v;
+    use[(size_t)b * L + l] = (prm->s3_adaptive && prm->has_s3_forced && forced) ? forced[(size_t)b * L + l] : v;
+    if (!prm->s3_adaptive) ent_out[(size_t)b * L + l] = 0.f;  // nothing measured this step
+  }
+  if (!prm->s3_adaptive) ent_valid[b] = 0;
 }
 
 // Row offsets of every layer: off[l][b] = sum of M[b'][l] over b' < b.
@@ -253,18 +295,24 @@ static cudaError_t select_smem_attr(size_t smem) {
   return cudaSuccess;
 }
 
+void launch_schedule(const StepParams* prm, const float* ent, uint8_t* ent_valid, const uint16_t* forced,
+                     const uint8_t* active, int B, int L, uint16_t* own, uint16_t* use, float* ent_out,
+                     cudaStream_t st) {
+  launch_k(schedule_kernel, dim3(B), dim3(32), 0, st, prm, ent, ent_valid, forced, L, active, own, use, ent_out);
+}
+
 cudaError_t launch_select(const int3* stats, const uint8_t* mask, const uint8_t* valid, const float* m_prev,
                           const StepParams* prm, const int8_t* override_, int B, int Nv, int S, int L, int P,
                           int parallel, int n_action, uint8_t* full, int* idx, int* M, int* off, int* emit_slot,
                           uint8_t* user_recomputed, uint8_t* user_gate_auto, int* user_idx, int* user_M,
                           const uint8_t* active, const float* rel, uint8_t* rel_valid, const uint8_t* s2_forced,
-                          uint8_t* relevant, float* rel_out, cudaStream_t st) {
+                          uint8_t* relevant, float* rel_out, const uint16_t* sched, cudaStream_t st) {
   const size_t smem = select_smem(Nv);
   cudaError_t e = select_smem_attr(smem);
   if (e != cudaSuccess) return e;
   e = launch_k(select_kernel, dim3(B), dim3(512), smem, st, stats, mask, valid, m_prev, prm, override_, Nv, S, L, P,
            parallel, n_action, full, idx, M, emit_slot, user_recomputed, user_gate_auto, user_idx, user_M, active, rel,
-           rel_valid, s2_forced, relevant, rel_out);
+           rel_valid, s2_forced, relevant, rel_out, sched);
   if (e != cudaSuccess) return e;
   return launch_k(plan_kernel, dim3(1), dim3(256), 0, st, M, B, L, off);
 }

@@ -102,7 +102,7 @@ extern "C" int vlac_select_noalloc(const vlac_dims* d, int batch, const uint8_t*
     return VLAC_ERR_CUDA;
   if (launch_select(stats, static_mask, valid, m_prev, prm, gate_override, batch, Nv, S, L, P, d->parallel,
                     d->n_action, full, idx, M, off, emit, recomputed, nullptr, nullptr, nullptr, nullptr, nullptr,
-                    nullptr, nullptr, nullptr, nullptr, st) != cudaSuccess)
+                    nullptr, nullptr, nullptr, nullptr, nullptr, st) != cudaSuccess)
     return VLAC_ERR_CUDA;
   return VLAC_OK;
 }

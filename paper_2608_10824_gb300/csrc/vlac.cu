@@ -103,6 +103,14 @@ struct vlac_ctx {
   void* vh_rows;            // whole-vocabulary margin: normed action rows [rows][hidden] (T)
   float* vh_logits;         // and their logits over the non-bin rows [rows][vocab - n_bins]
   bool vm_on = false;       // this step computes the whole-vocabulary margin
+  // Stage 3 adaptive: per-layer entropies per (sequence, head, text row)
+  // [L][B][n_heads][nt], the schedule derived [B][L] and applied [B][L], the
+  // replayed schedule [B][L] and the entropies returned [B][L]
+  float* ent_part;
+  uint16_t *sched_own, *sched_use, *in_s3_forced;
+  float* o_lent;
+  bool s3_on = false;  // this step measures the layer entropies
+  int text_lo = 0, n_textrows = 0;  // text rows after the image: positions text_lo .. P-1
   cudaStream_t cap_stream = nullptr;
   bool use_graph = true;
   bool fatal = false;  // a launch was refused for exceeding a workspace buffer
@@ -127,16 +135,19 @@ struct vlac_cache {
   cudaGraphExec_t gexec = nullptr;
   int eager_steps = 0;
   uint64_t graph_launches = 0;
-  int graph_sig = 0;  // what the graph was captured with: Stage 2 (0 off, 1 + layer) * 2 + the vocabulary margin
+  int graph_sig = 0;  // what the graph was captured with: Stage 2 (0 off, 1 + layer), the vocabulary margin, Stage 3
   void *K, *V;
   float* H;
   uint8_t *prev, *valid;
   float* m_prev;
   float* rel;          // [B][Nv] the last step's Stage-2 relevance
   uint8_t* rel_valid;  // [B] rel holds one
+  float* ent;          // [B][L] the last step's per-layer attention entropy (Stage 3 adaptive)
+  uint8_t* ent_valid;  // [B] ent holds it
   int32_t* prev_ids;   // [B][n_action] the previous step's action bins
   uint8_t* ids_valid;  // [B] prev_ids holds them
   size_t kv_seq_stride, h_seq_stride;  // elements per sequence
+  KvMaps kvm;                          // TMA maps of K and V (bf16)
 };
 
 #define CK(x)                                  \
@@ -196,6 +207,21 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t c
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 3-D bf16 tensor {cols, rows, planes} (cols contiguous, planes of rows x
+// cols), box = 64 columns x box_rows x 1, 128B swizzle; reads outside it are zeros.
+static bool make_map3(CUtensorMap* m, const void* base, uint64_t planes, uint64_t rows, uint64_t cols,
+                      uint32_t box_rows) {
+  EncodeTiledFn enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {cols, rows, planes};
+  cuuint64_t strides[2] = {cols * 2, rows * cols * 2};
+  cuuint32_t box[3] = {64, box_rows, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // ---- create / destroy -----------------------------------------------------------
 
 extern "C" int vlac_destroy(vlac_ctx* c) {
@@ -242,6 +268,8 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   c->Nv = d.n_views * (d.img_h / d.patch) * (d.img_w / d.patch);
   c->has_p = d.proprio_dim > 0;
   c->P = d.n_text + c->Nv + c->has_p;
+  c->text_lo = 1 + c->Nv + c->has_p;
+  c->n_textrows = c->P - c->text_lo;
   c->S = c->P + (d.parallel ? d.n_action : 0);
   c->Tc = c->S + (d.parallel ? 0 : d.n_action - 1);
   c->pdim = d.patch * d.patch * 3;
@@ -470,6 +498,11 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->in_forced, Bm * d.n_action * 4, base);
     sc.take(c->in_active, Bm, base);
     sc.take(c->in_s2_forced, Bm * c->Nv, base);
+    sc.take(c->in_s3_forced, Bm * L * 2, base);
+    sc.take(c->sched_own, Bm * L * 2, base);
+    sc.take(c->sched_use, Bm * L * 2, base);
+    sc.take(c->o_lent, Bm * L * 4, base);
+    sc.take(c->ent_part, L * Bm * d.n_heads * std::max(c->n_textrows, 1) * 4, base);
     sc.take(c->o_ids, Bm * d.n_action * 4, base);
     sc.take(c->o_margins, Bm * d.n_action * 4, base);
     sc.take(c->o_gaps, Bm * d.n_action * 4, base);
@@ -552,8 +585,8 @@ static size_t cache_layout(const vlac_ctx* c, int B, char* base, vlac_cache* k) 
   void* K;
   void* V;
   float* H;
-  uint8_t *prev, *valid, *rel_valid, *ids_valid;
-  float *m_prev, *rel;
+  uint8_t *prev, *valid, *rel_valid, *ids_valid, *ent_valid;
+  float *m_prev, *rel, *ent;
   int32_t* prev_ids;
   const size_t kv = (size_t)d.n_layers * d.n_heads * c->Tc * d.head_dim;
   const size_t hs = (size_t)d.n_layers * c->S * d.hidden;
@@ -567,7 +600,10 @@ static size_t cache_layout(const vlac_ctx* c, int B, char* base, vlac_cache* k) 
   cv.take(rel_valid, (size_t)B, base);
   cv.take(prev_ids, (size_t)B * d.n_action * 4, base);
   cv.take(ids_valid, (size_t)B, base);
+  cv.take(ent, (size_t)B * d.n_layers * 4, base);
+  cv.take(ent_valid, (size_t)B, base);
   if (k) {
+    k->ent = ent; k->ent_valid = ent_valid;
     k->K = K; k->V = V; k->H = H; k->prev = prev; k->m_prev = m_prev; k->valid = valid;
     k->rel = rel; k->rel_valid = rel_valid;
     k->prev_ids = prev_ids; k->ids_valid = ids_valid;
@@ -593,6 +629,15 @@ extern "C" int vlac_cache_init(vlac_ctx* c, void* mem, size_t bytes, int batch, 
   k->ctx = c;
   k->B = batch;
   cache_layout(c, batch, static_cast<char*>(mem), k);
+  if (c->bf16) {
+    // the prefix attention's K/V tiles: rows of head_dim, Tc positions per (sequence, layer, head)
+    const uint64_t planes = (uint64_t)batch * c->d.n_layers * c->d.n_heads;
+    if (!make_map3(&k->kvm.k, k->K, planes, c->Tc, c->d.head_dim, 64) ||
+        !make_map3(&k->kvm.v, k->V, planes, c->Tc, c->d.head_dim, 64)) {
+      delete k;
+      return VLAC_ERR_CUDA;
+    }
+  }
   if (cudaMemset(mem, 0, need) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
     (void)cudaGetLastError();
     delete k;
@@ -617,10 +662,12 @@ extern "C" int vlac_reset(vlac_cache* k, int seq, void* stream) {
     CK(cudaMemsetAsync(k->valid, 0, (size_t)k->B, st));
     CK(cudaMemsetAsync(k->rel_valid, 0, (size_t)k->B, st));
     CK(cudaMemsetAsync(k->ids_valid, 0, (size_t)k->B, st));
+    CK(cudaMemsetAsync(k->ent_valid, 0, (size_t)k->B, st));
   } else {
     CK(cudaMemsetAsync(k->valid + seq, 0, 1, st));
     CK(cudaMemsetAsync(k->rel_valid + seq, 0, 1, st));
     CK(cudaMemsetAsync(k->ids_valid + seq, 0, 1, st));
+    CK(cudaMemsetAsync(k->ent_valid + seq, 0, 1, st));
   }
   return VLAC_OK;
 }
@@ -664,6 +711,7 @@ template <typename T>
 void dgemv(vlac_ctx* c, const DGemv& a_in, int epi, int nb, cudaStream_t st) {
   DGemv a = a_in;
   a.ns = c->gemv_ns;
+  a.wait_limit = c->wait_limit;
   // the stage ring must fit next to the input vector in shared memory
   const size_t xs = ((size_t)nb * a.K * sizeof(T) + 1023) / 1024 * 1024;
   while (a.ns > 2 && (size_t)a.ns * dgemv_stage_bytes() + (xs > 64 * 1024 ? 0 : xs) > 200 * 1024) --a.ns;
@@ -700,10 +748,11 @@ void gemm(vlac_ctx* c, const ActMaps* tmA, const CUtensorMap* tmW, const T* A, c
 // the previous layer record their input there; H NULL at layer 0), q/k/v
 // with RoPE and the K/V scatter into Kc_l / Vc_l (this layer of the cache),
 // the mixed-cache attention, o-projection + residual, the MLP norm, gate/up +
-// SwiGLU and down + residual.
+// SwiGLU and down + residual.  The bf16 attention reads the K/V tiles through
+// the cache's maps kvm; seq0 is the batch's first sequence in the cache.
 template <typename T>
 void prefix_layer(vlac_ctx* c, const Rows& rl, const int* off_prev, int B, int l, float* H, size_t h_seq_stride,
-                  T* Kc_l, T* Vc_l, size_t kv_seq_stride, cudaStream_t st) {
+                  T* Kc_l, T* Vc_l, size_t kv_seq_stride, const KvMaps* kvm, int seq0, cudaStream_t st) {
   const vlac_dims& d = c->d;
   const int S = c->S, Hd = d.hidden, F = d.ffn, nh = d.n_heads, hd = d.head_dim;
   const float eps = d.rms_eps;
@@ -730,7 +779,8 @@ void prefix_layer(vlac_ctx* c, const Rows& rl, const int* off_prev, int B, int l
   }
   {
     ProfScope ps_(c, VLAC_PROF_PREFIX_ATTN, 0, st);
-    launch_attention<T>(rl, B, S, nh, hd, Q, Kc_l, Vc_l, kv_seq_stride, c->Tc, c->P, d.parallel, d.n_action, AO, st);
+    launch_attention<T>(rl, B, S, nh, hd, Q, Kc_l, Vc_l, kv_seq_stride, c->Tc, c->P, d.parallel, d.n_action, AO, kvm,
+                        d.n_layers * nh, (seq0 * d.n_layers + l) * nh, c->err, c->wait_limit, st);
   }
   gemm<T>(c, &c->tm_AO, c->bf16 ? &c->tm_o[l] : nullptr, AO, c->wo[l], ml, Hd, Hd, so, st);
   {
@@ -759,7 +809,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
                      c->o_entropy, c->o_vm,    c->o_delta};
   VocabHead vh{c->head_full, c->d.vocab - c->d.n_bins, c->vh_rows, c->vh_logits, c->o_vm};
   const VocabHead* vhp = c->vm_on ? &vh : nullptr;
-  const int head_launches = c->vm_on ? (vh.n_rows ? 5 : 4) : 2;
+  const int head_launches = c->vm_on ? (vh.n_rows ? 4 : 3) : 1;
   const vlac_step_out* out = &outv;
   const uint8_t* frames = c->in_frames;
   const int32_t* prompt = c->in_prompt;
@@ -787,12 +837,19 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
                        out->static_mask, st);
   }
   {
+    // Stage 3's per-sequence schedule (the caller's unless adaptive)
+    ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
+    launch_schedule(c->prm, k->ent, k->ent_valid, c->in_s3_forced, c->in_active, B, L, c->sched_own, c->sched_use,
+                    c->o_lent, st);
+  }
+  {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_select(c->stats, c->mask, k->valid, k->m_prev, c->prm, ovr, B, c->Nv, S, L, c->P, d.parallel, D, c->full,
                   c->idx, c->M, c->off, c->emit_slot, out->recomputed, out->gate_auto, out->idx, out->M,
-                  c->in_active, k->rel, k->rel_valid, c->in_s2_forced, out->relevant, out->relevance, st);
+                  c->in_active, k->rel, k->rel_valid, c->in_s2_forced, out->relevant, out->relevance, c->sched_use,
+                  st);
   }
-  c->launches += 3;
+  c->launches += 4;
 
   // layer-0 inputs of the recomputed rows
   Rows r0{c->off, c->idx, S, c->X};
@@ -813,7 +870,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
     Rows rl{c->off + (size_t)l * (B + 1), c->idx, S, c->X};
     const int* off_prev = l == 0 ? rl.off : c->off + (size_t)(l - 1) * (B + 1);
     prefix_layer<T>(c, rl, off_prev, B, l, l == 0 ? nullptr : k->H + (size_t)l * S * Hd, k->h_seq_stride,
-                    Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, st);
+                    Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, &k->kvm, 0, st);
     if (c->s2_on && l == c->s2_layer) {
       // Stage 2: the text rows' attention on the visual keys of this layer (Q
       // still holds this layer's rows)
@@ -824,6 +881,20 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
         c->fatal = true;
       c->launches += 2;
     }
+    if (c->s3_on) {
+      // Stage 3 adaptive: this layer's attention entropy of the text rows
+      ProfScope ps_(c, VLAC_PROF_PREFIX_ATTN, 0, st);
+      if (launch_layer_entropy<T>(rl, B, nh, hd, Q, Kc + l * kv_layer, k->kv_seq_stride, c->Tc, c->text_lo, c->P,
+                                  c->ent_part + (size_t)l * B * nh * c->n_textrows, st))
+        c->fatal = true;
+      c->launches += 1;
+    }
+  }
+  if (c->s3_on) {
+    ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
+    launch_entropy_finish(c->ent_part, L, B, nh, c->n_textrows, k->ent, k->ent_valid, c->o_lent, c->prm,
+                          c->in_active, st);
+    c->launches += 1;
   }
   // action head on the prefix pass: the last text row, or the parallel action block
   {
@@ -1025,10 +1096,10 @@ int run_body(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
 // the second captures the body into a graph, which every later step replays.
 int run_step(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   if (!c->use_graph || c->prof_on) return run_body(c, k, st);
-  const int sig = (c->s2_on ? 1 + c->s2_layer : 0) * 2 + (c->vm_on ? 1 : 0);
+  const int sig = ((c->s2_on ? 1 + c->s2_layer : 0) * 2 + (c->vm_on ? 1 : 0)) * 2 + (c->s3_on ? 1 : 0);
   if (k->gexec && k->graph_sig != sig) {
-    // Stage 2 or the whole-vocabulary margin switched on or off, or Stage 2
-    // moved to another layer: the launch list
+    // Stage 2, Stage 3 adaptive or the whole-vocabulary margin switched on or
+    // off, or Stage 2 moved to another layer: the launch list
     // differs, so the graph is captured again (after one eager step)
     cudaGraphExecDestroy(k->gexec);
     cudaGraphDestroy(k->graph);
@@ -1100,6 +1171,17 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   p.s2_top_k = s2_k;
   p.s2_layer = s2_k > 0 ? s2_l : 0;
   p.has_s2_forced = (s2_k > 0 && opts->s2_forced) ? 1 : 0;
+  p.s3_adaptive = (opts && opts->s3_adaptive) ? 1 : 0;
+  if (p.s3_adaptive) {
+    if (opts->s3_lo < 0 || opts->s3_lo > opts->s3_hi || opts->s3_hi > 1000 || opts->s3_weight < 0 ||
+        opts->s3_weight > 1000)
+      return VLAC_ERR_INVALID_ARG;
+    p.s3_lo = opts->s3_lo;
+    p.s3_hi = opts->s3_hi;
+    p.s3_weight = opts->s3_weight;
+    p.has_s3_forced = opts->s3_forced ? 1 : 0;
+    if (c->n_textrows < 1) return VLAC_ERR_UNSUPPORTED;  // no text rows after the image to measure
+  }
   // an error latched by an earlier step on this context is reported first
   if (*c->err_host) {
     const int e = *c->err_host;
@@ -1113,7 +1195,7 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   const size_t fb = (size_t)d.n_views * d.img_h * d.img_w * 3;
   CopyList in{};
   auto add = [](CopyList& l, const void* src, void* dst, size_t bytes) {
-    if (src && dst && bytes) l.span[l.n++] = CopySpan{src, dst, bytes};
+    if (src && dst && bytes && l.n < kMaxSpans) l.span[l.n++] = CopySpan{src, dst, bytes};
   };
   add(in, frames, c->in_frames, (size_t)B * fb);
   add(in, prompt_ids, c->in_prompt, (size_t)B * d.n_text * 4);
@@ -1122,6 +1204,7 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   if (p.has_forced) add(in, opts->forced_ids, c->in_forced, (size_t)B * D * 4);
   if (p.has_active) add(in, opts->active, c->in_active, (size_t)B);
   if (p.has_s2_forced) add(in, opts->s2_forced, c->in_s2_forced, (size_t)B * c->Nv);
+  if (p.has_s3_forced) add(in, opts->s3_forced, c->in_s3_forced, (size_t)B * d.n_layers * 2);
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_stage(p, c->prm, in, st);
@@ -1129,6 +1212,7 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   c->launches += 1;
   c->s2_on = p.s2_top_k > 0;
   c->s2_layer = p.s2_layer;
+  c->s3_on = p.s3_adaptive != 0;
   c->vm_on = mk == VLAC_MARGIN_VOCAB || out->vocab_margin != nullptr;
   int rc = run_step(c, k, st);
   if (rc) return rc;
@@ -1148,6 +1232,8 @@ extern "C" int vlac_step(vlac_ctx* c, vlac_cache* k, const uint8_t* frames, cons
   add(o, c->o_entropy, out->entropy, (size_t)B * D * 4);
   if (c->vm_on) add(o, c->o_vm, out->vocab_margin, (size_t)B * D * 4);
   add(o, c->o_delta, out->action_delta, (size_t)B * 4);
+  add(o, c->o_lent, out->layer_entropy, (size_t)B * d.n_layers * 4);
+  add(o, c->sched_own, out->schedule, (size_t)B * d.n_layers * 2);
   {
     ProfScope ps_(c, VLAC_PROF_OTHER, 0, st);
     launch_copies(o, st);
@@ -1171,7 +1257,7 @@ int layer_bench_impl(vlac_ctx* c, vlac_cache* k, int seq, int layer, const int32
   Rows rl{c->off, c->idx, c->S, c->X};
   T* Kc = static_cast<T*>(k->K) + (size_t)seq * k->kv_seq_stride + (size_t)layer * kv_layer;
   T* Vc = static_cast<T*>(k->V) + (size_t)seq * k->kv_seq_stride + (size_t)layer * kv_layer;
-  prefix_layer<T>(c, rl, rl.off, 1, layer, nullptr, 0, Kc, Vc, k->kv_seq_stride, st);
+  prefix_layer<T>(c, rl, rl.off, 1, layer, nullptr, 0, Kc, Vc, k->kv_seq_stride, &k->kvm, seq, st);
   CK(cudaMemcpyAsync(x, c->X, (size_t)M * Hd * sizeof(float), cudaMemcpyDeviceToDevice, st));
   CK(cudaGetLastError());
   return c->fatal ? VLAC_ERR_INVALID_ARG : VLAC_OK;
@@ -1235,6 +1321,12 @@ extern "C" int vlac_selftest_wait(vlac_ctx* c, uint32_t spin_limit) {
   CK(cudaMemcpy(&e, c->err, sizeof(int), cudaMemcpyDeviceToHost));
   CK(cudaMemset(c->err, 0, sizeof(int)));
   return e;
+}
+
+extern "C" int vlac_set_wait_limit(vlac_ctx* c, uint32_t polls) {
+  if (!c) return VLAC_ERR_INVALID_ARG;
+  c->wait_limit = polls;
+  return VLAC_OK;
 }
 
 extern "C" int vlac_prof_enable(vlac_ctx* c, int on) {

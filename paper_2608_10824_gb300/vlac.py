@@ -57,17 +57,20 @@ class Rational(C.Structure):
 class StepOpts(C.Structure):
     _fields_ = [("margin_kind", C.c_int32), ("reduction", C.c_int32), ("gate_override", C.c_void_p),
                 ("forced_ids", C.c_void_p), ("active", C.c_void_p), ("s2_top_k", C.c_int32), ("s2_layer", C.c_int32),
-                ("s2_forced", C.c_void_p)]
+                ("s2_forced", C.c_void_p), ("s3_adaptive", C.c_int32), ("s3_lo", C.c_int32),
+                ("s3_hi", C.c_int32), ("s3_weight", C.c_int32), ("s3_forced", C.c_void_p)]
 
 
 class StepOut(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in (
         "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
-        "static_mask", "idx", "M", "relevance", "relevant", "entropy", "vocab_margin", "action_delta")]
+        "static_mask", "idx", "M", "relevance", "relevant", "entropy", "vocab_margin", "action_delta",
+        "layer_entropy", "schedule")]
 
 
 EXPORTS = ["vlac_create", "vlac_destroy", "vlac_cache_bytes", "vlac_cache_init", "vlac_cache_destroy",
            "vlac_step", "vlac_reset", "vlac_sync_error", "vlac_launch_count", "vlac_selftest_wait",
+           "vlac_set_wait_limit",
            "vlac_prof_enable", "vlac_prof_read", "vlac_select_noalloc", "vlac_strerror", "vlac_layer_bench",
            "vlac_cache_load", "vlac_cache_store"]
 
@@ -93,6 +96,7 @@ def lib():
             L.vlac_launch_count.argtypes = [vp]
             L.vlac_launch_count.restype = C.c_uint64
             L.vlac_selftest_wait.argtypes = [vp, C.c_uint32]
+            L.vlac_set_wait_limit.argtypes = [vp, C.c_uint32]
             L.vlac_prof_enable.argtypes = [vp, i32]
             L.vlac_prof_read.argtypes = [vp, i32, C.POINTER(C.c_double), C.POINTER(C.c_uint64),
                                          C.POINTER(C.c_double)]
@@ -191,7 +195,9 @@ class Context:
                   "relevance": ((batch, d.n_visual), torch.float32),
                   "relevant": ((batch, d.n_visual), torch.uint8),
                   "entropy": ((batch, D), torch.float32), "vocab_margin": ((batch, D), torch.float32),
-                  "action_delta": ((batch,), torch.int32)}
+                  "action_delta": ((batch,), torch.int32),
+                  "layer_entropy": ((batch, d.n_layers), torch.float32),
+                  "schedule": ((batch, d.n_layers), torch.int16)}
         for k in want:
             shp, dt = shapes[k]
             out[k] = torch.zeros(shp, dtype=dt, device=dev)
@@ -200,12 +206,15 @@ class Context:
     def step(self, cache: "Cache", frames, prompt, proprio=None, tau_sim=(996, 1000), tau_margin: float = 0.0,
              permille=None, margin_kind: int = MARGIN_PROB, reduction: int = REDUCE_DEFAULT, gate_override=None,
              forced_ids=None, out: Optional[Dict] = None, want: Sequence[str] = (), stream=None,
-             active=None, s2_top_k: int = 0, s2_layer: Optional[int] = None, s2_forced=None) -> Dict:
+             active=None, s2_top_k: int = 0, s2_layer: Optional[int] = None, s2_forced=None,
+             s3_adaptive=None, s3_forced=None) -> Dict:
         """One step for every sequence of `cache`; inputs are CUDA tensors.
         Returns the dict of device output tensors (allocated unless given).
         s2_top_k > 0 turns on Stage 2 with the relevance of layer s2_layer
         (default: the middle layer); s2_forced (CUDA uint8 [B][Nv]) replaces
-        its removal set (lock-step replay)."""
+        its removal set (lock-step replay).  s3_adaptive = (lo, hi, weight)
+        per mille turns on the entropy-adaptive Stage 3; s3_forced (CUDA
+        uint16 [B][L]) replaces its schedule (lock-step replay)."""
         d = self.d
         if permille is None:
             permille = np.full(d.n_layers, 1000, dtype=np.uint16)
@@ -214,11 +223,14 @@ class Context:
             out = self.alloc_outputs(cache.batch, want)
         so = StepOut(*[_ptr(out.get(k)) for k in (
             "action_ids", "margins", "logit_gap", "recomputed", "step_margin", "gate_auto", "logits",
-            "static_mask", "idx", "M", "relevance", "relevant", "entropy", "vocab_margin", "action_delta")])
+            "static_mask", "idx", "M", "relevance", "relevant", "entropy", "vocab_margin", "action_delta",
+            "layer_entropy", "schedule")])
         if s2_layer is None:
             s2_layer = d.n_layers // 2
+        s3 = (0, 0, 0) if s3_adaptive is None else tuple(int(v) for v in s3_adaptive)
         opts = StepOpts(margin_kind, reduction, _ptr(gate_override), _ptr(forced_ids), _ptr(active), int(s2_top_k),
-                        int(s2_layer), _ptr(s2_forced))
+                        int(s2_layer), _ptr(s2_forced), int(s3_adaptive is not None), s3[0], s3[1], s3[2],
+                        _ptr(s3_forced))
         rc = lib().vlac_step(self._h, cache._h, frames.data_ptr(), prompt.data_ptr(), _ptr(proprio),
                              Rational(int(tau_sim[0]), int(tau_sim[1])), float(tau_margin),
                              permille.ctypes.data, C.byref(opts), C.byref(so), _stream_ptr(stream))
@@ -262,6 +274,10 @@ class Context:
 
     def selftest_wait(self, spin_limit: int) -> int:
         return lib().vlac_selftest_wait(self._h, spin_limit)
+
+    def set_wait_limit(self, polls: int):
+        """Test hook: polls after which the step kernels' bounded waits give up."""
+        _check(lib().vlac_set_wait_limit(self._h, int(polls)), "vlac_set_wait_limit")
 
 
 def select_noalloc(d, frames, prev_frames, valid, m_prev, tau_sim=(996, 1000), tau_margin: float = 0.0,

@@ -28,6 +28,10 @@ ID_EXEMPT_MARGIN = 1e-3
 # twice the bar.  The deep tests exempt exactly those ids, and require the
 # GPU's id to be the first maximum of the GPU's own logits.
 FLAG_TIE = 1e-4
+# At 32 layers the margins are held to 0.05 x LOGIT_TOL_DEEP (see compare), so
+# the library's m_{t-1} may sit on the other side of theta_m wherever the
+# oracle's lies within that band of it.
+FLAG_TIE_DEEP = 0.05 * LOGIT_TOL_DEEP
 # Stage 2 relevance, relative to the sequence's largest relevance.  At layer
 # 0 the kernel sums fp32 probabilities of the same bf16 (or fp32) Q and K the
 # oracle sums in fp64 (REL_TOL).  At a deeper layer of a bf16 model Q and K
@@ -39,6 +43,10 @@ FLAG_TIE = 1e-4
 # lies within twice the bar of the oracle's k-th / (k+1)-th midpoint.
 REL_TOL = {"bf16": 1e-4, "f32": 1e-5}
 REL_TOL_DEEP = {"bf16": 2e-3, "f32": 1e-5}
+# Stage 3 adaptive: a layer's normalized attention entropy is a mean of
+# functions of the same softmax probabilities the relevance sums, so it is held
+# to the deep relevance bar (absolute: the entropy is already normalized to 1).
+ENT_TOL = {"bf16": 2e-3, "f32": 1e-5}
 # Entropy of the bin softmax: H moves by at most max_j |l_j - E_p[l]| per unit
 # of logit error, about 5 for these models' logit spread, so the bar is five
 # times the logit bar; the library's entropy must also match the entropy of
@@ -94,15 +102,20 @@ class Lockstep:
         self.prev_m = None
         self.prev_rel = None
         self.prev_ids = None
+        self.prev_ent = None
         self.log = []
         self.logit_tol = logit_tol
 
     def step(self, frames, prompt, proprio, tau_sim, tau_m, permille, margin_kind=0, force_branch=None,
-             active=None, s2_top_k=0, s2_layer=None, s2_lockstep=True, want_vocab=False):
+             active=None, s2_top_k=0, s2_layer=None, s2_lockstep=True, want_vocab=False, s3=None,
+             s3_lockstep=True):
         """active: uint8 [B], 0 = the sequence sits the step out (both sides).
         s2_top_k > 0: Stage 2 on both sides; with s2_lockstep the library
         applies the oracle's removal set (its own is still compared).
-        want_vocab: also the whole-vocabulary margin (always with margin kind 2)."""
+        want_vocab: also the whole-vocabulary margin (always with margin kind 2).
+        s3 = (lo, hi, weight): the entropy-adaptive Stage 3 on both sides; with
+        s3_lockstep the library applies the oracle's schedule (its own is
+        still compared)."""
         torch = self.torch
         d, B = self.d, self.B
         act = None if active is None else np.ascontiguousarray(active, np.uint8)
@@ -112,7 +125,8 @@ class Lockstep:
         o = self.orc.step(self.oc, frames, prompt, proprio, tau_sim=tau_sim, tau_margin=tau_m,
                           permille=permille, margin_kind=margin_kind,
                           gate_override=None if force_branch is None else np.full(B, force_branch, np.int8),
-                          active=act, s2_top_k=s2_top_k, s2_layer=s2_layer, want_vocab_margin=vocab)
+                          active=act, s2_top_k=s2_top_k, s2_layer=s2_layer, want_vocab_margin=vocab,
+                          s3_adaptive=s3)
         # branch: free-running, except where the oracle's m_{t-1} sits in the tie zone
         ovr = np.full(B, -1, np.int8) if force_branch is None else np.full(B, force_branch, np.int8)
         if self.prev_m is not None and force_branch is None:
@@ -125,12 +139,16 @@ class Lockstep:
             tau_sim=tau_sim, tau_margin=tau_m, permille=permille, margin_kind=margin_kind,
             gate_override=torch.from_numpy(ovr).cuda(),
             forced_ids=torch.from_numpy(o["action_ids"].astype(np.int32)).cuda(),
-            want=("gate_auto", "logits", "static_mask", "idx", "M", "relevance", "relevant", "entropy", "action_delta")
+            want=("gate_auto", "logits", "static_mask", "idx", "M", "relevance", "relevant", "entropy", "action_delta",
+                  "layer_entropy", "schedule")
             + (("vocab_margin",) if vocab else ()),
             active=None if act is None else torch.from_numpy(act).cuda(),
             s2_top_k=s2_top_k, s2_layer=s2_layer,
             s2_forced=(torch.from_numpy(np.ascontiguousarray(o["relevant"])).cuda()
-                       if s2_top_k > 0 and s2_lockstep else None))
+                       if s2_top_k > 0 and s2_lockstep else None),
+            s3_adaptive=s3,
+            s3_forced=(torch.from_numpy(np.ascontiguousarray(o["schedule"]).view(np.int16)).cuda()
+                       if s3 is not None and s3_lockstep else None))
         torch.cuda.synchronize()
         g = {k: v.cpu().numpy() for k, v in g.items()}
         err = self.ctx.sync_error()
@@ -139,6 +157,12 @@ class Lockstep:
         stepped = np.ones(B, bool) if act is None else act != 0
         rep.update(compare_stage2(d, o, g, s2_top_k, self.prev_rel, stepped, s2_layer))
         rep.update(compare_signals(d, o, g, self.prev_ids, self.logit_tol, stepped))
+        rep.update(compare_stage3(d, o, g, s3, self.prev_ent, stepped))
+        if s3 is not None:
+            pe = o["layer_entropy"].copy()
+            if act is not None and self.prev_ent is not None:
+                pe[~stepped] = self.prev_ent[~stepped]
+            self.prev_ent = pe
         # the ids a sequence's next action delta is measured against: a sequence
         # that sat the step out keeps those of the last step it ran
         po, pg = o["action_ids"].copy(), g["action_ids"].copy()
@@ -157,13 +181,14 @@ class Lockstep:
         return o, g, rep
 
 
-def compare(d, o, g, prev_m, tau_m, logit_tol=None):
-    """Checks one step; returns a small report of the numeric gaps."""
+def compare(d, o, g, prev_m, tau_m, logit_tol=None, flag_tie=FLAG_TIE):
+    """Checks one step; returns a small report of the numeric gaps.  The
+    gate's own decision (gate_auto) must match outside `flag_tie` of theta_m."""
     B = o["action_ids"].shape[0]
     for k in ("static_mask", "idx", "M", "recomputed"):
         np.testing.assert_array_equal(g[k], o[k], err_msg=k)
     for b in range(B):
-        tie = prev_m is not None and abs(prev_m[b] - tau_m) < FLAG_TIE
+        tie = prev_m is not None and abs(prev_m[b] - tau_m) < flag_tie
         if not tie:
             assert g["gate_auto"][b] == o["gate_auto"][b], f"gate_auto[{b}]"
     tol = LOGIT_TOL[d.dtype] if logit_tol is None else logit_tol
@@ -213,6 +238,41 @@ def compare_stage2(d, o, g, top_k, prev_rel, stepped=None, s2_layer=0):
             assert not outside.any(), f"removal set differs outside the tie band: {np.flatnonzero(outside)}"
             diffs += int(bad.sum())
     return {"rel_diff": worst, "removal_diffs": diffs}
+def compare_stage3(d, o, g, s3, prev_ent, stepped=None):
+    """Stage 3 adaptive: the layer entropies within ENT_TOL of the oracle's;
+    the library's own schedule equal to the oracle's except for a layer whose
+    smoothed per-mille value, computed exactly from the oracle's previous
+    entropies, lies within (hi - lo) x ENT_TOL of an integer.  Off: the
+    caller's schedule is reported and nothing is measured."""
+    g_sched = g["schedule"].astype(np.int64) & 0xFFFF
+    if s3 is None:
+        assert not g["layer_entropy"].any()
+        np.testing.assert_array_equal(g_sched, o["schedule"])
+        return {"ent_diff": 0.0, "sched_diffs": 0}
+    lo, hi, w = s3
+    tol = ENT_TOL[d.dtype]
+    worst, diffs = 0.0, 0
+    for b in range(o["schedule"].shape[0]):
+        if stepped is not None and not stepped[b]:
+            assert not g["layer_entropy"][b].any() and not g_sched[b].any()
+            continue
+        err = float(np.max(np.abs(g["layer_entropy"][b].astype(np.float64) - o["layer_entropy"][b])))
+        assert err <= tol, f"layer entropy of sequence {b} differs by {err:.3e} > {tol}"
+        worst = max(worst, err)
+        bad = g_sched[b] != o["schedule"][b]
+        if bad.any():
+            assert prev_ent is not None, "a derived schedule without a previous step"
+            r, near = 0.0, []
+            for l, e in enumerate(prev_ent[b]):
+                t = hi - (hi - lo) * float(e)
+                r = t if l == 0 else r + (w / 1000.0) * (t - r)
+                near.append(abs(r - round(r)) <= (hi - lo) * tol + 1e-9)
+            outside = bad & ~np.array(near)
+            assert not outside.any(), f"schedule differs away from a rounding boundary at layers {np.flatnonzero(outside)}"
+            diffs += int(bad.sum())
+    return {"ent_diff": worst, "sched_diffs": diffs}
+
+
 def compare_signals(d, o, g, prev_ids, logit_tol=None, stepped=None):
     """Entropy within ENTROPY_FACTOR x the logit bar of the oracle's (and
     within fp32 rounding of the entropy of the library's own logits); the

@@ -74,3 +74,30 @@ def test_unsupported_dims():
     with pytest.raises(VlacError) as e:
         Context(d, synth.weights_to(synth.make_weights(d, seed=1), "cuda"))
     assert e.value.code in (-7, -1)
+
+
+@pytest.mark.parametrize("polls", [0, 1])
+def test_step_kernels_give_up_and_the_context_stays_usable(cuda_device, polls):
+    """The prefix GEMM's, the decode GEMV's and the prefix attention's bounded
+    waits, run out on purpose (0 polls: every wait gives up at once; 1 poll:
+    wherever a copy has not landed by the first poll): the step latches
+    VLAC_ERR_TIMEOUT (or, with 1 poll, may happen to finish), nothing hangs
+    or faults, and a normal step on a new cache of the same context then
+    matches the oracle."""
+    from paper_2608_10824_gb300.vlac import ERRORS
+    from tests.gpu_common import Lockstep
+    d = SMALL["small"]
+    w = synth.make_weights(d, seed=5)
+    ls = Lockstep(d, w)
+    frames, prompt, _ = episode(d, 2, seed=5)
+    f, p = torch.from_numpy(frames[0]).cuda(), torch.from_numpy(prompt).cuda()
+    ls.ctx.set_wait_limit(polls)
+    c = ls.ctx.new_cache(1)
+    ls.ctx.step(c, f, p)
+    torch.cuda.synchronize()
+    rc = ls.ctx.sync_error()
+    assert ERRORS.get(rc) == "VLAC_ERR_TIMEOUT" or (polls > 0 and rc == 0), rc
+    ls.ctx.set_wait_limit(1 << 24)
+    # the lock-step cache is a fresh one of the same context
+    for t in range(2):
+        ls.step(frames[t], prompt, None, (95, 100), 0.0, synth.linear_schedule(d.n_layers))

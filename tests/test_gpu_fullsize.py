@@ -21,7 +21,7 @@ import numpy as np
 import pytest
 
 import synth
-from tests.gpu_common import LOGIT_TOL_DEEP, Lockstep, compare
+from tests.gpu_common import FLAG_TIE_DEEP, LOGIT_TOL_DEEP, Lockstep, compare
 
 pytestmark = [pytest.mark.gpu, pytest.mark.timeout(1800)]
 
@@ -68,7 +68,13 @@ def test_oft7b_parity(cuda_device):
     assert _run_lockstep("oft7b", [0.0, 0.0], seed=12) == [1, 0]
 
 
-def test_batch7b_sampled_parity(cuda_device):
+@pytest.mark.parametrize("tau_m", [0.0, 0.02, 0.05, 0.1, 0.2])
+def test_batch7b_sampled_parity(cuda_device, tau_m):
+    """The batch of 8 at every theta_m of its sweep: the oracle runs two of the
+    eight sequences over the first frames (the parity window), the library
+    the whole batch.  The sampled sequences take the oracle's branch on both
+    sides; their gate's own decision must match the oracle's wherever the
+    oracle's m_{t-1} lies outside FLAG_TIE_DEEP of theta_m."""
     import torch
 
     import oracle
@@ -76,7 +82,7 @@ def test_batch7b_sampled_parity(cuda_device):
     d = synth.dims_for("batch7b")
     B, pick = d.max_batch, [0, 5]
     w_cpu, w_gpu = _weights(d, 13)
-    n = 2
+    n = 3 if tau_m == 0.0 else 2
     frames = synth.make_episode(d, n, seed=13, batch=B, kind="scene", speeds=synth.batch_speeds(B, seed=13))
     prompt = synth.make_prompt(d, seed=13, batch=B)
     pm = synth.linear_schedule(d.n_layers)
@@ -89,24 +95,37 @@ def test_batch7b_sampled_parity(cuda_device):
     pr = torch.from_numpy(np.ascontiguousarray(prompt)).cuda()
     want = ("gate_auto", "logits", "static_mask", "idx", "M")
     prev_m = None
+    branches = []
     for t in range(n):
-        o = orc.step(oc, frames[t][pick], prompt[pick], tau_sim=(996, 1000), tau_margin=0.0, permille=pm)
+        o = orc.step(oc, frames[t][pick], prompt[pick], tau_sim=(996, 1000), tau_margin=tau_m, permille=pm)
+        # the sampled sequences take the oracle's branch (their own gate
+        # decision is still compared, outside the deep tie band); the others
+        # follow their own gate
+        ovr = torch.full((B,), -1, dtype=torch.int8)
+        for i, b in enumerate(pick):
+            ovr[b] = int(o["recomputed"][i])
+        ovr = ovr.cuda()
         # the decoded bins are fed back, so the sampled rows take the oracle's
         # bins and the others their own: a copy of the cache runs the step
         # first to find those
         probe.mem.copy_(cache.mem)
-        own = ctx.step(probe, fr[t], pr, tau_sim=(996, 1000), tau_margin=0.0, permille=pm)["action_ids"]
+        own = ctx.step(probe, fr[t], pr, tau_sim=(996, 1000), tau_margin=tau_m, permille=pm,
+                       gate_override=ovr)["action_ids"]
         forced = own.clone()
         forced[pick] = torch.from_numpy(o["action_ids"].astype(np.int32)).cuda()
-        g = ctx.step(cache, fr[t], pr, tau_sim=(996, 1000), tau_margin=0.0, permille=pm, forced_ids=forced,
-                     want=want)
+        g = ctx.step(cache, fr[t], pr, tau_sim=(996, 1000), tau_margin=tau_m, permille=pm, forced_ids=forced,
+                     gate_override=ovr, want=want)
         torch.cuda.synchronize()
         assert ctx.sync_error() == 0
         g = {k: v.cpu().numpy()[pick] for k, v in g.items()}
-        rep = compare(d, o, g, prev_m, 0.0, LOGIT_TOL_DEEP)
-        print(f"batch7b frame {t}: max logit diff {rep['max_logit_diff']:.4e}, id mismatches {rep['id_mismatch']}")
+        rep = compare(d, o, g, prev_m, tau_m, LOGIT_TOL_DEEP, FLAG_TIE_DEEP)
+        branches.append(o["recomputed"].tolist())
+        print(f"batch7b tau {tau_m} frame {t}: recomputed {branches[-1]}, max logit diff "
+              f"{rep['max_logit_diff']:.4e}, id mismatches {rep['id_mismatch']}")
         prev_m = o["step_margin"].copy()
-    assert g["recomputed"].tolist() == [0, 0]
+    assert branches[0] == [1, 1]
+    if tau_m == 0.0:
+        assert all(b == [0, 0] for b in branches[1:])
     del ctx, cache, probe, orc
     gc.collect()
 
