@@ -34,6 +34,9 @@ import synth  # noqa: E402
 METRIC = "cached VLA steps/sec at OpenVLA-7B shape (1 GB300) and % of step roofline"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 EPISODE = 50
+# frames per synthetic episode: the batched serving workload runs 200-frame episodes
+EPISODE_LEN = {"batch7b": 200}
+TAU_SWEEP = (0.0, 0.02, 0.05, 0.1, 0.2)
 TAU_SIM = (996, 1000)
 CPU_LAYERS = 2  # the CPU oracle sample runs this many of the 32 layers
 # dram__bytes_read.sum + dram__bytes_write.sum of one dgemv_kernel launch,
@@ -327,6 +330,8 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-budget", type=float, default=25.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--tau-sweep", action="store_true",
+                    help="time K steps at every theta_m of the batched workload's sweep (0, .02, .05, .1, .2)")
     ap.add_argument("--layer-sweep", action="store_true",
                     help="time one decoder layer per recomputed-row count (the one-layer workload) instead")
     ap.add_argument("--stage2-top-k", type=int, default=0,
@@ -334,6 +339,8 @@ def main():
     ap.add_argument("--stage2-layer", type=int, default=None, help="layer whose attention gives the relevance")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    global EPISODE
+    EPISODE = EPISODE_LEN.get(args.config, EPISODE)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -437,10 +444,19 @@ def main():
     # ---- timed region: device-resident inputs ----
     ms, launches, clocks, step_roof, gemm_flops = timed_pass(W, None)
     value = aggregate_rate(world, B, K, ms / 1e3)   # sequence-steps per second
+    # ---- optionally: K more steps at every theta_m of the sweep ----
+    sweep = None
+    if args.tau_sweep:
+        sweep = []
+        for i, tau in enumerate(TAU_SWEEP):
+            s_ms, _, s_clocks, s_roof, _ = timed_pass(W + K * (1 + i), tau)
+            sweep.append({"tau_margin": tau, "value": aggregate_rate(world, B, K, s_ms / 1e3), "unit": "steps/s",
+                          "ms_per_step": s_ms / K, "fire_rate": s_roof["fire_rate"], "step_roofline": s_roof,
+                          "clocks": s_clocks})
     # ---- the same K frames once more at theta_m = 0: the gate never fires,
     # every step after the first of an episode takes the cached branch ----
     cached = None
-    if args.tau_margin != 0.0:
+    if args.tau_margin != 0.0 and not args.tau_sweep:
         c_ms, _, c_clocks, c_roof, _ = timed_pass(W + K, 0.0)
         cached = {"tau_margin": 0.0, "value": aggregate_rate(world, B, K, c_ms / 1e3), "unit": "steps/s",
                   "ms_per_step": c_ms / K, "step_roofline": c_roof, "clocks": c_clocks}
@@ -524,6 +540,7 @@ def main():
         "config": config_block(d, args),
         "step_roofline": step_roof,
         "cached_branch": cached,
+        "tau_sweep": sweep,
         "roofline": roof,
         "prefix_gemm": {"weight_gbs": gemm_gbs, "tflops": gemm_tfs, "launches": p_n,
                         "avg_launch_us": 1e3 * p_ms / max(p_n, 1)},
