@@ -194,6 +194,9 @@ def compare(d, o, g, prev_m, tau_m, logit_tol=None, flag_tie=FLAG_TIE):
     tol = LOGIT_TOL[d.dtype] if logit_tol is None else logit_tol
     diff = np.abs(g["logits"].astype(np.float64) - o["logits"])
     assert diff.max() <= tol, f"logits differ by {diff.max():.3e} > {tol}"
+    # at depth the largest difference is held to the floor-derived bar; the
+    # stated bar still holds for the typical (median) logit
+    assert np.median(diff) <= LOGIT_TOL[d.dtype], f"median logit difference {np.median(diff):.3e}"
     mism = g["action_ids"] != o["action_ids"]
     exempt = o["margins"] < ID_EXEMPT_MARGIN
     if logit_tol is not None:
@@ -206,7 +209,8 @@ def compare(d, o, g, prev_m, tau_m, logit_tol=None, flag_tie=FLAG_TIE):
     assert not bad.any(), (f"action ids differ outside the exemption: {np.argwhere(bad)}, "
                            f"oracle margins {o['margins'][bad]}")
     np.testing.assert_allclose(g["margins"], o["margins"], atol=max(tol * 0.05, 1e-6), rtol=0.05)
-    return {"max_logit_diff": float(diff.max()), "id_mismatch": int(mism.sum()),
+    return {"max_logit_diff": float(diff.max()), "median_logit_diff": float(np.median(diff)),
+            "id_mismatch": int(mism.sum()),
             "id_exempt": int(exempt.sum()), "recomputed": o["recomputed"].tolist()}
 
 

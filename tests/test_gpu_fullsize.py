@@ -48,7 +48,7 @@ def _run_lockstep(name, taus, seed):
         o, g, rep = ls.step(frames[t], prompt, None if prop is None else prop[t], (996, 1000), taus[t], pm)
         branches.append(int(o["recomputed"][0]))
         print(f"{name} frame {t}: recomputed {branches[-1]}, max logit diff {rep['max_logit_diff']:.4e}, "
-              f"id mismatches {rep['id_mismatch']}")
+              f"median {rep['median_logit_diff']:.4e}, id mismatches {rep['id_mismatch']}")
         if not branches[-1]:  # a cached step reused static patches at every layer
             assert g["M"][0].max() < d.pass_len
     del ls
@@ -121,7 +121,8 @@ def test_batch7b_sampled_parity(cuda_device, tau_m):
         rep = compare(d, o, g, prev_m, tau_m, LOGIT_TOL_DEEP, FLAG_TIE_DEEP)
         branches.append(o["recomputed"].tolist())
         print(f"batch7b tau {tau_m} frame {t}: recomputed {branches[-1]}, max logit diff "
-              f"{rep['max_logit_diff']:.4e}, id mismatches {rep['id_mismatch']}")
+              f"{rep['max_logit_diff']:.4e}, median {rep['median_logit_diff']:.4e}, "
+              f"id mismatches {rep['id_mismatch']}")
         prev_m = o["step_margin"].copy()
     assert branches[0] == [1, 1]
     if tau_m == 0.0:
