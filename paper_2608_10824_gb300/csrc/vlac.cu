@@ -255,6 +255,14 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
 
   vlac_ctx* c = new (std::nothrow) vlac_ctx();
   if (!c) return VLAC_ERR_OOM;
+  // test hook (fault injection on the host): VLAC_FAIL_ALLOC=n makes the
+  // n-th allocation of this call fail as cudaMalloc would, without calling it
+  int alloc_no = 0, fail_at = 0;
+  if (const char* e = std::getenv("VLAC_FAIL_ALLOC")) fail_at = std::atoi(e);
+  auto dev_alloc = [&](void** ptr, size_t bytes, bool host) {
+    if (++alloc_no == fail_at) return cudaErrorMemoryAllocation;
+    return host ? cudaMallocHost(ptr, bytes) : cudaMalloc(ptr, bytes);
+  };
   if (const char* e = std::getenv("VLAC_PDL")) g_pdl = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_GRAPH")) c->use_graph = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_GEMV_NS")) c->gemv_ns = std::max(2, std::min(24, std::atoi(e)));
@@ -307,7 +315,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     wc.take(c->rope_sin, (size_t)c->Tc * half * 4, base);
   };
   plan_w(nullptr);
-  if (cudaMalloc(&c->wmem, wc.off) != cudaSuccess) {
+  if (dev_alloc(reinterpret_cast<void**>(&c->wmem), wc.off, false) != cudaSuccess) {
     (void)cudaGetLastError();
     delete c;
     return VLAC_ERR_OOM;
@@ -353,7 +361,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
       }
     };
     plan_d(nullptr);
-    if (cudaMalloc(&c->dmem, dc.off) != cudaSuccess) {
+    if (dev_alloc(reinterpret_cast<void**>(&c->dmem), dc.off, false) != cudaSuccess) {
       (void)cudaGetLastError();
       return fail(VLAC_ERR_OOM);
     }
@@ -524,7 +532,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     sc.take(c->vh_logits, head_rows * std::max(d.vocab - d.n_bins, 1) * 4, base);
   };
   plan_s(nullptr);
-  if (cudaMalloc(&c->wsmem, sc.off) != cudaSuccess) {
+  if (dev_alloc(reinterpret_cast<void**>(&c->wsmem), sc.off, false) != cudaSuccess) {
     (void)cudaGetLastError();
     return fail(VLAC_ERR_OOM);
   }
@@ -549,7 +557,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
     if (cudaMemcpy(c->dp_ptrs, pp.data(), pp.size() * sizeof(void*), cudaMemcpyHostToDevice) != cudaSuccess)
       return fail(VLAC_ERR_CUDA);
   }
-  if (cudaMallocHost(&c->err_host, sizeof(int)) != cudaSuccess) {
+  if (dev_alloc(reinterpret_cast<void**>(&c->err_host), sizeof(int), true) != cudaSuccess) {
     (void)cudaGetLastError();
     c->err_host = nullptr;
     return fail(VLAC_ERR_OOM);

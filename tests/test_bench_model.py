@@ -87,3 +87,30 @@ def test_clock_samples_are_parsed():
     assert got["reasons"] == ["sw_power_cap"]
     c.p = None
     assert c.stop()["reasons"] == ["nvidia-smi unavailable"]
+
+
+def test_full_step_matches_the_papers_table_one():
+    """Table I counts one operation per multiply-add: 1.83-1.89 TFLOPs per full
+    OpenVLA step (average 1.87).  The benchmark counts 2 FLOPs per
+    multiply-add over the prefix pass and the six decode rows: half of it
+    lands inside the table's range."""
+    M, idx = _full()
+    F, _, _ = bench.batch_work(D, [M], [idx])
+    assert 1.83e12 <= F / 2 <= 1.89e12
+    assert F / 2 == pytest.approx(1.87e12, rel=0.01)
+
+
+def test_mean_flops_follow_the_mixture_law():
+    """Over an episode whose gate fires on a fraction f of the steps, the mean
+    counted work is f * F_full + (1 - f) * F_cached exactly; the paper's own
+    Long-suite figures obey the same law (0.24 * 1.88 + 0.76 * 1.43 = 1.54)."""
+    S = D.pass_len
+    M_full, idx = _full()
+    M_cached = [S - (int(p) * 230) // 1000 for p in synth.linear_schedule(D.n_layers)]
+    F_full = bench.batch_work(D, [M_full], [idx])[0]
+    F_cached = bench.batch_work(D, [M_cached], [idx])[0]
+    fired = [1, 0, 0, 0, 1, 0, 0, 0, 0, 0, 0, 0, 1, 0, 0, 0, 0, 0, 0, 0, 1, 0, 0, 0, 0]
+    total = sum(bench.batch_work(D, [M_full if b else M_cached], [idx])[0] for b in fired)
+    f = sum(fired) / len(fired)
+    assert total / len(fired) == pytest.approx(f * F_full + (1 - f) * F_cached, rel=1e-12)
+    assert 0.24 * 1.88 + 0.76 * 1.43 == pytest.approx(1.54, abs=0.005)

@@ -101,3 +101,56 @@ def test_step_kernels_give_up_and_the_context_stays_usable(cuda_device, polls):
     # the lock-step cache is a fresh one of the same context
     for t in range(2):
         ls.step(frames[t], prompt, None, (95, 100), 0.0, synth.linear_schedule(d.n_layers))
+
+
+@pytest.mark.parametrize("n", [1, 2, 3, 4])
+def test_allocation_failure_is_reported_and_leaks_nothing(cuda_device, monkeypatch, n):
+    """Host-side fault injection: the n-th allocation of vlac_create fails as
+    cudaMalloc would (VLAC_FAIL_ALLOC, no GPU fault involved).  The call
+    returns VLAC_ERR_OOM, frees what it had allocated, and the next create on
+    the same device works."""
+    from paper_2608_10824_gb300 import Context, VlacError
+    d = SMALL["small"]
+    w = synth.weights_to(synth.make_weights(d, seed=7), "cuda")
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    monkeypatch.setenv("VLAC_FAIL_ALLOC", str(n))
+    with pytest.raises(VlacError) as e:
+        Context(d, w, max_batch=1)
+    assert e.value.code == -3
+    torch.cuda.synchronize()
+    assert abs(torch.cuda.mem_get_info()[0] - free0) < (32 << 20)
+    monkeypatch.delenv("VLAC_FAIL_ALLOC")
+    ctx = Context(d, w, max_batch=1)
+    frames, prompt, _ = episode(d, 1, seed=7)
+    out = ctx.step(ctx.new_cache(1), torch.from_numpy(frames[0]).cuda(), torch.from_numpy(prompt).cuda())
+    torch.cuda.synchronize()
+    assert ctx.sync_error() == 0 and out["recomputed"].item() == 1
+
+
+def test_a_copied_cache_resumes_the_episode(cuda_device):
+    """The cache is the step's whole resumable state and lives in caller
+    memory: copying its bytes into a new cache of the same context (a
+    checkpoint) and stepping both gives the same outputs bit for bit."""
+    from paper_2608_10824_gb300 import Context
+    d = SMALL["small_oft"]
+    ctx = Context(d, synth.weights_to(synth.make_weights(d, seed=8), "cuda"), max_batch=1)
+    frames, prompt, prop = episode(d, 5, seed=8)
+    f = [torch.from_numpy(np.ascontiguousarray(x)).cuda() for x in frames]
+    p = torch.from_numpy(prompt).cuda()
+    pp = [torch.from_numpy(np.ascontiguousarray(x)).cuda() for x in prop]
+    pm = synth.linear_schedule(d.n_layers)
+    a = ctx.new_cache(1)
+    for t in range(3):
+        ctx.step(a, f[t], p, pp[t], permille=pm)
+    torch.cuda.synchronize()
+    b = ctx.new_cache(1)
+    b.mem.copy_(a.mem)
+    for t in (3, 4):
+        oa = ctx.step(a, f[t], p, pp[t], permille=pm, want=("logits", "idx"))
+        ob = ctx.step(b, f[t], p, pp[t], permille=pm, want=("logits", "idx"))
+        torch.cuda.synchronize()
+        for k in ("action_ids", "margins", "logits", "idx", "step_margin", "recomputed"):
+            assert torch.equal(oa[k], ob[k]), (t, k)
+    assert ctx.sync_error() == 0
+    assert torch.equal(a.mem, b.mem)
