@@ -197,13 +197,15 @@ int vlac_step(vlac_ctx* ctx, vlac_cache* cache, const uint8_t* frames, const int
               void* stream);
 
 /* Invalidates sequence `seq` (-1 = all): its next step runs the full pass as if
- * no cache existed (Algorithm 1, cache invalidation), and Stage 2 has no
- * previous relevance to use. */
+ * no cache existed (Algorithm 1, cache invalidation), and Stage 2 and Stage 3
+ * adaptive have no previous relevance or entropies to use. */
 int vlac_reset(vlac_cache* cache, int seq, void* stream);
 
-/* One decoder layer of the prefix pass on its own (the one-layer workload:
- * gather, q/k/v + RoPE + K/V scatter, mixed-cache attention, o-projection,
- * MLP, as vlac_step runs them for each layer).
+/* One decoder layer of the prefix pass on its own: Algorithm 1's partial
+ * forward ("recompute the non-cached tokens against the reused cache", Sec.
+ * III-B) for one layer, which is the one-layer workload: gather, q/k/v + RoPE
+ * + K/V scatter, mixed-cache attention, o-projection, MLP, as vlac_step runs
+ * them for each layer.
  *   seq, layer:  the cache sequence (< batch) and layer (< n_layers)
  *   pos:         device int32 [M], distinct positions of the rows, each below
  *                the prefix pass length S (n_text + visual + proprio, plus the
