@@ -464,7 +464,18 @@ struct DPass {
   size_t part_stride;
   float* attn_part;
   unsigned* attn_cnt;
+  // rolling L2 prefetch: the producer pulls the stage this many ring stages
+  // beyond the one it is issuing into L2 (0: off), so that HBM keeps
+  // streaming while the consumers wait at a grid barrier with the ring full
+  int pf_stages;
+  // grid barrier: 0 fence + atomic add + poll; 1 release add + acquire poll
+  int bar_mode;
+  // attention: up to kv_keys keys of the CTA's first item staged in shared
+  // memory a layer ahead (0: read from global)
+  int kv_keys;
 };
+size_t dpass_kv_bytes(int kv_keys);
+size_t dpass_smem_bytes(int hidden, int ffn, int nb, int ns, int kv_keys);
 bool dpass_supported(int hidden, int ffn, int n_heads, int head_dim, int nb, int ns);
 int launch_dpass(const DPass& a, int nb, int n_sm, cudaStream_t st);
 // Decode-streaming copy of a projection (W: [rows][K]); see k_decode.cu for the layout.

@@ -70,34 +70,134 @@ __device__ __forceinline__ Proj proj_of(const DPass& a, int l, int j) {
 }
 
 // Grid-wide barrier number `epoch` (1, 2, ...): every CTA arrives once.
+// bar_mode 1: the arrival is a release add at GPU scope (it orders the
+// CTA's writes before it, which the CTA barrier before it collects) and the
+// poll an acquire load; bar_mode 0: full fences around a relaxed add and a
+// volatile poll.
 __device__ __forceinline__ void grid_sync(const DPass& a, unsigned epoch, volatile int* abort) {
   consumers_sync();
   if (threadIdx.x == 0) {
-    __threadfence();
-    atomicAdd(a.bar, 1u);
     const unsigned target = epoch * gridDim.x;
     uint32_t it = 0;
-    if (!*abort) {
-      while (*reinterpret_cast<volatile unsigned*>(a.bar) < target) {
-        if (++it > kWaitLimit) {
-          set_error(a.err, VLAC_ERR_TIMEOUT);
-          *abort = 1;
-          break;
+    if (a.bar_mode == 1) {
+      asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(a.bar) : "memory");
+      if (!*abort) {
+        for (;;) {
+          unsigned v;
+          asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(a.bar) : "memory");
+          if (v >= target) break;
+          if (++it > kWaitLimit) {
+            set_error(a.err, VLAC_ERR_TIMEOUT);
+            *abort = 1;
+            break;
+          }
+          __nanosleep(20);
         }
-        __nanosleep(32);
       }
+    } else {
+      __threadfence();
+      atomicAdd(a.bar, 1u);
+      if (!*abort) {
+        while (*reinterpret_cast<volatile unsigned*>(a.bar) < target) {
+          if (++it > kWaitLimit) {
+            set_error(a.err, VLAC_ERR_TIMEOUT);
+            *abort = 1;
+            break;
+          }
+          __nanosleep(32);
+        }
+      }
+      __threadfence();
     }
-    __threadfence();
   }
   consumers_sync();
 }
 
+// The producer's walk over its ring stages: layer l, projection j, this
+// CTA's groups g of it, K chunks c, in the order the consumers take them.
+struct StageCursor {
+  int l, j, g, g1, c, nchunk, K, bx, nx;
+  const bf16* W;
+  bool done;
+  __device__ __forceinline__ StageCursor(const DPass& a, int bx_, int nx_)
+      : l(0), j(0), g(0), g1(0), c(0), nchunk(1), K(0), bx(bx_), nx(nx_), W(nullptr), done(a.L <= 0) {
+    if (!done) {
+      load(a);
+      skip(a);
+    }
+  }
+  __device__ __forceinline__ void load(const DPass& a) {
+    const Proj P = proj_of(a, l, j);
+    int g0;
+    dgemv_group_range((P.n_pairs + kDecGroupPairs - 1) / kDecGroupPairs, nx, bx, g0, g1);
+    g = g0;
+    c = 0;
+    K = P.K;
+    W = P.W;
+    nchunk = (P.K + kPKC - 1) / kPKC;
+  }
+  // past projections that give this CTA no group
+  __device__ __forceinline__ void skip(const DPass& a) {
+    while (!done && g >= g1) {
+      if (++j == 4) {
+        j = 0;
+        if (++l == a.L) {
+          done = true;
+          break;
+        }
+      }
+      load(a);
+    }
+  }
+  __device__ __forceinline__ void next(const DPass& a) {
+    if (++c == nchunk) {
+      c = 0;
+      ++g;
+      skip(a);
+    }
+  }
+  __device__ __forceinline__ const bf16* src() const { return W + (size_t)g * kPTR * K + (size_t)kPTR * c * kPKC; }
+  __device__ __forceinline__ uint32_t bytes() const { return (uint32_t)(kPTR * min(kPKC, K - c * kPKC) * 2); }
+};
+
 // xs[b] = bf16(RMSNorm(X[b]) * g) in A-fragment order; the mean square from
 // the producers' sums-of-squares partials (ssq_in[b][n_ssq], in index order).
+constexpr int kNormIt = 2;  // items (8 elements) per thread the norm prologue holds in registers
+
+// The gains a thread's first kNormIt prologue items use: constant, so they are
+// loaded before the grid barrier that precedes the prologue.
+template <int NB>
+__device__ __forceinline__ void load_gain(const bf16* gain, int K, uint4 (&pg)[kNormIt]) {
+  const int tid = threadIdx.x, n8 = K / 8;
+#pragma unroll
+  for (int j = 0; j < kNormIt; ++j) {
+    const int m = tid + j * kPC * 32;
+    pg[j] = make_uint4(0u, 0u, 0u, 0u);
+    if (m < NB * n8) pg[j] = *reinterpret_cast<const uint4*>(gain + (m - (m / n8) * n8) * 8);
+  }
+}
+
 template <int NB>
 __device__ void prologue_norm(const DPass& a, const float* ssq_in, int n_ssq, const bf16* gain, int K, bf16* xs,
-                              float (*red)[32], float* rr) {
+                              float (*red)[32], float* rr, const uint4 (&pg)[kNormIt]) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // the rows are loaded with the sums of squares, so that the prologue waits
+  // on one round trip to L2 (up to kNormIt items per thread)
+  constexpr int kIt = kNormIt;
+  const int n8 = K / 8, items = NB * n8;
+  const bool held = items <= kIt * kPC * 32;
+  float4 px0[kIt], px1[kIt];
+  if (held) {
+#pragma unroll
+    for (int j = 0; j < kIt; ++j) {
+      const int m = tid + j * kPC * 32;
+      if (m < items) {
+        const int b = m / n8, k = (m - b * n8) * 8;
+        px0[j] = __ldcg(reinterpret_cast<const float4*>(a.X + (size_t)b * K + k));
+        px1[j] = __ldcg(reinterpret_cast<const float4*>(a.X + (size_t)b * K + k + 4));
+      }
+    }
+  }
   float sacc[NB];
 #pragma unroll
   for (int b = 0; b < NB; ++b) sacc[b] = 0.f;
@@ -116,7 +216,28 @@ __device__ void prologue_norm(const DPass& a, const float* ssq_in, int n_ssq, co
     rr[tid] = 1.0f / sqrtf(t / (float)K + a.eps);
   }
   consumers_sync();
-  const int n8 = K / 8;
+  if (held) {
+#pragma unroll
+    for (int j = 0; j < kIt; ++j) {
+      const int m = tid + j * kPC * 32;
+      if (m < items) {
+        const int b = m / n8, k = (m - b * n8) * 8;
+        float gf[8];
+        bf16x8(pg[j], gf);
+        const float r = rr[b];
+        const float xv[8] = {px0[j].x, px0[j].y, px0[j].z, px0[j].w, px1[j].x, px1[j].y, px1[j].z, px1[j].w};
+        uint32_t* row = reinterpret_cast<uint32_t*>(xs + (size_t)b * K);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const __nv_bfloat162 v =
+              __floats2bfloat162_rn((xv[2 * q] * r) * gf[2 * q], (xv[2 * q + 1] * r) * gf[2 * q + 1]);
+          row[afrag_pos(k + 2 * q) >> 1] = *reinterpret_cast<const uint32_t*>(&v);
+        }
+      }
+    }
+    consumers_sync();
+    return;
+  }
 #pragma unroll 2
   for (int m = tid; m < NB * n8; m += kPC * 32) {
     const int b = m / n8, k = (m - b * n8) * 8;
@@ -140,16 +261,32 @@ __device__ void prologue_norm(const DPass& a, const float* ssq_in, int n_ssq, co
 // xs[b] = src[b] (bf16 rows of width K) in A-fragment order.
 template <int NB>
 __device__ void prologue_copy(const bf16* src, int K, bf16* xs) {
-  const int tid = threadIdx.x, n8 = K / 8;
-#pragma unroll 2
-  for (int m = tid; m < NB * n8; m += kPC * 32) {
-    const int b = m / n8, k = (m - b * n8) * 8;
-    const uint4 v = __ldcg(reinterpret_cast<const uint4*>(src + (size_t)b * K + k));
-    uint32_t* row = reinterpret_cast<uint32_t*>(xs + (size_t)b * K);
-    row[afrag_pos(k) >> 1] = v.x;
-    row[afrag_pos(k + 2) >> 1] = v.y;
-    row[afrag_pos(k + 4) >> 1] = v.z;
-    row[afrag_pos(k + 6) >> 1] = v.w;
+  const int tid = threadIdx.x, n8 = K / 8, items = NB * n8;
+  // batches of kIt items per thread, every load of a batch issued before its
+  // first store (a 9-warp block has 168 registers per thread)
+  constexpr int kIt = 4;
+  for (int base = 0; base < items; base += kIt * kPC * 32) {
+    uint4 v[kIt];
+#pragma unroll
+    for (int j = 0; j < kIt; ++j) {
+      const int m = base + tid + j * kPC * 32;
+      if (m < items) {
+        const int b = m / n8, k = (m - b * n8) * 8;
+        v[j] = __ldcg(reinterpret_cast<const uint4*>(src + (size_t)b * K + k));
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kIt; ++j) {
+      const int m = base + tid + j * kPC * 32;
+      if (m < items) {
+        const int b = m / n8, k = (m - b * n8) * 8;
+        uint32_t* row = reinterpret_cast<uint32_t*>(xs + (size_t)b * K);
+        row[afrag_pos(k) >> 1] = v[j].x;
+        row[afrag_pos(k + 2) >> 1] = v[j].y;
+        row[afrag_pos(k + 4) >> 1] = v[j].z;
+        row[afrag_pos(k + 6) >> 1] = v[j].w;
+      }
+    }
   }
   consumers_sync();
 }
@@ -302,12 +439,45 @@ __device__ void write_ssq(const DPass& a, float ssq, float (*red)[32]) {
 // one range per head the CTA writes the output row; with several, it writes
 // its range's partial and the last range to finish combines the ranges in
 // order (no CTA waits for another).
+// The key range [k0, k1) of attention item `item` (sequence, head, range).
+__device__ __forceinline__ void item_keys(const DPass& a, int item, int& b, int& h, int& ch, int& k0, int& k1) {
+  const int nkeys = min(a.pos + 1, a.Tc), nch = a.attn_chunks;
+  const int bh = item / nch;
+  ch = item - bh * nch;
+  b = bh / a.n_heads;
+  h = bh - b * a.n_heads;
+  k0 = (int)(((long long)nkeys * ch) / nch);
+  k1 = (int)(((long long)nkeys * (ch + 1)) / nch);
+}
+
+// Staging of the first item's K and V rows for layer l into shared memory
+// (thread 0): the keys before pos were written by earlier passes, so their
+// rows can be on their way a layer ahead.  [*lo, *hi): the staged keys.
+__device__ __forceinline__ void stage_kv(const DPass& a, int NBxH, int l, bf16* kvK, bf16* kvV, uint64_t* bar,
+                                         int* lo, int* hi) {
+  *lo = *hi = 0;
+  if (a.kv_keys <= 0 || (int)blockIdx.x >= NBxH * a.attn_chunks) return;
+  int b, h, ch, k0, k1;
+  item_keys(a, blockIdx.x, b, h, ch, k0, k1);
+  const int kend = min(k1, min(a.pos, k0 + a.kv_keys));
+  if (kend <= k0) return;
+  const size_t off = (size_t)l * a.kv_layer + (size_t)b * a.kv_seq_stride + ((size_t)h * a.Tc + k0) * kPHD;
+  const uint32_t bytes = (uint32_t)(kend - k0) * kPHD * 2;
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // after the generic reads of the last layer
+  mbar_expect_tx(bar, 2 * bytes);
+  bulk_g2s(kvK, a.Kc + off, bytes, bar);
+  bulk_g2s(kvV, a.Vc + off, bytes, bar);
+  *lo = k0;
+  *hi = kend;
+}
+
 template <int NB>
 __device__ void attention(const DPass& a, int l, float* qs, float* wm, float* wl, float (*wacc)[kPHD],
-                          volatile int* s_last) {
+                          volatile int* s_last, const bf16* kvK, const bf16* kvV, int kv_lo, int kv_hi) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int hidden = a.hidden, nkeys = min(a.pos + 1, a.Tc), nch = a.attn_chunks;
   for (int item = blockIdx.x; item < NB * a.n_heads * nch; item += gridDim.x) {
+    if (item != (int)blockIdx.x) kv_lo = kv_hi = 0;  // only the first item is staged
     const int bh = item / nch, ch = item - bh * nch;
     const int b = bh / a.n_heads, h = bh - b * a.n_heads;
     const int k0 = (int)(((long long)nkeys * ch) / nch), k1 = (int)(((long long)nkeys * (ch + 1)) / nch);
@@ -320,10 +490,16 @@ __device__ void attention(const DPass& a, int l, float* qs, float* wm, float* wl
       const int jn = min(32, k1 - j0), j = j0 + lane;
       float s = -INFINITY;
       if (lane < jn) {
-        const uint4* kr = reinterpret_cast<const uint4*>(Kh + (size_t)j * kPHD);
         uint4 kv[kPHD / 8];
+        if (j >= kv_lo && j < kv_hi) {
+          const uint4* kr = reinterpret_cast<const uint4*>(kvK + (size_t)(j - kv_lo) * kPHD);
 #pragma unroll
-        for (int v = 0; v < kPHD / 8; ++v) kv[v] = __ldcg(kr + v);
+          for (int v = 0; v < kPHD / 8; ++v) kv[v] = kr[v];
+        } else {
+          const uint4* kr = reinterpret_cast<const uint4*>(Kh + (size_t)j * kPHD);
+#pragma unroll
+          for (int v = 0; v < kPHD / 8; ++v) kv[v] = __ldcg(kr + v);
+        }
         float dot = 0.f;
 #pragma unroll
         for (int v = 0; v < kPHD / 8; ++v) {
@@ -343,7 +519,10 @@ __device__ void attention(const DPass& a, int l, float* qs, float* wm, float* wl
 #pragma unroll 8
       for (int jj = 0; jj < jn; ++jj) {
         const float pj = __shfl_sync(0xffffffffu, pr, jj);
-        const uint2 vv = __ldcg(reinterpret_cast<const uint2*>(Vh + (size_t)(j0 + jj) * kPHD + lane * 4));
+        const int jr = j0 + jj;
+        const uint2 vv = (jr >= kv_lo && jr < kv_hi)
+                             ? *reinterpret_cast<const uint2*>(kvV + (size_t)(jr - kv_lo) * kPHD + lane * 4)
+                             : __ldcg(reinterpret_cast<const uint2*>(Vh + (size_t)jr * kPHD + lane * 4));
         acc[0] = fmaf(pj, __uint_as_float(vv.x << 16), acc[0]);
         acc[1] = fmaf(pj, __uint_as_float(vv.x & 0xFFFF0000u), acc[1]);
         acc[2] = fmaf(pj, __uint_as_float(vv.y << 16), acc[2]);
@@ -381,12 +560,16 @@ __device__ void attention(const DPass& a, int l, float* qs, float* wm, float* wl
         part[(size_t)ch * (kPHD + 2) + 1] = L;
       }
     }
-    __threadfence();
+    // the CTA barrier collects the partial's stores; thread 0's ticket
+    // releases them at GPU scope and acquires the other ranges' partials
     consumers_sync();
-    if (tid == 0) *s_last = atomicAdd(a.attn_cnt + bh, 1u) == (unsigned)(nch - 1);
+    if (tid == 0) {
+      unsigned t;
+      asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(t) : "l"(a.attn_cnt + bh) : "memory");
+      *s_last = t == (unsigned)(nch - 1);
+    }
     consumers_sync();
     if (*s_last) {
-      __threadfence();
       if (tid < kPHD) {
         float Mx = -INFINITY;
         for (int c = 0; c < nch; ++c) Mx = fmaxf(Mx, __ldcg(part + (size_t)c * (kPHD + 2)));
@@ -416,18 +599,24 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
   __shared__ float qs[kPHD], wm[kPC], wl[kPC];
   __shared__ float wacc[kPC][kPHD];
   __shared__ int abort_flag, ring_flag, last_flag;
+  __shared__ __align__(8) uint64_t kv_bar;  // the staged K/V rows of the layer in flight
+  __shared__ int kv_lo, kv_hi, kv_dead;
   uint8_t* dsm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int xs_bytes = ((NB * max(a.hidden, a.ffn) * 2 + 1023) / 1024) * 1024;
   bf16* xs = reinterpret_cast<bf16*>(dsm);
   Ring R{dsm + xs_bytes, full_bar, empty_bar, a.ns, 0, 0u};
+  bf16* kvK = reinterpret_cast<bf16*>(dsm + xs_bytes + (size_t)a.ns * kPStage);
+  bf16* kvV = kvK + (size_t)a.kv_keys * kPHD;
   if (threadIdx.x == 0) {
     for (int s = 0; s < a.ns; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], kPC);
     }
+    mbar_init(&kv_bar, 1);
     abort_flag = 0;
     ring_flag = 0;
+    kv_dead = 0;
     mbar_fence_init();
   }
   __syncthreads();
@@ -438,34 +627,32 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
     // ---- producer: every projection of every layer, in consumption order ----
     if (lane == 0) {
       uint32_t issued = 0;
-      bool dead = false;
-      for (int l = 0; l < a.L && !dead; ++l)
-        for (int j = 0; j < 4 && !dead; ++j) {
-          const Proj P = proj_of(a, l, j);
-          const int G = (P.n_pairs + kDecGroupPairs - 1) / kDecGroupPairs, nchunk = (P.K + kPKC - 1) / kPKC;
-          int g0, g1;
-          dgemv_group_range(G, gridDim.x, blockIdx.x, g0, g1);
-          for (int g = g0; g < g1 && !dead; ++g)
-            for (int c = 0; c < nchunk; ++c) {
-              const int kn = min(kPKC, P.K - c * kPKC);
-              if (!mbar_wait(&R.empty[R.stage], R.phase ^ 1u, kWaitLimit, ring_dead)) {
-                // the consumers stopped releasing stages: nothing more is issued
-                set_error(a.err, VLAC_ERR_TIMEOUT);
-                *ring_dead = 1;
-                dead = true;
-                break;
-              }
-              const uint32_t bytes = (uint32_t)(kPTR * kn * 2);
-              mbar_expect_tx(&R.full[R.stage], bytes);
-              bulk_g2s(R.stages + (size_t)R.stage * kPStage, P.W + (size_t)g * kPTR * P.K + (size_t)kPTR * c * kPKC,
-                       bytes, &R.full[R.stage]);
-              ++issued;
-              if (++R.stage == R.ns) {
-                R.stage = 0;
-                R.phase ^= 1u;
-              }
-            }
+      StageCursor cur(a, blockIdx.x, gridDim.x), ahead = cur;
+      for (int i = 0; i < a.pf_stages && !ahead.done; ++i) {
+        prefetch_l2(ahead.src(), ahead.bytes());
+        ahead.next(a);
+      }
+      while (!cur.done) {
+        if (!ahead.done) {
+          prefetch_l2(ahead.src(), ahead.bytes());
+          ahead.next(a);
         }
+        if (!mbar_wait(&R.empty[R.stage], R.phase ^ 1u, kWaitLimit, ring_dead)) {
+          // the consumers stopped releasing stages: nothing more is issued
+          set_error(a.err, VLAC_ERR_TIMEOUT);
+          *ring_dead = 1;
+          break;
+        }
+        const uint32_t bytes = cur.bytes();
+        mbar_expect_tx(&R.full[R.stage], bytes);
+        bulk_g2s(R.stages + (size_t)R.stage * kPStage, cur.src(), bytes, &R.full[R.stage]);
+        ++issued;
+        if (++R.stage == R.ns) {
+          R.stage = 0;
+          R.phase ^= 1u;
+        }
+        cur.next(a);
+      }
       // no bulk copy may still be landing in this CTA's shared memory when it
       // exits; on the normal path the consumers waited for every one already
       ring_drain(R.full, R.ns, R.stage, R.phase, issued);
@@ -475,10 +662,15 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
 
   // ---- consumers ----
   unsigned epoch = 0;
+  if (threadIdx.x == 0) stage_kv(a, NB * a.n_heads, 0, kvK, kvV, &kv_bar, &kv_lo, &kv_hi);
+  int kv_issued = -1;  // the last layer whose staging copy was issued (thread 0's view is what counts)
+  if (threadIdx.x == 0 && kv_hi > kv_lo) kv_issued = 0;
   for (int l = 0; l < a.L; ++l) {
     int g0, g1;
     // q/k/v: RMSNorm of the residual rows (sums of squares from the decode
     // embedding for layer 0, else from the previous down-projection)
+    uint4 pga[kNormIt];
+    load_gain<NB>(a.g_attn[l], a.hidden, pga);  // constant: before the barrier
     if (l > 0) grid_sync(a, ++epoch, abort);
     if (threadIdx.x == 0) {
       // this CTA's attention items: their older K/V rows (written by earlier
@@ -495,12 +687,41 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
     }
     {
       const Proj P = proj_of(a, l, 0);
-      prologue_norm<NB>(a, l == 0 ? a.ssq0 : a.ssq, l == 0 ? a.n_ssq0 : (int)gridDim.x, a.g_attn[l], P.K, xs, red, rr);
+      prologue_norm<NB>(a, l == 0 ? a.ssq0 : a.ssq, l == 0 ? a.n_ssq0 : (int)gridDim.x, a.g_attn[l], P.K, xs, red, rr,
+                        pga);
       dgemv_group_range((P.n_pairs + kDecGroupPairs - 1) / kDecGroupPairs, gridDim.x, blockIdx.x, g0, g1);
       consume<NB, 0>(a, l, P, g0, g1, xs, R, pacc, ring_dead);
     }
     grid_sync(a, ++epoch, abort);
-    attention<NB>(a, l, qs, wm, wl, wacc, &last_flag);
+    {
+      // the staged rows of this layer (the CTA barrier inside the attention
+      // phase orders thread 0's flags before the other threads' reads)
+      int lo = 0, hi = 0;
+      if (threadIdx.x == 0 && kv_hi > kv_lo && !kv_dead) {
+        if (mbar_wait(&kv_bar, (uint32_t)l & 1u, kWaitLimit, ring_dead)) {
+          lo = kv_lo;
+          hi = kv_hi;
+        } else {
+          set_error(a.err, VLAC_ERR_TIMEOUT);
+          kv_dead = 1;  // read from global from now on; the copy is waited for at exit
+        }
+      }
+      if (threadIdx.x == 0) {
+        kv_lo = lo;
+        kv_hi = hi;
+      }
+      consumers_sync();
+      lo = kv_lo;
+      hi = kv_hi;
+      // every reader observes the copy's completion itself (it completed: no wait)
+      if (threadIdx.x != 0 && hi > lo) mbar_wait(&kv_bar, (uint32_t)l & 1u, kWaitLimit, ring_dead);
+      attention<NB>(a, l, qs, wm, wl, wacc, &last_flag, kvK, kvV, lo, hi);
+      // attention ended with a CTA barrier: the buffer is free for the next layer
+      if (threadIdx.x == 0 && !kv_dead && l + 1 < a.L) {
+        stage_kv(a, NB * a.n_heads, l + 1, kvK, kvV, &kv_bar, &kv_lo, &kv_hi);
+        if (kv_hi > kv_lo) kv_issued = l + 1;
+      }
+    }
     grid_sync(a, ++epoch, abort);
     {  // o-projection + residual
       const Proj P = proj_of(a, l, 1);
@@ -508,10 +729,12 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
       dgemv_group_range((P.n_pairs + kDecGroupPairs - 1) / kDecGroupPairs, gridDim.x, blockIdx.x, g0, g1);
       write_ssq<NB>(a, consume<NB, 1>(a, l, P, g0, g1, xs, R, pacc, ring_dead), red);
     }
+    uint4 pgf[kNormIt];
+    load_gain<NB>(a.g_ffn[l], a.hidden, pgf);
     grid_sync(a, ++epoch, abort);
     {  // gate/up with the MLP RMSNorm, SwiGLU
       const Proj P = proj_of(a, l, 2);
-      prologue_norm<NB>(a, a.ssq, (int)gridDim.x, a.g_ffn[l], P.K, xs, red, rr);
+      prologue_norm<NB>(a, a.ssq, (int)gridDim.x, a.g_ffn[l], P.K, xs, red, rr, pgf);
       dgemv_group_range((P.n_pairs + kDecGroupPairs - 1) / kDecGroupPairs, gridDim.x, blockIdx.x, g0, g1);
       consume<NB, 2>(a, l, P, g0, g1, xs, R, pacc, ring_dead);
     }
@@ -523,11 +746,18 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
       write_ssq<NB>(a, consume<NB, 3>(a, l, P, g0, g1, xs, R, pacc, ring_dead), red);
     }
   }
+  // a staging copy whose wait gave up may still be landing: wait for it
+  // (bounded, deaf to the give-up flags) before the CTA exits
+  if (threadIdx.x == 0 && kv_dead && kv_issued >= 0) {
+    int never = 0;
+    mbar_wait(&kv_bar, (uint32_t)kv_issued & 1u, kWaitLimit, &never);
+  }
 }
 
 template <int NB>
 int dpass_launch(const DPass& a, int n_sm, cudaStream_t st) {
-  const size_t smem = 1024 + ((size_t)NB * std::max(a.hidden, a.ffn) * 2 + 1023) / 1024 * 1024 + (size_t)a.ns * kPStage;
+  const size_t smem = 1024 + ((size_t)NB * std::max(a.hidden, a.ffn) * 2 + 1023) / 1024 * 1024 + (size_t)a.ns * kPStage +
+                      dpass_kv_bytes(a.kv_keys);
   static size_t smem_set = 0;
   if (smem > smem_set) {
     if (cudaFuncSetAttribute(dpass_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
@@ -555,6 +785,12 @@ int dpass_launch(const DPass& a, int n_sm, cudaStream_t st) {
 }
 
 }  // namespace
+
+size_t dpass_kv_bytes(int kv_keys) { return (size_t)2 * std::max(kv_keys, 0) * kPHD * 2; }
+size_t dpass_smem_bytes(int hidden, int ffn, int nb, int ns, int kv_keys) {
+  return 1024 + ((size_t)nb * std::max(hidden, ffn) * 2 + 1023) / 1024 * 1024 + (size_t)ns * kPStage +
+         dpass_kv_bytes(kv_keys);
+}
 
 bool dpass_supported(int hidden, int ffn, int n_heads, int head_dim, int nb, int ns) {
   return head_dim == kPHD && n_heads * head_dim == hidden && nb >= 1 && nb <= 2 && hidden % 64 == 0 && ffn % 64 == 0 &&

@@ -48,6 +48,9 @@ struct vlac_ctx {
   int n_sm = 1;
   int gemv_ns = 4;  // decode-GEMV weight ring stages (32 KB each)
   int gemv_pf_kb = 0;  // decode-GEMV L2 prefetch of the next projection, KB per CTA (measured: off is best)
+  int dpass_pf = 0;   // persistent pass: rolling L2 prefetch distance, ring stages (VLAC_DPASS_PF; measured: off is best)
+  int dpass_bar = 1;  // persistent pass: grid barrier kind (VLAC_DPASS_BAR: 1 release/acquire, 0 fences)
+  bool dpass_kv = true;  // persistent pass: attention K/V staged in shared memory (VLAC_DPASS_KV)
   bool use_dpass = false;  // decode passes as one persistent cooperative launch (k_dpass.cu) where supported
   int dpass_attn_chunks = 0;  // its key ranges per (sequence, head); 0 = chosen from the SM count
   void** dp_ptrs = nullptr;  // device: per-layer pointers [w_qkv | w_o | w_gu | w_d | g_attn | g_ffn][L]
@@ -268,6 +271,9 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (const char* e = std::getenv("VLAC_GEMV_NS")) c->gemv_ns = std::max(2, std::min(24, std::atoi(e)));
   if (const char* e = std::getenv("VLAC_GEMV_PF_KB")) c->gemv_pf_kb = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("VLAC_DPASS")) c->use_dpass = std::atoi(e) != 0;
+  if (const char* e = std::getenv("VLAC_DPASS_PF")) c->dpass_pf = std::max(0, std::min(64, std::atoi(e)));
+  if (const char* e = std::getenv("VLAC_DPASS_BAR")) c->dpass_bar = std::atoi(e) != 0 ? 1 : 0;
+  if (const char* e = std::getenv("VLAC_DPASS_KV")) c->dpass_kv = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_DPASS_ATTN_CHUNKS")) c->dpass_attn_chunks = std::max(0, std::atoi(e));
   c->d = *dims;
   const vlac_dims& d = c->d;
@@ -970,6 +976,8 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
           p.ssq = c->ssq_a;
           p.bar = c->dp_bar;
           p.err = c->err;
+          p.pf_stages = c->dpass_pf;
+          p.bar_mode = c->dpass_bar;
           {
             // key ranges per (sequence, head): enough items for the SMs, at
             // most one per 32 keys (the partial buffer's capacity) and 8
@@ -977,6 +985,14 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
             int chunks = std::max(1, std::min(cap, c->n_sm / std::max(1, B * nh)));
             if (c->dpass_attn_chunks > 0) chunks = std::min(cap, c->dpass_attn_chunks);
             p.attn_chunks = chunks;
+            // the first item's K/V rows staged in shared memory, as many as
+            // fit next to the ring (220 KB of dynamic shared memory)
+            p.kv_keys = 0;
+            if (c->dpass_kv) {
+              const size_t base = dpass_smem_bytes((int)Hd, (int)F, B, c->gemv_ns, 0), cap = 220 * 1024;
+              const int fit = base < cap ? (int)((cap - base) / dpass_kv_bytes(1)) : 0;
+              p.kv_keys = std::min((c->Tc + chunks - 1) / chunks, fit);
+            }
             p.part_stride = (size_t)((c->Tc + 31) / 32) * (hd + 2);
             p.attn_part = c->attn_part;
             p.attn_cnt = c->attn_cnt;

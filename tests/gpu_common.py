@@ -71,6 +71,12 @@ SMALL = {
     "small_wide": synth.Dims(n_layers=2, hidden=256, n_heads=2, head_dim=128, ffn=4160, vocab=1024, n_bins=256,
                              img_h=112, img_w=112, patch=14, n_views=1, n_text=8, proprio_dim=0, n_action=7,
                              parallel=0, dtype="bf16", max_batch=2),
+    # bf16, hidden 2304 (18 x 128 heads), MLP width 4608: every decode GEMV's K
+    # spans two or three 2048-element chunks (the last one partial), and the
+    # decode projections have more row groups than a GB300 has SMs
+    "wide": synth.Dims(n_layers=2, hidden=2304, n_heads=18, head_dim=128, ffn=4608, vocab=1024, n_bins=256,
+                       img_h=112, img_w=112, patch=14, n_views=1, n_text=8, proprio_dim=0, n_action=7,
+                       parallel=0, dtype="bf16", max_batch=2),
     # fp32 tiny model (SIMT path)
     "tiny": synth.dims_for("tiny"),
 }

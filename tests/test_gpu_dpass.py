@@ -24,7 +24,7 @@ def dpass_on():
 
 
 @pytest.mark.parametrize("chunks", ["auto", "1", "3"])
-@pytest.mark.parametrize("name,batch", [("small", 1), ("small_wide", 1), ("small_wide", 2)])
+@pytest.mark.parametrize("name,batch", [("small", 1), ("small_wide", 1), ("small_wide", 2), ("wide", 1), ("wide", 2)])
 def test_dpass_parity(name, batch, chunks, dpass_on, cuda_device, monkeypatch):
     """chunks: key ranges per (sequence, head) in the attention phase (1: one
     CTA per head; otherwise the ranges' partials are combined by the last)."""
