@@ -46,6 +46,10 @@ CPU_LAYERS = 2  # the CPU oracle sample runs this many of the 32 layers
 # Reported only while the kernel is the one the counters were taken on.
 DGEMV_TRAFFIC_PER_LAUNCH: dict = {c: 102.06e6 for c in ("openvla7b", "layer7b")}
 DGEMV_TRAFFIC_NOTE = "ncu capture only for the 7B-shaped decode layer"
+# The same counters for one persistent decode pass (dpass_kernel), per decoder
+# layer it streams (profiles/dpass_layer7b_decode.txt): a launch of the
+# one-layer 7B model; a launch over L layers moves L times as much.
+DPASS_TRAFFIC_PER_LAYER: dict = {}
 
 
 def peaks():
@@ -476,7 +480,18 @@ def main():
     gemv_gbs = g_bytes / (g_ms / 1e3) / 1e9 if g_ms > 0 else None
     gemm_gbs = p_bytes / (p_ms / 1e3) / 1e9 if p_ms > 0 else None
     gemm_tfs = gemm_flops / (p_ms / 1e3) / 1e12 if p_ms > 0 else None
-    if g_n:
+    # one launch per decode token: the persistent decode pass ran (bf16,
+    # head_dim 128, one or two sequences); else one per projection
+    persistent = 0 < g_n <= K * max(1, d.n_action - 1)
+    if g_n and persistent:
+        # the persistent pass (weights of every layer + attention) dominates
+        per_layer = DPASS_TRAFFIC_PER_LAYER.get("7b") if d.hidden == 4096 and d.ffn == 11008 else None
+        roof = {"bound": "hbm", "achieved": gemv_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": gemv_gbs / pk["hbm_gbs"], "traffic": None if per_layer is None else per_layer * d.n_layers,
+                "kernel": "dpass_kernel (persistent decode pass: every layer's weight stream and attention)",
+                "launches": g_n, "avg_launch_us": 1e3 * g_ms / g_n, "peak_source": f"{src} hbm_gbs",
+                **({} if per_layer is not None else {"traffic_note": "no ncu capture of this kernel at this shape"})}
+    elif g_n:
         # weight streaming of the decode passes dominates the step
         roof = {"bound": "hbm", "achieved": gemv_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
                 "frac": gemv_gbs / pk["hbm_gbs"], "traffic": DGEMV_TRAFFIC_PER_LAUNCH.get(args.config),
@@ -547,7 +562,9 @@ def main():
         "device_ms_per_step_by_kind": {k: round(v, 4) for k, v in breakdown.items()},
         "by_kind_note": (f"per-launch CUDA events in a second, non-graph pass of the same K steps serialise the "
                          f"launches: the kinds sum to {sum(breakdown.values()):.2f} ms per step against "
-                         f"{ms / K:.2f} ms of graph replay in the timed pass"),
+                         f"{ms / K:.2f} ms of graph replay in the timed pass"
+                         + ("; decode_gemv is the persistent decode pass, which also runs the decode attention"
+                            if persistent else "")),
         "clocks": clocks,
         "e2e": {"value": e2e, "unit": "steps/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "note": "frames + prompt (+ proprio) H2D from pinned memory, action ids/margins/flags D2H, "

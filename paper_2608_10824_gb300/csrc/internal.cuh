@@ -464,10 +464,6 @@ struct DPass {
   size_t part_stride;
   float* attn_part;
   unsigned* attn_cnt;
-  // rolling L2 prefetch: the producer pulls the stage this many ring stages
-  // beyond the one it is issuing into L2 (0: off), so that HBM keeps
-  // streaming while the consumers wait at a grid barrier with the ring full
-  int pf_stages;
   // grid barrier: 0 fence + atomic add + poll; 1 release add + acquire poll
   int bar_mode;
   // attention: up to kv_keys keys of the CTA's first item staged in shared

@@ -627,16 +627,8 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
     // ---- producer: every projection of every layer, in consumption order ----
     if (lane == 0) {
       uint32_t issued = 0;
-      StageCursor cur(a, blockIdx.x, gridDim.x), ahead = cur;
-      for (int i = 0; i < a.pf_stages && !ahead.done; ++i) {
-        prefetch_l2(ahead.src(), ahead.bytes());
-        ahead.next(a);
-      }
+      StageCursor cur(a, blockIdx.x, gridDim.x);
       while (!cur.done) {
-        if (!ahead.done) {
-          prefetch_l2(ahead.src(), ahead.bytes());
-          ahead.next(a);
-        }
         if (!mbar_wait(&R.empty[R.stage], R.phase ^ 1u, kWaitLimit, ring_dead)) {
           // the consumers stopped releasing stages: nothing more is issued
           set_error(a.err, VLAC_ERR_TIMEOUT);

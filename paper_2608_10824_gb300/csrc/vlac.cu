@@ -48,10 +48,9 @@ struct vlac_ctx {
   int n_sm = 1;
   int gemv_ns = 4;  // decode-GEMV weight ring stages (32 KB each)
   int gemv_pf_kb = 0;  // decode-GEMV L2 prefetch of the next projection, KB per CTA (measured: off is best)
-  int dpass_pf = 0;   // persistent pass: rolling L2 prefetch distance, ring stages (VLAC_DPASS_PF; measured: off is best)
   int dpass_bar = 1;  // persistent pass: grid barrier kind (VLAC_DPASS_BAR: 1 release/acquire, 0 fences)
   bool dpass_kv = true;  // persistent pass: attention K/V staged in shared memory (VLAC_DPASS_KV)
-  bool use_dpass = false;  // decode passes as one persistent cooperative launch (k_dpass.cu) where supported
+  bool use_dpass = true;  // decode passes as one persistent cooperative launch (k_dpass.cu) where supported
   int dpass_attn_chunks = 0;  // its key ranges per (sequence, head); 0 = chosen from the SM count
   void** dp_ptrs = nullptr;  // device: per-layer pointers [w_qkv | w_o | w_gu | w_d | g_attn | g_ffn][L]
   unsigned* dp_bar = nullptr;  // device: the persistent pass's grid-barrier counter
@@ -271,7 +270,6 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (const char* e = std::getenv("VLAC_GEMV_NS")) c->gemv_ns = std::max(2, std::min(24, std::atoi(e)));
   if (const char* e = std::getenv("VLAC_GEMV_PF_KB")) c->gemv_pf_kb = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("VLAC_DPASS")) c->use_dpass = std::atoi(e) != 0;
-  if (const char* e = std::getenv("VLAC_DPASS_PF")) c->dpass_pf = std::max(0, std::min(64, std::atoi(e)));
   if (const char* e = std::getenv("VLAC_DPASS_BAR")) c->dpass_bar = std::atoi(e) != 0 ? 1 : 0;
   if (const char* e = std::getenv("VLAC_DPASS_KV")) c->dpass_kv = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_DPASS_ATTN_CHUNKS")) c->dpass_attn_chunks = std::max(0, std::atoi(e));
@@ -976,7 +974,6 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
           p.ssq = c->ssq_a;
           p.bar = c->dp_bar;
           p.err = c->err;
-          p.pf_stages = c->dpass_pf;
           p.bar_mode = c->dpass_bar;
           {
             // key ranges per (sequence, head): enough items for the SMs, at
