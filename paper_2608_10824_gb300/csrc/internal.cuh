@@ -472,6 +472,7 @@ struct DPass {
 };
 size_t dpass_kv_bytes(int kv_keys);
 size_t dpass_smem_bytes(int hidden, int ffn, int nb, int ns, int kv_keys);
+int dpass_kv_fit(int hidden, int ffn, int nb, int ns);  // K/V rows the staging buffer can hold on this device
 bool dpass_supported(int hidden, int ffn, int n_heads, int head_dim, int nb, int ns);
 int launch_dpass(const DPass& a, int nb, int n_sm, cudaStream_t st);
 // Decode-streaming copy of a projection (W: [rows][K]); see k_decode.cu for the layout.

@@ -486,8 +486,10 @@ __device__ void attention(const DPass& a, int l, float* qs, float* wm, float* wl
     if (tid < kPHD) qs[tid] = __bfloat162float(__ldcg(a.Q + (size_t)b * hidden + (size_t)h * kPHD + tid));
     consumers_sync();
     float m_run = -INFINITY, l_run = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
-    for (int j0 = k0 + warp * 32; j0 < k1; j0 += kPC * 32) {
-      const int jn = min(32, k1 - j0), j = j0 + lane;
+    // the range's keys cut evenly over the eight warps (a key per lane)
+    const int kw = (k1 - k0 + kPC - 1) / kPC, w0 = k0 + warp * kw, w1 = min(k1, w0 + kw);
+    for (int j0 = w0; j0 < w1; j0 += 32) {
+      const int jn = min(32, w1 - j0), j = j0 + lane;
       float s = -INFINITY;
       if (lane < jn) {
         uint4 kv[kPHD / 8];
@@ -500,15 +502,17 @@ __device__ void attention(const DPass& a, int l, float* qs, float* wm, float* wl
 #pragma unroll
           for (int v = 0; v < kPHD / 8; ++v) kv[v] = __ldcg(kr + v);
         }
-        float dot = 0.f;
+        // four partial sums over the head dimension (element i mod 4),
+        // added in a fixed order
+        float dp[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int v = 0; v < kPHD / 8; ++v) {
           float f[8];
           bf16x8(kv[v], f);
 #pragma unroll
-          for (int i = 0; i < 8; ++i) dot = fmaf(f[i], qs[v * 8 + i], dot);
+          for (int i = 0; i < 8; ++i) dp[i & 3] = fmaf(f[i], qs[v * 8 + i], dp[i & 3]);
         }
-        s = dot * a.scale;
+        s = ((dp[0] + dp[1]) + (dp[2] + dp[3])) * a.scale;
       }
       const float m_new = fmaxf(m_run, p_allmax(s));
       const float corr = m_run == -INFINITY ? 0.f : expf(m_run - m_new);
@@ -753,7 +757,7 @@ int dpass_launch(const DPass& a, int n_sm, cudaStream_t st) {
   static size_t smem_set = 0;
   if (smem > smem_set) {
     if (cudaFuncSetAttribute(dpass_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
-      return VLAC_ERR_CUDA;
+      return VLAC_ERR_UNSUPPORTED;  // more than a block may have: the per-projection chain runs instead
     smem_set = smem;
   }
   int per_sm = 0;
@@ -782,6 +786,19 @@ size_t dpass_kv_bytes(int kv_keys) { return (size_t)2 * std::max(kv_keys, 0) * k
 size_t dpass_smem_bytes(int hidden, int ffn, int nb, int ns, int kv_keys) {
   return 1024 + ((size_t)nb * std::max(hidden, ffn) * 2 + 1023) / 1024 * 1024 + (size_t)ns * kPStage +
          dpass_kv_bytes(kv_keys);
+}
+
+int dpass_kv_fit(int hidden, int ffn, int nb, int ns) {
+  // what the device lets one block have, less the kernel's static shared
+  // memory and the dynamic part without staging
+  int dev = 0, optin = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+    return 0;
+  cudaFuncAttributes fa{};
+  if (cudaFuncGetAttributes(&fa, nb == 1 ? dpass_kernel<1> : dpass_kernel<2>) != cudaSuccess) return 0;
+  const long long room = (long long)optin - (long long)fa.sharedSizeBytes - (long long)dpass_smem_bytes(hidden, ffn, nb, ns, 0);
+  return room > 0 ? (int)(room / (long long)dpass_kv_bytes(1)) : 0;
 }
 
 bool dpass_supported(int hidden, int ffn, int n_heads, int head_dim, int nb, int ns) {

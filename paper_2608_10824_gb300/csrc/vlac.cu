@@ -983,13 +983,10 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
             if (c->dpass_attn_chunks > 0) chunks = std::min(cap, c->dpass_attn_chunks);
             p.attn_chunks = chunks;
             // the first item's K/V rows staged in shared memory, as many as
-            // fit next to the ring (220 KB of dynamic shared memory)
+            // fit next to the ring
             p.kv_keys = 0;
-            if (c->dpass_kv) {
-              const size_t base = dpass_smem_bytes((int)Hd, (int)F, B, c->gemv_ns, 0), cap = 220 * 1024;
-              const int fit = base < cap ? (int)((cap - base) / dpass_kv_bytes(1)) : 0;
-              p.kv_keys = std::min((c->Tc + chunks - 1) / chunks, fit);
-            }
+            if (c->dpass_kv)
+              p.kv_keys = std::min((c->Tc + chunks - 1) / chunks, dpass_kv_fit((int)Hd, (int)F, B, c->gemv_ns));
             p.part_stride = (size_t)((c->Tc + 31) / 32) * (hd + 2);
             p.attn_part = c->attn_part;
             p.attn_cnt = c->attn_cnt;
