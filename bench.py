@@ -47,9 +47,9 @@ CPU_LAYERS = 2  # the CPU oracle sample runs this many of the 32 layers
 DGEMV_TRAFFIC_PER_LAUNCH: dict = {c: 102.06e6 for c in ("openvla7b", "layer7b")}
 DGEMV_TRAFFIC_NOTE = "ncu capture only for the 7B-shaped decode layer"
 # The same counters for one persistent decode pass (dpass_kernel), per decoder
-# layer it streams (profiles/dpass_layer7b_decode.txt): a launch of the
+# layer it streams (profiles/dpass_openvla7b_decode.md): a launch of the
 # one-layer 7B model; a launch over L layers moves L times as much.
-DPASS_TRAFFIC_PER_LAYER: dict = {}
+DPASS_TRAFFIC_PER_LAYER: dict = {"7b": 409.77e6}
 
 
 def peaks():
