@@ -469,6 +469,7 @@ struct DPass {
   // attention: up to kv_keys keys of the CTA's first item staged in shared
   // memory a layer ahead (0: read from global)
   int kv_keys;
+  uint32_t wait_limit;  // polls of a ring, staging or grid-barrier wait before it gives up (drains keep kWaitLimit)
 };
 size_t dpass_kv_bytes(int kv_keys);
 size_t dpass_smem_bytes(int hidden, int ffn, int nb, int ns, int kv_keys);

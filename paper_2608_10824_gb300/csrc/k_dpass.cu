@@ -86,7 +86,7 @@ __device__ __forceinline__ void grid_sync(const DPass& a, unsigned epoch, volati
           unsigned v;
           asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(a.bar) : "memory");
           if (v >= target) break;
-          if (++it > kWaitLimit) {
+          if (++it > a.wait_limit) {
             set_error(a.err, VLAC_ERR_TIMEOUT);
             *abort = 1;
             break;
@@ -99,7 +99,7 @@ __device__ __forceinline__ void grid_sync(const DPass& a, unsigned epoch, volati
       atomicAdd(a.bar, 1u);
       if (!*abort) {
         while (*reinterpret_cast<volatile unsigned*>(a.bar) < target) {
-          if (++it > kWaitLimit) {
+          if (++it > a.wait_limit) {
             set_error(a.err, VLAC_ERR_TIMEOUT);
             *abort = 1;
             break;
@@ -339,7 +339,7 @@ __device__ float consume(const DPass& a, int l, const Proj& P, int g0, int g1, c
       // back only after its copy landed; once one ring wait times out the
       // ring is dead and the others return at once
       bool ok = true;
-      if (lane == 0) ok = mbar_wait(&R.full[R.stage], R.phase, kWaitLimit, ring_dead);
+      if (lane == 0) ok = mbar_wait(&R.full[R.stage], R.phase, a.wait_limit, ring_dead);
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (ok) {
         const uint32_t st = st_lane + (uint32_t)((size_t)R.stage * kPStage);
@@ -633,7 +633,7 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
       uint32_t issued = 0;
       StageCursor cur(a, blockIdx.x, gridDim.x);
       while (!cur.done) {
-        if (!mbar_wait(&R.empty[R.stage], R.phase ^ 1u, kWaitLimit, ring_dead)) {
+        if (!mbar_wait(&R.empty[R.stage], R.phase ^ 1u, a.wait_limit, ring_dead)) {
           // the consumers stopped releasing stages: nothing more is issued
           set_error(a.err, VLAC_ERR_TIMEOUT);
           *ring_dead = 1;
@@ -694,7 +694,7 @@ __global__ void __launch_bounds__((kPC + 1) * 32, 1) dpass_kernel(const __grid_c
       // phase orders thread 0's flags before the other threads' reads)
       int lo = 0, hi = 0;
       if (threadIdx.x == 0 && kv_hi > kv_lo && !kv_dead) {
-        if (mbar_wait(&kv_bar, (uint32_t)l & 1u, kWaitLimit, ring_dead)) {
+        if (mbar_wait(&kv_bar, (uint32_t)l & 1u, a.wait_limit, ring_dead)) {
           lo = kv_lo;
           hi = kv_hi;
         } else {

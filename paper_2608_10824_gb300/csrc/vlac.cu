@@ -975,6 +975,7 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
           p.bar = c->dp_bar;
           p.err = c->err;
           p.bar_mode = c->dpass_bar;
+          p.wait_limit = c->wait_limit;
           {
             // key ranges per (sequence, head): enough items for the SMs, at
             // most one per 32 keys (the partial buffer's capacity) and 8

@@ -76,16 +76,19 @@ def test_unsupported_dims():
     assert e.value.code in (-7, -1)
 
 
+@pytest.mark.parametrize("path", ["dpass", "chain"])
 @pytest.mark.parametrize("polls", [0, 1])
-def test_step_kernels_give_up_and_the_context_stays_usable(cuda_device, polls):
-    """The prefix GEMM's, the decode GEMV's and the prefix attention's bounded
-    waits, run out on purpose (0 polls: every wait gives up at once; 1 poll:
-    wherever a copy has not landed by the first poll): the step latches
-    VLAC_ERR_TIMEOUT (or, with 1 poll, may happen to finish), nothing hangs
-    or faults, and a normal step on a new cache of the same context then
-    matches the oracle."""
+def test_step_kernels_give_up_and_the_context_stays_usable(cuda_device, monkeypatch, polls, path):
+    """The prefix GEMM's, the prefix attention's and the decode path's bounded
+    waits (the persistent pass's ring, K/V staging and grid-barrier waits, or
+    the chain's GEMV ring waits), run out on purpose (0 polls: every wait
+    gives up at once; 1 poll: wherever a copy has not landed by the first
+    poll): the step latches VLAC_ERR_TIMEOUT (or, with 1 poll, may happen to
+    finish), nothing hangs or faults, and a normal step on a new cache of the
+    same context then matches the oracle."""
     from paper_2608_10824_gb300.vlac import ERRORS
     from tests.gpu_common import Lockstep
+    monkeypatch.setenv("VLAC_DPASS", "1" if path == "dpass" else "0")
     d = SMALL["small"]
     w = synth.make_weights(d, seed=5)
     ls = Lockstep(d, w)
