@@ -49,7 +49,7 @@ DGEMV_TRAFFIC_NOTE = "ncu capture only for the 7B-shaped decode layer"
 # The same counters for one persistent decode pass (dpass_kernel), per decoder
 # layer it streams (profiles/dpass_openvla7b_decode.md): a launch of the
 # one-layer 7B model; a launch over L layers moves L times as much.
-DPASS_TRAFFIC_PER_LAYER: dict = {"7b": 409.77e6}
+DPASS_TRAFFIC_PER_LAYER: dict = {"7b": 409.85e6}
 
 
 def peaks():
