@@ -12,16 +12,19 @@
 // ring keeps filling.
 //
 // Per layer: q/k/v (RMSNorm prologue, RoPE, Q and the K/V rows at pos) |
-// barrier | attention, one (sequence, head) per CTA | barrier | o-projection
-// + residual | barrier | gate/up (RMSNorm prologue, SwiGLU) | barrier |
-// down + residual | barrier (before the next layer).
+// barrier | attention, one (sequence, head, key range) per CTA, the CTA's
+// older K/V rows staged in shared memory during the layer before | barrier |
+// o-projection + residual | barrier | gate/up (RMSNorm prologue, SwiGLU) |
+// barrier | down + residual | barrier (before the next layer).
 //
 // Data one CTA writes and another reads inside the launch (Q, the K/V rows at
-// pos, the attention output, the residual rows, the SwiGLU output, the sums
-// of squares) is published by the barrier (fence, atomic arrive; acquire,
-// fence) and read through L2 (ld.global.cg).  Every wait is bounded; a CTA
-// that gives up latches VLAC_ERR_TIMEOUT, stops waiting and still arrives at
-// every later barrier, so the others finish.
+// pos, the attention output and partials, the residual rows, the SwiGLU
+// output, the sums of squares) is published by the barrier (a release add at
+// GPU scope after a CTA barrier; an acquire poll, then a CTA barrier) and
+// read through L2 (ld.global.cg).  Every wait is bounded (the context's wait
+// limit; drains before exit keep a fixed one); a CTA that gives up latches
+// VLAC_ERR_TIMEOUT, stops waiting and still arrives at every later barrier,
+// so the others finish.
 #include <algorithm>
 
 #include "internal.cuh"
@@ -434,11 +437,11 @@ __device__ void write_ssq(const DPass& a, float ssq, float (*red)[32]) {
 }
 
 // Single-query attention of layer l: items (sequence, head, key range) spread
-// over the CTAs.  Warp w takes keys k0 + w*32 + 256t + lane of the item's range
-// (online softmax per warp) and the eight warps are combined in order.  With
-// one range per head the CTA writes the output row; with several, it writes
-// its range's partial and the last range to finish combines the ranges in
-// order (no CTA waits for another).
+// over the CTAs.  The item's keys are cut evenly over the eight warps, a key
+// per lane (online softmax per warp), and the eight warps are combined in
+// order.  With one range per head the CTA writes the output row; with
+// several, it writes its range's partial and the last range to finish
+// combines the ranges in order (no CTA waits for another).
 // The key range [k0, k1) of attention item `item` (sequence, head, range).
 __device__ __forceinline__ void item_keys(const DPass& a, int item, int& b, int& h, int& ch, int& k0, int& k1) {
   const int nkeys = min(a.pos + 1, a.Tc), nch = a.attn_chunks;
