@@ -326,6 +326,12 @@ void launch_residual_norm(Rows rows, int B, int S, int hidden, const float* part
 template <typename T>
 void launch_swiglu(Rows rows, int B, int S, int ffn, const float* part, const SplitPlan& sp, T* G, cudaStream_t st);
 void launch_residual(Rows rows, int B, int S, int hidden, const float* part, const SplitPlan& sp, cudaStream_t st);
+// residual_kernel of layer l and layer_in_kernel of layer l+1 in one launch
+// (rows: layer l+1's; off_prev: layer l's offsets; H: layer l+1's H slice)
+template <typename T>
+void launch_residual_layer_in(Rows rows, const int* off_prev, int B, int S, int hidden, const float* part,
+                              const SplitPlan& sp, float* H, size_t h_seq_stride, const T* gain, float eps, T* A,
+                              cudaStream_t st);
 // TMA maps of a cache's K and V (bf16 caches): 3-D {head_dim, Tc, batch x
 // layers x heads}, boxes of 64 dimensions x 64 positions, 128-byte swizzle,
 // positions past Tc read as zeros.  The box of (sequence b, layer l, head h)

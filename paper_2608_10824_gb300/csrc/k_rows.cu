@@ -173,6 +173,51 @@ __global__ void layer_in_kernel(Rows rows, const int* __restrict__ off_prev, int
   rmsnorm_row<T>(x, ss, gain, hidden, eps, A + (size_t)(rows.off[b] + i) * hidden, red);
 }
 
+// The down-projection residual of layer l fused with layer l+1's input: rows
+// computed at layer l add their down-projection (summed over splits), and
+// the sum is their layer-(l+1) input, recorded in the H cache; rows that join
+// at layer l+1 start from H; every row of layer l+1 is normalised into A.
+// The same arithmetic, element for element, as residual_kernel followed by
+// layer_in_kernel.  rows: layer l+1's; off_prev: layer l's row offsets.
+template <typename T>
+__global__ void residual_layer_in_kernel(Rows rows, const int* __restrict__ off_prev, int hidden,
+                                         const float* __restrict__ part, SplitPlan sp, float* __restrict__ H,
+                                         size_t h_seq_stride, const T* __restrict__ gain, float eps,
+                                         T* __restrict__ A) {
+  pdl_wait();
+  pdl_trigger();
+  __shared__ float red[32];
+  const int b = blockIdx.y, i = blockIdx.x;
+  const int cnt = rows.off[b + 1] - rows.off[b];
+  const int cnt_prev = off_prev[b + 1] - off_prev[b];
+  if (i >= cnt && i >= cnt_prev) return;
+  const int pos = rows.idx[(size_t)b * rows.idx_stride + i];
+  float* x = rows.X + ((size_t)b * rows.idx_stride + i) * hidden;
+  float4* x4 = reinterpret_cast<float4*>(x);
+  float4* h4 = reinterpret_cast<float4*>(H + (size_t)b * h_seq_stride + (size_t)pos * hidden);
+  float ss = 0.f;
+  if (i < cnt_prev) {
+    const int r = off_prev[b] + i;
+    const float* pr = part + (size_t)r * hidden;
+#pragma unroll 4
+    for (int k = threadIdx.x; k < hidden / 4; k += blockDim.x) {
+      const float4 v = add4(x4[k], sum_splits4(pr, sp, r, 4 * (size_t)k));
+      x4[k] = v;
+      h4[k] = v;
+      ss = sq4(v, ss);
+    }
+  } else {
+#pragma unroll 4
+    for (int k = threadIdx.x; k < hidden / 4; k += blockDim.x) {
+      const float4 v = h4[k];
+      x4[k] = v;
+      ss = sq4(v, ss);
+    }
+  }
+  if (i >= cnt) return;
+  rmsnorm_row<T>(x, ss, gain, hidden, eps, A + (size_t)(rows.off[b] + i) * hidden, red);
+}
+
 // ---- GEMM epilogues ------------------------------------------------------------
 
 // q, k, v from the fused projection [q | k | v]; RoPE (rotate-half) on q and k
@@ -459,6 +504,13 @@ void launch_layer_in(Rows rows, const int* off_prev, int B, int S, int hidden, f
   launch_k(layer_in_kernel<T>, dim3(S, B), dim3(kNormThreads), 0, st, rows, off_prev, hidden, H, h_seq_stride, gain, eps, A);
 }
 template <typename T>
+void launch_residual_layer_in(Rows rows, const int* off_prev, int B, int S, int hidden, const float* part,
+                              const SplitPlan& sp, float* H, size_t h_seq_stride, const T* gain, float eps, T* A,
+                              cudaStream_t st) {
+  launch_k(residual_layer_in_kernel<T>, dim3(S, B), dim3(kNormThreads), 0, st, rows, off_prev, hidden, part, sp, H,
+           h_seq_stride, gain, eps, A);
+}
+template <typename T>
 void launch_qkv_epilogue(Rows rows, int B, int S, int n_heads, int head_dim, const float* part, const SplitPlan& sp,
                          const float* rope_cos, const float* rope_sin, T* Q, T* Kc, T* Vc, size_t kv_seq_stride,
                          int Tc, cudaStream_t st) {
@@ -548,6 +600,8 @@ void launch_commit(int B, int D, int n_bins, int Nv, int S, int L, size_t frame_
                                 const T*, const float*, const T*, const T*, int*, cudaStream_t);                 \
   template void launch_layer_in<T>(Rows, const int*, int, int, int, float*, size_t, const T*, float, T*,          \
                                    cudaStream_t);                                                                 \
+  template void launch_residual_layer_in<T>(Rows, const int*, int, int, int, const float*, const SplitPlan&,     \
+                                            float*, size_t, const T*, float, T*, cudaStream_t);                   \
   template void launch_qkv_epilogue<T>(Rows, int, int, int, int, const float*, const SplitPlan&, const float*,  \
                                        const float*, T*, T*, T*, size_t, int, cudaStream_t);                      \
   template void launch_residual_norm<T>(Rows, int, int, int, const float*, const SplitPlan&, const T*, float, T*, \

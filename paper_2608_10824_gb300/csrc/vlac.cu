@@ -50,6 +50,7 @@ struct vlac_ctx {
   int gemv_pf_kb = 0;  // decode-GEMV L2 prefetch of the next projection, KB per CTA (measured: off is best)
   int dpass_bar = 1;  // persistent pass: grid barrier kind (VLAC_DPASS_BAR: 1 release/acquire, 0 fences)
   bool dpass_kv = true;  // persistent pass: attention K/V staged in shared memory (VLAC_DPASS_KV)
+  bool fuse_rows = true;  // prefix: a layer's down residual and the next layer's input norm in one launch (VLAC_FUSE_ROWS)
   bool use_dpass = true;  // decode passes as one persistent cooperative launch (k_dpass.cu) where supported
   int dpass_attn_chunks = 0;  // its key ranges per (sequence, head); 0 = chosen from the SM count
   void** dp_ptrs = nullptr;  // device: per-layer pointers [w_qkv | w_o | w_gu | w_d | g_attn | g_ffn][L]
@@ -272,6 +273,7 @@ extern "C" int vlac_create(const vlac_dims* dims, const vlac_weights* w, vlac_ct
   if (const char* e = std::getenv("VLAC_DPASS")) c->use_dpass = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_DPASS_BAR")) c->dpass_bar = std::atoi(e) != 0 ? 1 : 0;
   if (const char* e = std::getenv("VLAC_DPASS_KV")) c->dpass_kv = std::atoi(e) != 0;
+  if (const char* e = std::getenv("VLAC_FUSE_ROWS")) c->fuse_rows = std::atoi(e) != 0;
   if (const char* e = std::getenv("VLAC_DPASS_ATTN_CHUNKS")) c->dpass_attn_chunks = std::max(0, std::atoi(e));
   c->d = *dims;
   const vlac_dims& d = c->d;
@@ -762,9 +764,13 @@ void gemm(vlac_ctx* c, const ActMaps* tmA, const CUtensorMap* tmW, const T* A, c
 // the mixed-cache attention, o-projection + residual, the MLP norm, gate/up +
 // SwiGLU and down + residual.  The bf16 attention reads the K/V tiles through
 // the cache's maps kvm; seq0 is the batch's first sequence in the cache.
+// do_in: this layer's input norm runs here (else the previous layer's last
+// launch ran it); rl_next / H_next: the next layer's rows and H slice, whose
+// input norm then runs fused with this layer's down residual.
 template <typename T>
 void prefix_layer(vlac_ctx* c, const Rows& rl, const int* off_prev, int B, int l, float* H, size_t h_seq_stride,
-                  T* Kc_l, T* Vc_l, size_t kv_seq_stride, const KvMaps* kvm, int seq0, cudaStream_t st) {
+                  T* Kc_l, T* Vc_l, size_t kv_seq_stride, const KvMaps* kvm, int seq0, cudaStream_t st,
+                  bool do_in = true, const Rows* rl_next = nullptr, float* H_next = nullptr) {
   const vlac_dims& d = c->d;
   const int S = c->S, Hd = d.hidden, F = d.ffn, nh = d.n_heads, hd = d.head_dim;
   const float eps = d.rms_eps;
@@ -779,7 +785,7 @@ void prefix_layer(vlac_ctx* c, const Rows& rl, const int* off_prev, int B, int l
   };
   const SplitPlan sq = with_tail(c->sp_qkv), so = with_tail(c->sp_o), sg = with_tail(c->sp_gu), sd = with_tail(c->sp_d);
   const int* ml = rl.off + B;
-  {
+  if (do_in) {
     ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
     launch_layer_in<T>(rl, off_prev, B, S, Hd, H, h_seq_stride, W(c->attn_norm[l]), eps, A, st);
   }
@@ -807,9 +813,13 @@ void prefix_layer(vlac_ctx* c, const Rows& rl, const int* off_prev, int B, int l
   gemm<T>(c, &c->tm_G, c->bf16 ? &c->tm_d[l] : nullptr, G, c->wd[l], ml, Hd, F, sd, st);
   {
     ProfScope ps_(c, VLAC_PROF_ROWS, 0, st);
-    launch_residual(rl, B, S, Hd, c->part, sd, st);
+    if (rl_next)
+      launch_residual_layer_in<T>(*rl_next, rl.off, B, S, Hd, c->part, sd, H_next, h_seq_stride,
+                                  W(c->attn_norm[l + 1]), eps, A, st);
+    else
+      launch_residual(rl, B, S, Hd, c->part, sd, st);
   }
-  c->launches += 6;
+  c->launches += do_in ? 6 : 5;
 }
 
 // The step body: reads only the staged inputs and writes only the context's
@@ -881,8 +891,13 @@ int step_impl(vlac_ctx* c, vlac_cache* k, cudaStream_t st) {
   for (int l = 0; l < L; ++l) {
     Rows rl{c->off + (size_t)l * (B + 1), c->idx, S, c->X};
     const int* off_prev = l == 0 ? rl.off : c->off + (size_t)(l - 1) * (B + 1);
+    // the next layer's input norm runs with this layer's down residual
+    const Rows rl_next{c->off + (size_t)(l + 1) * (B + 1), c->idx, S, c->X};
+    const bool fuse_next = c->fuse_rows && l + 1 < L;
     prefix_layer<T>(c, rl, off_prev, B, l, l == 0 ? nullptr : k->H + (size_t)l * S * Hd, k->h_seq_stride,
-                    Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, &k->kvm, 0, st);
+                    Kc + l * kv_layer, Vc + l * kv_layer, k->kv_seq_stride, &k->kvm, 0, st,
+                    l == 0 || !c->fuse_rows, fuse_next ? &rl_next : nullptr,
+                    fuse_next ? k->H + (size_t)(l + 1) * S * Hd : nullptr);
     if (c->s2_on && l == c->s2_layer) {
       // Stage 2: the text rows' attention on the visual keys of this layer (Q
       // still holds this layer's rows)
